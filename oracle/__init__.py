@@ -1,0 +1,220 @@
+"""fp64 CPU oracle for the BiSCo-LLM hot path -- TEST INFRASTRUCTURE ONLY.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may import this package.  The product library never loads it and
+shares no code with it.  The arithmetic lives in ``bisco_oracle.c`` (plain C,
+binary64, ``-ffp-contract=off``); this module compiles it with gcc and
+marshals numpy arrays through ctypes.
+
+Functions and the paper passages they follow:
+
+* :func:`encode`            Sec. III-E Eq. 8 (protected columns), Eq. 10 (Q8),
+                            Sec. III-C Eq. 3 and Sec. III-D Eq. 5-7 (stages)
+* :func:`select_protected`  Eq. 8
+* :func:`decode_rows`       Sec. III-F Eq. 12 with the Eq. 10 scatter
+* :func:`matmul`            y = What x (plain definition)
+* :func:`apply_rows`        decode + matmul on a list of rows
+* :func:`double_to_fp16`, :func:`fp16_to_double`, :func:`bf16_to_double`
+                            the number formats the storage uses
+
+Parity status: every function is pinned by ``tests/test_oracle_pins.py``
+except whole-model quality, which needs trained codecs and real checkpoints
+(parity unpinned, out of scope).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "bisco_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB = os.path.join(_BUILD, "libbisco_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+OK, ERR_INVALID_ARG, ERR_RANGE = 0, 1, 3
+
+CFLAGS = ["-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared"]
+
+
+def build(force: bool = False) -> str:
+    """Compile bisco_oracle.c into _build/libbisco_oracle.so (gcc, fp64)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if (not force and os.path.exists(_LIB)
+            and os.path.getmtime(_LIB) >= os.path.getmtime(_SRC)):
+        return _LIB
+    tmp = _LIB + ".%d.tmp" % os.getpid()
+    subprocess.check_call(["gcc", *CFLAGS, "-o", tmp, _SRC, "-lm"])
+    os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        lib = ctypes.CDLL(build())
+        P = ctypes.c_void_p
+        i32, i64 = ctypes.c_int32, ctypes.c_int64
+        lib.or_bf16_to_double.restype = ctypes.c_double
+        lib.or_bf16_to_double.argtypes = [ctypes.c_uint16]
+        lib.or_fp16_to_double.restype = ctypes.c_double
+        lib.or_fp16_to_double.argtypes = [ctypes.c_uint16]
+        lib.or_double_to_fp16.restype = ctypes.c_uint16
+        lib.or_double_to_fp16.argtypes = [ctypes.c_double]
+        lib.or_pad16.restype = i32
+        lib.or_pad16.argtypes = [i32]
+        lib.or_encoded_sizes.restype = ctypes.c_int
+        lib.or_encoded_sizes.argtypes = [i32, i32, i32, i32, P]
+        lib.or_select_protected.restype = ctypes.c_int
+        lib.or_select_protected.argtypes = [P, P, i32, i32, i32, P, P]
+        lib.or_quantize_protected.restype = ctypes.c_int
+        lib.or_quantize_protected.argtypes = [P, i32, i32, P, i32, P, P]
+        lib.or_encode_stages.restype = ctypes.c_int
+        lib.or_encode_stages.argtypes = [P, i32, i32, i32, P, i32, P, P]
+        lib.or_encode.restype = ctypes.c_int
+        lib.or_encode.argtypes = [P, P, i32, i32, i32, i32, P, P, P, P, P]
+        lib.or_decode_rows.restype = None
+        lib.or_decode_rows.argtypes = [P, P, P, P, P, i32, i32, i32, i32, i32, i32, P]
+        lib.or_matmul.restype = None
+        lib.or_matmul.argtypes = [P, i32, i32, P, i32, P]
+        lib.or_apply_rows.restype = ctypes.c_int
+        lib.or_apply_rows.argtypes = [P, P, P, P, P, i32, i32, i32, i32, P, i32, P, i32, P]
+        del i64
+        _lib = lib
+        return lib
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+class OracleError(RuntimeError):
+    def __init__(self, code):
+        super().__init__("oracle status %d" % code)
+        self.code = code
+
+
+# ------------------------------------------------------------------ numbers
+
+def bf16_to_double(b: int) -> float:
+    return _load().or_bf16_to_double(int(b))
+
+
+def fp16_to_double(h: int) -> float:
+    return _load().or_fp16_to_double(int(h))
+
+
+def double_to_fp16(x: float) -> int:
+    return int(_load().or_double_to_fp16(float(x)))
+
+
+def pad16(p: int) -> int:
+    return (p + 15) // 16 * 16
+
+
+def encoded_sizes(N, K, S, p):
+    out = np.zeros(5, np.int64)
+    rc = _load().or_encoded_sizes(N, K, S, p, _ptr(out))
+    if rc:
+        raise OracleError(rc)
+    return [int(v) for v in out]
+
+
+# ------------------------------------------------------------------ encode
+
+def select_protected(W_bits, p, g=None):
+    """Eq. 8: returns (idx ascending int32[p], scores float64[K])."""
+    W_bits = _c(W_bits, np.uint16)
+    N, K = W_bits.shape
+    idx = np.zeros(max(p, 1), np.int32)
+    scores = np.zeros(K, np.float64)
+    gg = None if g is None else _c(g, np.float32)
+    rc = _load().or_select_protected(_ptr(W_bits), _ptr(gg), N, K, p, _ptr(idx), _ptr(scores))
+    if rc:
+        raise OracleError(rc)
+    return idx[:p].copy(), scores
+
+
+def encode(W_bits, S, p, g=None):
+    """Whole encoder.  W_bits: uint16[N][K] bf16 bit patterns.
+
+    Returns a dict with codes uint8[S][N][K/8], norms uint16[S][N][K/8],
+    q8 int8[N][pad16(p)], scale uint16[p], idx int32[p]."""
+    W_bits = _c(W_bits, np.uint16)
+    N, K = W_bits.shape
+    C = K // 8 if K % 8 == 0 else 1
+    codes = np.zeros((S, N, C), np.uint8)
+    norms = np.zeros((S, N, C), np.uint16)
+    q8 = np.zeros((N, max(pad16(p), 16)), np.int8)
+    scale = np.zeros(max(p, 1), np.uint16)
+    idx = np.zeros(max(p, 1), np.int32)
+    gg = None if g is None else _c(g, np.float32)
+    rc = _load().or_encode(_ptr(W_bits), _ptr(gg), N, K, S, p, _ptr(codes), _ptr(norms),
+                           _ptr(q8), _ptr(scale), _ptr(idx))
+    if rc:
+        raise OracleError(rc)
+    return dict(N=N, K=K, S=S, p=p, codes=codes, norms=norms,
+                q8=q8[:, :pad16(p)].copy(), scale=scale[:p].copy(), idx=idx[:p].copy())
+
+
+def _layer_args(L):
+    codes = _c(L["codes"], np.uint8)
+    norms = _c(L["norms"], np.uint16)
+    q8 = _c(L["q8"], np.int8) if L["p"] > 0 else np.zeros((L["N"], 16), np.int8)
+    scale = _c(L["scale"], np.uint16) if L["p"] > 0 else np.zeros(1, np.uint16)
+    idx = _c(L["idx"], np.int32) if L["p"] > 0 else np.zeros(1, np.int32)
+    return codes, norms, q8, scale, idx
+
+
+def decode_rows(L, row0=0, nrows=None):
+    """Eq. 12 + Eq. 10: dense float64 rows [row0, row0+nrows) of What."""
+    N, K = L["N"], L["K"]
+    if nrows is None:
+        nrows = N - row0
+    codes, norms, q8, scale, idx = _layer_args(L)
+    out = np.zeros((nrows, K), np.float64)
+    _load().or_decode_rows(_ptr(codes), _ptr(norms), _ptr(q8), _ptr(scale), _ptr(idx),
+                           N, K, L["S"], L["p"], row0, nrows, _ptr(out))
+    return out
+
+
+def matmul(What, X_bits):
+    """y[b][i] = sum_j What[i][j] * x[b][j] in float64 (X_bits: bf16 bits)."""
+    What = _c(What, np.float64)
+    X_bits = _c(np.atleast_2d(X_bits), np.uint16)
+    nrows, K = What.shape
+    B = X_bits.shape[0]
+    Y = np.zeros((B, nrows), np.float64)
+    _load().or_matmul(_ptr(What), nrows, K, _ptr(X_bits), B, _ptr(Y))
+    return Y
+
+
+def apply_rows(L, rows, X_bits):
+    """Y[b][t] = What[rows[t], :] . x_b, decoding one row at a time."""
+    rows = _c(rows, np.int32)
+    X_bits = _c(np.atleast_2d(X_bits), np.uint16)
+    codes, norms, q8, scale, idx = _layer_args(L)
+    B = X_bits.shape[0]
+    Y = np.zeros((B, len(rows)), np.float64)
+    rc = _load().or_apply_rows(_ptr(codes), _ptr(norms), _ptr(q8), _ptr(scale), _ptr(idx),
+                               L["N"], L["K"], L["S"], L["p"], _ptr(rows), len(rows),
+                               _ptr(X_bits), B, _ptr(Y))
+    if rc:
+        raise OracleError(rc)
+    return Y
+
+
+def gemv(L, X_bits):
+    """Full output Y[B][N] = X What^T (decode to dense, then the naive matmul)."""
+    return matmul(decode_rows(L), X_bits)

@@ -1,0 +1,343 @@
+/*
+ * bisco_oracle.c -- plain, slow, fp64 CPU oracle for the BiSCo-LLM inference
+ * hot path (binary spherical coding of LLM weights, arxiv 2607.08643).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing in the product path may link, load or
+ * call this file: only the tests, the smoke check and the benchmark's CPU
+ * baseline leg use it.  It shares no code, header or constant with the CUDA
+ * library; the two agree only through the paper and the storage format.
+ *
+ * What it computes (all arithmetic in IEEE binary64, no FMA contraction --
+ * build with -ffp-contract=off -- and no reordering of sums):
+ *
+ *   encode   Sec. III-E Eq. 8 (protected input channels, TopK of g_j*||W_:,j||_2),
+ *            Sec. III-E Eq. 10 (8-bit quantiser on the protected slices),
+ *            Sec. III-C Eq. 3 (unit-sphere normalisation and sign binarisation,
+ *            q = sign(u)/sqrt(b)) with the identity encoder (b = d) and the
+ *            decoder read as "rescale the unit code by the chunk's stored
+ *            fp16 L2 norm", and Sec. III-D Eq. 5-7 (residual stages
+ *            r(s) = r(s-1) - rhat(s)).
+ *   decode   Sec. III-F Eq. 12 (stages decoded independently and summed)
+ *            with the Eq. 10 scatter of the protected columns.
+ *   matmul   y[b][i] = sum_j What[i][j] * x[b][j]  (plain definition).
+ *
+ * Storage format produced by encode (identical bytes are required from the
+ * GPU encoder):
+ *   codes [S][N][K/8] uint8  one byte per 8-element chunk; bit k = element k
+ *                            of the chunk, 1 = negative, 0 = positive (the
+ *                            sign of +0.0, -0.0 and exact zeros is positive)
+ *   norms [S][N][K/8] uint16 IEEE binary16 bits of the stage target's chunk
+ *                            L2 norm, rounded to nearest-even
+ *   q8    [N][p_pad]  int8   p_pad = p rounded up to a multiple of 16, zero pad
+ *   scale [p]         uint16 binary16 bits of max_i |W_ij| / 127
+ *   idx   [p]         int32  protected input columns, ascending
+ *
+ * Readings of the paper taken here (the paper is silent on them):
+ *   - no learned encoder/decoder: b = d = 8, the decoder is n16 * q;
+ *   - protected entries are masked to zero before every stage (Eq. 10's
+ *     complement realised by masking, not compaction);
+ *   - sign(0) = +1;  g = NULL means g_j = 1;  ties in TopK go to the lower
+ *     column index;  p is given by the caller (= ceil(rho * K)).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define OR_OK 0
+#define OR_ERR_INVALID_ARG 1
+#define OR_ERR_RANGE 3
+
+/* ---------------------------------------------------------------- numbers */
+
+/* bf16 -> binary64: bf16 is the upper half of a binary32, so widening is
+ * exact for every bit pattern. */
+double or_bf16_to_double(uint16_t b)
+{
+    uint32_t u = (uint32_t)b << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+/* binary16 bits -> binary64 (exact). */
+double or_fp16_to_double(uint16_t h)
+{
+    int sign = (h >> 15) & 1;
+    int e = (h >> 10) & 0x1f;
+    int m = h & 0x3ff;
+    double v;
+    if (e == 0)
+        v = ldexp((double)m, -24);                 /* zero or subnormal */
+    else if (e == 31)
+        v = m ? NAN : INFINITY;
+    else
+        v = ldexp((double)(1024 + m), e - 25);     /* 1.m * 2^(e-15) */
+    return sign ? -v : v;
+}
+
+/* binary64 -> binary16 bits, round to nearest, ties to even, gradual
+ * underflow, overflow to infinity.  The significand is scaled by a power of
+ * two (exact in binary64) so that the 11 kept bits form the integer part,
+ * and rounded once with nearbyint() in the default rounding mode. */
+uint16_t or_double_to_fp16(double x)
+{
+    uint16_t sign = signbit(x) ? 0x8000 : 0;
+    double a = fabs(x);
+    if (isnan(x))
+        return (uint16_t)(sign | 0x7e00);
+    if (a < ldexp(1.0, -14)) {
+        /* subnormal range: units of 2^-24; 1024 units is the least normal */
+        double m = nearbyint(a * ldexp(1.0, 24));
+        return (uint16_t)(sign | (uint16_t)m);
+    }
+    if (isinf(a))
+        return (uint16_t)(sign | 0x7c00);
+    int ex;
+    frexp(a, &ex);                 /* a = f * 2^ex, f in [0.5, 1) */
+    int E = ex - 1;                /* a in [2^E, 2^(E+1)) */
+    if (E > 15)
+        return (uint16_t)(sign | 0x7c00);
+    double m = nearbyint(ldexp(a, 10 - E));   /* in [1024, 2048] */
+    if (m == 2048.0) {
+        m = 1024.0;
+        E += 1;
+        if (E > 15)
+            return (uint16_t)(sign | 0x7c00);
+    }
+    return (uint16_t)(sign | (uint16_t)((E + 15) << 10) | (uint16_t)(m - 1024.0));
+}
+
+/* 1/sqrt(d) for d = 8, the spherical code's per-element magnitude (Eq. 3). */
+static double or_inv_sqrt8(void) { return 1.0 / sqrt(8.0); }
+
+int32_t or_pad16(int32_t p) { return (p + 15) / 16 * 16; }
+
+/* Byte sizes of the five buffers of one encoded layer (Eq. 2 real-size
+ * terms: S_code = codes, S_meta = norms + scales + indices, S_8bit = q8). */
+int or_encoded_sizes(int32_t N, int32_t K, int32_t S, int32_t p, int64_t out[5])
+{
+    if (N <= 0 || K <= 0 || K % 8 != 0 || S < 1 || p < 0 || p > K)
+        return OR_ERR_INVALID_ARG;
+    int64_t C = K / 8;
+    out[0] = (int64_t)S * N * C;                 /* codes  */
+    out[1] = (int64_t)S * N * C * 2;             /* norms  */
+    out[2] = (int64_t)N * or_pad16(p);           /* q8     */
+    out[3] = (int64_t)p * 2;                     /* scales */
+    out[4] = (int64_t)p * 4;                     /* idx    */
+    return OR_OK;
+}
+
+/* ------------------------------------------------ Eq. 8: protected columns */
+
+typedef struct { double score; int32_t j; } or_scored;
+
+static int or_cmp_scored(const void *a, const void *b)
+{
+    const or_scored *x = (const or_scored *)a, *y = (const or_scored *)b;
+    if (x->score > y->score) return -1;        /* larger score first */
+    if (x->score < y->score) return 1;
+    return (x->j < y->j) ? -1 : (x->j > y->j); /* tie: lower index first */
+}
+
+static int or_cmp_i32(const void *a, const void *b)
+{
+    int32_t x = *(const int32_t *)a, y = *(const int32_t *)b;
+    return (x > y) - (x < y);
+}
+
+/* score_j = g_j * sqrt(sum_{i=0..N-1} W_ij^2), the sum taken in ascending i;
+ * P = the p columns of largest score, returned ascending.  Also writes the
+ * scores when scores_out != NULL. */
+int or_select_protected(const uint16_t *W, const float *g, int32_t N, int32_t K,
+                        int32_t p, int32_t *idx_out, double *scores_out)
+{
+    if (p < 0 || p > K) return OR_ERR_INVALID_ARG;
+    or_scored *sc = (or_scored *)malloc(sizeof(or_scored) * (size_t)K);
+    if (!sc) return OR_ERR_INVALID_ARG;
+    for (int32_t j = 0; j < K; ++j) {
+        double sum = 0.0;
+        for (int32_t i = 0; i < N; ++i) {
+            double w = or_bf16_to_double(W[(int64_t)i * K + j]);
+            sum = sum + w * w;
+        }
+        double s = sqrt(sum);
+        if (g) s = (double)g[j] * s;
+        sc[j].score = s;
+        sc[j].j = j;
+        if (scores_out) scores_out[j] = s;
+    }
+    qsort(sc, (size_t)K, sizeof(or_scored), or_cmp_scored);
+    for (int32_t t = 0; t < p; ++t) idx_out[t] = sc[t].j;
+    qsort(idx_out, (size_t)p, sizeof(int32_t), or_cmp_i32);
+    free(sc);
+    return OR_OK;
+}
+
+/* ----------------------------------------- Eq. 10: 8-bit protected slices */
+
+/* Per protected column j (a per-channel 8-bit quantiser):
+ *   scale_j = fp16(max_i |W_ij| / 127)
+ *   q8_ij   = clamp(rint(W_ij / scale_j), -127, 127), or 0 if scale_j == 0. */
+int or_quantize_protected(const uint16_t *W, int32_t N, int32_t K,
+                          const int32_t *idx, int32_t p,
+                          int8_t *q8_out, uint16_t *scale_out)
+{
+    int32_t pp = or_pad16(p);
+    memset(q8_out, 0, (size_t)N * (size_t)pp);
+    for (int32_t t = 0; t < p; ++t) {
+        int32_t j = idx[t];
+        double m = 0.0;
+        for (int32_t i = 0; i < N; ++i) {
+            double a = fabs(or_bf16_to_double(W[(int64_t)i * K + j]));
+            if (a > m) m = a;
+        }
+        uint16_t s16 = or_double_to_fp16(m / 127.0);
+        if ((s16 & 0x7c00) == 0x7c00) return OR_ERR_RANGE;
+        scale_out[t] = s16;
+        double s = or_fp16_to_double(s16);
+        for (int32_t i = 0; i < N; ++i) {
+            double q = 0.0;
+            if (s != 0.0) {
+                q = nearbyint(or_bf16_to_double(W[(int64_t)i * K + j]) / s);
+                if (q > 127.0) q = 127.0;
+                if (q < -127.0) q = -127.0;
+            }
+            q8_out[(int64_t)i * pp + t] = (int8_t)q;
+        }
+    }
+    return OR_OK;
+}
+
+/* --------------------------------- Eq. 3 + Eq. 5-7: spherical sign stages */
+
+/* For every row i and chunk c (8 contiguous input columns), with
+ * r(0) = the chunk of W with protected entries set to zero, for s = 1..S:
+ *   n      = sqrt(((((((v0^2+v1^2)+v2^2)+v3^2)+v4^2)+v5^2)+v6^2)+v7^2)
+ *   n16    = fp16(n)                       (stored norm; overflow -> RANGE)
+ *   bit_k  = (v_k < 0)                     (stored sign pattern, Eq. 3)
+ *   rhat_k = (bit_k ? -1 : +1) * n16 / sqrt(8)
+ *   r(s)_k = r(s-1)_k - rhat_k, then 0 at protected entries   (Eq. 5-7)  */
+int or_encode_stages(const uint16_t *W, int32_t N, int32_t K, int32_t S,
+                     const int32_t *idx, int32_t p,
+                     uint8_t *codes_out, uint16_t *norms_out)
+{
+    int32_t C = K / 8;
+    double inv_sqrt8 = or_inv_sqrt8();
+    unsigned char *prot = (unsigned char *)calloc((size_t)K, 1);
+    if (!prot) return OR_ERR_INVALID_ARG;
+    for (int32_t t = 0; t < p; ++t) prot[idx[t]] = 1;
+    int rc = OR_OK;
+    for (int32_t i = 0; i < N && rc == OR_OK; ++i) {
+        for (int32_t c = 0; c < C; ++c) {
+            double v[8];
+            for (int k = 0; k < 8; ++k) {
+                int32_t j = 8 * c + k;
+                v[k] = prot[j] ? 0.0 : or_bf16_to_double(W[(int64_t)i * K + j]);
+            }
+            for (int32_t s = 0; s < S; ++s) {
+                double sum = v[0] * v[0];
+                for (int k = 1; k < 8; ++k) sum = sum + v[k] * v[k];
+                double n = sqrt(sum);
+                uint16_t n16 = or_double_to_fp16(n);
+                if ((n16 & 0x7c00) == 0x7c00) { rc = OR_ERR_RANGE; break; }
+                uint8_t bits = 0;
+                for (int k = 0; k < 8; ++k)
+                    if (v[k] < 0.0) bits |= (uint8_t)(1u << k);
+                double t = or_fp16_to_double(n16) * inv_sqrt8;
+                for (int k = 0; k < 8; ++k) {
+                    double rhat = ((bits >> k) & 1) ? -t : t;
+                    v[k] = v[k] - rhat;
+                    if (prot[8 * c + k]) v[k] = 0.0;
+                }
+                int64_t o = ((int64_t)s * N + i) * C + c;
+                codes_out[o] = bits;
+                norms_out[o] = n16;
+            }
+            if (rc != OR_OK) break;
+        }
+    }
+    free(prot);
+    return rc;
+}
+
+/* Whole offline encoder: non-finite weights are rejected with RANGE. */
+int or_encode(const uint16_t *W, const float *g, int32_t N, int32_t K,
+              int32_t S, int32_t p, uint8_t *codes, uint16_t *norms,
+              int8_t *q8, uint16_t *scale, int32_t *idx)
+{
+    if (N <= 0 || K <= 0 || K % 8 != 0 || S < 1 || S > 3 || p < 0 || p > K)
+        return OR_ERR_INVALID_ARG;
+    for (int64_t e = 0; e < (int64_t)N * K; ++e)
+        if (!isfinite(or_bf16_to_double(W[e]))) return OR_ERR_RANGE;
+    int rc = or_select_protected(W, g, N, K, p, idx, NULL);
+    if (rc) return rc;
+    rc = or_quantize_protected(W, N, K, idx, p, q8, scale);
+    if (rc) return rc;
+    return or_encode_stages(W, N, K, S, idx, p, codes, norms);
+}
+
+/* ------------------------------------------------ Eq. 12 + Eq. 10: decode */
+
+/* Dense reconstruction of rows [row0, row0+nrows):
+ *   What_ij = sum_{s=1..S} (bit ? -1 : +1) * n16_{s,i,c} / sqrt(8)   j not in P
+ *   What_ij = scale_j * q8_ij                                         j in P   */
+void or_decode_rows(const uint8_t *codes, const uint16_t *norms,
+                    const int8_t *q8, const uint16_t *scale, const int32_t *idx,
+                    int32_t N, int32_t K, int32_t S, int32_t p,
+                    int32_t row0, int32_t nrows, double *out)
+{
+    int32_t C = K / 8, pp = or_pad16(p);
+    double inv_sqrt8 = or_inv_sqrt8();
+    for (int32_t r = 0; r < nrows; ++r) {
+        int32_t i = row0 + r;
+        double *o = out + (int64_t)r * K;
+        for (int32_t j = 0; j < K; ++j) {
+            int32_t c = j / 8, k = j % 8;
+            double acc = 0.0;
+            for (int32_t s = 0; s < S; ++s) {
+                int64_t e = ((int64_t)s * N + i) * C + c;
+                double t = or_fp16_to_double(norms[e]) * inv_sqrt8;
+                acc = acc + (((codes[e] >> k) & 1) ? -t : t);
+            }
+            o[j] = acc;
+        }
+        for (int32_t t = 0; t < p; ++t)
+            o[idx[t]] = or_fp16_to_double(scale[t]) * (double)q8[(int64_t)i * pp + t];
+    }
+}
+
+/* y[b][r] = sum_j What[r][j] * x[b][j], ascending j, for a block of rows. */
+void or_matmul(const double *What, int32_t nrows, int32_t K,
+               const uint16_t *X, int32_t B, double *Y)
+{
+    for (int32_t b = 0; b < B; ++b)
+        for (int32_t r = 0; r < nrows; ++r) {
+            double acc = 0.0;
+            for (int32_t j = 0; j < K; ++j)
+                acc = acc + What[(int64_t)r * K + j] *
+                            or_bf16_to_double(X[(int64_t)b * K + j]);
+            Y[(int64_t)b * nrows + r] = acc;
+        }
+}
+
+/* Y[b][t] = (x_b . What[rows[t], :]) for a list of rows, decoding one row at
+ * a time (used to check full-size layers on sampled outputs). */
+int or_apply_rows(const uint8_t *codes, const uint16_t *norms,
+                  const int8_t *q8, const uint16_t *scale, const int32_t *idx,
+                  int32_t N, int32_t K, int32_t S, int32_t p,
+                  const int32_t *rows, int32_t nrows,
+                  const uint16_t *X, int32_t B, double *Y)
+{
+    double *w = (double *)malloc(sizeof(double) * (size_t)K);
+    double *y = (double *)malloc(sizeof(double) * (size_t)B);
+    if (!w || !y) { free(w); free(y); return OR_ERR_INVALID_ARG; }
+    for (int32_t t = 0; t < nrows; ++t) {
+        or_decode_rows(codes, norms, q8, scale, idx, N, K, S, p, rows[t], 1, w);
+        or_matmul(w, 1, K, X, B, y);
+        for (int32_t b = 0; b < B; ++b) Y[(int64_t)b * nrows + t] = y[b];
+    }
+    free(w);
+    free(y);
+    return OR_OK;
+}
