@@ -1,0 +1,379 @@
+"""Decode benchmark: BiSCo-coded Qwen3-8B attention projections on GB300.
+
+Workload (one "step" = one decode token through every projection):
+  q_proj/o_proj 4096x4096 and k_proj/v_proj 1024x4096 (N x K) for each of
+  the 36 layers of Qwen3-8B, each a distinct random layer (N(0, 0.02)
+  weights with 8 outlier input columns x20, drawn on the device from a
+  seeded generator), coded with d = 8, base + 1 residual stage (S = 2) and
+  1 % int8 protected columns (p = 41); batch 1 bf16 N(0,1) activations.
+  The 144 coded layers hold 1.15 GB, far more than the 129 MB L2, so every
+  step streams its weights from HBM (no L2 flush needed).
+
+Metric: decode GEMV GB/s on compressed bytes (signs + norms + int8 payload +
+scales + indices) and tokens/s; value = whole-job GB/s over all ranks.
+
+  python bench.py [--gpus N --steps K --warmup W --batch B --impl {bisco,reference}]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode GEMV GB/s (compressed bytes) & tokens/s, % of HBM/tensor roofline"
+ATTN = ("q_proj", "k_proj", "v_proj", "o_proj")
+N_LAYERS = 36
+S_STAGES = 2
+RHO_PCT = 1
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--batch", type=int, default=1)
+    ap.add_argument("--layers", type=int, default=N_LAYERS)
+    ap.add_argument("--impl", choices=("bisco", "reference"), default="bisco")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    return ap.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def workload_config(args):
+    return {
+        "workload": "Qwen3-8B attention projections q/k/v/o x %d layers, decode batch %d"
+                    % (args.layers, args.batch),
+        "shapes_NxK": {"q_proj": [4096, 4096], "k_proj": [1024, 4096],
+                       "v_proj": [1024, 4096], "o_proj": [4096, 4096]},
+        "chunk_dim": 8, "stages": S_STAGES, "protected_pct": RHO_PCT, "batch": args.batch,
+        "weights": "N(0,0.02) + 8 outlier cols x20, seeded on device",
+        "l2": "inputs larger than L2 (distinct coded layers per step, no flush)",
+    }
+
+
+# ---------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples taken during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.Q,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        mhz, mx, reasons = [], None, set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                mhz.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not mhz:
+            return None
+        return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(mhz)}
+
+
+# ---------------------------------------------------------------- layers
+
+def build_layers(args, dev):
+    import torch
+    from paper_2607_08643_gb300 import bisco, synth
+    layers = []
+    ws = None
+    for l in range(args.layers):
+        for j, name in enumerate(ATTN):
+            N, K = synth.QWEN3_8B_SHAPES[name]
+            p = synth.protected_count(K, RHO_PCT)
+            W = synth.layer_weights_torch(N, K, seed=1000 * l + j, device=dev)
+            need = bisco.bisco_encode_workspace_bytes(N, K)
+            if ws is None or ws.numel() < need:
+                ws = torch.empty(need, dtype=torch.uint8, device=dev)
+            layers.append((name, bisco.bisco_encode(W, S_STAGES, p, workspace=ws)))
+            del W
+    torch.cuda.synchronize()
+    if bisco.bisco_get_device_error() != bisco.OK:
+        raise RuntimeError("device error while encoding")
+    return layers
+
+
+def run_bisco(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+    from paper_2607_08643_gb300 import bisco, synth
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    bisco.load()
+    layers = build_layers(args, dev)
+    B = args.batch
+    K = 4096
+    # per step: one activation shared by q/k/v and one for o_proj, per layer
+    n_in = 2 * args.layers
+    x_dev = torch.empty((n_in, B, K), dtype=torch.int16, device=dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(7 + rank)
+    x_dev.copy_(torch.randn((n_in, B, K), generator=gen, device=dev).to(torch.bfloat16).view(torch.int16))
+    outs = [torch.empty((B, L.N), dtype=torch.float32, device=dev) for _, L in layers]
+    y_total = sum(o.numel() for o in outs)
+    y_flat = torch.empty(y_total, dtype=torch.float32, device=dev)
+    views, off = [], 0
+    for o in outs:
+        views.append(y_flat[off:off + o.numel()].view(o.shape))
+        off += o.numel()
+    bytes_step = sum(L.compressed_bytes for _, L in layers)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step():
+        for i, (name, L) in enumerate(layers):
+            li = i // 4
+            xi = 2 * li + (1 if name == "o_proj" else 0)
+            bisco.bisco_gemv(L, x_dev[xi], y=views[i], stream=stream)
+
+    # capture one step (144 launches through the public API) in a CUDA graph
+    with torch.cuda.stream(stream):
+        step()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            step()
+    torch.cuda.synchronize()
+    if bisco.bisco_get_device_error(stream) != bisco.OK:
+        raise RuntimeError("device error in warm-up")
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(max(args.warmup, 3)):
+        g.replay()
+    barrier()
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    time.sleep(0.3)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(args.steps):
+            g.replay()
+        e1.record(stream)
+    barrier()
+    ms_total = e0.elapsed_time(e1)
+    clk = clocks.stop()
+    if bisco.bisco_get_device_error(stream) != bisco.OK:
+        raise RuntimeError("device error in timed region")
+
+    # end to end: pinned host inputs in, graph of public-API calls, outputs out
+    x_host = torch.empty(x_dev.shape, dtype=torch.int16, pin_memory=True)
+    x_host.copy_(x_dev.cpu())
+    y_host = torch.empty(y_total, dtype=torch.float32, pin_memory=True)
+    for _ in range(2):
+        with torch.cuda.stream(stream):
+            x_dev.copy_(x_host, non_blocking=True)
+            g.replay()
+            y_host.copy_(y_flat, non_blocking=True)
+    barrier()
+    t0 = time.perf_counter()
+    f0 = torch.cuda.Event(enable_timing=True)
+    f1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        f0.record(stream)
+        for _ in range(args.steps):
+            x_dev.copy_(x_host, non_blocking=True)
+            g.replay()
+            y_host.copy_(y_flat, non_blocking=True)
+        f1.record(stream)
+    stream.synchronize()
+    wall_e2e = time.perf_counter() - t0
+    barrier()
+    ms_e2e = max(f0.elapsed_time(f1), wall_e2e * 1e3)
+
+    if world > 1:
+        t = torch.tensor([ms_total, ms_e2e], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_total, ms_e2e = float(t[0]), float(t[1])
+
+    ms_step = ms_total / args.steps
+    gbs = world * bytes_step / (ms_step * 1e-3) / 1e9
+    tok_s = world * B / (ms_step * 1e-3)
+    e2e_gbs = world * bytes_step / (ms_e2e / args.steps * 1e-3) / 1e9
+    launches = len(layers)
+    peak, peak_kind = peaks()
+    achieved = bytes_step / (ms_step * 1e-3) / 1e9          # per GPU, dominant kernel
+    return dict(
+        value=gbs, ms_per_step=ms_step, tokens_per_s=tok_s, bytes_per_step=bytes_step,
+        launches=launches, e2e_gbs=e2e_gbs, h2d=x_dev.numel() * 2, d2h=y_total * 4,
+        roofline={"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                  "frac": achieved / peak, "traffic": None,
+                  "peak_source": "%s hbm_gbs (MEASURED_PEAKS.json)" % peak_kind
+                  if peak_kind == "measured" else "fallback 6.8 TB/s",
+                  "kernel": "k_gemv (bisco_gemv)",
+                  "bytes_per_launch_avg": bytes_step / launches},
+        clocks=clk, ms_e2e=ms_e2e / args.steps)
+
+
+# ------------------------------------------------------------ CPU oracle
+
+def cpu_oracle_sample(seconds, batch):
+    """The fp64 oracle (decode to dense + naive matmul, single thread) on a
+    bounded sample of the same workload: whole projections of layer 0, in
+    q/k/v/o order, repeated until `seconds` of CPU time have passed."""
+    import numpy as np
+    import oracle
+    from paper_2607_08643_gb300 import synth
+    layers = []
+    for j, name in enumerate(ATTN):
+        N, K = synth.QWEN3_8B_SHAPES[name]
+        p = synth.protected_count(K, RHO_PCT)
+        W = synth.layer_weights(N, K, seed=j)
+        layers.append(oracle.encode(W, S=S_STAGES, p=p))
+    X = synth.activations(batch, 4096, seed=99)
+    done_bytes, n_calls, t0 = 0, 0, time.perf_counter()
+    while True:
+        L = layers[n_calls % 4]
+        oracle.gemv(L, X)
+        done_bytes += S_STAGES * L["N"] * (L["K"] // 8) * 3 + L["N"] * L["p"] + 6 * L["p"]
+        n_calls += 1
+        el = time.perf_counter() - t0
+        if el >= seconds and n_calls >= 1:
+            break
+    return {"value": done_bytes / el / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": "%d whole-projection calls of layer 0 (q/k/v/o cycle), %.1f s, "
+                      "fp64 decode-to-dense + naive matmul, batch %d" % (n_calls, el, batch)}
+
+
+def run_reference(args, rank, world):
+    """Reference arm: the CPU oracle as it stands, on the same metric."""
+    if rank != 0:
+        return None
+    per_step = max(2.0, min(20.0, 120.0 / max(1, args.steps + args.warmup)))
+    for _ in range(args.warmup):
+        cpu_oracle_sample(min(per_step, 2.0), args.batch)
+    vals, t0 = [], time.perf_counter()
+    for _ in range(args.steps):
+        vals.append(cpu_oracle_sample(per_step, args.batch))
+    el = time.perf_counter() - t0
+    gbs = statistics.median(v["value"] for v in vals)
+    bytes_step_full = 0
+    for name in ATTN:
+        N, K = (4096, 4096) if name in ("q_proj", "o_proj") else (1024, 4096)
+        bytes_step_full += S_STAGES * N * (K // 8) * 3 + N * 41 + 6 * 41
+    bytes_step_full *= args.layers
+    ms_step = bytes_step_full / (gbs * 1e9) * 1e3
+    line = {
+        "impl": "reference", "metric": METRIC, "value": gbs, "unit": "GB/s", "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": workload_config(args),
+        "tokens_per_s": args.batch / (ms_step * 1e-3),
+        "cpu_baseline": {"kind": "oracle", "cores": 1, "value": gbs, "unit": "GB/s",
+                         "sample": vals[0]["sample"] + "; each step a bounded sample"},
+        "e2e": {"value": gbs, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "wall_s": el,
+    }
+    return line
+
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        import torch
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    if args.impl == "reference":
+        line = run_reference(args, rank, world)
+        if line is not None:
+            print(json.dumps(line))
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return
+    # CPU baseline first (before any CUDA work), rank 0 at N = 1 only
+    cpu = None
+    if world == 1 and rank == 0 and not args.no_cpu_baseline:
+        cpu = cpu_oracle_sample(args.cpu_seconds, args.batch)
+    r = run_bisco(args, rank, world, local_rank)
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": r["value"], "unit": "GB/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": r["ms_per_step"],
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f16", "data": "synthetic", "config": workload_config(args),
+            "tokens_per_s": r["tokens_per_s"], "bytes_per_step": r["bytes_per_step"],
+            "e2e": {"value": r["e2e_gbs"], "unit": "GB/s",
+                    "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"],
+                    "how": "pinned H2D of the step's activations + CUDA graph of the step's "
+                           "bisco_gemv calls + D2H of all outputs, per step",
+                    "ms_per_step": r["ms_e2e"]},
+            "gpu_launches": r["launches"] * args.steps,
+            "roofline": r["roofline"],
+            "clocks": r["clocks"],
+            "cpu_baseline": cpu,
+            "parallelism": "replicas" if world > 1 else "single GPU",
+        }
+        print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

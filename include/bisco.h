@@ -1,0 +1,158 @@
+/*
+ * bisco.h -- C ABI of the GB300 (sm_103a) library for BiSCo-LLM binary
+ * spherical coded linear layers (arxiv 2607.08643).
+ *
+ * The paper states the problem, not an API: a weight matrix is cut into
+ * d-dimensional chunks, each chunk is stored as a bit-packed sign pattern of
+ * its unit-sphere direction (Sec. III-C, Eq. 3), further stages code the
+ * residual left by the earlier ones (Sec. III-D, Eq. 5-7), a small set of
+ * input channels chosen by Eq. 8 is kept in 8 bits instead (Sec. III-E,
+ * Eq. 10), and inference decodes the stages independently and sums them
+ * (Sec. III-F, Eq. 12) before the linear map y = W x.  This library runs
+ * that linear map straight from the coded bytes, without ever writing the
+ * dense weight to memory.
+ *
+ * Conventions for every entry point:
+ *   - All pointers are caller-owned DEVICE memory unless stated otherwise;
+ *     the library allocates nothing and keeps no state between calls other
+ *     than a per-device error word.
+ *   - Pointers must be 16-byte aligned, else BISCO_ERR_INVALID_ARG.
+ *   - Calls are asynchronous on `stream` (NULL = the legacy default stream).
+ *     Argument errors are returned synchronously and nothing is launched.
+ *     Errors found on the device (fp16 overflow in encode, an expired
+ *     bounded wait) are latched in the device error word and returned by
+ *     bisco_get_device_error().  No function aborts or prints.
+ *   - bf16 / fp16 values are passed as their uint16 bit patterns.
+ */
+#ifndef BISCO_H
+#define BISCO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t / CUstream. */
+typedef struct CUstream_st *bisco_stream_t;
+
+typedef enum {
+    BISCO_OK = 0,
+    BISCO_ERR_INVALID_ARG = 1,  /* bad size, NULL or misaligned pointer        */
+    BISCO_ERR_UNSUPPORTED = 2,  /* valid but not implemented (d != 8, axis 1)  */
+    BISCO_ERR_RANGE = 3,        /* encode: non-finite weight, fp16 norm/scale overflow */
+    BISCO_ERR_CUDA = 4,         /* a CUDA runtime call failed                  */
+    BISCO_ERR_TIMEOUT = 5       /* a bounded device-side wait expired          */
+} bisco_status;
+
+/*
+ * One coded linear layer W (N = out features x K = in features, the
+ * row-major layout of a PyTorch Linear weight).  Storage follows the paper's
+ * real-size accounting (Sec. III-A, Eq. 2: S_code + S_8bit + S_meta; there
+ * are no decoder or LoRA parameters):
+ *
+ *   codes    [S][N][K/8]  uint8   S_code.  Byte c of row i in stage s is
+ *                                 chunk c = input columns 8c..8c+7; bit k
+ *                                 is element k, 1 = negative (sign(0) = +).
+ *   norms    [S][N][K/8]  uint16  S_meta.  binary16 L2 norm of that stage's
+ *                                 chunk target; the chunk decodes to
+ *                                 (bit ? -1 : +1) * norm / sqrt(8).
+ *   q8       [N][p_pad]   int8    S_8bit.  Protected column t of row i at
+ *                                 q8[i*p_pad + t], p_pad = roundup(p, 16),
+ *                                 padding zero.
+ *   q8_scale [p]          uint16  binary16 per-column scale (Eq. 10 Q8).
+ *   prot_idx [p]          int32   protected input columns, strictly ascending.
+ *
+ * The decoded weight is  What[i][j] = sum_s (+-) norm_s[i][j/8] / sqrt(8)
+ * for j not protected, and q8_scale[t] * q8[i][t] for j = prot_idx[t].
+ */
+typedef struct {
+    int32_t n_out;        /* N >= 1                                       */
+    int32_t k_in;         /* K >= 8, K % 8 == 0                            */
+    int32_t chunk_dim;    /* d; only 8 is supported                        */
+    int32_t stages;       /* S in {1, 2, 3}                                */
+    int32_t n_protected;  /* p, 0 <= p <= K (the caller's ceil(rho * K))   */
+    int32_t protect_axis; /* 0 = input columns; 1 (output rows) unsupported */
+    uint8_t *codes;
+    uint16_t *norms;
+    int8_t *q8;
+    uint16_t *q8_scale;
+    int32_t *prot_idx;
+} bisco_layer;
+
+/* ABI version of this header (major * 100 + minor). */
+#define BISCO_ABI_VERSION 100
+int32_t bisco_abi_version(void);
+
+/* Static string for a status code (never NULL). */
+const char *bisco_status_string(int32_t status);
+
+/*
+ * Byte sizes of the five buffers of one layer, in the order codes, norms,
+ * q8, q8_scale, prot_idx (Sec. III-A, Eq. 2).  Host-only, no device access.
+ * Returns INVALID_ARG for N < 1, K < 8, K % 8 != 0, S not in 1..3, p out of
+ * [0, K] or out_bytes == NULL; UNSUPPORTED for d != 8.
+ */
+bisco_status bisco_encoded_sizes(int32_t N, int32_t K, int32_t d, int32_t S,
+                                 int32_t p, size_t out_bytes[5]);
+
+/*
+ * Scratch bytes bisco_encode needs for an N x K layer (per-column scores and
+ * the protected-column map); 0 on invalid sizes.
+ */
+size_t bisco_encode_workspace_bytes(int32_t N, int32_t K);
+
+/*
+ * Offline encoder (Sec. III-E Eq. 8, Eq. 10; Sec. III-C Eq. 3; Sec. III-D
+ * Eq. 5-7), deterministic and bit-identical to the fp64 definition:
+ *   1. score_j = g_j * sqrt(sum_i W_ij^2) (fp64, ascending i); P = the p
+ *      largest, ties to the lower column; stored ascending in prot_idx.
+ *   2. per protected column: scale = fp16(max_i |W_ij| / 127),
+ *      q8 = clamp(rint_even(W_ij / scale), -127, 127) (0 if scale == 0).
+ *   3. stage loop on r = W with protected entries zeroed: n = fp16(||r_c||),
+ *      bits = (r_c < 0), r_c -= (+-) n / sqrt(8), protected entries reset
+ *      to zero before the next stage.
+ * W_bf16: [N][K] device, 16-byte aligned.  g: [K] float device (finite,
+ * >= 0) or NULL for g = 1.  L: host struct; its sizes are inputs, its five
+ * device buffers outputs (sized by bisco_encoded_sizes).  workspace: device,
+ * at least bisco_encode_workspace_bytes(N, K) bytes.  Non-finite weights or
+ * an fp16 overflow latch BISCO_ERR_RANGE in the device error word; the
+ * outputs are then unspecified.
+ */
+bisco_status bisco_encode(const uint16_t *W_bf16, const float *g, const bisco_layer *L,
+                          void *workspace, size_t workspace_bytes, bisco_stream_t stream);
+
+/*
+ * Decode-time matrix-vector product for B in [0, 16] activation rows:
+ *     y[b][i] = sum_j What[i][j] * x[b][j]        (Sec. III-F Eq. 12, Eq. 10)
+ * computed straight from the coded layer (the dense weight is never
+ * formed).  x_bf16: [B][K] device bf16 bits; activations are used as fp16,
+ * which is exact for 2^-24 <= |x| <= 65504 (larger magnitudes become inf).
+ * y: [B][N] float32 device, fully overwritten.  B == 0 is a no-op.
+ */
+bisco_status bisco_gemv(const bisco_layer *L, const uint16_t *x_bf16, int32_t B, float *y,
+                        bisco_stream_t stream);
+
+/*
+ * Prefill matrix product Y[m][i] = sum_j What[i][j] * X[m][j] for any M >= 0,
+ * with the same arithmetic contract as bisco_gemv.  X_bf16: [M][K] device;
+ * Y: [M][N] float32 device, fully overwritten.  workspace: device, at least
+ * bisco_gemm_workspace_bytes(M, N, K) bytes (may be NULL when that is 0).
+ */
+size_t bisco_gemm_workspace_bytes(int32_t M, int32_t N, int32_t K);
+bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M, float *Y,
+                        void *workspace, size_t workspace_bytes, bisco_stream_t stream);
+
+/*
+ * Synchronises `stream`, returns the device error word of the current device
+ * (BISCO_OK if clear) and clears it.  BISCO_ERR_CUDA if the synchronisation
+ * itself fails.
+ */
+bisco_status bisco_get_device_error(bisco_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BISCO_H */

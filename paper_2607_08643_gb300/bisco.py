@@ -1,0 +1,214 @@
+"""Thin ctypes binding of libbisco.so (include/bisco.h), same entry-point
+names.  It only marshals arguments: PyTorch supplies device memory and the
+stream; every step of the computation runs in the library's CUDA kernels.
+There is no fallback -- if the library is missing this module raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libbisco.so")
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_RANGE, ERR_CUDA, ERR_TIMEOUT = range(6)
+
+# Functions declared in include/bisco.h (kept in sync by tests/test_abi.py).
+EXPORTS = (
+    "bisco_abi_version", "bisco_status_string", "bisco_encoded_sizes",
+    "bisco_encode_workspace_bytes", "bisco_encode", "bisco_gemv",
+    "bisco_gemm_workspace_bytes", "bisco_gemm", "bisco_get_device_error",
+)
+
+
+class BiscoError(RuntimeError):
+    def __init__(self, code: int, where: str = ""):
+        self.code = code
+        super().__init__("%s: bisco status %d (%s)" % (where, code, status_string(code)))
+
+
+class bisco_layer(ctypes.Structure):
+    _fields_ = [
+        ("n_out", ctypes.c_int32), ("k_in", ctypes.c_int32), ("chunk_dim", ctypes.c_int32),
+        ("stages", ctypes.c_int32), ("n_protected", ctypes.c_int32),
+        ("protect_axis", ctypes.c_int32),
+        ("codes", ctypes.c_void_p), ("norms", ctypes.c_void_p), ("q8", ctypes.c_void_p),
+        ("q8_scale", ctypes.c_void_p), ("prot_idx", ctypes.c_void_p),
+    ]
+
+
+_lib = None
+
+
+def load(path: str = LIB_PATH):
+    """Loads the CUDA library; raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError("libbisco.so not built (run __graft_entry__.build())")
+    lib = ctypes.CDLL(path)
+    P, i32, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t
+    st = ctypes.c_int
+    Lp = ctypes.POINTER(bisco_layer)
+    lib.bisco_abi_version.restype = i32
+    lib.bisco_abi_version.argtypes = []
+    lib.bisco_status_string.restype = ctypes.c_char_p
+    lib.bisco_status_string.argtypes = [i32]
+    lib.bisco_encoded_sizes.restype = st
+    lib.bisco_encoded_sizes.argtypes = [i32, i32, i32, i32, i32, ctypes.POINTER(sz)]
+    lib.bisco_encode_workspace_bytes.restype = sz
+    lib.bisco_encode_workspace_bytes.argtypes = [i32, i32]
+    lib.bisco_encode.restype = st
+    lib.bisco_encode.argtypes = [P, P, Lp, P, sz, P]
+    lib.bisco_gemv.restype = st
+    lib.bisco_gemv.argtypes = [Lp, P, i32, P, P]
+    lib.bisco_gemm_workspace_bytes.restype = sz
+    lib.bisco_gemm_workspace_bytes.argtypes = [i32, i32, i32]
+    lib.bisco_gemm.restype = st
+    lib.bisco_gemm.argtypes = [Lp, P, i32, P, P, sz, P]
+    lib.bisco_get_device_error.restype = st
+    lib.bisco_get_device_error.argtypes = [P]
+    _lib = lib
+    return lib
+
+
+def status_string(code: int) -> str:
+    return load().bisco_status_string(int(code)).decode()
+
+
+def _check(code: int, where: str):
+    if code != OK:
+        raise BiscoError(code, where)
+
+
+def _stream(stream):
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def bisco_abi_version() -> int:
+    return int(load().bisco_abi_version())
+
+
+def bisco_encoded_sizes(N, K, S, p, d=8):
+    out = (ctypes.c_size_t * 5)()
+    _check(load().bisco_encoded_sizes(N, K, d, S, p, out), "bisco_encoded_sizes")
+    return [int(v) for v in out]
+
+
+def bisco_encode_workspace_bytes(N, K) -> int:
+    return int(load().bisco_encode_workspace_bytes(N, K))
+
+
+def bisco_gemm_workspace_bytes(M, N, K) -> int:
+    return int(load().bisco_gemm_workspace_bytes(M, N, K))
+
+
+class Layer:
+    """A coded layer in device memory (torch tensors) plus its C struct."""
+
+    def __init__(self, N, K, S, p, device="cuda", d=8):
+        import torch
+        sizes = bisco_encoded_sizes(N, K, S, p, d)
+        self.N, self.K, self.S, self.p = N, K, S, p
+        self.p_pad = (p + 15) // 16 * 16
+        dev = torch.device(device)
+        self.codes = torch.empty((S, N, K // 8), dtype=torch.uint8, device=dev)
+        self.norms = torch.empty((S, N, K // 8), dtype=torch.int16, device=dev)
+        self.q8 = torch.empty((N, max(self.p_pad, 16)), dtype=torch.int8, device=dev)
+        self.scale = torch.empty((max(p, 8),), dtype=torch.int16, device=dev)
+        self.idx = torch.empty((max(p, 4),), dtype=torch.int32, device=dev)
+        assert sizes[0] == self.codes.numel() and sizes[1] == 2 * self.norms.numel()
+        self.c = bisco_layer(N, K, d, S, p, 0, self.codes.data_ptr(), self.norms.data_ptr(),
+                             self.q8.data_ptr(), self.scale.data_ptr(), self.idx.data_ptr())
+
+    @property
+    def compressed_bytes(self) -> int:
+        """Algorithmic payload: signs + norms + unpadded q8 + scales + indices."""
+        return self.S * self.N * (self.K // 8) * 3 + self.N * self.p + 6 * self.p
+
+    def to_numpy(self):
+        """Host copy in the oracle's dict layout."""
+        p = self.p
+        return dict(N=self.N, K=self.K, S=self.S, p=p,
+                    codes=self.codes.cpu().numpy(),
+                    norms=self.norms.cpu().numpy().view("uint16"),
+                    q8=self.q8[:, :self.p_pad].cpu().numpy(),
+                    scale=self.scale[:p].cpu().numpy().view("uint16"),
+                    idx=self.idx[:p].cpu().numpy())
+
+    @classmethod
+    def from_numpy(cls, L, device="cuda"):
+        import numpy as np
+        import torch
+        obj = cls(L["N"], L["K"], L["S"], L["p"], device)
+        obj.codes.copy_(torch.from_numpy(np.ascontiguousarray(L["codes"])))
+        obj.norms.copy_(torch.from_numpy(np.ascontiguousarray(L["norms"]).view(np.int16)))
+        if L["p"]:
+            obj.q8[:, :obj.p_pad].copy_(torch.from_numpy(np.ascontiguousarray(L["q8"])))
+            obj.scale[:L["p"]].copy_(torch.from_numpy(np.ascontiguousarray(L["scale"]).view(np.int16)))
+            obj.idx[:L["p"]].copy_(torch.from_numpy(np.ascontiguousarray(L["idx"])))
+        return obj
+
+
+def bisco_encode(W_bits, S, p, g=None, workspace=None, stream=None) -> Layer:
+    """Encodes a device tensor of bf16 bits [N][K] (int16 or bfloat16)."""
+    import torch
+    if W_bits.dtype == torch.bfloat16:
+        W_bits = W_bits.view(torch.int16)
+    assert W_bits.is_cuda and W_bits.is_contiguous() and W_bits.dim() == 2
+    N, K = W_bits.shape
+    L = Layer(N, K, S, p, W_bits.device)
+    need = bisco_encode_workspace_bytes(N, K)
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=W_bits.device)
+    if g is not None:
+        assert g.dtype == torch.float32 and g.is_cuda and g.numel() == K
+    _check(load().bisco_encode(_ptr(W_bits), _ptr(g), ctypes.byref(L.c), _ptr(workspace),
+                               workspace.numel(), _stream(stream)), "bisco_encode")
+    return L
+
+
+def bisco_gemv(L: Layer, x_bits, y=None, stream=None):
+    """y[B][N] (float32) = x What^T for B <= 16 activation rows (bf16 bits)."""
+    import torch
+    if x_bits.dtype == torch.bfloat16:
+        x_bits = x_bits.view(torch.int16)
+    if x_bits.dim() == 1:
+        x_bits = x_bits.unsqueeze(0)
+    B = x_bits.shape[0]
+    assert x_bits.is_contiguous() and x_bits.shape[1] == L.K
+    if y is None:
+        y = torch.empty((B, L.N), dtype=torch.float32, device=x_bits.device)
+    _check(load().bisco_gemv(ctypes.byref(L.c), _ptr(x_bits), B, _ptr(y), _stream(stream)),
+           "bisco_gemv")
+    return y
+
+
+def bisco_gemm(L: Layer, X_bits, Y=None, workspace=None, stream=None):
+    """Y[M][N] (float32) = X What^T for any M (prefill)."""
+    import torch
+    if X_bits.dtype == torch.bfloat16:
+        X_bits = X_bits.view(torch.int16)
+    M = X_bits.shape[0]
+    assert X_bits.is_contiguous() and X_bits.shape[1] == L.K
+    if Y is None:
+        Y = torch.empty((M, L.N), dtype=torch.float32, device=X_bits.device)
+    need = bisco_gemm_workspace_bytes(M, L.N, L.K)
+    if need and workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=X_bits.device)
+    nbytes = 0 if workspace is None else workspace.numel()
+    _check(load().bisco_gemm(ctypes.byref(L.c), _ptr(X_bits), M, _ptr(Y), _ptr(workspace),
+                             nbytes, _stream(stream)), "bisco_gemm")
+    return Y
+
+
+def bisco_get_device_error(stream=None) -> int:
+    return int(load().bisco_get_device_error(_stream(stream)))

@@ -1,0 +1,214 @@
+// api.cu -- the extern "C" entry points declared in include/bisco.h:
+// argument validation, the per-device error word, tensor-map encoding and
+// dispatch to the kernels in encode.cu / gemv.cu / gemm.cu.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+#include <stdint.h>
+
+#include <mutex>
+
+#include "bisco_host.h"
+
+namespace bisco {
+
+__device__ int g_device_error;
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+int *g_err_ptr[kMaxDevices] = {};
+int g_sms[kMaxDevices] = {};
+PFN_cuTensorMapEncodeTiled_v12000 g_encode_tiled = nullptr;
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int current_device() {
+    int d = -1;
+    if (cudaGetDevice(&d) != cudaSuccess || d < 0 || d >= kMaxDevices) return -1;
+    return d;
+}
+
+// Validates the sizes of a layer; buffers too when check_buffers.
+bisco_status check_layer(const bisco_layer *L, bool check_buffers) {
+    if (!L) return BISCO_ERR_INVALID_ARG;
+    if (L->n_out < 1 || L->k_in < 8 || L->k_in % 8 != 0) return BISCO_ERR_INVALID_ARG;
+    if (L->stages < 1 || L->stages > 3) return BISCO_ERR_INVALID_ARG;
+    if (L->n_protected < 0 || L->n_protected > L->k_in) return BISCO_ERR_INVALID_ARG;
+    if (L->protect_axis != 0 && L->protect_axis != 1) return BISCO_ERR_INVALID_ARG;
+    if (L->chunk_dim != 8 || L->protect_axis != 0) return BISCO_ERR_UNSUPPORTED;
+    if (static_cast<int64_t>(L->n_out) * L->k_in > (int64_t(1) << 40)) return BISCO_ERR_INVALID_ARG;
+    if (!check_buffers) return BISCO_OK;
+    if (!L->codes || !L->norms || !aligned16(L->codes) || !aligned16(L->norms))
+        return BISCO_ERR_INVALID_ARG;
+    if (L->n_protected > 0) {
+        if (!L->q8 || !L->q8_scale || !L->prot_idx) return BISCO_ERR_INVALID_ARG;
+        if (!aligned16(L->q8) || !aligned16(L->q8_scale) || !aligned16(L->prot_idx))
+            return BISCO_ERR_INVALID_ARG;
+    }
+    return BISCO_OK;
+}
+
+}  // namespace
+
+int *device_error_word(bisco_status *st) {
+    const int d = current_device();
+    if (d < 0) {
+        *st = BISCO_ERR_CUDA;
+        return nullptr;
+    }
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (!g_err_ptr[d]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_device_error) != cudaSuccess) {
+            *st = BISCO_ERR_CUDA;
+            return nullptr;
+        }
+        g_err_ptr[d] = static_cast<int *>(p);
+    }
+    *st = BISCO_OK;
+    return g_err_ptr[d];
+}
+
+int num_sms() {
+    const int d = current_device();
+    if (d < 0) return 148;
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (!g_sms[d]) {
+        int v = 0;
+        if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, d) != cudaSuccess || v <= 0)
+            v = 148;
+        g_sms[d] = v;
+    }
+    return g_sms[d];
+}
+
+bool encode_tensor_map(CUtensorMap *map, CUtensorMapDataType dtype, int rank, void *base,
+                       const uint64_t *dims, const uint64_t *strides_bytes, const uint32_t *box,
+                       CUtensorMapSwizzle swizzle) {
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        if (!g_encode_tiled) {
+            cudaDriverEntryPointQueryResult q;
+            void *fn = nullptr;
+            if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                 cudaEnableDefault, &q) != cudaSuccess ||
+                q != cudaDriverEntryPointSuccess || !fn)
+                return false;
+            g_encode_tiled = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+        }
+    }
+    cuuint64_t gdim[5], gstr[4];
+    cuuint32_t bdim[5], estr[5];
+    for (int i = 0; i < rank; ++i) {
+        gdim[i] = dims[i];
+        bdim[i] = box[i];
+        estr[i] = 1;
+        if (i + 1 < rank) gstr[i] = strides_bytes[i];
+    }
+    const CUresult r = g_encode_tiled(map, dtype, static_cast<cuuint32_t>(rank), base, gdim, gstr,
+                                      bdim, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
+                                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+}  // namespace bisco
+
+using namespace bisco;
+
+extern "C" {
+
+int32_t bisco_abi_version(void) { return BISCO_ABI_VERSION; }
+
+const char *bisco_status_string(int32_t status) {
+    switch (status) {
+        case BISCO_OK: return "ok";
+        case BISCO_ERR_INVALID_ARG: return "invalid argument";
+        case BISCO_ERR_UNSUPPORTED: return "unsupported configuration";
+        case BISCO_ERR_RANGE: return "value out of range (non-finite weight or fp16 overflow)";
+        case BISCO_ERR_CUDA: return "CUDA runtime error";
+        case BISCO_ERR_TIMEOUT: return "bounded device wait expired";
+        default: return "unknown status";
+    }
+}
+
+bisco_status bisco_encoded_sizes(int32_t N, int32_t K, int32_t d, int32_t S, int32_t p,
+                                 size_t out_bytes[5]) {
+    if (!out_bytes) return BISCO_ERR_INVALID_ARG;
+    if (N < 1 || K < 8 || K % 8 != 0 || S < 1 || S > 3 || p < 0 || p > K)
+        return BISCO_ERR_INVALID_ARG;
+    if (d != 8) return BISCO_ERR_UNSUPPORTED;
+    const size_t C = static_cast<size_t>(K) / 8;
+    const size_t p_pad = (static_cast<size_t>(p) + 15) / 16 * 16;
+    out_bytes[0] = static_cast<size_t>(S) * N * C;
+    out_bytes[1] = static_cast<size_t>(S) * N * C * 2;
+    out_bytes[2] = static_cast<size_t>(N) * p_pad;
+    out_bytes[3] = static_cast<size_t>(p) * 2;
+    out_bytes[4] = static_cast<size_t>(p) * 4;
+    return BISCO_OK;
+}
+
+size_t bisco_encode_workspace_bytes(int32_t N, int32_t K) { return encode_workspace_bytes(N, K); }
+
+bisco_status bisco_encode(const uint16_t *W_bf16, const float *g, const bisco_layer *L,
+                          void *workspace, size_t workspace_bytes, bisco_stream_t stream) {
+    bisco_status st = check_layer(L, true);
+    if (st != BISCO_OK) return st;
+    if (!W_bf16 || !aligned16(W_bf16) || (g && (reinterpret_cast<uintptr_t>(g) & 3u)))
+        return BISCO_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace) ||
+        workspace_bytes < encode_workspace_bytes(L->n_out, L->k_in))
+        return BISCO_ERR_INVALID_ARG;
+    int *err = device_error_word(&st);
+    if (!err) return st;
+    return launch_encode(W_bf16, g, *L, workspace, err, reinterpret_cast<cudaStream_t>(stream));
+}
+
+bisco_status bisco_gemv(const bisco_layer *L, const uint16_t *x_bf16, int32_t B, float *y,
+                        bisco_stream_t stream) {
+    bisco_status st = check_layer(L, true);
+    if (st != BISCO_OK) return st;
+    if (B < 0 || B > 16) return BISCO_ERR_INVALID_ARG;
+    if (B == 0) return BISCO_OK;
+    if (!x_bf16 || !y || !aligned16(x_bf16) || !aligned16(y)) return BISCO_ERR_INVALID_ARG;
+    int *err = device_error_word(&st);
+    if (!err) return st;
+    return launch_gemv(*L, x_bf16, B, y, err, reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t bisco_gemm_workspace_bytes(int32_t M, int32_t N, int32_t K) {
+    if (M < 0 || N < 1 || K < 8 || K % 8) return 0;
+    return gemm_workspace_bytes(M, N, K);
+}
+
+bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M, float *Y,
+                        void *workspace, size_t workspace_bytes, bisco_stream_t stream) {
+    bisco_status st = check_layer(L, true);
+    if (st != BISCO_OK) return st;
+    if (M < 0) return BISCO_ERR_INVALID_ARG;
+    if (M == 0) return BISCO_OK;
+    if (!X_bf16 || !Y || !aligned16(X_bf16) || !aligned16(Y)) return BISCO_ERR_INVALID_ARG;
+    const size_t need = gemm_workspace_bytes(M, L->n_out, L->k_in);
+    if (need && (!workspace || !aligned16(workspace) || workspace_bytes < need))
+        return BISCO_ERR_INVALID_ARG;
+    int *err = device_error_word(&st);
+    if (!err) return st;
+    return launch_gemm(*L, X_bf16, M, Y, workspace, workspace_bytes, err,
+                       reinterpret_cast<cudaStream_t>(stream));
+}
+
+bisco_status bisco_get_device_error(bisco_stream_t stream) {
+    bisco_status st;
+    int *err = device_error_word(&st);
+    if (!err) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaStreamSynchronize(s) != cudaSuccess) return BISCO_ERR_CUDA;
+    int v = 0;
+    if (cudaMemcpy(&v, err, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return BISCO_ERR_CUDA;
+    if (v != 0 && cudaMemset(err, 0, sizeof v) != cudaSuccess) return BISCO_ERR_CUDA;
+    return static_cast<bisco_status>(v);
+}
+
+}  // extern "C"

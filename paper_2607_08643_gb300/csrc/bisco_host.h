@@ -1,0 +1,33 @@
+// bisco_host.h -- host-side declarations shared by the library's
+// translation units (not part of the public ABI).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/bisco.h"
+
+namespace bisco {
+
+// Device error word of the current device (set up on first use).
+int *device_error_word(bisco_status *st);
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point.
+bool encode_tensor_map(CUtensorMap *map, CUtensorMapDataType dtype, int rank, void *base,
+                       const uint64_t *dims, const uint64_t *strides_bytes, const uint32_t *box,
+                       CUtensorMapSwizzle swizzle);
+
+int num_sms();
+
+size_t encode_workspace_bytes(int N, int K);
+bisco_status launch_encode(const uint16_t *W, const float *g, const bisco_layer &L,
+                           void *workspace, int *err, cudaStream_t stream);
+bisco_status launch_gemv(const bisco_layer &L, const uint16_t *x, int B, float *y, int *err,
+                         cudaStream_t stream);
+size_t gemm_workspace_bytes(int M, int N, int K);
+bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *Y,
+                         void *workspace, size_t ws_bytes, int *err, cudaStream_t stream);
+
+}  // namespace bisco

@@ -1,0 +1,246 @@
+// encode.cu -- offline BiSCo encoder on the GPU (Sec. III-E Eq. 8 and
+// Eq. 10, Sec. III-C Eq. 3, Sec. III-D Eq. 5-7).
+//
+// Every floating-point step is binary64 with an explicit rounding intrinsic
+// (no FMA contraction; this file is also compiled with --fmad=false), sums
+// run in a fixed order, and narrowing to binary16 uses the hardware's
+// round-to-nearest-even conversion, so the produced bytes are a pure
+// function of the input bits.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "bisco_dev.cuh"
+#include "bisco_host.h"
+
+namespace bisco {
+namespace {
+
+__device__ __forceinline__ uint16_t f64_to_f16_rn(double x) {
+    unsigned short r;
+    asm("cvt.rn.f16.f64 %0, %1;" : "=h"(r) : "d"(x));
+    return r;
+}
+
+__device__ __forceinline__ double f16_to_f64(uint16_t h) {
+    return static_cast<double>(__half2float(__ushort_as_half(h)));
+}
+
+__device__ __forceinline__ double bf16_to_f64(uint16_t b) {
+    return static_cast<double>(__uint_as_float(static_cast<uint32_t>(b) << 16));
+}
+
+__device__ __forceinline__ bool bf16_nonfinite(uint16_t b) { return (b & 0x7F80u) == 0x7F80u; }
+
+// Eq. 8 score of every input column: g_j * sqrt(sum_{i ascending} W_ij^2).
+// One thread per column; also rejects non-finite weights.
+__global__ void __launch_bounds__(128) k_colscore(const uint16_t *__restrict__ W,
+                                                  const float *__restrict__ g, int N, int K,
+                                                  double *__restrict__ score, int *err) {
+    const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    if (j >= K) return;
+    double sum = 0.0;
+    bool bad = false;
+    const uint16_t *col = W + j;
+    int i = 0;
+    for (; i + 8 <= N; i += 8) {
+        uint16_t b[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) b[u] = col[static_cast<int64_t>(i + u) * K];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            bad |= bf16_nonfinite(b[u]);
+            const double w = bf16_to_f64(b[u]);
+            sum = __dadd_rn(sum, __dmul_rn(w, w));
+        }
+    }
+    for (; i < N; ++i) {
+        const uint16_t b = col[static_cast<int64_t>(i) * K];
+        bad |= bf16_nonfinite(b);
+        const double w = bf16_to_f64(b);
+        sum = __dadd_rn(sum, __dmul_rn(w, w));
+    }
+    if (bad) latch_error(err, BISCO_ERR_RANGE);
+    double s = __dsqrt_rn(sum);
+    if (g) s = __dmul_rn(static_cast<double>(g[j]), s);
+    score[j] = s;
+}
+
+// Eq. 8 TopK, step 1: rank_j = number of columns that precede j in the
+// order (score descending, index ascending); column j is protected iff
+// rank_j < p.  One thread per column, scores staged through shared memory;
+// counting stops once every thread of the block has reached p.
+constexpr int kRankThreads = 256;
+constexpr int kRankTile = 2048;
+
+__global__ void __launch_bounds__(kRankThreads) k_rank(const double *__restrict__ score, int K,
+                                                       int p, int32_t *__restrict__ rank_out) {
+    __shared__ double s[kRankTile];
+    const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    const double sj = j < K ? score[j] : 0.0;
+    int rank = 0;
+    for (int q0 = 0; q0 < K; q0 += kRankTile) {
+        const int n = min(kRankTile, K - q0);
+        __syncthreads();
+        for (int q = threadIdx.x; q < n; q += blockDim.x) s[q] = score[q0 + q];
+        __syncthreads();
+        if (j < K && rank < p) {
+            for (int q = 0; q < n; ++q) {
+                const double sq = s[q];
+                rank += (sq > sj) || (sq == sj && q0 + q < j);
+            }
+        }
+        if (__syncthreads_and(j >= K || rank >= p)) break;
+    }
+    if (j < K) rank_out[j] = rank;
+}
+
+// Eq. 8 TopK, step 2 (one CTA): protected-column map and the ascending list
+// of protected columns, by an ordered compaction over contiguous ranges.
+constexpr int kCompactThreads = 1024;
+
+__global__ void __launch_bounds__(kCompactThreads) k_compact(const int32_t *__restrict__ rank,
+                                                             int K, int p,
+                                                             uint8_t *__restrict__ prot,
+                                                             int32_t *__restrict__ idx) {
+    __shared__ int counts[kCompactThreads];
+    const int per = (K + kCompactThreads - 1) / kCompactThreads;
+    const int j0 = min(K, static_cast<int>(threadIdx.x) * per);
+    const int j1 = min(K, j0 + per);
+    int mine = 0;
+    for (int j = j0; j < j1; ++j) {
+        const uint8_t f = rank[j] < p ? 1 : 0;
+        prot[j] = f;
+        mine += f;
+    }
+    counts[threadIdx.x] = mine;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int run = 0;
+        for (int t = 0; t < kCompactThreads; ++t) {
+            const int c = counts[t];
+            counts[t] = run;
+            run += c;
+        }
+    }
+    __syncthreads();
+    int pos = counts[threadIdx.x];
+    for (int j = j0; j < j1; ++j)
+        if (prot[j]) idx[pos++] = j;
+}
+
+// Eq. 10 per-channel 8-bit quantiser, one CTA per q8 column t < p_pad
+// (columns t >= p are the zero padding).
+__global__ void __launch_bounds__(256) k_q8(const uint16_t *__restrict__ W, int N, int K, int p,
+                                            int p_pad, const int32_t *__restrict__ idx,
+                                            int8_t *__restrict__ q8, uint16_t *__restrict__ scale,
+                                            int *err) {
+    const int t = blockIdx.x;
+    if (t >= p) {
+        for (int i = threadIdx.x; i < N; i += blockDim.x) q8[static_cast<int64_t>(i) * p_pad + t] = 0;
+        return;
+    }
+    const int j = idx[t];
+    double m = 0.0;
+    for (int i = threadIdx.x; i < N; i += blockDim.x)
+        m = fmax(m, fabs(bf16_to_f64(W[static_cast<int64_t>(i) * K + j])));
+    __shared__ double red[256];
+    red[threadIdx.x] = m;
+    __syncthreads();
+    for (int w = 128; w > 0; w >>= 1) {
+        if (threadIdx.x < w) red[threadIdx.x] = fmax(red[threadIdx.x], red[threadIdx.x + w]);
+        __syncthreads();
+    }
+    const uint16_t s16 = f64_to_f16_rn(__ddiv_rn(red[0], 127.0));
+    if ((s16 & 0x7C00u) == 0x7C00u) {
+        if (threadIdx.x == 0) latch_error(err, BISCO_ERR_RANGE);
+        return;
+    }
+    if (threadIdx.x == 0) scale[t] = s16;
+    const double s = f16_to_f64(s16);
+    for (int i = threadIdx.x; i < N; i += blockDim.x) {
+        double q = 0.0;
+        if (s != 0.0) {
+            q = rint(__ddiv_rn(bf16_to_f64(W[static_cast<int64_t>(i) * K + j]), s));
+            q = fmin(127.0, fmax(-127.0, q));
+        }
+        q8[static_cast<int64_t>(i) * p_pad + t] = static_cast<int8_t>(static_cast<int>(q));
+    }
+}
+
+// Eq. 3 + Eq. 5-7: one thread per (row, chunk); S sign/norm stages on the
+// residual, protected entries held at zero in every stage.
+__global__ void __launch_bounds__(256) k_stages(const uint16_t *__restrict__ W, int N, int K, int S,
+                                                const uint8_t *__restrict__ prot,
+                                                uint8_t *__restrict__ codes,
+                                                uint16_t *__restrict__ norms, int *err) {
+    const int C = K / 8;
+    const int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (e >= static_cast<int64_t>(N) * C) return;
+    const int i = static_cast<int>(e / C);
+    const int c = static_cast<int>(e % C);
+    const uint4 raw = *reinterpret_cast<const uint4 *>(W + static_cast<int64_t>(i) * K + 8 * c);
+    const uint2 pm = *reinterpret_cast<const uint2 *>(prot + 8 * c);
+    const uint32_t wv[4] = {raw.x, raw.y, raw.z, raw.w};
+    const uint32_t pv[2] = {pm.x, pm.y};
+    bool pr[8];
+    double v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        pr[k] = ((pv[k / 4] >> (8 * (k % 4))) & 0xFFu) != 0;
+        const uint16_t b = static_cast<uint16_t>(wv[k / 2] >> (16 * (k % 2)));
+        v[k] = pr[k] ? 0.0 : bf16_to_f64(b);
+    }
+    const double inv_sqrt8 = __ddiv_rn(1.0, __dsqrt_rn(8.0));
+    for (int s = 0; s < S; ++s) {
+        double sum = __dmul_rn(v[0], v[0]);
+#pragma unroll
+        for (int k = 1; k < 8; ++k) sum = __dadd_rn(sum, __dmul_rn(v[k], v[k]));
+        const uint16_t n16 = f64_to_f16_rn(__dsqrt_rn(sum));
+        if ((n16 & 0x7C00u) == 0x7C00u) latch_error(err, BISCO_ERR_RANGE);
+        uint32_t bits = 0;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) bits |= (v[k] < 0.0 ? 1u : 0u) << k;
+        const double t = __dmul_rn(f16_to_f64(n16), inv_sqrt8);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const double rhat = ((bits >> k) & 1u) ? -t : t;
+            v[k] = pr[k] ? 0.0 : __dsub_rn(v[k], rhat);
+        }
+        const int64_t o = (static_cast<int64_t>(s) * N + i) * C + c;
+        codes[o] = static_cast<uint8_t>(bits);
+        norms[o] = n16;
+    }
+}
+
+}  // namespace
+
+static size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+size_t encode_workspace_bytes(int N, int K) {
+    if (N < 1 || K < 8 || K % 8) return 0;
+    const size_t k = static_cast<size_t>(K);
+    return round_up(8 * k, 256) + round_up(4 * k, 256) + round_up(k, 256);
+}
+
+bisco_status launch_encode(const uint16_t *W, const float *g, const bisco_layer &L,
+                           void *workspace, int *err, cudaStream_t stream) {
+    const int N = L.n_out, K = L.k_in, S = L.stages, p = L.n_protected;
+    const int p_pad = (p + 15) / 16 * 16;
+    const size_t k = static_cast<size_t>(K);
+    unsigned char *ws = static_cast<unsigned char *>(workspace);
+    double *score = reinterpret_cast<double *>(ws);
+    int32_t *rank = reinterpret_cast<int32_t *>(ws + round_up(8 * k, 256));
+    uint8_t *prot = ws + round_up(8 * k, 256) + round_up(4 * k, 256);
+
+    k_colscore<<<(K + 127) / 128, 128, 0, stream>>>(W, g, N, K, score, err);
+    k_rank<<<(K + kRankThreads - 1) / kRankThreads, kRankThreads, 0, stream>>>(score, K, p, rank);
+    k_compact<<<1, kCompactThreads, 0, stream>>>(rank, K, p, prot, L.prot_idx);
+    if (p_pad > 0)
+        k_q8<<<p_pad, 256, 0, stream>>>(W, N, K, p, p_pad, L.prot_idx, L.q8, L.q8_scale, err);
+    const int64_t chunks = static_cast<int64_t>(N) * (K / 8);
+    k_stages<<<static_cast<unsigned>((chunks + 255) / 256), 256, 0, stream>>>(
+        W, N, K, S, prot, L.codes, L.norms, err);
+    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+}
+
+}  // namespace bisco

@@ -1,0 +1,111 @@
+"""C-ABI checks that need no GPU: the library loads, exports every function
+include/bisco.h declares, and rejects bad arguments before touching the
+device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import oracle
+from paper_2607_08643_gb300 import bisco, synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "bisco.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2607_08643_gb300 import build
+    build.build()
+    return bisco.load()
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(bisco_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_header_declarations_are_exported(lib):
+    names = declared_functions()
+    assert set(names) == set(bisco.EXPORTS)
+    for n in names:
+        assert getattr(lib, n) is not None
+
+
+def test_abi_version_and_status_strings(lib):
+    assert bisco.bisco_abi_version() == 100
+    for code in range(6):
+        assert bisco.status_string(code)
+    assert bisco.status_string(99) == "unknown status"
+
+
+def test_encoded_sizes_match_oracle_accounting(lib):
+    for (N, K, S, rho) in [(1024, 1024, 2, 1), (4096, 4096, 2, 1), (12288, 4096, 3, 2),
+                           (4096, 12288, 3, 2), (37, 136, 1, 0)]:
+        p = synth.protected_count(K, rho)
+        assert bisco.bisco_encoded_sizes(N, K, S, p) == oracle.encoded_sizes(N, K, S, p)
+
+
+@pytest.mark.parametrize("args,code", [
+    ((0, 64, 8, 1, 0), bisco.ERR_INVALID_ARG),
+    ((4, 60, 8, 1, 0), bisco.ERR_INVALID_ARG),
+    ((4, 64, 8, 4, 0), bisco.ERR_INVALID_ARG),
+    ((4, 64, 8, 1, 65), bisco.ERR_INVALID_ARG),
+    ((4, 64, 16, 1, 0), bisco.ERR_UNSUPPORTED),
+])
+def test_encoded_sizes_rejects(lib, args, code):
+    out = (ctypes.c_size_t * 5)()
+    assert lib.bisco_encoded_sizes(*args, out) == code
+
+
+def _fake_layer(**kw):
+    base = dict(n_out=64, k_in=256, chunk_dim=8, stages=2, n_protected=3, protect_axis=0,
+                codes=0x10000, norms=0x20000, q8=0x30000, q8_scale=0x40000, prot_idx=0x50000)
+    base.update(kw)
+    return bisco.bisco_layer(**base)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(k_in=252), bisco.ERR_INVALID_ARG),
+    (dict(stages=0), bisco.ERR_INVALID_ARG),
+    (dict(n_protected=-1), bisco.ERR_INVALID_ARG),
+    (dict(chunk_dim=16), bisco.ERR_UNSUPPORTED),
+    (dict(protect_axis=1), bisco.ERR_UNSUPPORTED),
+    (dict(protect_axis=2), bisco.ERR_INVALID_ARG),
+    (dict(codes=0x10004), bisco.ERR_INVALID_ARG),
+    (dict(codes=0), bisco.ERR_INVALID_ARG),
+    (dict(q8=0), bisco.ERR_INVALID_ARG),
+])
+def test_layer_validation_before_any_device_call(lib, kw, code):
+    L = _fake_layer(**kw)
+    x = ctypes.c_void_p(0x60000)
+    y = ctypes.c_void_p(0x70000)
+    assert lib.bisco_gemv(ctypes.byref(L), x, 1, y, None) == code
+    assert lib.bisco_gemm(ctypes.byref(L), x, 4, y, None, 0, None) == code
+    assert lib.bisco_encode(x, None, ctypes.byref(L), ctypes.c_void_p(0x80000), 1 << 20, None) == code
+
+
+def test_call_argument_validation(lib):
+    L = _fake_layer()
+    x, y = ctypes.c_void_p(0x60000), ctypes.c_void_p(0x70000)
+    assert lib.bisco_gemv(ctypes.byref(L), x, 17, y, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_gemv(ctypes.byref(L), x, -1, y, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_gemv(ctypes.byref(L), ctypes.c_void_p(0x60002), 1, y, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_gemv(ctypes.byref(L), None, 1, y, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_gemv(None, x, 1, y, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_gemv(ctypes.byref(L), x, 0, y, None) == bisco.OK          # empty batch
+    assert lib.bisco_gemm(ctypes.byref(L), x, -3, y, None, 0, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_gemm(ctypes.byref(L), x, 0, y, None, 0, None) == bisco.OK  # empty prefill
+    # encode: workspace too small / misaligned weights / misaligned g
+    ws = bisco.bisco_encode_workspace_bytes(64, 256)
+    assert ws >= 64 * 256 // 8 and ws % 256 == 0
+    assert lib.bisco_encode(x, None, ctypes.byref(L), ctypes.c_void_p(0x80000), ws - 1, None) \
+        == bisco.ERR_INVALID_ARG
+    assert lib.bisco_encode(ctypes.c_void_p(0x60008), None, ctypes.byref(L),
+                            ctypes.c_void_p(0x80000), ws, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_encode(x, ctypes.c_void_p(0x90002), ctypes.byref(L),
+                            ctypes.c_void_p(0x80000), ws, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_encode_workspace_bytes(0, 64) == 0
+    assert lib.bisco_gemm_workspace_bytes(16, 64, 12) == 0

@@ -1,0 +1,72 @@
+"""bisco_gemm (prefill) against the fp64 oracle, and against bisco_gemv."""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2607_08643_gb300 import synth
+
+from _helpers import TOL, max_rel_rows, sample_rows, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def env():
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_08643_gb300 import bisco
+    dev = torch.device("cuda:0")
+    torch.cuda.set_device(dev)
+    return bisco, dev
+
+
+def run_gemm(env, Lref, X):
+    import torch
+    bisco, dev = env
+    L = bisco.Layer.from_numpy(Lref, dev)
+    Y = bisco.bisco_gemm(L, to_dev(X, dev))
+    torch.cuda.synchronize()
+    assert bisco.bisco_get_device_error() == 0
+    return Y.cpu().numpy(), L
+
+
+@pytest.mark.parametrize("N,K,S,p,M", [
+    (1024, 1024, 2, 11, 2048),      # single layer 1024 x 1024, 2048 tokens
+    (1024, 1024, 2, 11, 37),        # ragged token count
+    (200, 1536, 3, 20, 130),        # ragged N, three stages
+    (64, 1000, 2, 10, 20),          # K % 128 != 0
+    (128, 512, 1, 0, 1),            # one token
+])
+def test_gemm_matches_oracle(env, N, K, S, p, M):
+    W = synth.layer_weights(N, K, seed=N ^ K)
+    X = synth.activations(M, K, seed=M)
+    Lref = oracle.encode(W, S=S, p=p)
+    Y, _ = run_gemm(env, Lref, X)
+    assert max_rel_rows(Y, oracle.gemv(Lref, X)) <= TOL
+
+
+@pytest.mark.parametrize("name", ["q_proj", "k_proj", "down_proj"])
+def test_gemm_full_size_sampled(env, name):
+    N, K = synth.QWEN3_8B_SHAPES[name]
+    S, p = 2, synth.protected_count(K, 1)
+    W = synth.layer_weights(N, K, seed=23)
+    X = synth.activations(2048, K, seed=24)
+    Lref = oracle.encode(W, S=S, p=p)
+    Y, _ = run_gemm(env, Lref, X)
+    rows = sample_rows(N, n=12)
+    toks = sample_rows(2048, n=40, seed=1)
+    ref = oracle.apply_rows(Lref, rows, X[toks])
+    assert max_rel_rows(Y[toks][:, rows], ref) <= TOL
+
+
+def test_gemm_equals_gemv(env):
+    import torch
+    bisco, dev = env
+    N, K, S, p = 512, 2048, 2, 21
+    W = synth.layer_weights(N, K, seed=31)
+    X = synth.activations(16, K, seed=32)
+    Lref = oracle.encode(W, S=S, p=p)
+    Y, L = run_gemm(env, Lref, X)
+    y = bisco.bisco_gemv(L, to_dev(X, dev)).cpu().numpy()
+    assert max_rel_rows(Y, y) <= 1e-4

@@ -1,0 +1,123 @@
+"""bisco_gemv (decode, B <= 16) against the fp64 oracle.
+
+Parity bar: per activation row, max|y - y_ref| / max|y_ref| <= 2e-3.  The
+oracle encodes its own layer and the GPU runs on a copy of those bytes, so
+no oracle input comes from the CUDA path."""
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2607_08643_gb300 import synth
+
+from _helpers import TOL, max_rel_rows, sample_rows, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def env():
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_08643_gb300 import bisco
+    dev = torch.device("cuda:0")
+    torch.cuda.set_device(dev)
+    return bisco, dev
+
+
+def run_gemv(env, Lref, X, plan=None):
+    import torch
+    bisco, dev = env
+    L = bisco.Layer.from_numpy(Lref, dev)
+    old = os.environ.get("BISCO_GEMV_PLAN")
+    if plan:
+        os.environ["BISCO_GEMV_PLAN"] = plan
+    try:
+        y = bisco.bisco_gemv(L, to_dev(X, dev))
+    finally:
+        if plan:
+            if old is None:
+                del os.environ["BISCO_GEMV_PLAN"]
+            else:
+                os.environ["BISCO_GEMV_PLAN"] = old
+    torch.cuda.synchronize()
+    assert bisco.bisco_get_device_error() == 0
+    return y.cpu().numpy()
+
+
+@pytest.mark.parametrize("N,K,S,p,B,dist", [
+    (1024, 1024, 2, 11, 1, "normal"),     # single layer 1024 x 1024, batch 1
+    (1024, 1024, 2, 11, 16, "normal"),
+    (100, 1536, 3, 20, 3, "t4"),          # ragged N, three stages
+    (256, 4096, 2, 41, 9, "normal"),      # B = 9: two MMA n-tiles
+    (64, 1000, 2, 10, 4, "normal"),       # K % 128 != 0
+    (48, 512, 1, 0, 1, "normal"),         # S = 1, no protection
+    (32, 640, 2, 640, 2, "normal"),       # every column protected
+    (16, 128, 3, 2, 16, "t4"),            # one slab, ragged slab
+    (200, 2176, 2, 23, 8, "t4"),          # K not a multiple of the 512 slab
+])
+def test_gemv_matches_oracle(env, N, K, S, p, B, dist):
+    W = synth.layer_weights(N, K, seed=N + K, dist=dist)
+    X = synth.activations(B, K, seed=B)
+    Lref = oracle.encode(W, S=S, p=p)
+    y = run_gemv(env, Lref, X)
+    assert max_rel_rows(y, oracle.gemv(Lref, X)) <= TOL
+
+
+@pytest.mark.parametrize("plan", ["1,1,2", "1,4,3", "2,2,4", "4,8,2", "4,3,2", "2,5,3",
+                                  "1,2,8", "4,1,2"])
+@pytest.mark.parametrize("B", [1, 5, 16])
+def test_gemv_every_tiling(env, plan, B):
+    """All tile heights, cluster split-K factors (including ranks left with
+    no slab) and ring depths give the same answer."""
+    N, K, S, p = 208, 4096, 2, 41
+    W = synth.layer_weights(N, K, seed=2)
+    X = synth.activations(B, K, seed=3)
+    Lref = oracle.encode(W, S=S, p=p)
+    y = run_gemv(env, Lref, X, plan=plan)
+    assert max_rel_rows(y, oracle.gemv(Lref, X)) <= TOL
+
+
+@pytest.mark.parametrize("name,S,rho,B", [("q_proj", 2, 1, 1), ("q_proj", 2, 1, 16),
+                                          ("k_proj", 2, 1, 1), ("o_proj", 2, 1, 4),
+                                          ("gate_proj", 3, 2, 1), ("down_proj", 3, 2, 1),
+                                          ("down_proj", 2, 1, 16)])
+def test_gemv_full_size_sampled_rows(env, name, S, rho, B):
+    N, K = synth.QWEN3_8B_SHAPES[name]
+    p = synth.protected_count(K, rho)
+    W = synth.layer_weights(N, K, seed=17, dist="t4" if S == 3 else "normal")
+    X = synth.activations(B, K, seed=18)
+    Lref = oracle.encode(W, S=S, p=p)
+    y = run_gemv(env, Lref, X)
+    rows = sample_rows(N)
+    assert max_rel_rows(y[:, rows], oracle.apply_rows(Lref, rows, X)) <= TOL
+
+
+def test_gemv_one_hot_columns_and_linearity(env):
+    """One-hot activations return columns of What (the protected ones exactly
+    scale * q8); the map is linear in x."""
+    N, K, S, p = 64, 512, 2, 6
+    W = synth.layer_weights(N, K, seed=5)
+    Lref = oracle.encode(W, S=S, p=p)
+    cols = [0, 7, 255, 511, int(Lref["idx"][0]), int(Lref["idx"][-1])]
+    X = np.zeros((len(cols), K), np.uint16)
+    for b, j in enumerate(cols):
+        X[b, j] = 0x3F80                                   # 1.0
+    y = run_gemv(env, Lref, X)
+    What = oracle.decode_rows(Lref)
+    for b, j in enumerate(cols):
+        assert np.allclose(y[b], What[:, j], rtol=0, atol=1e-6 * np.abs(What[:, j]).max())
+    X2 = synth.activations(2, K, seed=6)
+    y2 = run_gemv(env, Lref, X2)
+    ref = oracle.gemv(Lref, X2)
+    assert max_rel_rows(y2, ref) <= TOL
+
+
+def test_gemv_zero_and_tiny_activations(env):
+    N, K, S, p = 32, 256, 2, 3
+    W = synth.layer_weights(N, K, seed=8)
+    Lref = oracle.encode(W, S=S, p=p)
+    y = run_gemv(env, Lref, np.zeros((2, K), np.uint16))
+    assert np.all(y == 0)
