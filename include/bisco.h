@@ -124,6 +124,27 @@ bisco_status bisco_encode(const uint16_t *W_bf16, const float *g, const bisco_la
                           void *workspace, size_t workspace_bytes, bisco_stream_t stream);
 
 /*
+ * bisco_encode without a workspace argument, for callers that cannot
+ * allocate device memory (for example a host application whose own
+ * allocator has reserved the device memory and forbids other cudaMalloc
+ * calls, or code that must avoid the device-wide synchronisation that
+ * cudaMalloc/cudaFree can cause).  The paper has no counterpart; this is a
+ * library convenience.  It calls no cudaMalloc, cudaFree or allocating
+ * routine: its scratch is a fixed array inside the library, sized for
+ * K <= BISCO_ENCODE_NOALLOC_MAX_K (13 bytes per column, 416 KiB, held on
+ * every GPU that loads the library until the process exits).  Larger K
+ * returns BISCO_ERR_UNSUPPORTED.  The first call on each device looks up
+ * the array's device address (cudaGetSymbolAddress) with that device
+ * current; make that first call before any stream capture.  All calls share
+ * the one array, so calls that overlap on the GPU race and must be
+ * serialised by the caller.  Arguments, outputs and errors are otherwise
+ * those of bisco_encode.
+ */
+#define BISCO_ENCODE_NOALLOC_MAX_K 32768
+bisco_status bisco_encode_noalloc(const uint16_t *W_bf16, const float *g, const bisco_layer *L,
+                                  bisco_stream_t stream);
+
+/*
  * Decode-time matrix-vector product for B in [0, 16] activation rows:
  *     y[b][i] = sum_j What[i][j] * x[b][j]        (Sec. III-F Eq. 12, Eq. 10)
  * computed straight from the coded layer (the dense weight is never

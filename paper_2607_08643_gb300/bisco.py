@@ -16,7 +16,7 @@ OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_RANGE, ERR_CUDA, ERR_TIMEOUT = range(6
 # Functions declared in include/bisco.h (kept in sync by tests/test_abi.py).
 EXPORTS = (
     "bisco_abi_version", "bisco_status_string", "bisco_encoded_sizes",
-    "bisco_encode_workspace_bytes", "bisco_encode", "bisco_gemv",
+    "bisco_encode_workspace_bytes", "bisco_encode", "bisco_encode_noalloc", "bisco_gemv",
     "bisco_gemm_workspace_bytes", "bisco_gemm", "bisco_get_device_error",
 )
 
@@ -61,6 +61,8 @@ def load(path: str = LIB_PATH):
     lib.bisco_encode_workspace_bytes.argtypes = [i32, i32]
     lib.bisco_encode.restype = st
     lib.bisco_encode.argtypes = [P, P, Lp, P, sz, P]
+    lib.bisco_encode_noalloc.restype = st
+    lib.bisco_encode_noalloc.argtypes = [P, P, Lp, P]
     lib.bisco_gemv.restype = st
     lib.bisco_gemv.argtypes = [Lp, P, i32, P, P]
     lib.bisco_gemm_workspace_bytes.restype = sz
@@ -173,6 +175,24 @@ def bisco_encode(W_bits, S, p, g=None, workspace=None, stream=None) -> Layer:
         assert g.dtype == torch.float32 and g.is_cuda and g.numel() == K
     _check(load().bisco_encode(_ptr(W_bits), _ptr(g), ctypes.byref(L.c), _ptr(workspace),
                                workspace.numel(), _stream(stream)), "bisco_encode")
+    return L
+
+
+def bisco_encode_noalloc(W_bits, S, p, g=None, stream=None) -> Layer:
+    """bisco_encode with the library's fixed scratch array instead of a
+    workspace (for callers that cannot allocate device memory; K up to
+    BISCO_ENCODE_NOALLOC_MAX_K = 32768).  The output Layer's tensors are
+    still allocated here, by PyTorch."""
+    import torch
+    if W_bits.dtype == torch.bfloat16:
+        W_bits = W_bits.view(torch.int16)
+    assert W_bits.is_cuda and W_bits.is_contiguous() and W_bits.dim() == 2
+    N, K = W_bits.shape
+    L = Layer(N, K, S, p, W_bits.device)
+    if g is not None:
+        assert g.dtype == torch.float32 and g.is_cuda and g.numel() == K
+    _check(load().bisco_encode_noalloc(_ptr(W_bits), _ptr(g), ctypes.byref(L.c), _stream(stream)),
+           "bisco_encode_noalloc")
     return L
 
 

@@ -13,11 +13,11 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libbisco.so")
-SOURCES = ["api.cu", "encode.cu", "gemv.cu", "gemm.cu"]
+SOURCES = ["api.cu", "encode.cu", "encode_noalloc.cu", "gemv.cu", "gemm.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
           "-Xptxas", "-warn-spills"]
-PER_FILE = {"encode.cu": ["--fmad=false"]}
+PER_FILE = {"encode.cu": ["--fmad=false"], "encode_noalloc.cu": ["--fmad=false"]}
 
 
 def nvcc() -> str:
