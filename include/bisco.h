@@ -151,6 +151,11 @@ bisco_status bisco_encode_noalloc(const uint16_t *W_bf16, const float *g, const 
  * formed).  x_bf16: [B][K] device bf16 bits; activations are used as fp16,
  * which is exact for 2^-24 <= |x| <= 65504 (larger magnitudes become inf).
  * y: [B][N] float32 device, fully overwritten.  B == 0 is a no-op.
+ * The kernel is launched as a programmatic dependent of the previous kernel
+ * in the stream: it reads x only after that kernel has completed, but it
+ * starts fetching the layer's buffers before, so they must not be written
+ * by the kernel immediately ahead of it (bisco_encode ends with an empty
+ * kernel for this reason; copies and events order as usual).
  */
 bisco_status bisco_gemv(const bisco_layer *L, const uint16_t *x_bf16, int32_t B, float *y,
                         bisco_stream_t stream);

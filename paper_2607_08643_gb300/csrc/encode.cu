@@ -212,6 +212,12 @@ __global__ void __launch_bounds__(256) k_stages(const uint16_t *__restrict__ W, 
     }
 }
 
+// Empty kernel that ends every encode.  bisco_gemv starts reading a layer
+// before it waits on the kernels ahead of it in the stream (programmatic
+// dependent launch); with this ordinary launch between them, the stage
+// kernel has completed, with its writes visible, before the GEMV starts.
+__global__ void k_encode_done() {}
+
 }  // namespace
 
 static size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
@@ -240,6 +246,7 @@ bisco_status launch_encode(const uint16_t *W, const float *g, const bisco_layer 
     const int64_t chunks = static_cast<int64_t>(N) * (K / 8);
     k_stages<<<static_cast<unsigned>((chunks + 255) / 256), 256, 0, stream>>>(
         W, N, K, S, prot, L.codes, L.norms, err);
+    k_encode_done<<<1, 32, 0, stream>>>();
     return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
 }
 

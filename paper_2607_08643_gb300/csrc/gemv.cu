@@ -1,31 +1,41 @@
 // gemv.cu -- decode-time y = What x straight from the coded layer
 // (Sec. III-F Eq. 12 with the Eq. 10 protected scatter), batch 1..16.
 //
-// Design (GB300, HBM-bound):
-//  * Each CTA owns BM = 16*WM output rows and one K range; a cluster of CK
-//    CTAs splits K and reduces its partial sums in a fixed rank order
-//    through distributed shared memory (deterministic, no atomics).
-//  * One producer thread streams 512-column slabs of the sign bytes and the
-//    fp16 norms of all S stages into a shared-memory ring with TMA
-//    (cp.async.bulk.tensor, mbarrier complete_tx); the norm tile uses the
-//    128-byte swizzle so the consumers' 16-byte reads are conflict-free.
-//  * Consumer warps own 16 rows each and decode in registers: for a 32-bit
-//    code word holding chunks c..c+3 (byte per chunk), one shift brings the
-//    sign bits of element j of chunk c and of chunk c+2 to bits 15 and 31,
-//    and one LOP3 ((w << s) & 0x80008000) ^ (n_c | n_{c+2} << 16) yields the
-//    fp16 pair (+-n_c, +-n_{c+2}) exactly.  These pairs are the A fragments
-//    of mma.m16n8k16 (fp16 in, fp32 accumulate), one MMA per stage, so the
-//    stage sum of Eq. 12 is exact in fp32.  The activation operand is staged
-//    once per CTA as fp16 in the matching permuted order, with protected
-//    columns zeroed (Eq. 10's overwrite).
-//  * Epilogue: the int8 protected columns are one more small MMA pass
-//    (q8 as exact fp16 integers against scale_j * x_j split into fp16
-//    hi + lo parts), then y = acc / sqrt(8) + acc_protected.
+// Shared decode scheme (GB300, HBM-bound):
+//  * A producer thread streams ring slots of the sign bytes and fp16 norms
+//    of all S stages (rows x 512*WQ input columns) into shared memory with
+//    TMA (cp.async.bulk.tensor, mbarrier complete_tx).  Weights never depend
+//    on earlier kernels, so this starts before the wait on the previous grid
+//    (programmatic dependent launch), and every CTA lets the next kernel in
+//    the stream be scheduled at once: CTAs of consecutive layers share an SM
+//    and the next layer's weights stream in while this one finishes.
+//  * Consumer warps decode in registers: for a 32-bit code word holding
+//    chunks c..c+3 (byte per chunk), one shift brings the sign bits of
+//    element i of chunk c and of chunk c+2 to bits 15 and 31, and one LOP3
+//    ((w << s) & 0x80008000) ^ (n_c | n_{c+2} << 16) yields the fp16 pair
+//    (+-n_c, +-n_{c+2}) exactly.  These pairs are the A fragments of
+//    mma.m16n8k16 (fp16 in, fp32 accumulate), one MMA per stage, so the
+//    stage sum of Eq. 12 is exact in fp32.  The activations are staged once
+//    per CTA, as fp16 in the matching permuted order, with the protected
+//    columns zeroed (Eq. 10's overwrite); lanes whose activation row is >= B
+//    read a zero block, so every fragment load is unconditional.
+//  * The int8 protected columns are a few more k tiles on the same MMA: q8
+//    as exact fp16 integers against scale_j * x_j split into fp16 hi + lo;
+//    y = acc / sqrt(8) + acc_protected.
+//
+// k_gemv_stream (batch <= 8, at least one 16-row tile per SM): one
+// persistent CTA per SM walks its 16-row tiles while the ring keeps
+// streaming across tile boundaries; a reducer warp computes each tile's
+// protected term and writes y, so the consumer warps never stop decoding.
+// k_gemv (short layers, batch > 8): a cluster of CK CTAs splits K; ranks 1..
+// store their partial sums into rank 0's shared memory and arrive on an
+// mbarrier there; rank 0 adds them in rank order (deterministic, no atomics).
 #include <cuda_runtime.h>
 #include <stdint.h>
 #include <stdio.h>
 #include <stdlib.h>
 
+#include <algorithm>
 
 #include "bisco_dev.cuh"
 #include "bisco_host.h"
@@ -33,9 +43,7 @@
 namespace bisco {
 namespace {
 
-constexpr int kSlab = 512;            // input columns per ring slot
-constexpr int kCodeRow = kSlab / 8;   // 64 bytes of signs per row per stage
-constexpr int kNormRow = kSlab / 4;   // 128 bytes of norms per row per stage
+constexpr int kSlab = 512;   // input columns one consumer warp covers per slot
 constexpr float kInvSqrt8 = 0.35355339059327373f;
 
 struct GemvArgs {
@@ -45,153 +53,331 @@ struct GemvArgs {
     const int32_t *prot_idx;
     int *err;
     int N, K, B, p;
-    int slabs_per_rank, total_slabs, nslot;
-    uint32_t off_xt, off_q8, off_xs, off_red, off_bar;
-    int xt_pitch;   // bytes per activation row in the staged operand
-    int xs_pitch;   // halves per activation row of the protected operand
-    int q8_boxes;   // 128-column TMA boxes of q8 reserved per CTA
+    int wide_per_rank;   // ring slots' worth of columns per cluster rank (k_gemv)
+    int nslot;           // ring depth
+    uint32_t off_xt, off_q8, off_red, off_cl, off_bar, off_pidx, off_pmask, off_pu, off_zero,
+        off_prot;
+    int pidx_cap;        // protected entries staged per CTA (multiple of 16)
+    int xt_pitch;        // bytes per activation row in the staged operand
 };
 
 __device__ __forceinline__ uint32_t word_of(const uint4 &v, int i) {
     return i == 0 ? v.x : (i == 1 ? v.y : (i == 2 ? v.z : v.w));
 }
 
-// Position (in halves, within one activation row) of slab-relative column
-// kk in the permuted operand layout [slab][w][m][t][4 pairs][2].
-__device__ __forceinline__ int xt_pos(int kk) {
-    const int slab = kk >> 9, col = kk & 511;
-    const int t = col >> 7, cc = col & 127;
-    const int w = cc >> 5, cw = cc & 31;
-    const int c4 = cw >> 3, j = cw & 7;
-    const int i = 8 * (c4 & 1) + j, half = c4 >> 1;
-    return slab * 512 + (((w * 4 + (i >> 2)) * 4 + t) * 4 + (i & 3)) * 2 + half;
+// A fragment of one k16 tile from the code words of rows lo/hi: pairs i0
+// and i0+1 of each word, ((w << (15-i)) & 0x80008000) ^ norm pair.
+__device__ __forceinline__ void decode_pairs(int i0, uint32_t cl, uint32_t ch, uint32_t nl,
+                                             uint32_t nh, uint32_t (&af)[4]) {
+    af[0] = lop3_and_xor(cl << (15 - i0), 0x80008000u, nl);
+    af[1] = lop3_and_xor(ch << (15 - i0), 0x80008000u, nh);
+    af[2] = lop3_and_xor(cl << (14 - i0), 0x80008000u, nl);
+    af[3] = lop3_and_xor(ch << (14 - i0), 0x80008000u, nh);
 }
 
-__device__ __forceinline__ int lower_bound_i32(const int32_t *a, int n, int v) {
-    int lo = 0, hi = n;
-    while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if (a[mid] < v) lo = mid + 1; else hi = mid;
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+// 1024-byte aligned base of the dynamic shared memory, derived by pointer
+// arithmetic on the shared array so that accesses stay shared-space ones.
+__device__ __forceinline__ unsigned char *aligned_smem(unsigned char *raw) {
+    return raw + ((1024u - (smem_u32(raw) & 1023u)) & 1023u);
+}
+
+// Activation staging for the input columns [k_begin, k_begin + cols):
+// bf16 rows from global memory -> fp16 in the permuted fragment order
+// [512-column slab][w][m][t][4 pairs], protected columns zeroed, and
+// scale_u * x[b][j_u] of the protected columns (exact in fp32: 11 x 8
+// significant bits) taken from the same loads, so the activations cost one
+// round trip to memory.  Job = one 32-column group of one row (4 x 16 B in,
+// 4 x 16 B out).  Pair i of a 32-column group is element i&7 of chunk
+// (i>>3) and of chunk (i>>3)+2 -- bits i and i+16 of its code word.
+__device__ __forceinline__ void stage_activations(unsigned char *sm, const GemvArgs &a,
+                                                  int k_begin, int cols, int nnar,
+                                                  const uint32_t *s_pmask, const int *s_pu,
+                                                  const float *s_pscale, float *s_xs) {
+    const int groups_per_row = cols >> 5;   // cols % 128 == 0 on this path
+    const int njobs = a.B * nnar * 16;
+    for (int e = threadIdx.x; e < njobs; e += blockDim.x) {
+        const int t = e & 3, w = (e >> 2) & 3, sb = e >> 4;
+        const int b = sb / nnar, slab = sb - b * nnar;
+        const int g32 = slab * 16 + t * 4 + w;
+        unsigned char *dst = sm + a.off_xt + b * a.xt_pitch + slab * 1024 + t * 16;
+        if (g32 >= groups_per_row) {
+#pragma unroll
+            for (int m = 0; m < 4; ++m)
+                *reinterpret_cast<uint4 *>(dst + (w * 4 + m) * 64) = make_uint4(0, 0, 0, 0);
+            continue;
+        }
+        const uint4 *src = reinterpret_cast<const uint4 *>(
+            a.x + static_cast<int64_t>(b) * a.K + k_begin + g32 * 32);
+        uint32_t r[16];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const uint4 v = src[q];
+            r[4 * q] = v.x; r[4 * q + 1] = v.y; r[4 * q + 2] = v.z; r[4 * q + 3] = v.w;
+        }
+        const uint32_t pm = s_pmask[g32];
+        if (pm) {
+            const int u0 = s_pu[g32];   // protected columns before this group
+#pragma unroll
+            for (int k = 0; k < 32; ++k) {
+                if ((pm >> k) & 1u) {
+                    const int u = u0 + __popc(pm & ((1u << k) - 1u));
+                    const float xv = (k & 1) ? bf16_hi(r[k >> 1]) : bf16_lo(r[k >> 1]);
+                    s_xs[b * a.pidx_cap + u] = s_pscale[u] * xv;
+                    r[k >> 1] &= (k & 1) ? 0x0000FFFFu : 0xFFFF0000u;
+                }
+            }
+        }
+#pragma unroll
+        for (int m = 0; m < 4; ++m) {
+            // pairs 4m..4m+3: element 4(m&1)+q of chunk m>>1 and of chunk (m>>1)+2
+            const int wf = 4 * (m >> 1) + 2 * (m & 1);
+            uint32_t o[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const uint32_t f = r[wf + (q >> 1)], sw = r[8 + wf + (q >> 1)];
+                const __half2 h = __floats2half2_rn((q & 1) ? bf16_hi(f) : bf16_lo(f),
+                                                    (q & 1) ? bf16_hi(sw) : bf16_lo(sw));
+                o[q] = *reinterpret_cast<const uint32_t *>(&h);
+            }
+            *reinterpret_cast<uint4 *>(dst + (w * 4 + m) * 64) = make_uint4(o[0], o[1], o[2], o[3]);
+        }
     }
-    return lo;
 }
 
-__device__ __forceinline__ uint32_t pack_q8_pair(int8_t a, int8_t b) {
-    const __half2 h = __floats2half2_rn(static_cast<float>(a), static_cast<float>(b));
-    return *reinterpret_cast<const uint32_t *>(&h);
+// One ring slot's share of one consumer warp: rows lo/hi of column quarter
+// q (512 columns) for all S stages, accumulated into four MMA chains.
+template <int S, int BM, int kCodeRow, int kNormRow, bool kSwz, int NT>
+__device__ __forceinline__ void decode_slot(const unsigned char *cs, const unsigned char *ns,
+                                            int q, int rlo, int rhi, int t,
+                                            const unsigned char *const (&xr)[NT],
+                                            float (&acc)[4][NT][4]) {
+    // stages one after another: keeps one stage's codes and norms live
+#pragma unroll 1
+    for (int s = 0; s < S; ++s) {
+        const uint4 clo = *reinterpret_cast<const uint4 *>(cs + (s * BM + rlo) * kCodeRow + q * 64 + t * 16);
+        const uint4 chi = *reinterpret_cast<const uint4 *>(cs + (s * BM + rhi) * kCodeRow + q * 64 + t * 16);
+        const unsigned char *nlo = ns + (s * BM + rlo) * kNormRow + q * 128;
+        const unsigned char *nhi = ns + (s * BM + rhi) * kNormRow + q * 128;
+        const int sl = kSwz ? (rlo & 7) : 0, sh = kSwz ? (rhi & 7) : 0;
+        const uint4 nl0 = *reinterpret_cast<const uint4 *>(nlo + (((2 * t) ^ sl) << 4));
+        const uint4 nl1 = *reinterpret_cast<const uint4 *>(nlo + (((2 * t + 1) ^ sl) << 4));
+        const uint4 nh0 = *reinterpret_cast<const uint4 *>(nhi + (((2 * t) ^ sh) << 4));
+        const uint4 nh1 = *reinterpret_cast<const uint4 *>(nhi + (((2 * t + 1) ^ sh) << 4));
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+            const uint32_t cl = word_of(clo, w), ch = word_of(chi, w);
+            const uint32_t la = word_of(w < 2 ? nl0 : nl1, (2 * w) & 3);
+            const uint32_t lb = word_of(w < 2 ? nl0 : nl1, (2 * w + 1) & 3);
+            const uint32_t ha = word_of(w < 2 ? nh0 : nh1, (2 * w) & 3);
+            const uint32_t hb = word_of(w < 2 ? nh0 : nh1, (2 * w + 1) & 3);
+            // norm pairs (n_c, n_{c+2}) for chunks 0/2 and 1/3 of the word
+            const uint32_t np0l = prmt(la, lb, 0x5410), np1l = prmt(la, lb, 0x7632);
+            const uint32_t np0h = prmt(ha, hb, 0x5410), np1h = prmt(ha, hb, 0x7632);
+#pragma unroll
+            for (int m = 0; m < 4; ++m) {
+                uint4 xf[NT];
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt)
+                    xf[nt] = *reinterpret_cast<const uint4 *>(xr[nt] + (w * 4 + m) * 64);
+                // k tiles 2m, 2m+1: pairs 4m..4m+3 of the word
+                uint32_t af[2][4];
+                decode_pairs(4 * m, cl, ch, m < 2 ? np0l : np1l, m < 2 ? np0h : np1h, af[0]);
+                decode_pairs(4 * m + 2, cl, ch, m < 2 ? np0l : np1l, m < 2 ? np0h : np1h, af[1]);
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt) {
+                    mma_16816(acc[(w & 1) * 2][nt], af[0], xf[nt].x, xf[nt].y);
+                    mma_16816(acc[(w & 1) * 2 + 1][nt], af[1], xf[nt].z, xf[nt].w);
+                }
+            }
+        }
+    }
 }
 
-template <int WM, int NT, int S>
-__global__ void __launch_bounds__((WM + 1) * 32, 1)
+// Protected k tile u16..u16+15 for rows lo/hi (Eq. 10): q8 bytes from the
+// TMA'd int8 slab (column col0 + u of box-major [box][BM][128] storage) as
+// exact fp16 integers against scale * x (s_xs) split into fp16 hi + lo.
+template <int BM, int NT>
+__device__ __forceinline__ void protected_tile(const int8_t *q8s, int col0, int u16, int p_loc,
+                                               int rlo, int rhi, int g, int t, const float *s_xs,
+                                               int xs_pitch, int B, float (&accp)[NT][4]) {
+    auto q8v = [&](int r, int u) -> float {
+        if (u >= p_loc) return 0.f;
+        const int col = col0 + u;
+        return static_cast<float>(q8s[((col >> 7) * BM + r) * 128 + (col & 127)]);
+    };
+    const int u0 = u16 + 2 * t;
+    uint32_t af[4];
+    const int uu[4] = {u0, u0, u0 + 8, u0 + 8};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const int r = (e & 1) ? rhi : rlo;
+        const __half2 h = __floats2half2_rn(q8v(r, uu[e]), q8v(r, uu[e] + 1));
+        af[e] = *reinterpret_cast<const uint32_t *>(&h);
+    }
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+        const int bg = nt * 8 + g;
+        uint32_t hi[2] = {0u, 0u}, lo[2] = {0u, 0u};
+        if (bg < B) {
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int u = u0 + 8 * h;
+                const float v0 = u < p_loc ? s_xs[bg * xs_pitch + u] : 0.f;
+                const float v1 = u + 1 < p_loc ? s_xs[bg * xs_pitch + u + 1] : 0.f;
+                const __half2 vh = __floats2half2_rn(v0, v1);
+                const float2 back = __half22float2(vh);
+                const __half2 vl = __floats2half2_rn(v0 - back.x, v1 - back.y);
+                hi[h] = *reinterpret_cast<const uint32_t *>(&vh);
+                lo[h] = *reinterpret_cast<const uint32_t *>(&vl);
+            }
+        }
+        mma_16816(accp[nt], af, hi[0], hi[1]);
+        mma_16816(accp[nt], af, lo[0], lo[1]);
+    }
+}
+
+// Protected-column bookkeeping of one CTA (warp 0): indices in [k_begin,
+// k_end) (prot_idx is ascending), their scales, a bit mask over the CTA's
+// 32-column groups and the number of protected columns before each group.
+// Returns the index range [lo, hi) in prot_idx via s_lohi.
+__device__ __forceinline__ void stage_protected_meta(const GemvArgs &a, int k_begin, int k_end,
+                                                     int mwords, int *s_pidx, float *s_pscale,
+                                                     uint32_t *s_pmask, int *s_pu, int *s_lohi) {
+    const int lane = threadIdx.x & 31;
+    for (int i = lane; i < mwords; i += 32) s_pmask[i] = 0u;
+    int lo = 0, hi = 0;
+    for (int t0 = 0; t0 < a.p; t0 += 32) {
+        const int t = t0 + lane;
+        const int v = t < a.p ? a.prot_idx[t] : 0x7FFFFFFF;
+        lo += __popc(__ballot_sync(0xFFFFFFFFu, v < k_begin));
+        hi += __popc(__ballot_sync(0xFFFFFFFFu, v < k_end));
+    }
+    __syncwarp();
+    for (int u = lane; u < hi - lo; u += 32) {
+        const int j = a.prot_idx[lo + u];
+        s_pidx[u] = j;
+        s_pscale[u] = __half2float(__ushort_as_half(a.q8_scale[lo + u]));
+        atomicOr(&s_pmask[(j - k_begin) >> 5], 1u << ((j - k_begin) & 31));
+    }
+    __syncwarp();
+    int run = 0;
+    for (int base = 0; base < mwords; base += 32) {
+        const int i = base + lane;
+        const int c = i < mwords ? __popc(s_pmask[i]) : 0;
+        int incl = c;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+            if (lane >= o) incl += v;
+        }
+        if (i < mwords) s_pu[i] = run + incl - c;
+        run += __shfl_sync(0xFFFFFFFFu, incl, 31);
+    }
+    if (lane == 0) {
+        s_lohi[0] = lo;
+        s_lohi[1] = hi;
+    }
+}
+
+// ------------------------------------------------------------------------
+// Clustered kernel: BM = 16*WM rows x one K range per CTA.
+template <int WM, int WQ, int NT, int S>
+__global__ void __launch_bounds__((WM * WQ + 1) * 32, (NT == 1 && (WM * WQ + 1) * 32 <= 320) ? 2 : 1)
 k_gemv(const __grid_constant__ CUtensorMap tm_codes, const __grid_constant__ CUtensorMap tm_norms,
        const __grid_constant__ CUtensorMap tm_q8, const GemvArgs a) {
     constexpr int BM = 16 * WM;
     constexpr int BP = 8 * NT;
+    constexpr int NCW = WM * WQ;             // consumer warps; warp NCW is the producer
+    constexpr int SW = kSlab * WQ;           // columns per ring slot
+    constexpr int kCodeRow = SW / 8;
+    constexpr int kNormRow = SW / 4;
+    constexpr bool kSwz = (WQ == 1);         // 128-byte swizzle when a norm row is 128 B
     constexpr uint32_t kCodesBytes = S * BM * kCodeRow;
     constexpr uint32_t kSlotBytes = S * BM * (kCodeRow + kNormRow);
 
     extern __shared__ unsigned char smem_raw[];
-    unsigned char *sm = reinterpret_cast<unsigned char *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    unsigned char *sm = aligned_smem(smem_raw);
     const uint32_t sbase = smem_u32(sm);
-    __shared__ int s_abort, s_lo, s_hi;
+    __shared__ int s_abort, s_lohi[2];
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int rank = static_cast<int>(cluster_ctarank());
     const int nrank = static_cast<int>(cluster_nctarank());
     const int row0 = blockIdx.y * BM;
-    const int slab0 = rank * a.slabs_per_rank;
-    const int nsl = max(0, min(a.slabs_per_rank, a.total_slabs - slab0));
-    const int k_begin = slab0 * kSlab;
-    const int k_end = min(a.K, k_begin + nsl * kSlab);
+    const int k_begin = min(a.K, rank * a.wide_per_rank * SW);
+    const int k_end = min(a.K, k_begin + a.wide_per_rank * SW);
+    const int nwide = (k_end - k_begin + SW - 1) / SW;
+    const int nnar = (k_end - k_begin + kSlab - 1) / kSlab;
     const int nslot = a.nslot;
     const uint32_t bar_full = sbase + a.off_bar;
     const uint32_t bar_empty = bar_full + 8 * nslot;
     const uint32_t bar_q8 = bar_full + 16 * nslot;
+    const uint32_t bar_cl = bar_q8 + 8;
+    const bool producer = (warp == NCW) && (lane == 0);
+    const uint64_t pol = l2_evict_first_policy();
+    int *s_pidx = reinterpret_cast<int *>(sm + a.off_pidx);
+    float *s_pscale = reinterpret_cast<float *>(s_pidx + a.pidx_cap);
+    float *s_xs = s_pscale + a.pidx_cap;
+    uint32_t *s_pmask = reinterpret_cast<uint32_t *>(sm + a.off_pmask);
+    int *s_pu = reinterpret_cast<int *>(sm + a.off_pu);
 
-    if (threadIdx.x == 0) {
-        for (int i = 0; i < nslot; ++i) {
-            mbar_init(bar_full + 8 * i, 1);
-            mbar_init(bar_empty + 8 * i, WM);
-        }
-        mbar_init(bar_q8, 1);
-        fence_mbar_init();
-        s_abort = 0;
-    }
-    if (threadIdx.x == 32) {
-        s_lo = a.p ? lower_bound_i32(a.prot_idx, a.p, k_begin) : 0;
-        s_hi = a.p ? lower_bound_i32(a.prot_idx, a.p, k_end) : 0;
-    }
-    __syncthreads();
-    const int lo_t = s_lo, p_loc = s_hi - s_lo;
-    const bool producer = (warp == WM) && (lane == 0);
-
-    // Weights do not depend on earlier kernels: start streaming them before
-    // waiting on the previous grid (programmatic dependent launch).
     int issued = 0;
     if (producer) {
+        for (int i = 0; i < nslot; ++i) {
+            mbar_init(bar_full + 8 * i, 1);
+            mbar_init(bar_empty + 8 * i, NCW);
+        }
+        mbar_init(bar_q8, 1);
+        mbar_init(bar_cl, nrank > 1 ? (nrank - 1) * blockDim.x : 1);
+        fence_mbar_init();
+        s_abort = 0;
         prefetch_tmap(&tm_codes);
         prefetch_tmap(&tm_norms);
-        if (p_loc > 0) {
-            const int qx0 = lo_t & ~15;
-            const int nq = (lo_t + p_loc - qx0 + 127) >> 7;
-            mbar_arrive_expect_tx(bar_q8, static_cast<uint32_t>(nq * BM * 128));
-            for (int q = 0; q < nq; ++q)
-                tma_load_2d(sbase + a.off_q8 + q * BM * 128, &tm_q8, bar_q8, qx0 + 128 * q, row0);
-        }
-        for (; issued < nsl && issued < nslot; ++issued) {
+        for (; issued < nwide && issued < nslot; ++issued) {
             const uint32_t dst = sbase + issued * kSlotBytes;
             mbar_arrive_expect_tx(bar_full + 8 * issued, kSlotBytes);
-            const int kx = (k_begin + issued * kSlab) / 8;
-            tma_load_3d(dst, &tm_codes, bar_full + 8 * issued, kx, row0, 0);
-            tma_load_3d(dst + kCodesBytes, &tm_norms, bar_full + 8 * issued, kx, row0, 0);
+            const int kx = (k_begin + issued * SW) / 8;
+            tma_load_3d_hint(dst, &tm_codes, bar_full + 8 * issued, kx, row0, 0, pol);
+            tma_load_3d_hint(dst + kCodesBytes, &tm_norms, bar_full + 8 * issued, kx, row0, 0, pol);
         }
     }
-
-    pdl_wait();
-
-    // Stage the activation operand: fp16, permuted to fragment order,
-    // protected columns zeroed; and scale_j * x_j as fp16 hi + lo.
-    {
-        uint16_t *xt = reinterpret_cast<uint16_t *>(sm + a.off_xt);
-        const int cols = nsl * kSlab;
-        const int pitch_h = a.xt_pitch / 2;
-        for (int e = threadIdx.x; e < a.B * cols; e += blockDim.x) {
-            const int b = e / cols, kk = e - b * cols;
-            const int k = k_begin + kk;
-            const uint16_t v = k < k_end ? bf16_bits_to_f16_bits(a.x[static_cast<int64_t>(b) * a.K + k]) : 0;
-            xt[b * pitch_h + xt_pos(kk)] = v;
-        }
-        __syncthreads();
-        __half *xs_hi = reinterpret_cast<__half *>(sm + a.off_xs);
-        __half *xs_lo = xs_hi + a.B * a.xs_pitch;
-        const int p16 = (p_loc + 15) & ~15;
-        for (int e = threadIdx.x; e < a.B * p16; e += blockDim.x) {
-            const int b = e / p16, u = e - b * p16;
-            float v = 0.f;
-            if (u < p_loc) {
-                const int j = a.prot_idx[lo_t + u];
-                xt[b * pitch_h + xt_pos(j - k_begin)] = 0;
-                v = __half2float(__ushort_as_half(a.q8_scale[lo_t + u])) *
-                    bf16_bits_to_f32(a.x[static_cast<int64_t>(b) * a.K + j]);
-            }
-            const __half h = __float2half_rn(v);
-            xs_hi[b * a.xs_pitch + u] = h;
-            xs_lo[b * a.xs_pitch + u] = __float2half_rn(v - __half2float(h));
-        }
-    }
+    if (warp == 0)
+        stage_protected_meta(a, k_begin, k_end, nnar * (kSlab / 32), s_pidx, s_pscale, s_pmask,
+                             s_pu, s_lohi);
     __syncthreads();
+    // the next kernel in the stream may start streaming its own weights now
     pdl_launch_dependents();
+    // rank 0's reduction barrier is initialised before any rank arrives on
+    // it: arrive here, wait just before the hand-over at the end
+    if (nrank > 1) cluster_arrive();
+    const int lo_t = s_lohi[0], p_loc = s_lohi[1] - s_lohi[0];
+    const int q8x0 = lo_t & ~15;   // 16-byte aligned TMA start
+    const int q8_boxes = p_loc > 0 ? (lo_t + p_loc - q8x0 + 127) >> 7 : 0;
+    if (producer && q8_boxes > 0) {
+        mbar_arrive_expect_tx(bar_q8, static_cast<uint32_t>(q8_boxes * BM * 128));
+        for (int q = 0; q < q8_boxes; ++q)
+            tma_load_2d_hint(sbase + a.off_q8 + q * BM * 128, &tm_q8, bar_q8, q8x0 + 128 * q, row0,
+                             pol);
+    }
+
+    // activations may be written by the previous kernel
+    pdl_wait();
+    stage_activations(sm, a, k_begin, k_end - k_begin, nnar, s_pmask, s_pu, s_pscale, s_xs);
+    for (int i = threadIdx.x; i < 1024 / 16; i += blockDim.x)
+        reinterpret_cast<uint4 *>(sm + a.off_zero)[i] = make_uint4(0, 0, 0, 0);
+    __syncthreads();
 
     float *red = reinterpret_cast<float *>(sm + a.off_red);
 
-    if (warp == WM) {
+    if (warp == NCW) {
         // ------------------------------------------------ producer: refill
         if (producer) {
-            for (; issued < nsl; ++issued) {
+            for (; issued < nwide; ++issued) {
                 const int slot = issued % nslot;
-                const uint32_t par = ((issued / nslot) - 1) & 1;
-                if (!mbar_wait(bar_empty + 8 * slot, par)) {
+                if (!mbar_wait(bar_empty + 8 * slot, ((issued / nslot) - 1) & 1)) {
                     latch_error(a.err, BISCO_ERR_TIMEOUT);
                     atomicExch(&s_abort, 1);
                     break;
@@ -199,9 +385,9 @@ k_gemv(const __grid_constant__ CUtensorMap tm_codes, const __grid_constant__ CUt
                 if (*reinterpret_cast<volatile int *>(&s_abort)) break;
                 const uint32_t dst = sbase + slot * kSlotBytes;
                 mbar_arrive_expect_tx(bar_full + 8 * slot, kSlotBytes);
-                const int kx = (k_begin + issued * kSlab) / 8;
-                tma_load_3d(dst, &tm_codes, bar_full + 8 * slot, kx, row0, 0);
-                tma_load_3d(dst + kCodesBytes, &tm_norms, bar_full + 8 * slot, kx, row0, 0);
+                const int kx = (k_begin + issued * SW) / 8;
+                tma_load_3d_hint(dst, &tm_codes, bar_full + 8 * slot, kx, row0, 0, pol);
+                tma_load_3d_hint(dst + kCodesBytes, &tm_norms, bar_full + 8 * slot, kx, row0, 0, pol);
             }
             if (*reinterpret_cast<volatile int *>(&s_abort)) {
                 // let every copy already in flight land before the CTA exits
@@ -209,20 +395,32 @@ k_gemv(const __grid_constant__ CUtensorMap tm_codes, const __grid_constant__ CUt
                     const int last = slot + ((issued - 1 - slot) / nslot) * nslot;
                     mbar_wait(bar_full + 8 * slot, (last / nslot) & 1);
                 }
-                if (p_loc > 0) mbar_wait(bar_q8, 0);
+                if (q8_boxes > 0) mbar_wait(bar_q8, 0);
             }
         }
     } else {
         // ----------------------------------------------- consumers: decode
+        // warp (wm, q) owns rows 16*wm.. and column quarter q of every slot
+        const int wm = warp % WM, q = warp / WM;
         const int g = lane >> 2, t = lane & 3;
-        const int rlo = 16 * warp + g, rhi = rlo + 8;
-        float acc[NT][4];
+        const int rlo = 16 * wm + g, rhi = rlo + 8;
+        const unsigned char *xb[NT];
+        int xstep[NT];
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt)
+        for (int nt = 0; nt < NT; ++nt) {
+            const int bg = nt * 8 + g;
+            xb[nt] = bg < a.B ? sm + a.off_xt + bg * a.xt_pitch + t * 16 : sm + a.off_zero + t * 16;
+            xstep[nt] = bg < a.B ? 1024 : 0;
+        }
+        float acc[4][NT][4];
 #pragma unroll
-            for (int k = 0; k < 4; ++k) acc[nt][k] = 0.f;
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                for (int k = 0; k < 4; ++k) acc[c][nt][k] = 0.f;
 
-        for (int it = 0; it < nsl; ++it) {
+        for (int it = 0; it < nwide; ++it) {
             const int slot = it % nslot;
             if (*reinterpret_cast<volatile int *>(&s_abort)) break;
             if (!mbar_wait(bar_full + 8 * slot, (it / nslot) & 1)) {
@@ -230,101 +428,34 @@ k_gemv(const __grid_constant__ CUtensorMap tm_codes, const __grid_constant__ CUt
                 atomicExch(&s_abort, 1);
                 break;
             }
-            const unsigned char *cs = sm + slot * kSlotBytes;
-            const unsigned char *ns = cs + kCodesBytes;
-            const unsigned char *xrow = sm + a.off_xt + it * 1024 + t * 16;
+            const int nar = it * WQ + q;   // this warp's 512-column slab
+            if (nar < nnar) {
+                const unsigned char *cs = sm + slot * kSlotBytes;
+                const unsigned char *xr[NT];
 #pragma unroll
-            for (int s = 0; s < S; ++s) {
-                const uint4 clo = *reinterpret_cast<const uint4 *>(cs + (s * BM + rlo) * kCodeRow + t * 16);
-                const uint4 chi = *reinterpret_cast<const uint4 *>(cs + (s * BM + rhi) * kCodeRow + t * 16);
-                const unsigned char *nlo = ns + (s * BM + rlo) * kNormRow;
-                const unsigned char *nhi = ns + (s * BM + rhi) * kNormRow;
-                const uint4 nl0 = *reinterpret_cast<const uint4 *>(nlo + (((2 * t) ^ (rlo & 7)) << 4));
-                const uint4 nl1 = *reinterpret_cast<const uint4 *>(nlo + (((2 * t + 1) ^ (rlo & 7)) << 4));
-                const uint4 nh0 = *reinterpret_cast<const uint4 *>(nhi + (((2 * t) ^ (rhi & 7)) << 4));
-                const uint4 nh1 = *reinterpret_cast<const uint4 *>(nhi + (((2 * t + 1) ^ (rhi & 7)) << 4));
-#pragma unroll
-                for (int w = 0; w < 4; ++w) {
-                    const uint32_t cl = word_of(clo, w), ch = word_of(chi, w);
-                    const uint32_t la = word_of(w < 2 ? nl0 : nl1, (2 * w) & 3);
-                    const uint32_t lb = word_of(w < 2 ? nl0 : nl1, (2 * w + 1) & 3);
-                    const uint32_t ha = word_of(w < 2 ? nh0 : nh1, (2 * w) & 3);
-                    const uint32_t hb = word_of(w < 2 ? nh0 : nh1, (2 * w + 1) & 3);
-                    const uint32_t np0l = prmt(la, lb, 0x5410), np1l = prmt(la, lb, 0x7632);
-                    const uint32_t np0h = prmt(ha, hb, 0x5410), np1h = prmt(ha, hb, 0x7632);
-#pragma unroll
-                    for (int m = 0; m < 4; ++m) {
-                        uint4 xf[NT];
-#pragma unroll
-                        for (int nt = 0; nt < NT; ++nt) {
-                            const int bg = nt * 8 + g;
-                            xf[nt] = bg < a.B ? *reinterpret_cast<const uint4 *>(
-                                                    xrow + bg * a.xt_pitch + (w * 4 + m) * 64)
-                                              : make_uint4(0, 0, 0, 0);
-                        }
-#pragma unroll
-                        for (int qq = 0; qq < 2; ++qq) {
-                            const int q = 2 * m + qq;
-                            const int i0 = 2 * q, i1 = 2 * q + 1;
-                            const uint32_t nl = q < 4 ? np0l : np1l;
-                            const uint32_t nh = q < 4 ? np0h : np1h;
-                            uint32_t af[4];
-                            af[0] = lop3_and_xor(cl << (15 - i0), 0x80008000u, nl);
-                            af[1] = lop3_and_xor(ch << (15 - i0), 0x80008000u, nh);
-                            af[2] = lop3_and_xor(cl << (15 - i1), 0x80008000u, nl);
-                            af[3] = lop3_and_xor(ch << (15 - i1), 0x80008000u, nh);
-#pragma unroll
-                            for (int nt = 0; nt < NT; ++nt)
-                                mma_16816(acc[nt], af, word_of(xf[nt], 2 * qq), word_of(xf[nt], 2 * qq + 1));
-                        }
-                    }
-                }
+                for (int nt = 0; nt < NT; ++nt) xr[nt] = xb[nt] + nar * xstep[nt];
+                decode_slot<S, BM, kCodeRow, kNormRow, kSwz, NT>(cs, cs + kCodesBytes, q, rlo, rhi, t,
+                                                                 xr, acc);
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_empty + 8 * slot);
         }
 
-        // protected int8 columns (Eq. 10) as a second MMA pass
+        // protected columns: k tiles of a row group shared out over its WQ warps
         float accp[NT][4];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
             for (int k = 0; k < 4; ++k) accp[nt][k] = 0.f;
-        if (p_loc > 0) {
+        if (q8_boxes > 0 && q * 16 < p_loc) {
             if (!mbar_wait(bar_q8, 0)) {
                 latch_error(a.err, BISCO_ERR_TIMEOUT);
                 atomicExch(&s_abort, 1);
             } else {
-                const int8_t *q8s = reinterpret_cast<const int8_t *>(sm + a.off_q8);
-                const int qoff = lo_t - (lo_t & ~15);
-                const __half *xs_hi = reinterpret_cast<const __half *>(sm + a.off_xs);
-                const __half *xs_lo = xs_hi + a.B * a.xs_pitch;
-                auto q8at = [&](int r, int u) -> int8_t {
-                    if (u >= p_loc) return 0;
-                    const int col = qoff + u;
-                    return q8s[((col >> 7) * BM + r) * 128 + (col & 127)];
-                };
-                for (int u16 = 0; u16 < p_loc; u16 += 16) {
-                    const int u0 = u16 + 2 * t;
-                    uint32_t af[4];
-                    af[0] = pack_q8_pair(q8at(rlo, u0), q8at(rlo, u0 + 1));
-                    af[1] = pack_q8_pair(q8at(rhi, u0), q8at(rhi, u0 + 1));
-                    af[2] = pack_q8_pair(q8at(rlo, u0 + 8), q8at(rlo, u0 + 9));
-                    af[3] = pack_q8_pair(q8at(rhi, u0 + 8), q8at(rhi, u0 + 9));
-#pragma unroll
-                    for (int nt = 0; nt < NT; ++nt) {
-                        const int bg = nt * 8 + g;
-                        uint32_t h0 = 0, h1 = 0, l0 = 0, l1 = 0;
-                        if (bg < a.B) {
-                            h0 = *reinterpret_cast<const uint32_t *>(xs_hi + bg * a.xs_pitch + u0);
-                            h1 = *reinterpret_cast<const uint32_t *>(xs_hi + bg * a.xs_pitch + u0 + 8);
-                            l0 = *reinterpret_cast<const uint32_t *>(xs_lo + bg * a.xs_pitch + u0);
-                            l1 = *reinterpret_cast<const uint32_t *>(xs_lo + bg * a.xs_pitch + u0 + 8);
-                        }
-                        mma_16816(accp[nt], af, h0, h1);
-                        mma_16816(accp[nt], af, l0, l1);
-                    }
-                }
+                for (int u16 = 16 * q; u16 < p_loc; u16 += 16 * WQ)
+                    protected_tile<BM, NT>(reinterpret_cast<const int8_t *>(sm + a.off_q8),
+                                           lo_t - q8x0, u16, p_loc, rlo, rhi, g, t, s_xs,
+                                           a.pidx_cap, a.B, accp);
             }
         }
 #pragma unroll
@@ -333,35 +464,300 @@ k_gemv(const __grid_constant__ CUtensorMap tm_codes, const __grid_constant__ CUt
             for (int k = 0; k < 4; ++k) {
                 const int r = k < 2 ? rlo : rhi;
                 const int b = nt * 8 + 2 * t + (k & 1);
-                red[r * BP + b] = acc[nt][k] * kInvSqrt8 + accp[nt][k];
+                const float sum = (acc[0][nt][k] + acc[1][nt][k]) + (acc[2][nt][k] + acc[3][nt][k]);
+                red[(q * BM + r) * BP + b] = sum * kInvSqrt8 + accp[nt][k];
             }
     }
 
     __syncthreads();
-    __syncwarp();
-    if (nrank > 1) {
-        cluster_sync();
-        if (rank == 0) {
-            const uint32_t red_addr = sbase + a.off_red;
-            for (int e = threadIdx.x; e < a.B * BM; e += blockDim.x) {
-                const int b = e / BM, r = e - b * BM;
-                const uint32_t off = static_cast<uint32_t>((r * BP + b) * 4);
-                float v = 0.f;
-                for (int q = 0; q < nrank; ++q) v += ld_shared_cluster_f32(mapa_shared(red_addr + off, q));
-                if (row0 + r < a.N) a.y[static_cast<int64_t>(b) * a.N + row0 + r] = v;
-            }
+    // this CTA's partial for each (row, batch): column quarters in order
+    if (WQ > 1) {
+        for (int e = threadIdx.x; e < BM * BP; e += blockDim.x) {
+            float v = red[e];
+#pragma unroll
+            for (int qq = 1; qq < WQ; ++qq) v += red[qq * BM * BP + e];
+            red[e] = v;
         }
-        __syncwarp();
-        cluster_sync();
-    } else {
+        __syncthreads();
+    }
+    if (nrank == 1) {
         for (int e = threadIdx.x; e < a.B * BM; e += blockDim.x) {
             const int b = e / BM, r = e - b * BM;
             if (row0 + r < a.N) a.y[static_cast<int64_t>(b) * a.N + row0 + r] = red[r * BP + b];
         }
+        return;
+    }
+    cluster_wait();
+    if (rank != 0) {
+        // hand the partial to rank 0; every thread releases its own stores
+        const uint32_t dst = mapa_shared(sbase + a.off_cl + (rank - 1) * BM * BP * 4, 0);
+        for (int e = threadIdx.x; e < BM * BP; e += blockDim.x) st_shared_cluster_f32(dst + e * 4, red[e]);
+        mbar_arrive_cluster(mapa_shared(bar_cl, 0));
+        return;
+    }
+    if (!mbar_wait_cluster(bar_cl, 0)) {
+        latch_error(a.err, BISCO_ERR_TIMEOUT);
+        return;
+    }
+    const float *cl = reinterpret_cast<const float *>(sm + a.off_cl);
+    for (int e = threadIdx.x; e < a.B * BM; e += blockDim.x) {
+        const int b = e / BM, r = e - b * BM;
+        float v = red[r * BP + b];
+        for (int qq = 1; qq < nrank; ++qq) v += cl[((qq - 1) * BM + r) * BP + b];
+        if (row0 + r < a.N) a.y[static_cast<int64_t>(b) * a.N + row0 + r] = v;
     }
 }
 
-// Correctness path for layers whose row pitch rules out TMA (K % 128 != 0):
+// ------------------------------------------------------------------------
+// Streaming kernel: persistent CTA, 16-row tiles x all K, batch <= 8.
+// Warp (q, k) decodes column quarter q of every slot whose global index is
+// k modulo WK; warp NCW produces; warp NCW+1 reduces.  A slot's full
+// barrier is split into WK barriers taken in turn by its fills, so that a
+// consumer group always waits on a barrier whose previous phase it observed
+// itself, whatever the ring depth.
+template <int WQ, int WK, int S>
+__global__ void __launch_bounds__((WQ * WK + 2) * 32, 2)
+k_gemv_stream(const __grid_constant__ CUtensorMap tm_codes,
+              const __grid_constant__ CUtensorMap tm_norms,
+              const __grid_constant__ CUtensorMap tm_q8, const GemvArgs a) {
+    constexpr int BM = 16;
+    constexpr int BP = 8;
+    constexpr int NCW = WQ * WK;
+    constexpr int SW = kSlab * WQ;
+    constexpr int kCodeRow = SW / 8;
+    constexpr int kNormRow = SW / 4;
+    constexpr bool kSwz = (WQ == 1);
+    constexpr uint32_t kCodesBytes = S * BM * kCodeRow;
+    constexpr uint32_t kSlotBytes = S * BM * (kCodeRow + kNormRow);
+
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *sm = aligned_smem(smem_raw);
+    const uint32_t sbase = smem_u32(sm);
+    __shared__ int s_abort, s_lohi[2];
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int G = static_cast<int>(gridDim.x), cta = static_cast<int>(blockIdx.x);
+    const int ntiles = (a.N + BM - 1) / BM;
+    const int my_tiles = ntiles > cta ? (ntiles - 1 - cta) / G + 1 : 0;
+    const int nwide = (a.K + SW - 1) / SW;
+    const int nnar = (a.K + kSlab - 1) / kSlab;
+    const int total = my_tiles * nwide;   // ring fills of this CTA
+    const int nslot = a.nslot;
+    const int q8_boxes = a.p > 0 ? ((a.p + 15) / 16 * 16 + 127) / 128 : 0;
+    const uint32_t q8_buf_bytes = static_cast<uint32_t>(q8_boxes * BM * 128);
+    const uint32_t bar_full = sbase + a.off_bar;            // [nslot][WK]
+    const uint32_t bar_empty = bar_full + 8 * nslot * WK;   // [nslot]
+    const uint32_t bar_q8f = bar_empty + 8 * nslot;         // [2] int8 slab landed
+    const uint32_t bar_q8e = bar_q8f + 16;                  // [2] int8 slab consumed
+    const uint32_t bar_rf = bar_q8e + 16;                   // [2] tile partials written
+    const uint32_t bar_re = bar_rf + 16;                    // [2] tile partials read
+    const bool producer = (warp == NCW) && (lane == 0);
+    const uint64_t pol = l2_evict_first_policy();
+    int *s_pidx = reinterpret_cast<int *>(sm + a.off_pidx);
+    float *s_pscale = reinterpret_cast<float *>(s_pidx + a.pidx_cap);
+    float *s_xs = s_pscale + a.pidx_cap;
+    uint32_t *s_pmask = reinterpret_cast<uint32_t *>(sm + a.off_pmask);
+    int *s_pu = reinterpret_cast<int *>(sm + a.off_pu);
+    float *red = reinterpret_cast<float *>(sm + a.off_red);   // [2][NCW][BM][BP]
+
+    auto tile_row0 = [&](int ii) { return (cta + ii * G) * BM; };
+    auto full_bar = [&](int gidx) {
+        const int ph = gidx / nslot;
+        return bar_full + 8 * ((gidx % nslot) * WK + ph % WK);
+    };
+    auto full_parity = [&](int gidx) { return static_cast<uint32_t>((gidx / nslot) / WK) & 1u; };
+    auto issue_slot = [&](int gidx) {
+        const int ii = gidx / nwide, w = gidx - ii * nwide;
+        const uint32_t dst = sbase + (gidx % nslot) * kSlotBytes;
+        const uint32_t bar = full_bar(gidx);
+        mbar_arrive_expect_tx(bar, kSlotBytes);
+        tma_load_3d_hint(dst, &tm_codes, bar, w * (SW / 8), tile_row0(ii), 0, pol);
+        tma_load_3d_hint(dst + kCodesBytes, &tm_norms, bar, w * (SW / 8), tile_row0(ii), 0, pol);
+    };
+    auto issue_q8 = [&](int ii) {
+        const uint32_t dst = sbase + a.off_q8 + (ii & 1) * q8_buf_bytes;
+        mbar_arrive_expect_tx(bar_q8f + 8 * (ii & 1), q8_buf_bytes);
+        for (int q = 0; q < q8_boxes; ++q)
+            tma_load_2d_hint(dst + q * BM * 128, &tm_q8, bar_q8f + 8 * (ii & 1), 128 * q,
+                             tile_row0(ii), pol);
+    };
+
+    int issued = 0, q8_issued = 0;
+    if (producer) {
+        for (int i = 0; i < nslot; ++i) {
+            for (int k = 0; k < WK; ++k) mbar_init(bar_full + 8 * (i * WK + k), 1);
+            mbar_init(bar_empty + 8 * i, WQ);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar_q8f + 8 * i, 1);
+            mbar_init(bar_q8e + 8 * i, 1);
+            mbar_init(bar_rf + 8 * i, NCW);
+            mbar_init(bar_re + 8 * i, 1);
+        }
+        fence_mbar_init();
+        s_abort = 0;
+        prefetch_tmap(&tm_codes);
+        prefetch_tmap(&tm_norms);
+        for (; issued < total && issued < nslot; ++issued) {
+            // a tile's int8 slab goes out with its first slot (two buffers)
+            if (q8_boxes > 0 && issued % nwide == 0 && issued / nwide < 2) issue_q8(q8_issued++);
+            issue_slot(issued);
+        }
+    }
+    if (warp == 0)
+        stage_protected_meta(a, 0, a.K, nnar * (kSlab / 32), s_pidx, s_pscale, s_pmask, s_pu,
+                             s_lohi);
+    __syncthreads();
+    pdl_launch_dependents();
+
+    pdl_wait();
+    stage_activations(sm, a, 0, a.K, nnar, s_pmask, s_pu, s_pscale, s_xs);
+    for (int i = threadIdx.x; i < 1024 / 16; i += blockDim.x)
+        reinterpret_cast<uint4 *>(sm + a.off_zero)[i] = make_uint4(0, 0, 0, 0);
+    __syncthreads();
+
+    if (warp == NCW) {
+        // ------------------------------------------------ producer: refill
+        if (producer) {
+            // The int8 slab of tile ii (buffer ii & 1) goes out just before the
+            // tile's first slot, once tile ii-2 released the buffer; every slot
+            // of tile ii-1 is issued by then, so this never starves the decode.
+            auto issue_q8_upto = [&](int ii) -> bool {
+                while (q8_boxes > 0 && q8_issued <= ii && q8_issued < my_tiles) {
+                    if (q8_issued >= 2 &&
+                        !mbar_wait(bar_q8e + 8 * (q8_issued & 1), ((q8_issued >> 1) - 1) & 1))
+                        return false;
+                    issue_q8(q8_issued);
+                    ++q8_issued;
+                }
+                return true;
+            };
+            bool ok = true;
+            for (; issued < total; ++issued) {
+                const int slot = issued % nslot;
+                if (issued % nwide == 0 && !issue_q8_upto(issued / nwide)) {
+                    ok = false;
+                    break;
+                }
+                if (!mbar_wait(bar_empty + 8 * slot, ((issued / nslot) - 1) & 1)) {
+                    ok = false;
+                    break;
+                }
+                if (*reinterpret_cast<volatile int *>(&s_abort)) break;
+                issue_slot(issued);
+            }
+            if (ok && !*reinterpret_cast<volatile int *>(&s_abort) && !issue_q8_upto(my_tiles - 1))
+                ok = false;
+            if (!ok) {
+                latch_error(a.err, BISCO_ERR_TIMEOUT);
+                atomicExch(&s_abort, 1);
+            }
+            if (*reinterpret_cast<volatile int *>(&s_abort)) {
+                // let every copy already in flight land before the CTA exits
+                for (int gi = (issued > nslot ? issued - nslot : 0); gi < issued; ++gi)
+                    mbar_wait(full_bar(gi), full_parity(gi));
+                for (int ii = (q8_issued > 2 ? q8_issued - 2 : 0); ii < q8_issued; ++ii)
+                    mbar_wait(bar_q8f + 8 * (ii & 1), (ii >> 1) & 1);
+            }
+        }
+    } else if (warp == NCW + 1) {
+        // ------------------------------------------- reducer: protected + y
+        const int g = lane >> 2, t = lane & 3;
+        const int8_t *q8base = reinterpret_cast<const int8_t *>(sm + a.off_q8);
+        float *prot = reinterpret_cast<float *>(sm + a.off_prot);   // [BM][BP]
+        for (int ii = 0; ii < my_tiles; ++ii) {
+            if (*reinterpret_cast<volatile int *>(&s_abort)) break;
+            float accp[1][4] = {{0.f, 0.f, 0.f, 0.f}};
+            if (q8_boxes > 0) {
+                if (!mbar_wait(bar_q8f + 8 * (ii & 1), (ii >> 1) & 1)) {
+                    latch_error(a.err, BISCO_ERR_TIMEOUT);
+                    atomicExch(&s_abort, 1);
+                    break;
+                }
+                for (int u16 = 0; u16 < a.p; u16 += 16)
+                    protected_tile<BM, 1>(q8base + (ii & 1) * q8_buf_bytes, 0, u16, a.p, g, g + 8, g,
+                                          t, s_xs, a.pidx_cap, a.B, accp);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar_q8e + 8 * (ii & 1));
+            }
+#pragma unroll
+            for (int e = 0; e < 4; ++e) prot[(e < 2 ? g : g + 8) * BP + 2 * t + (e & 1)] = accp[0][e];
+            __syncwarp();
+            if (!mbar_wait(bar_rf + 8 * (ii & 1), (ii >> 1) & 1)) {
+                latch_error(a.err, BISCO_ERR_TIMEOUT);
+                atomicExch(&s_abort, 1);
+                break;
+            }
+            const float *rb = red + (ii & 1) * NCW * BM * BP;
+            const int row0 = tile_row0(ii);
+            for (int e = lane; e < a.B * BM; e += 32) {
+                const int b = e / BM, r = e - b * BM;
+                float v = 0.f;
+#pragma unroll
+                for (int wq = 0; wq < NCW; ++wq) v += rb[(wq * BM + r) * BP + b];
+                v += prot[r * BP + b];
+                if (row0 + r < a.N) a.y[static_cast<int64_t>(b) * a.N + row0 + r] = v;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_re + 8 * (ii & 1));
+        }
+    } else {
+        // ----------------------------------------------- consumers: decode
+        const int q = warp % WQ, k = warp / WQ;
+        const int g = lane >> 2, t = lane & 3;
+        const unsigned char *xb = g < a.B ? sm + a.off_xt + g * a.xt_pitch + t * 16
+                                          : sm + a.off_zero + t * 16;
+        const int xstep = g < a.B ? 1024 : 0;
+        for (int ii = 0; ii < my_tiles; ++ii) {
+            if (*reinterpret_cast<volatile int *>(&s_abort)) break;
+            float acc[4][1][4];
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) acc[c][0][e] = 0.f;
+            // this warp's slots of tile ii: global index ii*nwide + w == k (mod WK)
+            for (int w = (k - (ii * nwide) % WK + WK) % WK; w < nwide; w += WK) {
+                const int gidx = ii * nwide + w;
+                if (*reinterpret_cast<volatile int *>(&s_abort)) break;
+                if (!mbar_wait(full_bar(gidx), full_parity(gidx))) {
+                    latch_error(a.err, BISCO_ERR_TIMEOUT);
+                    atomicExch(&s_abort, 1);
+                    break;
+                }
+                const int nar = w * WQ + q;
+                if (nar < nnar) {
+                    const unsigned char *cs = sm + (gidx % nslot) * kSlotBytes;
+                    const unsigned char *xr[1] = {xb + nar * xstep};
+                    decode_slot<S, BM, kCodeRow, kNormRow, kSwz, 1>(cs, cs + kCodesBytes, q, g, g + 8,
+                                                                    t, xr, acc);
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar_empty + 8 * (gidx % nslot));
+            }
+            // hand this warp's partial of tile ii to the reducer (buffer ii & 1,
+            // free once the reducer has finished tile ii - 2)
+            if (ii >= 2 && !mbar_wait(bar_re + 8 * (ii & 1), ((ii >> 1) - 1) & 1)) {
+                latch_error(a.err, BISCO_ERR_TIMEOUT);
+                atomicExch(&s_abort, 1);
+                break;
+            }
+            float *rb = red + (ii & 1) * NCW * BM * BP;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int r = e < 2 ? g : g + 8;
+                const int b = 2 * t + (e & 1);
+                rb[(warp * BM + r) * BP + b] =
+                    ((acc[0][0][e] + acc[1][0][e]) + (acc[2][0][e] + acc[3][0][e])) * kInvSqrt8;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_rf + 8 * (ii & 1));
+        }
+    }
+}
+
+// ------------------------------------------------------------------------
+// Correctness path for layers whose row pitch rules out TMA (K % 128 != 0)
+// or whose protected set is too large for the fast kernels' shared memory:
 // one warp per output row, fp32 throughout.
 __global__ void __launch_bounds__(256) k_gemv_generic(const uint8_t *__restrict__ codes,
                                                       const uint16_t *__restrict__ norms,
@@ -424,92 +820,130 @@ __global__ void __launch_bounds__(256) k_gemv_generic(const uint8_t *__restrict_
 
 // ------------------------------------------------------------- planning
 
+constexpr size_t kMaxSmem = 227 * 1024;
+// Two CTAs (this layer's and the next one's) share an SM when each needs at
+// most this much dynamic shared memory (228 KB per SM, 1 KB reserved per CTA).
+constexpr size_t kCoresident = 112 * 1024;
+
 struct Plan {
-    int wm, ck, nslot;
+    int wm, wq, ck, nslot;
 };
 
-// "WM,CK,NSLOT" from BISCO_GEMV_PLAN overrides the tiling (tuning sweeps and
-// tests that cover every cluster/tile shape); read on every call.
+// (WM, WQ) tilings of k_gemv that are instantiated.
+constexpr int kTilings[][2] = {{1, 4}, {2, 4}, {4, 4}, {2, 2}, {4, 2}, {4, 1}, {8, 1}, {1, 2}};
+
+bool tiling_known(int wm, int wq) {
+    for (const auto &t : kTilings)
+        if (t[0] == wm && t[1] == wq) return true;
+    return false;
+}
+
+// Tuning overrides, read on every call (sweeps, and tests that cover every
+// path):  BISCO_GEMV_MODE  = "stream" | "cluster"   force a kernel
+//         BISCO_GEMV_PLAN  = "WM,CK,NSLOT[,WQ]"     k_gemv tiling
+//         BISCO_GEMV_NSLOT = n                      k_gemv_stream ring depth
 bool plan_override(Plan *pl) {
     const char *e = getenv("BISCO_GEMV_PLAN");
     if (!e) return false;
-    int v[3] = {0, 0, 0};
-    if (sscanf(e, "%d,%d,%d", &v[0], &v[1], &v[2]) != 3) return false;
-    if ((v[0] != 1 && v[0] != 2 && v[0] != 4) || v[1] < 1 || v[1] > 8 || v[2] < 0 || v[2] > 16)
+    int v[4] = {0, 0, 0, 1};
+    const int n = sscanf(e, "%d,%d,%d,%d", &v[0], &v[1], &v[2], &v[3]);
+    if (n < 3 || !tiling_known(v[0], v[3]) || v[1] < 1 || v[1] > 8 || v[2] < 0 || v[2] > 16)
         return false;
-    *pl = {v[0], v[1], v[2]};
+    *pl = {v[0], v[3], v[1], v[2]};
     return true;
 }
 
-constexpr int kSmemBudget = 110 * 1024;
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
-size_t smem_bytes_for(int wm, int S, int B, int p, int slabs_per_rank, int nslot, GemvArgs *a) {
-    const int BM = 16 * wm;
-    const int NT = B > 8 ? 2 : 1;
-    size_t off = static_cast<size_t>(nslot) * S * BM * (kCodeRow + kNormRow);
+// Shared-memory carve-up after the ring (common to both kernels).
+size_t layout_tail(size_t off, int B, int nar, int q8_bytes, int pidx_cap, int red_bytes,
+                   int cl_bytes, int prot_bytes, int nbars, GemvArgs *a) {
     a->off_xt = static_cast<uint32_t>(off);
-    a->xt_pitch = slabs_per_rank * 1024 + 64;
+    a->xt_pitch = nar * 1024 + 64;   // +64 B: rows g and g+1 land in different banks
     off += static_cast<size_t>(B) * a->xt_pitch;
-    off = (off + 127) & ~size_t(127);
+    off = align_up(off, 128);
     a->off_q8 = static_cast<uint32_t>(off);
-    a->q8_boxes = p > 0 ? (p + 15 + 127) / 128 : 0;
-    off += static_cast<size_t>(a->q8_boxes) * BM * 128;
-    a->off_xs = static_cast<uint32_t>(off);
-    a->xs_pitch = ((p + 15) & ~15) + 8;
-    off += static_cast<size_t>(2) * B * a->xs_pitch * 2;
-    off = (off + 15) & ~size_t(15);
+    off += q8_bytes;
+    a->pidx_cap = pidx_cap;
+    a->off_pidx = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(2 + B) * pidx_cap * 4;   // indices, scales, scale * x
+    a->off_pmask = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(nar) * (kSlab / 32) * 4;
+    a->off_pu = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(nar) * (kSlab / 32) * 4;
+    off = align_up(off, 16);
+    a->off_zero = static_cast<uint32_t>(off);
+    off += 1024;
     a->off_red = static_cast<uint32_t>(off);
-    off += static_cast<size_t>(BM) * 8 * NT * 4;
+    off += red_bytes;
+    a->off_cl = static_cast<uint32_t>(off);
+    off += cl_bytes;
+    a->off_prot = static_cast<uint32_t>(off);
+    off += prot_bytes;
+    off = align_up(off, 8);
     a->off_bar = static_cast<uint32_t>(off);
-    off += static_cast<size_t>(2 * nslot + 1) * 8;
-    return off + 1024;   // alignment slack for the 1024-byte aligned base
+    off += static_cast<size_t>(nbars) * 8;
+    return off + 1024;   // slack for the 1024-byte aligned base
 }
 
-Plan choose_plan(int N, int K, int B, int S) {
+size_t cluster_smem(int wm, int wq, int ck, int S, int B, int p, int wide_per_rank, int nslot,
+                    GemvArgs *a) {
+    const int BM = 16 * wm, BP = B > 8 ? 16 : 8, SW = kSlab * wq;
+    const int nar = wide_per_rank * wq;
+    const int cap = static_cast<int>(align_up(static_cast<size_t>(std::min(p, nar * kSlab)), 16));
+    const int q8_boxes = p > 0 ? (cap + 15 + 127) / 128 : 0;   // bound per CTA
+    const size_t ring = static_cast<size_t>(nslot) * S * BM * (SW / 8 + SW / 4);
+    return layout_tail(ring, B, nar, q8_boxes * BM * 128, cap, wq * BM * BP * 4,
+                       (ck > 1 ? ck - 1 : 0) * BM * BP * 4, 0, nslot * 2 + 2, a);
+}
+
+size_t stream_smem(int wq, int wk, int S, int B, int K, int p, int nslot, GemvArgs *a) {
+    const int BM = 16, BP = 8, SW = kSlab * wq;
+    const int nar = (K + kSlab - 1) / kSlab;
+    const int cap = static_cast<int>(align_up(static_cast<size_t>(p), 16));
+    const int q8_boxes = p > 0 ? (cap + 127) / 128 : 0;
+    const size_t ring = static_cast<size_t>(nslot) * S * BM * (SW / 8 + SW / 4);
+    return layout_tail(ring, B, nar, 2 * q8_boxes * BM * 128, cap, 2 * wq * wk * BM * BP * 4, 0,
+                       BM * BP * 4, nslot * (wk + 1) + 8, a);
+}
+
+// k_gemv tiling rule: 2048-column slots (four column-quarter warps per row
+// group), 32 rows per CTA (16 for short layers, 64 at batch > 8); the K split
+// grows until about one CTA per SM.
+Plan choose_plan(int N, int K, int B) {
     const int sms = num_sms();
-    const int total_slabs = (K + kSlab - 1) / kSlab;
-    Plan best{4, 1, 2};
-    long best_score = -1;
-    for (int wm : {4, 2, 1}) {
-        if (B > 8 && wm < 2) continue;
-        const int BM = 16 * wm;
-        const int mblocks = (N + BM - 1) / BM;
-        for (int ck = 1; ck <= 8; ++ck) {
-            const int spr = (total_slabs + ck - 1) / ck;
-            if ((ck - 1) * spr >= total_slabs) continue;          // an empty rank
-            if (static_cast<long>(B) * (spr * 1024 + 64) > 64 * 1024) continue;
-            const long ctas = static_cast<long>(mblocks) * ck;
-            // prefer ~2 resident CTAs per SM, then bigger tiles, then less split
-            const long fill = ctas >= 2L * sms ? 2L * sms : ctas;
-            const long score = fill * 64 + wm * 8 - ck;
-            if (score > best_score) {
-                best_score = score;
-                best = {wm, ck, 0};
-            }
-        }
-    }
-    return best;
+    Plan pl = B > 8 ? Plan{4, 4, 1, 0} : Plan{2, 4, 1, 0};
+    if (B <= 8 && N <= 2048) pl = {1, 4, 1, 0};
+    const int SW = kSlab * pl.wq;
+    const int total_wide = (K + SW - 1) / SW;
+    const int mblocks = (N + 16 * pl.wm - 1) / (16 * pl.wm);
+    while (pl.ck < 8 && pl.ck < total_wide && static_cast<long>(mblocks) * pl.ck < (sms * 4) / 5)
+        ++pl.ck;
+    return pl;
 }
 
-template <int WM, int NT, int S>
-bisco_status launch_t(const CUtensorMap &mc, const CUtensorMap &mn, const CUtensorMap &mq,
-                      const GemvArgs &a, int ck, size_t smem, cudaStream_t stream) {
-    auto kern = k_gemv<WM, NT, S>;
-    static size_t configured[64] = {};
+template <typename Kern>
+bool set_smem(Kern kern, size_t smem, size_t (&configured)[64]) {
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return BISCO_ERR_CUDA;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
     if (smem > configured[dev]) {
         if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  static_cast<int>(smem)) != cudaSuccess)
-            return BISCO_ERR_CUDA;
-        if (cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
-            cudaSuccess)
-            return BISCO_ERR_CUDA;
+            return false;
         configured[dev] = smem;
     }
+    return true;
+}
+
+template <int WM, int WQ, int NT, int S>
+bisco_status launch_t(const CUtensorMap &mc, const CUtensorMap &mn, const CUtensorMap &mq,
+                      const GemvArgs &a, int ck, size_t smem, cudaStream_t stream) {
+    auto kern = k_gemv<WM, WQ, NT, S>;
+    static size_t configured[64] = {};
+    if (!set_smem(kern, smem, configured)) return BISCO_ERR_CUDA;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(ck, (a.N + 16 * WM - 1) / (16 * WM), 1);
-    cfg.blockDim = dim3((WM + 1) * 32, 1, 1);
+    cfg.blockDim = dim3((WM * WQ + 1) * 32, 1, 1);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cudaLaunchAttribute attr[2];
@@ -524,13 +958,105 @@ bisco_status launch_t(const CUtensorMap &mc, const CUtensorMap &mn, const CUtens
     return cudaLaunchKernelEx(&cfg, kern, mc, mn, mq, a) == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
 }
 
-template <int WM, int NT>
+template <int WM, int WQ, int NT>
 bisco_status launch_s(int S, const CUtensorMap &mc, const CUtensorMap &mn, const CUtensorMap &mq,
                       const GemvArgs &a, int ck, size_t smem, cudaStream_t stream) {
     switch (S) {
-        case 1: return launch_t<WM, NT, 1>(mc, mn, mq, a, ck, smem, stream);
-        case 2: return launch_t<WM, NT, 2>(mc, mn, mq, a, ck, smem, stream);
-        default: return launch_t<WM, NT, 3>(mc, mn, mq, a, ck, smem, stream);
+        case 1: return launch_t<WM, WQ, NT, 1>(mc, mn, mq, a, ck, smem, stream);
+        case 2: return launch_t<WM, WQ, NT, 2>(mc, mn, mq, a, ck, smem, stream);
+        default: return launch_t<WM, WQ, NT, 3>(mc, mn, mq, a, ck, smem, stream);
+    }
+}
+
+template <int WM, int WQ>
+bisco_status launch_w(bool two, int S, const CUtensorMap &mc, const CUtensorMap &mn,
+                      const CUtensorMap &mq, const GemvArgs &a, int ck, size_t smem,
+                      cudaStream_t stream) {
+    if (two) {
+        if constexpr (WM >= 2) return launch_s<WM, WQ, 2>(S, mc, mn, mq, a, ck, smem, stream);
+        return BISCO_ERR_UNSUPPORTED;
+    }
+    return launch_s<WM, WQ, 1>(S, mc, mn, mq, a, ck, smem, stream);
+}
+
+template <int WQ, int WK, int S>
+bisco_status launch_stream_t(const CUtensorMap &mc, const CUtensorMap &mn, const CUtensorMap &mq,
+                             const GemvArgs &a, int grid, size_t smem, cudaStream_t stream) {
+    auto kern = k_gemv_stream<WQ, WK, S>;
+    static size_t configured[64] = {};
+    if (!set_smem(kern, smem, configured)) return BISCO_ERR_CUDA;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid, 1, 1);
+    cfg.blockDim = dim3((WQ * WK + 2) * 32, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, mc, mn, mq, a) == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+}
+
+// Tensor maps of one layer: signs and norms as [S][N][K/8] boxes of
+// rows x SW columns (all S stages), q8 as [N][p_pad] boxes of rows x 128.
+bool layer_maps(const bisco_layer &L, int rows, int SW, bool swz, CUtensorMap *mc, CUtensorMap *mn,
+                CUtensorMap *mq) {
+    const int N = L.n_out, K = L.k_in, S = L.stages, p = L.n_protected;
+    const uint64_t dims[3] = {static_cast<uint64_t>(K / 8), static_cast<uint64_t>(N),
+                              static_cast<uint64_t>(S)};
+    const uint64_t strides[2] = {static_cast<uint64_t>(K / 8), static_cast<uint64_t>(N) * (K / 8)};
+    const uint32_t box[3] = {static_cast<uint32_t>(SW / 8), static_cast<uint32_t>(rows),
+                             static_cast<uint32_t>(S)};
+    const uint64_t nstrides[2] = {static_cast<uint64_t>(K / 4), static_cast<uint64_t>(N) * (K / 4)};
+    if (!encode_tensor_map(mc, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, L.codes, dims, strides, box,
+                           CU_TENSOR_MAP_SWIZZLE_NONE) ||
+        !encode_tensor_map(mn, CU_TENSOR_MAP_DATA_TYPE_UINT16, 3, L.norms, dims, nstrides, box,
+                           swz ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE))
+        return false;
+    if (p > 0) {
+        const int p_pad = (p + 15) / 16 * 16;
+        const uint64_t qd[2] = {static_cast<uint64_t>(p_pad), static_cast<uint64_t>(N)};
+        const uint64_t qs[1] = {static_cast<uint64_t>(p_pad)};
+        const uint32_t qb[2] = {128, static_cast<uint32_t>(rows)};
+        if (!encode_tensor_map(mq, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, L.q8, qd, qs, qb,
+                               CU_TENSOR_MAP_SWIZZLE_NONE))
+            return false;
+    } else {
+        *mq = *mc;   // never dereferenced when p == 0
+    }
+    return true;
+}
+
+// Ring depth: as many slots as fit next to `rest` bytes within `budget`,
+// clamped to [lo, hi].
+int fit_slots(size_t rest, size_t slot, size_t budget, int lo, int hi) {
+    const long fit = rest < budget ? static_cast<long>((budget - rest) / slot) : 0;
+    return static_cast<int>(fit < lo ? lo : (fit > hi ? hi : fit));
+}
+
+bisco_status launch_stream(const bisco_layer &L, GemvArgs &a, int sms, cudaStream_t stream,
+                           bool *launched) {
+    constexpr int WQ = 4, WK = 2;
+    const int N = L.n_out, K = L.k_in, S = L.stages, p = L.n_protected, B = a.B;
+    *launched = false;
+    const size_t slot = static_cast<size_t>(S) * 16 * (kSlab * WQ / 8 + kSlab * WQ / 4);
+    int nslot = 0;
+    if (const char *e = getenv("BISCO_GEMV_NSLOT")) nslot = atoi(e);
+    if (nslot <= 0 || nslot > 16)
+        nslot = fit_slots(stream_smem(WQ, WK, S, B, K, p, 0, &a), slot, kCoresident, 2, 8);
+    const size_t smem = stream_smem(WQ, WK, S, B, K, p, nslot, &a);
+    if (smem > kMaxSmem) return BISCO_OK;   // caller falls back to k_gemv
+    a.nslot = nslot;
+    const int ntiles = (N + 15) / 16;
+    const int grid = ntiles < sms ? ntiles : sms;
+    CUtensorMap mc, mn, mq;
+    if (!layer_maps(L, 16, kSlab * WQ, false, &mc, &mn, &mq)) return BISCO_ERR_CUDA;
+    *launched = true;
+    switch (S) {
+        case 1: return launch_stream_t<WQ, WK, 1>(mc, mn, mq, a, grid, smem, stream);
+        case 2: return launch_stream_t<WQ, WK, 2>(mc, mn, mq, a, grid, smem, stream);
+        default: return launch_stream_t<WQ, WK, 3>(mc, mn, mq, a, grid, smem, stream);
     }
 }
 
@@ -539,19 +1065,13 @@ bisco_status launch_s(int S, const CUtensorMap &mc, const CUtensorMap &mn, const
 bisco_status launch_gemv(const bisco_layer &L, const uint16_t *x, int B, float *y, int *err,
                          cudaStream_t stream) {
     const int N = L.n_out, K = L.k_in, S = L.stages, p = L.n_protected;
-    if (K % 128 != 0) {
+    auto generic = [&]() -> bisco_status {
         const int rows_per_block = 8;
         k_gemv_generic<<<(N + rows_per_block - 1) / rows_per_block, 32 * rows_per_block, 0, stream>>>(
             L.codes, L.norms, L.q8, L.q8_scale, L.prot_idx, N, K, S, p, x, B, y);
         return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
-    }
-    Plan pl = choose_plan(N, K, B, S);
-    plan_override(&pl);
-    if (B > 8 && pl.wm < 2) pl.wm = 2;
-    const int BM = 16 * pl.wm;
-    const int total_slabs = (K + kSlab - 1) / kSlab;
-    if (pl.ck > total_slabs) pl.ck = total_slabs;
-    const int spr = (total_slabs + pl.ck - 1) / pl.ck;
+    };
+    if (K % 128 != 0) return generic();   // row pitch rules out TMA
 
     GemvArgs a = {};
     a.x = x;
@@ -563,61 +1083,61 @@ bisco_status launch_gemv(const bisco_layer &L, const uint16_t *x, int B, float *
     a.K = K;
     a.B = B;
     a.p = p;
-    a.slabs_per_rank = spr;
-    a.total_slabs = total_slabs;
-    // ring depth: as many slots as fit next to the rest, 2..8
-    int nslot = pl.nslot;
-    if (nslot <= 0) {
-        const size_t rest = smem_bytes_for(pl.wm, S, B, p, spr, 0, &a);
-        const size_t slot = static_cast<size_t>(S) * BM * (kCodeRow + kNormRow);
-        long fit = rest < static_cast<size_t>(kSmemBudget) ? (kSmemBudget - static_cast<long>(rest)) / static_cast<long>(slot) : 0;
-        nslot = static_cast<int>(fit < 2 ? 2 : (fit > 8 ? 8 : fit));
-        if (nslot > spr && spr >= 2) nslot = spr;
-        if (nslot < 2) nslot = 2;
-    }
-    a.nslot = nslot;
-    const size_t smem = smem_bytes_for(pl.wm, S, B, p, spr, nslot, &a);
-    if (smem > 227 * 1024) return BISCO_ERR_UNSUPPORTED;
 
+    // streaming kernel: small batch and at least one 16-row tile per SM
+    const char *mode = getenv("BISCO_GEMV_MODE");
+    const int sms = num_sms();
+    bool use_stream = B <= 8 && (N + 15) / 16 >= sms;
+    if (mode && mode[0] == 's') use_stream = B <= 8;
+    if (mode && mode[0] == 'c') use_stream = false;
+    if (use_stream) {
+        bool launched = false;
+        const bisco_status st = launch_stream(L, a, sms, stream, &launched);
+        if (launched || st != BISCO_OK) return st;
+    }
+
+    Plan pl = choose_plan(N, K, B);
+    plan_override(&pl);
+    if (B > 8 && pl.wm < 2) pl = {2, pl.wq, pl.ck, pl.nslot};
+    if (!tiling_known(pl.wm, pl.wq)) pl = {2, 4, pl.ck, pl.nslot};
+    const int BM = 16 * pl.wm;
+    const int SW = kSlab * pl.wq;
+    const int total_wide = (K + SW - 1) / SW;
+    if (pl.ck > total_wide) pl.ck = total_wide;
+    const size_t slot = static_cast<size_t>(S) * BM * (SW / 8 + SW / 4);
+    // split K further until the staged activations and a 2-slot ring fit
+    int wpr = 0, nslot = 0;
+    size_t smem = 0;
+    for (;;) {
+        wpr = (total_wide + pl.ck - 1) / pl.ck;
+        nslot = pl.nslot;
+        if (nslot <= 0) {
+            nslot = fit_slots(cluster_smem(pl.wm, pl.wq, pl.ck, S, B, p, wpr, 0, &a), slot,
+                              kCoresident, 2, 8);
+            if (nslot > wpr && wpr >= 2) nslot = wpr;
+        }
+        if (nslot < 2) nslot = 2;
+        smem = cluster_smem(pl.wm, pl.wq, pl.ck, S, B, p, wpr, nslot, &a);
+        if (smem <= kMaxSmem) break;
+        if (pl.ck >= 8 || pl.ck >= total_wide) return generic();   // e.g. p close to K
+        ++pl.ck;
+    }
+    a.wide_per_rank = wpr;
+    a.nslot = nslot;
     CUtensorMap mc, mn, mq;
-    {
-        const uint64_t dims[3] = {static_cast<uint64_t>(K / 8), static_cast<uint64_t>(N),
-                                  static_cast<uint64_t>(S)};
-        const uint64_t strides[2] = {static_cast<uint64_t>(K / 8),
-                                     static_cast<uint64_t>(N) * (K / 8)};
-        const uint32_t box[3] = {static_cast<uint32_t>(kCodeRow), static_cast<uint32_t>(BM),
-                                 static_cast<uint32_t>(S)};
-        if (!encode_tensor_map(&mc, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, L.codes, dims, strides, box,
-                               CU_TENSOR_MAP_SWIZZLE_NONE))
-            return BISCO_ERR_CUDA;
-        const uint64_t nstrides[2] = {static_cast<uint64_t>(K / 4),
-                                      static_cast<uint64_t>(N) * (K / 4)};
-        const uint32_t nbox[3] = {static_cast<uint32_t>(kCodeRow), static_cast<uint32_t>(BM),
-                                  static_cast<uint32_t>(S)};
-        if (!encode_tensor_map(&mn, CU_TENSOR_MAP_DATA_TYPE_UINT16, 3, L.norms, dims, nstrides,
-                               nbox, CU_TENSOR_MAP_SWIZZLE_128B))
-            return BISCO_ERR_CUDA;
-    }
-    if (p > 0) {
-        const int p_pad = (p + 15) / 16 * 16;
-        const uint64_t dims[2] = {static_cast<uint64_t>(p_pad), static_cast<uint64_t>(N)};
-        const uint64_t strides[1] = {static_cast<uint64_t>(p_pad)};
-        const uint32_t box[2] = {128, static_cast<uint32_t>(BM)};
-        if (!encode_tensor_map(&mq, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, L.q8, dims, strides, box,
-                               CU_TENSOR_MAP_SWIZZLE_NONE))
-            return BISCO_ERR_CUDA;
-    } else {
-        mq = mc;   // never dereferenced when p == 0
-    }
+    if (!layer_maps(L, BM, SW, pl.wq == 1, &mc, &mn, &mq)) return BISCO_ERR_CUDA;
 
     const bool two = B > 8;
-    switch (pl.wm) {
-        case 1: return two ? BISCO_ERR_UNSUPPORTED : launch_s<1, 1>(S, mc, mn, mq, a, pl.ck, smem, stream);
-        case 2: return two ? launch_s<2, 2>(S, mc, mn, mq, a, pl.ck, smem, stream)
-                           : launch_s<2, 1>(S, mc, mn, mq, a, pl.ck, smem, stream);
-        default: return two ? launch_s<4, 2>(S, mc, mn, mq, a, pl.ck, smem, stream)
-                            : launch_s<4, 1>(S, mc, mn, mq, a, pl.ck, smem, stream);
-    }
+    const int ck = pl.ck;
+    if (pl.wm == 1 && pl.wq == 4) return launch_w<1, 4>(two, S, mc, mn, mq, a, ck, smem, stream);
+    if (pl.wm == 2 && pl.wq == 4) return launch_w<2, 4>(two, S, mc, mn, mq, a, ck, smem, stream);
+    if (pl.wm == 4 && pl.wq == 4) return launch_w<4, 4>(two, S, mc, mn, mq, a, ck, smem, stream);
+    if (pl.wm == 2 && pl.wq == 2) return launch_w<2, 2>(two, S, mc, mn, mq, a, ck, smem, stream);
+    if (pl.wm == 4 && pl.wq == 2) return launch_w<4, 2>(two, S, mc, mn, mq, a, ck, smem, stream);
+    if (pl.wm == 4 && pl.wq == 1) return launch_w<4, 1>(two, S, mc, mn, mq, a, ck, smem, stream);
+    if (pl.wm == 8 && pl.wq == 1) return launch_w<8, 1>(two, S, mc, mn, mq, a, ck, smem, stream);
+    if (pl.wm == 1 && pl.wq == 2) return launch_w<1, 2>(two, S, mc, mn, mq, a, ck, smem, stream);
+    return BISCO_ERR_UNSUPPORTED;
 }
 
 }  // namespace bisco

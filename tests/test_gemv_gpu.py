@@ -27,21 +27,26 @@ def env():
     return bisco, dev
 
 
-def run_gemv(env, Lref, X, plan=None):
+def run_gemv(env, Lref, X, plan=None, extra_env=None):
+    """bisco_gemv on a device copy of the oracle's layer; `plan` forces the
+    clustered kernel with tiling "WM,CK,NSLOT,WQ", `extra_env` sets other
+    tuning variables for the call."""
     import torch
     bisco, dev = env
     L = bisco.Layer.from_numpy(Lref, dev)
-    old = os.environ.get("BISCO_GEMV_PLAN")
+    env_vars = dict(extra_env or {})
     if plan:
-        os.environ["BISCO_GEMV_PLAN"] = plan
+        env_vars.update(BISCO_GEMV_PLAN=plan, BISCO_GEMV_MODE="cluster")
+    old = {k: os.environ.get(k) for k in env_vars}
+    os.environ.update(env_vars)
     try:
         y = bisco.bisco_gemv(L, to_dev(X, dev))
     finally:
-        if plan:
-            if old is None:
-                del os.environ["BISCO_GEMV_PLAN"]
+        for k, v in old.items():
+            if v is None:
+                del os.environ[k]
             else:
-                os.environ["BISCO_GEMV_PLAN"] = old
+                os.environ[k] = v
     torch.cuda.synchronize()
     assert bisco.bisco_get_device_error() == 0
     return y.cpu().numpy()
@@ -66,17 +71,38 @@ def test_gemv_matches_oracle(env, N, K, S, p, B, dist):
     assert max_rel_rows(y, oracle.gemv(Lref, X)) <= TOL
 
 
-@pytest.mark.parametrize("plan", ["1,1,2", "1,4,3", "2,2,4", "4,8,2", "4,3,2", "2,5,3",
-                                  "1,2,8", "4,1,2"])
+@pytest.mark.parametrize("plan", ["1,1,0,4", "2,2,0,4", "4,4,3,4", "2,1,2,2", "4,3,2,2",
+                                  "4,8,2,1", "8,1,0,1", "1,2,0,2", "2,5,3,2", "4,1,8,1"])
 @pytest.mark.parametrize("B", [1, 5, 16])
 def test_gemv_every_tiling(env, plan, B):
-    """All tile heights, cluster split-K factors (including ranks left with
-    no slab) and ring depths give the same answer."""
+    """Every tile height and slot width of the clustered kernel, cluster
+    split-K factors (including ranks left with no columns) and ring depths
+    give the same answer."""
     N, K, S, p = 208, 4096, 2, 41
     W = synth.layer_weights(N, K, seed=2)
     X = synth.activations(B, K, seed=3)
     Lref = oracle.encode(W, S=S, p=p)
     y = run_gemv(env, Lref, X, plan=plan)
+    assert max_rel_rows(y, oracle.gemv(Lref, X)) <= TOL
+
+
+@pytest.mark.parametrize("N,K,S,p,B,nslot", [
+    (100, 1536, 3, 20, 3, 2),      # one tile per CTA, ragged rows, K not a slot multiple
+    (208, 4096, 2, 41, 1, 3),      # odd ring depth
+    (64, 640, 1, 0, 8, 2),         # no protection, B = 8
+    (2500, 1024, 2, 11, 1, 2),     # several tiles per CTA, ring wraps across tiles
+    (2500, 1024, 2, 11, 5, 7),
+    (2500, 2176, 3, 23, 2, 4),     # a slot straddles the end of K
+    (5000, 512, 2, 300, 1, 5),     # three q8 boxes per tile, many tiles per CTA
+])
+def test_gemv_streaming_path(env, N, K, S, p, B, nslot):
+    """The persistent streaming kernel (reducer warp, int8 slab double
+    buffer, ring carried across tiles) at forced ring depths."""
+    W = synth.layer_weights(N, K, seed=N + p)
+    X = synth.activations(B, K, seed=B + 1)
+    Lref = oracle.encode(W, S=S, p=p)
+    y = run_gemv(env, Lref, X, extra_env={"BISCO_GEMV_MODE": "stream",
+                                         "BISCO_GEMV_NSLOT": str(nslot)})
     assert max_rel_rows(y, oracle.gemv(Lref, X)) <= TOL
 
 
