@@ -82,7 +82,7 @@ typedef struct {
 } bisco_layer;
 
 /* ABI version of this header (major * 100 + minor). */
-#define BISCO_ABI_VERSION 100
+#define BISCO_ABI_VERSION 101
 int32_t bisco_abi_version(void);
 
 /* Static string for a status code (never NULL). */
@@ -161,16 +161,28 @@ bisco_status bisco_gemv(const bisco_layer *L, const uint16_t *x_bf16, int32_t B,
                         bisco_stream_t stream);
 
 /*
- * Prefill matrix product Y[m][i] = sum_j What[i][j] * X[m][j] for any M >= 0,
- * with the same arithmetic contract as bisco_gemv.  X_bf16: [M][K] device;
- * Y: [M][N] float32 device, fully overwritten.  workspace: device, at least
- * bisco_gemm_workspace_bytes(M, N, K) bytes (may be NULL when that is 0).
+ * Prefill matrix product Y[m][i] = sum_j What[i][j] * X[m][j] for any M >= 0
+ * (Sec. III-F Eq. 12 with Eq. 10), the same quantity as bisco_gemv.  For
+ * M > 64 and K % 128 == 0 it runs on the tcgen05 tensor cores: the decoded
+ * weight (fp16, the S stages summed in fp16 -- one rounding of relative
+ * size <= 2^-11 per weight for S >= 2) against fp16 activations, fp32
+ * accumulation; the protected columns use the int8 values exactly.  Smaller
+ * M, or other K, run the decode kernels of bisco_gemv.
+ * X_bf16: [M][K] device; Y: [M][N] float32 device, fully overwritten.
+ * workspace: device, 16-byte aligned, at least
+ * bisco_gemm_workspace_bytes(L, M) bytes (M * (roundup(K,128) +
+ * 2 * roundup(p,64)) * 2 on the tensor-core path; NULL when that is 0).
+ * It holds the fp16 copy of X and is overwritten.
  */
-size_t bisco_gemm_workspace_bytes(int32_t M, int32_t N, int32_t K);
+size_t bisco_gemm_workspace_bytes(const bisco_layer *L, int32_t M);
 bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M, float *Y,
                         void *workspace, size_t workspace_bytes, bisco_stream_t stream);
 
 /*
+ * A protected-column index outside [0, K) (or a list that is not ascending)
+ * found by a kernel is skipped and latches BISCO_ERR_INVALID_ARG in the
+ * device error word.
+ *
  * Synchronises `stream`, returns the device error word of the current device
  * (BISCO_OK if clear) and clears it.  BISCO_ERR_CUDA if the synchronisation
  * itself fails.

@@ -66,7 +66,7 @@ def load(path: str = LIB_PATH):
     lib.bisco_gemv.restype = st
     lib.bisco_gemv.argtypes = [Lp, P, i32, P, P]
     lib.bisco_gemm_workspace_bytes.restype = sz
-    lib.bisco_gemm_workspace_bytes.argtypes = [i32, i32, i32]
+    lib.bisco_gemm_workspace_bytes.argtypes = [Lp, i32]
     lib.bisco_gemm.restype = st
     lib.bisco_gemm.argtypes = [Lp, P, i32, P, P, sz, P]
     lib.bisco_get_device_error.restype = st
@@ -109,8 +109,10 @@ def bisco_encode_workspace_bytes(N, K) -> int:
     return int(load().bisco_encode_workspace_bytes(N, K))
 
 
-def bisco_gemm_workspace_bytes(M, N, K) -> int:
-    return int(load().bisco_gemm_workspace_bytes(M, N, K))
+def bisco_gemm_workspace_bytes(L, M) -> int:
+    """Workspace bytes bisco_gemm needs for layer L (a Layer or its C struct)."""
+    c = L.c if isinstance(L, Layer) else L
+    return int(load().bisco_gemm_workspace_bytes(ctypes.byref(c), M))
 
 
 class Layer:
@@ -221,7 +223,7 @@ def bisco_gemm(L: Layer, X_bits, Y=None, workspace=None, stream=None):
     assert X_bits.is_contiguous() and X_bits.shape[1] == L.K
     if Y is None:
         Y = torch.empty((M, L.N), dtype=torch.float32, device=X_bits.device)
-    need = bisco_gemm_workspace_bytes(M, L.N, L.K)
+    need = bisco_gemm_workspace_bytes(L, M)
     if need and workspace is None:
         workspace = torch.empty(need, dtype=torch.uint8, device=X_bits.device)
     nbytes = 0 if workspace is None else workspace.numel()

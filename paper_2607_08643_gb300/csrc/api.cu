@@ -178,9 +178,9 @@ bisco_status bisco_gemv(const bisco_layer *L, const uint16_t *x_bf16, int32_t B,
     return launch_gemv(*L, x_bf16, B, y, err, reinterpret_cast<cudaStream_t>(stream));
 }
 
-size_t bisco_gemm_workspace_bytes(int32_t M, int32_t N, int32_t K) {
-    if (M < 0 || N < 1 || K < 8 || K % 8) return 0;
-    return gemm_workspace_bytes(M, N, K);
+size_t bisco_gemm_workspace_bytes(const bisco_layer *L, int32_t M) {
+    if (M < 0 || check_layer(L, false) != BISCO_OK) return 0;
+    return gemm_workspace_bytes(*L, M);
 }
 
 bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M, float *Y,
@@ -190,7 +190,7 @@ bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M,
     if (M < 0) return BISCO_ERR_INVALID_ARG;
     if (M == 0) return BISCO_OK;
     if (!X_bf16 || !Y || !aligned16(X_bf16) || !aligned16(Y)) return BISCO_ERR_INVALID_ARG;
-    const size_t need = gemm_workspace_bytes(M, L->n_out, L->k_in);
+    const size_t need = gemm_workspace_bytes(*L, M);
     if (need && (!workspace || !aligned16(workspace) || workspace_bytes < need))
         return BISCO_ERR_INVALID_ARG;
     int *err = device_error_word(&st);

@@ -1,23 +1,397 @@
-// gemm.cu -- prefill Y = X What^T (Sec. III-F Eq. 12 with Eq. 10).
-// Interim path: tiles of 16 activation rows through the decode kernel.
+// gemm.cu -- prefill Y = X What^T (Sec. III-F Eq. 12 with the Eq. 10
+// protected scatter) on the 5th-generation tensor cores.
+//
+// Prefill is a dense contraction, so the decoded weight feeds tcgen05.mma
+// (kind::f16, fp32 accumulation in tensor memory).  The weight is never
+// written out: per 128-column step, decoder warps expand the TMA-staged sign
+// bytes and fp16 norms of 128 output features into fp16 values in registers
+// (shift + LOP3 per element pair, the S stages summed with one fp16 add per
+// stage, Eq. 12) and store them straight into tensor memory, where they are
+// the MMA's A operand (M = 128 features).  The activations are the B operand
+// (N = 256 tokens), TMA-staged in the 128-byte swizzle.
+//
+// The activations are bf16 and the decoded weight fp16; one MMA needs one
+// type, so a pre-pass writes an fp16 copy of X into the workspace with the
+// protected columns zeroed (Eq. 10's overwrite) and, appended after the
+// K columns, sqrt(8) * scale_j * x_j split into fp16 hi and lo parts in
+// blocks of 64 protected columns [hi | lo].  The matching A columns are the
+// int8 q8 values (exact in fp16), so the protected term is a few more k
+// steps of the same MMA, and the epilogue is Y = D / sqrt(8).
+//
+// CTA roles (512 threads, one CTA per SM, persistent over output tiles):
+//   warps 0-3  epilogue: TMEM -> registers -> Y (fp32), lane quarter w
+//   warp 4     TMA producer (activation ring, compressed-weight ring)
+//   warp 5     TMEM allocator and MMA issuer (one thread)
+//   warps 8-15 decoders: lane quarter w % 4, K half (w - 8) / 4
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "bisco_dev.cuh"
 #include "bisco_host.h"
 
 namespace bisco {
+namespace {
 
-size_t gemm_workspace_bytes(int M, int N, int K) {
-    (void)M;
-    (void)N;
-    (void)K;
-    return 0;
+constexpr int GM = 128;     // output features per tile (MMA M, TMEM lanes)
+constexpr int GN = 256;     // tokens per tile (MMA N)
+constexpr int GK = 128;     // K columns per weight step (one TMEM A stage)
+constexpr int NX = 4;       // activation ring (64-column, 32 KB stages)
+constexpr int NW = 4;       // compressed-weight ring (128-column stages)
+constexpr int NA = 3;       // TMEM A ring (128 K columns = 64 TMEM columns each)
+constexpr int kThreads = 512;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kColD = 0;     // accumulator: 256 fp32 columns
+constexpr uint32_t kColA = 256;   // A stages
+constexpr uint32_t kXStage = GN * 128;   // 256 rows x 64 fp16
+constexpr float kInvSqrt8 = 0.35355339059327373f;
+constexpr float kSqrt8 = 2.8284271247461903f;
+
+struct GemmArgs {
+    float *Y;
+    int *err;
+    int M, N, S;
+    int ks_main;    // 128-column weight steps over K (K_pad / 128)
+    int ks_ext;     // extension steps (one per 64 protected columns)
+    int tiles_t;    // token tiles
+    int ntiles;
+    uint32_t w_stage;   // bytes of one compressed-weight stage
+};
+
+// idesc of kind::f16: D f32, A = B = f16, both K-major, N = GN, M = GM.
+constexpr uint32_t kIdesc = (1u << 4) | (static_cast<uint32_t>(GN >> 3) << 17) |
+                            (static_cast<uint32_t>(GM >> 4) << 24);
+
+// Decoded fp16 pairs of 8 chunks (64 columns) of one row and S stages:
+// element pair (2j, 2j+1) of chunk c is ((t << (15-2j)) & 0x80008000) ^
+// (n|n<<16) with t = byte * 0x8001 (bit k at k and at k+15), stages summed
+// in fp16.  out[4c + j] holds K columns 8c + 2j, 8c + 2j + 1.
+__device__ __forceinline__ void decode_row64(const unsigned char *codes, const unsigned char *norms,
+                                             int S, int r, int h, uint32_t (&out)[32]) {
+#pragma unroll 1
+    for (int s = 0; s < S; ++s) {
+        const uint2 cw = *reinterpret_cast<const uint2 *>(codes + (s * GM + r) * 16 + h * 8);
+        const uint4 nw = *reinterpret_cast<const uint4 *>(norms + (s * GM + r) * 32 + h * 16);
+        const uint32_t nv[4] = {nw.x, nw.y, nw.z, nw.w};
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+            const uint32_t word = c < 4 ? cw.x : cw.y;
+            const uint32_t b = prmt(word, 0u, 0x4440u + (c & 3));       // byte c, zero-extended
+            const uint32_t t = b * 0x8001u;
+            const uint32_t np = prmt(nv[c >> 1], 0u, (c & 1) ? 0x3232u : 0x1010u);   // n | n << 16
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const uint32_t v = lop3_and_xor(t << (15 - 2 * j), 0x80008000u, np);
+                if (s == 0) {
+                    out[4 * c + j] = v;
+                } else {
+                    __half2 a = *reinterpret_cast<const __half2 *>(&out[4 * c + j]);
+                    a = __hadd2(a, *reinterpret_cast<const __half2 *>(&v));
+                    out[4 * c + j] = *reinterpret_cast<const uint32_t *>(&a);
+                }
+            }
+        }
+    }
 }
 
-bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *Y,
-                         void *workspace, size_t ws_bytes, int *err, cudaStream_t stream) {
-    (void)workspace;
-    (void)ws_bytes;
+// 64 int8 q8 values of one row -> fp16 pairs (exact): bytes biased by 128
+// become the mantissa of 1024 + u, minus 1152.
+__device__ __forceinline__ void decode_q8_row(const unsigned char *q8s, int r, uint32_t (&out)[32]) {
+    const __half2 bias = __floats2half2_rn(1152.f, 1152.f);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const uint4 v = *reinterpret_cast<const uint4 *>(q8s + r * 64 + 16 * i);
+        const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const uint32_t x = w4[q] ^ 0x80808080u;
+            uint32_t lo = prmt(x, 0x64646464u, 0x5140u);
+            uint32_t hi = prmt(x, 0x64646464u, 0x7362u);
+            __half2 a = __hsub2(*reinterpret_cast<const __half2 *>(&lo), bias);
+            __half2 b = __hsub2(*reinterpret_cast<const __half2 *>(&hi), bias);
+            out[8 * i + 2 * q] = *reinterpret_cast<const uint32_t *>(&a);
+            out[8 * i + 2 * q + 1] = *reinterpret_cast<const uint32_t *>(&b);
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_codes,
+       const __grid_constant__ CUtensorMap tm_norms, const __grid_constant__ CUtensorMap tm_q8,
+       const GemmArgs a) {
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    const uint32_t sbase = smem_u32(sm);
+    __shared__ uint32_t s_tmem;
+    __shared__ int s_abort;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t x_ring = sbase;
+    const uint32_t w_ring = sbase + NX * kXStage;
+    const uint32_t bars = w_ring + NW * a.w_stage;
+    const uint32_t xfull = bars, xempty = xfull + 8 * NX;
+    const uint32_t wfull = xempty + 8 * NX, wempty = wfull + 8 * NW;
+    const uint32_t afull = wempty + 8 * NW, aempty = afull + 8 * NA;
+    const uint32_t dfull = aempty + 8 * NA, dempty = dfull + 8, drain = dempty + 8;
+    const int ksteps = a.ks_main + a.ks_ext;
+    const int S = a.S;
+    const uint32_t wbytes_main = static_cast<uint32_t>(S) * GM * 48;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < NX; ++i) {
+            mbar_init(xfull + 8 * i, 1);
+            mbar_init(xempty + 8 * i, 1);
+        }
+        for (int i = 0; i < NW; ++i) {
+            mbar_init(wfull + 8 * i, 1);
+            mbar_init(wempty + 8 * i, 8);
+        }
+        for (int i = 0; i < NA; ++i) {
+            mbar_init(afull + 8 * i, 8);
+            mbar_init(aempty + 8 * i, 1);
+        }
+        mbar_init(dfull, 1);
+        mbar_init(dempty, 4);
+        mbar_init(drain, 1);
+        fence_mbar_init();
+        s_abort = 0;
+    }
+    if (warp == 5) tmem_alloc(smem_u32(&s_tmem), kTmemCols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = s_tmem;
+    auto aborted = [&]() { return *reinterpret_cast<volatile int *>(&s_abort) != 0; };
+    auto fail = [&]() {
+        latch_error(a.err, BISCO_ERR_TIMEOUT);
+        atomicExch(&s_abort, 1);
+    };
+
+    if (warp == 4) {
+        // ------------------------------------------------------ producer
+        if (lane == 0) {
+            prefetch_tmap(&tm_x);
+            prefetch_tmap(&tm_codes);
+            prefetch_tmap(&tm_norms);
+            int xi = 0, wi = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; ok && t < a.ntiles; t += gridDim.x) {
+                const int f0 = (t / a.tiles_t) * GM, t0 = (t % a.tiles_t) * GN;
+                for (int ks = 0; ks < ksteps; ++ks) {
+                    const int ws = wi % NW;
+                    if (wi >= NW && !mbar_wait(wempty + 8 * ws, ((wi / NW) - 1) & 1)) { ok = false; break; }
+                    if (aborted()) { ok = false; break; }
+                    const uint32_t wdst = w_ring + ws * a.w_stage;
+                    if (ks < a.ks_main) {
+                        mbar_arrive_expect_tx(wfull + 8 * ws, wbytes_main);
+                        // weights are re-read by the CTAs working on the other token tiles
+                        // of this feature tile: normal L2 policy
+                        tma_load_3d(wdst, &tm_codes, wfull + 8 * ws, ks * (GK / 8), f0, 0);
+                        tma_load_3d(wdst + S * GM * 16, &tm_norms, wfull + 8 * ws, ks * (GK / 8), f0, 0);
+                    } else {
+                        mbar_arrive_expect_tx(wfull + 8 * ws, GM * 64);
+                        tma_load_2d(wdst, &tm_q8, wfull + 8 * ws, (ks - a.ks_main) * 64, f0);
+                    }
+                    ++wi;
+                    for (int hh = 0; hh < 2; ++hh) {
+                        const int xs = xi % NX;
+                        if (xi >= NX && !mbar_wait(xempty + 8 * xs, ((xi / NX) - 1) & 1)) { ok = false; break; }
+                        mbar_arrive_expect_tx(xfull + 8 * xs, kXStage);
+                        tma_load_2d(x_ring + xs * kXStage, &tm_x, xfull + 8 * xs, ks * GK + hh * 64, t0);
+                        ++xi;
+                    }
+                    if (!ok) break;
+                }
+            }
+            if (!ok) fail();
+            // every copy issued has landed before this thread leaves (in the
+            // normal case the consumers saw them all, so this returns at once)
+            for (int i = (wi > NW ? wi - NW : 0); i < wi; ++i) mbar_wait(wfull + 8 * (i % NW), (i / NW) & 1);
+            for (int i = (xi > NX ? xi - NX : 0); i < xi; ++i) mbar_wait(xfull + 8 * (i % NX), (i / NX) & 1);
+        }
+    } else if (warp == 5) {
+        // --------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            int xi = 0, ai = 0, ti = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; ok && t < a.ntiles; t += gridDim.x, ++ti) {
+                if (ti > 0 && !mbar_wait(dempty, (ti - 1) & 1)) { ok = false; break; }
+                tc_fence_after();
+                for (int ks = 0; ks < ksteps && ok; ++ks) {
+                    const int as = ai % NA;
+                    if (!mbar_wait(afull + 8 * as, (ai / NA) & 1) || aborted()) { ok = false; break; }
+                    tc_fence_after();
+                    for (int hh = 0; hh < 2; ++hh) {
+                        const int xs = xi % NX;
+                        if (!mbar_wait(xfull + 8 * xs, (xi / NX) & 1)) { ok = false; break; }
+                        tc_fence_after();
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk) {
+                            const uint32_t a_tmem = tmem + kColA + as * 64 + hh * 32 + kk * 8;
+                            const uint64_t bdesc = smem_desc_sw128(x_ring + xs * kXStage + kk * 32);
+                            tc_mma_f16_ta(tmem + kColD, a_tmem, bdesc, kIdesc, (ks | hh | kk) != 0);
+                        }
+                        tc_commit(xempty + 8 * xs);
+                        ++xi;
+                    }
+                    tc_commit(aempty + 8 * as);
+                    ++ai;
+                }
+                if (ok) tc_commit(dfull);
+            }
+            if (!ok) fail();
+            // nothing may still be running on the tensor core when TMEM is freed
+            tc_commit(drain);
+            mbar_wait(drain, 0);
+        }
+    } else if (warp >= 8) {
+        // ------------------------------------------------------ decoders
+        const int q = warp & 3, h = (warp - 8) >> 2;
+        const int r = 32 * q + lane;
+        int wi = 0, ai = 0;
+        for (int t = blockIdx.x; t < a.ntiles; t += gridDim.x) {
+            bool ok = true;
+            for (int ks = 0; ks < ksteps; ++ks) {
+                const int ws = wi % NW, as = ai % NA;
+                if (!mbar_wait_all(wfull + 8 * ws, (wi / NW) & 1)) { ok = false; break; }
+                if (ai >= NA && !mbar_wait_all(aempty + 8 * as, ((ai / NA) - 1) & 1)) { ok = false; break; }
+                if (__any_sync(0xFFFFFFFFu, aborted())) { ok = false; break; }
+                tc_fence_after();
+                const unsigned char *wst = sm + (w_ring - sbase) + ws * a.w_stage;
+                uint32_t out[32];
+                if (ks < a.ks_main)
+                    decode_row64(wst, wst + S * GM * 16, S, r, h, out);
+                else
+                    decode_q8_row(wst, r, out);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(wempty + 8 * ws);
+                tmem_st32(tmem + (static_cast<uint32_t>(32 * q) << 16) + kColA + as * 64 + h * 32, out);
+                tmem_wait_st();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(afull + 8 * as);
+                ++wi;
+                ++ai;
+            }
+            if (!ok) {
+                if (lane == 0) fail();
+                break;
+            }
+        }
+    } else if (warp < 4) {
+        // ------------------------------------------------------ epilogue
+        const int q = warp;
+        int ti = 0;
+        for (int t = blockIdx.x; t < a.ntiles; t += gridDim.x, ++ti) {
+            if (!mbar_wait_all(dfull, ti & 1) || __any_sync(0xFFFFFFFFu, aborted())) {
+                if (lane == 0) fail();
+                break;
+            }
+            tc_fence_after();
+            const int f0 = (t / a.tiles_t) * GM, t0 = (t % a.tiles_t) * GN;
+            const int feat = f0 + 32 * q + lane;
+#pragma unroll 1
+            for (int c = 0; c < GN / 32; ++c) {
+                uint32_t v[32];
+                tmem_ld32(tmem + (static_cast<uint32_t>(32 * q) << 16) + kColD + c * 32, v);
+                tmem_wait_ld();
+                if (feat < a.N) {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) {
+                        const int tok = t0 + c * 32 + i;
+                        if (tok < a.M)
+                            a.Y[static_cast<int64_t>(tok) * a.N + feat] = __uint_as_float(v[i]) * kInvSqrt8;
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(dempty);
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 5) tmem_dealloc(tmem, kTmemCols);
+}
+
+// Activation pre-pass: X16[m][k] = fp16(x[m][k]) for k < K (0 for
+// protected k and for K <= k < K_pad); for protected block bq and u < 64,
+// X16[m][K_pad + 128 bq + u] = hi(v), X16[m][K_pad + 128 bq + 64 + u] = lo(v)
+// with v = sqrt(8) * scale_{64bq+u} * x[m][j_{64bq+u}] (0 past p).
+constexpr int kPrepRows = 16;
+
+__global__ void __launch_bounds__(256) k_gemm_prep(const uint16_t *__restrict__ X, int M, int K,
+                                                   int K_pad, int K_ext, int p,
+                                                   const int32_t *__restrict__ prot_idx,
+                                                   const uint16_t *__restrict__ q8_scale,
+                                                   uint16_t *__restrict__ X16, int *err) {
+    extern __shared__ uint32_t s_mask[];   // K_pad / 32 words
+    const int mw = K_pad / 32;
+    for (int i = threadIdx.x; i < mw; i += blockDim.x) s_mask[i] = 0u;
+    __syncthreads();
+    for (int u = threadIdx.x; u < p; u += blockDim.x) {
+        const int j = prot_idx[u];
+        if (j < 0 || j >= K) {
+            latch_error(err, BISCO_ERR_INVALID_ARG);   // not a column of this layer
+            continue;
+        }
+        atomicOr(&s_mask[j >> 5], 1u << (j & 31));
+    }
+    __syncthreads();
+    const int groups = K_ext / 8;
+    const int m0 = blockIdx.x * kPrepRows;
+    for (int e = threadIdx.x; e < kPrepRows * groups; e += blockDim.x) {
+        const int m = m0 + e / groups, k = (e % groups) * 8;
+        if (m >= M) break;
+        uint32_t o[4] = {0u, 0u, 0u, 0u};
+        const uint16_t *xr = X + static_cast<int64_t>(m) * K;
+        if (k < K_pad) {
+            if (k < K) {
+                const uint4 v = *reinterpret_cast<const uint4 *>(xr + k);
+                const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+                const uint32_t pm = (s_mask[k >> 5] >> (k & 31)) & 0xFFu;
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const float lo = (pm >> (2 * i)) & 1u ? 0.f : __uint_as_float(w[i] << 16);
+                    const float hi = (pm >> (2 * i + 1)) & 1u ? 0.f : __uint_as_float(w[i] & 0xFFFF0000u);
+                    const __half2 h2 = __floats2half2_rn(lo, hi);
+                    o[i] = *reinterpret_cast<const uint32_t *>(&h2);
+                }
+            }
+        } else {
+            const int e2 = k - K_pad, bq = e2 >> 7, part = (e2 >> 6) & 1, u0 = bq * 64 + (e2 & 63);
+            uint16_t hv[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int u = u0 + i;
+                float v = 0.f;
+                const int j = u < p ? prot_idx[u] : -1;
+                if (j >= 0 && j < K)
+                    v = (__half2float(__ushort_as_half(q8_scale[u])) *
+                         __uint_as_float(static_cast<uint32_t>(xr[j]) << 16)) * kSqrt8;
+                const __half vh = __float2half_rn(v);
+                hv[i] = part ? __half_as_ushort(__float2half_rn(v - __half2float(vh)))
+                             : __half_as_ushort(vh);
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) o[i] = hv[2 * i] | (static_cast<uint32_t>(hv[2 * i + 1]) << 16);
+        }
+        *reinterpret_cast<uint4 *>(X16 + static_cast<int64_t>(m) * K_ext + k) =
+            make_uint4(o[0], o[1], o[2], o[3]);
+    }
+}
+
+int k_pad_of(int K) { return (K + GK - 1) / GK * GK; }
+int p_ext_of(int p) { return (p + 63) / 64 * 64; }
+int k_ext_of(int K, int p) { return k_pad_of(K) + 2 * p_ext_of(p); }
+
+// The tcgen05 path needs TMA-legal strides and enough tokens to fill tiles;
+// small prefills go through the decode kernels instead.
+bool tensor_path(const bisco_layer &L, int M) { return M > 64 && L.k_in % 128 == 0; }
+
+bisco_status gemm_via_gemv(const bisco_layer &L, const uint16_t *X, int M, float *Y, int *err,
+                           cudaStream_t stream) {
     for (int m0 = 0; m0 < M; m0 += 16) {
         const int b = M - m0 < 16 ? M - m0 : 16;
         const bisco_status st = launch_gemv(L, X + static_cast<int64_t>(m0) * L.k_in, b,
@@ -25,6 +399,97 @@ bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *
         if (st != BISCO_OK) return st;
     }
     return BISCO_OK;
+}
+
+}  // namespace
+
+size_t gemm_workspace_bytes(const bisco_layer &L, int M) {
+    if (!tensor_path(L, M)) return 0;
+    return static_cast<size_t>(M) * k_ext_of(L.k_in, L.n_protected) * 2;
+}
+
+bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *Y,
+                         void *workspace, size_t ws_bytes, int *err, cudaStream_t stream) {
+    if (!tensor_path(L, M)) return gemm_via_gemv(L, X, M, Y, err, stream);
+    const int N = L.n_out, K = L.k_in, S = L.stages, p = L.n_protected;
+    const int K_pad = k_pad_of(K), K_ext = k_ext_of(K, p);
+    if (ws_bytes < gemm_workspace_bytes(L, M)) return BISCO_ERR_INVALID_ARG;
+    uint16_t *X16 = static_cast<uint16_t *>(workspace);
+
+    const size_t prep_smem = static_cast<size_t>(K_pad / 32) * 4;
+    if (prep_smem > 48 * 1024) {
+        static size_t configured[64] = {};
+        int dev = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return BISCO_ERR_CUDA;
+        if (prep_smem > configured[dev]) {
+            if (cudaFuncSetAttribute(k_gemm_prep, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(prep_smem)) != cudaSuccess)
+                return BISCO_ERR_CUDA;
+            configured[dev] = prep_smem;
+        }
+    }
+    k_gemm_prep<<<(M + kPrepRows - 1) / kPrepRows, 256, prep_smem, stream>>>(
+        X, M, K, K_pad, K_ext, p, L.prot_idx, L.q8_scale, X16, err);
+    if (cudaGetLastError() != cudaSuccess) return BISCO_ERR_CUDA;
+
+    CUtensorMap mx, mc, mn, mq;
+    {
+        const uint64_t dims[2] = {static_cast<uint64_t>(K_ext), static_cast<uint64_t>(M)};
+        const uint64_t strides[1] = {static_cast<uint64_t>(K_ext) * 2};
+        const uint32_t box[2] = {64, GN};
+        if (!encode_tensor_map(&mx, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, X16, dims, strides, box,
+                               CU_TENSOR_MAP_SWIZZLE_128B))
+            return BISCO_ERR_CUDA;
+    }
+    {
+        const uint64_t dims[3] = {static_cast<uint64_t>(K / 8), static_cast<uint64_t>(N),
+                                  static_cast<uint64_t>(S)};
+        const uint64_t cs[2] = {static_cast<uint64_t>(K / 8), static_cast<uint64_t>(N) * (K / 8)};
+        const uint64_t ns[2] = {static_cast<uint64_t>(K / 4), static_cast<uint64_t>(N) * (K / 4)};
+        const uint32_t box[3] = {GK / 8, GM, static_cast<uint32_t>(S)};
+        if (!encode_tensor_map(&mc, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, L.codes, dims, cs, box,
+                               CU_TENSOR_MAP_SWIZZLE_NONE) ||
+            !encode_tensor_map(&mn, CU_TENSOR_MAP_DATA_TYPE_UINT16, 3, L.norms, dims, ns, box,
+                               CU_TENSOR_MAP_SWIZZLE_NONE))
+            return BISCO_ERR_CUDA;
+    }
+    if (p > 0) {
+        const int p_pad = (p + 15) / 16 * 16;
+        const uint64_t dims[2] = {static_cast<uint64_t>(p_pad), static_cast<uint64_t>(N)};
+        const uint64_t strides[1] = {static_cast<uint64_t>(p_pad)};
+        const uint32_t box[2] = {64, GM};
+        if (!encode_tensor_map(&mq, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, L.q8, dims, strides, box,
+                               CU_TENSOR_MAP_SWIZZLE_NONE))
+            return BISCO_ERR_CUDA;
+    } else {
+        mq = mc;   // never dereferenced when p == 0
+    }
+
+    GemmArgs a = {};
+    a.Y = Y;
+    a.err = err;
+    a.M = M;
+    a.N = N;
+    a.S = S;
+    a.ks_main = K_pad / GK;
+    a.ks_ext = p_ext_of(p) / 64;
+    a.tiles_t = (M + GN - 1) / GN;
+    a.ntiles = a.tiles_t * ((N + GM - 1) / GM);
+    a.w_stage = static_cast<uint32_t>(S * GM * 48 > GM * 64 ? S * GM * 48 : GM * 64);
+    const size_t smem = 1024 + NX * kXStage + NW * a.w_stage + 8 * (2 * NX + 2 * NW + 2 * NA + 3);
+    static size_t configured[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return BISCO_ERR_CUDA;
+    if (smem > configured[dev]) {
+        if (cudaFuncSetAttribute(k_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(smem)) != cudaSuccess)
+            return BISCO_ERR_CUDA;
+        configured[dev] = smem;
+    }
+    const int sms = num_sms();
+    const int grid = a.ntiles < sms ? a.ntiles : sms;
+    k_gemm<<<grid, kThreads, smem, stream>>>(mx, mc, mn, mq, a);
+    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
 }
 
 }  // namespace bisco

@@ -256,11 +256,19 @@ __device__ __forceinline__ void stage_protected_meta(const GemvArgs &a, int k_be
         hi += __popc(__ballot_sync(0xFFFFFFFFu, v < k_end));
     }
     __syncwarp();
+    // an ascending index list puts at most pidx_cap entries in [k_begin,
+    // k_end); anything else is not a valid layer and is reported, not used
+    if (hi - lo > a.pidx_cap) {
+        if (lane == 0) latch_error(a.err, BISCO_ERR_INVALID_ARG);
+        hi = lo + a.pidx_cap;
+    }
     for (int u = lane; u < hi - lo; u += 32) {
         const int j = a.prot_idx[lo + u];
-        s_pidx[u] = j;
-        s_pscale[u] = __half2float(__ushort_as_half(a.q8_scale[lo + u]));
-        atomicOr(&s_pmask[(j - k_begin) >> 5], 1u << ((j - k_begin) & 31));
+        const bool in_range = j >= k_begin && j < k_end;
+        if (!in_range) latch_error(a.err, BISCO_ERR_INVALID_ARG);
+        s_pidx[u] = in_range ? j : k_begin;
+        s_pscale[u] = in_range ? __half2float(__ushort_as_half(a.q8_scale[lo + u])) : 0.f;
+        if (in_range) atomicOr(&s_pmask[(j - k_begin) >> 5], 1u << ((j - k_begin) & 31));
     }
     __syncwarp();
     int run = 0;
@@ -766,7 +774,7 @@ __global__ void __launch_bounds__(256) k_gemv_generic(const uint8_t *__restrict_
                                                       const int32_t *__restrict__ prot_idx,
                                                       int N, int K, int S, int p,
                                                       const uint16_t *__restrict__ x, int B,
-                                                      float *__restrict__ y) {
+                                                      float *__restrict__ y, int *err) {
     const int C = K / 8, p_pad = (p + 15) / 16 * 16;
     const int lane = threadIdx.x & 31;
     const int i = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
@@ -796,6 +804,10 @@ __global__ void __launch_bounds__(256) k_gemv_generic(const uint8_t *__restrict_
     // (kept in the same 1/sqrt(8) units as acc until the final scaling)
     for (int t = lane; t < p; t += 32) {
         const int j = prot_idx[t], c = j / 8, k = j % 8;
+        if (j < 0 || j >= K) {   // not a column of this layer
+            latch_error(err, BISCO_ERR_INVALID_ARG);
+            continue;
+        }
         float wb = 0.f;
         for (int s = 0; s < S; ++s) {
             const int64_t e = (static_cast<int64_t>(s) * N + i) * C + c;
@@ -1068,7 +1080,7 @@ bisco_status launch_gemv(const bisco_layer &L, const uint16_t *x, int B, float *
     auto generic = [&]() -> bisco_status {
         const int rows_per_block = 8;
         k_gemv_generic<<<(N + rows_per_block - 1) / rows_per_block, 32 * rows_per_block, 0, stream>>>(
-            L.codes, L.norms, L.q8, L.q8_scale, L.prot_idx, N, K, S, p, x, B, y);
+            L.codes, L.norms, L.q8, L.q8_scale, L.prot_idx, N, K, S, p, x, B, y, err);
         return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
     };
     if (K % 128 != 0) return generic();   // row pitch rules out TMA

@@ -35,7 +35,7 @@ def test_header_declarations_are_exported(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert bisco.bisco_abi_version() == 100
+    assert bisco.bisco_abi_version() == 101
     for code in range(6):
         assert bisco.status_string(code)
     assert bisco.status_string(99) == "unknown status"
@@ -108,4 +108,10 @@ def test_call_argument_validation(lib):
     assert lib.bisco_encode(x, ctypes.c_void_p(0x90002), ctypes.byref(L),
                             ctypes.c_void_p(0x80000), ws, None) == bisco.ERR_INVALID_ARG
     assert lib.bisco_encode_workspace_bytes(0, 64) == 0
-    assert lib.bisco_gemm_workspace_bytes(16, 64, 12) == 0
+    assert lib.bisco_gemm_workspace_bytes(ctypes.byref(_fake_layer(k_in=12)), 128) == 0
+    assert lib.bisco_gemm_workspace_bytes(ctypes.byref(L), -1) == 0
+    assert lib.bisco_gemm_workspace_bytes(ctypes.byref(L), 64) == 0        # decode-kernel path
+    # tensor-core path: fp16 activations plus hi/lo protected columns
+    L2 = _fake_layer(k_in=4096, n_protected=41)
+    assert lib.bisco_gemm_workspace_bytes(ctypes.byref(L2), 2048) == 2048 * (4096 + 128) * 2
+    assert lib.bisco_gemm(ctypes.byref(L2), x, 2048, y, None, 0, None) == bisco.ERR_INVALID_ARG

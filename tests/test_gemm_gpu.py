@@ -32,10 +32,14 @@ def run_gemm(env, Lref, X):
 
 
 @pytest.mark.parametrize("N,K,S,p,M", [
-    (1024, 1024, 2, 11, 2048),      # single layer 1024 x 1024, 2048 tokens
-    (1024, 1024, 2, 11, 37),        # ragged token count
-    (200, 1536, 3, 20, 130),        # ragged N, three stages
-    (64, 1000, 2, 10, 20),          # K % 128 != 0
+    (1024, 1024, 2, 11, 2048),      # single layer 1024 x 1024, 2048 tokens (tensor cores)
+    (1024, 1024, 2, 11, 37),        # small prefill: decode kernels
+    (200, 1536, 3, 20, 130),        # ragged N and M, three stages
+    (128, 512, 1, 0, 100),          # S = 1, no protected columns
+    (384, 2048, 2, 130, 300),       # three 64-column protected blocks, two token tiles
+    (96, 512, 2, 512, 80),          # every column protected
+    (256, 12288, 2, 123, 260),      # K = 12288 (down_proj width)
+    (64, 1000, 2, 10, 90),          # K % 128 != 0: decode kernels
     (128, 512, 1, 0, 1),            # one token
 ])
 def test_gemm_matches_oracle(env, N, K, S, p, M):
