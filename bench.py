@@ -45,6 +45,9 @@ def parse():
     ap.add_argument("--impl", choices=("bisco", "reference"), default="bisco")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--mode", choices=("both", "decode", "prefill"), default="both",
+                    help="decode: the GEMV step only; prefill: the tcgen05 GEMM only")
+    ap.add_argument("--prefill-tokens", type=int, default=2048)
     return ap.parse_args()
 
 
@@ -55,6 +58,17 @@ def peaks():
         return float(d["hbm_gbs"]), "measured"
     except Exception:
         return 6800.0, "fallback"
+
+
+def tensor_peaks():
+    """bf16 dense tensor peaks (TFLOP/s): burst and sustained; the fp16
+    kind::f16 MMA runs at the bf16 rate."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["bf16_tflops"]), float(d["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return 1900.0, 1700.0, "fallback"
 
 
 # DRAM bytes (read + write) of one q_proj/o_proj launch of the dominant
@@ -308,6 +322,67 @@ def run_bisco(args, rank, world, local_rank):
         clocks=clk, ms_e2e=ms_e2e / args.steps)
 
 
+# ---------------------------------------------------------------- prefill
+
+def run_prefill(args, local_rank):
+    """Prefill (bisco_gemm on the tensor cores): the four attention
+    projections of one layer at M tokens, a CUDA graph of the four calls
+    (fp16 pre-pass + tcgen05 kernel each), CUDA events over `steps` replays.
+    TFLOP/s on the algorithmic 2*M*N*K."""
+    import torch
+    from paper_2607_08643_gb300 import bisco, synth
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    M = args.prefill_tokens
+    layers = []
+    for j, name in enumerate(ATTN):
+        N, K = synth.QWEN3_8B_SHAPES[name]
+        W = synth.layer_weights_torch(N, K, seed=500 + j, device=dev)
+        layers.append((name, bisco.bisco_encode(W, S_STAGES, synth.protected_count(K, RHO_PCT))))
+        del W
+    X = torch.randn((M, 4096), device=dev).to(torch.bfloat16).view(torch.int16)
+    Ys = [torch.empty((M, L.N), device=dev) for _, L in layers]
+    ws = torch.empty(max(bisco.bisco_gemm_workspace_bytes(L, M) for _, L in layers),
+                     dtype=torch.uint8, device=dev)
+    torch.cuda.synchronize()
+    stream = torch.cuda.Stream(device=dev)
+    with torch.cuda.stream(stream):
+        for (_, L), Y in zip(layers, Ys):
+            bisco.bisco_gemm(L, X, Y=Y, workspace=ws, stream=stream)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for (_, L), Y in zip(layers, Ys):
+                bisco.bisco_gemm(L, X, Y=Y, workspace=ws, stream=stream)
+    torch.cuda.synchronize()
+    for _ in range(max(args.warmup, 3)):
+        g.replay()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(args.steps):
+            g.replay()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    if bisco.bisco_get_device_error(stream) != bisco.OK:
+        raise RuntimeError("device error in prefill")
+    ms = e0.elapsed_time(e1) / args.steps
+    flops = sum(2.0 * M * L.N * L.K for _, L in layers)
+    tf = flops / (ms * 1e-3) / 1e12
+    burst, sustained, kind = tensor_peaks()
+    return {"metric": "prefill GEMM TFLOP/s (2*M*N*K, decoded weight never written)",
+            "workload": "Qwen3-8B q/k/v/o projections, %d tokens, S=%d, %d%% protected"
+                        % (M, S_STAGES, RHO_PCT),
+            "value": tf, "unit": "TFLOP/s", "ms_per_step": ms, "tokens_per_s": M / (ms * 1e-3),
+            "roofline": {"bound": "tensor", "achieved": tf, "peak": burst, "unit": "TFLOP/s",
+                         "frac": tf / burst, "frac_of_sustained": tf / sustained,
+                         "peak_source": "%s bf16_tflops (MEASURED_PEAKS.json; fp16 rate = bf16)" % kind,
+                         "kernels": "k_gemm_prep + k_gemm per projection"},
+            "dtype": "f16 x f16 -> f32", "launches_per_step": 2 * len(layers)}
+
+
 # ------------------------------------------------------------ CPU oracle
 
 def cpu_oracle_sample(seconds, batch):
@@ -388,11 +463,21 @@ def main():
             import torch.distributed as dist
             dist.destroy_process_group()
         return
+    if args.mode == "prefill":
+        pf = run_prefill(args, local_rank)
+        if rank == 0:
+            print(json.dumps(dict(pf, n_gpus=world, steps=args.steps, warmup=args.warmup,
+                                  higher_is_better=True, data="synthetic")))
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return
     # CPU baseline first (before any CUDA work), rank 0 at N = 1 only
     cpu = None
     if world == 1 and rank == 0 and not args.no_cpu_baseline:
         cpu = cpu_oracle_sample(args.cpu_seconds, args.batch)
     r = run_bisco(args, rank, world, local_rank)
+    prefill = run_prefill(args, local_rank) if args.mode == "both" else None
     if rank == 0:
         line = {
             "metric": METRIC, "value": r["value"], "unit": "GB/s", "n_gpus": world,
@@ -410,6 +495,7 @@ def main():
             "clocks": r["clocks"],
             "cpu_baseline": cpu,
             "parallelism": "replicas" if world > 1 else "single GPU",
+            "prefill": prefill,
         }
         print(json.dumps(line))
     if world > 1:
