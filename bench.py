@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--mode", choices=("both", "decode", "prefill"), default="both",
                     help="decode: the GEMV step only; prefill: the tcgen05 GEMM only")
     ap.add_argument("--prefill-tokens", type=int, default=2048)
+    ap.add_argument("--ungrouped", action="store_true",
+                    help="one bisco_gemv per projection instead of bisco_gemv_multi for q/k/v")
     return ap.parse_args()
 
 
@@ -96,6 +98,8 @@ def workload_config(args):
         "chunk_dim": 8, "stages": S_STAGES, "protected_pct": RHO_PCT, "batch": args.batch,
         "weights": "N(0,0.02) + 8 outlier cols x20, seeded on device",
         "l2": "inputs larger than L2 (distinct coded layers per step, no flush)",
+        "launches": ("one bisco_gemv per projection" if args.ungrouped else
+                     "q/k/v in one bisco_gemv_multi launch per layer, o_proj in its own"),
     }
 
 
@@ -207,10 +211,18 @@ def run_bisco(args, rank, world, local_rank):
     stream = torch.cuda.Stream(device=dev)
 
     def step():
-        for i, (name, L) in enumerate(layers):
-            li = i // 4
-            xi = 2 * li + (1 if name == "o_proj" else 0)
-            bisco.bisco_gemv(L, x_dev[xi], y=views[i], stream=stream)
+        if args.ungrouped:
+            for i, (name, L) in enumerate(layers):
+                li = i // 4
+                xi = 2 * li + (1 if name == "o_proj" else 0)
+                bisco.bisco_gemv(L, x_dev[xi], y=views[i], stream=stream)
+            return
+        for li in range(args.layers):
+            # q/k/v read the same activation: one grouped launch; o_proj its own
+            qkv = [layers[4 * li + j][1] for j in range(3)]
+            bisco.bisco_gemv_multi(qkv, x_dev[2 * li], ys=views[4 * li:4 * li + 3], stream=stream)
+            bisco.bisco_gemv(layers[4 * li + 3][1], x_dev[2 * li + 1], y=views[4 * li + 3],
+                             stream=stream)
 
     # capture one step (144 launches through the public API) in a CUDA graph
     with torch.cuda.stream(stream):
@@ -277,17 +289,23 @@ def run_bisco(args, rank, world, local_rank):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms_total, ms_e2e = float(t[0]), float(t[1])
 
-    # dominant kernel (the 4096 x 4096 q/o projections, about 80 % of the
-    # step's bytes): the same launches on the same stream, timed alone
-    dom = [i for i, (name, _) in enumerate(layers) if name in ("q_proj", "o_proj")]
+    # dominant kernel: the grouped q/k/v launch (60 % of the step's bytes;
+    # the q/o projections when ungrouped), timed alone on the same stream
+    if args.ungrouped:
+        dom_calls = [[i] for i, (name, _) in enumerate(layers) if name in ("q_proj", "o_proj")]
+    else:
+        dom_calls = [[4 * li, 4 * li + 1, 4 * li + 2] for li in range(args.layers)]
     with torch.cuda.stream(stream):
         g_dom = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g_dom, stream=stream):
-            for i in dom:
-                name, L = layers[i]
-                li = i // 4
-                bisco.bisco_gemv(L, x_dev[2 * li + (1 if name == "o_proj" else 0)], y=views[i],
-                                 stream=stream)
+            for idx in dom_calls:
+                li = idx[0] // 4
+                xi = 2 * li + (1 if layers[idx[0]][0] == "o_proj" else 0)
+                if len(idx) == 1:
+                    bisco.bisco_gemv(layers[idx[0]][1], x_dev[xi], y=views[idx[0]], stream=stream)
+                else:
+                    bisco.bisco_gemv_multi([layers[i][1] for i in idx], x_dev[xi],
+                                           ys=[views[i] for i in idx], stream=stream)
     for _ in range(3):
         g_dom.replay()
     barrier()
@@ -299,14 +317,14 @@ def run_bisco(args, rank, world, local_rank):
             g_dom.replay()
         d1.record(stream)
     barrier()
-    us_dom = d0.elapsed_time(d1) * 1e3 / (args.steps * len(dom))
-    bytes_dom = layers[dom[0]][1].compressed_bytes
+    us_dom = d0.elapsed_time(d1) * 1e3 / (args.steps * len(dom_calls))
+    bytes_dom = sum(layers[i][1].compressed_bytes for i in dom_calls[0])
 
     ms_step = ms_total / args.steps
     gbs = world * bytes_step / (ms_step * 1e-3) / 1e9
     tok_s = world * B / (ms_step * 1e-3)
     e2e_gbs = world * bytes_step / (ms_e2e / args.steps * 1e-3) / 1e9
-    launches = len(layers)
+    launches = len(layers) if args.ungrouped else 2 * args.layers
     peak, peak_kind = peaks()
     achieved = bytes_dom / (us_dom * 1e-6) / 1e9
     return dict(
@@ -316,9 +334,11 @@ def run_bisco(args, rank, world, local_rank):
                   "frac": achieved / peak, "traffic": dominant_traffic(),
                   "peak_source": "%s hbm_gbs (MEASURED_PEAKS.json, copy burst)" % peak_kind
                   if peak_kind == "measured" else "fallback 6.8 TB/s",
-                  "kernel": "k_gemv_stream<4,2,2> (bisco_gemv, q_proj/o_proj 4096x4096, batch %d)" % B,
+                  "kernel": ("k_gemv_stream<4,2,2> (bisco_gemv, q_proj/o_proj 4096x4096, batch %d)"
+                             if args.ungrouped else
+                             "k_gemv_stream<4,2,2> (bisco_gemv_multi, q+k+v 6144x4096, batch %d)") % B,
                   "bytes_per_launch": bytes_dom, "us_per_launch": us_dom,
-                  "launches_timed": args.steps * len(dom)},
+                  "launches_timed": args.steps * len(dom_calls)},
         clocks=clk, ms_e2e=ms_e2e / args.steps)
 
 
@@ -488,7 +508,8 @@ def main():
             "e2e": {"value": r["e2e_gbs"], "unit": "GB/s",
                     "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"],
                     "how": "pinned H2D of the step's activations + CUDA graph of the step's "
-                           "bisco_gemv calls + D2H of all outputs, per step",
+                           "bisco_gemv_multi (q/k/v) and bisco_gemv (o) calls + D2H of all "
+                           "outputs, per step",
                     "ms_per_step": r["ms_e2e"]},
             "gpu_launches": r["launches"] * args.steps,
             "roofline": r["roofline"],

@@ -82,7 +82,7 @@ typedef struct {
 } bisco_layer;
 
 /* ABI version of this header (major * 100 + minor). */
-#define BISCO_ABI_VERSION 101
+#define BISCO_ABI_VERSION 102
 int32_t bisco_abi_version(void);
 
 /* Static string for a status code (never NULL). */
@@ -159,6 +159,23 @@ bisco_status bisco_encode_noalloc(const uint16_t *W_bf16, const float *g, const 
  */
 bisco_status bisco_gemv(const bisco_layer *L, const uint16_t *x_bf16, int32_t B, float *y,
                         bisco_stream_t stream);
+
+/*
+ * bisco_gemv for G layers that read the same activations, for example the
+ * q, k and v projections of one attention layer (Sec. III-F Eq. 12 for each):
+ *     y[g][b][i] = sum_j What_g[i][j] * x[b][j]      for g < G
+ * in one launch, so the fixed per-launch latency (dependency release,
+ * activation staging, reduction tail) is paid once for the group.
+ * layers: host array of G structs; all must have the same k_in and stages
+ * (n_out and n_protected may differ).  G in [1, BISCO_GEMV_MULTI_MAX].
+ * y: host array of G device pointers, y[g] is [B][n_out of layer g] float32,
+ * 16-byte aligned, fully overwritten.  x_bf16, B and the launch contract
+ * are those of bisco_gemv.  Combinations the grouped kernel does not take
+ * (B > 8, K % 128 != 0, shared memory) run as G bisco_gemv launches.
+ */
+#define BISCO_GEMV_MULTI_MAX 4
+bisco_status bisco_gemv_multi(const bisco_layer *layers, int32_t G, const uint16_t *x_bf16,
+                              int32_t B, float *const *y, bisco_stream_t stream);
 
 /*
  * Prefill matrix product Y[m][i] = sum_j What[i][j] * X[m][j] for any M >= 0

@@ -17,6 +17,7 @@ OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_RANGE, ERR_CUDA, ERR_TIMEOUT = range(6
 EXPORTS = (
     "bisco_abi_version", "bisco_status_string", "bisco_encoded_sizes",
     "bisco_encode_workspace_bytes", "bisco_encode", "bisco_encode_noalloc", "bisco_gemv",
+    "bisco_gemv_multi",
     "bisco_gemm_workspace_bytes", "bisco_gemm", "bisco_get_device_error",
 )
 
@@ -65,6 +66,8 @@ def load(path: str = LIB_PATH):
     lib.bisco_encode_noalloc.argtypes = [P, P, Lp, P]
     lib.bisco_gemv.restype = st
     lib.bisco_gemv.argtypes = [Lp, P, i32, P, P]
+    lib.bisco_gemv_multi.restype = st
+    lib.bisco_gemv_multi.argtypes = [Lp, i32, P, i32, ctypes.POINTER(P), P]
     lib.bisco_gemm_workspace_bytes.restype = sz
     lib.bisco_gemm_workspace_bytes.argtypes = [Lp, i32]
     lib.bisco_gemm.restype = st
@@ -212,6 +215,25 @@ def bisco_gemv(L: Layer, x_bits, y=None, stream=None):
     _check(load().bisco_gemv(ctypes.byref(L.c), _ptr(x_bits), B, _ptr(y), _stream(stream)),
            "bisco_gemv")
     return y
+
+
+def bisco_gemv_multi(layers, x_bits, ys=None, stream=None):
+    """[y_g] = x What_g^T for layers sharing K and S, one launch (q/k/v)."""
+    import torch
+    if x_bits.dtype == torch.bfloat16:
+        x_bits = x_bits.view(torch.int16)
+    if x_bits.dim() == 1:
+        x_bits = x_bits.unsqueeze(0)
+    B = x_bits.shape[0]
+    G = len(layers)
+    assert x_bits.is_contiguous() and all(L.K == x_bits.shape[1] for L in layers)
+    if ys is None:
+        ys = [torch.empty((B, L.N), dtype=torch.float32, device=x_bits.device) for L in layers]
+    structs = (bisco_layer * G)(*[L.c for L in layers])
+    yp = (ctypes.c_void_p * G)(*[y.data_ptr() for y in ys])
+    _check(load().bisco_gemv_multi(structs, G, _ptr(x_bits), B, yp, _stream(stream)),
+           "bisco_gemv_multi")
+    return ys
 
 
 def bisco_gemm(L: Layer, X_bits, Y=None, workspace=None, stream=None):

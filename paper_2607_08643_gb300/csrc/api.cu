@@ -178,6 +178,26 @@ bisco_status bisco_gemv(const bisco_layer *L, const uint16_t *x_bf16, int32_t B,
     return launch_gemv(*L, x_bf16, B, y, err, reinterpret_cast<cudaStream_t>(stream));
 }
 
+bisco_status bisco_gemv_multi(const bisco_layer *layers, int32_t G, const uint16_t *x_bf16,
+                              int32_t B, float *const *y, bisco_stream_t stream) {
+    if (!layers || !y || G < 1 || G > BISCO_GEMV_MULTI_MAX) return BISCO_ERR_INVALID_ARG;
+    for (int g = 0; g < G; ++g) {
+        const bisco_status st = check_layer(&layers[g], true);
+        if (st != BISCO_OK) return st;
+        if (layers[g].k_in != layers[0].k_in || layers[g].stages != layers[0].stages)
+            return BISCO_ERR_INVALID_ARG;
+    }
+    if (B < 0 || B > 16) return BISCO_ERR_INVALID_ARG;
+    if (B == 0) return BISCO_OK;
+    if (!x_bf16 || !aligned16(x_bf16)) return BISCO_ERR_INVALID_ARG;
+    for (int g = 0; g < G; ++g)
+        if (!y[g] || !aligned16(y[g])) return BISCO_ERR_INVALID_ARG;
+    bisco_status st;
+    int *err = device_error_word(&st);
+    if (!err) return st;
+    return launch_gemv_multi(layers, G, x_bf16, B, y, err, reinterpret_cast<cudaStream_t>(stream));
+}
+
 size_t bisco_gemm_workspace_bytes(const bisco_layer *L, int32_t M) {
     if (M < 0 || check_layer(L, false) != BISCO_OK) return 0;
     return gemm_workspace_bytes(*L, M);

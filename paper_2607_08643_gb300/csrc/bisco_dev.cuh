@@ -137,6 +137,14 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_
         ::"r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
 }
 
+// Warms L2 with [src, src + bytes) (16-byte aligned, bytes % 16 == 0).  A
+// prefetch moves no data into the CTA, so it is safe ahead of the wait on an
+// earlier kernel that may still write the range: L2 is the point of
+// coherence and the later real load sees the final values.
+__device__ __forceinline__ void prefetch_l2(const void *src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap *map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");
 }

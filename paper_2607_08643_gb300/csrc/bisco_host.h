@@ -26,6 +26,8 @@ bisco_status launch_encode(const uint16_t *W, const float *g, const bisco_layer 
                            void *workspace, int *err, cudaStream_t stream);
 bisco_status launch_gemv(const bisco_layer &L, const uint16_t *x, int B, float *y, int *err,
                          cudaStream_t stream);
+bisco_status launch_gemv_multi(const bisco_layer *Ls, int G, const uint16_t *x, int B,
+                               float *const *y, int *err, cudaStream_t stream);
 size_t gemm_workspace_bytes(const bisco_layer &L, int M);
 bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *Y,
                          void *workspace, size_t ws_bytes, int *err, cudaStream_t stream);

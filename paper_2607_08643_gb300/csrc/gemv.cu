@@ -84,65 +84,90 @@ __device__ __forceinline__ unsigned char *aligned_smem(unsigned char *raw) {
     return raw + ((1024u - (smem_u32(raw) & 1023u)) & 1023u);
 }
 
-// Activation staging for the input columns [k_begin, k_begin + cols):
-// bf16 rows from global memory -> fp16 in the permuted fragment order
-// [512-column slab][w][m][t][4 pairs], protected columns zeroed, and
-// scale_u * x[b][j_u] of the protected columns (exact in fp32: 11 x 8
-// significant bits) taken from the same loads, so the activations cost one
-// round trip to memory.  Job = one 32-column group of one row (4 x 16 B in,
-// 4 x 16 B out).  Pair i of a 32-column group is element i&7 of chunk
-// (i>>3) and of chunk (i>>3)+2 -- bits i and i+16 of its code word.
-__device__ __forceinline__ void stage_activations(unsigned char *sm, const GemvArgs &a,
-                                                  int k_begin, int cols, int nnar,
-                                                  const uint32_t *s_pmask, const int *s_pu,
-                                                  const float *s_pscale, float *s_xs) {
+constexpr int kMaxGroup = 4;   // layers sharing one activation in a grouped launch
+
+// Per-layer shared-memory view used by the activation staging.
+struct StageView {
+    unsigned char *xt;        // [B][xt_pitch] staged fp16 operand
+    const uint32_t *pmask;    // protected-column bits per 32-column group
+    const int *pu;            // protected columns before each group
+    const float *pscale;      // scale of each protected column
+    float *xs;                // [B][cap] scale * x of each protected column
+};
+
+// Activation staging for the input columns [k_begin, k_begin + cols) of G
+// layers that share x: bf16 rows from global memory -> fp16 in the permuted
+// fragment order [512-column slab][w][m][t][4 pairs], converted once, then
+// stored per layer with that layer's protected columns zeroed; scale_u *
+// x[b][j_u] of the protected columns (exact in fp32: 11 x 8 significant
+// bits) is taken from the same cache lines, so the activations cost one
+// round trip to memory.  Job = one 32-column group of one row.  Pair i of a
+// 32-column group is element i&7 of chunk (i>>3) and of chunk (i>>3)+2 --
+// bits i and i+16 of its code word, columns (i>>3)*8 + (i&7) and that + 16.
+template <int MAXG>
+__device__ __forceinline__ void stage_activations(const uint16_t *x, int K, int B, int k_begin,
+                                                  int cols, int nnar, int xt_pitch, int cap,
+                                                  int G, const StageView (&v)[MAXG]) {
     const int groups_per_row = cols >> 5;   // cols % 128 == 0 on this path
-    const int njobs = a.B * nnar * 16;
+    const int njobs = B * nnar * 16;
     for (int e = threadIdx.x; e < njobs; e += blockDim.x) {
         const int t = e & 3, w = (e >> 2) & 3, sb = e >> 4;
         const int b = sb / nnar, slab = sb - b * nnar;
         const int g32 = slab * 16 + t * 4 + w;
-        unsigned char *dst = sm + a.off_xt + b * a.xt_pitch + slab * 1024 + t * 16;
-        if (g32 >= groups_per_row) {
-#pragma unroll
-            for (int m = 0; m < 4; ++m)
-                *reinterpret_cast<uint4 *>(dst + (w * 4 + m) * 64) = make_uint4(0, 0, 0, 0);
-            continue;
-        }
-        const uint4 *src = reinterpret_cast<const uint4 *>(
-            a.x + static_cast<int64_t>(b) * a.K + k_begin + g32 * 32);
-        uint32_t r[16];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const uint4 v = src[q];
-            r[4 * q] = v.x; r[4 * q + 1] = v.y; r[4 * q + 2] = v.z; r[4 * q + 3] = v.w;
-        }
-        const uint32_t pm = s_pmask[g32];
-        if (pm) {
-            const int u0 = s_pu[g32];   // protected columns before this group
-#pragma unroll
-            for (int k = 0; k < 32; ++k) {
-                if ((pm >> k) & 1u) {
-                    const int u = u0 + __popc(pm & ((1u << k) - 1u));
-                    const float xv = (k & 1) ? bf16_hi(r[k >> 1]) : bf16_lo(r[k >> 1]);
-                    s_xs[b * a.pidx_cap + u] = s_pscale[u] * xv;
-                    r[k >> 1] &= (k & 1) ? 0x0000FFFFu : 0xFFFF0000u;
-                }
-            }
-        }
-#pragma unroll
-        for (int m = 0; m < 4; ++m) {
-            // pairs 4m..4m+3: element 4(m&1)+q of chunk m>>1 and of chunk (m>>1)+2
-            const int wf = 4 * (m >> 1) + 2 * (m & 1);
-            uint32_t o[4];
+        const int dst_off = b * xt_pitch + slab * 1024 + t * 16 + w * 256;
+        uint32_t o[16];
+        const uint16_t *src = x + static_cast<int64_t>(b) * K + k_begin + g32 * 32;
+        if (g32 < groups_per_row) {
+            uint32_t r[16];
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
-                const uint32_t f = r[wf + (q >> 1)], sw = r[8 + wf + (q >> 1)];
-                const __half2 h = __floats2half2_rn((q & 1) ? bf16_hi(f) : bf16_lo(f),
-                                                    (q & 1) ? bf16_hi(sw) : bf16_lo(sw));
-                o[q] = *reinterpret_cast<const uint32_t *>(&h);
+                const uint4 u4 = reinterpret_cast<const uint4 *>(src)[q];
+                r[4 * q] = u4.x; r[4 * q + 1] = u4.y; r[4 * q + 2] = u4.z; r[4 * q + 3] = u4.w;
             }
-            *reinterpret_cast<uint4 *>(dst + (w * 4 + m) * 64) = make_uint4(o[0], o[1], o[2], o[3]);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                // pair i: columns c0 = (i>>3)*8 + (i&7) (low half) and c0 + 16
+                const int c0 = (i >> 3) * 8 + (i & 7);
+                const uint32_t f = r[c0 >> 1], sw = r[(c0 + 16) >> 1];
+                const __half2 h = __floats2half2_rn((c0 & 1) ? bf16_hi(f) : bf16_lo(f),
+                                                    (c0 & 1) ? bf16_hi(sw) : bf16_lo(sw));
+                o[i] = *reinterpret_cast<const uint32_t *>(&h);
+            }
+        } else {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) o[i] = 0u;
+        }
+#pragma unroll
+        for (int g = 0; g < MAXG; ++g) {
+            if (g >= G) break;
+            uint32_t pm = g32 < groups_per_row ? v[g].pmask[g32] : 0u;
+            unsigned char *dst = v[g].xt + dst_off;
+            if (pm == 0u) {
+#pragma unroll
+                for (int m = 0; m < 4; ++m)
+                    *reinterpret_cast<uint4 *>(dst + m * 64) =
+                        make_uint4(o[4 * m], o[4 * m + 1], o[4 * m + 2], o[4 * m + 3]);
+                continue;
+            }
+            // protected columns of this group: record scale * x, zero the halves
+            const int u0 = v[g].pu[g32];   // protected columns before this group
+            for (uint32_t bits = pm; bits; bits &= bits - 1u) {
+                const int k = __ffs(bits) - 1;
+                const int u = u0 + __popc(pm & ((1u << k) - 1u));
+                v[g].xs[b * cap + u] = v[g].pscale[u] * bf16_bits_to_f32(src[k]);
+            }
+            uint32_t om[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                const int c0 = (i >> 3) * 8 + (i & 7);
+                const uint32_t keep = (((pm >> c0) & 1u) ? 0u : 0x0000FFFFu) |
+                                      (((pm >> (c0 + 16)) & 1u) ? 0u : 0xFFFF0000u);
+                om[i] = o[i] & keep;
+            }
+#pragma unroll
+            for (int m = 0; m < 4; ++m)
+                *reinterpret_cast<uint4 *>(dst + m * 64) =
+                    make_uint4(om[4 * m], om[4 * m + 1], om[4 * m + 2], om[4 * m + 3]);
         }
     }
 }
@@ -248,12 +273,24 @@ __device__ __forceinline__ void stage_protected_meta(const GemvArgs &a, int k_be
                                                      uint32_t *s_pmask, int *s_pu, int *s_lohi) {
     const int lane = threadIdx.x & 31;
     for (int i = lane; i < mwords; i += 32) s_pmask[i] = 0u;
-    int lo = 0, hi = 0;
-    for (int t0 = 0; t0 < a.p; t0 += 32) {
-        const int t = t0 + lane;
-        const int v = t < a.p ? a.prot_idx[t] : 0x7FFFFFFF;
-        lo += __popc(__ballot_sync(0xFFFFFFFFu, v < k_begin));
-        hi += __popc(__ballot_sync(0xFFFFFFFFu, v < k_end));
+    int lo = 0, hi = a.p;
+    if (k_begin > 0 || k_end < a.K) {
+        // position of [k_begin, k_end) in the ascending list; four loads in
+        // flight per lane
+        hi = 0;
+        for (int t0 = 0; t0 < a.p; t0 += 128) {
+            int v[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int t = t0 + 32 * i + lane;
+                v[i] = t < a.p ? a.prot_idx[t] : 0x7FFFFFFF;
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                lo += __popc(__ballot_sync(0xFFFFFFFFu, v[i] < k_begin));
+                hi += __popc(__ballot_sync(0xFFFFFFFFu, v[i] < k_end));
+            }
+        }
     }
     __syncwarp();
     // an ascending index list puts at most pidx_cap entries in [k_begin,
@@ -262,6 +299,7 @@ __device__ __forceinline__ void stage_protected_meta(const GemvArgs &a, int k_be
         if (lane == 0) latch_error(a.err, BISCO_ERR_INVALID_ARG);
         hi = lo + a.pidx_cap;
     }
+#pragma unroll 4
     for (int u = lane; u < hi - lo; u += 32) {
         const int j = a.prot_idx[lo + u];
         const bool in_range = j >= k_begin && j < k_end;
@@ -355,6 +393,11 @@ k_gemv(const __grid_constant__ CUtensorMap tm_codes, const __grid_constant__ CUt
     if (warp == 0)
         stage_protected_meta(a, k_begin, k_end, nnar * (kSlab / 32), s_pidx, s_pscale, s_pmask,
                              s_pu, s_lohi);
+    if (producer && k_end > k_begin) {
+        for (int b = 0; b < a.B; ++b)
+            prefetch_l2(a.x + static_cast<int64_t>(b) * a.K + k_begin,
+                        static_cast<uint32_t>(k_end - k_begin) * 2);
+    }
     __syncthreads();
     // the next kernel in the stream may start streaming its own weights now
     pdl_launch_dependents();
@@ -373,7 +416,11 @@ k_gemv(const __grid_constant__ CUtensorMap tm_codes, const __grid_constant__ CUt
 
     // activations may be written by the previous kernel
     pdl_wait();
-    stage_activations(sm, a, k_begin, k_end - k_begin, nnar, s_pmask, s_pu, s_pscale, s_xs);
+    {
+        StageView v[1] = {{sm + a.off_xt, s_pmask, s_pu, s_pscale, s_xs}};
+        stage_activations<1>(a.x, a.K, a.B, k_begin, k_end - k_begin, nnar, a.xt_pitch, a.pidx_cap,
+                             1, v);
+    }
     for (int i = threadIdx.x; i < 1024 / 16; i += blockDim.x)
         reinterpret_cast<uint4 *>(sm + a.off_zero)[i] = make_uint4(0, 0, 0, 0);
     __syncthreads();
@@ -517,42 +564,84 @@ k_gemv(const __grid_constant__ CUtensorMap tm_codes, const __grid_constant__ CUt
 }
 
 // ------------------------------------------------------------------------
-// Streaming kernel: persistent CTA, 16-row tiles x all K, batch <= 8.
+// Streaming kernel: persistent CTA over 16-row tiles x all K of G <= 4 layers
+// that share the activations (G = 1 for a plain bisco_gemv), batch <= 8.
 // Warp (q, k) decodes column quarter q of every slot whose global index is
 // k modulo WK; warp NCW produces; warp NCW+1 reduces.  A slot's full
 // barrier is split into WK barriers taken in turn by its fills, so that a
 // consumer group always waits on a barrier whose previous phase it observed
 // itself, whatever the ring depth.
-template <int WQ, int WK, int S>
+
+struct StreamLayer {
+    float *y;
+    const uint16_t *q8_scale;
+    const int32_t *prot_idx;
+    int N, p;
+    int tile0;       // first tile of this layer in the launch's tile list
+    int q8_boxes;    // 128-column boxes of the int8 slab of one tile
+};
+
+template <int MAXG>
+struct StreamArgs {
+    CUtensorMap mc[MAXG], mn[MAXG], mq[MAXG];
+    StreamLayer L[MAXG];
+    const uint16_t *x;
+    int *err;
+    int K, B, G, ntiles, nslot;
+    int q8_boxes;    // the largest of the layers' (int8 double buffer size)
+    int pidx_cap, xt_pitch, mwords;
+    uint32_t off_xt, off_q8, off_red, off_bar, off_pidx, off_pmask, off_zero, off_prot;
+};
+
+template <int WQ, int WK, int S, int MAXG>
 __global__ void __launch_bounds__((WQ * WK + 2) * 32, 2)
-k_gemv_stream(const __grid_constant__ CUtensorMap tm_codes,
-              const __grid_constant__ CUtensorMap tm_norms,
-              const __grid_constant__ CUtensorMap tm_q8, const GemvArgs a) {
+k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
     constexpr int BM = 16;
     constexpr int BP = 8;
     constexpr int NCW = WQ * WK;
     constexpr int SW = kSlab * WQ;
     constexpr int kCodeRow = SW / 8;
     constexpr int kNormRow = SW / 4;
-    constexpr bool kSwz = (WQ == 1);
     constexpr uint32_t kCodesBytes = S * BM * kCodeRow;
     constexpr uint32_t kSlotBytes = S * BM * (kCodeRow + kNormRow);
 
     extern __shared__ unsigned char smem_raw[];
     unsigned char *sm = aligned_smem(smem_raw);
     const uint32_t sbase = smem_u32(sm);
-    __shared__ int s_abort, s_lohi[2];
+    __shared__ int s_abort, s_lohi[MAXG][2];
+    // layer descriptors, read with a run-time layer index: from shared memory
+    // (a run-time index into the parameter block is a slow generic load)
+    __shared__ StreamLayer s_L[MAXG];
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int G = static_cast<int>(gridDim.x), cta = static_cast<int>(blockIdx.x);
-    const int ntiles = (a.N + BM - 1) / BM;
-    const int my_tiles = ntiles > cta ? (ntiles - 1 - cta) / G + 1 : 0;
-    const int nwide = (a.K + SW - 1) / SW;
-    const int nnar = (a.K + kSlab - 1) / kSlab;
+    const int Gd = static_cast<int>(gridDim.x), cta = static_cast<int>(blockIdx.x);
+    if (threadIdx.x < MAXG) {
+#pragma unroll
+        for (int i = 0; i < MAXG; ++i)
+            if (static_cast<int>(threadIdx.x) == i) s_L[i] = a.L[i];
+    }
+    __syncthreads();
+    // every scalar the loops use, read once: the tensor maps are addressed
+    // with a run-time layer index, after which parameter reads inside loops
+    // are not hoisted
+    const int K = a.K, B = a.B, G = a.G, xt_pitch = a.xt_pitch, mwords = a.mwords;
+    const uint32_t off_xt = a.off_xt, off_q8 = a.off_q8, off_zero = a.off_zero;
+    const uint32_t off_pidx = a.off_pidx, off_pmask = a.off_pmask, off_prot = a.off_prot;
+    const uint16_t *const x = a.x;
+    int *const err = a.err;
+    int tile0[MAXG];
+#pragma unroll
+    for (int i = 0; i < MAXG; ++i) tile0[i] = a.L[i].tile0;
+    const CUtensorMap *const maps_c = &a.mc[0];
+    const CUtensorMap *const maps_n = &a.mn[0];
+    const CUtensorMap *const maps_q = &a.mq[0];
+    const int my_tiles = a.ntiles > cta ? (a.ntiles - 1 - cta) / Gd + 1 : 0;
+    const int nwide = (K + SW - 1) / SW;
+    const int nnar = (K + kSlab - 1) / kSlab;
     const int total = my_tiles * nwide;   // ring fills of this CTA
     const int nslot = a.nslot;
-    const int q8_boxes = a.p > 0 ? ((a.p + 15) / 16 * 16 + 127) / 128 : 0;
-    const uint32_t q8_buf_bytes = static_cast<uint32_t>(q8_boxes * BM * 128);
+    const int cap = a.pidx_cap;
+    const uint32_t q8_buf_bytes = static_cast<uint32_t>(a.q8_boxes * BM * 128);
     const uint32_t bar_full = sbase + a.off_bar;            // [nslot][WK]
     const uint32_t bar_empty = bar_full + 8 * nslot * WK;   // [nslot]
     const uint32_t bar_q8f = bar_empty + 8 * nslot;         // [2] int8 slab landed
@@ -561,33 +650,64 @@ k_gemv_stream(const __grid_constant__ CUtensorMap tm_codes,
     const uint32_t bar_re = bar_rf + 16;                    // [2] tile partials read
     const bool producer = (warp == NCW) && (lane == 0);
     const uint64_t pol = l2_evict_first_policy();
-    int *s_pidx = reinterpret_cast<int *>(sm + a.off_pidx);
-    float *s_pscale = reinterpret_cast<float *>(s_pidx + a.pidx_cap);
-    float *s_xs = s_pscale + a.pidx_cap;
-    uint32_t *s_pmask = reinterpret_cast<uint32_t *>(sm + a.off_pmask);
-    int *s_pu = reinterpret_cast<int *>(sm + a.off_pu);
-    float *red = reinterpret_cast<float *>(sm + a.off_red);   // [2][NCW][BM][BP]
+    float *red = reinterpret_cast<float *>(sm + a.off_red);   // [2][NCW][BM][B]
 
-    auto tile_row0 = [&](int ii) { return (cta + ii * G) * BM; };
+    // per-layer shared-memory views
+    auto pidx_of = [&](int g) {
+        return reinterpret_cast<int *>(sm + off_pidx) + g * (2 + B) * cap;
+    };
+    auto pscale_of = [&](int g) { return reinterpret_cast<float *>(pidx_of(g) + cap); };
+    auto xs_of = [&](int g) { return pscale_of(g) + cap; };
+    auto pmask_of = [&](int g) {
+        return reinterpret_cast<uint32_t *>(sm + off_pmask) + g * 2 * mwords;
+    };
+    auto pu_of = [&](int g) { return reinterpret_cast<int *>(pmask_of(g) + mwords); };
+    auto xt_of = [&](int g) { return sm + off_xt + g * B * xt_pitch; };
+    // tile ii of this CTA -> (layer, first row)
+    auto layer_of = [&](int ii) {
+        const int T = cta + ii * Gd;
+        int g = 0;
+#pragma unroll
+        for (int i = 1; i < MAXG; ++i)
+            if (i < G && T >= tile0[i]) g = i;
+        return g;
+    };
+    auto row0_of = [&](int ii, int g) { return (cta + ii * Gd - s_L[g].tile0) * BM; };
     auto full_bar = [&](int gidx) {
         const int ph = gidx / nslot;
         return bar_full + 8 * ((gidx % nslot) * WK + ph % WK);
     };
     auto full_parity = [&](int gidx) { return static_cast<uint32_t>((gidx / nslot) / WK) & 1u; };
+    // the producer walks its tiles in order: layer and first row of the
+    // current tile are kept in registers
+    int cur_ii = -1, cur_g = 0, cur_row0 = 0;
     auto issue_slot = [&](int gidx) {
         const int ii = gidx / nwide, w = gidx - ii * nwide;
+        if (ii != cur_ii) {
+            cur_ii = ii;
+            cur_g = layer_of(ii);
+            cur_row0 = row0_of(ii, cur_g);
+        }
         const uint32_t dst = sbase + (gidx % nslot) * kSlotBytes;
         const uint32_t bar = full_bar(gidx);
+        const CUtensorMap *mc = maps_c + cur_g, *mn = maps_n + cur_g;
         mbar_arrive_expect_tx(bar, kSlotBytes);
-        tma_load_3d_hint(dst, &tm_codes, bar, w * (SW / 8), tile_row0(ii), 0, pol);
-        tma_load_3d_hint(dst + kCodesBytes, &tm_norms, bar, w * (SW / 8), tile_row0(ii), 0, pol);
+        tma_load_3d_hint(dst, mc, bar, w * (SW / 8), cur_row0, 0, pol);
+        tma_load_3d_hint(dst + kCodesBytes, mn, bar, w * (SW / 8), cur_row0, 0, pol);
     };
+    // the int8 slab of tile ii (a plain arrive when its layer has none)
     auto issue_q8 = [&](int ii) {
-        const uint32_t dst = sbase + a.off_q8 + (ii & 1) * q8_buf_bytes;
-        mbar_arrive_expect_tx(bar_q8f + 8 * (ii & 1), q8_buf_bytes);
-        for (int q = 0; q < q8_boxes; ++q)
-            tma_load_2d_hint(dst + q * BM * 128, &tm_q8, bar_q8f + 8 * (ii & 1), 128 * q,
-                             tile_row0(ii), pol);
+        const int g = layer_of(ii);
+        const uint32_t bar = bar_q8f + 8 * (ii & 1);
+        const int boxes = s_L[g].q8_boxes;
+        if (boxes == 0) {
+            mbar_arrive(bar);
+            return;
+        }
+        const uint32_t dst = sbase + off_q8 + (ii & 1) * q8_buf_bytes;
+        mbar_arrive_expect_tx(bar, static_cast<uint32_t>(boxes * BM * 128));
+        for (int q = 0; q < boxes; ++q)
+            tma_load_2d_hint(dst + q * BM * 128, maps_q + g, bar, 128 * q, row0_of(ii, g), pol);
     };
 
     int issued = 0, q8_issued = 0;
@@ -604,24 +724,45 @@ k_gemv_stream(const __grid_constant__ CUtensorMap tm_codes,
         }
         fence_mbar_init();
         s_abort = 0;
-        prefetch_tmap(&tm_codes);
-        prefetch_tmap(&tm_norms);
+        for (int g = 0; g < G; ++g) {
+            prefetch_tmap(maps_c + g);
+            prefetch_tmap(maps_n + g);
+        }
         for (; issued < total && issued < nslot; ++issued) {
             // a tile's int8 slab goes out with its first slot (two buffers)
-            if (q8_boxes > 0 && issued % nwide == 0 && issued / nwide < 2) issue_q8(q8_issued++);
+            if (issued % nwide == 0 && issued / nwide < 2) issue_q8(q8_issued++);
             issue_slot(issued);
         }
+        // activations: into L2 now, into the CTA after the wait
+        for (int b = 0; b < B; ++b)
+            prefetch_l2(x + static_cast<int64_t>(b) * K, static_cast<uint32_t>(K) * 2);
     }
-    if (warp == 0)
-        stage_protected_meta(a, 0, a.K, nnar * (kSlab / 32), s_pidx, s_pscale, s_pmask, s_pu,
-                             s_lohi);
+    if (warp < G) {
+        // one warp per layer: its protected columns, scales and masks
+        GemvArgs la = {};
+        la.q8_scale = s_L[warp].q8_scale;
+        la.prot_idx = s_L[warp].prot_idx;
+        la.err = err;
+        la.K = K;
+        la.p = s_L[warp].p;
+        la.pidx_cap = cap;
+        stage_protected_meta(la, 0, K, nnar * (kSlab / 32), pidx_of(warp), pscale_of(warp),
+                             pmask_of(warp), pu_of(warp), s_lohi[warp]);
+    }
     __syncthreads();
     pdl_launch_dependents();
 
+    // activations may be written by the previous kernel
     pdl_wait();
-    stage_activations(sm, a, 0, a.K, nnar, s_pmask, s_pu, s_pscale, s_xs);
+    {
+        StageView v[MAXG] = {};
+#pragma unroll
+        for (int g = 0; g < MAXG; ++g)
+            if (g < G) v[g] = {xt_of(g), pmask_of(g), pu_of(g), pscale_of(g), xs_of(g)};
+        stage_activations<MAXG>(x, K, B, 0, K, nnar, xt_pitch, cap, G, v);
+    }
     for (int i = threadIdx.x; i < 1024 / 16; i += blockDim.x)
-        reinterpret_cast<uint4 *>(sm + a.off_zero)[i] = make_uint4(0, 0, 0, 0);
+        reinterpret_cast<uint4 *>(sm + off_zero)[i] = make_uint4(0, 0, 0, 0);
     __syncthreads();
 
     if (warp == NCW) {
@@ -631,7 +772,7 @@ k_gemv_stream(const __grid_constant__ CUtensorMap tm_codes,
             // tile's first slot, once tile ii-2 released the buffer; every slot
             // of tile ii-1 is issued by then, so this never starves the decode.
             auto issue_q8_upto = [&](int ii) -> bool {
-                while (q8_boxes > 0 && q8_issued <= ii && q8_issued < my_tiles) {
+                while (q8_issued <= ii && q8_issued < my_tiles) {
                     if (q8_issued >= 2 &&
                         !mbar_wait(bar_q8e + 8 * (q8_issued & 1), ((q8_issued >> 1) - 1) & 1))
                         return false;
@@ -657,54 +798,57 @@ k_gemv_stream(const __grid_constant__ CUtensorMap tm_codes,
             if (ok && !*reinterpret_cast<volatile int *>(&s_abort) && !issue_q8_upto(my_tiles - 1))
                 ok = false;
             if (!ok) {
-                latch_error(a.err, BISCO_ERR_TIMEOUT);
+                latch_error(err, BISCO_ERR_TIMEOUT);
                 atomicExch(&s_abort, 1);
             }
-            if (*reinterpret_cast<volatile int *>(&s_abort)) {
-                // let every copy already in flight land before the CTA exits
-                for (int gi = (issued > nslot ? issued - nslot : 0); gi < issued; ++gi)
-                    mbar_wait(full_bar(gi), full_parity(gi));
-                for (int ii = (q8_issued > 2 ? q8_issued - 2 : 0); ii < q8_issued; ++ii)
-                    mbar_wait(bar_q8f + 8 * (ii & 1), (ii >> 1) & 1);
-            }
+            // every copy issued has landed before this thread leaves
+            for (int gi = (issued > nslot ? issued - nslot : 0); gi < issued; ++gi)
+                mbar_wait(full_bar(gi), full_parity(gi));
+            for (int ii = (q8_issued > 2 ? q8_issued - 2 : 0); ii < q8_issued; ++ii)
+                mbar_wait(bar_q8f + 8 * (ii & 1), (ii >> 1) & 1);
         }
     } else if (warp == NCW + 1) {
         // ------------------------------------------- reducer: protected + y
-        const int g = lane >> 2, t = lane & 3;
-        const int8_t *q8base = reinterpret_cast<const int8_t *>(sm + a.off_q8);
-        float *prot = reinterpret_cast<float *>(sm + a.off_prot);   // [BM][BP]
+        const int gq = lane >> 2, t = lane & 3;
+        const int8_t *q8base = reinterpret_cast<const int8_t *>(sm + off_q8);
+        float *prot = reinterpret_cast<float *>(sm + off_prot);   // [BM][BP]
         for (int ii = 0; ii < my_tiles; ++ii) {
             if (*reinterpret_cast<volatile int *>(&s_abort)) break;
+            const int g = layer_of(ii);
             float accp[1][4] = {{0.f, 0.f, 0.f, 0.f}};
-            if (q8_boxes > 0) {
-                if (!mbar_wait(bar_q8f + 8 * (ii & 1), (ii >> 1) & 1)) {
-                    latch_error(a.err, BISCO_ERR_TIMEOUT);
+            if (!mbar_wait_all(bar_q8f + 8 * (ii & 1), (ii >> 1) & 1)) {
+                if (lane == 0) {
+                    latch_error(err, BISCO_ERR_TIMEOUT);
                     atomicExch(&s_abort, 1);
-                    break;
                 }
-                for (int u16 = 0; u16 < a.p; u16 += 16)
-                    protected_tile<BM, 1>(q8base + (ii & 1) * q8_buf_bytes, 0, u16, a.p, g, g + 8, g,
-                                          t, s_xs, a.pidx_cap, a.B, accp);
-                __syncwarp();
-                if (lane == 0) mbar_arrive(bar_q8e + 8 * (ii & 1));
-            }
-#pragma unroll
-            for (int e = 0; e < 4; ++e) prot[(e < 2 ? g : g + 8) * BP + 2 * t + (e & 1)] = accp[0][e];
-            __syncwarp();
-            if (!mbar_wait(bar_rf + 8 * (ii & 1), (ii >> 1) & 1)) {
-                latch_error(a.err, BISCO_ERR_TIMEOUT);
-                atomicExch(&s_abort, 1);
                 break;
             }
-            const float *rb = red + (ii & 1) * NCW * BM * BP;
-            const int row0 = tile_row0(ii);
-            for (int e = lane; e < a.B * BM; e += 32) {
+            const int pg = s_L[g].p;
+            for (int u16 = 0; u16 < pg; u16 += 16)
+                protected_tile<BM, 1>(q8base + (ii & 1) * q8_buf_bytes, 0, u16, pg, gq, gq + 8, gq,
+                                      t, xs_of(g), cap, B, accp);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_q8e + 8 * (ii & 1));
+#pragma unroll
+            for (int e = 0; e < 4; ++e) prot[(e < 2 ? gq : gq + 8) * BP + 2 * t + (e & 1)] = accp[0][e];
+            __syncwarp();
+            if (!mbar_wait_all(bar_rf + 8 * (ii & 1), (ii >> 1) & 1)) {
+                if (lane == 0) {
+                    latch_error(err, BISCO_ERR_TIMEOUT);
+                    atomicExch(&s_abort, 1);
+                }
+                break;
+            }
+            const float *rb = red + (ii & 1) * NCW * BM * B;
+            const int row0 = row0_of(ii, g), N = s_L[g].N;
+            float *y = s_L[g].y;
+            for (int e = lane; e < B * BM; e += 32) {
                 const int b = e / BM, r = e - b * BM;
                 float v = 0.f;
 #pragma unroll
-                for (int wq = 0; wq < NCW; ++wq) v += rb[(wq * BM + r) * BP + b];
+                for (int wq = 0; wq < NCW; ++wq) v += rb[(wq * BM + r) * B + b];
                 v += prot[r * BP + b];
-                if (row0 + r < a.N) a.y[static_cast<int64_t>(b) * a.N + row0 + r] = v;
+                if (row0 + r < N) y[static_cast<int64_t>(b) * N + row0 + r] = v;
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_re + 8 * (ii & 1));
@@ -712,50 +856,55 @@ k_gemv_stream(const __grid_constant__ CUtensorMap tm_codes,
     } else {
         // ----------------------------------------------- consumers: decode
         const int q = warp % WQ, k = warp / WQ;
-        const int g = lane >> 2, t = lane & 3;
-        const unsigned char *xb = g < a.B ? sm + a.off_xt + g * a.xt_pitch + t * 16
-                                          : sm + a.off_zero + t * 16;
-        const int xstep = g < a.B ? 1024 : 0;
+        const int gq = lane >> 2, t = lane & 3;
+        const int xstep = gq < B ? 1024 : 0;
         for (int ii = 0; ii < my_tiles; ++ii) {
             if (*reinterpret_cast<volatile int *>(&s_abort)) break;
+            const int g = layer_of(ii);
+            const unsigned char *xb = gq < B ? xt_of(g) + gq * xt_pitch + t * 16
+                                             : sm + off_zero + t * 16;
             float acc[4][1][4];
 #pragma unroll
             for (int c = 0; c < 4; ++c)
 #pragma unroll
                 for (int e = 0; e < 4; ++e) acc[c][0][e] = 0.f;
+            bool ok = true;
             // this warp's slots of tile ii: global index ii*nwide + w == k (mod WK)
             for (int w = (k - (ii * nwide) % WK + WK) % WK; w < nwide; w += WK) {
                 const int gidx = ii * nwide + w;
-                if (*reinterpret_cast<volatile int *>(&s_abort)) break;
-                if (!mbar_wait(full_bar(gidx), full_parity(gidx))) {
-                    latch_error(a.err, BISCO_ERR_TIMEOUT);
-                    atomicExch(&s_abort, 1);
+                if (!mbar_wait_all(full_bar(gidx), full_parity(gidx)) ||
+                    __any_sync(0xFFFFFFFFu, *reinterpret_cast<volatile int *>(&s_abort) != 0)) {
+                    ok = false;
                     break;
                 }
                 const int nar = w * WQ + q;
                 if (nar < nnar) {
                     const unsigned char *cs = sm + (gidx % nslot) * kSlotBytes;
                     const unsigned char *xr[1] = {xb + nar * xstep};
-                    decode_slot<S, BM, kCodeRow, kNormRow, kSwz, 1>(cs, cs + kCodesBytes, q, g, g + 8,
-                                                                    t, xr, acc);
+                    decode_slot<S, BM, kCodeRow, kNormRow, false, 1>(cs, cs + kCodesBytes, q, gq,
+                                                                     gq + 8, t, xr, acc);
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar_empty + 8 * (gidx % nslot));
             }
             // hand this warp's partial of tile ii to the reducer (buffer ii & 1,
             // free once the reducer has finished tile ii - 2)
-            if (ii >= 2 && !mbar_wait(bar_re + 8 * (ii & 1), ((ii >> 1) - 1) & 1)) {
-                latch_error(a.err, BISCO_ERR_TIMEOUT);
-                atomicExch(&s_abort, 1);
+            if (ok && ii >= 2 && !mbar_wait_all(bar_re + 8 * (ii & 1), ((ii >> 1) - 1) & 1)) ok = false;
+            if (!ok) {
+                if (lane == 0) {
+                    latch_error(err, BISCO_ERR_TIMEOUT);
+                    atomicExch(&s_abort, 1);
+                }
                 break;
             }
-            float *rb = red + (ii & 1) * NCW * BM * BP;
+            float *rb = red + (ii & 1) * NCW * BM * B;
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
-                const int r = e < 2 ? g : g + 8;
+                const int r = e < 2 ? gq : gq + 8;
                 const int b = 2 * t + (e & 1);
-                rb[(warp * BM + r) * BP + b] =
-                    ((acc[0][0][e] + acc[1][0][e]) + (acc[2][0][e] + acc[3][0][e])) * kInvSqrt8;
+                if (b < B)
+                    rb[(warp * BM + r) * B + b] =
+                        ((acc[0][0][e] + acc[1][0][e]) + (acc[2][0][e] + acc[3][0][e])) * kInvSqrt8;
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_rf + 8 * (ii & 1));
@@ -909,14 +1058,37 @@ size_t cluster_smem(int wm, int wq, int ck, int S, int B, int p, int wide_per_ra
                        (ck > 1 ? ck - 1 : 0) * BM * BP * 4, 0, nslot * 2 + 2, a);
 }
 
-size_t stream_smem(int wq, int wk, int S, int B, int K, int p, int nslot, GemvArgs *a) {
+// Shared memory of k_gemv_stream for G layers (largest protected count
+// p_max, largest int8 slab q8_boxes).
+template <int MAXG>
+size_t stream_smem(int wq, int wk, int S, int B, int K, int G, int p_max, int q8_boxes, int nslot,
+                   StreamArgs<MAXG> *a) {
     const int BM = 16, BP = 8, SW = kSlab * wq;
     const int nar = (K + kSlab - 1) / kSlab;
-    const int cap = static_cast<int>(align_up(static_cast<size_t>(p), 16));
-    const int q8_boxes = p > 0 ? (cap + 127) / 128 : 0;
-    const size_t ring = static_cast<size_t>(nslot) * S * BM * (SW / 8 + SW / 4);
-    return layout_tail(ring, B, nar, 2 * q8_boxes * BM * 128, cap, 2 * wq * wk * BM * BP * 4, 0,
-                       BM * BP * 4, nslot * (wk + 1) + 8, a);
+    a->pidx_cap = static_cast<int>(align_up(static_cast<size_t>(p_max), 16));
+    a->mwords = nar * (kSlab / 32);
+    size_t off = static_cast<size_t>(nslot) * S * BM * (SW / 8 + SW / 4);
+    a->off_xt = static_cast<uint32_t>(off);
+    a->xt_pitch = nar * 1024 + 64;   // +64 B: rows g and g+1 land in different banks
+    off += static_cast<size_t>(G) * B * a->xt_pitch;
+    off = align_up(off, 128);
+    a->off_q8 = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(2) * q8_boxes * BM * 128;
+    a->off_pidx = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(G) * (2 + B) * a->pidx_cap * 4;   // indices, scales, scale * x
+    a->off_pmask = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(G) * 2 * a->mwords * 4;           // masks, prefix counts
+    off = align_up(off, 16);
+    a->off_zero = static_cast<uint32_t>(off);
+    off += 1024;
+    a->off_red = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(2) * wq * wk * BM * B * 4;   // partials of the B rows
+    a->off_prot = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(BM) * BP * 4;
+    off = align_up(off, 8);
+    a->off_bar = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(nslot * (wk + 1) + 8) * 8;
+    return off + 1024;   // slack for the 1024-byte aligned base
 }
 
 // k_gemv tiling rule: 2048-column slots (four column-quarter warps per row
@@ -991,10 +1163,9 @@ bisco_status launch_w(bool two, int S, const CUtensorMap &mc, const CUtensorMap 
     return launch_s<WM, WQ, 1>(S, mc, mn, mq, a, ck, smem, stream);
 }
 
-template <int WQ, int WK, int S>
-bisco_status launch_stream_t(const CUtensorMap &mc, const CUtensorMap &mn, const CUtensorMap &mq,
-                             const GemvArgs &a, int grid, size_t smem, cudaStream_t stream) {
-    auto kern = k_gemv_stream<WQ, WK, S>;
+template <int WQ, int WK, int S, int MAXG>
+bisco_status launch_stream_t(const StreamArgs<MAXG> &a, int grid, size_t smem, cudaStream_t stream) {
+    auto kern = k_gemv_stream<WQ, WK, S, MAXG>;
     static size_t configured[64] = {};
     if (!set_smem(kern, smem, configured)) return BISCO_ERR_CUDA;
     cudaLaunchConfig_t cfg = {};
@@ -1007,7 +1178,7 @@ bisco_status launch_stream_t(const CUtensorMap &mc, const CUtensorMap &mn, const
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, mc, mn, mq, a) == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+    return cudaLaunchKernelEx(&cfg, kern, a) == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
 }
 
 // Tensor maps of one layer: signs and norms as [S][N][K/8] boxes of
@@ -1047,29 +1218,64 @@ int fit_slots(size_t rest, size_t slot, size_t budget, int lo, int hi) {
     return static_cast<int>(fit < lo ? lo : (fit > hi ? hi : fit));
 }
 
-bisco_status launch_stream(const bisco_layer &L, GemvArgs &a, int sms, cudaStream_t stream,
-                           bool *launched) {
+// One k_gemv_stream launch over G layers that share x (same K and S).
+// *launched stays false when the shared memory does not fit.
+template <int MAXG>
+bisco_status launch_stream_g(const bisco_layer *Ls, int G, const uint16_t *x, int B,
+                             float *const *y, int *err, int sms, cudaStream_t stream, bool *launched) {
     constexpr int WQ = 4, WK = 2;
-    const int N = L.n_out, K = L.k_in, S = L.stages, p = L.n_protected, B = a.B;
+    const int K = Ls[0].k_in, S = Ls[0].stages;
     *launched = false;
+    StreamArgs<MAXG> a = {};
+    a.x = x;
+    a.err = err;
+    a.K = K;
+    a.B = B;
+    a.G = G;
+    int p_max = 0, q8_max = 0, tiles = 0;
+    for (int g = 0; g < G; ++g) {
+        const bisco_layer &L = Ls[g];
+        StreamLayer &sl = a.L[g];
+        sl.y = y[g];
+        sl.q8_scale = L.q8_scale;
+        sl.prot_idx = L.prot_idx;
+        sl.N = L.n_out;
+        sl.p = L.n_protected;
+        sl.tile0 = tiles;
+        sl.q8_boxes = L.n_protected > 0 ? ((L.n_protected + 15) / 16 * 16 + 127) / 128 : 0;
+        tiles += (L.n_out + 15) / 16;
+        p_max = p_max > sl.p ? p_max : sl.p;
+        q8_max = q8_max > sl.q8_boxes ? q8_max : sl.q8_boxes;
+    }
+    a.ntiles = tiles;
+    a.q8_boxes = q8_max;
     const size_t slot = static_cast<size_t>(S) * 16 * (kSlab * WQ / 8 + kSlab * WQ / 4);
     int nslot = 0;
     if (const char *e = getenv("BISCO_GEMV_NSLOT")) nslot = atoi(e);
     if (nslot <= 0 || nslot > 16)
-        nslot = fit_slots(stream_smem(WQ, WK, S, B, K, p, 0, &a), slot, kCoresident, 2, 8);
-    const size_t smem = stream_smem(WQ, WK, S, B, K, p, nslot, &a);
-    if (smem > kMaxSmem) return BISCO_OK;   // caller falls back to k_gemv
+        nslot = fit_slots(stream_smem(WQ, WK, S, B, K, G, p_max, q8_max, 0, &a), slot, kCoresident,
+                          2, 8);
+    const size_t smem = stream_smem(WQ, WK, S, B, K, G, p_max, q8_max, nslot, &a);
+    if (smem > kMaxSmem) return BISCO_OK;
     a.nslot = nslot;
-    const int ntiles = (N + 15) / 16;
-    const int grid = ntiles < sms ? ntiles : sms;
-    CUtensorMap mc, mn, mq;
-    if (!layer_maps(L, 16, kSlab * WQ, false, &mc, &mn, &mq)) return BISCO_ERR_CUDA;
+    for (int g = 0; g < G; ++g)
+        if (!layer_maps(Ls[g], 16, kSlab * WQ, false, &a.mc[g], &a.mn[g], &a.mq[g]))
+            return BISCO_ERR_CUDA;
+    const int grid = tiles < sms ? tiles : sms;
     *launched = true;
     switch (S) {
-        case 1: return launch_stream_t<WQ, WK, 1>(mc, mn, mq, a, grid, smem, stream);
-        case 2: return launch_stream_t<WQ, WK, 2>(mc, mn, mq, a, grid, smem, stream);
-        default: return launch_stream_t<WQ, WK, 3>(mc, mn, mq, a, grid, smem, stream);
+        case 1: return launch_stream_t<WQ, WK, 1, MAXG>(a, grid, smem, stream);
+        case 2: return launch_stream_t<WQ, WK, 2, MAXG>(a, grid, smem, stream);
+        default: return launch_stream_t<WQ, WK, 3, MAXG>(a, grid, smem, stream);
     }
+}
+
+// A single layer gets the one-layer instantiation: a run-time layer index
+// (and the larger parameter block) cost about 5 % per launch.
+bisco_status launch_stream(const bisco_layer *Ls, int G, const uint16_t *x, int B, float *const *y,
+                           int *err, int sms, cudaStream_t stream, bool *launched) {
+    if (G == 1) return launch_stream_g<1>(Ls, G, x, B, y, err, sms, stream, launched);
+    return launch_stream_g<kMaxGroup>(Ls, G, x, B, y, err, sms, stream, launched);
 }
 
 }  // namespace
@@ -1104,7 +1310,7 @@ bisco_status launch_gemv(const bisco_layer &L, const uint16_t *x, int B, float *
     if (mode && mode[0] == 'c') use_stream = false;
     if (use_stream) {
         bool launched = false;
-        const bisco_status st = launch_stream(L, a, sms, stream, &launched);
+        const bisco_status st = launch_stream(&L, 1, x, B, &y, err, sms, stream, &launched);
         if (launched || st != BISCO_OK) return st;
     }
 
@@ -1150,6 +1356,20 @@ bisco_status launch_gemv(const bisco_layer &L, const uint16_t *x, int B, float *
     if (pl.wm == 8 && pl.wq == 1) return launch_w<8, 1>(two, S, mc, mn, mq, a, ck, smem, stream);
     if (pl.wm == 1 && pl.wq == 2) return launch_w<1, 2>(two, S, mc, mn, mq, a, ck, smem, stream);
     return BISCO_ERR_UNSUPPORTED;
+}
+
+bisco_status launch_gemv_multi(const bisco_layer *Ls, int G, const uint16_t *x, int B,
+                               float *const *y, int *err, cudaStream_t stream) {
+    if (B <= 8 && Ls[0].k_in % 128 == 0) {
+        bool launched = false;
+        const bisco_status st = launch_stream(Ls, G, x, B, y, err, num_sms(), stream, &launched);
+        if (launched || st != BISCO_OK) return st;
+    }
+    for (int g = 0; g < G; ++g) {   // one launch per layer
+        const bisco_status st = launch_gemv(Ls[g], x, B, y[g], err, stream);
+        if (st != BISCO_OK) return st;
+    }
+    return BISCO_OK;
 }
 
 }  // namespace bisco

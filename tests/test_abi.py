@@ -35,7 +35,7 @@ def test_header_declarations_are_exported(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert bisco.bisco_abi_version() == 101
+    assert bisco.bisco_abi_version() == 102
     for code in range(6):
         assert bisco.status_string(code)
     assert bisco.status_string(99) == "unknown status"
@@ -115,3 +115,26 @@ def test_call_argument_validation(lib):
     L2 = _fake_layer(k_in=4096, n_protected=41)
     assert lib.bisco_gemm_workspace_bytes(ctypes.byref(L2), 2048) == 2048 * (4096 + 128) * 2
     assert lib.bisco_gemm(ctypes.byref(L2), x, 2048, y, None, 0, None) == bisco.ERR_INVALID_ARG
+
+
+def test_gemv_multi_validation(lib):
+    L = _fake_layer()
+    x = ctypes.c_void_p(0x60000)
+    ys = (ctypes.c_void_p * 4)(0x70000, 0x71000, 0x72000, 0x73000)
+    arr = (bisco.bisco_layer * 4)(L, L, L, L)
+    assert lib.bisco_gemv_multi(arr, 0, x, 1, ys, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_gemv_multi(arr, 5, x, 1, ys, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_gemv_multi(None, 1, x, 1, ys, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_gemv_multi(arr, 2, x, 1, None, None) == bisco.ERR_INVALID_ARG
+    mixed = (bisco.bisco_layer * 2)(L, _fake_layer(k_in=512))          # K differs
+    assert lib.bisco_gemv_multi(mixed, 2, x, 1, ys, None) == bisco.ERR_INVALID_ARG
+    mixed = (bisco.bisco_layer * 2)(L, _fake_layer(stages=3))          # S differs
+    assert lib.bisco_gemv_multi(mixed, 2, x, 1, ys, None) == bisco.ERR_INVALID_ARG
+    bad = (bisco.bisco_layer * 2)(L, _fake_layer(codes=0x10004))       # layer invalid
+    assert lib.bisco_gemv_multi(bad, 2, x, 1, ys, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_gemv_multi(arr, 2, x, 17, ys, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_gemv_multi(arr, 2, ctypes.c_void_p(0x60002), 1, ys, None) \
+        == bisco.ERR_INVALID_ARG
+    odd = (ctypes.c_void_p * 2)(0x70000, 0x70004)                       # y[1] misaligned
+    assert lib.bisco_gemv_multi(arr, 2, x, 1, odd, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_gemv_multi(arr, 2, x, 0, ys, None) == bisco.OK   # empty batch

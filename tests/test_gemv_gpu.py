@@ -147,3 +147,63 @@ def test_gemv_zero_and_tiny_activations(env):
     Lref = oracle.encode(W, S=S, p=p)
     y = run_gemv(env, Lref, np.zeros((2, K), np.uint16))
     assert np.all(y == 0)
+
+
+def _multi(env, Lrefs, X, extra_env=None):
+    import torch
+    bisco, dev = env
+    Ls = [bisco.Layer.from_numpy(L, dev) for L in Lrefs]
+    old = {k: os.environ.get(k) for k in (extra_env or {})}
+    os.environ.update(extra_env or {})
+    try:
+        ys = bisco.bisco_gemv_multi(Ls, to_dev(X, dev))
+    finally:
+        for k, v in old.items():
+            if v is None:
+                del os.environ[k]
+            else:
+                os.environ[k] = v
+    torch.cuda.synchronize()
+    assert bisco.bisco_get_device_error() == 0
+    return [y.cpu().numpy() for y in ys]
+
+
+@pytest.mark.parametrize("B", [1, 3, 8, 12])
+@pytest.mark.parametrize("nslot", [None, 3])
+def test_gemv_multi_matches_oracle(env, B, nslot):
+    """Grouped launch over layers sharing x with different N and protected
+    sets (one layer unprotected); B = 12 takes the per-layer path."""
+    K, S = 2048, 2
+    shapes = [(300, 21), (64, 0), (1000, 33)]
+    Lrefs = [oracle.encode(synth.layer_weights(N, K, seed=40 + i), S=S, p=p)
+             for i, (N, p) in enumerate(shapes)]
+    X = synth.activations(B, K, seed=41)
+    ys = _multi(env, Lrefs, X, {"BISCO_GEMV_NSLOT": str(nslot)} if nslot else None)
+    for y, L in zip(ys, Lrefs):
+        assert max_rel_rows(y, oracle.gemv(L, X)) <= TOL
+
+
+def test_gemv_multi_qkv_full_size(env):
+    """q/k/v of one Qwen3-8B attention layer in one launch, batch 1."""
+    K, S = 4096, 2
+    p = synth.protected_count(K, 1)
+    names = ("q_proj", "k_proj", "v_proj")
+    Lrefs = [oracle.encode(synth.layer_weights(synth.QWEN3_8B_SHAPES[n][0], K, seed=60 + i),
+                           S=S, p=p) for i, n in enumerate(names)]
+    X = synth.activations(1, K, seed=61)
+    ys = _multi(env, Lrefs, X)
+    for y, L, n in zip(ys, Lrefs, names):
+        rows = sample_rows(L["N"], n=24)
+        assert max_rel_rows(y[:, rows], oracle.apply_rows(L, rows, X)) <= TOL, n
+
+
+def test_gemv_multi_single_layer_matches_gemv(env):
+    import torch
+    bisco, dev = env
+    K, S = 1024, 3
+    Lref = oracle.encode(synth.layer_weights(2500, K, seed=70, dist="t4"), S=S, p=11)
+    X = synth.activations(2, K, seed=71)
+    (ym,) = _multi(env, [Lref], X)
+    y = run_gemv(env, Lref, X)
+    assert max_rel_rows(ym, y) <= 1e-5
+    assert max_rel_rows(ym, oracle.gemv(Lref, X)) <= TOL
