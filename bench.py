@@ -45,8 +45,11 @@ def parse():
     ap.add_argument("--impl", choices=("bisco", "reference"), default="bisco")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
-    ap.add_argument("--mode", choices=("both", "decode", "prefill"), default="both",
-                    help="decode: the GEMV step only; prefill: the tcgen05 GEMM only")
+    ap.add_argument("--mode", choices=("both", "decode", "prefill", "shapes"), default="both",
+                    help="decode: the GEMV step only; prefill: the tcgen05 GEMM only; "
+                         "shapes: batch-1 GEMV per Qwen3-8B layer shape")
+    ap.add_argument("--shape-mb", type=float, default=500.0,
+                    help="--mode shapes: MB of distinct coded layers per shape (> L2)")
     ap.add_argument("--prefill-tokens", type=int, default=2048)
     ap.add_argument("--ungrouped", action="store_true",
                     help="one bisco_gemv per projection instead of bisco_gemv_multi for q/k/v")
@@ -76,8 +79,8 @@ def tensor_peaks():
 # DRAM bytes (read + write) of one q_proj/o_proj launch of the dominant
 # kernel, from the ncu capture summarised in profiles/ (see the file for the
 # command), valid while the kernel source hashes to the recorded digest.
-DOMINANT_TRAFFIC = {"bytes": None, "gemv_cu_sha256": None,
-                    "profile": "profiles/k_gemv_stream_q_proj_4096x4096_b1.md"}
+DOMINANT_TRAFFIC = {"bytes": 19249664, "gemv_cu_sha256": "b9f38afc1f4233b05754d37a4b91881fb046c03dc9e0b99cd266c9f025928c2e",
+                    "profile": "profiles/k_gemv_stream_qkv_group_b1.md"}
 
 
 def dominant_traffic():
@@ -403,6 +406,67 @@ def run_prefill(args, local_rank):
             "dtype": "f16 x f16 -> f32", "launches_per_step": 2 * len(layers)}
 
 
+# ----------------------------------------------------------------- shapes
+
+def run_shapes(args, local_rank):
+    """Batch-1 bisco_gemv per Qwen3-8B linear shape: a CUDA graph of one call
+    on each of about --shape-mb MB of distinct coded layers of that shape
+    (larger than L2, so every call streams from HBM), CUDA events over
+    `steps` replays; GB/s on the algorithmic compressed bytes.  Attention
+    shapes use S=2 and 1 % protection (N(0,0.02) weights), MLP shapes S=3
+    and 2 % (Student-t(4) weights), as in the paper-derived configurations."""
+    import torch
+    from paper_2607_08643_gb300 import bisco, synth
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    peak, _ = peaks()
+    out = []
+    for name, (N, K) in synth.QWEN3_8B_SHAPES.items():
+        mlp = name in synth.MLP
+        S, rho, dist = (3, 2, "t4") if mlp else (2, 1, "normal")
+        p = synth.protected_count(K, rho)
+        one = S * N * (K // 8) * 3 + N * p + 6 * p
+        nl = max(4, int(args.shape_mb * 1e6 / one))
+        W = synth.layer_weights_torch(N, K, seed=900, device=dev, dist=dist)
+        ws = torch.empty(bisco.bisco_encode_workspace_bytes(N, K), dtype=torch.uint8, device=dev)
+        layers = [bisco.bisco_encode(W, S, p, workspace=ws) for _ in range(nl)]
+        del W
+        xs = torch.randn((nl, 1, K), device=dev).to(torch.bfloat16).view(torch.int16)
+        ys = torch.empty((nl, 1, N), device=dev)
+        torch.cuda.synchronize()
+        stream = torch.cuda.Stream(device=dev)
+        with torch.cuda.stream(stream):
+            for i, L in enumerate(layers):
+                bisco.bisco_gemv(L, xs[i], y=ys[i], stream=stream)
+            torch.cuda.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for i, L in enumerate(layers):
+                    bisco.bisco_gemv(L, xs[i], y=ys[i], stream=stream)
+        torch.cuda.synchronize()
+        for _ in range(max(args.warmup, 3)):
+            g.replay()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(args.steps):
+                g.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        if bisco.bisco_get_device_error(stream) != bisco.OK:
+            raise RuntimeError("device error in shape sweep")
+        us = e0.elapsed_time(e1) * 1e3 / (args.steps * nl)
+        gbs = one / (us * 1e-6) / 1e9
+        out.append({"shape": name, "N": N, "K": K, "S": S, "p": p, "layers": nl,
+                    "bytes_per_launch": one, "us_per_launch": us, "gbs": gbs,
+                    "frac_of_hbm": gbs / peak})
+        del layers, xs, ys, g
+        torch.cuda.empty_cache()
+    return out
+
+
 # ------------------------------------------------------------ CPU oracle
 
 def cpu_oracle_sample(seconds, batch):
@@ -482,6 +546,13 @@ def main():
         if world > 1:
             import torch.distributed as dist
             dist.destroy_process_group()
+        return
+    if args.mode == "shapes":
+        res = run_shapes(args, local_rank)
+        if rank == 0:
+            print(json.dumps({"metric": "batch-1 GEMV GB/s per Qwen3-8B shape (compressed bytes)",
+                              "unit": "GB/s", "hbm_peak_gbs": peaks()[0], "steps": args.steps,
+                              "data": "synthetic", "shapes": res}))
         return
     if args.mode == "prefill":
         pf = run_prefill(args, local_rank)

@@ -9,7 +9,8 @@ import ctypes
 import os
 
 HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(HERE, "libbisco.so")
+# BISCO_LIB selects another build of the same library (for A/B timing).
+LIB_PATH = os.environ.get("BISCO_LIB") or os.path.join(HERE, "libbisco.so")
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_RANGE, ERR_CUDA, ERR_TIMEOUT = range(6)
 
