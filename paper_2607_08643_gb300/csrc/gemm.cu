@@ -35,8 +35,10 @@ namespace {
 constexpr int GM = 128;     // output features per tile (MMA M, TMEM lanes)
 constexpr int GN = 256;     // tokens per tile (MMA N)
 constexpr int GK = 128;     // K columns per weight step (one TMEM A stage)
-constexpr int NX = 4;       // activation ring (64-column, 32 KB stages)
-constexpr int NW = 4;       // compressed-weight ring (128-column stages)
+// Ring depths are template parameters (NX activation stages of 64 columns
+// = 32 KB, NW compressed-weight stages of 128 columns): the activation ring
+// must cover the L2 latency of a stream consumed at 64 B/clk, so it takes
+// what the weight ring leaves of the 227 KB.
 constexpr int NA = 3;       // TMEM A ring (128 K columns = 64 TMEM columns each)
 constexpr int kThreads = 512;
 constexpr uint32_t kTmemCols = 512;
@@ -114,6 +116,7 @@ __device__ __forceinline__ void decode_q8_row(const unsigned char *q8s, int r, u
     }
 }
 
+template <int NX, int NW>
 __global__ void __launch_bounds__(kThreads, 1)
 k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_codes,
        const __grid_constant__ CUtensorMap tm_norms, const __grid_constant__ CUtensorMap tm_q8,
@@ -401,6 +404,24 @@ bisco_status gemm_via_gemv(const bisco_layer &L, const uint16_t *X, int M, float
     return BISCO_OK;
 }
 
+template <int NX, int NW>
+bisco_status launch_gemm_t(const CUtensorMap &mx, const CUtensorMap &mc, const CUtensorMap &mn,
+                           const CUtensorMap &mq, const GemmArgs &a, int grid, cudaStream_t stream) {
+    const size_t smem = 1024 + NX * kXStage + NW * a.w_stage + 8 * (2 * NX + 2 * NW + 2 * NA + 3);
+    if (smem > 227 * 1024) return BISCO_ERR_UNSUPPORTED;
+    static size_t configured[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return BISCO_ERR_CUDA;
+    if (smem > configured[dev]) {
+        if (cudaFuncSetAttribute(k_gemm<NX, NW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(smem)) != cudaSuccess)
+            return BISCO_ERR_CUDA;
+        configured[dev] = smem;
+    }
+    k_gemm<NX, NW><<<grid, kThreads, smem, stream>>>(mx, mc, mn, mq, a);
+    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+}
+
 }  // namespace
 
 size_t gemm_workspace_bytes(const bisco_layer &L, int M) {
@@ -476,20 +497,11 @@ bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *
     a.tiles_t = (M + GN - 1) / GN;
     a.ntiles = a.tiles_t * ((N + GM - 1) / GM);
     a.w_stage = static_cast<uint32_t>(S * GM * 48 > GM * 64 ? S * GM * 48 : GM * 64);
-    const size_t smem = 1024 + NX * kXStage + NW * a.w_stage + 8 * (2 * NX + 2 * NW + 2 * NA + 3);
-    static size_t configured[64] = {};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return BISCO_ERR_CUDA;
-    if (smem > configured[dev]) {
-        if (cudaFuncSetAttribute(k_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 static_cast<int>(smem)) != cudaSuccess)
-            return BISCO_ERR_CUDA;
-        configured[dev] = smem;
-    }
     const int sms = num_sms();
     const int grid = a.ntiles < sms ? a.ntiles : sms;
-    k_gemm<<<grid, kThreads, smem, stream>>>(mx, mc, mn, mq, a);
-    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+    // S = 1: 6 x 32 KB + 3 x 8 KB; S = 2, 3: 5 x 32 KB + 3 x 12/18 KB (<= 227 KB)
+    if (S == 1) return launch_gemm_t<6, 3>(mx, mc, mn, mq, a, grid, stream);
+    return launch_gemm_t<5, 3>(mx, mc, mn, mq, a, grid, stream);
 }
 
 }  // namespace bisco
