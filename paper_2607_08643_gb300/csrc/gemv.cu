@@ -1252,9 +1252,14 @@ bisco_status launch_stream_g(const bisco_layer *Ls, int G, const uint16_t *x, in
     const size_t slot = static_cast<size_t>(S) * 16 * (kSlab * WQ / 8 + kSlab * WQ / 4);
     int nslot = 0;
     if (const char *e = getenv("BISCO_GEMV_NSLOT")) nslot = atoi(e);
-    if (nslot <= 0 || nslot > 16)
+    if (nslot <= 0 || nslot > 16) {
+        // at least three slots: with two, the refills of a long launch are
+        // exposed (measured -15 % on the S = 3 MLP shapes), which costs more
+        // than sharing the SM with the next kernel gains
         nslot = fit_slots(stream_smem(WQ, WK, S, B, K, G, p_max, q8_max, 0, &a), slot, kCoresident,
-                          2, 8);
+                          3, 8);
+        if (stream_smem(WQ, WK, S, B, K, G, p_max, q8_max, nslot, &a) > kMaxSmem) nslot = 2;
+    }
     const size_t smem = stream_smem(WQ, WK, S, B, K, G, p_max, q8_max, nslot, &a);
     if (smem > kMaxSmem) return BISCO_OK;
     a.nslot = nslot;
