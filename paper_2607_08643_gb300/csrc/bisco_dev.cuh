@@ -22,6 +22,19 @@ __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+// Shared-space loads by 32-bit shared address (never a generic access).
+__device__ __forceinline__ uint32_t lds_u32(uint32_t addr) {
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ uint2 lds_u64(uint32_t addr) {
+    uint2 v;
+    asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
+    return v;
+}
+
 __device__ __forceinline__ uint64_t globaltimer() {
     uint64_t t;
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
@@ -336,6 +349,42 @@ __device__ __forceinline__ uint32_t lop3_and_xor(uint32_t a, uint32_t mask, uint
     uint32_t r;
     asm("lop3.b32 %0, %1, %2, %3, 0x6A;" : "=r"(r) : "r"(a), "r"(mask), "r"(c));
     return r;
+}
+
+__device__ __forceinline__ uint32_t lop3_and_or(uint32_t a, uint32_t mask, uint32_t c) {
+    // (a & mask) | c
+    uint32_t r;
+    asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(r) : "r"(a), "r"(mask), "r"(c));
+    return r;
+}
+
+__device__ __forceinline__ uint16_t lo_half(uint32_t w) {
+    uint16_t l, h;
+    asm("mov.b32 {%0, %1}, %2;" : "=h"(l), "=h"(h) : "r"(w));
+    return l;
+}
+
+__device__ __forceinline__ uint16_t hi_half(uint32_t w) {
+    uint16_t l, h;
+    asm("mov.b32 {%0, %1}, %2;" : "=h"(l), "=h"(h) : "r"(w));
+    return h;
+}
+
+// c + a * b for fp16 a, b (bit patterns) and fp32 c: the product of two fp16
+// values is exact in fp32, so the result is rounded once, to fp32
+__device__ __forceinline__ float fma_f16_f32(uint16_t a, uint16_t b, float c) {
+    float d;
+    asm("fma.rn.f32.f16 %0, %1, %2, %3;" : "=f"(d) : "h"(a), "h"(b), "f"(c));
+    return d;
+}
+
+// Two int8 (low 16 bits of v) -> exact fp16 pair: with the sign bits
+// flipped each byte is b + 128, which as the low mantissa byte of 1024.0 is
+// 1024 + b + 128 exactly; subtracting 1152 leaves b.
+__device__ __forceinline__ uint32_t i8x2_to_h2(uint32_t v) {
+    uint32_t h = prmt(v ^ 0x8080u, 0x64646464u, 0x5140u);
+    const __half2 r = __hsub2(*reinterpret_cast<const __half2 *>(&h), __floats2half2_rn(1152.f, 1152.f));
+    return *reinterpret_cast<const uint32_t *>(&r);
 }
 
 __device__ __forceinline__ uint16_t bf16_bits_to_f16_bits(uint16_t b) {

@@ -78,10 +78,12 @@ __device__ __forceinline__ void decode_pairs(int i0, uint32_t cl, uint32_t ch, u
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
-// 1024-byte aligned base of the dynamic shared memory, derived by pointer
-// arithmetic on the shared array so that accesses stay shared-space ones.
+// A-byte aligned base of the dynamic shared memory (1024 for the 128-byte
+// swizzle, 128 for plain TMA boxes), derived by pointer arithmetic on the
+// shared array so that accesses stay shared-space ones.
+template <uint32_t A = 1024>
 __device__ __forceinline__ unsigned char *aligned_smem(unsigned char *raw) {
-    return raw + ((1024u - (smem_u32(raw) & 1023u)) & 1023u);
+    return raw + ((A - (smem_u32(raw) & (A - 1u))) & (A - 1u));
 }
 
 constexpr int kMaxGroup = 4;   // layers sharing one activation in a grouped launch
@@ -104,7 +106,7 @@ struct StageView {
 // round trip to memory.  Job = one 32-column group of one row.  Pair i of a
 // 32-column group is element i&7 of chunk (i>>3) and of chunk (i>>3)+2 --
 // bits i and i+16 of its code word, columns (i>>3)*8 + (i&7) and that + 16.
-template <int MAXG>
+template <int MAXG, bool kHalfXs = false>
 __device__ __forceinline__ void stage_activations(const uint16_t *x, int K, int B, int k_begin,
                                                   int cols, int nnar, int xt_pitch, int cap,
                                                   int G, const StageView (&v)[MAXG]) {
@@ -154,7 +156,15 @@ __device__ __forceinline__ void stage_activations(const uint16_t *x, int K, int 
             for (uint32_t bits = pm; bits; bits &= bits - 1u) {
                 const int k = __ffs(bits) - 1;
                 const int u = u0 + __popc(pm & ((1u << k) - 1u));
-                v[g].xs[b * cap + u] = v[g].pscale[u] * bf16_bits_to_f32(src[k]);
+                const float sx = v[g].pscale[u] * bf16_bits_to_f32(src[k]);
+                if constexpr (kHalfXs) {
+                    __half *xh = reinterpret_cast<__half *>(v[g].xs);
+                    const __half hi = __float2half_rn(sx);
+                    xh[b * cap + u] = hi;
+                    xh[(B + b) * cap + u] = __float2half_rn(sx - __half2float(hi));
+                } else {
+                    v[g].xs[b * cap + u] = sx;
+                }
             }
             uint32_t om[16];
 #pragma unroll
@@ -222,16 +232,19 @@ __device__ __forceinline__ void decode_slot(const unsigned char *cs, const unsig
 }
 
 // Protected k tile u16..u16+15 for rows lo/hi (Eq. 10): q8 bytes from the
-// TMA'd int8 slab (column col0 + u of box-major [box][BM][128] storage) as
-// exact fp16 integers against scale * x (s_xs) split into fp16 hi + lo.
+// int8 slab in shared memory (column col0 + u; box-major [box][BM][128]
+// storage, or rows of q8_pitch bytes when q8_pitch > 0) as exact fp16
+// integers against scale * x (s_xs) split into fp16 hi + lo.
 template <int BM, int NT>
 __device__ __forceinline__ void protected_tile(const int8_t *q8s, int col0, int u16, int p_loc,
                                                int rlo, int rhi, int g, int t, const float *s_xs,
-                                               int xs_pitch, int B, float (&accp)[NT][4]) {
+                                               int xs_pitch, int B, float (&accp)[NT][4],
+                                               int q8_pitch = 0) {
     auto q8v = [&](int r, int u) -> float {
         if (u >= p_loc) return 0.f;
         const int col = col0 + u;
-        return static_cast<float>(q8s[((col >> 7) * BM + r) * 128 + (col & 127)]);
+        return static_cast<float>(q8_pitch > 0 ? q8s[r * q8_pitch + col]
+                                               : q8s[((col >> 7) * BM + r) * 128 + (col & 127)]);
     };
     const int u0 = u16 + 2 * t;
     uint32_t af[4];
@@ -262,6 +275,29 @@ __device__ __forceinline__ void protected_tile(const int8_t *q8s, int col0, int 
         mma_16816(accp[nt], af, hi[0], hi[1]);
         mma_16816(accp[nt], af, lo[0], lo[1]);
     }
+}
+
+// Protected k tile u16..u16+15 of rows g and g + 8 (Eq. 10), batch column g
+// of the MMA: q8 from a tile slab of rows of `pitch` bytes (16-bit loads of
+// column pairs, exact int8 -> fp16), scale * x as fp16 hi + lo halves
+// xsh/xsl [B][cap], zero past the layer's p, so no bounds checks.
+__device__ __forceinline__ void protected_rows(const int8_t *q8s, int pitch, int u16, int g, int t,
+                                               const __half *xsh, const __half *xsl, int cap, int B,
+                                               float (&acc)[4]) {
+    const int u0 = u16 + 2 * t;
+    auto pair = [&](int r, int u) {
+        return i8x2_to_h2(*reinterpret_cast<const uint16_t *>(q8s + r * pitch + u));
+    };
+    const uint32_t af[4] = {pair(g, u0), pair(g + 8, u0), pair(g, u0 + 8), pair(g + 8, u0 + 8)};
+    uint32_t h0 = 0u, h1 = 0u, l0 = 0u, l1 = 0u;
+    if (g < B) {
+        h0 = *reinterpret_cast<const uint32_t *>(xsh + g * cap + u0);
+        h1 = *reinterpret_cast<const uint32_t *>(xsh + g * cap + u0 + 8);
+        l0 = *reinterpret_cast<const uint32_t *>(xsl + g * cap + u0);
+        l1 = *reinterpret_cast<const uint32_t *>(xsl + g * cap + u0 + 8);
+    }
+    mma_16816(acc, af, h0, h1);
+    mma_16816(acc, af, l0, l1);
 }
 
 // Protected-column bookkeeping of one CTA (warp 0): indices in [k_begin,
@@ -572,28 +608,202 @@ k_gemv(const __grid_constant__ CUtensorMap tm_codes, const __grid_constant__ CUt
 // consumer group always waits on a barrier whose previous phase it observed
 // itself, whatever the ring depth.
 
+// ------------------------------------------------------------------------
+// Table-lookup decode for a single activation row (batch 1).
+//
+// Per sign byte b of chunk c, Eq. 12's inner product sum_e s_e x[8c+e] is
+// the sum of two signed sums of four activations, one per half of the byte.
+// The tables hold them for every chunk and every v = 0..15:
+//   T_lo(c, v) = sum_{e<4} (bit e of v ? -x[8c+e] : +x[8c+e])
+//   T_hi(c, v) = the same over x[8c+4+e]
+// as one fp16 pair (T_lo low, T_hi high) per 32-bit word.  A chunk-stage
+// then costs two shared-memory lookups, T_lo(c, b & 15) and T_hi(c, b >> 4),
+// and two fp16 x fp16 -> fp32 FMAs with its norm, instead of decoding eight
+// signs.  Rounding T to fp16 is this path's one approximation (relative
+// 2^-11 of each half sum).
+//
+// Placement: chunk c sits at position P, where within each group of 128
+// chunks chunk 4l + j is at 32j + l, and entry (P, v) is at byte
+//   (P >> 6) * 4096 + v * 256 + (P & 63) * 4.
+// Lane l reading chunk 4l + j of its code word thus hits bank l, and the
+// address is one byte permute: byte 0 the lane's slot (P & 63) * 4, byte 1
+// the nibble with (P >> 6) & 15 above it, byte 2 (P >> 6) >> 4.
+constexpr int kLutSlotCols = 2048;                    // ring slot width the placement assumes
+constexpr int kLutSlotBytes = kLutSlotCols / 8 * 64;  // table bytes per slot of columns
+
+// Tables of x[0, K) for nchunk chunk positions (a multiple of 128; chunks at
+// or past K/8 get zero tables, so a ragged last slot reads zeros).  With a
+// protected-column mask (a bit per column, 32 per word) those columns count
+// as zero, which is Eq. 10's overwrite for a launch of one layer.
+__device__ __forceinline__ void build_nibble_tables(const uint16_t *x, int K, int nchunk,
+                                                    const uint32_t *pmask, unsigned char *tab) {
+    // a warp's jobs go in batches whose loads are all issued before any
+    // table is written: one round trip to memory per batch (one in all for
+    // K up to 2 * 32 * 8 * warps columns; larger batches measured slower on
+    // the short layers)
+    constexpr int kBatch = 2;
+    const int lane = threadIdx.x & 31, nwarp = static_cast<int>(blockDim.x >> 5);
+    const int njobs = nchunk / 32;
+    for (int J0 = static_cast<int>(threadIdx.x >> 5); J0 < njobs; J0 += kBatch * nwarp) {
+        uint4 u[kBatch];
+        uint32_t m[kBatch];
+#pragma unroll
+        for (int i = 0; i < kBatch; ++i) {
+            const int J = J0 + i * nwarp;
+            const int c = (J >> 2) * 128 + 4 * lane + (J & 3);
+            u[i] = make_uint4(0u, 0u, 0u, 0u);
+            m[i] = 0u;
+            if (J < njobs && 8 * c < K) {
+                u[i] = *reinterpret_cast<const uint4 *>(x + 8 * c);
+                if (pmask != nullptr) m[i] = (pmask[c >> 2] >> ((c & 3) * 8)) & 0xFFu;
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < kBatch; ++i) {
+            const int J = J0 + i * nwarp;
+            if (J >= njobs) break;
+            const int P = (J >> 2) * 128 + 32 * (J & 3) + lane;
+            float e[8] = {bf16_lo(u[i].x), bf16_hi(u[i].x), bf16_lo(u[i].y), bf16_hi(u[i].y),
+                          bf16_lo(u[i].z), bf16_hi(u[i].z), bf16_lo(u[i].w), bf16_hi(u[i].w)};
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                if ((m[i] >> k) & 1u) e[k] = 0.f;
+            // signed sums of element pairs: index bit 0 negates the first, bit 1 the second
+            float a[2][4], d[2][4];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const float x0 = e[4 * h], x1 = e[4 * h + 1], x2 = e[4 * h + 2], x3 = e[4 * h + 3];
+                a[h][0] = x0 + x1; a[h][1] = x1 - x0; a[h][2] = x0 - x1; a[h][3] = -(x0 + x1);
+                d[h][0] = x2 + x3; d[h][1] = x3 - x2; d[h][2] = x2 - x3; d[h][3] = -(x2 + x3);
+            }
+            unsigned char *dst = tab + (P >> 6) * 4096 + (P & 63) * 4;
+#pragma unroll
+            for (int v = 0; v < 16; ++v) {
+                const __half2 t = __floats2half2_rn(a[0][v & 3] + d[0][v >> 2], a[1][v & 3] + d[1][v >> 2]);
+                *reinterpret_cast<__half2 *>(dst + v * 256) = t;
+            }
+        }
+    }
+}
+
+// One ring slot (2048 columns, slot index w along K) for rows row0..row0+R-1
+// and all S stages: lane l takes code words l and 32 + l of each row, i.e.
+// chunks 4(32m + l) + j at table positions 256w + 128m + 32j + l.
+template <int S, int R, int kCodeRow, int kNormRow>
+__device__ __forceinline__ void lut_slot(uint32_t cs, uint32_t ns, uint32_t tab, int w, int row0,
+                                         int lane, float (&acc)[R]) {
+    uint32_t sgpat[2], base[2][4];
+#pragma unroll
+    for (int m = 0; m < 2; ++m) {
+        // 64-position table blocks of chunks j = 0, 1 and j = 2, 3 of word m
+        const uint32_t g0 = 4u * static_cast<uint32_t>(w) + 2u * m, g1 = g0 + 1u;
+        sgpat[m] = (g0 & 15u) * 0x1010u | (g1 & 15u) * 0x10100000u;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            base[m][j] = static_cast<uint32_t>(lane) * 4u + (j & 1) * 128u + (((j < 2 ? g0 : g1) >> 4) << 16);
+    }
+#pragma unroll 1
+    for (int s = 0; s < S; ++s) {
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            const uint32_t crow = cs + (s * 16 + row0 + r) * kCodeRow + lane * 4;
+            const uint32_t nrow = ns + (s * 16 + row0 + r) * kNormRow + lane * 8;
+#pragma unroll
+            for (int m = 0; m < 2; ++m) {
+                const uint32_t cw = lds_u32(crow + m * 128);
+                const uint2 nw = lds_u64(nrow + m * 256);
+                const uint32_t wl = lop3_and_or(cw, 0x0F0F0F0Fu, sgpat[m]);
+                const uint32_t wh = lop3_and_or(cw >> 4, 0x0F0F0F0Fu, sgpat[m]);
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const uint32_t sel = 0x7604u | (static_cast<uint32_t>(j) << 4);
+                    const uint32_t tl = lds_u32(tab + prmt(wl, base[m][j], sel));
+                    const uint32_t th = lds_u32(tab + prmt(wh, base[m][j], sel));
+                    const uint32_t nj = j < 2 ? nw.x : nw.y;
+                    const uint16_t n = (j & 1) ? hi_half(nj) : lo_half(nj);
+                    acc[r] = fma_f16_f32(lo_half(tl), n, acc[r]);
+                    acc[r] = fma_f16_f32(hi_half(th), n, acc[r]);
+                }
+            }
+        }
+    }
+}
+
+// A launch over several layers shares one set of tables built from x itself,
+// so the BSQ terms of a layer's protected columns (Eq. 10 replaces them) are
+// removed here: for the protected columns u0..u1 of slot w, acc[r] of row
+// row0 + r loses sum_s (+-n_s) * x_j.  One column per lane (all R rows and S
+// stages loaded at once); the warp sum of acc[r] then carries the total.
+template <int S, int R, int kCodeRow, int kNormRow>
+__device__ __forceinline__ void lut_protected(const unsigned char *cs, const unsigned char *ns,
+                                              int w, int row0, int lane, const int *pidx,
+                                              const float *xj, int u0, int u1, float (&acc)[R]) {
+    for (int u = u0 + lane; u < u1; u += 32) {
+        const int jc = pidx[u] - w * kLutSlotCols;   // column within the slot
+        if (jc < 0 || jc >= kLutSlotCols) continue;   // only for a list that is not ascending
+        const int ch = jc >> 3, e = jc & 7;
+        const float xv = xj[u];
+        uint32_t b[R][S];
+        uint16_t n[R][S];
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+#pragma unroll
+            for (int s = 0; s < S; ++s) {
+                b[r][s] = cs[(s * 16 + row0 + r) * kCodeRow + ch];
+                n[r][s] = *reinterpret_cast<const uint16_t *>(ns + (s * 16 + row0 + r) * kNormRow + 2 * ch);
+            }
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            float sum = 0.f;
+#pragma unroll
+            for (int s = 0; s < S; ++s) {
+                const float v = __half2float(__ushort_as_half(n[r][s]));
+                sum += ((b[r][s] >> e) & 1u) ? -v : v;
+            }
+            acc[r] = fmaf(-sum, xv, acc[r]);
+        }
+    }
+}
+
+// Sum of acc[r] over the warp's 32 lanes for r = 0, 1: afterwards every lane
+// holds the total of row bit4(lane).
+__device__ __forceinline__ float reduce_rows2(const float (&acc)[2], int lane) {
+    const bool h16 = (lane & 16) != 0;
+    float k = h16 ? acc[1] : acc[0];
+    k += __shfl_xor_sync(0xFFFFFFFFu, h16 ? acc[0] : acc[1], 16);
+    k += __shfl_xor_sync(0xFFFFFFFFu, k, 8);
+    k += __shfl_xor_sync(0xFFFFFFFFu, k, 4);
+    k += __shfl_xor_sync(0xFFFFFFFFu, k, 2);
+    k += __shfl_xor_sync(0xFFFFFFFFu, k, 1);
+    return k;
+}
+
 struct StreamLayer {
     float *y;
     const uint16_t *q8_scale;
     const int32_t *prot_idx;
     int N, p;
     int tile0;       // first tile of this layer in the launch's tile list
-    int q8_boxes;    // 128-column boxes of the int8 slab of one tile
+    const int8_t *q8;
+    int q8_pitch;    // bytes per row of q8 (p rounded up to 16), 0 without protection
 };
 
 template <int MAXG>
 struct StreamArgs {
-    CUtensorMap mc[MAXG], mn[MAXG], mq[MAXG];
+    CUtensorMap mc[MAXG], mn[MAXG];
     StreamLayer L[MAXG];
     const uint16_t *x;
     int *err;
     int K, B, G, ntiles, nslot;
-    int q8_boxes;    // the largest of the layers' (int8 double buffer size)
+    int q8_pitch;    // the largest of the layers' (int8 double buffer size)
     int pidx_cap, xt_pitch, mwords;
-    uint32_t off_xt, off_q8, off_red, off_bar, off_pidx, off_pmask, off_zero, off_prot;
+    int pblk;        // ints per layer in the protected-column block
+    uint32_t off_xt, off_q8, off_red, off_bar, off_pidx, off_pmask, off_zero, off_prot, off_tab;
 };
 
-template <int WQ, int WK, int S, int MAXG>
+// LUT: batch 1 through the nibble tables (x staged as tables, rows 4q..4q+3
+// per consumer warp); otherwise the MMA decode for batch <= 8.
+template <int WQ, int WK, int S, int MAXG, bool LUT>
 __global__ void __launch_bounds__((WQ * WK + 2) * 32, 2)
 k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
     constexpr int BM = 16;
@@ -604,9 +814,15 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
     constexpr int kNormRow = SW / 4;
     constexpr uint32_t kCodesBytes = S * BM * kCodeRow;
     constexpr uint32_t kSlotBytes = S * BM * (kCodeRow + kNormRow);
+    static_assert(!LUT || (SW == kLutSlotCols && NCW == 8), "table decode: 2048-column slots, 8 warps");
+    // table decode: every consumer warp takes every slot, two rows each; a
+    // launch of one layer masks its protected columns in the tables, a
+    // grouped launch shares unmasked tables and corrects per layer
+    constexpr int kLutRows = BM / NCW;
+    constexpr bool kLutMasked = (MAXG == 1);
 
     extern __shared__ unsigned char smem_raw[];
-    unsigned char *sm = aligned_smem(smem_raw);
+    unsigned char *sm = aligned_smem<128>(smem_raw);   // unswizzled boxes only
     const uint32_t sbase = smem_u32(sm);
     __shared__ int s_abort, s_lohi[MAXG][2];
     // layer descriptors, read with a run-time layer index: from shared memory
@@ -627,6 +843,7 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
     const int K = a.K, B = a.B, G = a.G, xt_pitch = a.xt_pitch, mwords = a.mwords;
     const uint32_t off_xt = a.off_xt, off_q8 = a.off_q8, off_zero = a.off_zero;
     const uint32_t off_pidx = a.off_pidx, off_pmask = a.off_pmask, off_prot = a.off_prot;
+    const int pblk = a.pblk;
     const uint16_t *const x = a.x;
     int *const err = a.err;
     int tile0[MAXG];
@@ -634,30 +851,31 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
     for (int i = 0; i < MAXG; ++i) tile0[i] = a.L[i].tile0;
     const CUtensorMap *const maps_c = &a.mc[0];
     const CUtensorMap *const maps_n = &a.mn[0];
-    const CUtensorMap *const maps_q = &a.mq[0];
     const int my_tiles = a.ntiles > cta ? (a.ntiles - 1 - cta) / Gd + 1 : 0;
     const int nwide = (K + SW - 1) / SW;
     const int nnar = (K + kSlab - 1) / kSlab;
     const int total = my_tiles * nwide;   // ring fills of this CTA
     const int nslot = a.nslot;
     const int cap = a.pidx_cap;
-    const uint32_t q8_buf_bytes = static_cast<uint32_t>(a.q8_boxes * BM * 128);
+    const uint32_t q8_buf_bytes = static_cast<uint32_t>(a.q8_pitch * BM);
     const uint32_t bar_full = sbase + a.off_bar;            // [nslot][WK]
     const uint32_t bar_empty = bar_full + 8 * nslot * WK;   // [nslot]
     const uint32_t bar_q8f = bar_empty + 8 * nslot;         // [2] int8 slab landed
-    const uint32_t bar_q8e = bar_q8f + 16;                  // [2] int8 slab consumed
-    const uint32_t bar_rf = bar_q8e + 16;                   // [2] tile partials written
+    const uint32_t bar_rf = bar_q8f + 32;                   // [2] tile partials written
     const uint32_t bar_re = bar_rf + 16;                    // [2] tile partials read
     const bool producer = (warp == NCW) && (lane == 0);
     const uint64_t pol = l2_evict_first_policy();
     float *red = reinterpret_cast<float *>(sm + a.off_red);   // [2][NCW][BM][B]
 
     // per-layer shared-memory views
-    auto pidx_of = [&](int g) {
-        return reinterpret_cast<int *>(sm + off_pidx) + g * (2 + B) * cap;
-    };
+    // per layer: indices, scales, scale * x [B][cap]; the table decode adds
+    // x of each protected column [cap] and the first protected column of
+    // every slot [nwide + 1]
+    auto pidx_of = [&](int g) { return reinterpret_cast<int *>(sm + off_pidx) + g * pblk; };
     auto pscale_of = [&](int g) { return reinterpret_cast<float *>(pidx_of(g) + cap); };
     auto xs_of = [&](int g) { return pscale_of(g) + cap; };
+    auto xj_of = [&](int g) { return xs_of(g) + B * cap; };
+    auto su_of = [&](int g) { return reinterpret_cast<int *>(xj_of(g) + cap); };
     auto pmask_of = [&](int g) {
         return reinterpret_cast<uint32_t *>(sm + off_pmask) + g * 2 * mwords;
     };
@@ -695,30 +913,32 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
         tma_load_3d_hint(dst, mc, bar, w * (SW / 8), cur_row0, 0, pol);
         tma_load_3d_hint(dst + kCodesBytes, mn, bar, w * (SW / 8), cur_row0, 0, pol);
     };
-    // the int8 slab of tile ii (a plain arrive when its layer has none)
+    // the int8 slab of tile ii (a plain arrive when its layer has none): the
+    // tile's rows of q8 are contiguous, one bulk copy (no tensor map)
     auto issue_q8 = [&](int ii) {
         const int g = layer_of(ii);
         const uint32_t bar = bar_q8f + 8 * (ii & 1);
-        const int boxes = s_L[g].q8_boxes;
-        if (boxes == 0) {
+        const int pitch = s_L[g].q8_pitch;
+        if (pitch == 0) {
             mbar_arrive(bar);
             return;
         }
+        const int row0 = row0_of(ii, g);
+        const int rows = min(BM, s_L[g].N - row0);
+        const uint32_t bytes = static_cast<uint32_t>(rows * pitch);
         const uint32_t dst = sbase + off_q8 + (ii & 1) * q8_buf_bytes;
-        mbar_arrive_expect_tx(bar, static_cast<uint32_t>(boxes * BM * 128));
-        for (int q = 0; q < boxes; ++q)
-            tma_load_2d_hint(dst + q * BM * 128, maps_q + g, bar, 128 * q, row0_of(ii, g), pol);
+        mbar_arrive_expect_tx(bar, bytes);
+        bulk_load(dst, s_L[g].q8 + static_cast<int64_t>(row0) * pitch, bytes, bar);
     };
 
-    int issued = 0, q8_issued = 0;
+    int issued = 0;
     if (producer) {
         for (int i = 0; i < nslot; ++i) {
             for (int k = 0; k < WK; ++k) mbar_init(bar_full + 8 * (i * WK + k), 1);
-            mbar_init(bar_empty + 8 * i, WQ);
+            mbar_init(bar_empty + 8 * i, LUT ? NCW : WQ);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar_q8f + 8 * i, 1);
-            mbar_init(bar_q8e + 8 * i, 1);
             mbar_init(bar_rf + 8 * i, NCW);
             mbar_init(bar_re + 8 * i, 1);
         }
@@ -728,11 +948,10 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
             prefetch_tmap(maps_c + g);
             prefetch_tmap(maps_n + g);
         }
-        for (; issued < total && issued < nslot; ++issued) {
-            // a tile's int8 slab goes out with its first slot (two buffers)
-            if (issued % nwide == 0 && issued / nwide < 2) issue_q8(q8_issued++);
-            issue_slot(issued);
-        }
+        // the first ring fills, then the int8 slabs of the first two tiles
+        // (two buffers; the reducer issues the rest as it frees them)
+        for (; issued < total && issued < nslot; ++issued) issue_slot(issued);
+        for (int t = 0; t < 2 && t < my_tiles; ++t) issue_q8(t);
         // activations: into L2 now, into the CTA after the wait
         for (int b = 0; b < B; ++b)
             prefetch_l2(x + static_cast<int64_t>(b) * K, static_cast<uint32_t>(K) * 2);
@@ -748,46 +967,85 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
         la.pidx_cap = cap;
         stage_protected_meta(la, 0, K, nnar * (kSlab / 32), pidx_of(warp), pscale_of(warp),
                              pmask_of(warp), pu_of(warp), s_lohi[warp]);
+        __syncwarp();
+        {
+            // scale * x halves past the layer's protected count are zero (the
+            // protected k tiles run to a multiple of 16); the staging after the
+            // wait writes the others
+            const int np = s_lohi[warp][1] - s_lohi[warp][0];
+            __half *xh = reinterpret_cast<__half *>(xs_of(warp));
+            for (int b = 0; b < B; ++b)
+                for (int u = np + lane; u < cap; u += 32) {
+                    xh[b * cap + u] = __float2half_rn(0.f);
+                    xh[(B + b) * cap + u] = __float2half_rn(0.f);
+                }
+        }
+        if constexpr (LUT) {
+            // protected columns before each slot (the masks live in the table
+            // area until the tables are built)
+            __syncwarp();
+            const int *pu = pu_of(warp);
+            int *su = su_of(warp);
+            const int np = s_lohi[warp][1] - s_lohi[warp][0];
+            for (int w = lane; w <= nwide; w += 32) su[w] = w < nwide ? pu[w * (kLutSlotCols / 32)] : np;
+        }
     }
     __syncthreads();
     pdl_launch_dependents();
 
     // activations may be written by the previous kernel
     pdl_wait();
-    {
+    if constexpr (LUT) {
+        // protected activations of every layer (flat list over layers), x and
+        // scale * x as fp16 hi + lo; the first blockDim.x are loaded before the
+        // table build so that both share one round trip to memory
+        auto protected_entry = [&](int e, int &g, int &u) {
+            for (g = 0; g < G; ++g) {
+                const int np = s_lohi[g][1] - s_lohi[g][0];
+                if (e < np) {
+                    u = e;
+                    return true;
+                }
+                e -= np;
+            }
+            return false;
+        };
+        auto store_protected = [&](int g, int u, float xv) {
+            const float sx = pscale_of(g)[u] * xv;
+            __half *xh = reinterpret_cast<__half *>(xs_of(g));
+            const __half hi = __float2half_rn(sx);
+            xh[u] = hi;
+            xh[cap + u] = __float2half_rn(sx - __half2float(hi));
+            xj_of(g)[u] = xv;
+        };
+        int g0 = 0, u0 = 0;
+        const bool has0 = protected_entry(threadIdx.x, g0, u0);
+        const float x0 = has0 ? bf16_bits_to_f32(x[pidx_of(g0)[u0]]) : 0.f;
+        build_nibble_tables(x, K, nwide * (kLutSlotCols / 8), kLutMasked ? pmask_of(0) : nullptr,
+                            sm + a.off_tab);
+        if (has0) store_protected(g0, u0, x0);
+        for (int e = threadIdx.x + blockDim.x;; e += blockDim.x) {
+            int g, u;
+            if (!protected_entry(e, g, u)) break;
+            store_protected(g, u, bf16_bits_to_f32(x[pidx_of(g)[u]]));
+        }
+    } else {
         StageView v[MAXG] = {};
 #pragma unroll
         for (int g = 0; g < MAXG; ++g)
             if (g < G) v[g] = {xt_of(g), pmask_of(g), pu_of(g), pscale_of(g), xs_of(g)};
-        stage_activations<MAXG>(x, K, B, 0, K, nnar, xt_pitch, cap, G, v);
+        stage_activations<MAXG, true>(x, K, B, 0, K, nnar, xt_pitch, cap, G, v);
+        for (int i = threadIdx.x; i < 1024 / 16; i += blockDim.x)
+            reinterpret_cast<uint4 *>(sm + off_zero)[i] = make_uint4(0, 0, 0, 0);
     }
-    for (int i = threadIdx.x; i < 1024 / 16; i += blockDim.x)
-        reinterpret_cast<uint4 *>(sm + off_zero)[i] = make_uint4(0, 0, 0, 0);
     __syncthreads();
 
     if (warp == NCW) {
         // ------------------------------------------------ producer: refill
         if (producer) {
-            // The int8 slab of tile ii (buffer ii & 1) goes out just before the
-            // tile's first slot, once tile ii-2 released the buffer; every slot
-            // of tile ii-1 is issued by then, so this never starves the decode.
-            auto issue_q8_upto = [&](int ii) -> bool {
-                while (q8_issued <= ii && q8_issued < my_tiles) {
-                    if (q8_issued >= 2 &&
-                        !mbar_wait(bar_q8e + 8 * (q8_issued & 1), ((q8_issued >> 1) - 1) & 1))
-                        return false;
-                    issue_q8(q8_issued);
-                    ++q8_issued;
-                }
-                return true;
-            };
             bool ok = true;
             for (; issued < total; ++issued) {
                 const int slot = issued % nslot;
-                if (issued % nwide == 0 && !issue_q8_upto(issued / nwide)) {
-                    ok = false;
-                    break;
-                }
                 if (!mbar_wait(bar_empty + 8 * slot, ((issued / nslot) - 1) & 1)) {
                     ok = false;
                     break;
@@ -795,8 +1053,6 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
                 if (*reinterpret_cast<volatile int *>(&s_abort)) break;
                 issue_slot(issued);
             }
-            if (ok && !*reinterpret_cast<volatile int *>(&s_abort) && !issue_q8_upto(my_tiles - 1))
-                ok = false;
             if (!ok) {
                 latch_error(err, BISCO_ERR_TIMEOUT);
                 atomicExch(&s_abort, 1);
@@ -804,18 +1060,17 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
             // every copy issued has landed before this thread leaves
             for (int gi = (issued > nslot ? issued - nslot : 0); gi < issued; ++gi)
                 mbar_wait(full_bar(gi), full_parity(gi));
-            for (int ii = (q8_issued > 2 ? q8_issued - 2 : 0); ii < q8_issued; ++ii)
-                mbar_wait(bar_q8f + 8 * (ii & 1), (ii >> 1) & 1);
         }
     } else if (warp == NCW + 1) {
         // ------------------------------------------- reducer: protected + y
         const int gq = lane >> 2, t = lane & 3;
         const int8_t *q8base = reinterpret_cast<const int8_t *>(sm + off_q8);
         float *prot = reinterpret_cast<float *>(sm + off_prot);   // [BM][BP]
-        for (int ii = 0; ii < my_tiles; ++ii) {
+        int ii = 0;
+        for (; ii < my_tiles; ++ii) {
             if (*reinterpret_cast<volatile int *>(&s_abort)) break;
             const int g = layer_of(ii);
-            float accp[1][4] = {{0.f, 0.f, 0.f, 0.f}};
+            float accp[4] = {0.f, 0.f, 0.f, 0.f};
             if (!mbar_wait_all(bar_q8f + 8 * (ii & 1), (ii >> 1) & 1)) {
                 if (lane == 0) {
                     latch_error(err, BISCO_ERR_TIMEOUT);
@@ -824,13 +1079,18 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
                 break;
             }
             const int pg = s_L[g].p;
+            const __half *xsh = reinterpret_cast<const __half *>(xs_of(g)), *xsl = xsh + B * cap;
+            const int8_t *slab = q8base + (ii & 1) * q8_buf_bytes;
             for (int u16 = 0; u16 < pg; u16 += 16)
-                protected_tile<BM, 1>(q8base + (ii & 1) * q8_buf_bytes, 0, u16, pg, gq, gq + 8, gq,
-                                      t, xs_of(g), cap, B, accp);
+                protected_rows(slab, s_L[g].q8_pitch, u16, gq, t, xsh, xsl, cap, B, accp);
             __syncwarp();
-            if (lane == 0) mbar_arrive(bar_q8e + 8 * (ii & 1));
+            // buffer ii & 1 is free: the slab of tile ii + 2 goes into it
+            if (lane == 0 && ii + 2 < my_tiles) {
+                fence_proxy_async_smem();
+                issue_q8(ii + 2);
+            }
 #pragma unroll
-            for (int e = 0; e < 4; ++e) prot[(e < 2 ? gq : gq + 8) * BP + 2 * t + (e & 1)] = accp[0][e];
+            for (int e = 0; e < 4; ++e) prot[(e < 2 ? gq : gq + 8) * BP + 2 * t + (e & 1)] = accp[e];
             __syncwarp();
             if (!mbar_wait_all(bar_rf + 8 * (ii & 1), (ii >> 1) & 1)) {
                 if (lane == 0) {
@@ -845,13 +1105,65 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
             for (int e = lane; e < B * BM; e += 32) {
                 const int b = e / BM, r = e - b * BM;
                 float v = 0.f;
+                // table decode: one partial per row; MMA decode: one per warp
 #pragma unroll
-                for (int wq = 0; wq < NCW; ++wq) v += rb[(wq * BM + r) * B + b];
+                for (int wq = 0; wq < (LUT ? 1 : NCW); ++wq) v += rb[(wq * BM + r) * B + b];
                 v += prot[r * BP + b];
                 if (row0 + r < N) y[static_cast<int64_t>(b) * N + row0 + r] = v;
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_re + 8 * (ii & 1));
+        }
+        // the slabs of the two tiles after the last one consumed (issued by the
+        // prologue or above) have landed before this warp leaves
+        if (lane == 0)
+            for (int t2 = ii; t2 < my_tiles && t2 < ii + 2; ++t2)
+                mbar_wait(bar_q8f + 8 * (t2 & 1), (t2 >> 1) & 1);
+    } else if constexpr (LUT) {
+        // --------------------------------- consumers: table decode, batch 1
+        const int row0 = warp * kLutRows;
+        const uint32_t tab = sbase + a.off_tab;
+        for (int ii = 0; ii < my_tiles; ++ii) {
+            if (*reinterpret_cast<volatile int *>(&s_abort)) break;
+            const int g = layer_of(ii);
+            const int *pidx = pidx_of(g), *su = su_of(g);
+            const float *xj = xj_of(g);
+            float acc[kLutRows] = {};
+            bool ok = true;
+            for (int w = 0; w < nwide; ++w) {
+                const int gidx = ii * nwide + w;
+                if (!mbar_wait_all(full_bar(gidx), full_parity(gidx)) ||
+                    __any_sync(0xFFFFFFFFu, *reinterpret_cast<volatile int *>(&s_abort) != 0)) {
+                    ok = false;
+                    break;
+                }
+                const unsigned char *cs = sm + (gidx % nslot) * kSlotBytes;
+                lut_slot<S, kLutRows, kCodeRow, kNormRow>(smem_u32(cs), smem_u32(cs) + kCodesBytes, tab,
+                                                          w, row0, lane, acc);
+                if constexpr (!kLutMasked) {
+                    const int u0 = su[w], u1 = su[w + 1];
+                    if (u1 > u0)
+                        lut_protected<S, kLutRows, kCodeRow, kNormRow>(cs, cs + kCodesBytes, w, row0, lane,
+                                                                       pidx, xj, u0, u1, acc);
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar_empty + 8 * (gidx % nslot));
+            }
+            if (ok && ii >= 2 && !mbar_wait_all(bar_re + 8 * (ii & 1), ((ii >> 1) - 1) & 1)) ok = false;
+            if (!ok) {
+                if (lane == 0) {
+                    latch_error(err, BISCO_ERR_TIMEOUT);
+                    atomicExch(&s_abort, 1);
+                }
+                break;
+            }
+            const float v = reduce_rows2(acc, lane);
+            if ((lane & 15) == 0) {
+                float *rb = red + (ii & 1) * NCW * BM * B;
+                rb[row0 + (lane >> 4)] = v * kInvSqrt8;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_rf + 8 * (ii & 1));
         }
     } else {
         // ----------------------------------------------- consumers: decode
@@ -1059,28 +1371,52 @@ size_t cluster_smem(int wm, int wq, int ck, int S, int B, int p, int wide_per_ra
 }
 
 // Shared memory of k_gemv_stream for G layers (largest protected count
-// p_max, largest int8 slab q8_boxes).
+// p_max, largest int8 row pitch q8_pitch).  The table decode (lut) keeps nibble
+// tables of x instead of staged fp16 copies.  A grouped launch (MAXG > 1)
+// keeps the protected-column masks of its prologue as scratch in the table
+// area, built over afterwards; a single layer's tables are built from the
+// masks, which therefore get their own area.
 template <int MAXG>
-size_t stream_smem(int wq, int wk, int S, int B, int K, int G, int p_max, int q8_boxes, int nslot,
-                   StreamArgs<MAXG> *a) {
+size_t stream_smem(int wq, int wk, int S, int B, int K, int G, int p_max, int q8_pitch, int nslot,
+                   bool lut, StreamArgs<MAXG> *a) {
     const int BM = 16, BP = 8, SW = kSlab * wq;
     const int nar = (K + kSlab - 1) / kSlab;
+    const int nwide = (K + SW - 1) / SW;
     a->pidx_cap = static_cast<int>(align_up(static_cast<size_t>(p_max), 16));
     a->mwords = nar * (kSlab / 32);
+    // indices, scales, scale * x [B]; the table decode adds x and slot starts
+    a->pblk = lut ? (3 + B) * a->pidx_cap + static_cast<int>(align_up(nwide + 1, 4))
+                  : (2 + B) * a->pidx_cap;
     size_t off = static_cast<size_t>(nslot) * S * BM * (SW / 8 + SW / 4);
-    a->off_xt = static_cast<uint32_t>(off);
-    a->xt_pitch = nar * 1024 + 64;   // +64 B: rows g and g+1 land in different banks
-    off += static_cast<size_t>(G) * B * a->xt_pitch;
+    if (lut) {
+        a->off_tab = static_cast<uint32_t>(off);
+        a->off_pmask = static_cast<uint32_t>(off);   // G * 2 * mwords words <= K bytes
+        a->off_xt = a->off_zero = 0;
+        a->xt_pitch = 0;
+        off += static_cast<size_t>(nwide) * kLutSlotBytes;
+        if (MAXG == 1) {
+            a->off_pmask = static_cast<uint32_t>(off);
+            off += static_cast<size_t>(2) * a->mwords * 4;
+        }
+    } else {
+        a->off_tab = 0;
+        a->off_xt = static_cast<uint32_t>(off);
+        a->xt_pitch = nar * 1024 + 64;   // +64 B: rows g and g+1 land in different banks
+        off += static_cast<size_t>(G) * B * a->xt_pitch;
+    }
     off = align_up(off, 128);
     a->off_q8 = static_cast<uint32_t>(off);
-    off += static_cast<size_t>(2) * q8_boxes * BM * 128;
+    off += static_cast<size_t>(2) * q8_pitch * BM;
     a->off_pidx = static_cast<uint32_t>(off);
-    off += static_cast<size_t>(G) * (2 + B) * a->pidx_cap * 4;   // indices, scales, scale * x
-    a->off_pmask = static_cast<uint32_t>(off);
-    off += static_cast<size_t>(G) * 2 * a->mwords * 4;           // masks, prefix counts
+    off += static_cast<size_t>(G) * a->pblk * 4;
+    if (!lut) {
+        a->off_pmask = static_cast<uint32_t>(off);
+        off += static_cast<size_t>(G) * 2 * a->mwords * 4;       // masks, prefix counts
+        off = align_up(off, 16);
+        a->off_zero = static_cast<uint32_t>(off);
+        off += 1024;
+    }
     off = align_up(off, 16);
-    a->off_zero = static_cast<uint32_t>(off);
-    off += 1024;
     a->off_red = static_cast<uint32_t>(off);
     off += static_cast<size_t>(2) * wq * wk * BM * B * 4;   // partials of the B rows
     a->off_prot = static_cast<uint32_t>(off);
@@ -1088,7 +1424,7 @@ size_t stream_smem(int wq, int wk, int S, int B, int K, int G, int p_max, int q8
     off = align_up(off, 8);
     a->off_bar = static_cast<uint32_t>(off);
     off += static_cast<size_t>(nslot * (wk + 1) + 8) * 8;
-    return off + 1024;   // slack for the 1024-byte aligned base
+    return off + 128;   // slack for the 128-byte aligned base
 }
 
 // k_gemv tiling rule: 2048-column slots (four column-quarter warps per row
@@ -1163,9 +1499,9 @@ bisco_status launch_w(bool two, int S, const CUtensorMap &mc, const CUtensorMap 
     return launch_s<WM, WQ, 1>(S, mc, mn, mq, a, ck, smem, stream);
 }
 
-template <int WQ, int WK, int S, int MAXG>
+template <int WQ, int WK, int S, int MAXG, bool LUT>
 bisco_status launch_stream_t(const StreamArgs<MAXG> &a, int grid, size_t smem, cudaStream_t stream) {
-    auto kern = k_gemv_stream<WQ, WK, S, MAXG>;
+    auto kern = k_gemv_stream<WQ, WK, S, MAXG, LUT>;
     static size_t configured[64] = {};
     if (!set_smem(kern, smem, configured)) return BISCO_ERR_CUDA;
     cudaLaunchConfig_t cfg = {};
@@ -1225,6 +1561,9 @@ bisco_status launch_stream_g(const bisco_layer *Ls, int G, const uint16_t *x, in
                              float *const *y, int *err, int sms, cudaStream_t stream, bool *launched) {
     constexpr int WQ = 4, WK = 2;
     const int K = Ls[0].k_in, S = Ls[0].stages;
+    // batch 1 decodes through nibble tables of x unless BISCO_GEMV_LUT=0
+    const char *lut_env = getenv("BISCO_GEMV_LUT");
+    const bool lut = B == 1 && !(lut_env && lut_env[0] == '0');
     *launched = false;
     StreamArgs<MAXG> a = {};
     a.x = x;
@@ -1242,13 +1581,14 @@ bisco_status launch_stream_g(const bisco_layer *Ls, int G, const uint16_t *x, in
         sl.N = L.n_out;
         sl.p = L.n_protected;
         sl.tile0 = tiles;
-        sl.q8_boxes = L.n_protected > 0 ? ((L.n_protected + 15) / 16 * 16 + 127) / 128 : 0;
+        sl.q8 = L.q8;
+        sl.q8_pitch = L.n_protected > 0 ? (L.n_protected + 15) / 16 * 16 : 0;
         tiles += (L.n_out + 15) / 16;
         p_max = p_max > sl.p ? p_max : sl.p;
-        q8_max = q8_max > sl.q8_boxes ? q8_max : sl.q8_boxes;
+        q8_max = q8_max > sl.q8_pitch ? q8_max : sl.q8_pitch;
     }
     a.ntiles = tiles;
-    a.q8_boxes = q8_max;
+    a.q8_pitch = q8_max;
     const size_t slot = static_cast<size_t>(S) * 16 * (kSlab * WQ / 8 + kSlab * WQ / 4);
     int nslot = 0;
     if (const char *e = getenv("BISCO_GEMV_NSLOT")) nslot = atoi(e);
@@ -1256,22 +1596,31 @@ bisco_status launch_stream_g(const bisco_layer *Ls, int G, const uint16_t *x, in
         // at least three slots: with two, the refills of a long launch are
         // exposed (measured -15 % on the S = 3 MLP shapes), which costs more
         // than sharing the SM with the next kernel gains
-        nslot = fit_slots(stream_smem(WQ, WK, S, B, K, G, p_max, q8_max, 0, &a), slot, kCoresident,
-                          3, 8);
-        if (stream_smem(WQ, WK, S, B, K, G, p_max, q8_max, nslot, &a) > kMaxSmem) nslot = 2;
+        nslot = fit_slots(stream_smem(WQ, WK, S, B, K, G, p_max, q8_max, 0, lut, &a), slot,
+                          kCoresident, 3, 8);
+        if (stream_smem(WQ, WK, S, B, K, G, p_max, q8_max, nslot, lut, &a) > kMaxSmem) nslot = 2;
     }
-    const size_t smem = stream_smem(WQ, WK, S, B, K, G, p_max, q8_max, nslot, &a);
+    const size_t smem = stream_smem(WQ, WK, S, B, K, G, p_max, q8_max, nslot, lut, &a);
     if (smem > kMaxSmem) return BISCO_OK;
     a.nslot = nslot;
-    for (int g = 0; g < G; ++g)
-        if (!layer_maps(Ls[g], 16, kSlab * WQ, false, &a.mc[g], &a.mn[g], &a.mq[g]))
+    for (int g = 0; g < G; ++g) {
+        CUtensorMap unused_q8;   // the int8 slab goes by bulk copy
+        if (!layer_maps(Ls[g], 16, kSlab * WQ, false, &a.mc[g], &a.mn[g], &unused_q8))
             return BISCO_ERR_CUDA;
+    }
     const int grid = tiles < sms ? tiles : sms;
     *launched = true;
+    if (lut) {
+        switch (S) {
+            case 1: return launch_stream_t<WQ, WK, 1, MAXG, true>(a, grid, smem, stream);
+            case 2: return launch_stream_t<WQ, WK, 2, MAXG, true>(a, grid, smem, stream);
+            default: return launch_stream_t<WQ, WK, 3, MAXG, true>(a, grid, smem, stream);
+        }
+    }
     switch (S) {
-        case 1: return launch_stream_t<WQ, WK, 1, MAXG>(a, grid, smem, stream);
-        case 2: return launch_stream_t<WQ, WK, 2, MAXG>(a, grid, smem, stream);
-        default: return launch_stream_t<WQ, WK, 3, MAXG>(a, grid, smem, stream);
+        case 1: return launch_stream_t<WQ, WK, 1, MAXG, false>(a, grid, smem, stream);
+        case 2: return launch_stream_t<WQ, WK, 2, MAXG, false>(a, grid, smem, stream);
+        default: return launch_stream_t<WQ, WK, 3, MAXG, false>(a, grid, smem, stream);
     }
 }
 

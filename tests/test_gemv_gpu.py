@@ -207,3 +207,79 @@ def test_gemv_multi_single_layer_matches_gemv(env):
     y = run_gemv(env, Lref, X)
     assert max_rel_rows(ym, y) <= 1e-5
     assert max_rel_rows(ym, oracle.gemv(Lref, X)) <= TOL
+
+
+# ---------------------------------------------------------------- batch 1
+# Batch 1 decodes through nibble tables of x: a launch of one layer builds
+# them with its protected columns masked, a grouped launch shares unmasked
+# tables and removes each layer's protected BSQ terms afterwards.  Both are
+# checked where the layout has edges: protected columns on chunk and ring-slot
+# boundaries (2048-column slots), whole protected chunks, K not a slot multiple.
+
+def _boosted(N, K, cols, seed, S_dist="normal"):
+    """Weights whose protected set (Eq. 8 top-p) is exactly `cols`."""
+    W = synth.layer_weights(N, K, seed=seed, dist=S_dist, n_outliers=0)
+    w = synth.bf16_bits_to_f32(W).astype(np.float64)
+    w[:, cols] *= 50.0
+    return synth.f32_to_bf16_bits(w.astype(np.float32))
+
+
+BOUNDARY_COLS = [0, 7, 8, 15, 2040, 2041, 2042, 2043, 2044, 2045, 2046, 2047, 2048, 2055, 4095]
+
+
+@pytest.mark.parametrize("K,S", [(4096, 2), (4096, 3), (2176, 2)])
+def test_gemv_table_decode_protected_on_boundaries(env, K, S):
+    cols = [c for c in BOUNDARY_COLS if c < K]
+    Lref = oracle.encode(_boosted(2500, K, cols, seed=80 + K), S=S, p=len(cols))
+    assert sorted(Lref["idx"].tolist()) == cols
+    X = synth.activations(1, K, seed=81)
+    y = run_gemv(env, Lref, X)
+    assert max_rel_rows(y, oracle.gemv(Lref, X)) <= TOL
+
+
+def test_gemv_table_decode_grouped_correction_on_boundaries(env):
+    """Grouped launch: shared unmasked tables, per-layer correction of the
+    protected BSQ terms, with protected sets that differ between layers."""
+    K, S = 4096, 2
+    sets = [BOUNDARY_COLS, [1, 2047, 2049, 3000], []]
+    Lrefs = []
+    for i, cols in enumerate(sets):
+        W = _boosted(400 + 300 * i, K, cols, seed=90 + i) if cols else \
+            synth.layer_weights(400 + 300 * i, K, seed=90 + i)
+        Lrefs.append(oracle.encode(W, S=S, p=len(cols)))
+    X = synth.activations(1, K, seed=93)
+    ys = _multi(env, Lrefs, X)
+    for y, L in zip(ys, Lrefs):
+        assert max_rel_rows(y, oracle.gemv(L, X)) <= TOL
+
+
+def test_gemv_multi_fully_protected_layer(env):
+    """A layer with every column protected (its tables are all correction)
+    next to an unprotected one, batch 1."""
+    K, S = 512, 2
+    Lrefs = [oracle.encode(synth.layer_weights(300, K, seed=95), S=S, p=K),
+             oracle.encode(synth.layer_weights(200, K, seed=96), S=S, p=0)]
+    X = synth.activations(1, K, seed=97)
+    ys = _multi(env, Lrefs, X)
+    for y, L in zip(ys, Lrefs):
+        assert max_rel_rows(y, oracle.gemv(L, X)) <= TOL
+
+
+@pytest.mark.parametrize("N,K,S,p", [(2500, 4096, 2, 41), (2500, 2176, 3, 23), (300, 1024, 1, 11)])
+def test_gemv_batch1_both_decodes(env, N, K, S, p):
+    """Batch 1 through the table decode and through the MMA decode
+    (BISCO_GEMV_LUT=0) on the streaming kernel: both meet the bar."""
+    W = synth.layer_weights(N, K, seed=N + K + S)
+    X = synth.activations(1, K, seed=98)
+    Lref = oracle.encode(W, S=S, p=p)
+    ref = oracle.gemv(Lref, X)
+    for lut in ("1", "0"):
+        y = run_gemv(env, Lref, X, extra_env={"BISCO_GEMV_MODE": "stream", "BISCO_GEMV_LUT": lut})
+        assert max_rel_rows(y, ref) <= TOL, lut
+
+
+def test_gemv_batch1_zero_activations(env):
+    N, K, S, p = 2500, 2048, 2, 21
+    Lref = oracle.encode(synth.layer_weights(N, K, seed=99), S=S, p=p)
+    y = run_gemv(env, Lref, np.zeros((1, K), np.uint16))
+    assert np.all(y == 0)
