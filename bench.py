@@ -76,16 +76,26 @@ def tensor_peaks():
         return 1900.0, 1700.0, "fallback"
 
 
-# DRAM bytes (read + write) of one q_proj/o_proj launch of the dominant
-# kernel, from the ncu capture summarised in profiles/ (see the file for the
-# command), valid while the kernel source hashes to the recorded digest.
-DOMINANT_TRAFFIC = {"bytes": 19249664, "gemv_cu_sha256": "319eee6a6187726e1bc7dcce12ef98c71080af17a61c17dbfed7917f3f2f9b63",
+# DRAM bytes (read + write) of one grouped q/k/v launch of the dominant
+# kernel (batch 1, table-lookup decode), from the ncu capture summarised in
+# profiles/ (the file gives the command), valid while the kernel source
+# hashes to the recorded digest.
+DOMINANT_TRAFFIC = {"bytes": 19243008, "gemv_cu_sha256": "d37a2f84c70aee3cee6969395324d54d35f492f0b452245f658e42e5539cbcb4",
                     "profile": "profiles/k_gemv_stream_qkv_group_b1.md"}
 
 
-def dominant_traffic():
+def decode_kind(B):
+    """Template flag and name of the streaming kernel's decode for batch B."""
+    table = B == 1 and os.environ.get("BISCO_GEMV_LUT", "1")[:1] != "0"
+    return ("1", "table-lookup decode") if table else ("0", "mma decode")
+
+
+def dominant_traffic(B, grouped):
+    """DRAM bytes of one dominant launch from the committed ncu capture, or None
+    when the capture does not describe the kernel being timed (another
+    gemv.cu, batch, decode or launch grouping)."""
     import hashlib
-    if DOMINANT_TRAFFIC["bytes"] is None:
+    if DOMINANT_TRAFFIC["bytes"] is None or B != 1 or not grouped or decode_kind(B)[0] != "1":
         return None
     with open(os.path.join(ROOT, "paper_2607_08643_gb300", "csrc", "gemv.cu"), "rb") as f:
         digest = hashlib.sha256(f.read()).hexdigest()
@@ -334,12 +344,13 @@ def run_bisco(args, rank, world, local_rank):
         value=gbs, ms_per_step=ms_step, tokens_per_s=tok_s, bytes_per_step=bytes_step,
         launches=launches, e2e_gbs=e2e_gbs, h2d=x_dev.numel() * 2, d2h=y_total * 4,
         roofline={"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                  "frac": achieved / peak, "traffic": dominant_traffic(),
+                  "frac": achieved / peak, "traffic": dominant_traffic(B, not args.ungrouped),
                   "peak_source": "%s hbm_gbs (MEASURED_PEAKS.json, copy burst)" % peak_kind
                   if peak_kind == "measured" else "fallback 6.8 TB/s",
-                  "kernel": ("k_gemv_stream<4,2,2> (bisco_gemv, q_proj/o_proj 4096x4096, batch %d)"
+                  "kernel": ("k_gemv_stream<4,2,2,1,%s> (bisco_gemv, q_proj/o_proj 4096x4096, batch %d, %s)"
                              if args.ungrouped else
-                             "k_gemv_stream<4,2,2> (bisco_gemv_multi, q+k+v 6144x4096, batch %d)") % B,
+                             "k_gemv_stream<4,2,2,4,%s> (bisco_gemv_multi, q+k+v 6144x4096, batch %d, %s)")
+                            % (decode_kind(B)[0], B, decode_kind(B)[1]),
                   "bytes_per_launch": bytes_dom, "us_per_launch": us_dom,
                   "launches_timed": args.steps * len(dom_calls)},
         clocks=clk, ms_e2e=ms_e2e / args.steps)
