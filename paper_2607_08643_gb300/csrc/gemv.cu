@@ -1668,32 +1668,57 @@ bisco_status launch_gemv(const bisco_layer &L, const uint16_t *x, int B, float *
         if (launched || st != BISCO_OK) return st;
     }
 
-    Plan pl = choose_plan(N, K, B);
-    plan_override(&pl);
-    if (B > 8 && pl.wm < 2) pl = {2, pl.wq, pl.ck, pl.nslot};
-    if (!tiling_known(pl.wm, pl.wq)) pl = {2, 4, pl.ck, pl.nslot};
-    const int BM = 16 * pl.wm;
-    const int SW = kSlab * pl.wq;
-    const int total_wide = (K + SW - 1) / SW;
-    if (pl.ck > total_wide) pl.ck = total_wide;
-    const size_t slot = static_cast<size_t>(S) * BM * (SW / 8 + SW / 4);
-    // split K further until the staged activations and a 2-slot ring fit
+    // k_gemv plan: the preferred tiling (or BISCO_GEMV_PLAN), then smaller
+    // ones; for each, split K further until the staged activations and a
+    // 2-slot ring fit (at batch 9..16 the activations alone are 16 rows of
+    // K fp16, so large K needs narrow slots and wide splits)
+    Plan first = choose_plan(N, K, B);
+    const bool forced = plan_override(&first);
+    if (B > 8 && first.wm < 2) first = {2, first.wq, first.ck, first.nslot};
+    if (!tiling_known(first.wm, first.wq)) first = {2, 4, first.ck, first.nslot};
+    Plan cands[1 + sizeof(kTilings) / sizeof(kTilings[0])];
+    int ncand = 0;
+    cands[ncand++] = first;
+    if (!forced) {
+        // fallbacks, largest row block first (two MMA n-tiles need WM >= 2)
+        static const int order[][2] = {{4, 4}, {2, 4}, {4, 2}, {2, 2}, {1, 4}, {1, 2}, {4, 1}, {8, 1}};
+        for (const auto &t : order) {
+            if (B > 8 && t[0] < 2) continue;
+            if (t[0] == first.wm && t[1] == first.wq) continue;
+            cands[ncand++] = {t[0], t[1], 1, 0};
+        }
+    }
+    Plan pl = {};
     int wpr = 0, nslot = 0;
     size_t smem = 0;
-    for (;;) {
-        wpr = (total_wide + pl.ck - 1) / pl.ck;
-        nslot = pl.nslot;
-        if (nslot <= 0) {
-            nslot = fit_slots(cluster_smem(pl.wm, pl.wq, pl.ck, S, B, p, wpr, 0, &a), slot,
-                              kCoresident, 2, 8);
-            if (nslot > wpr && wpr >= 2) nslot = wpr;
+    bool fits = false;
+    for (int ci = 0; ci < ncand && !fits; ++ci) {
+        pl = cands[ci];
+        const int BMc = 16 * pl.wm, SWc = kSlab * pl.wq;
+        const int total_wide_c = (K + SWc - 1) / SWc;
+        if (pl.ck > total_wide_c) pl.ck = total_wide_c;
+        const size_t slot = static_cast<size_t>(S) * BMc * (SWc / 8 + SWc / 4);
+        for (;;) {
+            wpr = (total_wide_c + pl.ck - 1) / pl.ck;
+            nslot = pl.nslot;
+            if (nslot <= 0) {
+                nslot = fit_slots(cluster_smem(pl.wm, pl.wq, pl.ck, S, B, p, wpr, 0, &a), slot,
+                                  kCoresident, 2, 8);
+                if (nslot > wpr && wpr >= 2) nslot = wpr;
+            }
+            if (nslot < 2) nslot = 2;
+            smem = cluster_smem(pl.wm, pl.wq, pl.ck, S, B, p, wpr, nslot, &a);
+            if (smem <= kMaxSmem) {
+                fits = true;
+                break;
+            }
+            if (pl.ck >= 8 || pl.ck >= total_wide_c) break;
+            ++pl.ck;
         }
-        if (nslot < 2) nslot = 2;
-        smem = cluster_smem(pl.wm, pl.wq, pl.ck, S, B, p, wpr, nslot, &a);
-        if (smem <= kMaxSmem) break;
-        if (pl.ck >= 8 || pl.ck >= total_wide) return generic();   // e.g. p close to K
-        ++pl.ck;
     }
+    if (!fits) return generic();   // e.g. p close to K
+    const int BM = 16 * pl.wm;
+    const int SW = kSlab * pl.wq;
     a.wide_per_rank = wpr;
     a.nslot = nslot;
     CUtensorMap mc, mn, mq;
