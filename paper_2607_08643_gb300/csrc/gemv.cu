@@ -106,78 +106,95 @@ struct StageView {
 // round trip to memory.  Job = one 32-column group of one row.  Pair i of a
 // 32-column group is element i&7 of chunk (i>>3) and of chunk (i>>3)+2 --
 // bits i and i+16 of its code word, columns (i>>3)*8 + (i&7) and that + 16.
-template <int MAXG, bool kHalfXs = false>
+template <int MAXG, bool kHalfXs = false, int kBatch = 1>
 __device__ __forceinline__ void stage_activations(const uint16_t *x, int K, int B, int k_begin,
                                                   int cols, int nnar, int xt_pitch, int cap,
                                                   int G, const StageView (&v)[MAXG]) {
     const int groups_per_row = cols >> 5;   // cols % 128 == 0 on this path
     const int njobs = B * nnar * 16;
-    for (int e = threadIdx.x; e < njobs; e += blockDim.x) {
-        const int t = e & 3, w = (e >> 2) & 3, sb = e >> 4;
-        const int b = sb / nnar, slab = sb - b * nnar;
-        const int g32 = slab * 16 + t * 4 + w;
-        const int dst_off = b * xt_pitch + slab * 1024 + t * 16 + w * 256;
-        uint32_t o[16];
-        const uint16_t *src = x + static_cast<int64_t>(b) * K + k_begin + g32 * 32;
-        if (g32 < groups_per_row) {
-            uint32_t r[16];
+    const int nthr = static_cast<int>(blockDim.x);
+    // kBatch jobs per thread have their loads in flight together (one round
+    // trip to memory per batch; more than one job per batch measured no
+    // faster at batch 8..16)
+    for (int e0 = threadIdx.x; e0 < njobs; e0 += kBatch * nthr) {
+        uint32_t rr[kBatch][16];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const uint4 u4 = reinterpret_cast<const uint4 *>(src)[q];
-                r[4 * q] = u4.x; r[4 * q + 1] = u4.y; r[4 * q + 2] = u4.z; r[4 * q + 3] = u4.w;
+        for (int i = 0; i < kBatch; ++i) {
+            const int e = e0 + i * nthr;
+            const int t = e & 3, w = (e >> 2) & 3, sb = e >> 4;
+            const int b = sb / nnar, slab = sb - b * nnar;
+            const int g32 = slab * 16 + t * 4 + w;
+            if (e < njobs && g32 < groups_per_row) {
+                const uint16_t *src = x + static_cast<int64_t>(b) * K + k_begin + g32 * 32;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const uint4 u4 = reinterpret_cast<const uint4 *>(src)[q];
+                    rr[i][4 * q] = u4.x; rr[i][4 * q + 1] = u4.y; rr[i][4 * q + 2] = u4.z; rr[i][4 * q + 3] = u4.w;
+                }
+            } else {
+#pragma unroll
+                for (int q = 0; q < 16; ++q) rr[i][q] = 0u;
             }
-#pragma unroll
-            for (int i = 0; i < 16; ++i) {
-                // pair i: columns c0 = (i>>3)*8 + (i&7) (low half) and c0 + 16
-                const int c0 = (i >> 3) * 8 + (i & 7);
-                const uint32_t f = r[c0 >> 1], sw = r[(c0 + 16) >> 1];
-                const __half2 h = __floats2half2_rn((c0 & 1) ? bf16_hi(f) : bf16_lo(f),
-                                                    (c0 & 1) ? bf16_hi(sw) : bf16_lo(sw));
-                o[i] = *reinterpret_cast<const uint32_t *>(&h);
-            }
-        } else {
-#pragma unroll
-            for (int i = 0; i < 16; ++i) o[i] = 0u;
         }
 #pragma unroll
-        for (int g = 0; g < MAXG; ++g) {
-            if (g >= G) break;
-            uint32_t pm = g32 < groups_per_row ? v[g].pmask[g32] : 0u;
-            unsigned char *dst = v[g].xt + dst_off;
-            if (pm == 0u) {
+        for (int i = 0; i < kBatch; ++i) {
+            const int e = e0 + i * nthr;
+            if (e >= njobs) break;
+            const int t = e & 3, w = (e >> 2) & 3, sb = e >> 4;
+            const int b = sb / nnar, slab = sb - b * nnar;
+            const int g32 = slab * 16 + t * 4 + w;
+            const int dst_off = b * xt_pitch + slab * 1024 + t * 16 + w * 256;
+            const uint16_t *src = x + static_cast<int64_t>(b) * K + k_begin + g32 * 32;
+            uint32_t o[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                // pair j: columns c0 = (j>>3)*8 + (j&7) (low half) and c0 + 16
+                const int c0 = (j >> 3) * 8 + (j & 7);
+                const uint32_t f = rr[i][c0 >> 1], sw = rr[i][(c0 + 16) >> 1];
+                const __half2 h = __floats2half2_rn((c0 & 1) ? bf16_hi(f) : bf16_lo(f),
+                                                    (c0 & 1) ? bf16_hi(sw) : bf16_lo(sw));
+                o[j] = *reinterpret_cast<const uint32_t *>(&h);
+            }
+#pragma unroll
+            for (int g = 0; g < MAXG; ++g) {
+                if (g >= G) break;
+                uint32_t pm = g32 < groups_per_row ? v[g].pmask[g32] : 0u;
+                unsigned char *dst = v[g].xt + dst_off;
+                if (pm == 0u) {
+#pragma unroll
+                    for (int m = 0; m < 4; ++m)
+                        *reinterpret_cast<uint4 *>(dst + m * 64) =
+                            make_uint4(o[4 * m], o[4 * m + 1], o[4 * m + 2], o[4 * m + 3]);
+                    continue;
+                }
+                // protected columns of this group: record scale * x, zero the halves
+                const int u0 = v[g].pu[g32];   // protected columns before this group
+                for (uint32_t bits = pm; bits; bits &= bits - 1u) {
+                    const int k = __ffs(bits) - 1;
+                    const int u = u0 + __popc(pm & ((1u << k) - 1u));
+                    const float sx = v[g].pscale[u] * bf16_bits_to_f32(src[k]);
+                    if constexpr (kHalfXs) {
+                        __half *xh = reinterpret_cast<__half *>(v[g].xs);
+                        const __half hi = __float2half_rn(sx);
+                        xh[b * cap + u] = hi;
+                        xh[(B + b) * cap + u] = __float2half_rn(sx - __half2float(hi));
+                    } else {
+                        v[g].xs[b * cap + u] = sx;
+                    }
+                }
+                uint32_t om[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                    const int c0 = (j >> 3) * 8 + (j & 7);
+                    const uint32_t keep = (((pm >> c0) & 1u) ? 0u : 0x0000FFFFu) |
+                                          (((pm >> (c0 + 16)) & 1u) ? 0u : 0xFFFF0000u);
+                    om[j] = o[j] & keep;
+                }
 #pragma unroll
                 for (int m = 0; m < 4; ++m)
                     *reinterpret_cast<uint4 *>(dst + m * 64) =
-                        make_uint4(o[4 * m], o[4 * m + 1], o[4 * m + 2], o[4 * m + 3]);
-                continue;
+                        make_uint4(om[4 * m], om[4 * m + 1], om[4 * m + 2], om[4 * m + 3]);
             }
-            // protected columns of this group: record scale * x, zero the halves
-            const int u0 = v[g].pu[g32];   // protected columns before this group
-            for (uint32_t bits = pm; bits; bits &= bits - 1u) {
-                const int k = __ffs(bits) - 1;
-                const int u = u0 + __popc(pm & ((1u << k) - 1u));
-                const float sx = v[g].pscale[u] * bf16_bits_to_f32(src[k]);
-                if constexpr (kHalfXs) {
-                    __half *xh = reinterpret_cast<__half *>(v[g].xs);
-                    const __half hi = __float2half_rn(sx);
-                    xh[b * cap + u] = hi;
-                    xh[(B + b) * cap + u] = __float2half_rn(sx - __half2float(hi));
-                } else {
-                    v[g].xs[b * cap + u] = sx;
-                }
-            }
-            uint32_t om[16];
-#pragma unroll
-            for (int i = 0; i < 16; ++i) {
-                const int c0 = (i >> 3) * 8 + (i & 7);
-                const uint32_t keep = (((pm >> c0) & 1u) ? 0u : 0x0000FFFFu) |
-                                      (((pm >> (c0 + 16)) & 1u) ? 0u : 0xFFFF0000u);
-                om[i] = o[i] & keep;
-            }
-#pragma unroll
-            for (int m = 0; m < 4; ++m)
-                *reinterpret_cast<uint4 *>(dst + m * 64) =
-                    make_uint4(om[4 * m], om[4 * m + 1], om[4 * m + 2], om[4 * m + 3]);
         }
     }
 }
@@ -277,27 +294,33 @@ __device__ __forceinline__ void protected_tile(const int8_t *q8s, int col0, int 
     }
 }
 
-// Protected k tile u16..u16+15 of rows g and g + 8 (Eq. 10), batch column g
-// of the MMA: q8 from a tile slab of rows of `pitch` bytes (16-bit loads of
-// column pairs, exact int8 -> fp16), scale * x as fp16 hi + lo halves
-// xsh/xsl [B][cap], zero past the layer's p, so no bounds checks.
+// Protected k tile u16..u16+15 of rows g and g + 8 (Eq. 10), batch columns
+// nt * 8 + g of the MMA n-tiles: q8 from a tile slab of rows of `pitch`
+// bytes (16-bit loads of column pairs, exact int8 -> fp16), scale * x as fp16
+// hi + lo halves xsh/xsl [B][cap], zero past the layer's p, so no bounds
+// checks.
+template <int NT>
 __device__ __forceinline__ void protected_rows(const int8_t *q8s, int pitch, int u16, int g, int t,
                                                const __half *xsh, const __half *xsl, int cap, int B,
-                                               float (&acc)[4]) {
+                                               float (&acc)[NT][4]) {
     const int u0 = u16 + 2 * t;
     auto pair = [&](int r, int u) {
         return i8x2_to_h2(*reinterpret_cast<const uint16_t *>(q8s + r * pitch + u));
     };
     const uint32_t af[4] = {pair(g, u0), pair(g + 8, u0), pair(g, u0 + 8), pair(g + 8, u0 + 8)};
-    uint32_t h0 = 0u, h1 = 0u, l0 = 0u, l1 = 0u;
-    if (g < B) {
-        h0 = *reinterpret_cast<const uint32_t *>(xsh + g * cap + u0);
-        h1 = *reinterpret_cast<const uint32_t *>(xsh + g * cap + u0 + 8);
-        l0 = *reinterpret_cast<const uint32_t *>(xsl + g * cap + u0);
-        l1 = *reinterpret_cast<const uint32_t *>(xsl + g * cap + u0 + 8);
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+        const int bg = nt * 8 + g;
+        uint32_t h0 = 0u, h1 = 0u, l0 = 0u, l1 = 0u;
+        if (bg < B) {
+            h0 = *reinterpret_cast<const uint32_t *>(xsh + bg * cap + u0);
+            h1 = *reinterpret_cast<const uint32_t *>(xsh + bg * cap + u0 + 8);
+            l0 = *reinterpret_cast<const uint32_t *>(xsl + bg * cap + u0);
+            l1 = *reinterpret_cast<const uint32_t *>(xsl + bg * cap + u0 + 8);
+        }
+        mma_16816(acc[nt], af, h0, h1);
+        mma_16816(acc[nt], af, l0, l1);
     }
-    mma_16816(acc, af, h0, h1);
-    mma_16816(acc, af, l0, l1);
 }
 
 // Protected-column bookkeeping of one CTA (warp 0): indices in [k_begin,
@@ -801,13 +824,15 @@ struct StreamArgs {
     uint32_t off_xt, off_q8, off_red, off_bar, off_pidx, off_pmask, off_zero, off_prot, off_tab;
 };
 
-// LUT: batch 1 through the nibble tables (x staged as tables, rows 4q..4q+3
-// per consumer warp); otherwise the MMA decode for batch <= 8.
-template <int WQ, int WK, int S, int MAXG, bool LUT>
-__global__ void __launch_bounds__((WQ * WK + 2) * 32, 2)
+// LUT: batch 1 through the nibble tables (x staged as tables); otherwise the
+// MMA decode for batch <= 8 * NT (NT n-tiles of 8 activation rows; at NT = 2
+// the staged activations fill most of the shared memory: one CTA per SM).
+template <int WQ, int WK, int S, int MAXG, bool LUT, int NT = 1>
+__global__ void __launch_bounds__((WQ * WK + 2) * 32, NT == 1 ? 2 : 1)
 k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
     constexpr int BM = 16;
-    constexpr int BP = 8;
+    constexpr int BP = 8 * NT;
+    static_assert(!LUT || NT == 1, "the table decode is batch 1");
     constexpr int NCW = WQ * WK;
     constexpr int SW = kSlab * WQ;
     constexpr int kCodeRow = SW / 8;
@@ -1070,7 +1095,7 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
         for (; ii < my_tiles; ++ii) {
             if (*reinterpret_cast<volatile int *>(&s_abort)) break;
             const int g = layer_of(ii);
-            float accp[4] = {0.f, 0.f, 0.f, 0.f};
+            float accp[NT][4] = {};
             if (!mbar_wait_all(bar_q8f + 8 * (ii & 1), (ii >> 1) & 1)) {
                 if (lane == 0) {
                     latch_error(err, BISCO_ERR_TIMEOUT);
@@ -1082,7 +1107,7 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
             const __half *xsh = reinterpret_cast<const __half *>(xs_of(g)), *xsl = xsh + B * cap;
             const int8_t *slab = q8base + (ii & 1) * q8_buf_bytes;
             for (int u16 = 0; u16 < pg; u16 += 16)
-                protected_rows(slab, s_L[g].q8_pitch, u16, gq, t, xsh, xsl, cap, B, accp);
+                protected_rows<NT>(slab, s_L[g].q8_pitch, u16, gq, t, xsh, xsl, cap, B, accp);
             __syncwarp();
             // buffer ii & 1 is free: the slab of tile ii + 2 goes into it
             if (lane == 0 && ii + 2 < my_tiles) {
@@ -1090,7 +1115,10 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
                 issue_q8(ii + 2);
             }
 #pragma unroll
-            for (int e = 0; e < 4; ++e) prot[(e < 2 ? gq : gq + 8) * BP + 2 * t + (e & 1)] = accp[e];
+            for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    prot[(e < 2 ? gq : gq + 8) * BP + nt * 8 + 2 * t + (e & 1)] = accp[nt][e];
             __syncwarp();
             if (!mbar_wait_all(bar_rf + 8 * (ii & 1), (ii >> 1) & 1)) {
                 if (lane == 0) {
@@ -1169,17 +1197,19 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
         // ----------------------------------------------- consumers: decode
         const int q = warp % WQ, k = warp / WQ;
         const int gq = lane >> 2, t = lane & 3;
-        const int xstep = gq < B ? 1024 : 0;
         for (int ii = 0; ii < my_tiles; ++ii) {
             if (*reinterpret_cast<volatile int *>(&s_abort)) break;
             const int g = layer_of(ii);
-            const unsigned char *xb = gq < B ? xt_of(g) + gq * xt_pitch + t * 16
-                                             : sm + off_zero + t * 16;
-            float acc[4][1][4];
+            // activation row nt * 8 + gq of each n-tile (rows >= B read a zero block)
+            const unsigned char *xb[NT];
+            int xstep[NT];
 #pragma unroll
-            for (int c = 0; c < 4; ++c)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) acc[c][0][e] = 0.f;
+            for (int nt = 0; nt < NT; ++nt) {
+                const int bg = nt * 8 + gq;
+                xb[nt] = bg < B ? xt_of(g) + bg * xt_pitch + t * 16 : sm + off_zero + t * 16;
+                xstep[nt] = bg < B ? 1024 : 0;
+            }
+            float acc[4][NT][4] = {};
             bool ok = true;
             // this warp's slots of tile ii: global index ii*nwide + w == k (mod WK)
             for (int w = (k - (ii * nwide) % WK + WK) % WK; w < nwide; w += WK) {
@@ -1192,9 +1222,11 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
                 const int nar = w * WQ + q;
                 if (nar < nnar) {
                     const unsigned char *cs = sm + (gidx % nslot) * kSlotBytes;
-                    const unsigned char *xr[1] = {xb + nar * xstep};
-                    decode_slot<S, BM, kCodeRow, kNormRow, false, 1>(cs, cs + kCodesBytes, q, gq,
-                                                                     gq + 8, t, xr, acc);
+                    const unsigned char *xr[NT];
+#pragma unroll
+                    for (int nt = 0; nt < NT; ++nt) xr[nt] = xb[nt] + nar * xstep[nt];
+                    decode_slot<S, BM, kCodeRow, kNormRow, false, NT>(cs, cs + kCodesBytes, q, gq,
+                                                                      gq + 8, t, xr, acc);
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar_empty + 8 * (gidx % nslot));
@@ -1211,13 +1243,15 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
             }
             float *rb = red + (ii & 1) * NCW * BM * B;
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const int r = e < 2 ? gq : gq + 8;
-                const int b = 2 * t + (e & 1);
-                if (b < B)
-                    rb[(warp * BM + r) * B + b] =
-                        ((acc[0][0][e] + acc[1][0][e]) + (acc[2][0][e] + acc[3][0][e])) * kInvSqrt8;
-            }
+            for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int r = e < 2 ? gq : gq + 8;
+                    const int b = nt * 8 + 2 * t + (e & 1);
+                    if (b < B)
+                        rb[(warp * BM + r) * B + b] =
+                            ((acc[0][nt][e] + acc[1][nt][e]) + (acc[2][nt][e] + acc[3][nt][e])) * kInvSqrt8;
+                }
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_rf + 8 * (ii & 1));
         }
@@ -1379,7 +1413,7 @@ size_t cluster_smem(int wm, int wq, int ck, int S, int B, int p, int wide_per_ra
 template <int MAXG>
 size_t stream_smem(int wq, int wk, int S, int B, int K, int G, int p_max, int q8_pitch, int nslot,
                    bool lut, StreamArgs<MAXG> *a) {
-    const int BM = 16, BP = 8, SW = kSlab * wq;
+    const int BM = 16, BP = B > 8 ? 16 : 8, SW = kSlab * wq;
     const int nar = (K + kSlab - 1) / kSlab;
     const int nwide = (K + SW - 1) / SW;
     a->pidx_cap = static_cast<int>(align_up(static_cast<size_t>(p_max), 16));
@@ -1499,9 +1533,9 @@ bisco_status launch_w(bool two, int S, const CUtensorMap &mc, const CUtensorMap 
     return launch_s<WM, WQ, 1>(S, mc, mn, mq, a, ck, smem, stream);
 }
 
-template <int WQ, int WK, int S, int MAXG, bool LUT>
+template <int WQ, int WK, int S, int MAXG, bool LUT, int NT = 1>
 bisco_status launch_stream_t(const StreamArgs<MAXG> &a, int grid, size_t smem, cudaStream_t stream) {
-    auto kern = k_gemv_stream<WQ, WK, S, MAXG, LUT>;
+    auto kern = k_gemv_stream<WQ, WK, S, MAXG, LUT, NT>;
     static size_t configured[64] = {};
     if (!set_smem(kern, smem, configured)) return BISCO_ERR_CUDA;
     cudaLaunchConfig_t cfg = {};
@@ -1565,6 +1599,8 @@ bisco_status launch_stream_g(const bisco_layer *Ls, int G, const uint16_t *x, in
     const char *lut_env = getenv("BISCO_GEMV_LUT");
     const bool lut = B == 1 && !(lut_env && lut_env[0] == '0');
     *launched = false;
+    // batch 9..16 (two MMA n-tiles) for single layers only
+    if (B > 8 && (MAXG > 1 || B > 16)) return BISCO_OK;
     StreamArgs<MAXG> a = {};
     a.x = x;
     a.err = err;
@@ -1617,6 +1653,15 @@ bisco_status launch_stream_g(const bisco_layer *Ls, int G, const uint16_t *x, in
             default: return launch_stream_t<WQ, WK, 3, MAXG, true>(a, grid, smem, stream);
         }
     }
+    if constexpr (MAXG == 1) {
+        if (B > 8) {
+            switch (S) {
+                case 1: return launch_stream_t<WQ, WK, 1, MAXG, false, 2>(a, grid, smem, stream);
+                case 2: return launch_stream_t<WQ, WK, 2, MAXG, false, 2>(a, grid, smem, stream);
+                default: return launch_stream_t<WQ, WK, 3, MAXG, false, 2>(a, grid, smem, stream);
+            }
+        }
+    }
     switch (S) {
         case 1: return launch_stream_t<WQ, WK, 1, MAXG, false>(a, grid, smem, stream);
         case 2: return launch_stream_t<WQ, WK, 2, MAXG, false>(a, grid, smem, stream);
@@ -1659,8 +1704,8 @@ bisco_status launch_gemv(const bisco_layer &L, const uint16_t *x, int B, float *
     // streaming kernel: small batch and at least one 16-row tile per SM
     const char *mode = getenv("BISCO_GEMV_MODE");
     const int sms = num_sms();
-    bool use_stream = B <= 8 && (N + 15) / 16 >= sms;
-    if (mode && mode[0] == 's') use_stream = B <= 8;
+    bool use_stream = B <= 16 && (N + 15) / 16 >= sms;
+    if (mode && mode[0] == 's') use_stream = B <= 16;
     if (mode && mode[0] == 'c') use_stream = false;
     if (use_stream) {
         bool launched = false;

@@ -94,6 +94,9 @@ def test_gemv_every_tiling(env, plan, B):
     (2500, 1024, 2, 11, 5, 7),
     (2500, 2176, 3, 23, 2, 4),     # a slot straddles the end of K
     (5000, 512, 2, 300, 1, 5),     # three q8 boxes per tile, many tiles per CTA
+    (2500, 1024, 2, 11, 16, 3),    # batch 16: two MMA n-tiles
+    (2500, 2176, 3, 23, 12, 2),    # batch 12, K not a slot multiple
+    (300, 4096, 2, 41, 9, 3),      # batch 9: second n-tile one row wide
 ])
 def test_gemv_streaming_path(env, N, K, S, p, B, nslot):
     """The persistent streaming kernel (reducer warp, int8 slab double
