@@ -175,6 +175,9 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
             prefetch_tmap(&tm_x);
             prefetch_tmap(&tm_codes);
             prefetch_tmap(&tm_norms);
+            // the activation copy X16 is written by the pre-pass launched just
+            // before this kernel (programmatic dependent launch)
+            pdl_wait();
             int xi = 0, wi = 0;
             bool ok = true;
             for (int t = blockIdx.x; ok && t < a.ntiles; t += gridDim.x) {
@@ -322,14 +325,33 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
 // protected k and for K <= k < K_pad); for protected block bq and u < 64,
 // X16[m][K_pad + 128 bq + u] = hi(v), X16[m][K_pad + 128 bq + 64 + u] = lo(v)
 // with v = sqrt(8) * scale_{64bq+u} * x[m][j_{64bq+u}] (0 past p).
-constexpr int kPrepRows = 16;
+constexpr int kPrepThreads = 256;
+constexpr int kPrepJobs = 4;   // 8-column groups per thread, their loads in flight together
 
-__global__ void __launch_bounds__(256) k_gemm_prep(const uint16_t *__restrict__ X, int M, int K,
-                                                   int K_pad, int K_ext, int p,
-                                                   const int32_t *__restrict__ prot_idx,
-                                                   const uint16_t *__restrict__ q8_scale,
-                                                   uint16_t *__restrict__ X16, int *err) {
+__global__ void __launch_bounds__(kPrepThreads) k_gemm_prep(const uint16_t *__restrict__ X, int M, int K,
+                                                            int K_pad, int K_ext, int p,
+                                                            const int32_t *__restrict__ prot_idx,
+                                                            const uint16_t *__restrict__ q8_scale,
+                                                            uint16_t *__restrict__ X16, int *err) {
     extern __shared__ uint32_t s_mask[];   // K_pad / 32 words
+    // the GEMM launched after this kernel may set itself up meanwhile; it
+    // waits for this grid's completion before it reads X16
+    pdl_launch_dependents();
+    const int groups = K_ext / 8;
+    const int64_t njobs = static_cast<int64_t>(M) * groups;
+    const int64_t base = static_cast<int64_t>(blockIdx.x) * kPrepThreads * kPrepJobs + threadIdx.x;
+    // the plain columns' loads go out first; the protected-column mask is
+    // built while they are in flight
+    uint4 v[kPrepJobs];
+#pragma unroll
+    for (int i = 0; i < kPrepJobs; ++i) {
+        const int64_t e = base + static_cast<int64_t>(i) * kPrepThreads;
+        v[i] = make_uint4(0u, 0u, 0u, 0u);
+        if (e < njobs) {
+            const int m = static_cast<int>(e / groups), k = static_cast<int>(e % groups) * 8;
+            if (k < K) v[i] = *reinterpret_cast<const uint4 *>(X + static_cast<int64_t>(m) * K + k);
+        }
+    }
     const int mw = K_pad / 32;
     for (int i = threadIdx.x; i < mw; i += blockDim.x) s_mask[i] = 0u;
     __syncthreads();
@@ -342,43 +364,43 @@ __global__ void __launch_bounds__(256) k_gemm_prep(const uint16_t *__restrict__ 
         atomicOr(&s_mask[j >> 5], 1u << (j & 31));
     }
     __syncthreads();
-    const int groups = K_ext / 8;
-    const int m0 = blockIdx.x * kPrepRows;
-    for (int e = threadIdx.x; e < kPrepRows * groups; e += blockDim.x) {
-        const int m = m0 + e / groups, k = (e % groups) * 8;
-        if (m >= M) break;
+#pragma unroll
+    for (int i = 0; i < kPrepJobs; ++i) {
+        const int64_t e = base + static_cast<int64_t>(i) * kPrepThreads;
+        if (e >= njobs) break;
+        const int m = static_cast<int>(e / groups), k = static_cast<int>(e % groups) * 8;
         uint32_t o[4] = {0u, 0u, 0u, 0u};
-        const uint16_t *xr = X + static_cast<int64_t>(m) * K;
         if (k < K_pad) {
             if (k < K) {
-                const uint4 v = *reinterpret_cast<const uint4 *>(xr + k);
-                const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+                const uint32_t w[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
                 const uint32_t pm = (s_mask[k >> 5] >> (k & 31)) & 0xFFu;
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const float lo = (pm >> (2 * i)) & 1u ? 0.f : __uint_as_float(w[i] << 16);
-                    const float hi = (pm >> (2 * i + 1)) & 1u ? 0.f : __uint_as_float(w[i] & 0xFFFF0000u);
+                for (int q = 0; q < 4; ++q) {
+                    const float lo = (pm >> (2 * q)) & 1u ? 0.f : __uint_as_float(w[q] << 16);
+                    const float hi = (pm >> (2 * q + 1)) & 1u ? 0.f : __uint_as_float(w[q] & 0xFFFF0000u);
                     const __half2 h2 = __floats2half2_rn(lo, hi);
-                    o[i] = *reinterpret_cast<const uint32_t *>(&h2);
+                    o[q] = *reinterpret_cast<const uint32_t *>(&h2);
                 }
             }
         } else {
+            // protected block bq, part hi (0) or lo (1): sqrt(8) * scale_u * x[m][j_u]
+            const uint16_t *xr = X + static_cast<int64_t>(m) * K;
             const int e2 = k - K_pad, bq = e2 >> 7, part = (e2 >> 6) & 1, u0 = bq * 64 + (e2 & 63);
             uint16_t hv[8];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const int u = u0 + i;
-                float v = 0.f;
+            for (int q = 0; q < 8; ++q) {
+                const int u = u0 + q;
+                float val = 0.f;
                 const int j = u < p ? prot_idx[u] : -1;
                 if (j >= 0 && j < K)
-                    v = (__half2float(__ushort_as_half(q8_scale[u])) *
-                         __uint_as_float(static_cast<uint32_t>(xr[j]) << 16)) * kSqrt8;
-                const __half vh = __float2half_rn(v);
-                hv[i] = part ? __half_as_ushort(__float2half_rn(v - __half2float(vh)))
+                    val = (__half2float(__ushort_as_half(q8_scale[u])) *
+                           __uint_as_float(static_cast<uint32_t>(xr[j]) << 16)) * kSqrt8;
+                const __half vh = __float2half_rn(val);
+                hv[q] = part ? __half_as_ushort(__float2half_rn(val - __half2float(vh)))
                              : __half_as_ushort(vh);
             }
 #pragma unroll
-            for (int i = 0; i < 4; ++i) o[i] = hv[2 * i] | (static_cast<uint32_t>(hv[2 * i + 1]) << 16);
+            for (int q = 0; q < 4; ++q) o[q] = hv[2 * q] | (static_cast<uint32_t>(hv[2 * q + 1]) << 16);
         }
         *reinterpret_cast<uint4 *>(X16 + static_cast<int64_t>(m) * K_ext + k) =
             make_uint4(o[0], o[1], o[2], o[3]);
@@ -418,8 +440,20 @@ bisco_status launch_gemm_t(const CUtensorMap &mx, const CUtensorMap &mc, const C
             return BISCO_ERR_CUDA;
         configured[dev] = smem;
     }
-    k_gemm<NX, NW><<<grid, kThreads, smem, stream>>>(mx, mc, mn, mq, a);
-    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+    // programmatic dependent launch after the pre-pass: barrier set-up and
+    // the TMEM allocation overlap it; the producer waits before its first copy
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid, 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_gemm<NX, NW>, mx, mc, mn, mq, a) == cudaSuccess ? BISCO_OK
+                                                                                     : BISCO_ERR_CUDA;
 }
 
 }  // namespace
@@ -449,7 +483,9 @@ bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *
             configured[dev] = prep_smem;
         }
     }
-    k_gemm_prep<<<(M + kPrepRows - 1) / kPrepRows, 256, prep_smem, stream>>>(
+    const int64_t prep_jobs = static_cast<int64_t>(M) * (K_ext / 8);
+    const int prep_grid = static_cast<int>((prep_jobs + kPrepThreads * kPrepJobs - 1) / (kPrepThreads * kPrepJobs));
+    k_gemm_prep<<<prep_grid, kPrepThreads, prep_smem, stream>>>(
         X, M, K, K_pad, K_ext, p, L.prot_idx, L.q8_scale, X16, err);
     if (cudaGetLastError() != cudaSuccess) return BISCO_ERR_CUDA;
 
