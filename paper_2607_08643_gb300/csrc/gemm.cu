@@ -20,8 +20,9 @@
 //
 // CTA roles (512 threads, one CTA per SM, persistent over output tiles):
 //   warps 0-3  epilogue: TMEM -> registers -> Y (fp32), lane quarter w
-//   warp 4     TMA producer (activation ring, compressed-weight ring)
+//   warp 4     TMA producer of the compressed-weight ring
 //   warp 5     TMEM allocator and MMA issuer (one thread)
+//   warp 6     TMA producer of the activation ring
 //   warps 8-15 decoders: lane quarter w % 4, K half (w - 8) / 4
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -33,7 +34,7 @@ namespace bisco {
 namespace {
 
 constexpr int GM = 128;     // output features per tile (MMA M, TMEM lanes)
-constexpr int GN = 256;     // tokens per tile (MMA N)
+constexpr int GN = 256;     // tokens per tile (MMA N); 128 when 256 leaves SMs idle
 constexpr int GK = 128;     // K columns per weight step (one TMEM A stage)
 // Ring depths are template parameters (NX activation stages of 64 columns
 // = 32 KB, NW compressed-weight stages of 128 columns): the activation ring
@@ -42,9 +43,10 @@ constexpr int GK = 128;     // K columns per weight step (one TMEM A stage)
 constexpr int NA = 3;       // TMEM A ring (128 K columns = 64 TMEM columns each)
 constexpr int kThreads = 512;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColD = 0;     // accumulator: 256 fp32 columns
+constexpr uint32_t kColD = 0;     // accumulator: TN <= 256 fp32 columns
 constexpr uint32_t kColA = 256;   // A stages
-constexpr uint32_t kXStage = GN * 128;   // 256 rows x 64 fp16
+// one 64-column activation stage of a TN-token tile: TN rows x 64 fp16
+constexpr uint32_t x_stage_bytes(int tn) { return static_cast<uint32_t>(tn) * 128; }
 constexpr float kInvSqrt8 = 0.35355339059327373f;
 constexpr float kSqrt8 = 2.8284271247461903f;
 
@@ -59,9 +61,10 @@ struct GemmArgs {
     uint32_t w_stage;   // bytes of one compressed-weight stage
 };
 
-// idesc of kind::f16: D f32, A = B = f16, both K-major, N = GN, M = GM.
-constexpr uint32_t kIdesc = (1u << 4) | (static_cast<uint32_t>(GN >> 3) << 17) |
-                            (static_cast<uint32_t>(GM >> 4) << 24);
+// idesc of kind::f16: D f32, A = B = f16, both K-major, N = tn, M = GM.
+constexpr uint32_t idesc_f16(int tn) {
+    return (1u << 4) | (static_cast<uint32_t>(tn >> 3) << 17) | (static_cast<uint32_t>(GM >> 4) << 24);
+}
 
 // Decoded fp16 pairs of 8 chunks (64 columns) of one row and S stages:
 // element pair (2j, 2j+1) of chunk c is ((t << (15-2j)) & 0x80008000) ^
@@ -116,11 +119,13 @@ __device__ __forceinline__ void decode_q8_row(const unsigned char *q8s, int r, u
     }
 }
 
-template <int NX, int NW>
+template <int NX, int NW, int TN>
 __global__ void __launch_bounds__(kThreads, 1)
 k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_codes,
        const __grid_constant__ CUtensorMap tm_norms, const __grid_constant__ CUtensorMap tm_q8,
        const GemmArgs a) {
+    constexpr uint32_t kXStage = x_stage_bytes(TN);
+    constexpr uint32_t kIdesc = idesc_f16(TN);
     extern __shared__ unsigned char smem_raw[];
     unsigned char *sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     const uint32_t sbase = smem_u32(sm);
@@ -170,18 +175,16 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
     };
 
     if (warp == 4) {
-        // ------------------------------------------------------ producer
+        // ----------------------------------- producer: compressed weights
+        // (its own thread: the weight ring runs ahead of the decoders without
+        // waiting for the MMAs to free activation stages)
         if (lane == 0) {
-            prefetch_tmap(&tm_x);
             prefetch_tmap(&tm_codes);
             prefetch_tmap(&tm_norms);
-            // the activation copy X16 is written by the pre-pass launched just
-            // before this kernel (programmatic dependent launch)
-            pdl_wait();
-            int xi = 0, wi = 0;
+            int wi = 0;
             bool ok = true;
             for (int t = blockIdx.x; ok && t < a.ntiles; t += gridDim.x) {
-                const int f0 = (t / a.tiles_t) * GM, t0 = (t % a.tiles_t) * GN;
+                const int f0 = (t / a.tiles_t) * GM;
                 for (int ks = 0; ks < ksteps; ++ks) {
                     const int ws = wi % NW;
                     if (wi >= NW && !mbar_wait(wempty + 8 * ws, ((wi / NW) - 1) & 1)) { ok = false; break; }
@@ -198,20 +201,36 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
                         tma_load_2d(wdst, &tm_q8, wfull + 8 * ws, (ks - a.ks_main) * 64, f0);
                     }
                     ++wi;
-                    for (int hh = 0; hh < 2; ++hh) {
-                        const int xs = xi % NX;
-                        if (xi >= NX && !mbar_wait(xempty + 8 * xs, ((xi / NX) - 1) & 1)) { ok = false; break; }
-                        mbar_arrive_expect_tx(xfull + 8 * xs, kXStage);
-                        tma_load_2d(x_ring + xs * kXStage, &tm_x, xfull + 8 * xs, ks * GK + hh * 64, t0);
-                        ++xi;
-                    }
-                    if (!ok) break;
                 }
             }
             if (!ok) fail();
             // every copy issued has landed before this thread leaves (in the
             // normal case the consumers saw them all, so this returns at once)
             for (int i = (wi > NW ? wi - NW : 0); i < wi; ++i) mbar_wait(wfull + 8 * (i % NW), (i / NW) & 1);
+        }
+    } else if (warp == 6) {
+        // ----------------------------------------- producer: activations
+        if (lane == 0) {
+            prefetch_tmap(&tm_x);
+            // the activation copy X16 is written by the pre-pass launched just
+            // before this kernel (programmatic dependent launch)
+            pdl_wait();
+            int xi = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; ok && t < a.ntiles; t += gridDim.x) {
+                const int t0 = (t % a.tiles_t) * TN;
+                for (int ks = 0; ok && ks < ksteps; ++ks) {
+                    for (int hh = 0; hh < 2; ++hh) {
+                        const int xs = xi % NX;
+                        if (xi >= NX && !mbar_wait(xempty + 8 * xs, ((xi / NX) - 1) & 1)) { ok = false; break; }
+                        if (aborted()) { ok = false; break; }
+                        mbar_arrive_expect_tx(xfull + 8 * xs, kXStage);
+                        tma_load_2d(x_ring + xs * kXStage, &tm_x, xfull + 8 * xs, ks * GK + hh * 64, t0);
+                        ++xi;
+                    }
+                }
+            }
+            if (!ok) fail();
             for (int i = (xi > NX ? xi - NX : 0); i < xi; ++i) mbar_wait(xfull + 8 * (i % NX), (i / NX) & 1);
         }
     } else if (warp == 5) {
@@ -259,9 +278,7 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
             for (int ks = 0; ks < ksteps; ++ks) {
                 const int ws = wi % NW, as = ai % NA;
                 if (!mbar_wait_all(wfull + 8 * ws, (wi / NW) & 1)) { ok = false; break; }
-                if (ai >= NA && !mbar_wait_all(aempty + 8 * as, ((ai / NA) - 1) & 1)) { ok = false; break; }
                 if (__any_sync(0xFFFFFFFFu, aborted())) { ok = false; break; }
-                tc_fence_after();
                 const unsigned char *wst = sm + (w_ring - sbase) + ws * a.w_stage;
                 uint32_t out[32];
                 if (ks < a.ks_main)
@@ -270,6 +287,10 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
                     decode_q8_row(wst, r, out);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(wempty + 8 * ws);
+                // the TMEM stage is needed only for the store: decode first, so
+                // the decode overlaps the MMAs still reading this stage
+                if (ai >= NA && !mbar_wait_all(aempty + 8 * as, ((ai / NA) - 1) & 1)) { ok = false; break; }
+                tc_fence_after();
                 tmem_st32(tmem + (static_cast<uint32_t>(32 * q) << 16) + kColA + as * 64 + h * 32, out);
                 tmem_wait_st();
                 tc_fence_before();
@@ -293,10 +314,10 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
                 break;
             }
             tc_fence_after();
-            const int f0 = (t / a.tiles_t) * GM, t0 = (t % a.tiles_t) * GN;
+            const int f0 = (t / a.tiles_t) * GM, t0 = (t % a.tiles_t) * TN;
             const int feat = f0 + 32 * q + lane;
 #pragma unroll 1
-            for (int c = 0; c < GN / 32; ++c) {
+            for (int c = 0; c < TN / 32; ++c) {
                 uint32_t v[32];
                 tmem_ld32(tmem + (static_cast<uint32_t>(32 * q) << 16) + kColD + c * 32, v);
                 tmem_wait_ld();
@@ -426,16 +447,17 @@ bisco_status gemm_via_gemv(const bisco_layer &L, const uint16_t *X, int M, float
     return BISCO_OK;
 }
 
-template <int NX, int NW>
+template <int NX, int NW, int TN>
 bisco_status launch_gemm_t(const CUtensorMap &mx, const CUtensorMap &mc, const CUtensorMap &mn,
                            const CUtensorMap &mq, const GemmArgs &a, int grid, cudaStream_t stream) {
-    const size_t smem = 1024 + NX * kXStage + NW * a.w_stage + 8 * (2 * NX + 2 * NW + 2 * NA + 3);
+    const size_t smem =
+        1024 + NX * x_stage_bytes(TN) + NW * a.w_stage + 8 * (2 * NX + 2 * NW + 2 * NA + 3);
     if (smem > 227 * 1024) return BISCO_ERR_UNSUPPORTED;
     static size_t configured[64] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return BISCO_ERR_CUDA;
     if (smem > configured[dev]) {
-        if (cudaFuncSetAttribute(k_gemm<NX, NW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        if (cudaFuncSetAttribute(k_gemm<NX, NW, TN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  static_cast<int>(smem)) != cudaSuccess)
             return BISCO_ERR_CUDA;
         configured[dev] = smem;
@@ -452,8 +474,9 @@ bisco_status launch_gemm_t(const CUtensorMap &mx, const CUtensorMap &mc, const C
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, k_gemm<NX, NW>, mx, mc, mn, mq, a) == cudaSuccess ? BISCO_OK
-                                                                                     : BISCO_ERR_CUDA;
+    return cudaLaunchKernelEx(&cfg, k_gemm<NX, NW, TN>, mx, mc, mn, mq, a) == cudaSuccess
+               ? BISCO_OK
+               : BISCO_ERR_CUDA;
 }
 
 }  // namespace
@@ -489,11 +512,17 @@ bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *
         X, M, K, K_pad, K_ext, p, L.prot_idx, L.q8_scale, X16, err);
     if (cudaGetLastError() != cudaSuccess) return BISCO_ERR_CUDA;
 
+    // token tile: 256, or 128 when 256-token tiles would leave SMs idle
+    // (e.g. k_proj / v_proj: 8 feature tiles); the decode per k-step is the
+    // same, the MMA work halves
+    const int sms = num_sms();
+    const int feat_tiles = (N + GM - 1) / GM;
+    const int TN = (static_cast<long>((M + GN - 1) / GN) * feat_tiles < sms && M > 128) ? 128 : GN;
     CUtensorMap mx, mc, mn, mq;
     {
         const uint64_t dims[2] = {static_cast<uint64_t>(K_ext), static_cast<uint64_t>(M)};
         const uint64_t strides[1] = {static_cast<uint64_t>(K_ext) * 2};
-        const uint32_t box[2] = {64, GN};
+        const uint32_t box[2] = {64, static_cast<uint32_t>(TN)};
         if (!encode_tensor_map(&mx, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, X16, dims, strides, box,
                                CU_TENSOR_MAP_SWIZZLE_128B))
             return BISCO_ERR_CUDA;
@@ -530,14 +559,15 @@ bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *
     a.S = S;
     a.ks_main = K_pad / GK;
     a.ks_ext = p_ext_of(p) / 64;
-    a.tiles_t = (M + GN - 1) / GN;
-    a.ntiles = a.tiles_t * ((N + GM - 1) / GM);
+    a.tiles_t = (M + TN - 1) / TN;
+    a.ntiles = a.tiles_t * feat_tiles;
     a.w_stage = static_cast<uint32_t>(S * GM * 48 > GM * 64 ? S * GM * 48 : GM * 64);
-    const int sms = num_sms();
     const int grid = a.ntiles < sms ? a.ntiles : sms;
-    // S = 1: 6 x 32 KB + 3 x 8 KB; S = 2, 3: 5 x 32 KB + 3 x 12/18 KB (<= 227 KB)
-    if (S == 1) return launch_gemm_t<6, 3>(mx, mc, mn, mq, a, grid, stream);
-    return launch_gemm_t<5, 3>(mx, mc, mn, mq, a, grid, stream);
+    // 256 tokens: S = 1: 6 x 32 KB + 3 x 8 KB; S = 2, 3: 5 x 32 KB + 3 x 12/18 KB;
+    // 128 tokens: 8 x 16 KB + 3 x 8/12/18 KB (all <= 227 KB)
+    if (TN == 128) return launch_gemm_t<8, 3, 128>(mx, mc, mn, mq, a, grid, stream);
+    if (S == 1) return launch_gemm_t<6, 3, GN>(mx, mc, mn, mq, a, grid, stream);
+    return launch_gemm_t<5, 3, GN>(mx, mc, mn, mq, a, grid, stream);
 }
 
 }  // namespace bisco
