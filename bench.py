@@ -45,7 +45,7 @@ def parse():
     ap.add_argument("--impl", choices=("bisco", "reference"), default="bisco")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
-    ap.add_argument("--mode", choices=("both", "decode", "prefill", "shapes"), default="both",
+    ap.add_argument("--mode", choices=("both", "decode", "prefill", "shapes", "dense"), default="both",
                     help="decode: the GEMV step only; prefill: the tcgen05 GEMM only; "
                          "shapes: batch-1 GEMV per Qwen3-8B layer shape")
     ap.add_argument("--shape-mb", type=float, default=500.0,
@@ -417,6 +417,88 @@ def run_prefill(args, local_rank):
             "dtype": "f16 x f16 -> f32", "launches_per_step": 2 * len(layers)}
 
 
+# ------------------------------------------------------------------ dense
+
+def run_dense(args, local_rank):
+    """The materialise-then-multiply comparison: the same 36-layer q/k/v/o
+    stack decoded once to dense bf16 weights with bisco_decode_dense (q/k/v
+    of a layer into one [6144][4096] matrix), then the decode step as two
+    cuBLAS products per layer (torch.matmul, a CUDA graph of the step), the
+    same launch structure as the fused step.  Reports the one-time decode
+    and the dense step (its GB/s counts the dense bf16 weight bytes)."""
+    import torch
+    from paper_2607_08643_gb300 import bisco
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    bisco.load()
+    layers = build_layers(args, dev)
+    B, K = args.batch, 4096
+    dense = []
+    for li in range(args.layers):
+        qkv = [layers[4 * li + j][1] for j in range(3)]
+        W_qkv = torch.empty((sum(L.N for L in qkv), K), dtype=torch.bfloat16, device=dev)
+        W_o = torch.empty((layers[4 * li + 3][1].N, K), dtype=torch.bfloat16, device=dev)
+        dense.append((qkv, W_qkv, layers[4 * li + 3][1], W_o))
+    stream = torch.cuda.Stream(device=dev)
+
+    def materialise():
+        for qkv, W_qkv, L_o, W_o in dense:
+            r0 = 0
+            for L in qkv:
+                bisco.bisco_decode_dense(L, "bf16", out=W_qkv[r0:r0 + L.N], stream=stream)
+                r0 += L.N
+            bisco.bisco_decode_dense(L_o, "bf16", out=W_o, stream=stream)
+
+    with torch.cuda.stream(stream):
+        materialise()   # warm-up
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        materialise()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    if bisco.bisco_get_device_error(stream) != bisco.OK:
+        raise RuntimeError("device error in bisco_decode_dense")
+    ms_mat = e0.elapsed_time(e1)
+    comp = sum(L.compressed_bytes for _, L in layers)
+    dense_bytes = sum((W_qkv.numel() + W_o.numel()) * 2 for _, W_qkv, _, W_o in dense)
+
+    x = torch.randn((2 * args.layers, K, B), device=dev).to(torch.bfloat16)
+    ys = [(torch.empty((W_qkv.shape[0], B), dtype=torch.bfloat16, device=dev),
+           torch.empty((W_o.shape[0], B), dtype=torch.bfloat16, device=dev)) for _, W_qkv, _, W_o in dense]
+
+    def step():
+        for li, (_, W_qkv, _, W_o) in enumerate(dense):
+            torch.matmul(W_qkv, x[2 * li], out=ys[li][0])
+            torch.matmul(W_o, x[2 * li + 1], out=ys[li][1])
+
+    with torch.cuda.stream(stream):
+        step()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            step()
+    torch.cuda.synchronize()
+    for _ in range(max(args.warmup, 3)):
+        g.replay()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(args.steps):
+            g.replay()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / args.steps
+    return {"how": "bisco_decode_dense to bf16 once, then torch.matmul (cuBLAS) per step: "
+                   "q/k/v concatenated + o_proj per layer, CUDA graph",
+            "materialise_ms": ms_mat,
+            "materialise_gbs": (comp + dense_bytes) / (ms_mat * 1e-3) / 1e9,
+            "dense_bytes_per_step": dense_bytes, "compressed_bytes": comp,
+            "ms_per_step": ms, "tokens_per_s": B / (ms * 1e-3),
+            "dense_gbs": dense_bytes / (ms * 1e-3) / 1e9, "batch": B}
+
+
 # ----------------------------------------------------------------- shapes
 
 def run_shapes(args, local_rank):
@@ -565,6 +647,13 @@ def main():
                               "unit": "GB/s", "hbm_peak_gbs": peaks()[0], "steps": args.steps,
                               "data": "synthetic", "shapes": res}))
         return
+    if args.mode == "dense":
+        dn = run_dense(args, local_rank)
+        if rank == 0:
+            print(json.dumps(dict(dn, metric="decode step through materialised bf16 weights",
+                                  n_gpus=world, steps=args.steps, warmup=args.warmup,
+                                  data="synthetic", config=workload_config(args))))
+        return
     if args.mode == "prefill":
         pf = run_prefill(args, local_rank)
         if rank == 0:
@@ -580,6 +669,11 @@ def main():
         cpu = cpu_oracle_sample(args.cpu_seconds, args.batch)
     r = run_bisco(args, rank, world, local_rank)
     prefill = run_prefill(args, local_rank) if args.mode == "both" else None
+    dense_cmp = None
+    if args.mode == "both" and world == 1:
+        dn = run_dense(args, local_rank)
+        dense_cmp = dict(dn, fused_tokens_per_s=r["tokens_per_s"],
+                         fused_over_dense=r["tokens_per_s"] / dn["tokens_per_s"])
     if rank == 0:
         line = {
             "metric": METRIC, "value": r["value"], "unit": "GB/s", "n_gpus": world,
@@ -599,6 +693,7 @@ def main():
             "cpu_baseline": cpu,
             "parallelism": "replicas" if world > 1 else "single GPU",
             "prefill": prefill,
+            "dense_comparison": dense_cmp,
         }
         print(json.dumps(line))
     if world > 1:

@@ -82,7 +82,7 @@ typedef struct {
 } bisco_layer;
 
 /* ABI version of this header (major * 100 + minor). */
-#define BISCO_ABI_VERSION 102
+#define BISCO_ABI_VERSION 103
 int32_t bisco_abi_version(void);
 
 /* Static string for a status code (never NULL). */
@@ -194,6 +194,24 @@ bisco_status bisco_gemv_multi(const bisco_layer *layers, int32_t G, const uint16
 size_t bisco_gemm_workspace_bytes(const bisco_layer *L, int32_t M);
 bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M, float *Y,
                         void *workspace, size_t workspace_bytes, bisco_stream_t stream);
+
+/*
+ * The coded layer decoded to a dense row-major matrix (Sec. III-F Eq. 12
+ * with the Eq. 10 overwrite), the materialise-then-multiply alternative to
+ * the fused kernels:
+ *     out[i][j] = sum_s (bit ? -1 : +1) * n16_{s,i,j/8} / sqrt(8)   j not protected
+ *     out[i][j] = scale_j * q8[i][j]                                 j protected
+ * The stage sum is formed in fp32 and rounded once after the 1/sqrt(8)
+ * scale (to fp32, or from there to bf16 / fp16 with round-to-nearest-even);
+ * the protected values are exact in fp32.
+ * out: [N][K] device, 16-byte aligned, fully overwritten; dtype one of
+ * BISCO_DENSE_*.  Asynchronous on `stream` (two kernels).
+ */
+#define BISCO_DENSE_F32 0
+#define BISCO_DENSE_BF16 1
+#define BISCO_DENSE_F16 2
+bisco_status bisco_decode_dense(const bisco_layer *L, void *out, int32_t dtype,
+                                bisco_stream_t stream);
 
 /*
  * A protected-column index outside [0, K) (or a list that is not ascending)

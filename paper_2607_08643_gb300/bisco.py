@@ -19,8 +19,10 @@ EXPORTS = (
     "bisco_abi_version", "bisco_status_string", "bisco_encoded_sizes",
     "bisco_encode_workspace_bytes", "bisco_encode", "bisco_encode_noalloc", "bisco_gemv",
     "bisco_gemv_multi",
-    "bisco_gemm_workspace_bytes", "bisco_gemm", "bisco_get_device_error",
+    "bisco_gemm_workspace_bytes", "bisco_gemm", "bisco_decode_dense", "bisco_get_device_error",
 )
+
+DENSE_F32, DENSE_BF16, DENSE_F16 = 0, 1, 2
 
 
 class BiscoError(RuntimeError):
@@ -73,6 +75,8 @@ def load(path: str = LIB_PATH):
     lib.bisco_gemm_workspace_bytes.argtypes = [Lp, i32]
     lib.bisco_gemm.restype = st
     lib.bisco_gemm.argtypes = [Lp, P, i32, P, P, sz, P]
+    lib.bisco_decode_dense.restype = st
+    lib.bisco_decode_dense.argtypes = [Lp, P, i32, P]
     lib.bisco_get_device_error.restype = st
     lib.bisco_get_device_error.argtypes = [P]
     _lib = lib
@@ -253,6 +257,20 @@ def bisco_gemm(L: Layer, X_bits, Y=None, workspace=None, stream=None):
     _check(load().bisco_gemm(ctypes.byref(L.c), _ptr(X_bits), M, _ptr(Y), _ptr(workspace),
                              nbytes, _stream(stream)), "bisco_gemm")
     return Y
+
+
+def bisco_decode_dense(L: Layer, dtype: str = "f32", out=None, stream=None):
+    """The layer's decoded weight What [N][K] as a dense tensor ("f32", "bf16"
+    or "f16"): the materialise-then-multiply path."""
+    import torch
+    code = {"f32": DENSE_F32, "bf16": DENSE_BF16, "f16": DENSE_F16}[dtype]
+    tdt = {"f32": torch.float32, "bf16": torch.bfloat16, "f16": torch.float16}[dtype]
+    if out is None:
+        out = torch.empty((L.N, L.K), dtype=tdt, device=L.codes.device)
+    assert out.is_contiguous() and out.dtype == tdt and tuple(out.shape) == (L.N, L.K)
+    _check(load().bisco_decode_dense(ctypes.byref(L.c), _ptr(out), code, _stream(stream)),
+           "bisco_decode_dense")
+    return out
 
 
 def bisco_get_device_error(stream=None) -> int:

@@ -219,6 +219,18 @@ bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M,
                        reinterpret_cast<cudaStream_t>(stream));
 }
 
+bisco_status bisco_decode_dense(const bisco_layer *L, void *out, int32_t dtype,
+                                bisco_stream_t stream) {
+    bisco_status st = check_layer(L, true);
+    if (st != BISCO_OK) return st;
+    if (dtype != BISCO_DENSE_F32 && dtype != BISCO_DENSE_BF16 && dtype != BISCO_DENSE_F16)
+        return BISCO_ERR_INVALID_ARG;
+    if (!out || !aligned16(out)) return BISCO_ERR_INVALID_ARG;
+    int *err = device_error_word(&st);
+    if (!err) return st;
+    return launch_decode_dense(*L, out, dtype, err, reinterpret_cast<cudaStream_t>(stream));
+}
+
 bisco_status bisco_get_device_error(bisco_stream_t stream) {
     bisco_status st;
     int *err = device_error_word(&st);

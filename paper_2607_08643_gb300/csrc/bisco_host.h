@@ -31,5 +31,7 @@ bisco_status launch_gemv_multi(const bisco_layer *Ls, int G, const uint16_t *x, 
 size_t gemm_workspace_bytes(const bisco_layer &L, int M);
 bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *Y,
                          void *workspace, size_t ws_bytes, int *err, cudaStream_t stream);
+bisco_status launch_decode_dense(const bisco_layer &L, void *out, int dtype, int *err,
+                                 cudaStream_t stream);
 
 }  // namespace bisco

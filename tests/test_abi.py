@@ -35,7 +35,7 @@ def test_header_declarations_are_exported(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert bisco.bisco_abi_version() == 102
+    assert bisco.bisco_abi_version() == 103
     for code in range(6):
         assert bisco.status_string(code)
     assert bisco.status_string(99) == "unknown status"
@@ -115,6 +115,19 @@ def test_call_argument_validation(lib):
     L2 = _fake_layer(k_in=4096, n_protected=41)
     assert lib.bisco_gemm_workspace_bytes(ctypes.byref(L2), 2048) == 2048 * (4096 + 128) * 2
     assert lib.bisco_gemm(ctypes.byref(L2), x, 2048, y, None, 0, None) == bisco.ERR_INVALID_ARG
+
+
+def test_decode_dense_validation(lib):
+    L = _fake_layer()
+    out = ctypes.c_void_p(0x70000)
+    assert lib.bisco_decode_dense(ctypes.byref(L), out, 3, None) == bisco.ERR_INVALID_ARG     # dtype
+    assert lib.bisco_decode_dense(ctypes.byref(L), out, -1, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_decode_dense(ctypes.byref(L), None, bisco.DENSE_F32, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_decode_dense(ctypes.byref(L), ctypes.c_void_p(0x70004), bisco.DENSE_BF16,
+                                  None) == bisco.ERR_INVALID_ARG                               # alignment
+    assert lib.bisco_decode_dense(None, out, bisco.DENSE_F16, None) == bisco.ERR_INVALID_ARG
+    assert lib.bisco_decode_dense(ctypes.byref(_fake_layer(codes=0x10004)), out, bisco.DENSE_F32,
+                                  None) == bisco.ERR_INVALID_ARG
 
 
 def test_gemv_multi_validation(lib):
