@@ -95,15 +95,19 @@ struct StageView {
     const int *pu;            // protected columns before each group
     const float *pscale;      // scale of each protected column
     float *xs;                // [B][cap] scale * x of each protected column
+    const int *pidx;          // the protected columns (absolute indices)
+    int np;                   // how many
 };
 
 // Activation staging for the input columns [k_begin, k_begin + cols) of G
 // layers that share x: bf16 rows from global memory -> fp16 in the permuted
 // fragment order [512-column slab][w][m][t][4 pairs], converted once, then
-// stored per layer with that layer's protected columns zeroed; scale_u *
-// x[b][j_u] of the protected columns (exact in fp32: 11 x 8 significant
-// bits) is taken from the same cache lines, so the activations cost one
-// round trip to memory.  Job = one 32-column group of one row.  Pair i of a
+// stored per layer with that layer's protected columns zeroed; then
+// scale_u * x[b][j_u] of the protected columns (exact in fp32: 11 x 8
+// significant bits) in a flat second loop, whose loads are all independent
+// (gathering them inside the first loop put a dependent round trip on every
+// job with a protected column: 7 us of a 17.6 us launch at batch 16).
+// Job = one 32-column group of one row.  Pair i of a
 // 32-column group is element i&7 of chunk (i>>3) and of chunk (i>>3)+2 --
 // bits i and i+16 of its code word, columns (i>>3)*8 + (i&7) and that + 16.
 template <int MAXG, bool kHalfXs = false, int kBatch = 1>
@@ -144,7 +148,6 @@ __device__ __forceinline__ void stage_activations(const uint16_t *x, int K, int 
             const int b = sb / nnar, slab = sb - b * nnar;
             const int g32 = slab * 16 + t * 4 + w;
             const int dst_off = b * xt_pitch + slab * 1024 + t * 16 + w * 256;
-            const uint16_t *src = x + static_cast<int64_t>(b) * K + k_begin + g32 * 32;
             uint32_t o[16];
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
@@ -167,21 +170,7 @@ __device__ __forceinline__ void stage_activations(const uint16_t *x, int K, int 
                             make_uint4(o[4 * m], o[4 * m + 1], o[4 * m + 2], o[4 * m + 3]);
                     continue;
                 }
-                // protected columns of this group: record scale * x, zero the halves
-                const int u0 = v[g].pu[g32];   // protected columns before this group
-                for (uint32_t bits = pm; bits; bits &= bits - 1u) {
-                    const int k = __ffs(bits) - 1;
-                    const int u = u0 + __popc(pm & ((1u << k) - 1u));
-                    const float sx = v[g].pscale[u] * bf16_bits_to_f32(src[k]);
-                    if constexpr (kHalfXs) {
-                        __half *xh = reinterpret_cast<__half *>(v[g].xs);
-                        const __half hi = __float2half_rn(sx);
-                        xh[b * cap + u] = hi;
-                        xh[(B + b) * cap + u] = __float2half_rn(sx - __half2float(hi));
-                    } else {
-                        v[g].xs[b * cap + u] = sx;
-                    }
-                }
+                // protected columns of this group: zero their halves
                 uint32_t om[16];
 #pragma unroll
                 for (int j = 0; j < 16; ++j) {
@@ -194,6 +183,24 @@ __device__ __forceinline__ void stage_activations(const uint16_t *x, int K, int 
                 for (int m = 0; m < 4; ++m)
                     *reinterpret_cast<uint4 *>(dst + m * 64) =
                         make_uint4(om[4 * m], om[4 * m + 1], om[4 * m + 2], om[4 * m + 3]);
+            }
+        }
+    }
+    // scale * x of every protected column of every layer and row
+#pragma unroll
+    for (int g = 0; g < MAXG; ++g) {
+        if (g >= G) break;
+        const int np = v[g].np;
+        for (int e = threadIdx.x; e < B * np; e += nthr) {
+            const int b = e / np, u = e - b * np;
+            const float sx = v[g].pscale[u] * bf16_bits_to_f32(x[static_cast<int64_t>(b) * K + v[g].pidx[u]]);
+            if constexpr (kHalfXs) {
+                __half *xh = reinterpret_cast<__half *>(v[g].xs);
+                const __half hi = __float2half_rn(sx);
+                xh[b * cap + u] = hi;
+                xh[(B + b) * cap + u] = __float2half_rn(sx - __half2float(hi));
+            } else {
+                v[g].xs[b * cap + u] = sx;
             }
         }
     }
@@ -476,7 +483,7 @@ k_gemv(const __grid_constant__ CUtensorMap tm_codes, const __grid_constant__ CUt
     // activations may be written by the previous kernel
     pdl_wait();
     {
-        StageView v[1] = {{sm + a.off_xt, s_pmask, s_pu, s_pscale, s_xs}};
+        StageView v[1] = {{sm + a.off_xt, s_pmask, s_pu, s_pscale, s_xs, s_pidx, p_loc}};
         stage_activations<1>(a.x, a.K, a.B, k_begin, k_end - k_begin, nnar, a.xt_pitch, a.pidx_cap,
                              1, v);
     }
@@ -1058,7 +1065,9 @@ k_gemv_stream(const __grid_constant__ StreamArgs<MAXG> a) {
         StageView v[MAXG] = {};
 #pragma unroll
         for (int g = 0; g < MAXG; ++g)
-            if (g < G) v[g] = {xt_of(g), pmask_of(g), pu_of(g), pscale_of(g), xs_of(g)};
+            if (g < G)
+                v[g] = {xt_of(g), pmask_of(g), pu_of(g), pscale_of(g), xs_of(g), pidx_of(g),
+                        s_lohi[g][1] - s_lohi[g][0]};
         stage_activations<MAXG, true>(x, K, B, 0, K, nnar, xt_pitch, cap, G, v);
         for (int i = threadIdx.x; i < 1024 / 16; i += blockDim.x)
             reinterpret_cast<uint4 *>(sm + off_zero)[i] = make_uint4(0, 0, 0, 0);
