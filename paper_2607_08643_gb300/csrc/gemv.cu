@@ -732,31 +732,41 @@ __device__ __forceinline__ void lut_slot(uint32_t cs, uint32_t ns, uint32_t tab,
         for (int j = 0; j < 4; ++j)
             base[m][j] = static_cast<uint32_t>(lane) * 4u + (j & 1) * 128u + (((j < 2 ? g0 : g1) >> 4) << 16);
     }
-#pragma unroll 1
-    for (int s = 0; s < S; ++s) {
+    // every code and norm word of the slot first, so that no lookup waits
+    // behind another stage's or row's code load
+    uint32_t cw[S][R][2];
+    uint2 nw[S][R][2];
+#pragma unroll
+    for (int s = 0; s < S; ++s)
 #pragma unroll
         for (int r = 0; r < R; ++r) {
             const uint32_t crow = cs + (s * 16 + row0 + r) * kCodeRow + lane * 4;
             const uint32_t nrow = ns + (s * 16 + row0 + r) * kNormRow + lane * 8;
 #pragma unroll
             for (int m = 0; m < 2; ++m) {
-                const uint32_t cw = lds_u32(crow + m * 128);
-                const uint2 nw = lds_u64(nrow + m * 256);
-                const uint32_t wl = lop3_and_or(cw, 0x0F0F0F0Fu, sgpat[m]);
-                const uint32_t wh = lop3_and_or(cw >> 4, 0x0F0F0F0Fu, sgpat[m]);
+                cw[s][r][m] = lds_u32(crow + m * 128);
+                nw[s][r][m] = lds_u64(nrow + m * 256);
+            }
+        }
+#pragma unroll
+    for (int s = 0; s < S; ++s)
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+#pragma unroll
+            for (int m = 0; m < 2; ++m) {
+                const uint32_t wl = lop3_and_or(cw[s][r][m], 0x0F0F0F0Fu, sgpat[m]);
+                const uint32_t wh = lop3_and_or(cw[s][r][m] >> 4, 0x0F0F0F0Fu, sgpat[m]);
 #pragma unroll
                 for (int j = 0; j < 4; ++j) {
                     const uint32_t sel = 0x7604u | (static_cast<uint32_t>(j) << 4);
                     const uint32_t tl = lds_u32(tab + prmt(wl, base[m][j], sel));
                     const uint32_t th = lds_u32(tab + prmt(wh, base[m][j], sel));
-                    const uint32_t nj = j < 2 ? nw.x : nw.y;
+                    const uint32_t nj = j < 2 ? nw[s][r][m].x : nw[s][r][m].y;
                     const uint16_t n = (j & 1) ? hi_half(nj) : lo_half(nj);
                     acc[r] = fma_f16_f32(lo_half(tl), n, acc[r]);
                     acc[r] = fma_f16_f32(hi_half(th), n, acc[r]);
                 }
             }
-        }
-    }
 }
 
 // A launch over several layers shares one set of tables built from x itself,
