@@ -11,7 +11,7 @@ Functions and the paper passages they follow:
 * :func:`encode`            Sec. III-E Eq. 8 (protected columns), Eq. 10 (Q8),
                             Sec. III-C Eq. 3 and Sec. III-D Eq. 5-7 (stages)
 * :func:`select_protected`  Eq. 8
-* :func:`decode_rows`       Sec. III-F Eq. 12 with the Eq. 10 scatter
+* :func:`decode_rows`       Sec. III-G Eq. 12 with the Eq. 10 scatter
 * :func:`matmul`            y = What x (plain definition)
 * :func:`apply_rows`        decode + matmul on a list of rows
 * :func:`double_to_fp16`, :func:`fp16_to_double`, :func:`bf16_to_double`

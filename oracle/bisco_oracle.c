@@ -17,7 +17,7 @@
  *            decoder read as "rescale the unit code by the chunk's stored
  *            fp16 L2 norm", and Sec. III-D Eq. 5-7 (residual stages
  *            r(s) = r(s-1) - rhat(s)).
- *   decode   Sec. III-F Eq. 12 (stages decoded independently and summed)
+ *   decode   Sec. III-G Eq. 12 (stages decoded independently and summed)
  *            with the Eq. 10 scatter of the protected columns.
  *   matmul   y[b][i] = sum_j What[i][j] * x[b][j]  (plain definition).
  *

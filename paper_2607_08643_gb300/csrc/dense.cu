@@ -1,5 +1,5 @@
 // dense.cu -- the coded layer decoded to a dense matrix in device memory
-// (Sec. III-F Eq. 12 with the Eq. 10 overwrite):
+// (Sec. III-G Eq. 12 with the Eq. 10 overwrite):
 //     What[i][j] = sum_s (bit_{s,i,j} ? -1 : +1) * n16_{s,i,j/8} / sqrt(8)   j not protected
 //     What[i][j] = scale_j * q8[i][j]                                         j protected
 // This is the materialise-then-multiply path (the decoded weight written to

@@ -1,4 +1,4 @@
-// gemm.cu -- prefill Y = X What^T (Sec. III-F Eq. 12 with the Eq. 10
+// gemm.cu -- prefill Y = X What^T (Sec. III-G Eq. 12 with the Eq. 10
 // protected scatter) on the 5th-generation tensor cores.
 //
 // Prefill is a dense contraction, so the decoded weight feeds tcgen05.mma

@@ -1,5 +1,5 @@
 // gemv.cu -- decode-time y = What x straight from the coded layer
-// (Sec. III-F Eq. 12 with the Eq. 10 protected scatter), batch 1..16.
+// (Sec. III-G Eq. 12 with the Eq. 10 protected scatter), batch 1..16.
 //
 // Shared decode scheme (GB300, HBM-bound):
 //  * A producer thread streams ring slots of the sign bytes and fp16 norms
