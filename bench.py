@@ -45,9 +45,12 @@ def parse():
     ap.add_argument("--impl", choices=("bisco", "reference"), default="bisco")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
-    ap.add_argument("--mode", choices=("both", "decode", "prefill", "shapes", "dense"), default="both",
+    ap.add_argument("--mode", choices=("both", "decode", "prefill", "shapes", "dense", "lora"),
+                    default="both",
                     help="decode: the GEMV step only; prefill: the tcgen05 GEMM only; "
-                         "shapes: batch-1 GEMV per Qwen3-8B layer shape")
+                         "shapes: batch-1 GEMV per Qwen3-8B layer shape; lora: the decode step "
+                         "with a low-rank compensation on every projection")
+    ap.add_argument("--lora-rank", type=int, default=16)
     ap.add_argument("--shape-mb", type=float, default=500.0,
                     help="--mode shapes: MB of distinct coded layers per shape (> L2)")
     ap.add_argument("--prefill-tokens", type=int, default=2048)
@@ -513,6 +516,107 @@ def run_dense(args, local_rank):
             "dense_gbs": dense_bytes / (ms * 1e-3) / 1e9, "batch": B}
 
 
+# ------------------------------------------------------------------- lora
+
+def run_lora(args, local_rank):
+    """Low-rank compensation (bisco_lora_apply, rank --lora-rank) on every
+    projection of the 36-layer q/k/v/o decode step.  Times the step with and
+    without it (CUDA graphs of the same calls, CUDA events over `steps`
+    replays) and the compensation alone: a graph of its calls for every
+    projection, timed replay by replay with L2 flushed in between (the
+    adapters of the stack are smaller than L2).  Adapter bytes are
+    rank * (K + N) bf16 per projection; the roofline counts those plus x, t
+    and the read-modify-write of y."""
+    import torch
+    from paper_2607_08643_gb300 import bisco
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    bisco.load()
+    layers = build_layers(args, dev)
+    B, K, R = args.batch, 4096, args.lora_rank
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(4242)
+    adapters = []
+    for _, L in layers:
+        A = (torch.randn((R, L.K), generator=gen, device=dev) / L.K ** 0.5).to(torch.bfloat16)
+        Bm = (torch.randn((L.N, R), generator=gen, device=dev) * 0.02).to(torch.bfloat16)
+        adapters.append((A, Bm))
+    x = torch.randn((2 * args.layers, B, K), generator=gen, device=dev).to(torch.bfloat16)
+    ys = [torch.zeros((B, L.N), dtype=torch.float32, device=dev) for _, L in layers]
+    t = torch.empty((B, R), dtype=torch.float32, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step(with_lora, with_gemv=True):
+        for li in range(args.layers):
+            q = [4 * li + j for j in range(3)]
+            if with_gemv:
+                bisco.bisco_gemv_multi([layers[i][1] for i in q], x[2 * li],
+                                       ys=[ys[i] for i in q], stream=stream)
+            if with_lora:
+                for i in q:
+                    bisco.bisco_lora_apply(*adapters[i], x[2 * li], ys[i], 1.0, t=t, stream=stream)
+            o = 4 * li + 3
+            if with_gemv:
+                bisco.bisco_gemv(layers[o][1], x[2 * li + 1], y=ys[o], stream=stream)
+            if with_lora:
+                bisco.bisco_lora_apply(*adapters[o], x[2 * li + 1], ys[o], 1.0, t=t, stream=stream)
+
+    graphs = {}
+    for key, (wl, wg) in {"plain": (False, True), "lora": (True, True), "only": (True, False)}.items():
+        with torch.cuda.stream(stream):
+            step(wl, wg)
+            torch.cuda.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                step(wl, wg)
+        graphs[key] = g
+    torch.cuda.synchronize()
+    if bisco.bisco_get_device_error(stream) != bisco.OK:
+        raise RuntimeError("device error in the lora step")
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ms = {}
+    for key in ("plain", "lora"):
+        for _ in range(max(args.warmup, 3)):
+            graphs[key].replay()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(args.steps):
+                graphs[key].replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        ms[key] = e0.elapsed_time(e1) / args.steps
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    only = []
+    for it in range(max(args.warmup, 3) + args.steps):
+        with torch.cuda.stream(stream):
+            flush.fill_(it & 255)
+            e0.record(stream)
+            graphs["only"].replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        if it >= max(args.warmup, 3):
+            only.append(e0.elapsed_time(e1))
+    ms_only = sum(only) / len(only)
+    calls = len(layers)
+    adapter_bytes = sum((A.numel() + Bm.numel()) * 2 for A, Bm in adapters)
+    io_bytes = sum(B * (L.K * 2 + L.N * 8) + 2 * B * R * 4 for _, L in layers)
+    peak, peak_kind = peaks()
+    gbs = (adapter_bytes + io_bytes) / (ms_only * 1e-3) / 1e9
+    return {"metric": "decode step with low-rank compensation on every projection",
+            "rank": R, "batch": B, "layers": args.layers,
+            "step_ms_without": ms["plain"], "step_ms_with": ms["lora"],
+            "overhead_pct": 100.0 * (ms["lora"] / ms["plain"] - 1.0),
+            "tokens_per_s_with": B / (ms["lora"] * 1e-3),
+            "compensation_alone": {"ms_per_step": ms_only, "calls": calls,
+                                   "us_per_call": ms_only * 1e3 / calls,
+                                   "adapter_bytes": adapter_bytes, "io_bytes": io_bytes,
+                                   "gbs": gbs, "frac_of_hbm": gbs / peak,
+                                   "peak_source": peak_kind,
+                                   "l2": "flushed (256 MB write) before every replay"},
+            "kernels": "k_lora_down + k_lora_up per projection"}
+
+
 # ----------------------------------------------------------------- shapes
 
 def run_shapes(args, local_rank):
@@ -660,6 +764,12 @@ def main():
             print(json.dumps({"metric": "batch-1 GEMV GB/s per Qwen3-8B shape (compressed bytes)",
                               "unit": "GB/s", "hbm_peak_gbs": peaks()[0], "steps": args.steps,
                               "data": "synthetic", "shapes": res}))
+        return
+    if args.mode == "lora":
+        lr = run_lora(args, local_rank)
+        if rank == 0:
+            print(json.dumps(dict(lr, n_gpus=world, steps=args.steps, warmup=args.warmup,
+                                  data="synthetic", config=workload_config(args))))
         return
     if args.mode == "dense":
         dn = run_dense(args, local_rank)

@@ -8,7 +8,7 @@
  * residual left by the earlier ones (Sec. III-D, Eq. 5-7), a small set of
  * input channels chosen by Eq. 8 is kept in 8 bits instead (Sec. III-E,
  * Eq. 10), and inference decodes the stages independently and sums them
- * (Sec. III-F, Eq. 12) before the linear map y = W x.  This library runs
+ * (Sec. III-G, Eq. 12) before the linear map y = W x.  This library runs
  * that linear map straight from the coded bytes, without ever writing the
  * dense weight to memory.
  *
@@ -82,7 +82,7 @@ typedef struct {
 } bisco_layer;
 
 /* ABI version of this header (major * 100 + minor). */
-#define BISCO_ABI_VERSION 103
+#define BISCO_ABI_VERSION 104
 int32_t bisco_abi_version(void);
 
 /* Static string for a status code (never NULL). */
@@ -146,7 +146,7 @@ bisco_status bisco_encode_noalloc(const uint16_t *W_bf16, const float *g, const 
 
 /*
  * Decode-time matrix-vector product for B in [0, 16] activation rows:
- *     y[b][i] = sum_j What[i][j] * x[b][j]        (Sec. III-F Eq. 12, Eq. 10)
+ *     y[b][i] = sum_j What[i][j] * x[b][j]        (Sec. III-G Eq. 12, Eq. 10)
  * computed straight from the coded layer (the dense weight is never
  * formed).  x_bf16: [B][K] device bf16 bits; activations are used as fp16,
  * which is exact for 2^-24 <= |x| <= 65504 (larger magnitudes become inf).
@@ -162,7 +162,7 @@ bisco_status bisco_gemv(const bisco_layer *L, const uint16_t *x_bf16, int32_t B,
 
 /*
  * bisco_gemv for G layers that read the same activations, for example the
- * q, k and v projections of one attention layer (Sec. III-F Eq. 12 for each):
+ * q, k and v projections of one attention layer (Sec. III-G Eq. 12 for each):
  *     y[g][b][i] = sum_j What_g[i][j] * x[b][j]      for g < G
  * in one launch, so the fixed per-launch latency (dependency release,
  * activation staging, reduction tail) is paid once for the group.
@@ -179,7 +179,7 @@ bisco_status bisco_gemv_multi(const bisco_layer *layers, int32_t G, const uint16
 
 /*
  * Prefill matrix product Y[m][i] = sum_j What[i][j] * X[m][j] for any M >= 0
- * (Sec. III-F Eq. 12 with Eq. 10), the same quantity as bisco_gemv.  For
+ * (Sec. III-G Eq. 12 with Eq. 10), the same quantity as bisco_gemv.  For
  * M > 64 and K % 128 == 0 it runs on the tcgen05 tensor cores: the decoded
  * weight (fp16, the S stages summed in fp16 -- one rounding of relative
  * size <= 2^-11 per weight for S >= 2) against fp16 activations, fp32
@@ -196,7 +196,7 @@ bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M,
                         void *workspace, size_t workspace_bytes, bisco_stream_t stream);
 
 /*
- * The coded layer decoded to a dense row-major matrix (Sec. III-F Eq. 12
+ * The coded layer decoded to a dense row-major matrix (Sec. III-G Eq. 12
  * with the Eq. 10 overwrite), the materialise-then-multiply alternative to
  * the fused kernels:
  *     out[i][j] = sum_s (bit ? -1 : +1) * n16_{s,i,j/8} / sqrt(8)   j not protected
@@ -212,6 +212,26 @@ bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M,
 #define BISCO_DENSE_F16 2
 bisco_status bisco_decode_dense(const bisco_layer *L, void *out, int32_t dtype,
                                 bisco_stream_t stream);
+
+/*
+ * Low-rank compensation (the optional LoRA path of Sec. II-D and Sec. III-F:
+ * adapters trained after the codes are fixed, kept apart from the coded
+ * layer's storage), added to an output the layer has already written:
+ *     t[b][r]  = sum_k A[r][k] * x[b][k]                (fp32 accumulation)
+ *     y[b][n] += scale * sum_r Bm[n][r] * t[b][r]        (fp32)
+ * A: [rank][K] bf16 and Bm: [N][rank] bf16 (the layouts of a PyTorch
+ * lora_A / lora_B weight); x_bf16: [batch][K]; y: [batch][N] float32, read
+ * and written (call it after bisco_gemv / bisco_gemm on the same stream);
+ * t: [batch][rank] float32 scratch, overwritten.  K >= 8, K % 8 == 0,
+ * N >= 1, 8 <= rank <= BISCO_LORA_MAX_RANK with rank % 8 == 0,
+ * 1 <= batch <= 65535, scale finite; else BISCO_ERR_INVALID_ARG.  Every
+ * pointer 16-byte aligned.  Asynchronous on `stream` (two kernels); the
+ * result does not depend on the launch (fixed summation order).
+ */
+#define BISCO_LORA_MAX_RANK 256
+bisco_status bisco_lora_apply(const uint16_t *A, const uint16_t *Bm, int32_t rank, int32_t N,
+                              int32_t K, float scale, const uint16_t *x_bf16, int32_t batch,
+                              float *y, float *t, bisco_stream_t stream);
 
 /*
  * A protected-column index outside [0, K) (or a list that is not ascending)

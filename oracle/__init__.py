@@ -13,6 +13,8 @@ Functions and the paper passages they follow:
 * :func:`select_protected`  Eq. 8
 * :func:`decode_rows`       Sec. III-G Eq. 12 with the Eq. 10 scatter
 * :func:`matmul`            y = What x (plain definition)
+* :func:`lora_apply`        y0 + scale * Bm (A x), the optional low-rank
+                            compensation of Sec. III-F (plain definition)
 * :func:`apply_rows`        decode + matmul on a list of rows
 * :func:`double_to_fp16`, :func:`fp16_to_double`, :func:`bf16_to_double`
                             the number formats the storage uses
@@ -86,6 +88,8 @@ def _load():
         lib.or_matmul.argtypes = [P, i32, i32, P, i32, P]
         lib.or_apply_rows.restype = ctypes.c_int
         lib.or_apply_rows.argtypes = [P, P, P, P, P, i32, i32, i32, i32, P, i32, P, i32, P]
+        lib.or_lora_apply.restype = ctypes.c_int
+        lib.or_lora_apply.argtypes = [P, P, i32, i32, i32, ctypes.c_double, P, i32, P, P]
         del i64
         _lib = lib
         return lib
@@ -197,6 +201,26 @@ def matmul(What, X_bits):
     B = X_bits.shape[0]
     Y = np.zeros((B, nrows), np.float64)
     _load().or_matmul(_ptr(What), nrows, K, _ptr(X_bits), B, _ptr(Y))
+    return Y
+
+
+def lora_apply(A_bits, Bm_bits, X_bits, Y0, scale=1.0):
+    """Y0 + scale * (X A^T) Bm^T in float64: A [rank][K], Bm [N][rank] and
+    X [B][K] as bf16 bits, Y0 [B][N]."""
+    A_bits = _c(A_bits, np.uint16)
+    Bm_bits = _c(Bm_bits, np.uint16)
+    X_bits = _c(np.atleast_2d(X_bits), np.uint16)
+    rank, K = A_bits.shape
+    N = Bm_bits.shape[0]
+    B = X_bits.shape[0]
+    if Bm_bits.shape[1] != rank or X_bits.shape[1] != K:
+        raise OracleError(ERR_INVALID_ARG)
+    Y0 = _c(np.asarray(Y0, np.float64).reshape(B, N), np.float64)
+    Y = np.zeros((B, N), np.float64)
+    rc = _load().or_lora_apply(_ptr(A_bits), _ptr(Bm_bits), rank, N, K, float(scale),
+                               _ptr(X_bits), B, _ptr(Y0), _ptr(Y))
+    if rc:
+        raise OracleError(rc)
     return Y
 
 

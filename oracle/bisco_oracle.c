@@ -20,6 +20,9 @@
  *   decode   Sec. III-G Eq. 12 (stages decoded independently and summed)
  *            with the Eq. 10 scatter of the protected columns.
  *   matmul   y[b][i] = sum_j What[i][j] * x[b][j]  (plain definition).
+ *   lora     y[b][n] + scale * sum_r Bm[n][r] * (sum_k A[r][k] * x[b][k]),
+ *            the optional low-rank compensation of Sec. III-F (plain
+ *            definition, the adapter's down projection first).
  *
  * Storage format produced by encode (identical bytes are required from the
  * GPU encoder):
@@ -339,5 +342,35 @@ int or_apply_rows(const uint8_t *codes, const uint16_t *norms,
     }
     free(w);
     free(y);
+    return OR_OK;
+}
+
+/* Low-rank compensation added to a layer output (Sec. III-F: LoRA adapters
+ * trained with the codes fixed).  A [rank][K], Bm [N][rank] and X [B][K] are
+ * bf16 bits, Y0 [B][N] the output before compensation.  First
+ * t[b][r] = sum_k A[r][k] x[b][k] (ascending k), then
+ * Y[b][n] = Y0[b][n] + scale * sum_r Bm[n][r] t[b][r] (ascending r). */
+int or_lora_apply(const uint16_t *A, const uint16_t *Bm, int32_t rank, int32_t N, int32_t K,
+                  double scale, const uint16_t *X, int32_t B, const double *Y0, double *Y)
+{
+    if (rank < 1 || N < 1 || K < 1 || B < 1) return OR_ERR_INVALID_ARG;
+    double *t = (double *)malloc(sizeof(double) * (size_t)rank);
+    if (!t) return OR_ERR_INVALID_ARG;
+    for (int32_t b = 0; b < B; ++b) {
+        for (int32_t r = 0; r < rank; ++r) {
+            double acc = 0.0;
+            for (int32_t k = 0; k < K; ++k)
+                acc = acc + or_bf16_to_double(A[(int64_t)r * K + k]) *
+                            or_bf16_to_double(X[(int64_t)b * K + k]);
+            t[r] = acc;
+        }
+        for (int32_t n = 0; n < N; ++n) {
+            double acc = 0.0;
+            for (int32_t r = 0; r < rank; ++r)
+                acc = acc + or_bf16_to_double(Bm[(int64_t)n * rank + r]) * t[r];
+            Y[(int64_t)b * N + n] = Y0[(int64_t)b * N + n] + scale * acc;
+        }
+    }
+    free(t);
     return OR_OK;
 }

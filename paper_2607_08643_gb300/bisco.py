@@ -19,7 +19,8 @@ EXPORTS = (
     "bisco_abi_version", "bisco_status_string", "bisco_encoded_sizes",
     "bisco_encode_workspace_bytes", "bisco_encode", "bisco_encode_noalloc", "bisco_gemv",
     "bisco_gemv_multi",
-    "bisco_gemm_workspace_bytes", "bisco_gemm", "bisco_decode_dense", "bisco_get_device_error",
+    "bisco_gemm_workspace_bytes", "bisco_gemm", "bisco_decode_dense", "bisco_lora_apply",
+    "bisco_get_device_error",
 )
 
 DENSE_F32, DENSE_BF16, DENSE_F16 = 0, 1, 2
@@ -77,6 +78,8 @@ def load(path: str = LIB_PATH):
     lib.bisco_gemm.argtypes = [Lp, P, i32, P, P, sz, P]
     lib.bisco_decode_dense.restype = st
     lib.bisco_decode_dense.argtypes = [Lp, P, i32, P]
+    lib.bisco_lora_apply.restype = st
+    lib.bisco_lora_apply.argtypes = [P, P, i32, i32, i32, ctypes.c_float, P, i32, P, P, P]
     lib.bisco_get_device_error.restype = st
     lib.bisco_get_device_error.argtypes = [P]
     _lib = lib
@@ -271,6 +274,31 @@ def bisco_decode_dense(L: Layer, dtype: str = "f32", out=None, stream=None):
     _check(load().bisco_decode_dense(ctypes.byref(L.c), _ptr(out), code, _stream(stream)),
            "bisco_decode_dense")
     return out
+
+
+def bisco_lora_apply(A, Bm, x_bits, y, scale: float = 1.0, t=None, stream=None):
+    """y[B][N] += scale * (x A^T) Bm^T in place: the low-rank compensation of a
+    layer's output.  A [rank][K] and Bm [N][rank] bf16, x [B][K] bf16 bits,
+    y [B][N] float32; t [B][rank] float32 scratch (allocated if None)."""
+    import torch
+    if x_bits.dtype == torch.bfloat16:
+        x_bits = x_bits.view(torch.int16)
+    if x_bits.dim() == 1:
+        x_bits = x_bits.unsqueeze(0)
+    A = A.view(torch.int16) if A.dtype == torch.bfloat16 else A
+    Bm = Bm.view(torch.int16) if Bm.dtype == torch.bfloat16 else Bm
+    rank, K = A.shape
+    N = Bm.shape[0]
+    batch = x_bits.shape[0]
+    assert Bm.shape[1] == rank and x_bits.shape[1] == K and tuple(y.shape) == (batch, N)
+    assert A.is_contiguous() and Bm.is_contiguous() and x_bits.is_contiguous() and y.is_contiguous()
+    assert y.dtype == torch.float32
+    if t is None:
+        t = torch.empty((batch, rank), dtype=torch.float32, device=y.device)
+    _check(load().bisco_lora_apply(_ptr(A), _ptr(Bm), rank, N, K, float(scale), _ptr(x_bits),
+                                   batch, _ptr(y), _ptr(t), _stream(stream)),
+           "bisco_lora_apply")
+    return y
 
 
 def bisco_get_device_error(stream=None) -> int:

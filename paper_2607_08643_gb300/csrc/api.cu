@@ -6,6 +6,7 @@
 #include <cudaTypedefs.h>
 #include <stdint.h>
 
+#include <cmath>
 #include <mutex>
 
 #include "bisco_host.h"
@@ -229,6 +230,19 @@ bisco_status bisco_decode_dense(const bisco_layer *L, void *out, int32_t dtype,
     int *err = device_error_word(&st);
     if (!err) return st;
     return launch_decode_dense(*L, out, dtype, err, reinterpret_cast<cudaStream_t>(stream));
+}
+
+bisco_status bisco_lora_apply(const uint16_t *A, const uint16_t *Bm, int32_t rank, int32_t N,
+                              int32_t K, float scale, const uint16_t *x_bf16, int32_t batch,
+                              float *y, float *t, bisco_stream_t stream) {
+    if (rank < 8 || rank > BISCO_LORA_MAX_RANK || rank % 8 != 0) return BISCO_ERR_INVALID_ARG;
+    if (N < 1 || K < 8 || K % 8 != 0 || batch < 1 || batch > 65535) return BISCO_ERR_INVALID_ARG;
+    if (!std::isfinite(scale)) return BISCO_ERR_INVALID_ARG;
+    const void *ptrs[5] = {A, Bm, x_bf16, y, t};
+    for (const void *q : ptrs)
+        if (!q || !aligned16(q)) return BISCO_ERR_INVALID_ARG;
+    return launch_lora_apply(A, Bm, rank, N, K, scale, x_bf16, batch, y, t,
+                             reinterpret_cast<cudaStream_t>(stream));
 }
 
 bisco_status bisco_get_device_error(bisco_stream_t stream) {

@@ -34,4 +34,9 @@ bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *
 bisco_status launch_decode_dense(const bisco_layer &L, void *out, int dtype, int *err,
                                  cudaStream_t stream);
 
+// bisco_lora_apply's two kernels (arguments already validated).
+bisco_status launch_lora_apply(const uint16_t *A, const uint16_t *Bm, int rank, int N, int K,
+                               float scale, const uint16_t *x, int batch, float *y, float *t,
+                               cudaStream_t stream);
+
 }  // namespace bisco

@@ -87,6 +87,19 @@ def activations(B: int, K: int, seed: int, scale: float = 1.0) -> np.ndarray:
     return f32_to_bf16_bits((rng.standard_normal((B, K)) * scale).astype(np.float32))
 
 
+def lora_adapter(N: int, K: int, rank: int, seed: int, sigma_a: float = None,
+                 sigma_b: float = 0.02):
+    """bf16 bits of one synthetic low-rank adapter: A uint16[rank][K] with
+    N(0, 1/K) entries (unless sigma_a is given) and Bm uint16[N][rank] with
+    N(0, sigma_b^2) entries (a trained adapter, not the all-zero Bm of LoRA's
+    initialisation)."""
+    rng = np.random.default_rng(seed)
+    sa = (1.0 / np.sqrt(K)) if sigma_a is None else sigma_a
+    A = f32_to_bf16_bits((rng.standard_normal((rank, K)) * sa).astype(np.float32))
+    Bm = f32_to_bf16_bits((rng.standard_normal((N, rank)) * sigma_b).astype(np.float32))
+    return A, Bm
+
+
 # --------------------------------------------------- device-side generation
 
 def layer_weights_torch(N: int, K: int, seed: int, device, dist: str = "normal",

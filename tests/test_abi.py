@@ -35,7 +35,7 @@ def test_header_declarations_are_exported(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert bisco.bisco_abi_version() == 103
+    assert bisco.bisco_abi_version() == 104
     for code in range(6):
         assert bisco.status_string(code)
     assert bisco.status_string(99) == "unknown status"
@@ -151,3 +151,23 @@ def test_gemv_multi_validation(lib):
     odd = (ctypes.c_void_p * 2)(0x70000, 0x70004)                       # y[1] misaligned
     assert lib.bisco_gemv_multi(arr, 2, x, 1, odd, None) == bisco.ERR_INVALID_ARG
     assert lib.bisco_gemv_multi(arr, 2, x, 0, ys, None) == bisco.OK   # empty batch
+
+
+def test_lora_validation(lib):
+    A, Bm, x, y, t = (ctypes.c_void_p(a) for a in (0x10000, 0x20000, 0x30000, 0x40000, 0x50000))
+    f = lib.bisco_lora_apply
+    E = bisco.ERR_INVALID_ARG
+    for rank in (0, 4, 12, 264, -8):                                   # rank: 8..256, % 8
+        assert f(A, Bm, rank, 64, 64, 1.0, x, 1, y, t, None) == E
+    for N, K in ((0, 64), (64, 0), (64, 4), (64, 12)):                 # N >= 1, K >= 8, K % 8
+        assert f(A, Bm, 16, N, K, 1.0, x, 1, y, t, None) == E
+    for batch in (0, -1, 65536):
+        assert f(A, Bm, 16, 64, 64, 1.0, x, batch, y, t, None) == E
+    for scale in (float("nan"), float("inf"), -float("inf")):
+        assert f(A, Bm, 16, 64, 64, scale, x, 1, y, t, None) == E
+    ptrs = [A, Bm, x, y, t]
+    for i in range(5):                                                  # NULL, misaligned
+        for bad in (None, ctypes.c_void_p(0x60008)):
+            p = list(ptrs)
+            p[i] = bad
+            assert f(p[0], p[1], 16, 64, 64, 1.0, p[2], 1, p[3], p[4], None) == E

@@ -401,3 +401,70 @@ def test_encoded_sizes_closed_form():
     # algorithmic compressed bytes (unpadded q8), 1024 x 1024, S = 2, 1 %
     p = 11
     assert 2 * 1024 * 128 * 3 + 1024 * p + 6 * p == 797762
+
+
+# ------------------------------------------------- low-rank compensation
+
+def test_lora_exact_rational_brute_force():
+    """lora_apply against the exact rational value of y0 + s * Bm (A x) on a
+    tiny case: the fp64 result lies within the rounding bound of a sum of
+    K + rank + 2 terms."""
+    from fractions import Fraction
+    rank, N, K, B = 3, 5, 16, 2
+    A, Bm = synth.lora_adapter(N, K, rank, seed=11, sigma_a=0.25, sigma_b=0.5)
+    X = synth.activations(B, K, seed=12)
+    Y0 = synth.bf16_bits_to_f32(synth.activations(B, N, seed=13)).astype(np.float64)
+    scale = 0.75
+    got = oracle.lora_apply(A, Bm, X, Y0, scale)
+    fa, fb, fx = f64(A), f64(Bm), f64(X)
+    u = 2.0 ** -53
+    for b in range(B):
+        t = [sum(Fraction(fa[r, k]) * Fraction(fx[b, k]) for k in range(K)) for r in range(rank)]
+        tabs = [sum(abs(fa[r, k] * fx[b, k]) for k in range(K)) for r in range(rank)]
+        for n in range(N):
+            exact = Fraction(Y0[b, n]) + Fraction(scale) * sum(Fraction(fb[n, r]) * t[r]
+                                                               for r in range(rank))
+            mag = abs(Y0[b, n]) + scale * sum(abs(fb[n, r]) * tabs[r] for r in range(rank))
+            assert abs(got[b, n] - float(exact)) <= 2 * (K + rank + 2) * u * mag + 1e-300
+
+
+def test_lora_rank1_one_hot_closed_form():
+    """A rank-1 adapter on a one-hot activation adds s * Bm[n][0] * A[0][k]
+    to every output: one product, exact in fp64."""
+    N, K = 7, 24
+    A, Bm = synth.lora_adapter(N, K, 1, seed=21)
+    for k in (0, 5, K - 1):
+        x = np.zeros((1, K), np.uint16)
+        x[0, k] = bf16([1.0])[0]
+        y0 = np.arange(N, dtype=np.float64)[None, :] * 0.5
+        got = oracle.lora_apply(A, Bm, x, y0, 0.5)
+        want = y0[0] + 0.5 * f64(Bm)[:, 0] * f64(A)[0, k]
+        assert np.array_equal(got[0], want)
+
+
+def test_lora_against_product_matrix_and_invariants():
+    """The adapter's down projection first (oracle) against the product
+    matrix Bm A formed first (numpy, another association); doubling x
+    doubles the correction exactly; scale 0 returns y0 bit for bit; a
+    transposed Bm or a missing scale would fail."""
+    rank, N, K, B = 16, 48, 256, 3
+    A, Bm = synth.lora_adapter(N, K, rank, seed=31)
+    X = synth.activations(B, K, seed=32)
+    Y0 = synth.bf16_bits_to_f32(synth.activations(B, N, seed=33)).astype(np.float64)
+    got = oracle.lora_apply(A, Bm, X, Y0, 2.0)
+    want = Y0 + 2.0 * f64(X) @ (f64(Bm) @ f64(A)).T
+    assert np.max(np.abs(got - want)) <= 1e-12 * np.max(np.abs(want - Y0))
+    X2 = f32_bits_times_two(X)
+    zero = np.zeros_like(Y0)
+    assert np.array_equal(oracle.lora_apply(A, Bm, X2, zero, 1.0),
+                          2.0 * oracle.lora_apply(A, Bm, X, zero, 1.0))
+    assert np.array_equal(oracle.lora_apply(A, Bm, X, Y0, 0.0), Y0)
+
+
+def f32_bits_times_two(bits):
+    """bf16 bits of 2 * x (exponent + 1; the test values are normal and far
+    from overflow)."""
+    v = synth.bf16_bits_to_f32(bits)
+    assert np.all(np.abs(v[v != 0]) > 1e-30) and np.all(np.abs(v) < 1e30)
+    out = bf16(2.0 * v)
+    return out
