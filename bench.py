@@ -216,6 +216,29 @@ def build_layers(args, dev):
     return layers
 
 
+def max_over_ranks(values, world, device=None):
+    """Each value's maximum over the ranks, on every rank: the job ends when
+    its slowest replica does."""
+    if world <= 1:
+        return [float(v) for v in values]
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.cpu()]
+
+
+def replica_rates(world, bytes_per_step, batch, steps, ms_total, ms_e2e):
+    """Whole-job rates of `world` independent replicas, each of which ran
+    `steps` steps of `bytes_per_step` compressed bytes and `batch` tokens, from
+    the max-over-ranks device time and end-to-end time (ms)."""
+    ms_step = ms_total / steps
+    return {"ms_per_step": ms_step,
+            "gbs": world * bytes_per_step / (ms_step * 1e-3) / 1e9,
+            "tokens_per_s": world * batch / (ms_step * 1e-3),
+            "e2e_gbs": world * bytes_per_step / (ms_e2e / steps * 1e-3) / 1e9}
+
+
 def run_bisco(args, rank, world, local_rank):
     import torch
     import torch.distributed as dist
@@ -317,10 +340,7 @@ def run_bisco(args, rank, world, local_rank):
     barrier()
     ms_e2e = max(f0.elapsed_time(f1), wall_e2e * 1e3)
 
-    if world > 1:
-        t = torch.tensor([ms_total, ms_e2e], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_total, ms_e2e = float(t[0]), float(t[1])
+    ms_total, ms_e2e = max_over_ranks([ms_total, ms_e2e], world, device=dev)
 
     # dominant kernel: the grouped q/k/v launch (60 % of the step's bytes;
     # the q/o projections when ungrouped), timed alone on the same stream
@@ -353,10 +373,9 @@ def run_bisco(args, rank, world, local_rank):
     us_dom = d0.elapsed_time(d1) * 1e3 / (args.steps * len(dom_calls))
     bytes_dom = sum(layers[i][1].compressed_bytes for i in dom_calls[0])
 
-    ms_step = ms_total / args.steps
-    gbs = world * bytes_step / (ms_step * 1e-3) / 1e9
-    tok_s = world * B / (ms_step * 1e-3)
-    e2e_gbs = world * bytes_step / (ms_e2e / args.steps * 1e-3) / 1e9
+    rates = replica_rates(world, bytes_step, B, args.steps, ms_total, ms_e2e)
+    ms_step, gbs, tok_s, e2e_gbs = (rates["ms_per_step"], rates["gbs"], rates["tokens_per_s"],
+                                    rates["e2e_gbs"])
     launches = len(layers) if args.ungrouped else 2 * args.layers
     peak, peak_kind = peaks()
     achieved = bytes_dom / (us_dom * 1e-6) / 1e9
