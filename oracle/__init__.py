@@ -38,6 +38,9 @@ _BUILD = os.path.join(_HERE, "_build")
 _LIB = os.path.join(_BUILD, "libbisco_oracle.so")
 _lock = threading.Lock()
 _lib = None
+# Tests that plant a mistake in a copy of bisco_oracle.c point this at the
+# copy's build, to check that the pins catch it.
+_LIB_OVERRIDE = os.environ.get("BISCO_ORACLE_LIB")
 
 OK, ERR_INVALID_ARG, ERR_RANGE = 0, 1, 3
 
@@ -61,7 +64,7 @@ def _load():
     with _lock:
         if _lib is not None:
             return _lib
-        lib = ctypes.CDLL(build())
+        lib = ctypes.CDLL(_LIB_OVERRIDE or build())
         P = ctypes.c_void_p
         i32, i64 = ctypes.c_int32, ctypes.c_int64
         lib.or_bf16_to_double.restype = ctypes.c_double

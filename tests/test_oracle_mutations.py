@@ -1,0 +1,63 @@
+"""Planted mistakes: each case below copies bisco_oracle.c with one
+plausible slip (a dropped term, a wrong sign, index or bit order, a rounding
+mode), builds the copy, and runs the pin suite against it.  The pins must
+fail for every one of them -- otherwise they would not pin the oracle.  All
+of it runs on the CPU; nothing here touches the CUDA library."""
+import os
+import subprocess
+import sys
+
+import pytest
+
+import oracle
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+ROOT = os.path.dirname(HERE)
+
+# name -> (text in bisco_oracle.c, replacement)
+MUTATIONS = {
+    "residual_sign": ("v[k] = v[k] - rhat;", "v[k] = v[k] + rhat;"),
+    "mask_dropped_after_stage_1": ("if (prot[8 * c + k]) v[k] = 0.0;", ";"),
+    "bit_order_reversed": ("bits |= (uint8_t)(1u << k);", "bits |= (uint8_t)(1u << (7 - k));"),
+    "zero_encoded_negative": ("if (v[k] < 0.0) bits", "if (v[k] <= 0.0) bits"),
+    "decode_without_inv_sqrt8": ("double t = or_fp16_to_double(norms[e]) * inv_sqrt8;",
+                                 "double t = or_fp16_to_double(norms[e]);"),
+    "decode_drops_last_stage": ("for (int32_t s = 0; s < S; ++s) {\n                int64_t e",
+                                "for (int32_t s = 0; s < S - 1; ++s) {\n                int64_t e"),
+    "protected_scatter_missing": (
+        "o[idx[t]] = or_fp16_to_double(scale[t]) * (double)q8[(int64_t)i * pp + t];", ";"),
+    "q8_truncates": ("q = nearbyint(or_bf16_to_double(W[(int64_t)i * K + j]) / s);",
+                     "q = trunc(or_bf16_to_double(W[(int64_t)i * K + j]) / s);"),
+    "q8_divides_by_unrounded_scale": ("double s = or_fp16_to_double(s16);", "double s = m / 127.0;"),
+    "selection_ties_to_higher_index": ("return (x->j < y->j) ? -1 : (x->j > y->j);",
+                                       "return (x->j > y->j) ? -1 : (x->j < y->j);"),
+    "fp16_rounds_toward_zero": ("double m = nearbyint(ldexp(a, 10 - E));",
+                                "double m = floor(ldexp(a, 10 - E));"),
+    "matmul_reversed_activation": ("or_bf16_to_double(X[(int64_t)b * K + j]);",
+                                   "or_bf16_to_double(X[(int64_t)b * K + (K - 1 - j)]);"),
+    "lora_bm_transposed": ("or_bf16_to_double(Bm[(int64_t)n * rank + r]) * t[r];",
+                           "or_bf16_to_double(Bm[(int64_t)r * N + n]) * t[r];"),
+    "lora_scale_dropped": ("Y0[(int64_t)b * N + n] + scale * acc;", "Y0[(int64_t)b * N + n] + acc;"),
+}
+
+
+@pytest.fixture(scope="module")
+def source():
+    with open(os.path.join(ROOT, "oracle", "bisco_oracle.c")) as f:
+        return f.read()
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_pins_catch_planted_mistake(name, source, tmp_path):
+    old, new = MUTATIONS[name]
+    assert source.count(old) == 1, "mutation anchor not found once: " + name
+    src = tmp_path / "bisco_oracle_mutant.c"
+    src.write_text(source.replace(old, new))
+    lib = tmp_path / "libbisco_oracle_mutant.so"
+    subprocess.check_call(["gcc", *oracle.CFLAGS, "-o", str(lib), str(src), "-lm"])
+    env = dict(os.environ, BISCO_ORACLE_LIB=str(lib))
+    r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
+                        os.path.join(HERE, "test_oracle_pins.py")],
+                       cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    assert r.returncode == 1, "pins passed with the planted mistake %r:\n%s" % (
+        name, r.stdout[-2000:])
