@@ -171,3 +171,18 @@ def test_lora_validation(lib):
             p = list(ptrs)
             p[i] = bad
             assert f(p[0], p[1], 16, 64, 64, 1.0, p[2], 1, p[3], p[4], None) == E
+
+
+def test_binding_argument_counts_match_header(lib):
+    """Every prototype in bisco.h has as many parameters as the ctypes
+    binding declares for it (a drifted binding would pass garbage)."""
+    src = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    protos = re.findall(r"\b(bisco_[a-z_0-9]+)\s*\(([^;{]*?)\)\s*;", src, flags=re.S)
+    assert protos
+    seen = set()
+    for name, params in protos:
+        params = params.strip()
+        n = 0 if params in ("", "void") else params.count(",") + 1
+        assert len(getattr(lib, name).argtypes) == n, name
+        seen.add(name)
+    assert seen == set(bisco.EXPORTS)
