@@ -13,6 +13,11 @@ Functions and the paper passages they follow:
 * :func:`select_protected`  Eq. 8
 * :func:`decode_rows`       Sec. III-G Eq. 12 with the Eq. 10 scatter
 * :func:`matmul`            y = What x (plain definition)
+* :func:`select_rows`, :func:`select_coupled`, :func:`encode_rows`,
+  :func:`encode_given`, :func:`encode_coupled`
+                            output-row protection and the coupled MLP
+                            channel score (Sec. III-E Eq. 9) with Eq. 10 on
+                            rows; the CUDA library does not take this axis yet
 * :func:`lora_apply`        y0 + scale * Bm (A x), the optional low-rank
                             compensation of Sec. III-F (plain definition)
 * :func:`apply_rows`        decode + matmul on a list of rows
@@ -91,6 +96,16 @@ def _load():
         lib.or_matmul.argtypes = [P, i32, i32, P, i32, P]
         lib.or_apply_rows.restype = ctypes.c_int
         lib.or_apply_rows.argtypes = [P, P, P, P, P, i32, i32, i32, i32, P, i32, P, i32, P]
+        lib.or_select_rows.restype = ctypes.c_int
+        lib.or_select_rows.argtypes = [P, P, i32, i32, i32, P, P]
+        lib.or_select_coupled.restype = ctypes.c_int
+        lib.or_select_coupled.argtypes = [P, P, P, P, P, P, i32, i32, i32, P, P]
+        lib.or_quantize_protected_rows.restype = ctypes.c_int
+        lib.or_quantize_protected_rows.argtypes = [P, i32, i32, P, i32, P, P]
+        lib.or_encode_rows.restype = ctypes.c_int
+        lib.or_encode_rows.argtypes = [P, P, i32, i32, i32, i32, P, P, P, P, P, P]
+        lib.or_decode_rows_axis1.restype = None
+        lib.or_decode_rows_axis1.argtypes = [P, P, P, P, P, i32, i32, i32, i32, i32, i32, P]
         lib.or_lora_apply.restype = ctypes.c_int
         lib.or_lora_apply.argtypes = [P, P, i32, i32, i32, ctypes.c_double, P, i32, P, P]
         del i64
@@ -175,6 +190,102 @@ def encode(W_bits, S, p, g=None):
                 q8=q8[:, :pad16(p)].copy(), scale=scale[:p].copy(), idx=idx[:p].copy())
 
 
+def select_rows(W_bits, p, g=None):
+    """Output-row selection: returns (idx ascending int32[p], scores float64[N])."""
+    W_bits = _c(W_bits, np.uint16)
+    N, K = W_bits.shape
+    idx = np.zeros(max(p, 1), np.int32)
+    scores = np.zeros(N, np.float64)
+    gg = None if g is None else _c(g, np.float32)
+    rc = _load().or_select_rows(_ptr(W_bits), _ptr(gg), N, K, p, _ptr(idx), _ptr(scores))
+    if rc:
+        raise OracleError(rc)
+    return idx[:p].copy(), scores
+
+
+def select_coupled(Wg_bits, Wu_bits, Wd_bits, p, gg=None, gu=None, gd=None):
+    """Eq. 9: the coupled intermediate-channel set of a gated MLP (gate/up
+    [F][H], down [H][F]).  Returns (idx ascending int32[p], scores float64[F])."""
+    Wg_bits, Wu_bits, Wd_bits = (_c(w, np.uint16) for w in (Wg_bits, Wu_bits, Wd_bits))
+    F, H = Wg_bits.shape
+    if Wu_bits.shape != (F, H) or Wd_bits.shape != (H, F):
+        raise OracleError(ERR_INVALID_ARG)
+    idx = np.zeros(max(p, 1), np.int32)
+    scores = np.zeros(F, np.float64)
+    g3 = [None if g is None else _c(g, np.float32) for g in (gg, gu, gd)]
+    rc = _load().or_select_coupled(_ptr(Wg_bits), _ptr(Wu_bits), _ptr(Wd_bits), _ptr(g3[0]),
+                                   _ptr(g3[1]), _ptr(g3[2]), F, H, p, _ptr(idx), _ptr(scores))
+    if rc:
+        raise OracleError(rc)
+    return idx[:p].copy(), scores
+
+
+def encode_rows(W_bits, S, p, g=None, idx=None):
+    """Encoder with output-row protection (axis 1).  The protected rows come
+    from :func:`select_rows` unless ``idx`` gives them.  Returns a dict like
+    :func:`encode` with axis=1, q8 int8[p][pad16(K)], scale/idx per row."""
+    W_bits = _c(W_bits, np.uint16)
+    N, K = W_bits.shape
+    C = K // 8 if K % 8 == 0 else 1
+    kp = pad16(K)
+    codes = np.zeros((S, N, C), np.uint8)
+    norms = np.zeros((S, N, C), np.uint16)
+    q8 = np.zeros((max(p, 1), kp), np.int8)
+    scale = np.zeros(max(p, 1), np.uint16)
+    out_idx = np.zeros(max(p, 1), np.int32)
+    gg = None if g is None else _c(g, np.float32)
+    given = None if idx is None else _c(idx, np.int32)
+    if given is not None and len(given) != p:
+        raise OracleError(ERR_INVALID_ARG)
+    rc = _load().or_encode_rows(_ptr(W_bits), _ptr(gg), N, K, S, p, _ptr(given), _ptr(codes),
+                                _ptr(norms), _ptr(q8), _ptr(scale), _ptr(out_idx))
+    if rc:
+        raise OracleError(rc)
+    return dict(N=N, K=K, S=S, p=p, axis=1, codes=codes, norms=norms, q8=q8[:p].copy(),
+                scale=scale[:p].copy(), idx=out_idx[:p].copy())
+
+
+def encode_given(W_bits, S, idx):
+    """Column protection (axis 0) with a given ascending column set, e.g. the
+    down projection's share of the coupled MLP set: Eq. 10 on those columns,
+    then the stages on the masked complement."""
+    W_bits = _c(W_bits, np.uint16)
+    N, K = W_bits.shape
+    idx = _c(idx, np.int32)
+    p = len(idx)
+    if (K % 8 or np.any(idx < 0) or np.any(idx >= K) or np.any(np.diff(idx) <= 0)):
+        raise OracleError(ERR_INVALID_ARG)
+    if not np.all(np.isfinite(_bf16_bits_to_f64(W_bits))):
+        raise OracleError(ERR_RANGE)
+    q8 = np.zeros((N, max(pad16(p), 16)), np.int8)
+    scale = np.zeros(max(p, 1), np.uint16)
+    codes = np.zeros((S, N, K // 8), np.uint8)
+    norms = np.zeros((S, N, K // 8), np.uint16)
+    lib = _load()
+    idx_arg = idx if p else np.zeros(1, np.int32)
+    rc = lib.or_quantize_protected(_ptr(W_bits), N, K, _ptr(idx_arg), p, _ptr(q8), _ptr(scale))
+    if rc == 0:
+        rc = lib.or_encode_stages(_ptr(W_bits), N, K, S, _ptr(idx_arg), p, _ptr(codes), _ptr(norms))
+    if rc:
+        raise OracleError(rc)
+    return dict(N=N, K=K, S=S, p=p, codes=codes, norms=norms, q8=q8[:, :pad16(p)].copy(),
+                scale=scale[:p].copy(), idx=idx.copy())
+
+
+def encode_coupled(Wg_bits, Wu_bits, Wd_bits, S, p):
+    """Eq. 9 + Eq. 10 for a gated MLP: one protected intermediate set P
+    (:func:`select_coupled`), the rows P of gate and up and the columns P of
+    down kept in 8 bits.  Returns (gate, up, down) layer dicts."""
+    idx, _ = select_coupled(Wg_bits, Wu_bits, Wd_bits, p)
+    return (encode_rows(Wg_bits, S, p, idx=idx), encode_rows(Wu_bits, S, p, idx=idx),
+            encode_given(Wd_bits, S, idx))
+
+
+def _bf16_bits_to_f64(bits):
+    """bf16 bit patterns -> float64 (exact), without importing the generators."""
+    return (np.asarray(bits, np.uint16).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
 def _layer_args(L):
     codes = _c(L["codes"], np.uint8)
     norms = _c(L["norms"], np.uint16)
@@ -185,12 +296,23 @@ def _layer_args(L):
 
 
 def decode_rows(L, row0=0, nrows=None):
-    """Eq. 12 + Eq. 10: dense float64 rows [row0, row0+nrows) of What."""
+    """Eq. 12 + Eq. 10: dense float64 rows [row0, row0+nrows) of What (input
+    columns protected, or output rows for a layer with axis=1)."""
     N, K = L["N"], L["K"]
     if nrows is None:
         nrows = N - row0
-    codes, norms, q8, scale, idx = _layer_args(L)
     out = np.zeros((nrows, K), np.float64)
+    if L.get("axis", 0) == 1:
+        codes = _c(L["codes"], np.uint8)
+        norms = _c(L["norms"], np.uint16)
+        p = L["p"]
+        q8 = _c(L["q8"], np.int8) if p > 0 else np.zeros((1, pad16(K)), np.int8)
+        scale = _c(L["scale"], np.uint16) if p > 0 else np.zeros(1, np.uint16)
+        idx = _c(L["idx"], np.int32) if p > 0 else np.zeros(1, np.int32)
+        _load().or_decode_rows_axis1(_ptr(codes), _ptr(norms), _ptr(q8), _ptr(scale), _ptr(idx),
+                                     N, K, L["S"], p, row0, nrows, _ptr(out))
+        return out
+    codes, norms, q8, scale, idx = _layer_args(L)
     _load().or_decode_rows(_ptr(codes), _ptr(norms), _ptr(q8), _ptr(scale), _ptr(idx),
                            N, K, L["S"], L["p"], row0, nrows, _ptr(out))
     return out

@@ -20,6 +20,9 @@
  *   decode   Sec. III-G Eq. 12 (stages decoded independently and summed)
  *            with the Eq. 10 scatter of the protected columns.
  *   matmul   y[b][i] = sum_j What[i][j] * x[b][j]  (plain definition).
+ *   rows     output-row protection and the coupled MLP channel score of
+ *            Sec. III-E Eq. 9 (gate/up rows and down columns share one
+ *            protected set), with Eq. 10's 8-bit quantiser on the rows.
  *   lora     y[b][n] + scale * sum_r Bm[n][r] * (sum_k A[r][k] * x[b][k]),
  *            the optional low-rank compensation of Sec. III-F (plain
  *            definition, the adapter's down projection first).
@@ -374,3 +377,165 @@ int or_lora_apply(const uint16_t *A, const uint16_t *Bm, int32_t rank, int32_t N
     free(t);
     return OR_OK;
 }
+
+/* ------------------------------- output-row protection (Eq. 9, Eq. 10) */
+
+/* score_i = g_i * sqrt(sum_k W_ik^2) (ascending k) for output row i; P = the
+ * p rows of largest score, ties to the lower index, returned ascending. */
+int or_select_rows(const uint16_t *W, const float *g, int32_t N, int32_t K, int32_t p,
+                   int32_t *idx_out, double *scores_out)
+{
+    if (p < 0 || p > N) return OR_ERR_INVALID_ARG;
+    or_scored *sc = (or_scored *)malloc(sizeof(or_scored) * (size_t)N);
+    if (!sc) return OR_ERR_INVALID_ARG;
+    for (int32_t i = 0; i < N; ++i) {
+        double sum = 0.0;
+        for (int32_t k = 0; k < K; ++k) {
+            double w = or_bf16_to_double(W[(int64_t)i * K + k]);
+            sum = sum + w * w;
+        }
+        double s = sqrt(sum);
+        if (g) s = (double)g[i] * s;
+        sc[i].score = s;
+        sc[i].j = i;
+        if (scores_out) scores_out[i] = s;
+    }
+    qsort(sc, (size_t)N, sizeof(or_scored), or_cmp_scored);
+    for (int32_t t = 0; t < p; ++t) idx_out[t] = sc[t].j;
+    qsort(idx_out, (size_t)p, sizeof(int32_t), or_cmp_i32);
+    free(sc);
+    return OR_OK;
+}
+
+/* Eq. 9, the coupled score of intermediate channel j of a gated MLP:
+ *   S_j = gg_j ||Wg[j,:]||_2 + gu_j ||Wu[j,:]||_2 + gd_j ||Wd[:,j]||_2
+ * with Wg, Wu [F][H] (gate/up rows) and Wd [H][F] (down columns); each norm
+ * is the square root of a sum in ascending index, and the three terms are
+ * added in that order.  A NULL g means 1.  P = TopK_j, ties to the lower j,
+ * returned ascending. */
+int or_select_coupled(const uint16_t *Wg, const uint16_t *Wu, const uint16_t *Wd,
+                      const float *gg, const float *gu, const float *gd,
+                      int32_t F, int32_t H, int32_t p, int32_t *idx_out, double *scores_out)
+{
+    if (F <= 0 || H <= 0 || p < 0 || p > F) return OR_ERR_INVALID_ARG;
+    or_scored *sc = (or_scored *)malloc(sizeof(or_scored) * (size_t)F);
+    if (!sc) return OR_ERR_INVALID_ARG;
+    for (int32_t j = 0; j < F; ++j) {
+        double sg = 0.0, su = 0.0, sd = 0.0;
+        for (int32_t h = 0; h < H; ++h) {
+            double a = or_bf16_to_double(Wg[(int64_t)j * H + h]);
+            double b = or_bf16_to_double(Wu[(int64_t)j * H + h]);
+            sg = sg + a * a;
+            su = su + b * b;
+        }
+        for (int32_t h = 0; h < H; ++h) {
+            double c = or_bf16_to_double(Wd[(int64_t)h * F + j]);
+            sd = sd + c * c;
+        }
+        double tg = sqrt(sg), tu = sqrt(su), td = sqrt(sd);
+        if (gg) tg = (double)gg[j] * tg;
+        if (gu) tu = (double)gu[j] * tu;
+        if (gd) td = (double)gd[j] * td;
+        double s = (tg + tu) + td;
+        sc[j].score = s;
+        sc[j].j = j;
+        if (scores_out) scores_out[j] = s;
+    }
+    qsort(sc, (size_t)F, sizeof(or_scored), or_cmp_scored);
+    for (int32_t t = 0; t < p; ++t) idx_out[t] = sc[t].j;
+    qsort(idx_out, (size_t)p, sizeof(int32_t), or_cmp_i32);
+    free(sc);
+    return OR_OK;
+}
+
+/* Eq. 10 on protected rows, one scale per row (the protected channel):
+ *   scale_t = fp16(max_k |W_{i_t,k}| / 127)
+ *   q8[t][k] = clamp(rint(W_{i_t,k} / scale_t), -127, 127), or 0 if scale_t == 0
+ * q8 is [p][kp], kp = K rounded up to a multiple of 16, zero padding. */
+int or_quantize_protected_rows(const uint16_t *W, int32_t N, int32_t K,
+                               const int32_t *idx, int32_t p,
+                               int8_t *q8_out, uint16_t *scale_out)
+{
+    int32_t kp = or_pad16(K);
+    memset(q8_out, 0, (size_t)(p > 0 ? p : 0) * (size_t)kp);
+    for (int32_t t = 0; t < p; ++t) {
+        int32_t i = idx[t];
+        if (i < 0 || i >= N) return OR_ERR_INVALID_ARG;
+        double m = 0.0;
+        for (int32_t k = 0; k < K; ++k) {
+            double a = fabs(or_bf16_to_double(W[(int64_t)i * K + k]));
+            if (a > m) m = a;
+        }
+        uint16_t s16 = or_double_to_fp16(m / 127.0);
+        if ((s16 & 0x7c00) == 0x7c00) return OR_ERR_RANGE;
+        scale_out[t] = s16;
+        double s = or_fp16_to_double(s16);
+        for (int32_t k = 0; k < K; ++k) {
+            double q = 0.0;
+            if (s != 0.0) {
+                q = nearbyint(or_bf16_to_double(W[(int64_t)i * K + k]) / s);
+                if (q > 127.0) q = 127.0;
+                if (q < -127.0) q = -127.0;
+            }
+            q8_out[(int64_t)t * kp + k] = (int8_t)q;
+        }
+    }
+    return OR_OK;
+}
+
+/* Whole encoder with output-row protection.  P is selected by
+ * or_select_rows when idx_in is NULL, else taken from idx_in (ascending,
+ * e.g. the coupled MLP set of or_select_coupled).  The protected rows are
+ * zero in the BSQ target (masking, as for columns), so each of their chunks
+ * stores norm 0 and sign byte 0; the stages are or_encode_stages on that
+ * masked matrix with no protected columns. */
+int or_encode_rows(const uint16_t *W, const float *g, int32_t N, int32_t K, int32_t S,
+                   int32_t p, const int32_t *idx_in, uint8_t *codes, uint16_t *norms,
+                   int8_t *q8, uint16_t *scale, int32_t *idx)
+{
+    if (N <= 0 || K <= 0 || K % 8 != 0 || S < 1 || S > 3 || p < 0 || p > N)
+        return OR_ERR_INVALID_ARG;
+    for (int64_t e = 0; e < (int64_t)N * K; ++e)
+        if (!isfinite(or_bf16_to_double(W[e]))) return OR_ERR_RANGE;
+    int rc = OR_OK;
+    if (idx_in) {
+        for (int32_t t = 0; t < p; ++t) {
+            if (idx_in[t] < 0 || idx_in[t] >= N || (t > 0 && idx_in[t] <= idx_in[t - 1]))
+                return OR_ERR_INVALID_ARG;
+            idx[t] = idx_in[t];
+        }
+    } else {
+        rc = or_select_rows(W, g, N, K, p, idx, NULL);
+        if (rc) return rc;
+    }
+    rc = or_quantize_protected_rows(W, N, K, idx, p, q8, scale);
+    if (rc) return rc;
+    uint16_t *Wm = (uint16_t *)malloc(sizeof(uint16_t) * (size_t)N * (size_t)K);
+    if (!Wm) return OR_ERR_INVALID_ARG;
+    memcpy(Wm, W, sizeof(uint16_t) * (size_t)N * (size_t)K);
+    for (int32_t t = 0; t < p; ++t)
+        memset(Wm + (int64_t)idx[t] * K, 0, sizeof(uint16_t) * (size_t)K);
+    rc = or_encode_stages(Wm, N, K, S, NULL, 0, codes, norms);
+    free(Wm);
+    return rc;
+}
+
+/* Dense rows [row0, row0+nrows) of a row-protected layer:
+ *   What[i][:] = scale_t * q8[t][:]                  i = idx[t]
+ *   What[i][:] = the BSQ rows of Eq. 12              otherwise */
+void or_decode_rows_axis1(const uint8_t *codes, const uint16_t *norms,
+                          const int8_t *q8, const uint16_t *scale, const int32_t *idx,
+                          int32_t N, int32_t K, int32_t S, int32_t p,
+                          int32_t row0, int32_t nrows, double *out)
+{
+    int32_t kp = or_pad16(K);
+    or_decode_rows(codes, norms, NULL, NULL, NULL, N, K, S, 0, row0, nrows, out);
+    for (int32_t t = 0; t < p; ++t) {
+        int32_t i = idx[t];
+        if (i < row0 || i >= row0 + nrows) continue;
+        double s = or_fp16_to_double(scale[t]);
+        for (int32_t k = 0; k < K; ++k)
+            out[(int64_t)(i - row0) * K + k] = s * (double)q8[(int64_t)t * kp + k];
+    }
+}
+

@@ -28,13 +28,24 @@ MUTATIONS = {
         "o[idx[t]] = or_fp16_to_double(scale[t]) * (double)q8[(int64_t)i * pp + t];", ";"),
     "q8_truncates": ("q = nearbyint(or_bf16_to_double(W[(int64_t)i * K + j]) / s);",
                      "q = trunc(or_bf16_to_double(W[(int64_t)i * K + j]) / s);"),
-    "q8_divides_by_unrounded_scale": ("double s = or_fp16_to_double(s16);", "double s = m / 127.0;"),
+    "q8_divides_by_unrounded_scale": (
+        "double s = or_fp16_to_double(s16);\n        for (int32_t i = 0; i < N; ++i) {",
+        "double s = m / 127.0;\n        for (int32_t i = 0; i < N; ++i) {"),
+    "row_q8_divides_by_unrounded_scale": (
+        "double s = or_fp16_to_double(s16);\n        for (int32_t k = 0; k < K; ++k) {",
+        "double s = m / 127.0;\n        for (int32_t k = 0; k < K; ++k) {"),
     "selection_ties_to_higher_index": ("return (x->j < y->j) ? -1 : (x->j > y->j);",
                                        "return (x->j > y->j) ? -1 : (x->j < y->j);"),
     "fp16_rounds_toward_zero": ("double m = nearbyint(ldexp(a, 10 - E));",
                                 "double m = floor(ldexp(a, 10 - E));"),
     "matmul_reversed_activation": ("or_bf16_to_double(X[(int64_t)b * K + j]);",
                                    "or_bf16_to_double(X[(int64_t)b * K + (K - 1 - j)]);"),
+    "coupled_drops_down_term": ("double s = (tg + tu) + td;", "double s = tg + tu;"),
+    "rows_not_masked": ("memset(Wm + (int64_t)idx[t] * K, 0, sizeof(uint16_t) * (size_t)K);", ";"),
+    "row_scale_from_half_row": (
+        "for (int32_t k = 0; k < K; ++k) {\n            double a = fabs(or_bf16_to_double(W[(int64_t)i * K + k]));",
+        "for (int32_t k = 0; k < K / 2; ++k) {\n            double a = fabs(or_bf16_to_double(W[(int64_t)i * K + k]));"),
+    "row_decode_keeps_bsq": ("out[(int64_t)(i - row0) * K + k] = s * (double)q8[(int64_t)t * kp + k];", ";"),
     "lora_bm_transposed": ("or_bf16_to_double(Bm[(int64_t)n * rank + r]) * t[r];",
                            "or_bf16_to_double(Bm[(int64_t)r * N + n]) * t[r];"),
     "lora_scale_dropped": ("Y0[(int64_t)b * N + n] + scale * acc;", "Y0[(int64_t)b * N + n] + acc;"),

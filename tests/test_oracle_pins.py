@@ -468,3 +468,97 @@ def f32_bits_times_two(bits):
     assert np.all(np.abs(v[v != 0]) > 1e-30) and np.all(np.abs(v) < 1e30)
     out = bf16(2.0 * v)
     return out
+
+
+# ------------------------------------- output-row and coupled MLP protection
+
+def _outlier_rows(N, K, seed):
+    """bf16 bits [N][K] with 8 outlier rows (the generator's outlier columns of
+    the transposed shape)."""
+    return np.ascontiguousarray(synth.layer_weights(K, N, seed=seed).T)
+
+
+def test_row_selection_matches_full_sort_and_catches_outliers():
+    N, K, p = 96, 64, 10
+    W = _outlier_rows(N, K, seed=41)
+    idx, scores = oracle.select_rows(W, p)
+    norms = np.sqrt((f64(W) ** 2).sum(axis=1))
+    assert np.allclose(scores, norms, rtol=1e-14, atol=0)
+    order = sorted(range(N), key=lambda i: (-norms[i], i))
+    assert list(idx) == sorted(order[:p])
+    outliers = np.argsort(-np.abs(f64(W)).max(axis=1))[:8]
+    assert set(outliers.tolist()) <= set(idx.tolist())
+    # ties go to the lower row; g weights the rows
+    Wt = np.zeros((6, 8), np.uint16)
+    Wt[[1, 3, 4]] = bf16([0.5] * 8)
+    assert list(oracle.select_rows(Wt, 2)[0]) == [1, 3]
+    g = np.array([1, 1, 1, 0.5, 1, 1], np.float32)
+    assert list(oracle.select_rows(Wt, 2, g=g)[0]) == [1, 4]
+
+
+def test_coupled_score_is_the_sum_of_three_slice_norms():
+    """Eq. 9: gate row norm + up row norm + down column norm, TopK."""
+    F, H, p = 80, 48, 7
+    Wg = synth.layer_weights(F, H, seed=51)
+    Wu = synth.layer_weights(F, H, seed=52)
+    Wd = synth.layer_weights(H, F, seed=53)
+    idx, scores = oracle.select_coupled(Wg, Wu, Wd, p)
+    want = (np.sqrt((f64(Wg) ** 2).sum(1)) + np.sqrt((f64(Wu) ** 2).sum(1))
+            + np.sqrt((f64(Wd) ** 2).sum(0)))
+    assert np.allclose(scores, want, rtol=1e-14, atol=0)
+    assert list(idx) == sorted(sorted(range(F), key=lambda j: (-want[j], j))[:p])
+    # zero weight on gate and up leaves down's column selection (Eq. 8)
+    z = np.zeros(F, np.float32)
+    assert list(oracle.select_coupled(Wg, Wu, Wd, p, gg=z, gu=z)[0]) == \
+        list(oracle.select_protected(Wd, p)[0])
+    # zero weight on up and down leaves gate's row selection
+    assert list(oracle.select_coupled(Wg, Wu, Wd, p, gu=z, gd=z)[0]) == \
+        list(oracle.select_rows(Wg, p)[0])
+
+
+def test_row_protection_encode_and_decode():
+    """Eq. 10 on rows: one scale per protected row (closed form with numpy's
+    fp16 rounding and rint), the BSQ stages of the row-masked matrix, and a
+    decode that returns scale * q8 on the protected rows exactly."""
+    N, K, S, p = 72, 136, 2, 6
+    W = _outlier_rows(N, K, seed=61)
+    L = oracle.encode_rows(W, S, p)
+    idx = L["idx"]
+    assert list(idx) == list(oracle.select_rows(W, p)[0])
+    fw = f64(W)
+    s = (np.abs(fw[idx]).max(axis=1) / 127.0).astype(np.float16)
+    assert np.array_equal(L["scale"], s.view(np.uint16))
+    sd = s.astype(np.float64)[:, None]
+    q = np.clip(np.rint(fw[idx] / sd), -127, 127)
+    assert np.array_equal(L["q8"][:, :K], q.astype(np.int8))
+    assert not L["q8"][:, K:].any()
+    assert np.all(np.abs(fw[idx] - sd * q) <= sd / 2 + 1e-300)
+    # stages: the row-masked matrix through the column encoder with p = 0
+    Wm = W.copy()
+    Wm[idx] = 0
+    ref = oracle.encode(Wm, S=S, p=0)
+    assert np.array_equal(L["codes"], ref["codes"]) and np.array_equal(L["norms"], ref["norms"])
+    assert not L["norms"][:, idx].any()
+    What = oracle.decode_rows(L)
+    assert np.array_equal(What[idx], sd * L["q8"][:, :K].astype(np.float64))
+    keep = np.setdiff1d(np.arange(N), idx)
+    assert np.array_equal(What[keep], oracle.decode_rows(ref)[keep])
+    assert np.array_equal(oracle.decode_rows(L, row0=5, nrows=20), What[5:25])
+
+
+def test_coupled_encode_shares_one_set():
+    F, H, S, p = 64, 32, 2, 4
+    Wg = synth.layer_weights(F, H, seed=71)
+    Wu = synth.layer_weights(F, H, seed=72)
+    Wd = synth.layer_weights(H, F, seed=73)
+    Lg, Lu, Ld = oracle.encode_coupled(Wg, Wu, Wd, S, p)
+    idx = oracle.select_coupled(Wg, Wu, Wd, p)[0]
+    for L in (Lg, Lu, Ld):
+        assert list(L["idx"]) == list(idx)
+    assert Lg["axis"] == 1 and Lu["axis"] == 1 and Ld.get("axis", 0) == 0
+    # down keeps the coupled set as columns: scale * q8 there, within half a
+    # quantisation step of the weight
+    sd = Ld["scale"].view(np.float16).astype(np.float64)[None, :]
+    cols = oracle.decode_rows(Ld)[:, idx]
+    assert np.array_equal(cols, sd * Ld["q8"][:, :p])
+    assert np.all(np.abs(f64(Wd)[:, idx] - cols) <= sd / 2 + 1e-300)
