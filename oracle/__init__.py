@@ -18,6 +18,11 @@ Functions and the paper passages they follow:
                             output-row protection and the coupled MLP
                             channel score (Sec. III-E Eq. 9) with Eq. 10 on
                             rows; the CUDA library does not take this axis yet
+* :func:`double_to_fp8`, :func:`fp8_to_double`, :func:`quantize_protected_fmt`,
+  :func:`protected_values_fmt`
+                            FP8 E4M3 / E5M2 and BF16 protected payloads (the
+                            paper's protected-format ablation) as variants of
+                            Eq. 10; not taken by the CUDA library yet
 * :func:`lora_apply`        y0 + scale * Bm (A x), the optional low-rank
                             compensation of Sec. III-F (plain definition)
 * :func:`apply_rows`        decode + matmul on a list of rows
@@ -48,6 +53,7 @@ _lib = None
 _LIB_OVERRIDE = os.environ.get("BISCO_ORACLE_LIB")
 
 OK, ERR_INVALID_ARG, ERR_RANGE = 0, 1, 3
+FMT_INT8, FMT_E4M3, FMT_E5M2, FMT_BF16 = 0, 1, 2, 3
 
 CFLAGS = ["-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared"]
 
@@ -106,6 +112,14 @@ def _load():
         lib.or_encode_rows.argtypes = [P, P, i32, i32, i32, i32, P, P, P, P, P, P]
         lib.or_decode_rows_axis1.restype = None
         lib.or_decode_rows_axis1.argtypes = [P, P, P, P, P, i32, i32, i32, i32, i32, i32, P]
+        lib.or_double_to_fp8.restype = ctypes.c_uint8
+        lib.or_double_to_fp8.argtypes = [ctypes.c_double, ctypes.c_int]
+        lib.or_fp8_to_double.restype = ctypes.c_double
+        lib.or_fp8_to_double.argtypes = [ctypes.c_uint8, ctypes.c_int]
+        lib.or_quantize_protected_fmt.restype = ctypes.c_int
+        lib.or_quantize_protected_fmt.argtypes = [P, i32, i32, P, i32, ctypes.c_int, P, P]
+        lib.or_protected_value_fmt.restype = ctypes.c_double
+        lib.or_protected_value_fmt.argtypes = [P, P, i32, ctypes.c_int, i32, i32]
         lib.or_lora_apply.restype = ctypes.c_int
         lib.or_lora_apply.argtypes = [P, P, i32, i32, i32, ctypes.c_double, P, i32, P, P]
         del i64
@@ -327,6 +341,52 @@ def matmul(What, X_bits):
     Y = np.zeros((B, nrows), np.float64)
     _load().or_matmul(_ptr(What), nrows, K, _ptr(X_bits), B, _ptr(Y))
     return Y
+
+
+def double_to_fp8(x: float, fmt: int) -> int:
+    """FP8 bits of x (FMT_E4M3 / FMT_E5M2): nearest even, saturating."""
+    return int(_load().or_double_to_fp8(float(x), int(fmt)))
+
+
+def fp8_to_double(v: int, fmt: int) -> float:
+    return _load().or_fp8_to_double(int(v), int(fmt))
+
+
+def quantize_protected_fmt(W_bits, idx, fmt):
+    """Eq. 10 with the protected payload in format ``fmt``: returns
+    (q [N][pad16(p)] uint8 FP8 bits / uint16 bf16 bits / int8, scale uint16[p])."""
+    W_bits = _c(W_bits, np.uint16)
+    N, K = W_bits.shape
+    idx = _c(idx, np.int32)
+    p = len(idx)
+    pp = max(pad16(p), 16)
+    dt = {FMT_INT8: np.int8, FMT_E4M3: np.uint8, FMT_E5M2: np.uint8, FMT_BF16: np.uint16}[fmt]
+    q = np.zeros((N, pp), dt)
+    scale = np.zeros(max(p, 1), np.uint16)
+    idx_arg = idx if p else np.zeros(1, np.int32)
+    if fmt == FMT_INT8:
+        rc = _load().or_quantize_protected(_ptr(W_bits), N, K, _ptr(idx_arg), p, _ptr(q), _ptr(scale))
+    else:
+        rc = _load().or_quantize_protected_fmt(_ptr(W_bits), N, K, _ptr(idx_arg), p, int(fmt),
+                                               _ptr(q), _ptr(scale))
+    if rc:
+        raise OracleError(rc)
+    return q[:, :pad16(p)].copy(), scale[:p].copy()
+
+
+def protected_values_fmt(q, scale, fmt):
+    """Decoded protected values [N][p] = scale_t * value(q[i][t])."""
+    q = np.ascontiguousarray(q)
+    scale = _c(scale, np.uint16)
+    N, pp = q.shape
+    p = len(scale)
+    assert pp == pad16(p)
+    out = np.zeros((N, p), np.float64)
+    lib = _load()
+    for i in range(N):
+        for t in range(p):
+            out[i, t] = lib.or_protected_value_fmt(_ptr(q), _ptr(scale), p, int(fmt), i, t)
+    return out
 
 
 def lora_apply(A_bits, Bm_bits, X_bits, Y0, scale=1.0):

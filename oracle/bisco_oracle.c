@@ -23,6 +23,9 @@
  *   rows     output-row protection and the coupled MLP channel score of
  *            Sec. III-E Eq. 9 (gate/up rows and down columns share one
  *            protected set), with Eq. 10's 8-bit quantiser on the rows.
+ *   fp8      the FP8 (E4M3, E5M2) and BF16 protected-payload formats of the
+ *            paper's protected-format ablation, as variants of Eq. 10's
+ *            quantiser.
  *   lora     y[b][n] + scale * sum_r Bm[n][r] * (sum_k A[r][k] * x[b][k]),
  *            the optional low-rank compensation of Sec. III-F (plain
  *            definition, the adapter's down projection first).
@@ -537,5 +540,134 @@ void or_decode_rows_axis1(const uint8_t *codes, const uint16_t *norms,
         for (int32_t k = 0; k < K; ++k)
             out[(int64_t)(i - row0) * K + k] = s * (double)q8[(int64_t)t * kp + k];
     }
+}
+
+/* ------------------------------- FP8 and BF16 protected payloads (Eq. 10) */
+
+/* Formats of the protected payload: 0 = INT8 (or_quantize_protected),
+ * 1 = FP8 E4M3 (bias 7, largest finite 448, S.1111.111 is NaN, no
+ * infinities), 2 = FP8 E5M2 (bias 15, largest finite 57344, IEEE-style
+ * infinities and NaNs), 3 = BF16 (the weight itself). */
+#define OR_FMT_INT8 0
+#define OR_FMT_E4M3 1
+#define OR_FMT_E5M2 2
+#define OR_FMT_BF16 3
+
+static int or_fp8_params(int fmt, int *mbits, int *bias, double *maxf, uint8_t *maxcode)
+{
+    if (fmt == OR_FMT_E4M3) { *mbits = 3; *bias = 7; *maxf = 448.0; *maxcode = 0x7e; return 1; }
+    if (fmt == OR_FMT_E5M2) { *mbits = 2; *bias = 15; *maxf = 57344.0; *maxcode = 0x7b; return 1; }
+    return 0;
+}
+
+/* binary64 -> FP8 bits: round to nearest, ties to even, gradual underflow;
+ * a finite value that rounds above the largest finite one gives the largest
+ * finite one (saturation), +-inf too; NaN gives the format's NaN.  Same
+ * method as or_double_to_fp16: scale the significand by a power of two so
+ * that the kept bits are the integer part, and round once with nearbyint(). */
+uint8_t or_double_to_fp8(double x, int fmt)
+{
+    int mb, bias;
+    double maxf;
+    uint8_t maxcode;
+    if (!or_fp8_params(fmt, &mb, &bias, &maxf, &maxcode)) return 0;
+    uint8_t sign = signbit(x) ? 0x80 : 0;
+    if (isnan(x)) return (uint8_t)(sign | (fmt == OR_FMT_E4M3 ? 0x7f : 0x7e));
+    double a = fabs(x);
+    if (isinf(a)) return (uint8_t)(sign | maxcode);
+    if (a < ldexp(1.0, 1 - bias)) {
+        /* subnormal range: units of 2^(1 - bias - mb); 2^mb units is the
+         * least normal, whose code is the same integer */
+        double m = nearbyint(ldexp(a, bias - 1 + mb));
+        return (uint8_t)(sign | (uint8_t)m);
+    }
+    int ex;
+    frexp(a, &ex);                  /* a = f * 2^ex, f in [0.5, 1) */
+    int E = ex - 1;                 /* a in [2^E, 2^(E+1)) */
+    double m = nearbyint(ldexp(a, mb - E));   /* in [2^mb, 2^(mb+1)] */
+    if (m == ldexp(1.0, mb + 1)) {
+        m = ldexp(1.0, mb);
+        E += 1;
+    }
+    double v = ldexp(m, E - mb);
+    if (v > maxf) return (uint8_t)(sign | maxcode);
+    return (uint8_t)(sign | (uint8_t)((E + bias) << mb) | (uint8_t)(m - ldexp(1.0, mb)));
+}
+
+/* FP8 bits -> binary64 (exact). */
+double or_fp8_to_double(uint8_t v, int fmt)
+{
+    int mb, bias;
+    double maxf;
+    uint8_t maxcode;
+    if (!or_fp8_params(fmt, &mb, &bias, &maxf, &maxcode)) return NAN;
+    int sign = v >> 7;
+    int emax = (1 << (7 - mb)) - 1;
+    int e = (v >> mb) & emax;
+    int mant = v & ((1 << mb) - 1);
+    double r;
+    if (fmt == OR_FMT_E4M3 && e == emax && mant == (1 << mb) - 1)
+        r = NAN;
+    else if (fmt == OR_FMT_E5M2 && e == emax)
+        r = mant ? NAN : INFINITY;
+    else if (e == 0)
+        r = ldexp((double)mant, 1 - bias - mb);
+    else
+        r = ldexp((double)((1 << mb) + mant), e - bias - mb);
+    return sign ? -r : r;
+}
+
+/* Eq. 10 with an FP8 payload, per protected column j:
+ *   scale_j = fp16(max_i |W_ij| / largest finite FP8 value)
+ *   q_ij    = fp8(W_ij / scale_j), or +0 if scale_j == 0
+ * With BF16 the payload is the weight's own bits and the scale is 1.0.
+ * q is [N][p_pad] bytes (FP8) or [N][p_pad] bf16 (BF16), zero padding. */
+int or_quantize_protected_fmt(const uint16_t *W, int32_t N, int32_t K,
+                              const int32_t *idx, int32_t p, int fmt,
+                              void *q_out, uint16_t *scale_out)
+{
+    int32_t pp = or_pad16(p);
+    int mb, bias;
+    double maxf;
+    uint8_t maxcode;
+    if (fmt == OR_FMT_BF16) {
+        uint16_t *q = (uint16_t *)q_out;
+        memset(q, 0, sizeof(uint16_t) * (size_t)N * (size_t)pp);
+        for (int32_t t = 0; t < p; ++t) {
+            scale_out[t] = 0x3c00;   /* 1.0 */
+            for (int32_t i = 0; i < N; ++i) q[(int64_t)i * pp + t] = W[(int64_t)i * K + idx[t]];
+        }
+        return OR_OK;
+    }
+    if (!or_fp8_params(fmt, &mb, &bias, &maxf, &maxcode)) return OR_ERR_INVALID_ARG;
+    uint8_t *q = (uint8_t *)q_out;
+    memset(q, 0, (size_t)N * (size_t)pp);
+    for (int32_t t = 0; t < p; ++t) {
+        int32_t j = idx[t];
+        double m = 0.0;
+        for (int32_t i = 0; i < N; ++i) {
+            double a = fabs(or_bf16_to_double(W[(int64_t)i * K + j]));
+            if (a > m) m = a;
+        }
+        uint16_t s16 = or_double_to_fp16(m / maxf);
+        if ((s16 & 0x7c00) == 0x7c00) return OR_ERR_RANGE;
+        scale_out[t] = s16;
+        double s = or_fp16_to_double(s16);
+        for (int32_t i = 0; i < N; ++i)
+            q[(int64_t)i * pp + t] =
+                s != 0.0 ? or_double_to_fp8(or_bf16_to_double(W[(int64_t)i * K + j]) / s, fmt) : 0;
+    }
+    return OR_OK;
+}
+
+/* The decoded protected value of column t in row i: scale_t * value(q). */
+double or_protected_value_fmt(const void *q, const uint16_t *scale, int32_t p,
+                              int fmt, int32_t i, int32_t t)
+{
+    int32_t pp = or_pad16(p);
+    double s = or_fp16_to_double(scale[t]);
+    if (fmt == OR_FMT_BF16) return s * or_bf16_to_double(((const uint16_t *)q)[(int64_t)i * pp + t]);
+    if (fmt == OR_FMT_INT8) return s * (double)((const int8_t *)q)[(int64_t)i * pp + t];
+    return s * or_fp8_to_double(((const uint8_t *)q)[(int64_t)i * pp + t], fmt);
 }
 

@@ -49,6 +49,13 @@ MUTATIONS = {
     "lora_bm_transposed": ("or_bf16_to_double(Bm[(int64_t)n * rank + r]) * t[r];",
                            "or_bf16_to_double(Bm[(int64_t)r * N + n]) * t[r];"),
     "lora_scale_dropped": ("Y0[(int64_t)b * N + n] + scale * acc;", "Y0[(int64_t)b * N + n] + acc;"),
+    "fp8_rounds_toward_zero": ("double m = nearbyint(ldexp(a, mb - E));",
+                               "double m = floor(ldexp(a, mb - E));"),
+    "fp8_e4m3_bias_off_by_one": ("*mbits = 3; *bias = 7;", "*mbits = 3; *bias = 8;"),
+    "fp8_scale_over_127": ("uint16_t s16 = or_double_to_fp16(m / maxf);",
+                           "uint16_t s16 = or_double_to_fp16(m / 127.0);"),
+    "fp8_subnormal_step_wrong": ("double m = nearbyint(ldexp(a, bias - 1 + mb));",
+                                 "double m = nearbyint(ldexp(a, bias + mb));"),
 }
 
 

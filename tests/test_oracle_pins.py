@@ -14,6 +14,7 @@ import os
 
 import numpy as np
 import pytest
+import torch
 
 import oracle
 from paper_2607_08643_gb300 import synth
@@ -562,3 +563,135 @@ def test_coupled_encode_shares_one_set():
     cols = oracle.decode_rows(Ld)[:, idx]
     assert np.array_equal(cols, sd * Ld["q8"][:, :p])
     assert np.all(np.abs(f64(Wd)[:, idx] - cols) <= sd / 2 + 1e-300)
+
+
+# ------------------------------------------- FP8 / BF16 protected payloads
+
+
+
+_FP8 = {oracle.FMT_E4M3: (torch.float8_e4m3fn, 3, 7, 448.0),
+        oracle.FMT_E5M2: (torch.float8_e5m2, 2, 15, 57344.0)}
+
+
+def _fp8_value_closed_form(v, mb, bias, e4m3):
+    """Value of an FP8 bit pattern from the format's definition (sign,
+    exponent field, mantissa field), written out independently of the
+    oracle's decoder."""
+    s = -1.0 if v & 0x80 else 1.0
+    e = (v >> mb) & ((1 << (7 - mb)) - 1)
+    m = v & ((1 << mb) - 1)
+    emax = (1 << (7 - mb)) - 1
+    if e4m3 and e == emax and m == (1 << mb) - 1:
+        return math.nan
+    if not e4m3 and e == emax:
+        return math.nan if m else s * math.inf
+    if e == 0:
+        return s * m * 2.0 ** (1 - bias - mb)
+    return s * (1 + m / 2.0 ** mb) * 2.0 ** (e - bias)
+
+
+@pytest.mark.parametrize("fmt", [oracle.FMT_E4M3, oracle.FMT_E5M2])
+def test_fp8_widening_all_patterns(fmt):
+    """All 256 codes against torch's FP8 dtype and the format's closed form."""
+    dt, mb, bias, _ = _FP8[fmt]
+    mine = np.array([oracle.fp8_to_double(v, fmt) for v in range(256)])
+    ref = torch.arange(256, dtype=torch.uint8).view(dt).to(torch.float64).numpy()
+    assert np.array_equal(mine, ref, equal_nan=True)
+    cf = np.array([_fp8_value_closed_form(v, mb, bias, fmt == oracle.FMT_E4M3) for v in range(256)])
+    assert np.array_equal(mine, cf, equal_nan=True)
+
+
+@pytest.mark.parametrize("fmt", [oracle.FMT_E4M3, oracle.FMT_E5M2])
+def test_fp8_rounding_brute_force_nearest_ties_to_even(fmt):
+    """Within range the code is the nearest finite code (brute force over all
+    of them), ties to the even mantissa; exact midpoints between neighbours
+    are included, and so are subnormals and both zeros."""
+    dt, mb, bias, maxf = _FP8[fmt]
+    codes = [v for v in range(256) if math.isfinite(oracle.fp8_to_double(v, fmt))]
+    vals = np.array([oracle.fp8_to_double(v, fmt) for v in codes])
+    pos = sorted({x for x in vals if x >= 0})
+    rng = np.random.default_rng(5)
+    xs = list(rng.uniform(-maxf, maxf, 400)) + list(rng.normal(0, 1, 400)) + \
+        list(rng.normal(0, 2.0 ** (1 - bias), 200))
+    xs += [(a + b) / 2 for a, b in zip(pos, pos[1:])]          # every midpoint
+    xs += [-(a + b) / 2 for a, b in zip(pos, pos[1:])]
+    xs += [0.0, -0.0, maxf, -maxf]
+    for x in xs:
+        got = oracle.double_to_fp8(x, fmt)
+        d = np.abs(vals - x)
+        best = np.flatnonzero(d == d.min())
+        cand = [codes[i] for i in best]
+        if x == 0.0:
+            want = 0x80 if math.copysign(1.0, x) < 0 else 0x00
+        elif len(cand) == 1:
+            want = cand[0]
+        else:                                  # a tie: the even mantissa
+            cand = [c for c in cand if (c & 0x80) == (0x80 if x < 0 else 0)]
+            even = [c for c in cand if c % 2 == 0]
+            assert len(even) == 1
+            want = even[0]
+        assert got == want, (x, got, want)
+        ref = int(torch.tensor([x], dtype=torch.float64).to(dt).view(torch.uint8)[0])
+        assert got == ref, (x, got, ref)
+
+
+@pytest.mark.parametrize("fmt", [oracle.FMT_E4M3, oracle.FMT_E5M2])
+def test_fp8_saturates_above_the_largest_finite(fmt):
+    """Reading for the protected payload: a value that rounds past the
+    largest finite code takes that code, with its sign; NaN stays NaN."""
+    _, _, _, maxf = _FP8[fmt]
+    top = oracle.double_to_fp8(maxf, fmt)
+    for x in (maxf * 1.5, maxf * 1e6, math.inf):
+        assert oracle.double_to_fp8(x, fmt) == top
+        assert oracle.double_to_fp8(-x, fmt) == top | 0x80
+    assert math.isnan(oracle.fp8_to_double(oracle.double_to_fp8(math.nan, fmt), fmt))
+
+
+@pytest.mark.parametrize("fmt", [oracle.FMT_E4M3, oracle.FMT_E5M2])
+def test_fp8_protected_quantiser_closed_form(fmt):
+    """Eq. 10 with an FP8 payload: scale = fp16(max|W_:,j| / largest FP8),
+    q = fp8(W / scale) with torch's FP8 cast as the rounding reference,
+    and a decoded value within half an FP8 step of the weight."""
+    dt, mb, bias, maxf = _FP8[fmt]
+    W = synth.layer_weights(96, 256, seed=81)
+    idx = oracle.select_protected(W, 7)[0]
+    q, scale = oracle.quantize_protected_fmt(W, idx, fmt)
+    assert q.shape == (96, 16) and q.dtype == np.uint8
+    assert not q[:, 7:].any()
+    Wd = f64(W)
+    got = oracle.protected_values_fmt(q, scale, fmt)
+    for t, j in enumerate(idx):
+        col = Wd[:, j]
+        s16 = np.float16(np.abs(col).max() / maxf)
+        assert scale[t] == s16.view(np.uint16)
+        s = float(s16)
+        r = col / s
+        assert np.all(np.abs(r) <= maxf * (1 + 2.0 ** -10))
+        rc = np.clip(r, -maxf, maxf)
+        ref = torch.from_numpy(rc).to(dt).view(torch.uint8).numpy()
+        assert np.array_equal(q[:, t], ref)
+        # decoded = s * value(q); the error is at most half an FP8 ulp of
+        # |W/s| (relative 2^-(mb+1) for normals, absolute half the
+        # subnormal step below), plus the saturation margin at the top
+        ulp_half = np.maximum(np.abs(rc) * 2.0 ** -(mb + 1), 2.0 ** (-bias - mb))
+        assert np.all(np.abs(got[:, t] - s * rc) <= s * ulp_half)
+        assert np.all(np.abs(r - rc) <= maxf * 2.0 ** -10)
+
+
+def test_bf16_protected_payload_is_the_weight():
+    W = synth.layer_weights(40, 128, seed=82)
+    idx = oracle.select_protected(W, 5)[0]
+    q, scale = oracle.quantize_protected_fmt(W, idx, oracle.FMT_BF16)
+    assert q.dtype == np.uint16 and np.all(scale == 0x3C00)
+    assert np.array_equal(q[:, :5], W[:, idx]) and not q[:, 5:].any()
+    assert np.array_equal(oracle.protected_values_fmt(q, scale, oracle.FMT_BF16), f64(W)[:, idx])
+
+
+def test_int8_format_matches_the_int8_quantiser():
+    """FMT_INT8 through the format-generic entry is Eq. 10's INT8 quantiser."""
+    W = synth.layer_weights(48, 256, seed=83)
+    L = oracle.encode(W, S=1, p=6)
+    q, scale = oracle.quantize_protected_fmt(W, L["idx"], oracle.FMT_INT8)
+    assert np.array_equal(q, L["q8"]) and np.array_equal(scale, L["scale"])
+    dec = oracle.protected_values_fmt(q, scale, oracle.FMT_INT8)
+    assert np.array_equal(dec, oracle.decode_rows(L)[:, L["idx"]])
