@@ -23,6 +23,11 @@ Functions and the paper passages they follow:
                             FP8 E4M3 / E5M2 and BF16 protected payloads (the
                             paper's protected-format ablation) as variants of
                             Eq. 10; not taken by the CUDA library yet
+* :func:`decoder_table_linear`, :func:`decoder_table_mlp`, :func:`decode_rows_table`
+                            the decoder step of Eq. 1 as a table over the 256
+                            code bytes (linear, or odd tanh perceptron with an
+                            optional residual block), decoded per Eq. 12; not
+                            taken by the CUDA library yet
 * :func:`lora_apply`        y0 + scale * Bm (A x), the optional low-rank
                             compensation of Sec. III-F (plain definition)
 * :func:`apply_rows`        decode + matmul on a list of rows
@@ -120,6 +125,12 @@ def _load():
         lib.or_quantize_protected_fmt.argtypes = [P, i32, i32, P, i32, ctypes.c_int, P, P]
         lib.or_protected_value_fmt.restype = ctypes.c_double
         lib.or_protected_value_fmt.argtypes = [P, P, i32, ctypes.c_int, i32, i32]
+        lib.or_decoder_table_linear.restype = None
+        lib.or_decoder_table_linear.argtypes = [P, P]
+        lib.or_decoder_table_mlp.restype = ctypes.c_int
+        lib.or_decoder_table_mlp.argtypes = [P, i32, P, P, P]
+        lib.or_decode_rows_table.restype = None
+        lib.or_decode_rows_table.argtypes = [P, P, P, P, P, P, i32, i32, i32, i32, i32, i32, P]
         lib.or_lora_apply.restype = ctypes.c_int
         lib.or_lora_apply.argtypes = [P, P, i32, i32, i32, ctypes.c_double, P, i32, P, P]
         del i64
@@ -386,6 +397,57 @@ def protected_values_fmt(q, scale, fmt):
     for i in range(N):
         for t in range(p):
             out[i, t] = lib.or_protected_value_fmt(_ptr(q), _ptr(scale), p, int(fmt), i, t)
+    return out
+
+
+def decoder_table_linear(A):
+    """Table [256][8] (float64) of the linear decoder D(q) = A q, A [8][8]."""
+    A = _c(A, np.float64)
+    assert A.shape == (8, 8)
+    T = np.zeros((256, 8), np.float64)
+    _load().or_decoder_table_linear(_ptr(A), _ptr(T))
+    return T
+
+
+def decoder_table_mlp(W1, W2, Wr=None):
+    """Table [256][8] (float64) of the odd decoder W2 (h + tanh(Wr h)),
+    h = tanh(W1 q); W1 [hdim][8], W2 [8][hdim], Wr [hdim][hdim] or None
+    (no residual block)."""
+    W1 = _c(W1, np.float64)
+    W2 = _c(W2, np.float64)
+    hdim = W1.shape[0]
+    assert W1.shape == (hdim, 8) and W2.shape == (8, hdim)
+    if Wr is not None:
+        Wr = _c(Wr, np.float64)
+        assert Wr.shape == (hdim, hdim)
+    T = np.zeros((256, 8), np.float64)
+    rc = _load().or_decoder_table_mlp(_ptr(W1), hdim, _ptr(Wr) if Wr is not None else None,
+                                      _ptr(W2), _ptr(T))
+    if rc:
+        raise OracleError(rc)
+    return T
+
+
+def table_to_fp16(T):
+    """Binary16 bits of a float64 decoder table, each value rounded once
+    (nearest even) by the oracle's own conversion."""
+    T = np.asarray(T, np.float64)
+    return np.array([double_to_fp16(float(v)) for v in T.ravel()], np.uint16).reshape(T.shape)
+
+
+def decode_rows_table(L, tables16, row0=0, nrows=None):
+    """Dense float64 rows of What with per-stage decoder tables
+    (tables16 [S][256][8] binary16 bits): Eq. 12 with Eq. 1, and the Eq. 10
+    protected columns."""
+    N, K, S = L["N"], L["K"], L["S"]
+    tables16 = _c(tables16, np.uint16)
+    assert tables16.shape == (S, 256, 8)
+    if nrows is None:
+        nrows = N - row0
+    out = np.zeros((nrows, K), np.float64)
+    codes, norms, q8, scale, idx = _layer_args(L)
+    _load().or_decode_rows_table(_ptr(codes), _ptr(norms), _ptr(tables16), _ptr(q8), _ptr(scale),
+                                 _ptr(idx), N, K, S, L["p"], row0, nrows, _ptr(out))
     return out
 
 

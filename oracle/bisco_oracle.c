@@ -26,6 +26,11 @@
  *   fp8      the FP8 (E4M3, E5M2) and BF16 protected-payload formats of the
  *            paper's protected-format ablation, as variants of Eq. 10's
  *            quantiser.
+ *   decoder  the decoder step of Eq. 1 as per-stage tables over the 256
+ *            code bytes: a linear decoder A q, or an odd (sign-symmetric)
+ *            tanh perceptron with an optional residual block, the table
+ *            form of the paper's decoder ablation; decode with the tables
+ *            follows Eq. 12.
  *   lora     y[b][n] + scale * sum_r Bm[n][r] * (sum_k A[r][k] * x[b][k]),
  *            the optional low-rank compensation of Sec. III-F (plain
  *            definition, the adapter's down projection first).
@@ -671,3 +676,99 @@ double or_protected_value_fmt(const void *q, const uint16_t *scale, int32_t p,
     return s * or_fp8_to_double(((const uint8_t *)q)[(int64_t)i * pp + t], fmt);
 }
 
+
+/* ------------------------------------- learned decoder step (Eq. 1, Eq. 12) */
+
+/* The decoder D of Eq. 1 maps a stage's code q in {-1/sqrt(8), +1/sqrt(8)}^8
+ * (Eq. 3 with b = d = 8) to a chunk.  With the stored norm kept, a chunk of
+ * stage s decodes to n16 * D_s(q).  Since q takes only 256 values, D_s is
+ * fully described by its table T_s[v][k] = D_s(q(v))_k, v the code byte
+ * (bit k of v set <=> q_k = -1/sqrt(8)).  The identity decoder q -> q is the
+ * norm-rescale decoder of the rest of this file. */
+
+/* q(v)_k = (bit k of v ? -1 : +1) / sqrt(8) */
+static double or_code_elem(int v, int k)
+{
+    double t = or_inv_sqrt8();
+    return ((v >> k) & 1) ? -t : t;
+}
+
+/* Linear decoder D(q) = A q, A [8][8] row-major (output k, code position j):
+ * T[v][k] = sum_j A[k][j] * q(v)_j, ascending j. */
+void or_decoder_table_linear(const double *A, double *T)
+{
+    for (int v = 0; v < 256; ++v)
+        for (int k = 0; k < 8; ++k) {
+            double acc = 0.0;
+            for (int j = 0; j < 8; ++j) acc = acc + A[k * 8 + j] * or_code_elem(v, j);
+            T[v * 8 + k] = acc;
+        }
+}
+
+/* Symmetric (odd) nonlinear decoder, D(-q) = -D(q): a bias-free perceptron
+ * with the odd activation tanh,
+ *   h   = tanh(W1 q)                 W1 [hdim][8]
+ *   h   = h + tanh(Wr h)             Wr [hdim][hdim], only if Wr != NULL
+ *                                    (the residual block)
+ *   out = W2 h                       W2 [8][hdim]
+ * every product summed in ascending index order. */
+int or_decoder_table_mlp(const double *W1, int32_t hdim, const double *Wr,
+                         const double *W2, double *T)
+{
+    if (hdim <= 0) return OR_ERR_INVALID_ARG;
+    double *h = (double *)malloc(sizeof(double) * (size_t)hdim);
+    double *g = (double *)malloc(sizeof(double) * (size_t)hdim);
+    if (!h || !g) { free(h); free(g); return OR_ERR_INVALID_ARG; }
+    for (int v = 0; v < 256; ++v) {
+        for (int32_t a = 0; a < hdim; ++a) {
+            double acc = 0.0;
+            for (int j = 0; j < 8; ++j) acc = acc + W1[(int64_t)a * 8 + j] * or_code_elem(v, j);
+            h[a] = tanh(acc);
+        }
+        if (Wr) {
+            for (int32_t a = 0; a < hdim; ++a) {
+                double acc = 0.0;
+                for (int32_t c = 0; c < hdim; ++c) acc = acc + Wr[(int64_t)a * hdim + c] * h[c];
+                g[a] = tanh(acc);
+            }
+            for (int32_t a = 0; a < hdim; ++a) h[a] = h[a] + g[a];
+        }
+        for (int k = 0; k < 8; ++k) {
+            double acc = 0.0;
+            for (int32_t a = 0; a < hdim; ++a) acc = acc + W2[(int64_t)k * hdim + a] * h[a];
+            T[v * 8 + k] = acc;
+        }
+    }
+    free(h);
+    free(g);
+    return OR_OK;
+}
+
+/* Dense reconstruction with per-stage decoder tables (Eq. 12 with Eq. 1):
+ *   What_ij = sum_{s=1..S} n16_{s,i,c} * T_s[code_{s,i,c}][j % 8]   j not in P
+ *   What_ij = scale_j * q8_ij                                       j in P
+ * tables [S][256][8] are binary16 bits: the evaluated decoder as a kernel
+ * would hold it. */
+void or_decode_rows_table(const uint8_t *codes, const uint16_t *norms, const uint16_t *tables,
+                          const int8_t *q8, const uint16_t *scale, const int32_t *idx,
+                          int32_t N, int32_t K, int32_t S, int32_t p,
+                          int32_t row0, int32_t nrows, double *out)
+{
+    int32_t C = K / 8, pp = or_pad16(p);
+    for (int32_t r = 0; r < nrows; ++r) {
+        int32_t i = row0 + r;
+        double *o = out + (int64_t)r * K;
+        for (int32_t j = 0; j < K; ++j) {
+            int32_t c = j / 8, k = j % 8;
+            double acc = 0.0;
+            for (int32_t s = 0; s < S; ++s) {
+                int64_t e = ((int64_t)s * N + i) * C + c;
+                double t = or_fp16_to_double(tables[((int64_t)s * 256 + codes[e]) * 8 + k]);
+                acc = acc + or_fp16_to_double(norms[e]) * t;
+            }
+            o[j] = acc;
+        }
+        for (int32_t t = 0; t < p; ++t)
+            o[idx[t]] = or_fp16_to_double(scale[t]) * (double)q8[(int64_t)i * pp + t];
+    }
+}

@@ -56,6 +56,17 @@ MUTATIONS = {
                            "uint16_t s16 = or_double_to_fp16(m / 127.0);"),
     "fp8_subnormal_step_wrong": ("double m = nearbyint(ldexp(a, bias - 1 + mb));",
                                  "double m = nearbyint(ldexp(a, bias + mb));"),
+    "decoder_table_ignores_stage": ("tables[((int64_t)s * 256 + codes[e]) * 8 + k]",
+                                    "tables[((int64_t)0 * 256 + codes[e]) * 8 + k]"),
+    "decoder_table_transposed": ("tables[((int64_t)s * 256 + codes[e]) * 8 + k]",
+                                 "tables[(int64_t)s * 2048 + (int64_t)k * 256 + codes[e]]"),
+    "linear_decoder_transposed": ("acc = acc + A[k * 8 + j] * or_code_elem(v, j);",
+                                  "acc = acc + A[j * 8 + k] * or_code_elem(v, j);"),
+    "code_element_sign_flipped": ("return ((v >> k) & 1) ? -t : t;", "return ((v >> k) & 1) ? t : -t;"),
+    "mlp_residual_replaces_hidden": ("for (int32_t a = 0; a < hdim; ++a) h[a] = h[a] + g[a];",
+                                     "for (int32_t a = 0; a < hdim; ++a) h[a] = g[a];"),
+    "mlp_output_weights_transposed": ("acc = acc + W2[(int64_t)k * hdim + a] * h[a];",
+                                      "acc = acc + W2[(int64_t)a * 8 + k] * h[a];"),
 }
 
 

@@ -695,3 +695,146 @@ def test_int8_format_matches_the_int8_quantiser():
     assert np.array_equal(q, L["q8"]) and np.array_equal(scale, L["scale"])
     dec = oracle.protected_values_fmt(q, scale, oracle.FMT_INT8)
     assert np.array_equal(dec, oracle.decode_rows(L)[:, L["idx"]])
+
+
+# ------------------------------------------------ learned decoder step (Eq. 1)
+
+def _signs(v):
+    """The +-1 sign vector of code byte v (bit k set <=> element k negative),
+    by numpy's own bit unpacking."""
+    b = np.unpackbits(np.array([v], np.uint8), bitorder="little")
+    return 1.0 - 2.0 * b.astype(np.float64)
+
+
+def test_linear_decoder_table_identity_permutation_and_scaling():
+    T = oracle.decoder_table_linear(np.eye(8))
+    for v in range(256):
+        assert np.array_equal(T[v], _signs(v) * INV_SQRT8)
+    perm = [3, 0, 7, 1, 6, 2, 5, 4]                   # not an involution
+    P = np.zeros((8, 8))
+    P[np.arange(8), perm] = 1.0                       # output k reads code position perm[k]
+    T = oracle.decoder_table_linear(P)
+    for v in range(256):
+        assert np.array_equal(T[v], _signs(v)[perm] * INV_SQRT8)
+    d = np.array([1, 2, 4, 8, 0.5, 0.25, -1, -2.0])
+    T = oracle.decoder_table_linear(np.diag(d))
+    for v in range(256):
+        assert np.array_equal(T[v], d * (_signs(v) * INV_SQRT8))
+
+
+def _dyadic_linear_table(seed):
+    """A linear decoder whose fp16 table is exact: A = sqrt(8) * B with B of
+    small dyadic entries, so T = A q rounds to B * signs exactly."""
+    rng = np.random.default_rng(seed)
+    B = rng.integers(-8, 9, size=(8, 8)) / 8.0
+    T16 = oracle.table_to_fp16(oracle.decoder_table_linear(math.sqrt(8.0) * B))
+    vals = T16.view(np.float16).astype(np.float64)
+    for v in range(256):
+        assert np.array_equal(vals[v], B @ _signs(v))
+    return B, T16
+
+
+def test_linear_decoder_equals_transformed_activations():
+    """With D(q) = A q, y = sum_c n * (A q_c) . x_c = sum_c n * q_c . (A^T x_c):
+    decoding with the table and multiplying gives the same output as the
+    identity-decoder sign codes against per-chunk transformed activations."""
+    N, K, S, p = 24, 96, 2, 3
+    W = synth.layer_weights(N, K, seed=91)
+    L = oracle.encode(W, S=S, p=p)
+    tabs, Bs = [], []
+    for s in range(S):
+        B, T16 = _dyadic_linear_table(92 + s)
+        tabs.append(T16)
+        Bs.append(B)
+    What = oracle.decode_rows_table(L, np.stack(tabs))
+    x = synth.activations(2, K, seed=93)
+    y = oracle.matmul(What, x)
+    xd = f64(x)
+    prot = np.zeros(K, bool)
+    prot[L["idx"]] = True
+    xm = np.where(prot, 0.0, xd)                       # BSQ part sees masked x
+    C = K // 8
+    bits = np.unpackbits(L["codes"].reshape(S, N, C, 1), axis=3, bitorder="little")
+    sg = 1.0 - 2.0 * bits.astype(np.float64)           # [S][N][C][8]
+    n = L["norms"].view(np.float16).astype(np.float64)  # [S][N][C]
+    ref = np.zeros((2, N))
+    for s in range(S):
+        xt = np.einsum("kj,bck->bcj", Bs[s], xm.reshape(2, C, 8))   # B^T x per chunk
+        ref += np.einsum("nc,ncj,bcj->bn", n[s], sg[s], xt)
+    sc = L["scale"].view(np.float16).astype(np.float64)
+    ref += xd[:, L["idx"]] @ (sc[None, :] * L["q8"][:, :p].astype(np.float64)).T
+    assert np.allclose(y, ref, rtol=1e-12, atol=1e-12 * np.abs(ref).max())
+
+
+def test_table_decode_with_exact_identity_table():
+    """A table of +-1/2 (exact in binary16) is the norm-rescale decoder with
+    1/sqrt(8) replaced by 1/2: the BSQ columns are numpy's sum of
+    n * sign / 2 exactly, and the protected columns are scale * q8."""
+    N, K, S = 16, 64, 3
+    W = synth.layer_weights(N, K, seed=94)
+    L = oracle.encode(W, S=S, p=2)
+    half = np.array([[oracle.double_to_fp16(0.5 * sv) for sv in _signs(v)] for v in range(256)],
+                    np.uint16)
+    What = oracle.decode_rows_table(L, np.stack([half] * S))
+    C = K // 8
+    bits = np.unpackbits(L["codes"].reshape(S, N, C, 1), axis=3, bitorder="little")
+    n = L["norms"].view(np.float16).astype(np.float64)[..., None]
+    ref = ((1.0 - 2.0 * bits) * n * 0.5).sum(axis=0).reshape(N, K)
+    base = oracle.decode_rows(L)
+    ref[:, L["idx"]] = base[:, L["idx"]]
+    assert np.array_equal(What, ref)
+
+
+def test_table_decode_one_hot_table_picks_its_code():
+    """A table that is 1 at one (code byte, element) and 0 elsewhere, on one
+    stage only, returns that stage's norm exactly where that stage's chunk
+    carries that code, and 0 everywhere else outside the protected set."""
+    N, K, S = 12, 64, 2
+    W = synth.layer_weights(N, K, seed=95)
+    L = oracle.encode(W, S=S, p=0)
+    C = K // 8
+    for s0 in range(S):
+        v0 = int(L["codes"].reshape(S, N, C)[s0, 3, 5])
+        k0 = 6
+        tabs = np.zeros((S, 256, 8), np.uint16)
+        tabs[s0, v0, k0] = 0x3C00                     # 1.0
+        What = oracle.decode_rows_table(L, tabs)
+        want = np.zeros((N, K))
+        cs = L["codes"].reshape(S, N, C)[s0]
+        ns = L["norms"].reshape(S, N, C)[s0].view(np.float16).astype(np.float64)
+        for i in range(N):
+            for c in range(C):
+                if cs[i, c] == v0:
+                    want[i, 8 * c + k0] = ns[i, c]
+        assert np.array_equal(What, want)
+        assert What[3, 8 * 5 + k0] != 0 or ns[3, 5] == 0
+
+
+def test_mlp_decoder_odd_residual_and_limits():
+    rng = np.random.default_rng(96)
+    hdim = 16
+    W1 = rng.normal(size=(hdim, 8))
+    W2 = rng.normal(size=(8, hdim))
+    Wr = rng.normal(size=(hdim, hdim)) / 4
+    for wr in (None, Wr):
+        T = oracle.decoder_table_mlp(W1, W2, wr)
+        assert np.array_equal(T[255 - np.arange(256)], -T)      # D(-q) = -D(q)
+    # a zero residual block adds tanh(0) = 0
+    assert np.array_equal(oracle.decoder_table_mlp(W1, W2, np.zeros((hdim, hdim))),
+                          oracle.decoder_table_mlp(W1, W2))
+    # one hidden unit: T[v] = W2[:, 0] * tanh(W1[0] . q(v))
+    T = oracle.decoder_table_mlp(W1[:1], W2[:, :1])
+    for v in (0, 1, 77, 200, 255):
+        h = math.tanh(float(np.dot(W1[0], _signs(v) * INV_SQRT8)))
+        assert np.allclose(T[v], W2[:, 0] * h, rtol=1e-14, atol=1e-15)
+    # small inputs: tanh(e z) = e z (1 - (e z)^2/3 + ...), so the table tends to
+    # the linear decoder e W2 W1 q; with the residual block, e (W2 (I + Wr) W1) q
+    eps = 1e-5
+    lin = oracle.decoder_table_linear(W2 @ W1)
+    T = oracle.decoder_table_mlp(eps * W1, W2)
+    assert np.allclose(T / eps, lin, rtol=0, atol=1e-8 * np.abs(lin).max())
+    lin_r = oracle.decoder_table_linear(W2 @ (np.eye(hdim) + Wr) @ W1)
+    T = oracle.decoder_table_mlp(eps * W1, W2, Wr)
+    assert np.allclose(T / eps, lin_r, rtol=0, atol=1e-8 * np.abs(lin_r).max())
+    with pytest.raises(oracle.OracleError):
+        oracle.decoder_table_mlp(np.zeros((0, 8)), np.zeros((8, 0)))
