@@ -40,7 +40,7 @@ typedef struct CUstream_st *bisco_stream_t;
 typedef enum {
     BISCO_OK = 0,
     BISCO_ERR_INVALID_ARG = 1,  /* bad size, NULL or misaligned pointer        */
-    BISCO_ERR_UNSUPPORTED = 2,  /* valid but not implemented (d != 8, axis 1)  */
+    BISCO_ERR_UNSUPPORTED = 2,  /* valid but not implemented (d != 8)          */
     BISCO_ERR_RANGE = 3,        /* encode: non-finite weight, fp16 norm/scale overflow */
     BISCO_ERR_CUDA = 4,         /* a CUDA runtime call failed                  */
     BISCO_ERR_TIMEOUT = 5       /* a bounded device-side wait expired          */
@@ -66,14 +66,24 @@ typedef enum {
  *
  * The decoded weight is  What[i][j] = sum_s (+-) norm_s[i][j/8] / sqrt(8)
  * for j not protected, and q8_scale[t] * q8[i][t] for j = prot_idx[t].
+ *
+ * With protect_axis = 1 the protected channels are OUTPUT ROWS (Sec. III-E
+ * Eq. 9: the gate/up rows of a gated MLP, coupled with the down columns):
+ *   q8       [p][kp]      int8    protected row t at q8[t*kp + k],
+ *                                 kp = roundup(K, 16), padding zero.
+ *   q8_scale [p]          uint16  binary16 per-row scale, max_k |W_ik| / 127.
+ *   prot_idx [p]          int32   protected output rows, strictly ascending.
+ * Those rows decode to What[i][k] = q8_scale[t] * q8[t][k] (i = prot_idx[t]);
+ * the encoder zeroes them in the stage target, so their chunks store norm 0
+ * and sign byte 0.  0 <= p <= N.
  */
 typedef struct {
     int32_t n_out;        /* N >= 1                                       */
     int32_t k_in;         /* K >= 8, K % 8 == 0                            */
     int32_t chunk_dim;    /* d; only 8 is supported                        */
     int32_t stages;       /* S in {1, 2, 3}                                */
-    int32_t n_protected;  /* p, 0 <= p <= K (the caller's ceil(rho * K))   */
-    int32_t protect_axis; /* 0 = input columns; 1 (output rows) unsupported */
+    int32_t n_protected;  /* p: 0 <= p <= K (axis 0), 0 <= p <= N (axis 1) */
+    int32_t protect_axis; /* 0 = input columns; 1 = output rows            */
     uint8_t *codes;
     uint16_t *norms;
     int8_t *q8;
@@ -82,7 +92,7 @@ typedef struct {
 } bisco_layer;
 
 /* ABI version of this header (major * 100 + minor). */
-#define BISCO_ABI_VERSION 104
+#define BISCO_ABI_VERSION 105
 int32_t bisco_abi_version(void);
 
 /* Static string for a status code (never NULL). */
@@ -98,10 +108,25 @@ bisco_status bisco_encoded_sizes(int32_t N, int32_t K, int32_t d, int32_t S,
                                  int32_t p, size_t out_bytes[5]);
 
 /*
+ * bisco_encoded_sizes for either protection axis: with axis = 1 the q8
+ * buffer is p * roundup(K, 16) bytes and 0 <= p <= N (INVALID_ARG else, and
+ * for an axis other than 0 or 1).  Axis 0 gives bisco_encoded_sizes.
+ */
+bisco_status bisco_encoded_sizes_axis(int32_t N, int32_t K, int32_t d, int32_t S, int32_t p,
+                                      int32_t axis, size_t out_bytes[5]);
+
+/*
  * Scratch bytes bisco_encode needs for an N x K layer (per-column scores and
  * the protected-column map); 0 on invalid sizes.
  */
 size_t bisco_encode_workspace_bytes(int32_t N, int32_t K);
+
+/*
+ * The same for either protection axis (axis 1: per-row scores, ranks and the
+ * protected-row map, 13 bytes per row rounded up); it also covers
+ * bisco_encode_with_set.  0 on invalid sizes or axis.
+ */
+size_t bisco_encode_workspace_bytes_axis(int32_t N, int32_t K, int32_t axis);
 
 /*
  * Offline encoder (Sec. III-E Eq. 8, Eq. 10; Sec. III-C Eq. 3; Sec. III-D
@@ -119,9 +144,48 @@ size_t bisco_encode_workspace_bytes(int32_t N, int32_t K);
  * at least bisco_encode_workspace_bytes(N, K) bytes.  Non-finite weights or
  * an fp16 overflow latch BISCO_ERR_RANGE in the device error word; the
  * outputs are then unspecified.
+ * With L->protect_axis = 1 the protected channels are output rows: step 1
+ * scores rows, score_i = g_i * sqrt(sum_k W_ik^2) (g: [N], ascending k),
+ * step 2 quantises each protected row with one scale (max_k |W_ik| / 127),
+ * and step 3 runs on W with the protected rows zeroed.  The workspace is
+ * then bisco_encode_workspace_bytes_axis(N, K, 1) bytes.
  */
 bisco_status bisco_encode(const uint16_t *W_bf16, const float *g, const bisco_layer *L,
                           void *workspace, size_t workspace_bytes, bisco_stream_t stream);
+
+/*
+ * bisco_encode with the protected set given instead of selected: steps 2
+ * and 3 above with P = idx_in (device, [p] int32, strictly ascending,
+ * columns in [0, K) for axis 0, rows in [0, N) for axis 1; NULL allowed
+ * when p == 0), copied to L->prot_idx.  This encodes the three projections
+ * of a gated MLP on the one coupled set of bisco_select_coupled (gate and
+ * up with axis 1, down with axis 0).  An index out of range or out of order
+ * latches BISCO_ERR_INVALID_ARG in the device error word (an out-of-range
+ * one is stored as 0; the outputs are then unspecified).  workspace: at
+ * least bisco_encode_workspace_bytes_axis(N, K, axis) bytes.
+ */
+bisco_status bisco_encode_with_set(const uint16_t *W_bf16, const int32_t *idx_in,
+                                   const bisco_layer *L, void *workspace, size_t workspace_bytes,
+                                   bisco_stream_t stream);
+
+/*
+ * Coupled protected set of a gated MLP (Sec. III-E Eq. 9): for intermediate
+ * channel j < F,
+ *   S_j = gg_j ||Wg[j,:]||_2 + gu_j ||Wu[j,:]||_2 + gd_j ||Wd[:,j]||_2
+ * (fp64, each sum of squares in ascending index, the three terms added in
+ * that order; a NULL g means 1), and idx_out = the p channels of largest
+ * S_j, ties to the lower j, ascending.  Wg, Wu: [F][H] bf16 (gate_proj and
+ * up_proj weights), Wd: [H][F] bf16 (down_proj), 16-byte aligned; gg, gu,
+ * gd: [F] float or NULL.  F >= 1, H >= 1, 0 <= p <= F.  idx_out: [p] int32
+ * device.  workspace: at least bisco_select_coupled_workspace_bytes(F)
+ * bytes.  Non-finite weights latch BISCO_ERR_RANGE.
+ */
+size_t bisco_select_coupled_workspace_bytes(int32_t F);
+bisco_status bisco_select_coupled(const uint16_t *Wg_bf16, const uint16_t *Wu_bf16,
+                                  const uint16_t *Wd_bf16, const float *gg, const float *gu,
+                                  const float *gd, int32_t F, int32_t H, int32_t p,
+                                  int32_t *idx_out, void *workspace, size_t workspace_bytes,
+                                  bisco_stream_t stream);
 
 /*
  * bisco_encode without a workspace argument, for callers that cannot
@@ -156,6 +220,10 @@ bisco_status bisco_encode_noalloc(const uint16_t *W_bf16, const float *g, const 
  * starts fetching the layer's buffers before, so they must not be written
  * by the kernel immediately ahead of it (bisco_encode ends with an empty
  * kernel for this reason; copies and events order as usual).
+ * For a layer with protect_axis = 1, a second kernel then overwrites the
+ * protected rows: y[b][prot_idx[t]] = q8_scale[t] * sum_k q8[t][k] * x[b][k]
+ * (int8 x bf16 products, exact in fp32, summed in fp32).  The same holds
+ * for bisco_gemv_multi and bisco_gemm.
  */
 bisco_status bisco_gemv(const bisco_layer *L, const uint16_t *x_bf16, int32_t B, float *y,
                         bisco_stream_t stream);
@@ -188,8 +256,9 @@ bisco_status bisco_gemv_multi(const bisco_layer *layers, int32_t G, const uint16
  * X_bf16: [M][K] device; Y: [M][N] float32 device, fully overwritten.
  * workspace: device, 16-byte aligned, at least
  * bisco_gemm_workspace_bytes(L, M) bytes (M * (roundup(K,128) +
- * 2 * roundup(p,64)) * 2 on the tensor-core path; NULL when that is 0).
- * It holds the fp16 copy of X and is overwritten.
+ * 2 * roundup(p,64)) * 2 on the tensor-core path, with p = 0 for a
+ * row-protected layer; NULL when that is 0).  It holds the fp16 copy of X
+ * and is overwritten.
  */
 size_t bisco_gemm_workspace_bytes(const bisco_layer *L, int32_t M);
 bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M, float *Y,
@@ -203,7 +272,8 @@ bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M,
  *     out[i][j] = scale_j * q8[i][j]                                 j protected
  * The stage sum is formed in fp32 and rounded once after the 1/sqrt(8)
  * scale (to fp32, or from there to bf16 / fp16 with round-to-nearest-even);
- * the protected values are exact in fp32.
+ * the protected values are exact in fp32.  With protect_axis = 1 the
+ * protected rows are out[prot_idx[t]][k] = q8_scale[t] * q8[t][k].
  * out: [N][K] device, 16-byte aligned, fully overwritten; dtype one of
  * BISCO_DENSE_*.  Asynchronous on `stream` (two kernels).
  */

@@ -17,8 +17,10 @@ OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_RANGE, ERR_CUDA, ERR_TIMEOUT = range(6
 # Functions declared in include/bisco.h (kept in sync by tests/test_abi.py).
 EXPORTS = (
     "bisco_abi_version", "bisco_status_string", "bisco_encoded_sizes",
-    "bisco_encode_workspace_bytes", "bisco_encode", "bisco_encode_noalloc", "bisco_gemv",
-    "bisco_gemv_multi",
+    "bisco_encoded_sizes_axis", "bisco_encode_workspace_bytes",
+    "bisco_encode_workspace_bytes_axis", "bisco_encode", "bisco_encode_with_set",
+    "bisco_select_coupled_workspace_bytes", "bisco_select_coupled",
+    "bisco_encode_noalloc", "bisco_gemv", "bisco_gemv_multi",
     "bisco_gemm_workspace_bytes", "bisco_gemm", "bisco_decode_dense", "bisco_lora_apply",
     "bisco_get_device_error",
 )
@@ -62,10 +64,20 @@ def load(path: str = LIB_PATH):
     lib.bisco_status_string.argtypes = [i32]
     lib.bisco_encoded_sizes.restype = st
     lib.bisco_encoded_sizes.argtypes = [i32, i32, i32, i32, i32, ctypes.POINTER(sz)]
+    lib.bisco_encoded_sizes_axis.restype = st
+    lib.bisco_encoded_sizes_axis.argtypes = [i32, i32, i32, i32, i32, i32, ctypes.POINTER(sz)]
     lib.bisco_encode_workspace_bytes.restype = sz
     lib.bisco_encode_workspace_bytes.argtypes = [i32, i32]
+    lib.bisco_encode_workspace_bytes_axis.restype = sz
+    lib.bisco_encode_workspace_bytes_axis.argtypes = [i32, i32, i32]
     lib.bisco_encode.restype = st
     lib.bisco_encode.argtypes = [P, P, Lp, P, sz, P]
+    lib.bisco_encode_with_set.restype = st
+    lib.bisco_encode_with_set.argtypes = [P, P, Lp, P, sz, P]
+    lib.bisco_select_coupled_workspace_bytes.restype = sz
+    lib.bisco_select_coupled_workspace_bytes.argtypes = [i32]
+    lib.bisco_select_coupled.restype = st
+    lib.bisco_select_coupled.argtypes = [P, P, P, P, P, P, i32, i32, i32, P, P, sz, P]
     lib.bisco_encode_noalloc.restype = st
     lib.bisco_encode_noalloc.argtypes = [P, P, Lp, P]
     lib.bisco_gemv.restype = st
@@ -116,8 +128,22 @@ def bisco_encoded_sizes(N, K, S, p, d=8):
     return [int(v) for v in out]
 
 
+def bisco_encoded_sizes_axis(N, K, S, p, axis, d=8):
+    out = (ctypes.c_size_t * 5)()
+    _check(load().bisco_encoded_sizes_axis(N, K, d, S, p, axis, out), "bisco_encoded_sizes_axis")
+    return [int(v) for v in out]
+
+
 def bisco_encode_workspace_bytes(N, K) -> int:
     return int(load().bisco_encode_workspace_bytes(N, K))
+
+
+def bisco_encode_workspace_bytes_axis(N, K, axis) -> int:
+    return int(load().bisco_encode_workspace_bytes_axis(N, K, axis))
+
+
+def bisco_select_coupled_workspace_bytes(F) -> int:
+    return int(load().bisco_select_coupled_workspace_bytes(F))
 
 
 def bisco_gemm_workspace_bytes(L, M) -> int:
@@ -127,68 +153,133 @@ def bisco_gemm_workspace_bytes(L, M) -> int:
 
 
 class Layer:
-    """A coded layer in device memory (torch tensors) plus its C struct."""
+    """A coded layer in device memory (torch tensors) plus its C struct.
+    axis 0 protects input columns (q8 [N][p_pad]); axis 1 protects output
+    rows (q8 [p][roundup(K, 16)])."""
 
-    def __init__(self, N, K, S, p, device="cuda", d=8):
+    def __init__(self, N, K, S, p, device="cuda", d=8, axis=0):
         import torch
-        sizes = bisco_encoded_sizes(N, K, S, p, d)
-        self.N, self.K, self.S, self.p = N, K, S, p
+        sizes = bisco_encoded_sizes(N, K, S, p, d) if axis == 0 else \
+            bisco_encoded_sizes_axis(N, K, S, p, axis, d)
+        self.N, self.K, self.S, self.p, self.axis = N, K, S, p, axis
         self.p_pad = (p + 15) // 16 * 16
+        self.kp = (K + 15) // 16 * 16
         dev = torch.device(device)
         self.codes = torch.empty((S, N, K // 8), dtype=torch.uint8, device=dev)
         self.norms = torch.empty((S, N, K // 8), dtype=torch.int16, device=dev)
-        self.q8 = torch.empty((N, max(self.p_pad, 16)), dtype=torch.int8, device=dev)
+        if axis == 1:
+            self.q8 = torch.empty((max(p, 1), self.kp), dtype=torch.int8, device=dev)
+        else:
+            self.q8 = torch.empty((N, max(self.p_pad, 16)), dtype=torch.int8, device=dev)
         self.scale = torch.empty((max(p, 8),), dtype=torch.int16, device=dev)
         self.idx = torch.empty((max(p, 4),), dtype=torch.int32, device=dev)
         assert sizes[0] == self.codes.numel() and sizes[1] == 2 * self.norms.numel()
-        self.c = bisco_layer(N, K, d, S, p, 0, self.codes.data_ptr(), self.norms.data_ptr(),
+        assert sizes[2] <= self.q8.numel()
+        self.c = bisco_layer(N, K, d, S, p, axis, self.codes.data_ptr(), self.norms.data_ptr(),
                              self.q8.data_ptr(), self.scale.data_ptr(), self.idx.data_ptr())
 
     @property
     def compressed_bytes(self) -> int:
         """Algorithmic payload: signs + norms + unpadded q8 + scales + indices."""
-        return self.S * self.N * (self.K // 8) * 3 + self.N * self.p + 6 * self.p
+        q8 = self.p * (self.K if self.axis == 1 else self.N)
+        return self.S * self.N * (self.K // 8) * 3 + q8 + 6 * self.p
 
     def to_numpy(self):
         """Host copy in the oracle's dict layout."""
         p = self.p
-        return dict(N=self.N, K=self.K, S=self.S, p=p,
-                    codes=self.codes.cpu().numpy(),
-                    norms=self.norms.cpu().numpy().view("uint16"),
-                    q8=self.q8[:, :self.p_pad].cpu().numpy(),
-                    scale=self.scale[:p].cpu().numpy().view("uint16"),
-                    idx=self.idx[:p].cpu().numpy())
+        L = dict(N=self.N, K=self.K, S=self.S, p=p,
+                 codes=self.codes.cpu().numpy(),
+                 norms=self.norms.cpu().numpy().view("uint16"),
+                 scale=self.scale[:p].cpu().numpy().view("uint16"),
+                 idx=self.idx[:p].cpu().numpy())
+        if self.axis == 1:
+            L["axis"] = 1
+            L["q8"] = self.q8[:p].cpu().numpy()
+        else:
+            L["q8"] = self.q8[:, :self.p_pad].cpu().numpy()
+        return L
 
     @classmethod
     def from_numpy(cls, L, device="cuda"):
         import numpy as np
         import torch
-        obj = cls(L["N"], L["K"], L["S"], L["p"], device)
+        axis = L.get("axis", 0)
+        obj = cls(L["N"], L["K"], L["S"], L["p"], device, axis=axis)
         obj.codes.copy_(torch.from_numpy(np.ascontiguousarray(L["codes"])))
         obj.norms.copy_(torch.from_numpy(np.ascontiguousarray(L["norms"]).view(np.int16)))
         if L["p"]:
-            obj.q8[:, :obj.p_pad].copy_(torch.from_numpy(np.ascontiguousarray(L["q8"])))
+            q8 = torch.from_numpy(np.ascontiguousarray(L["q8"]))
+            if axis == 1:
+                obj.q8[:L["p"]].copy_(q8)
+            else:
+                obj.q8[:, :obj.p_pad].copy_(q8)
             obj.scale[:L["p"]].copy_(torch.from_numpy(np.ascontiguousarray(L["scale"]).view(np.int16)))
             obj.idx[:L["p"]].copy_(torch.from_numpy(np.ascontiguousarray(L["idx"])))
         return obj
 
 
-def bisco_encode(W_bits, S, p, g=None, workspace=None, stream=None) -> Layer:
-    """Encodes a device tensor of bf16 bits [N][K] (int16 or bfloat16)."""
+def _bits2d(W_bits):
     import torch
     if W_bits.dtype == torch.bfloat16:
         W_bits = W_bits.view(torch.int16)
     assert W_bits.is_cuda and W_bits.is_contiguous() and W_bits.dim() == 2
+    return W_bits
+
+
+def bisco_encode(W_bits, S, p, g=None, workspace=None, stream=None, axis=0) -> Layer:
+    """Encodes a device tensor of bf16 bits [N][K] (int16 or bfloat16);
+    axis 1 protects the p output rows of largest norm instead of columns."""
+    import torch
+    W_bits = _bits2d(W_bits)
     N, K = W_bits.shape
-    L = Layer(N, K, S, p, W_bits.device)
-    need = bisco_encode_workspace_bytes(N, K)
+    L = Layer(N, K, S, p, W_bits.device, axis=axis)
+    need = bisco_encode_workspace_bytes_axis(N, K, axis)
     if workspace is None:
         workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=W_bits.device)
     if g is not None:
-        assert g.dtype == torch.float32 and g.is_cuda and g.numel() == K
+        assert g.dtype == torch.float32 and g.is_cuda and g.numel() == (N if axis == 1 else K)
     _check(load().bisco_encode(_ptr(W_bits), _ptr(g), ctypes.byref(L.c), _ptr(workspace),
                                workspace.numel(), _stream(stream)), "bisco_encode")
     return L
+
+
+def bisco_encode_with_set(W_bits, S, idx, axis, workspace=None, stream=None) -> Layer:
+    """Encodes with the protected set given (device int32 [p], ascending):
+    columns for axis 0, rows for axis 1."""
+    import torch
+    W_bits = _bits2d(W_bits)
+    N, K = W_bits.shape
+    p = int(idx.numel())
+    assert idx.dtype == torch.int32 and idx.is_cuda and idx.is_contiguous()
+    L = Layer(N, K, S, p, W_bits.device, axis=axis)
+    need = bisco_encode_workspace_bytes_axis(N, K, axis)
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=W_bits.device)
+    _check(load().bisco_encode_with_set(_ptr(W_bits), _ptr(idx) if p else None, ctypes.byref(L.c),
+                                        _ptr(workspace), workspace.numel(), _stream(stream)),
+           "bisco_encode_with_set")
+    return L
+
+
+def bisco_select_coupled(Wg_bits, Wu_bits, Wd_bits, p, gg=None, gu=None, gd=None,
+                         workspace=None, stream=None):
+    """The coupled protected set (Eq. 9) of a gated MLP: gate/up [F][H],
+    down [H][F]; returns the p channels as a device int32 tensor."""
+    import torch
+    Wg_bits, Wu_bits, Wd_bits = _bits2d(Wg_bits), _bits2d(Wu_bits), _bits2d(Wd_bits)
+    F, H = Wg_bits.shape
+    assert tuple(Wu_bits.shape) == (F, H) and tuple(Wd_bits.shape) == (H, F)
+    idx = torch.empty((max(p, 1),), dtype=torch.int32, device=Wg_bits.device)
+    need = bisco_select_coupled_workspace_bytes(F)
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=Wg_bits.device)
+    for g in (gg, gu, gd):
+        assert g is None or (g.dtype == torch.float32 and g.is_cuda and g.numel() == F)
+    _check(load().bisco_select_coupled(_ptr(Wg_bits), _ptr(Wu_bits), _ptr(Wd_bits), _ptr(gg),
+                                       _ptr(gu), _ptr(gd), F, H, p, _ptr(idx), _ptr(workspace),
+                                       workspace.numel(), _stream(stream)),
+           "bisco_select_coupled")
+    return idx[:p]
 
 
 def bisco_encode_noalloc(W_bits, S, p, g=None, stream=None) -> Layer:

@@ -36,9 +36,10 @@ bisco_status check_layer(const bisco_layer *L, bool check_buffers) {
     if (!L) return BISCO_ERR_INVALID_ARG;
     if (L->n_out < 1 || L->k_in < 8 || L->k_in % 8 != 0) return BISCO_ERR_INVALID_ARG;
     if (L->stages < 1 || L->stages > 3) return BISCO_ERR_INVALID_ARG;
-    if (L->n_protected < 0 || L->n_protected > L->k_in) return BISCO_ERR_INVALID_ARG;
     if (L->protect_axis != 0 && L->protect_axis != 1) return BISCO_ERR_INVALID_ARG;
-    if (L->chunk_dim != 8 || L->protect_axis != 0) return BISCO_ERR_UNSUPPORTED;
+    const int32_t p_max = L->protect_axis == 1 ? L->n_out : L->k_in;
+    if (L->n_protected < 0 || L->n_protected > p_max) return BISCO_ERR_INVALID_ARG;
+    if (L->chunk_dim != 8) return BISCO_ERR_UNSUPPORTED;
     if (static_cast<int64_t>(L->n_out) * L->k_in > (int64_t(1) << 40)) return BISCO_ERR_INVALID_ARG;
     if (!check_buffers) return BISCO_OK;
     if (!L->codes || !L->norms || !aligned16(L->codes) || !aligned16(L->norms))
@@ -49,6 +50,17 @@ bisco_status check_layer(const bisco_layer *L, bool check_buffers) {
             return BISCO_ERR_INVALID_ARG;
     }
     return BISCO_OK;
+}
+
+// The binary spherical stages of a row-protected layer alone: the decode
+// kernels run on this copy (no protected columns; they read none of the
+// protected buffers when p == 0) and rows.cu then overwrites the protected
+// rows.
+bisco_layer bsq_only(const bisco_layer &L) {
+    bisco_layer b = L;
+    b.n_protected = 0;
+    b.protect_axis = 0;
+    return b;
 }
 
 }  // namespace
@@ -151,7 +163,30 @@ bisco_status bisco_encoded_sizes(int32_t N, int32_t K, int32_t d, int32_t S, int
     return BISCO_OK;
 }
 
+bisco_status bisco_encoded_sizes_axis(int32_t N, int32_t K, int32_t d, int32_t S, int32_t p,
+                                      int32_t axis, size_t out_bytes[5]) {
+    if (axis == 0) return bisco_encoded_sizes(N, K, d, S, p, out_bytes);
+    if (axis != 1 || !out_bytes) return BISCO_ERR_INVALID_ARG;
+    if (N < 1 || K < 8 || K % 8 != 0 || S < 1 || S > 3 || p < 0 || p > N)
+        return BISCO_ERR_INVALID_ARG;
+    if (d != 8) return BISCO_ERR_UNSUPPORTED;
+    const size_t C = static_cast<size_t>(K) / 8;
+    const size_t kp = (static_cast<size_t>(K) + 15) / 16 * 16;
+    out_bytes[0] = static_cast<size_t>(S) * N * C;
+    out_bytes[1] = static_cast<size_t>(S) * N * C * 2;
+    out_bytes[2] = static_cast<size_t>(p) * kp;
+    out_bytes[3] = static_cast<size_t>(p) * 2;
+    out_bytes[4] = static_cast<size_t>(p) * 4;
+    return BISCO_OK;
+}
+
 size_t bisco_encode_workspace_bytes(int32_t N, int32_t K) { return encode_workspace_bytes(N, K); }
+
+size_t bisco_encode_workspace_bytes_axis(int32_t N, int32_t K, int32_t axis) {
+    return encode_workspace_bytes_axis(N, K, axis);
+}
+
+size_t bisco_select_coupled_workspace_bytes(int32_t F) { return select_coupled_workspace_bytes(F); }
 
 bisco_status bisco_encode(const uint16_t *W_bf16, const float *g, const bisco_layer *L,
                           void *workspace, size_t workspace_bytes, bisco_stream_t stream) {
@@ -160,11 +195,56 @@ bisco_status bisco_encode(const uint16_t *W_bf16, const float *g, const bisco_la
     if (!W_bf16 || !aligned16(W_bf16) || (g && (reinterpret_cast<uintptr_t>(g) & 3u)))
         return BISCO_ERR_INVALID_ARG;
     if (!workspace || !aligned16(workspace) ||
-        workspace_bytes < encode_workspace_bytes(L->n_out, L->k_in))
+        workspace_bytes < encode_workspace_bytes_axis(L->n_out, L->k_in, L->protect_axis))
         return BISCO_ERR_INVALID_ARG;
     int *err = device_error_word(&st);
     if (!err) return st;
+    if (L->protect_axis == 1)
+        return launch_encode_rows(W_bf16, g, *L, workspace, err,
+                                  reinterpret_cast<cudaStream_t>(stream));
     return launch_encode(W_bf16, g, *L, workspace, err, reinterpret_cast<cudaStream_t>(stream));
+}
+
+bisco_status bisco_encode_with_set(const uint16_t *W_bf16, const int32_t *idx_in,
+                                   const bisco_layer *L, void *workspace, size_t workspace_bytes,
+                                   bisco_stream_t stream) {
+    bisco_status st = check_layer(L, true);
+    if (st != BISCO_OK) return st;
+    if (!W_bf16 || !aligned16(W_bf16)) return BISCO_ERR_INVALID_ARG;
+    if (L->n_protected > 0 && (!idx_in || (reinterpret_cast<uintptr_t>(idx_in) & 3u)))
+        return BISCO_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace) ||
+        workspace_bytes < encode_workspace_bytes_axis(L->n_out, L->k_in, L->protect_axis))
+        return BISCO_ERR_INVALID_ARG;
+    int *err = device_error_word(&st);
+    if (!err) return st;
+    return launch_encode_with_set(W_bf16, idx_in, *L, workspace, err,
+                                  reinterpret_cast<cudaStream_t>(stream));
+}
+
+bisco_status bisco_select_coupled(const uint16_t *Wg_bf16, const uint16_t *Wu_bf16,
+                                  const uint16_t *Wd_bf16, const float *gg, const float *gu,
+                                  const float *gd, int32_t F, int32_t H, int32_t p,
+                                  int32_t *idx_out, void *workspace, size_t workspace_bytes,
+                                  bisco_stream_t stream) {
+    if (F < 1 || H < 1 || p < 0 || p > F) return BISCO_ERR_INVALID_ARG;
+    if (static_cast<int64_t>(F) * H > (int64_t(1) << 40)) return BISCO_ERR_INVALID_ARG;
+    const void *w[3] = {Wg_bf16, Wu_bf16, Wd_bf16};
+    for (const void *q : w)
+        if (!q || !aligned16(q)) return BISCO_ERR_INVALID_ARG;
+    const float *g[3] = {gg, gu, gd};
+    for (const float *q : g)
+        if (q && (reinterpret_cast<uintptr_t>(q) & 3u)) return BISCO_ERR_INVALID_ARG;
+    if (p > 0 && (!idx_out || (reinterpret_cast<uintptr_t>(idx_out) & 3u)))
+        return BISCO_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace) ||
+        workspace_bytes < select_coupled_workspace_bytes(F))
+        return BISCO_ERR_INVALID_ARG;
+    bisco_status st;
+    int *err = device_error_word(&st);
+    if (!err) return st;
+    return launch_select_coupled(Wg_bf16, Wu_bf16, Wd_bf16, gg, gu, gd, F, H, p, idx_out,
+                                 workspace, err, reinterpret_cast<cudaStream_t>(stream));
 }
 
 bisco_status bisco_gemv(const bisco_layer *L, const uint16_t *x_bf16, int32_t B, float *y,
@@ -176,7 +256,13 @@ bisco_status bisco_gemv(const bisco_layer *L, const uint16_t *x_bf16, int32_t B,
     if (!x_bf16 || !y || !aligned16(x_bf16) || !aligned16(y)) return BISCO_ERR_INVALID_ARG;
     int *err = device_error_word(&st);
     if (!err) return st;
-    return launch_gemv(*L, x_bf16, B, y, err, reinterpret_cast<cudaStream_t>(stream));
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (L->protect_axis == 1) {
+        st = launch_gemv(bsq_only(*L), x_bf16, B, y, err, s);
+        if (st != BISCO_OK) return st;
+        return launch_rows_apply(*L, x_bf16, B, y, err, s);
+    }
+    return launch_gemv(*L, x_bf16, B, y, err, s);
 }
 
 bisco_status bisco_gemv_multi(const bisco_layer *layers, int32_t G, const uint16_t *x_bf16,
@@ -196,12 +282,23 @@ bisco_status bisco_gemv_multi(const bisco_layer *layers, int32_t G, const uint16
     bisco_status st;
     int *err = device_error_word(&st);
     if (!err) return st;
-    return launch_gemv_multi(layers, G, x_bf16, B, y, err, reinterpret_cast<cudaStream_t>(stream));
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    bisco_layer stages[BISCO_GEMV_MULTI_MAX];
+    bool rows = false;
+    for (int g = 0; g < G; ++g) {
+        rows |= layers[g].protect_axis == 1;
+        stages[g] = layers[g].protect_axis == 1 ? bsq_only(layers[g]) : layers[g];
+    }
+    if (!rows) return launch_gemv_multi(layers, G, x_bf16, B, y, err, s);
+    st = launch_gemv_multi(stages, G, x_bf16, B, y, err, s);
+    for (int g = 0; g < G && st == BISCO_OK; ++g)
+        if (layers[g].protect_axis == 1) st = launch_rows_apply(layers[g], x_bf16, B, y[g], err, s);
+    return st;
 }
 
 size_t bisco_gemm_workspace_bytes(const bisco_layer *L, int32_t M) {
     if (M < 0 || check_layer(L, false) != BISCO_OK) return 0;
-    return gemm_workspace_bytes(*L, M);
+    return gemm_workspace_bytes(L->protect_axis == 1 ? bsq_only(*L) : *L, M);
 }
 
 bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M, float *Y,
@@ -211,13 +308,16 @@ bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M,
     if (M < 0) return BISCO_ERR_INVALID_ARG;
     if (M == 0) return BISCO_OK;
     if (!X_bf16 || !Y || !aligned16(X_bf16) || !aligned16(Y)) return BISCO_ERR_INVALID_ARG;
-    const size_t need = gemm_workspace_bytes(*L, M);
+    const bisco_layer Ls = L->protect_axis == 1 ? bsq_only(*L) : *L;
+    const size_t need = gemm_workspace_bytes(Ls, M);
     if (need && (!workspace || !aligned16(workspace) || workspace_bytes < need))
         return BISCO_ERR_INVALID_ARG;
     int *err = device_error_word(&st);
     if (!err) return st;
-    return launch_gemm(*L, X_bf16, M, Y, workspace, workspace_bytes, err,
-                       reinterpret_cast<cudaStream_t>(stream));
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    st = launch_gemm(Ls, X_bf16, M, Y, workspace, workspace_bytes, err, s);
+    if (st != BISCO_OK || L->protect_axis != 1) return st;
+    return launch_rows_apply(*L, X_bf16, M, Y, err, s);
 }
 
 bisco_status bisco_decode_dense(const bisco_layer *L, void *out, int32_t dtype,
@@ -229,7 +329,13 @@ bisco_status bisco_decode_dense(const bisco_layer *L, void *out, int32_t dtype,
     if (!out || !aligned16(out)) return BISCO_ERR_INVALID_ARG;
     int *err = device_error_word(&st);
     if (!err) return st;
-    return launch_decode_dense(*L, out, dtype, err, reinterpret_cast<cudaStream_t>(stream));
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (L->protect_axis == 1) {
+        st = launch_decode_dense(bsq_only(*L), out, dtype, err, s);
+        if (st != BISCO_OK) return st;
+        return launch_rows_dense(*L, out, dtype, err, s);
+    }
+    return launch_decode_dense(*L, out, dtype, err, s);
 }
 
 bisco_status bisco_lora_apply(const uint16_t *A, const uint16_t *Bm, int32_t rank, int32_t N,

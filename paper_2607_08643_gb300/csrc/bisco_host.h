@@ -28,6 +28,22 @@ bisco_status launch_gemv(const bisco_layer &L, const uint16_t *x, int B, float *
                          cudaStream_t stream);
 bisco_status launch_gemv_multi(const bisco_layer *Ls, int G, const uint16_t *x, int B,
                                float *const *y, int *err, cudaStream_t stream);
+// Output-row protection and the coupled MLP set (encode.cu, rows.cu).
+size_t encode_workspace_bytes_axis(int N, int K, int axis);
+size_t select_coupled_workspace_bytes(int F);
+bisco_status launch_encode_rows(const uint16_t *W, const float *g, const bisco_layer &L,
+                                void *workspace, int *err, cudaStream_t stream);
+bisco_status launch_encode_with_set(const uint16_t *W, const int32_t *idx_in,
+                                    const bisco_layer &L, void *workspace, int *err,
+                                    cudaStream_t stream);
+bisco_status launch_select_coupled(const uint16_t *Wg, const uint16_t *Wu, const uint16_t *Wd,
+                                   const float *gg, const float *gu, const float *gd, int F,
+                                   int H, int p, int32_t *idx_out, void *workspace, int *err,
+                                   cudaStream_t stream);
+bisco_status launch_rows_apply(const bisco_layer &L, const uint16_t *X, int M, float *Y, int *err,
+                               cudaStream_t stream);
+bisco_status launch_rows_dense(const bisco_layer &L, void *out, int dtype, int *err,
+                               cudaStream_t stream);
 size_t gemm_workspace_bytes(const bisco_layer &L, int M);
 bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *Y,
                          void *workspace, size_t ws_bytes, int *err, cudaStream_t stream);

@@ -1,5 +1,6 @@
 // encode.cu -- offline BiSCo encoder on the GPU (Sec. III-E Eq. 8 and
-// Eq. 10, Sec. III-C Eq. 3, Sec. III-D Eq. 5-7).
+// Eq. 10, Sec. III-C Eq. 3, Sec. III-D Eq. 5-7), with output-row
+// protection and the coupled MLP channel set of Sec. III-E Eq. 9.
 //
 // Every floating-point step is binary64 with an explicit rounding intrinsic
 // (no FMA contraction; this file is also compiled with --fmad=false), sums
@@ -168,7 +169,10 @@ __global__ void __launch_bounds__(256) k_q8(const uint16_t *__restrict__ W, int 
 }
 
 // Eq. 3 + Eq. 5-7: one thread per (row, chunk); S sign/norm stages on the
-// residual, protected entries held at zero in every stage.
+// residual, protected entries held at zero in every stage.  `prot` maps the
+// protected input columns ([K] bytes), or with kRows the protected output
+// rows ([N] bytes), whose chunks then code as norm 0, sign byte 0.
+template <bool kRows>
 __global__ void __launch_bounds__(256) k_stages(const uint16_t *__restrict__ W, int N, int K, int S,
                                                 const uint8_t *__restrict__ prot,
                                                 uint8_t *__restrict__ codes,
@@ -179,9 +183,15 @@ __global__ void __launch_bounds__(256) k_stages(const uint16_t *__restrict__ W, 
     const int i = static_cast<int>(e / C);
     const int c = static_cast<int>(e % C);
     const uint4 raw = *reinterpret_cast<const uint4 *>(W + static_cast<int64_t>(i) * K + 8 * c);
-    const uint2 pm = *reinterpret_cast<const uint2 *>(prot + 8 * c);
+    uint32_t pv[2];
+    if (kRows) {
+        pv[0] = pv[1] = prot[i] ? 0xFFFFFFFFu : 0u;
+    } else {
+        const uint2 pm = *reinterpret_cast<const uint2 *>(prot + 8 * c);
+        pv[0] = pm.x;
+        pv[1] = pm.y;
+    }
     const uint32_t wv[4] = {raw.x, raw.y, raw.z, raw.w};
-    const uint32_t pv[2] = {pm.x, pm.y};
     bool pr[8];
     double v[8];
 #pragma unroll
@@ -209,6 +219,121 @@ __global__ void __launch_bounds__(256) k_stages(const uint16_t *__restrict__ W, 
         const int64_t o = (static_cast<int64_t>(s) * N + i) * C + c;
         codes[o] = static_cast<uint8_t>(bits);
         norms[o] = n16;
+    }
+}
+
+// Row score for output-row protection: g_i * sqrt(sum_{k ascending} W_ik^2).
+// One thread per row; also rejects non-finite weights.
+__global__ void __launch_bounds__(128) k_rowscore(const uint16_t *__restrict__ W,
+                                                  const float *__restrict__ g, int N, int K,
+                                                  double *__restrict__ score, int *err) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= N) return;
+    const uint4 *row = reinterpret_cast<const uint4 *>(W + static_cast<int64_t>(i) * K);
+    double sum = 0.0;
+    bool bad = false;
+    for (int c = 0; c < K / 8; ++c) {
+        const uint4 raw = row[c];
+        const uint32_t wv[4] = {raw.x, raw.y, raw.z, raw.w};
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const uint16_t b = static_cast<uint16_t>(wv[k / 2] >> (16 * (k % 2)));
+            bad |= bf16_nonfinite(b);
+            const double w = bf16_to_f64(b);
+            sum = __dadd_rn(sum, __dmul_rn(w, w));
+        }
+    }
+    if (bad) latch_error(err, BISCO_ERR_RANGE);
+    double s = __dsqrt_rn(sum);
+    if (g) s = __dmul_rn(static_cast<double>(g[i]), s);
+    score[i] = s;
+}
+
+// Eq. 9 coupled score of intermediate channel j of a gated MLP (gate and up
+// [F][H], down [H][F]): the gate row norm, the up row norm and the down
+// column norm, each weighted by its own g (NULL = 1) and added in that
+// order.  One thread per channel.
+__global__ void __launch_bounds__(128) k_coupled_score(
+    const uint16_t *__restrict__ Wg, const uint16_t *__restrict__ Wu,
+    const uint16_t *__restrict__ Wd, const float *__restrict__ gg, const float *__restrict__ gu,
+    const float *__restrict__ gd, int F, int H, double *__restrict__ score, int *err) {
+    const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    if (j >= F) return;
+    double sg = 0.0, su = 0.0, sd = 0.0;
+    bool bad = false;
+    for (int h = 0; h < H; ++h) {
+        const uint16_t a = Wg[static_cast<int64_t>(j) * H + h];
+        const uint16_t b = Wu[static_cast<int64_t>(j) * H + h];
+        const uint16_t c = Wd[static_cast<int64_t>(h) * F + j];
+        bad |= bf16_nonfinite(a) | bf16_nonfinite(b) | bf16_nonfinite(c);
+        const double da = bf16_to_f64(a), db = bf16_to_f64(b), dc = bf16_to_f64(c);
+        sg = __dadd_rn(sg, __dmul_rn(da, da));
+        su = __dadd_rn(su, __dmul_rn(db, db));
+        sd = __dadd_rn(sd, __dmul_rn(dc, dc));
+    }
+    if (bad) latch_error(err, BISCO_ERR_RANGE);
+    double tg = __dsqrt_rn(sg), tu = __dsqrt_rn(su), td = __dsqrt_rn(sd);
+    if (gg) tg = __dmul_rn(static_cast<double>(gg[j]), tg);
+    if (gu) tu = __dmul_rn(static_cast<double>(gu[j]), tu);
+    if (gd) td = __dmul_rn(static_cast<double>(gd[j]), td);
+    score[j] = __dadd_rn(__dadd_rn(tg, tu), td);
+}
+
+// A caller-given protected set (one CTA): the map over the n channels and
+// the stored index list.  An index outside [0, n) or out of ascending
+// order latches BISCO_ERR_INVALID_ARG; an out-of-range one is stored as 0
+// so that the kernels after this one stay inside the weight.
+__global__ void __launch_bounds__(1024) k_set_map(const int32_t *__restrict__ idx_in, int p, int n,
+                                                  uint8_t *__restrict__ map,
+                                                  int32_t *__restrict__ idx_out, int *err) {
+    for (int j = threadIdx.x; j < n; j += blockDim.x) map[j] = 0;
+    __syncthreads();
+    for (int t = threadIdx.x; t < p; t += blockDim.x) {
+        const int i = idx_in[t];
+        const bool in_range = i >= 0 && i < n;
+        if (!in_range || (t > 0 && idx_in[t - 1] >= i)) latch_error(err, BISCO_ERR_INVALID_ARG);
+        idx_out[t] = in_range ? i : 0;
+        if (in_range) map[i] = 1;
+    }
+}
+
+// Eq. 10 on protected output rows, one CTA per row t < p: one fp16 scale
+// per row, q8 [p][kp] with kp = roundup(K, 16), zero padding.
+__global__ void __launch_bounds__(256) k_q8_rows(const uint16_t *__restrict__ W, int N, int K,
+                                                 int kp, const int32_t *__restrict__ idx,
+                                                 int8_t *__restrict__ q8,
+                                                 uint16_t *__restrict__ scale, int *err) {
+    const int t = blockIdx.x;
+    const int i = idx[t];
+    int8_t *qrow = q8 + static_cast<int64_t>(t) * kp;
+    if (i < 0 || i >= N) {   // only after a latched k_set_map error
+        for (int k = threadIdx.x; k < kp; k += blockDim.x) qrow[k] = 0;
+        return;
+    }
+    const uint16_t *wrow = W + static_cast<int64_t>(i) * K;
+    double m = 0.0;
+    for (int k = threadIdx.x; k < K; k += blockDim.x) m = fmax(m, fabs(bf16_to_f64(wrow[k])));
+    __shared__ double red[256];
+    red[threadIdx.x] = m;
+    __syncthreads();
+    for (int w = 128; w > 0; w >>= 1) {
+        if (threadIdx.x < w) red[threadIdx.x] = fmax(red[threadIdx.x], red[threadIdx.x + w]);
+        __syncthreads();
+    }
+    const uint16_t s16 = f64_to_f16_rn(__ddiv_rn(red[0], 127.0));
+    if ((s16 & 0x7C00u) == 0x7C00u) {
+        if (threadIdx.x == 0) latch_error(err, BISCO_ERR_RANGE);
+        return;
+    }
+    if (threadIdx.x == 0) scale[t] = s16;
+    const double s = f16_to_f64(s16);
+    for (int k = threadIdx.x; k < kp; k += blockDim.x) {
+        double q = 0.0;
+        if (k < K && s != 0.0) {
+            q = rint(__ddiv_rn(bf16_to_f64(wrow[k]), s));
+            q = fmin(127.0, fmax(-127.0, q));
+        }
+        qrow[k] = static_cast<int8_t>(static_cast<int>(q));
     }
 }
 
@@ -244,8 +369,92 @@ bisco_status launch_encode(const uint16_t *W, const float *g, const bisco_layer 
     if (p_pad > 0)
         k_q8<<<p_pad, 256, 0, stream>>>(W, N, K, p, p_pad, L.prot_idx, L.q8, L.q8_scale, err);
     const int64_t chunks = static_cast<int64_t>(N) * (K / 8);
-    k_stages<<<static_cast<unsigned>((chunks + 255) / 256), 256, 0, stream>>>(
+    k_stages<false><<<static_cast<unsigned>((chunks + 255) / 256), 256, 0, stream>>>(
         W, N, K, S, prot, L.codes, L.norms, err);
+    k_encode_done<<<1, 32, 0, stream>>>();
+    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+}
+
+// Scratch of the selection paths over n channels: scores (8n), ranks (4n)
+// and the protected map (n), each 256-byte aligned.
+static size_t select_ws_bytes(size_t n) {
+    return round_up(8 * n, 256) + round_up(4 * n, 256) + round_up(n, 256);
+}
+
+size_t encode_workspace_bytes_axis(int N, int K, int axis) {
+    if (N < 1 || K < 8 || K % 8) return 0;
+    if (axis == 0) return encode_workspace_bytes(N, K);
+    if (axis == 1) return select_ws_bytes(static_cast<size_t>(N));
+    return 0;
+}
+
+size_t select_coupled_workspace_bytes(int F) {
+    return F < 1 ? 0 : select_ws_bytes(static_cast<size_t>(F));
+}
+
+// Output-row protection: row scores, TopK over rows, Eq. 10 on the rows, and
+// the stages of the row-masked weight.
+bisco_status launch_encode_rows(const uint16_t *W, const float *g, const bisco_layer &L,
+                                void *workspace, int *err, cudaStream_t stream) {
+    const int N = L.n_out, K = L.k_in, S = L.stages, p = L.n_protected;
+    const int kp = (K + 15) / 16 * 16;
+    const size_t n = static_cast<size_t>(N);
+    unsigned char *ws = static_cast<unsigned char *>(workspace);
+    double *score = reinterpret_cast<double *>(ws);
+    int32_t *rank = reinterpret_cast<int32_t *>(ws + round_up(8 * n, 256));
+    uint8_t *prot = ws + round_up(8 * n, 256) + round_up(4 * n, 256);
+
+    k_rowscore<<<(N + 127) / 128, 128, 0, stream>>>(W, g, N, K, score, err);
+    k_rank<<<(N + kRankThreads - 1) / kRankThreads, kRankThreads, 0, stream>>>(score, N, p, rank);
+    k_compact<<<1, kCompactThreads, 0, stream>>>(rank, N, p, prot, L.prot_idx);
+    if (p > 0) k_q8_rows<<<p, 256, 0, stream>>>(W, N, K, kp, L.prot_idx, L.q8, L.q8_scale, err);
+    const int64_t chunks = static_cast<int64_t>(N) * (K / 8);
+    k_stages<true><<<static_cast<unsigned>((chunks + 255) / 256), 256, 0, stream>>>(
+        W, N, K, S, prot, L.codes, L.norms, err);
+    k_encode_done<<<1, 32, 0, stream>>>();
+    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+}
+
+// The encoder with a caller-given protected set (columns for axis 0, rows
+// for axis 1), for example the coupled MLP set of launch_select_coupled.
+bisco_status launch_encode_with_set(const uint16_t *W, const int32_t *idx_in,
+                                    const bisco_layer &L, void *workspace, int *err,
+                                    cudaStream_t stream) {
+    const int N = L.n_out, K = L.k_in, S = L.stages, p = L.n_protected;
+    const bool rows = L.protect_axis == 1;
+    const size_t n = static_cast<size_t>(rows ? N : K);
+    uint8_t *prot = static_cast<unsigned char *>(workspace) + round_up(8 * n, 256) +
+                    round_up(4 * n, 256);
+    k_set_map<<<1, 1024, 0, stream>>>(idx_in, p, static_cast<int>(n), prot, L.prot_idx, err);
+    const int64_t chunks = static_cast<int64_t>(N) * (K / 8);
+    const unsigned sgrid = static_cast<unsigned>((chunks + 255) / 256);
+    if (rows) {
+        const int kp = (K + 15) / 16 * 16;
+        if (p > 0) k_q8_rows<<<p, 256, 0, stream>>>(W, N, K, kp, L.prot_idx, L.q8, L.q8_scale, err);
+        k_stages<true><<<sgrid, 256, 0, stream>>>(W, N, K, S, prot, L.codes, L.norms, err);
+    } else {
+        const int p_pad = (p + 15) / 16 * 16;
+        if (p_pad > 0)
+            k_q8<<<p_pad, 256, 0, stream>>>(W, N, K, p, p_pad, L.prot_idx, L.q8, L.q8_scale, err);
+        k_stages<false><<<sgrid, 256, 0, stream>>>(W, N, K, S, prot, L.codes, L.norms, err);
+    }
+    k_encode_done<<<1, 32, 0, stream>>>();
+    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+}
+
+// Eq. 9 coupled selection over the F intermediate channels of a gated MLP.
+bisco_status launch_select_coupled(const uint16_t *Wg, const uint16_t *Wu, const uint16_t *Wd,
+                                   const float *gg, const float *gu, const float *gd, int F,
+                                   int H, int p, int32_t *idx_out, void *workspace, int *err,
+                                   cudaStream_t stream) {
+    const size_t n = static_cast<size_t>(F);
+    unsigned char *ws = static_cast<unsigned char *>(workspace);
+    double *score = reinterpret_cast<double *>(ws);
+    int32_t *rank = reinterpret_cast<int32_t *>(ws + round_up(8 * n, 256));
+    uint8_t *prot = ws + round_up(8 * n, 256) + round_up(4 * n, 256);
+    k_coupled_score<<<(F + 127) / 128, 128, 0, stream>>>(Wg, Wu, Wd, gg, gu, gd, F, H, score, err);
+    k_rank<<<(F + kRankThreads - 1) / kRankThreads, kRankThreads, 0, stream>>>(score, F, p, rank);
+    k_compact<<<1, kCompactThreads, 0, stream>>>(rank, F, p, prot, idx_out);
     k_encode_done<<<1, 32, 0, stream>>>();
     return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
 }

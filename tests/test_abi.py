@@ -35,7 +35,7 @@ def test_header_declarations_are_exported(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert bisco.bisco_abi_version() == 104
+    assert bisco.bisco_abi_version() == 105
     for code in range(6):
         assert bisco.status_string(code)
     assert bisco.status_string(99) == "unknown status"
@@ -72,7 +72,8 @@ def _fake_layer(**kw):
     (dict(stages=0), bisco.ERR_INVALID_ARG),
     (dict(n_protected=-1), bisco.ERR_INVALID_ARG),
     (dict(chunk_dim=16), bisco.ERR_UNSUPPORTED),
-    (dict(protect_axis=1), bisco.ERR_UNSUPPORTED),
+    (dict(protect_axis=1, n_protected=65), bisco.ERR_INVALID_ARG),   # p > N for rows
+    (dict(n_protected=257), bisco.ERR_INVALID_ARG),                 # p > K for columns
     (dict(protect_axis=2), bisco.ERR_INVALID_ARG),
     (dict(codes=0x10004), bisco.ERR_INVALID_ARG),
     (dict(codes=0), bisco.ERR_INVALID_ARG),
@@ -186,3 +187,81 @@ def test_binding_argument_counts_match_header(lib):
         assert len(getattr(lib, name).argtypes) == n, name
         seen.add(name)
     assert seen == set(bisco.EXPORTS)
+
+
+def test_row_layout_sizes_match_oracle(lib):
+    """axis 1: the buffers the oracle's row encoder fills, byte for byte."""
+    for (N, K, S, p) in [(64, 136, 2, 3), (12288, 4096, 2, 123), (40, 64, 1, 0), (16, 64, 3, 16)]:
+        sizes = bisco.bisco_encoded_sizes_axis(N, K, S, p, 1)
+        kp = oracle.pad16(K)
+        assert sizes == [S * N * (K // 8), 2 * S * N * (K // 8), p * kp, 2 * p, 4 * p]
+        if N * K <= 1 << 14:
+            L = oracle.encode_rows(synth.layer_weights(N, K, seed=7), S, p)
+            assert sizes[:2] == [L["codes"].nbytes, L["norms"].nbytes]
+            assert sizes[2:] == [L["q8"].nbytes, L["scale"].nbytes, L["idx"].nbytes]
+    assert bisco.bisco_encoded_sizes_axis(64, 64, 2, 5, 0) == bisco.bisco_encoded_sizes(64, 64, 2, 5)
+    out = (ctypes.c_size_t * 5)()
+    f = lib.bisco_encoded_sizes_axis
+    assert f(64, 64, 8, 2, 65, 1, out) == bisco.ERR_INVALID_ARG        # p > N
+    assert f(64, 128, 8, 2, 65, 1, out) == bisco.ERR_INVALID_ARG       # p > N although <= K
+    assert f(128, 64, 8, 2, 65, 1, out) == bisco.OK                    # rows may exceed K
+    assert f(64, 64, 8, 2, 4, 2, out) == bisco.ERR_INVALID_ARG         # axis
+    assert f(64, 64, 16, 2, 4, 1, out) == bisco.ERR_UNSUPPORTED
+    assert f(64, 64, 8, 2, 4, 1, None) == bisco.ERR_INVALID_ARG
+
+
+def test_encode_workspace_by_axis(lib):
+    assert bisco.bisco_encode_workspace_bytes_axis(300, 64, 0) == bisco.bisco_encode_workspace_bytes(300, 64)
+    ws = bisco.bisco_encode_workspace_bytes_axis(300, 64, 1)
+    assert ws % 256 == 0 and ws >= 13 * 300
+    assert bisco.bisco_encode_workspace_bytes_axis(300, 64, 2) == 0
+    assert bisco.bisco_encode_workspace_bytes_axis(300, 60, 1) == 0
+    assert bisco.bisco_select_coupled_workspace_bytes(0) == 0
+    assert bisco.bisco_select_coupled_workspace_bytes(1000) >= 13 * 1000
+    # a row-protected encode wants the row workspace
+    L = _fake_layer(n_out=300, k_in=64, n_protected=3, protect_axis=1)
+    x = ctypes.c_void_p(0x60000)
+    small = bisco.bisco_encode_workspace_bytes_axis(300, 64, 0)
+    assert small < ws
+    assert lib.bisco_encode(x, None, ctypes.byref(L), ctypes.c_void_p(0x80000), small, None) \
+        == bisco.ERR_INVALID_ARG
+
+
+def test_encode_with_set_validation(lib):
+    f = lib.bisco_encode_with_set
+    E = bisco.ERR_INVALID_ARG
+    x, idx, ws = ctypes.c_void_p(0x60000), ctypes.c_void_p(0x50000), ctypes.c_void_p(0x80000)
+    big = 1 << 20
+    for axis in (0, 1):
+        L = _fake_layer(protect_axis=axis)
+        assert f(None, idx, ctypes.byref(L), ws, big, None) == E                 # weights
+        assert f(ctypes.c_void_p(0x60008), idx, ctypes.byref(L), ws, big, None) == E
+        assert f(x, None, ctypes.byref(L), ws, big, None) == E                   # p > 0, no set
+        assert f(x, ctypes.c_void_p(0x50002), ctypes.byref(L), ws, big, None) == E
+        assert f(x, idx, ctypes.byref(L), None, big, None) == E                  # workspace
+        assert f(x, idx, ctypes.byref(L), ws, 16, None) == E
+        assert f(x, idx, None, ws, big, None) == E
+    assert f(x, idx, ctypes.byref(_fake_layer(protect_axis=1, n_protected=65)), ws, big, None) == E
+    assert f(x, idx, ctypes.byref(_fake_layer(chunk_dim=16)), ws, big, None) == bisco.ERR_UNSUPPORTED
+
+
+def test_select_coupled_validation(lib):
+    f = lib.bisco_select_coupled
+    E = bisco.ERR_INVALID_ARG
+    g, u, d = ctypes.c_void_p(0x10000), ctypes.c_void_p(0x20000), ctypes.c_void_p(0x30000)
+    idx, ws = ctypes.c_void_p(0x40000), ctypes.c_void_p(0x80000)
+    big = 1 << 20
+    ok = [g, u, d, None, None, None, 96, 64, 4, idx, ws, big, None]
+
+    def call(**kw):
+        a = list(ok)
+        names = ["g", "u", "d", "gg", "gu", "gd", "F", "H", "p", "idx", "ws", "bytes", "s"]
+        for k, v in kw.items():
+            a[names.index(k)] = v
+        return f(*a)
+
+    for bad in (dict(F=0), dict(H=0), dict(p=-1), dict(p=97), dict(g=None), dict(d=None),
+                dict(u=ctypes.c_void_p(0x20008)), dict(gg=ctypes.c_void_p(0x90002)),
+                dict(gd=ctypes.c_void_p(0x90001)), dict(idx=None), dict(idx=ctypes.c_void_p(0x40002)),
+                dict(ws=None), dict(ws=ctypes.c_void_p(0x80008)), dict(bytes=64)):
+        assert call(**bad) == E, bad

@@ -22,10 +22,21 @@ MUTATIONS = {
     "zero_encoded_negative": ("if (v[k] < 0.0) bits", "if (v[k] <= 0.0) bits"),
     "decode_without_inv_sqrt8": ("double t = or_fp16_to_double(norms[e]) * inv_sqrt8;",
                                  "double t = or_fp16_to_double(norms[e]);"),
-    "decode_drops_last_stage": ("for (int32_t s = 0; s < S; ++s) {\n                int64_t e",
-                                "for (int32_t s = 0; s < S - 1; ++s) {\n                int64_t e"),
+    "decode_drops_last_stage": (
+        "for (int32_t s = 0; s < S; ++s) {\n                int64_t e = ((int64_t)s * N + i) * C + c;\n"
+        "                double t = or_fp16_to_double(norms[e]) * inv_sqrt8;",
+        "for (int32_t s = 0; s < S - 1; ++s) {\n                int64_t e = ((int64_t)s * N + i) * C + c;\n"
+        "                double t = or_fp16_to_double(norms[e]) * inv_sqrt8;"),
     "protected_scatter_missing": (
-        "o[idx[t]] = or_fp16_to_double(scale[t]) * (double)q8[(int64_t)i * pp + t];", ";"),
+        "acc = acc + (((codes[e] >> k) & 1) ? -t : t);\n            }\n            o[j] = acc;\n        }\n"
+        "        for (int32_t t = 0; t < p; ++t)\n"
+        "            o[idx[t]] = or_fp16_to_double(scale[t]) * (double)q8[(int64_t)i * pp + t];",
+        "acc = acc + (((codes[e] >> k) & 1) ? -t : t);\n            }\n            o[j] = acc;\n        }\n"),
+    "table_decode_protected_scatter_missing": (
+        "acc = acc + or_fp16_to_double(norms[e]) * t;\n            }\n            o[j] = acc;\n        }\n"
+        "        for (int32_t t = 0; t < p; ++t)\n"
+        "            o[idx[t]] = or_fp16_to_double(scale[t]) * (double)q8[(int64_t)i * pp + t];",
+        "acc = acc + or_fp16_to_double(norms[e]) * t;\n            }\n            o[j] = acc;\n        }\n"),
     "q8_truncates": ("q = nearbyint(or_bf16_to_double(W[(int64_t)i * K + j]) / s);",
                      "q = trunc(or_bf16_to_double(W[(int64_t)i * K + j]) / s);"),
     "q8_divides_by_unrounded_scale": (
