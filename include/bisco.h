@@ -284,6 +284,31 @@ bisco_status bisco_decode_dense(const bisco_layer *L, void *out, int32_t dtype,
                                 bisco_stream_t stream);
 
 /*
+ * The learned decoder step (Sec. III-A Eq. 1; the decoder ablation compares
+ * a symmetric, sign-symmetric decoder with a linear one).  A stage's chunk
+ * decodes to n16 * D_s(q); with b = 8 the code q takes 256 values, so D_s is
+ * passed as its table:
+ *   tables [S][256][8] uint16, binary16 bits, device, 16-byte aligned;
+ *   tables[s][v][k] = D_s(q(v))_k, with bit k of v set <=> q_k < 0.
+ * The identity decoder is (bit k of v ? -1 : +1) / sqrt(8) (rounded to
+ * binary16); a linear decoder A_s q and the perceptron of the ablation are
+ * evaluated by the caller into the same form.  The decoded weight is
+ *   What[i][8c + k] = sum_s n16_{s,i,c} * tables[s][code_{s,i,c}][k]
+ * (fp16 x fp16 products, exact in fp32, summed in fp32), with the protected
+ * columns (or rows, protect_axis = 1) as for bisco_gemv.
+ * bisco_gemv_table: y[b][i] = sum_j What[i][j] * x[b][j] for B in [0, 16],
+ * one warp per output row (not tuned for bandwidth), fp32 throughout.
+ * bisco_decode_dense_table: What as a dense [N][K] fp32 / bf16 / fp16
+ * matrix (BISCO_DENSE_*), rounded once from fp32.
+ * Arguments and errors are otherwise those of bisco_gemv and
+ * bisco_decode_dense.
+ */
+bisco_status bisco_gemv_table(const bisco_layer *L, const uint16_t *tables, const uint16_t *x_bf16,
+                              int32_t B, float *y, bisco_stream_t stream);
+bisco_status bisco_decode_dense_table(const bisco_layer *L, const uint16_t *tables, void *out,
+                                      int32_t dtype, bisco_stream_t stream);
+
+/*
  * Low-rank compensation (the optional LoRA path of Sec. II-D and Sec. III-F:
  * adapters trained after the codes are fixed, kept apart from the coded
  * layer's storage), added to an output the layer has already written:

@@ -21,7 +21,8 @@ EXPORTS = (
     "bisco_encode_workspace_bytes_axis", "bisco_encode", "bisco_encode_with_set",
     "bisco_select_coupled_workspace_bytes", "bisco_select_coupled",
     "bisco_encode_noalloc", "bisco_gemv", "bisco_gemv_multi",
-    "bisco_gemm_workspace_bytes", "bisco_gemm", "bisco_decode_dense", "bisco_lora_apply",
+    "bisco_gemm_workspace_bytes", "bisco_gemm", "bisco_decode_dense", "bisco_gemv_table",
+    "bisco_decode_dense_table", "bisco_lora_apply",
     "bisco_get_device_error",
 )
 
@@ -90,6 +91,10 @@ def load(path: str = LIB_PATH):
     lib.bisco_gemm.argtypes = [Lp, P, i32, P, P, sz, P]
     lib.bisco_decode_dense.restype = st
     lib.bisco_decode_dense.argtypes = [Lp, P, i32, P]
+    lib.bisco_gemv_table.restype = st
+    lib.bisco_gemv_table.argtypes = [Lp, P, P, i32, P, P]
+    lib.bisco_decode_dense_table.restype = st
+    lib.bisco_decode_dense_table.argtypes = [Lp, P, P, i32, P]
     lib.bisco_lora_apply.restype = st
     lib.bisco_lora_apply.argtypes = [P, P, i32, i32, i32, ctypes.c_float, P, i32, P, P, P]
     lib.bisco_get_device_error.restype = st
@@ -364,6 +369,48 @@ def bisco_decode_dense(L: Layer, dtype: str = "f32", out=None, stream=None):
     assert out.is_contiguous() and out.dtype == tdt and tuple(out.shape) == (L.N, L.K)
     _check(load().bisco_decode_dense(ctypes.byref(L.c), _ptr(out), code, _stream(stream)),
            "bisco_decode_dense")
+    return out
+
+
+def _tables(L: Layer, tables):
+    import torch
+    if tables.dtype == torch.float16:
+        tables = tables.view(torch.int16)
+    assert tables.is_cuda and tables.is_contiguous() and tuple(tables.shape) == (L.S, 256, 8)
+    return tables
+
+
+def bisco_gemv_table(L: Layer, tables, x_bits, y=None, stream=None):
+    """y[B][N] = x What^T with the learned decoder step given as per-stage
+    tables [S][256][8] (float16 or their int16 bits) of the decoded unit code
+    of every code byte."""
+    import torch
+    tables = _tables(L, tables)
+    if x_bits.dtype == torch.bfloat16:
+        x_bits = x_bits.view(torch.int16)
+    if x_bits.dim() == 1:
+        x_bits = x_bits.unsqueeze(0)
+    B = x_bits.shape[0]
+    assert x_bits.is_contiguous() and x_bits.shape[1] == L.K
+    if y is None:
+        y = torch.empty((B, L.N), dtype=torch.float32, device=x_bits.device)
+    _check(load().bisco_gemv_table(ctypes.byref(L.c), _ptr(tables), _ptr(x_bits), B, _ptr(y),
+                                   _stream(stream)), "bisco_gemv_table")
+    return y
+
+
+def bisco_decode_dense_table(L: Layer, tables, dtype: str = "f32", out=None, stream=None):
+    """The layer decoded with per-stage decoder tables, as a dense [N][K]
+    tensor ("f32", "bf16" or "f16")."""
+    import torch
+    tables = _tables(L, tables)
+    code = {"f32": DENSE_F32, "bf16": DENSE_BF16, "f16": DENSE_F16}[dtype]
+    tdt = {"f32": torch.float32, "bf16": torch.bfloat16, "f16": torch.float16}[dtype]
+    if out is None:
+        out = torch.empty((L.N, L.K), dtype=tdt, device=L.codes.device)
+    assert out.is_contiguous() and out.dtype == tdt and tuple(out.shape) == (L.N, L.K)
+    _check(load().bisco_decode_dense_table(ctypes.byref(L.c), _ptr(tables), _ptr(out), code,
+                                           _stream(stream)), "bisco_decode_dense_table")
     return out
 
 

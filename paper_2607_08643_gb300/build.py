@@ -14,7 +14,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libbisco.so")
 SOURCES = ["api.cu", "encode.cu", "encode_noalloc.cu", "gemv.cu", "gemm.cu", "dense.cu", "lora.cu",
-           "rows.cu"]
+           "rows.cu", "decoder.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
           "-Xptxas", "-warn-spills"]

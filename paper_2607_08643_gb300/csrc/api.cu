@@ -338,6 +338,43 @@ bisco_status bisco_decode_dense(const bisco_layer *L, void *out, int32_t dtype,
     return launch_decode_dense(*L, out, dtype, err, s);
 }
 
+bisco_status bisco_gemv_table(const bisco_layer *L, const uint16_t *tables, const uint16_t *x_bf16,
+                              int32_t B, float *y, bisco_stream_t stream) {
+    bisco_status st = check_layer(L, true);
+    if (st != BISCO_OK) return st;
+    if (B < 0 || B > 16) return BISCO_ERR_INVALID_ARG;
+    if (!tables || !aligned16(tables)) return BISCO_ERR_INVALID_ARG;
+    if (B == 0) return BISCO_OK;
+    if (!x_bf16 || !y || !aligned16(x_bf16) || !aligned16(y)) return BISCO_ERR_INVALID_ARG;
+    int *err = device_error_word(&st);
+    if (!err) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (L->protect_axis == 1) {
+        st = launch_gemv_table(bsq_only(*L), tables, x_bf16, B, y, err, s);
+        if (st != BISCO_OK) return st;
+        return launch_rows_apply(*L, x_bf16, B, y, err, s);
+    }
+    return launch_gemv_table(*L, tables, x_bf16, B, y, err, s);
+}
+
+bisco_status bisco_decode_dense_table(const bisco_layer *L, const uint16_t *tables, void *out,
+                                      int32_t dtype, bisco_stream_t stream) {
+    bisco_status st = check_layer(L, true);
+    if (st != BISCO_OK) return st;
+    if (dtype != BISCO_DENSE_F32 && dtype != BISCO_DENSE_BF16 && dtype != BISCO_DENSE_F16)
+        return BISCO_ERR_INVALID_ARG;
+    if (!tables || !aligned16(tables) || !out || !aligned16(out)) return BISCO_ERR_INVALID_ARG;
+    int *err = device_error_word(&st);
+    if (!err) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (L->protect_axis == 1) {
+        st = launch_dense_table(bsq_only(*L), tables, out, dtype, err, s);
+        if (st != BISCO_OK) return st;
+        return launch_rows_dense(*L, out, dtype, err, s);
+    }
+    return launch_dense_table(*L, tables, out, dtype, err, s);
+}
+
 bisco_status bisco_lora_apply(const uint16_t *A, const uint16_t *Bm, int32_t rank, int32_t N,
                               int32_t K, float scale, const uint16_t *x_bf16, int32_t batch,
                               float *y, float *t, bisco_stream_t stream) {

@@ -44,6 +44,11 @@ bisco_status launch_rows_apply(const bisco_layer &L, const uint16_t *X, int M, f
                                cudaStream_t stream);
 bisco_status launch_rows_dense(const bisco_layer &L, void *out, int dtype, int *err,
                                cudaStream_t stream);
+// The learned decoder step in table form (decoder.cu).
+bisco_status launch_gemv_table(const bisco_layer &L, const uint16_t *tables, const uint16_t *x,
+                               int B, float *y, int *err, cudaStream_t stream);
+bisco_status launch_dense_table(const bisco_layer &L, const uint16_t *tables, void *out, int dtype,
+                                int *err, cudaStream_t stream);
 size_t gemm_workspace_bytes(const bisco_layer &L, int M);
 bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *Y,
                          void *workspace, size_t ws_bytes, int *err, cudaStream_t stream);

@@ -1,0 +1,218 @@
+// decoder.cu -- the learned decoder step (Sec. III-A Eq. 1, decoded per
+// Sec. III-G Eq. 12) in table form.  Stage s of a chunk decodes to
+// n16 * D_s(q), and since the code q of a chunk takes only 256 values, D_s
+// is held as its table T_s[v][k] = D_s(q(v))_k in binary16 ([S][256][8],
+// 4 KB per stage): a linear decoder A q, a sign-symmetric perceptron, or
+// any other map the caller evaluated.  The identity decoder is the table
+// (bit k of v ? -1 : +1) / sqrt(8).
+//
+//   What[i][8c + k] = sum_s n16_{s,i,c} * T_s[code_{s,i,c}][k]   (column not protected)
+//   What[i][j]      = scale_t * q8[i][t]                          (j = prot_idx[t])
+//
+// Products fp16 x fp16 are exact in fp32; every sum runs in fp32.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "bisco_dev.cuh"
+#include "bisco_host.h"
+
+namespace bisco {
+namespace {
+
+constexpr int kTableEntries = 256 * 8;   // halves per stage
+
+__device__ __forceinline__ float bf16_to_f32(uint16_t b) {
+    return __uint_as_float(static_cast<uint32_t>(b) << 16);
+}
+
+// Stages S tables into shared memory (S * 4 KB, 16-byte copies).
+__device__ __forceinline__ void stage_tables(const uint16_t *__restrict__ tables, int S,
+                                             uint4 *s_tab) {
+    const uint4 *src = reinterpret_cast<const uint4 *>(tables);
+    for (int u = threadIdx.x; u < S * kTableEntries / 8; u += blockDim.x) s_tab[u] = src[u];
+    __syncthreads();
+}
+
+// The 8 decoded values of one chunk: w[k] = sum_s n_s * T_s[code_s][k].
+__device__ __forceinline__ void decode_chunk(const uint8_t *__restrict__ codes,
+                                             const uint16_t *__restrict__ norms,
+                                             const uint4 *s_tab, int S, int64_t e0,
+                                             int64_t stage_stride, float (&w)[8]) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) w[k] = 0.f;
+    for (int s = 0; s < S; ++s) {
+        const int64_t e = e0 + s * stage_stride;
+        const uint32_t v = codes[e];
+        const float n = __half2float(__ushort_as_half(norms[e]));
+        const uint4 row = s_tab[s * 256 + v];
+        const uint32_t hw[4] = {row.x, row.y, row.z, row.w};
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+            const float2 t = __half22float2(*reinterpret_cast<const __half2 *>(&hw[h]));
+            w[2 * h] = fmaf(n, t.x, w[2 * h]);
+            w[2 * h + 1] = fmaf(n, t.y, w[2 * h + 1]);
+        }
+    }
+}
+
+// Decode GEMV with a decoder table: one warp per output row, B <= 16.
+// Protected columns replace their decoded value by scale * q8 (Eq. 10).
+__global__ void __launch_bounds__(256) k_gemv_table(const uint8_t *__restrict__ codes,
+                                                    const uint16_t *__restrict__ norms,
+                                                    const uint16_t *__restrict__ tables,
+                                                    const int8_t *__restrict__ q8,
+                                                    const uint16_t *__restrict__ q8_scale,
+                                                    const int32_t *__restrict__ prot_idx, int N,
+                                                    int K, int S, int p,
+                                                    const uint16_t *__restrict__ x, int B,
+                                                    float *__restrict__ y, int *err) {
+    __shared__ uint4 s_tab[3 * kTableEntries / 8];
+    stage_tables(tables, S, s_tab);
+    const int C = K / 8, p_pad = (p + 15) / 16 * 16;
+    const int lane = threadIdx.x & 31;
+    const int i = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
+    if (i >= N) return;
+    const int64_t stride = static_cast<int64_t>(N) * C;
+    float acc[16];
+#pragma unroll
+    for (int b = 0; b < 16; ++b) acc[b] = 0.f;
+    for (int c = lane; c < C; c += 32) {
+        float w[8];
+        decode_chunk(codes, norms, s_tab, S, static_cast<int64_t>(i) * C + c, stride, w);
+#pragma unroll
+        for (int b = 0; b < 16; ++b) {
+            if (b >= B) break;
+            const uint4 xr = *reinterpret_cast<const uint4 *>(x + static_cast<int64_t>(b) * K + 8 * c);
+            const uint32_t xw[4] = {xr.x, xr.y, xr.z, xr.w};
+            float d = 0.f;
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+                d = fmaf(w[2 * h], __uint_as_float(xw[h] << 16), d);
+                d = fmaf(w[2 * h + 1], __uint_as_float(xw[h] & 0xFFFF0000u), d);
+            }
+            acc[b] += d;
+        }
+    }
+    // Eq. 10: the protected columns' decoded value is replaced by scale * q8
+    for (int t = lane; t < p; t += 32) {
+        const int j = prot_idx[t];
+        if (j < 0 || j >= K) {   // not a column of this layer
+            latch_error(err, BISCO_ERR_INVALID_ARG);
+            continue;
+        }
+        float w[8];
+        decode_chunk(codes, norms, s_tab, S, static_cast<int64_t>(i) * C + j / 8, stride, w);
+        float wb = 0.f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) wb = (k == j % 8) ? w[k] : wb;
+        const float wq = __half2float(__ushort_as_half(q8_scale[t])) *
+                         static_cast<float>(q8[static_cast<int64_t>(i) * p_pad + t]);
+#pragma unroll
+        for (int b = 0; b < 16; ++b) {
+            if (b >= B) break;
+            acc[b] += (wq - wb) * bf16_to_f32(x[static_cast<int64_t>(b) * K + j]);
+        }
+    }
+#pragma unroll
+    for (int b = 0; b < 16; ++b)
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) acc[b] += __shfl_xor_sync(0xffffffffu, acc[b], o);
+    if (lane == 0) {
+#pragma unroll
+        for (int b = 0; b < 16; ++b)
+            if (b < B) y[static_cast<int64_t>(b) * N + i] = acc[b];
+    }
+}
+
+template <typename T>
+__device__ __forceinline__ T from_f32(float v);
+template <>
+__device__ __forceinline__ float from_f32<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+template <>
+__device__ __forceinline__ __half from_f32<__half>(float v) { return __float2half_rn(v); }
+
+// Dense decode with a decoder table: one thread per chunk.
+template <typename T>
+__global__ void __launch_bounds__(256) k_dense_table(const uint8_t *__restrict__ codes,
+                                                     const uint16_t *__restrict__ norms,
+                                                     const uint16_t *__restrict__ tables, int N,
+                                                     int K, int S, T *__restrict__ out) {
+    __shared__ uint4 s_tab[3 * kTableEntries / 8];
+    stage_tables(tables, S, s_tab);
+    const int64_t chunks = static_cast<int64_t>(N) * (K / 8);
+    const int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (e >= chunks) return;
+    float w[8];
+    decode_chunk(codes, norms, s_tab, S, e, chunks, w);
+    T *o = out + e * 8;   // chunk e covers out[i][8c .. 8c+7], i*K + 8c = 8e
+#pragma unroll
+    for (int k = 0; k < 8; ++k) o[k] = from_f32<T>(w[k]);
+}
+
+// Protected columns of the dense decode: out[i][prot_idx[u]] = scale_u * q8[i][u].
+template <typename T>
+__global__ void __launch_bounds__(256) k_dense_table_protected(const int8_t *__restrict__ q8,
+                                                               const uint16_t *__restrict__ q8_scale,
+                                                               const int32_t *__restrict__ prot_idx,
+                                                               int N, int K, int p,
+                                                               T *__restrict__ out, int *err) {
+    const int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (e >= static_cast<int64_t>(N) * p) return;
+    const int i = static_cast<int>(e / p), u = static_cast<int>(e % p);
+    const int j = prot_idx[u];
+    if (j < 0 || j >= K) {
+        latch_error(err, BISCO_ERR_INVALID_ARG);   // not a column of this layer
+        return;
+    }
+    const int p_pad = (p + 15) / 16 * 16;
+    const float sc = __half2float(__ushort_as_half(q8_scale[u]));
+    out[static_cast<int64_t>(i) * K + j] =
+        from_f32<T>(sc * static_cast<float>(q8[static_cast<int64_t>(i) * p_pad + u]));
+}
+
+template <typename T>
+bisco_status launch_dense_table_t(const bisco_layer &L, const uint16_t *tables, T *out, int *err,
+                                  cudaStream_t stream) {
+    const int N = L.n_out, K = L.k_in, S = L.stages, p = L.n_protected;
+    const int64_t chunks = static_cast<int64_t>(N) * (K / 8);
+    k_dense_table<T><<<static_cast<unsigned>((chunks + 255) / 256), 256, 0, stream>>>(
+        L.codes, L.norms, tables, N, K, S, out);
+    if (cudaGetLastError() != cudaSuccess) return BISCO_ERR_CUDA;
+    if (p > 0) {
+        const int64_t n = static_cast<int64_t>(N) * p;
+        k_dense_table_protected<T><<<static_cast<unsigned>((n + 255) / 256), 256, 0, stream>>>(
+            L.q8, L.q8_scale, L.prot_idx, N, K, p, out, err);
+        if (cudaGetLastError() != cudaSuccess) return BISCO_ERR_CUDA;
+    }
+    return BISCO_OK;
+}
+
+}  // namespace
+
+bisco_status launch_gemv_table(const bisco_layer &L, const uint16_t *tables, const uint16_t *x,
+                               int B, float *y, int *err, cudaStream_t stream) {
+    const int rows_per_block = 8;
+    k_gemv_table<<<(L.n_out + rows_per_block - 1) / rows_per_block, 32 * rows_per_block, 0,
+                   stream>>>(L.codes, L.norms, tables, L.q8, L.q8_scale, L.prot_idx, L.n_out,
+                             L.k_in, L.stages, L.n_protected, x, B, y, err);
+    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+}
+
+bisco_status launch_dense_table(const bisco_layer &L, const uint16_t *tables, void *out, int dtype,
+                                int *err, cudaStream_t stream) {
+    switch (dtype) {
+        case BISCO_DENSE_F32:
+            return launch_dense_table_t(L, tables, static_cast<float *>(out), err, stream);
+        case BISCO_DENSE_BF16:
+            return launch_dense_table_t(L, tables, static_cast<__nv_bfloat16 *>(out), err, stream);
+        case BISCO_DENSE_F16:
+            return launch_dense_table_t(L, tables, static_cast<__half *>(out), err, stream);
+        default: return BISCO_ERR_INVALID_ARG;
+    }
+}
+
+}  // namespace bisco

@@ -265,3 +265,24 @@ def test_select_coupled_validation(lib):
                 dict(gd=ctypes.c_void_p(0x90001)), dict(idx=None), dict(idx=ctypes.c_void_p(0x40002)),
                 dict(ws=None), dict(ws=ctypes.c_void_p(0x80008)), dict(bytes=64)):
         assert call(**bad) == E, bad
+
+
+def test_decoder_table_validation(lib):
+    E = bisco.ERR_INVALID_ARG
+    L = _fake_layer()
+    tab, x, y = ctypes.c_void_p(0x90000), ctypes.c_void_p(0x60000), ctypes.c_void_p(0x70000)
+    g, d = lib.bisco_gemv_table, lib.bisco_decode_dense_table
+    for bad_tab in (None, ctypes.c_void_p(0x90008)):
+        assert g(ctypes.byref(L), bad_tab, x, 1, y, None) == E
+        assert d(ctypes.byref(L), bad_tab, y, bisco.DENSE_F32, None) == E
+    assert g(ctypes.byref(L), tab, x, 17, y, None) == E
+    assert g(ctypes.byref(L), tab, x, -1, y, None) == E
+    assert g(ctypes.byref(L), tab, ctypes.c_void_p(0x60002), 1, y, None) == E
+    assert g(ctypes.byref(L), tab, x, 1, None, None) == E
+    assert g(ctypes.byref(L), tab, x, 0, y, None) == bisco.OK                  # empty batch
+    assert g(None, tab, x, 1, y, None) == E
+    assert g(ctypes.byref(_fake_layer(chunk_dim=16)), tab, x, 1, y, None) == bisco.ERR_UNSUPPORTED
+    assert d(ctypes.byref(L), tab, y, 3, None) == E
+    assert d(ctypes.byref(L), tab, None, bisco.DENSE_BF16, None) == E
+    assert d(ctypes.byref(L), tab, ctypes.c_void_p(0x70004), bisco.DENSE_F16, None) == E
+    assert d(ctypes.byref(_fake_layer(stages=4)), tab, y, bisco.DENSE_F32, None) == E
