@@ -89,7 +89,29 @@ typedef struct {
     int8_t *q8;
     uint16_t *q8_scale;
     int32_t *prot_idx;
+    int32_t protect_format; /* BISCO_PROT_*: the protected payload's type */
 } bisco_layer;
+
+/*
+ * Protected payload formats (the paper's protected-format ablation compares
+ * INT8, FP8 E4M3, FP8 E5M2 and BF16 for the protected channels).  INT8 is
+ * Eq. 10 as above.  For FP8 the per-column scale is
+ * fp16(max_i |W_ij| / F), F the format's largest finite value (448 for
+ * E4M3, 57344 for E5M2), and q = fp8(W_ij / scale) rounded to nearest, ties
+ * to even, with gradual underflow; a quotient that rounds past F takes F
+ * (saturation).  The q8 buffer then holds FP8 bytes in the same [N][p_pad]
+ * layout (E4M3: bias 7, no infinities; E5M2: bias 15).  For BF16 the
+ * payload is the weight itself, scale 1.0, and the buffer is [N][p_pad]
+ * uint16 (twice the bytes).  Formats other than INT8 are supported for
+ * protected columns (protect_axis 0) only, else BISCO_ERR_UNSUPPORTED.
+ * The decode kernels run the binary spherical stages without the protected
+ * set and then replace each protected column's decoded value by
+ * scale * value(q) in a second kernel.
+ */
+#define BISCO_PROT_INT8 0
+#define BISCO_PROT_E4M3 1
+#define BISCO_PROT_E5M2 2
+#define BISCO_PROT_BF16 3
 
 /* ABI version of this header (major * 100 + minor). */
 #define BISCO_ABI_VERSION 105
@@ -108,12 +130,13 @@ bisco_status bisco_encoded_sizes(int32_t N, int32_t K, int32_t d, int32_t S,
                                  int32_t p, size_t out_bytes[5]);
 
 /*
- * bisco_encoded_sizes for either protection axis: with axis = 1 the q8
- * buffer is p * roundup(K, 16) bytes and 0 <= p <= N (INVALID_ARG else, and
- * for an axis other than 0 or 1).  Axis 0 gives bisco_encoded_sizes.
+ * Byte sizes of the five buffers of the layer *L describes (its sizes,
+ * protect_axis and protect_format; the pointers are not read): the q8
+ * buffer is N * p_pad bytes for columns (twice that for BF16) and
+ * p * roundup(K, 16) bytes for rows.  INVALID_ARG or UNSUPPORTED as for the
+ * decode calls.  Host-only.
  */
-bisco_status bisco_encoded_sizes_axis(int32_t N, int32_t K, int32_t d, int32_t S, int32_t p,
-                                      int32_t axis, size_t out_bytes[5]);
+bisco_status bisco_layer_sizes(const bisco_layer *L, size_t out_bytes[5]);
 
 /*
  * Scratch bytes bisco_encode needs for an N x K layer (per-column scores and

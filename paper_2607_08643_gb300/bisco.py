@@ -17,7 +17,7 @@ OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_RANGE, ERR_CUDA, ERR_TIMEOUT = range(6
 # Functions declared in include/bisco.h (kept in sync by tests/test_abi.py).
 EXPORTS = (
     "bisco_abi_version", "bisco_status_string", "bisco_encoded_sizes",
-    "bisco_encoded_sizes_axis", "bisco_encode_workspace_bytes",
+    "bisco_layer_sizes", "bisco_encode_workspace_bytes",
     "bisco_encode_workspace_bytes_axis", "bisco_encode", "bisco_encode_with_set",
     "bisco_select_coupled_workspace_bytes", "bisco_select_coupled",
     "bisco_encode_noalloc", "bisco_gemv", "bisco_gemv_multi",
@@ -27,6 +27,7 @@ EXPORTS = (
 )
 
 DENSE_F32, DENSE_BF16, DENSE_F16 = 0, 1, 2
+PROT_INT8, PROT_E4M3, PROT_E5M2, PROT_BF16 = 0, 1, 2, 3
 
 
 class BiscoError(RuntimeError):
@@ -42,6 +43,7 @@ class bisco_layer(ctypes.Structure):
         ("protect_axis", ctypes.c_int32),
         ("codes", ctypes.c_void_p), ("norms", ctypes.c_void_p), ("q8", ctypes.c_void_p),
         ("q8_scale", ctypes.c_void_p), ("prot_idx", ctypes.c_void_p),
+        ("protect_format", ctypes.c_int32),
     ]
 
 
@@ -65,8 +67,8 @@ def load(path: str = LIB_PATH):
     lib.bisco_status_string.argtypes = [i32]
     lib.bisco_encoded_sizes.restype = st
     lib.bisco_encoded_sizes.argtypes = [i32, i32, i32, i32, i32, ctypes.POINTER(sz)]
-    lib.bisco_encoded_sizes_axis.restype = st
-    lib.bisco_encoded_sizes_axis.argtypes = [i32, i32, i32, i32, i32, i32, ctypes.POINTER(sz)]
+    lib.bisco_layer_sizes.restype = st
+    lib.bisco_layer_sizes.argtypes = [Lp, ctypes.POINTER(sz)]
     lib.bisco_encode_workspace_bytes.restype = sz
     lib.bisco_encode_workspace_bytes.argtypes = [i32, i32]
     lib.bisco_encode_workspace_bytes_axis.restype = sz
@@ -133,9 +135,12 @@ def bisco_encoded_sizes(N, K, S, p, d=8):
     return [int(v) for v in out]
 
 
-def bisco_encoded_sizes_axis(N, K, S, p, axis, d=8):
+def bisco_layer_sizes(N, K, S, p, axis=0, fmt=PROT_INT8, d=8):
+    """Byte sizes of the five buffers of a layer with these sizes, protection
+    axis and protected payload format."""
+    c = bisco_layer(N, K, d, S, p, axis, None, None, None, None, None, fmt)
     out = (ctypes.c_size_t * 5)()
-    _check(load().bisco_encoded_sizes_axis(N, K, d, S, p, axis, out), "bisco_encoded_sizes_axis")
+    _check(load().bisco_layer_sizes(ctypes.byref(c), out), "bisco_layer_sizes")
     return [int(v) for v in out]
 
 
@@ -160,13 +165,14 @@ def bisco_gemm_workspace_bytes(L, M) -> int:
 class Layer:
     """A coded layer in device memory (torch tensors) plus its C struct.
     axis 0 protects input columns (q8 [N][p_pad]); axis 1 protects output
-    rows (q8 [p][roundup(K, 16)])."""
+    rows (q8 [p][roundup(K, 16)]).  fmt is the protected payload's format
+    (PROT_*; BF16 payloads are [N][p_pad] uint16)."""
 
-    def __init__(self, N, K, S, p, device="cuda", d=8, axis=0):
+    def __init__(self, N, K, S, p, device="cuda", d=8, axis=0, fmt=PROT_INT8):
         import torch
-        sizes = bisco_encoded_sizes(N, K, S, p, d) if axis == 0 else \
-            bisco_encoded_sizes_axis(N, K, S, p, axis, d)
-        self.N, self.K, self.S, self.p, self.axis = N, K, S, p, axis
+        sizes = bisco_encoded_sizes(N, K, S, p, d) if (axis, fmt) == (0, PROT_INT8) else \
+            bisco_layer_sizes(N, K, S, p, axis, fmt, d)
+        self.N, self.K, self.S, self.p, self.axis, self.fmt = N, K, S, p, axis, fmt
         self.p_pad = (p + 15) // 16 * 16
         self.kp = (K + 15) // 16 * 16
         dev = torch.device(device)
@@ -175,18 +181,20 @@ class Layer:
         if axis == 1:
             self.q8 = torch.empty((max(p, 1), self.kp), dtype=torch.int8, device=dev)
         else:
-            self.q8 = torch.empty((N, max(self.p_pad, 16)), dtype=torch.int8, device=dev)
+            qdt = {PROT_INT8: torch.int8, PROT_E4M3: torch.uint8, PROT_E5M2: torch.uint8,
+                   PROT_BF16: torch.int16}[fmt]
+            self.q8 = torch.empty((N, max(self.p_pad, 16)), dtype=qdt, device=dev)
         self.scale = torch.empty((max(p, 8),), dtype=torch.int16, device=dev)
         self.idx = torch.empty((max(p, 4),), dtype=torch.int32, device=dev)
         assert sizes[0] == self.codes.numel() and sizes[1] == 2 * self.norms.numel()
-        assert sizes[2] <= self.q8.numel()
+        assert sizes[2] <= self.q8.numel() * self.q8.element_size()
         self.c = bisco_layer(N, K, d, S, p, axis, self.codes.data_ptr(), self.norms.data_ptr(),
-                             self.q8.data_ptr(), self.scale.data_ptr(), self.idx.data_ptr())
+                             self.q8.data_ptr(), self.scale.data_ptr(), self.idx.data_ptr(), fmt)
 
     @property
     def compressed_bytes(self) -> int:
         """Algorithmic payload: signs + norms + unpadded q8 + scales + indices."""
-        q8 = self.p * (self.K if self.axis == 1 else self.N)
+        q8 = self.p * (self.K if self.axis == 1 else self.N) * (2 if self.fmt == PROT_BF16 else 1)
         return self.S * self.N * (self.K // 8) * 3 + q8 + 6 * self.p
 
     def to_numpy(self):
@@ -202,6 +210,10 @@ class Layer:
             L["q8"] = self.q8[:p].cpu().numpy()
         else:
             L["q8"] = self.q8[:, :self.p_pad].cpu().numpy()
+            if self.fmt == PROT_BF16:
+                L["q8"] = L["q8"].view("uint16")
+        if self.fmt != PROT_INT8:
+            L["fmt"] = self.fmt
         return L
 
     @classmethod
@@ -209,11 +221,13 @@ class Layer:
         import numpy as np
         import torch
         axis = L.get("axis", 0)
-        obj = cls(L["N"], L["K"], L["S"], L["p"], device, axis=axis)
+        fmt = L.get("fmt", PROT_INT8)
+        obj = cls(L["N"], L["K"], L["S"], L["p"], device, axis=axis, fmt=fmt)
         obj.codes.copy_(torch.from_numpy(np.ascontiguousarray(L["codes"])))
         obj.norms.copy_(torch.from_numpy(np.ascontiguousarray(L["norms"]).view(np.int16)))
         if L["p"]:
-            q8 = torch.from_numpy(np.ascontiguousarray(L["q8"]))
+            q8 = np.ascontiguousarray(L["q8"])
+            q8 = torch.from_numpy(q8.view(np.int16) if q8.dtype == np.uint16 else q8)
             if axis == 1:
                 obj.q8[:L["p"]].copy_(q8)
             else:
@@ -231,13 +245,15 @@ def _bits2d(W_bits):
     return W_bits
 
 
-def bisco_encode(W_bits, S, p, g=None, workspace=None, stream=None, axis=0) -> Layer:
+def bisco_encode(W_bits, S, p, g=None, workspace=None, stream=None, axis=0,
+                 fmt=PROT_INT8) -> Layer:
     """Encodes a device tensor of bf16 bits [N][K] (int16 or bfloat16);
-    axis 1 protects the p output rows of largest norm instead of columns."""
+    axis 1 protects the p output rows of largest norm instead of columns;
+    fmt selects the protected payload's format."""
     import torch
     W_bits = _bits2d(W_bits)
     N, K = W_bits.shape
-    L = Layer(N, K, S, p, W_bits.device, axis=axis)
+    L = Layer(N, K, S, p, W_bits.device, axis=axis, fmt=fmt)
     need = bisco_encode_workspace_bytes_axis(N, K, axis)
     if workspace is None:
         workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=W_bits.device)

@@ -14,11 +14,12 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libbisco.so")
 SOURCES = ["api.cu", "encode.cu", "encode_noalloc.cu", "gemv.cu", "gemm.cu", "dense.cu", "lora.cu",
-           "rows.cu", "decoder.cu"]
+           "rows.cu", "decoder.cu", "formats.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
           "-Xptxas", "-warn-spills"]
-PER_FILE = {"encode.cu": ["--fmad=false"], "encode_noalloc.cu": ["--fmad=false"]}
+PER_FILE = {"encode.cu": ["--fmad=false"], "encode_noalloc.cu": ["--fmad=false"],
+            "formats.cu": ["--fmad=false"]}
 
 
 def nvcc() -> str:

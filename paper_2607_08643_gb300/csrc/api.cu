@@ -39,7 +39,10 @@ bisco_status check_layer(const bisco_layer *L, bool check_buffers) {
     if (L->protect_axis != 0 && L->protect_axis != 1) return BISCO_ERR_INVALID_ARG;
     const int32_t p_max = L->protect_axis == 1 ? L->n_out : L->k_in;
     if (L->n_protected < 0 || L->n_protected > p_max) return BISCO_ERR_INVALID_ARG;
+    if (L->protect_format < BISCO_PROT_INT8 || L->protect_format > BISCO_PROT_BF16)
+        return BISCO_ERR_INVALID_ARG;
     if (L->chunk_dim != 8) return BISCO_ERR_UNSUPPORTED;
+    if (L->protect_format != BISCO_PROT_INT8 && L->protect_axis != 0) return BISCO_ERR_UNSUPPORTED;
     if (static_cast<int64_t>(L->n_out) * L->k_in > (int64_t(1) << 40)) return BISCO_ERR_INVALID_ARG;
     if (!check_buffers) return BISCO_OK;
     if (!L->codes || !L->norms || !aligned16(L->codes) || !aligned16(L->norms))
@@ -52,15 +55,33 @@ bisco_status check_layer(const bisco_layer *L, bool check_buffers) {
     return BISCO_OK;
 }
 
-// The binary spherical stages of a row-protected layer alone: the decode
-// kernels run on this copy (no protected columns; they read none of the
-// protected buffers when p == 0) and rows.cu then overwrites the protected
-// rows.
+// Layers whose protected set the decode kernels do not take themselves:
+// output rows (rows.cu) and payloads other than INT8 (formats.cu).
+bool needs_epilogue(const bisco_layer &L) {
+    return L.n_protected > 0 &&
+           (L.protect_axis == 1 || L.protect_format != BISCO_PROT_INT8);
+}
+
+// The binary spherical stages of such a layer alone: the decode kernels run
+// on this copy (no protected set; they read none of the protected buffers
+// when p == 0), then epilogue() applies the protected set.
 bisco_layer bsq_only(const bisco_layer &L) {
     bisco_layer b = L;
     b.n_protected = 0;
     b.protect_axis = 0;
+    b.protect_format = BISCO_PROT_INT8;
     return b;
+}
+
+bisco_status epilogue(const bisco_layer &L, const uint16_t *X, int M, float *Y, int *err,
+                      cudaStream_t s) {
+    if (L.protect_axis == 1) return launch_rows_apply(L, X, M, Y, err, s);
+    return launch_prot_fix(L, X, M, Y, err, s);
+}
+
+bisco_status dense_epilogue(const bisco_layer &L, void *out, int dtype, int *err, cudaStream_t s) {
+    if (L.protect_axis == 1) return launch_rows_dense(L, out, dtype, err, s);
+    return launch_dense_fmt(L, out, dtype, err, s);
 }
 
 }  // namespace
@@ -163,20 +184,21 @@ bisco_status bisco_encoded_sizes(int32_t N, int32_t K, int32_t d, int32_t S, int
     return BISCO_OK;
 }
 
-bisco_status bisco_encoded_sizes_axis(int32_t N, int32_t K, int32_t d, int32_t S, int32_t p,
-                                      int32_t axis, size_t out_bytes[5]) {
-    if (axis == 0) return bisco_encoded_sizes(N, K, d, S, p, out_bytes);
-    if (axis != 1 || !out_bytes) return BISCO_ERR_INVALID_ARG;
-    if (N < 1 || K < 8 || K % 8 != 0 || S < 1 || S > 3 || p < 0 || p > N)
-        return BISCO_ERR_INVALID_ARG;
-    if (d != 8) return BISCO_ERR_UNSUPPORTED;
-    const size_t C = static_cast<size_t>(K) / 8;
-    const size_t kp = (static_cast<size_t>(K) + 15) / 16 * 16;
-    out_bytes[0] = static_cast<size_t>(S) * N * C;
-    out_bytes[1] = static_cast<size_t>(S) * N * C * 2;
-    out_bytes[2] = static_cast<size_t>(p) * kp;
-    out_bytes[3] = static_cast<size_t>(p) * 2;
-    out_bytes[4] = static_cast<size_t>(p) * 4;
+bisco_status bisco_layer_sizes(const bisco_layer *L, size_t out_bytes[5]) {
+    if (!out_bytes) return BISCO_ERR_INVALID_ARG;
+    const bisco_status st = check_layer(L, false);
+    if (st != BISCO_OK) return st;
+    const size_t N = static_cast<size_t>(L->n_out), K = static_cast<size_t>(L->k_in);
+    const size_t S = static_cast<size_t>(L->stages), p = static_cast<size_t>(L->n_protected);
+    const size_t C = K / 8;
+    out_bytes[0] = S * N * C;
+    out_bytes[1] = S * N * C * 2;
+    if (L->protect_axis == 1)
+        out_bytes[2] = p * ((K + 15) / 16 * 16);
+    else
+        out_bytes[2] = N * ((p + 15) / 16 * 16) * (L->protect_format == BISCO_PROT_BF16 ? 2 : 1);
+    out_bytes[3] = p * 2;
+    out_bytes[4] = p * 4;
     return BISCO_OK;
 }
 
@@ -257,10 +279,10 @@ bisco_status bisco_gemv(const bisco_layer *L, const uint16_t *x_bf16, int32_t B,
     int *err = device_error_word(&st);
     if (!err) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    if (L->protect_axis == 1) {
+    if (needs_epilogue(*L)) {
         st = launch_gemv(bsq_only(*L), x_bf16, B, y, err, s);
         if (st != BISCO_OK) return st;
-        return launch_rows_apply(*L, x_bf16, B, y, err, s);
+        return epilogue(*L, x_bf16, B, y, err, s);
     }
     return launch_gemv(*L, x_bf16, B, y, err, s);
 }
@@ -284,21 +306,22 @@ bisco_status bisco_gemv_multi(const bisco_layer *layers, int32_t G, const uint16
     if (!err) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     bisco_layer stages[BISCO_GEMV_MULTI_MAX];
-    bool rows = false;
+    bool any = false;
     for (int g = 0; g < G; ++g) {
-        rows |= layers[g].protect_axis == 1;
-        stages[g] = layers[g].protect_axis == 1 ? bsq_only(layers[g]) : layers[g];
+        const bool e = needs_epilogue(layers[g]);
+        any |= e;
+        stages[g] = e ? bsq_only(layers[g]) : layers[g];
     }
-    if (!rows) return launch_gemv_multi(layers, G, x_bf16, B, y, err, s);
+    if (!any) return launch_gemv_multi(layers, G, x_bf16, B, y, err, s);
     st = launch_gemv_multi(stages, G, x_bf16, B, y, err, s);
     for (int g = 0; g < G && st == BISCO_OK; ++g)
-        if (layers[g].protect_axis == 1) st = launch_rows_apply(layers[g], x_bf16, B, y[g], err, s);
+        if (needs_epilogue(layers[g])) st = epilogue(layers[g], x_bf16, B, y[g], err, s);
     return st;
 }
 
 size_t bisco_gemm_workspace_bytes(const bisco_layer *L, int32_t M) {
     if (M < 0 || check_layer(L, false) != BISCO_OK) return 0;
-    return gemm_workspace_bytes(L->protect_axis == 1 ? bsq_only(*L) : *L, M);
+    return gemm_workspace_bytes(needs_epilogue(*L) ? bsq_only(*L) : *L, M);
 }
 
 bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M, float *Y,
@@ -308,7 +331,7 @@ bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M,
     if (M < 0) return BISCO_ERR_INVALID_ARG;
     if (M == 0) return BISCO_OK;
     if (!X_bf16 || !Y || !aligned16(X_bf16) || !aligned16(Y)) return BISCO_ERR_INVALID_ARG;
-    const bisco_layer Ls = L->protect_axis == 1 ? bsq_only(*L) : *L;
+    const bisco_layer Ls = needs_epilogue(*L) ? bsq_only(*L) : *L;
     const size_t need = gemm_workspace_bytes(Ls, M);
     if (need && (!workspace || !aligned16(workspace) || workspace_bytes < need))
         return BISCO_ERR_INVALID_ARG;
@@ -316,8 +339,8 @@ bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M,
     if (!err) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     st = launch_gemm(Ls, X_bf16, M, Y, workspace, workspace_bytes, err, s);
-    if (st != BISCO_OK || L->protect_axis != 1) return st;
-    return launch_rows_apply(*L, X_bf16, M, Y, err, s);
+    if (st != BISCO_OK || !needs_epilogue(*L)) return st;
+    return epilogue(*L, X_bf16, M, Y, err, s);
 }
 
 bisco_status bisco_decode_dense(const bisco_layer *L, void *out, int32_t dtype,
@@ -330,10 +353,10 @@ bisco_status bisco_decode_dense(const bisco_layer *L, void *out, int32_t dtype,
     int *err = device_error_word(&st);
     if (!err) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    if (L->protect_axis == 1) {
+    if (needs_epilogue(*L)) {
         st = launch_decode_dense(bsq_only(*L), out, dtype, err, s);
         if (st != BISCO_OK) return st;
-        return launch_rows_dense(*L, out, dtype, err, s);
+        return dense_epilogue(*L, out, dtype, err, s);
     }
     return launch_decode_dense(*L, out, dtype, err, s);
 }
@@ -342,6 +365,7 @@ bisco_status bisco_gemv_table(const bisco_layer *L, const uint16_t *tables, cons
                               int32_t B, float *y, bisco_stream_t stream) {
     bisco_status st = check_layer(L, true);
     if (st != BISCO_OK) return st;
+    if (L->protect_format != BISCO_PROT_INT8) return BISCO_ERR_UNSUPPORTED;
     if (B < 0 || B > 16) return BISCO_ERR_INVALID_ARG;
     if (!tables || !aligned16(tables)) return BISCO_ERR_INVALID_ARG;
     if (B == 0) return BISCO_OK;
@@ -361,6 +385,7 @@ bisco_status bisco_decode_dense_table(const bisco_layer *L, const uint16_t *tabl
                                       int32_t dtype, bisco_stream_t stream) {
     bisco_status st = check_layer(L, true);
     if (st != BISCO_OK) return st;
+    if (L->protect_format != BISCO_PROT_INT8) return BISCO_ERR_UNSUPPORTED;
     if (dtype != BISCO_DENSE_F32 && dtype != BISCO_DENSE_BF16 && dtype != BISCO_DENSE_F16)
         return BISCO_ERR_INVALID_ARG;
     if (!tables || !aligned16(tables) || !out || !aligned16(out)) return BISCO_ERR_INVALID_ARG;

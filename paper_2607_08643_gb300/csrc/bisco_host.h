@@ -44,6 +44,14 @@ bisco_status launch_rows_apply(const bisco_layer &L, const uint16_t *X, int M, f
                                cudaStream_t stream);
 bisco_status launch_rows_dense(const bisco_layer &L, void *out, int dtype, int *err,
                                cudaStream_t stream);
+// Protected payloads other than INT8 (formats.cu): the encoder's
+// quantiser, the correction after the stage-only decode kernels, and the
+// dense overwrite.
+bisco_status launch_q_fmt(const uint16_t *W, const bisco_layer &L, int *err, cudaStream_t stream);
+bisco_status launch_prot_fix(const bisco_layer &L, const uint16_t *X, int M, float *Y, int *err,
+                             cudaStream_t stream);
+bisco_status launch_dense_fmt(const bisco_layer &L, void *out, int dtype, int *err,
+                              cudaStream_t stream);
 // The learned decoder step in table form (decoder.cu).
 bisco_status launch_gemv_table(const bisco_layer &L, const uint16_t *tables, const uint16_t *x,
                                int B, float *y, int *err, cudaStream_t stream);

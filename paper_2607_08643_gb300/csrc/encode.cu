@@ -366,8 +366,11 @@ bisco_status launch_encode(const uint16_t *W, const float *g, const bisco_layer 
     k_colscore<<<(K + 127) / 128, 128, 0, stream>>>(W, g, N, K, score, err);
     k_rank<<<(K + kRankThreads - 1) / kRankThreads, kRankThreads, 0, stream>>>(score, K, p, rank);
     k_compact<<<1, kCompactThreads, 0, stream>>>(rank, K, p, prot, L.prot_idx);
-    if (p_pad > 0)
+    if (L.protect_format != BISCO_PROT_INT8) {
+        if (launch_q_fmt(W, L, err, stream) != BISCO_OK) return BISCO_ERR_CUDA;
+    } else if (p_pad > 0) {
         k_q8<<<p_pad, 256, 0, stream>>>(W, N, K, p, p_pad, L.prot_idx, L.q8, L.q8_scale, err);
+    }
     const int64_t chunks = static_cast<int64_t>(N) * (K / 8);
     k_stages<false><<<static_cast<unsigned>((chunks + 255) / 256), 256, 0, stream>>>(
         W, N, K, S, prot, L.codes, L.norms, err);
@@ -434,8 +437,11 @@ bisco_status launch_encode_with_set(const uint16_t *W, const int32_t *idx_in,
         k_stages<true><<<sgrid, 256, 0, stream>>>(W, N, K, S, prot, L.codes, L.norms, err);
     } else {
         const int p_pad = (p + 15) / 16 * 16;
-        if (p_pad > 0)
+        if (L.protect_format != BISCO_PROT_INT8) {
+            if (launch_q_fmt(W, L, err, stream) != BISCO_OK) return BISCO_ERR_CUDA;
+        } else if (p_pad > 0) {
             k_q8<<<p_pad, 256, 0, stream>>>(W, N, K, p, p_pad, L.prot_idx, L.q8, L.q8_scale, err);
+        }
         k_stages<false><<<sgrid, 256, 0, stream>>>(W, N, K, S, prot, L.codes, L.norms, err);
     }
     k_encode_done<<<1, 32, 0, stream>>>();

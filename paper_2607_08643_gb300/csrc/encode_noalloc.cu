@@ -64,7 +64,8 @@ extern "C" bisco_status bisco_encode_noalloc(const uint16_t *W_bf16, const float
         L->n_protected < 0 || L->n_protected > L->k_in ||
         (L->protect_axis != 0 && L->protect_axis != 1))
         return BISCO_ERR_INVALID_ARG;
-    if (L->chunk_dim != 8 || L->protect_axis != 0) return BISCO_ERR_UNSUPPORTED;
+    if (L->chunk_dim != 8 || L->protect_axis != 0 || L->protect_format != BISCO_PROT_INT8)
+        return BISCO_ERR_UNSUPPORTED;
     if (L->k_in > BISCO_ENCODE_NOALLOC_MAX_K) return BISCO_ERR_UNSUPPORTED;   // beyond the array
     if (static_cast<int64_t>(L->n_out) * L->k_in > (int64_t(1) << 40)) return BISCO_ERR_INVALID_ARG;
     if (!L->codes || !L->norms || !aligned16(L->codes) || !aligned16(L->norms))

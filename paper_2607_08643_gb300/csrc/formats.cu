@@ -1,0 +1,279 @@
+// formats.cu -- protected payloads other than INT8 (the paper's
+// protected-format ablation: FP8 E4M3, FP8 E5M2, BF16 for the protected
+// channels of Sec. III-E Eq. 10).
+//
+// Encode: per protected column j, scale = fp16(max_i |W_ij| / F) with F the
+// format's largest finite value, and q_ij = fp8(W_ij / scale) (binary64
+// quotient rounded once to FP8, nearest even, gradual underflow, saturating
+// at F); BF16 keeps the weight itself with scale 1.0.
+//
+// Decode: the binary spherical kernels run without the protected set, so a
+// protected column carries its decoded stage value w_b; this file then adds
+//   y[m][i] += sum_t (scale_t * value(q[i][t]) - w_b(i, j_t)) * x[m][j_t]
+// which leaves scale * value(q) in place of the stage value (Eq. 10's
+// overwrite).  All of it in fp32 except the encoder (binary64).
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "bisco_dev.cuh"
+#include "bisco_host.h"
+
+namespace bisco {
+namespace {
+
+struct Fp8Format {
+    int mbits, bias;
+    double maxf;
+    uint8_t maxcode;
+};
+
+__device__ __forceinline__ Fp8Format fp8_format(int fmt) {
+    if (fmt == BISCO_PROT_E4M3) return {3, 7, 448.0, 0x7E};
+    return {2, 15, 57344.0, 0x7B};   // BISCO_PROT_E5M2
+}
+
+__device__ __forceinline__ uint16_t f64_to_f16_rn(double x) {
+    unsigned short r;
+    asm("cvt.rn.f16.f64 %0, %1;" : "=h"(r) : "d"(x));
+    return r;
+}
+
+__device__ __forceinline__ double f16_to_f64(uint16_t h) {
+    return static_cast<double>(__half2float(__ushort_as_half(h)));
+}
+
+__device__ __forceinline__ double bf16_to_f64(uint16_t b) {
+    return static_cast<double>(__uint_as_float(static_cast<uint32_t>(b) << 16));
+}
+
+// binary64 -> FP8 bits, nearest even: the significand scaled so that the
+// kept bits are its integer part (exact, a power of two), rounded once by
+// rint; subnormals share the least normal exponent; above F saturates.
+__device__ __forceinline__ uint8_t f64_to_fp8(double x, const Fp8Format &f) {
+    const uint8_t sign = signbit(x) ? 0x80 : 0x00;
+    const double a = fabs(x);
+    if (a == 0.0) return sign;
+    int E = ilogb(a);
+    if (E < 1 - f.bias) E = 1 - f.bias;
+    double m = rint(ldexp(a, f.mbits - E));
+    if (m == ldexp(1.0, f.mbits + 1)) {   // rounded up to the next binade
+        m = ldexp(1.0, f.mbits);
+        E += 1;
+    }
+    if (ldexp(m, E - f.mbits) > f.maxf) return sign | f.maxcode;
+    const int mi = static_cast<int>(m);
+    if (mi >= (1 << f.mbits))
+        return sign | static_cast<uint8_t>(((E + f.bias) << f.mbits) | (mi - (1 << f.mbits)));
+    return sign | static_cast<uint8_t>(mi);
+}
+
+// The value of a protected payload element (exact in fp32).
+__device__ __forceinline__ float payload_value(const void *q, int64_t e, int fmt) {
+    if (fmt == BISCO_PROT_BF16)
+        return __uint_as_float(static_cast<uint32_t>(static_cast<const uint16_t *>(q)[e]) << 16);
+    const uint32_t v = static_cast<const uint8_t *>(q)[e];
+    if (fmt == BISCO_PROT_E5M2)   // E5M2 is the upper byte of a binary16
+        return __half2float(__ushort_as_half(static_cast<uint16_t>(v << 8)));
+    const uint32_t ex = (v >> 3) & 0xFu, mn = v & 7u;   // E4M3
+    float r;
+    if (ex == 15u && mn == 7u)
+        r = __uint_as_float(0x7FC00000u);
+    else if (ex == 0u)
+        r = ldexpf(static_cast<float>(mn), -9);
+    else
+        r = ldexpf(static_cast<float>(8u + mn), static_cast<int>(ex) - 10);
+    return (v & 0x80u) ? -r : r;
+}
+
+// Encoder: one CTA per payload column t < p_pad (t >= p: zero padding).
+__global__ void __launch_bounds__(256) k_q_fmt(const uint16_t *__restrict__ W, int N, int K, int p,
+                                               int p_pad, const int32_t *__restrict__ idx, int fmt,
+                                               void *__restrict__ q, uint16_t *__restrict__ scale,
+                                               int *err) {
+    const int t = blockIdx.x;
+    uint8_t *q8 = static_cast<uint8_t *>(q);
+    uint16_t *q16 = static_cast<uint16_t *>(q);
+    if (t >= p) {
+        for (int i = threadIdx.x; i < N; i += blockDim.x) {
+            const int64_t e = static_cast<int64_t>(i) * p_pad + t;
+            if (fmt == BISCO_PROT_BF16) q16[e] = 0; else q8[e] = 0;
+        }
+        return;
+    }
+    const int j = idx[t];
+    if (fmt == BISCO_PROT_BF16) {
+        if (threadIdx.x == 0) scale[t] = 0x3C00u;   // 1.0
+        for (int i = threadIdx.x; i < N; i += blockDim.x)
+            q16[static_cast<int64_t>(i) * p_pad + t] = W[static_cast<int64_t>(i) * K + j];
+        return;
+    }
+    const Fp8Format f = fp8_format(fmt);
+    double m = 0.0;
+    for (int i = threadIdx.x; i < N; i += blockDim.x)
+        m = fmax(m, fabs(bf16_to_f64(W[static_cast<int64_t>(i) * K + j])));
+    __shared__ double red[256];
+    red[threadIdx.x] = m;
+    __syncthreads();
+    for (int w = 128; w > 0; w >>= 1) {
+        if (threadIdx.x < w) red[threadIdx.x] = fmax(red[threadIdx.x], red[threadIdx.x + w]);
+        __syncthreads();
+    }
+    const uint16_t s16 = f64_to_f16_rn(__ddiv_rn(red[0], f.maxf));
+    if ((s16 & 0x7C00u) == 0x7C00u) {
+        if (threadIdx.x == 0) latch_error(err, BISCO_ERR_RANGE);
+        return;
+    }
+    if (threadIdx.x == 0) scale[t] = s16;
+    const double s = f16_to_f64(s16);
+    for (int i = threadIdx.x; i < N; i += blockDim.x) {
+        const double w = bf16_to_f64(W[static_cast<int64_t>(i) * K + j]);
+        q8[static_cast<int64_t>(i) * p_pad + t] = s != 0.0 ? f64_to_fp8(__ddiv_rn(w, s), f) : 0;
+    }
+}
+
+constexpr int kFixRows = 32, kFixTok = 32, kFixT = 32;
+
+// The correction of the decode kernels' output, for a tile of 32 output
+// rows x 32 activation rows, the protected columns taken 32 at a time
+// through shared memory.  Thread (r = tid / 8, c = tid % 8) owns rows r and
+// activation rows 4c..4c+3 of the tile; every (m, i) belongs to one thread.
+__global__ void __launch_bounds__(256) k_prot_fix(const uint8_t *__restrict__ codes,
+                                                  const uint16_t *__restrict__ norms,
+                                                  const void *__restrict__ q,
+                                                  const uint16_t *__restrict__ scale,
+                                                  const int32_t *__restrict__ idx, int fmt, int N,
+                                                  int K, int S, int p,
+                                                  const uint16_t *__restrict__ X, int M,
+                                                  float *__restrict__ Y, int *err) {
+    __shared__ float s_d[kFixRows][kFixT + 1];
+    __shared__ float s_x[kFixTok][kFixT + 1];
+    const int tid = threadIdx.x;
+    const int r = tid >> 3, c = tid & 7;
+    const int i0 = blockIdx.x * kFixRows, m0 = blockIdx.y * kFixTok;
+    const int C = K / 8, p_pad = (p + 15) / 16 * 16;
+    const float inv_sqrt8 = 0.35355339059327373f;   // the decode kernels' 1/sqrt(8) in fp32
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int t0 = 0; t0 < p; t0 += kFixT) {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int tt = 4 * c + u, t = t0 + tt;
+            // d = scale * value(q) - (stage value of that weight), row i0 + r
+            float d = 0.f;
+            const int i = i0 + r;
+            if (t < p && i < N) {
+                const int j = idx[t];
+                if (j >= 0 && j < K) {
+                    float wb = 0.f;
+                    for (int s = 0; s < S; ++s) {
+                        const int64_t e = (static_cast<int64_t>(s) * N + i) * C + j / 8;
+                        const float n = __half2float(__ushort_as_half(norms[e]));
+                        wb += ((codes[e] >> (j % 8)) & 1u) ? -n : n;
+                    }
+                    const float sc = __half2float(__ushort_as_half(scale[t]));
+                    d = sc * payload_value(q, static_cast<int64_t>(i) * p_pad + t, fmt) -
+                        wb * inv_sqrt8;
+                } else if (r == 0) {
+                    latch_error(err, BISCO_ERR_INVALID_ARG);   // not a column of this layer
+                }
+            }
+            s_d[r][tt] = d;
+            // activation (m0 + r, column j_t)
+            float xv = 0.f;
+            const int m = m0 + r;
+            if (t < p && m < M) {
+                const int j = idx[t];
+                if (j >= 0 && j < K)
+                    xv = __uint_as_float(static_cast<uint32_t>(X[static_cast<int64_t>(m) * K + j]) << 16);
+            }
+            s_x[r][tt] = xv;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int tt = 0; tt < kFixT; ++tt) {
+            const float d = s_d[r][tt];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) acc[u] = fmaf(d, s_x[4 * c + u][tt], acc[u]);
+        }
+        __syncthreads();
+    }
+    const int i = i0 + r;
+    if (i >= N) return;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const int m = m0 + 4 * c + u;
+        if (m < M) Y[static_cast<int64_t>(m) * N + i] += acc[u];
+    }
+}
+
+template <typename T>
+__device__ __forceinline__ T from_f32(float v);
+template <>
+__device__ __forceinline__ float from_f32<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+template <>
+__device__ __forceinline__ __half from_f32<__half>(float v) { return __float2half_rn(v); }
+
+// Dense decode: out[i][idx[u]] = scale_u * value(q[i][u]), one thread per (i, u).
+template <typename T>
+__global__ void __launch_bounds__(256) k_dense_fmt(const void *__restrict__ q,
+                                                   const uint16_t *__restrict__ scale,
+                                                   const int32_t *__restrict__ idx, int fmt, int N,
+                                                   int K, int p, T *__restrict__ out, int *err) {
+    const int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (e >= static_cast<int64_t>(N) * p) return;
+    const int i = static_cast<int>(e / p), u = static_cast<int>(e % p);
+    const int j = idx[u];
+    if (j < 0 || j >= K) {
+        latch_error(err, BISCO_ERR_INVALID_ARG);   // not a column of this layer
+        return;
+    }
+    const int p_pad = (p + 15) / 16 * 16;
+    const float sc = __half2float(__ushort_as_half(scale[u]));
+    out[static_cast<int64_t>(i) * K + j] =
+        from_f32<T>(sc * payload_value(q, static_cast<int64_t>(i) * p_pad + u, fmt));
+}
+
+template <typename T>
+bisco_status launch_dense_fmt_t(const bisco_layer &L, T *out, int *err, cudaStream_t stream) {
+    const int64_t n = static_cast<int64_t>(L.n_out) * L.n_protected;
+    k_dense_fmt<T><<<static_cast<unsigned>((n + 255) / 256), 256, 0, stream>>>(
+        L.q8, L.q8_scale, L.prot_idx, L.protect_format, L.n_out, L.k_in, L.n_protected, out, err);
+    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+}
+
+}  // namespace
+
+bisco_status launch_q_fmt(const uint16_t *W, const bisco_layer &L, int *err, cudaStream_t stream) {
+    const int p = L.n_protected, p_pad = (p + 15) / 16 * 16;
+    if (p_pad == 0) return BISCO_OK;
+    k_q_fmt<<<p_pad, 256, 0, stream>>>(W, L.n_out, L.k_in, p, p_pad, L.prot_idx, L.protect_format,
+                                       L.q8, L.q8_scale, err);
+    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+}
+
+bisco_status launch_prot_fix(const bisco_layer &L, const uint16_t *X, int M, float *Y, int *err,
+                             cudaStream_t stream) {
+    if (L.n_protected <= 0 || M <= 0) return BISCO_OK;
+    const dim3 grid((L.n_out + kFixRows - 1) / kFixRows, (M + kFixTok - 1) / kFixTok);
+    k_prot_fix<<<grid, 256, 0, stream>>>(L.codes, L.norms, L.q8, L.q8_scale, L.prot_idx,
+                                         L.protect_format, L.n_out, L.k_in, L.stages,
+                                         L.n_protected, X, M, Y, err);
+    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+}
+
+bisco_status launch_dense_fmt(const bisco_layer &L, void *out, int dtype, int *err,
+                              cudaStream_t stream) {
+    if (L.n_protected <= 0) return BISCO_OK;
+    switch (dtype) {
+        case BISCO_DENSE_F32: return launch_dense_fmt_t(L, static_cast<float *>(out), err, stream);
+        case BISCO_DENSE_BF16:
+            return launch_dense_fmt_t(L, static_cast<__nv_bfloat16 *>(out), err, stream);
+        case BISCO_DENSE_F16: return launch_dense_fmt_t(L, static_cast<__half *>(out), err, stream);
+        default: return BISCO_ERR_INVALID_ARG;
+    }
+}
+
+}  // namespace bisco

@@ -189,25 +189,63 @@ def test_binding_argument_counts_match_header(lib):
     assert seen == set(bisco.EXPORTS)
 
 
-def test_row_layout_sizes_match_oracle(lib):
-    """axis 1: the buffers the oracle's row encoder fills, byte for byte."""
+def test_layer_sizes_match_oracle_layouts(lib):
+    """bisco_layer_sizes: the buffers the oracle's encoders fill, byte for
+    byte, for protected rows and for every protected payload format."""
     for (N, K, S, p) in [(64, 136, 2, 3), (12288, 4096, 2, 123), (40, 64, 1, 0), (16, 64, 3, 16)]:
-        sizes = bisco.bisco_encoded_sizes_axis(N, K, S, p, 1)
+        sizes = bisco.bisco_layer_sizes(N, K, S, p, axis=1)
         kp = oracle.pad16(K)
         assert sizes == [S * N * (K // 8), 2 * S * N * (K // 8), p * kp, 2 * p, 4 * p]
         if N * K <= 1 << 14:
             L = oracle.encode_rows(synth.layer_weights(N, K, seed=7), S, p)
             assert sizes[:2] == [L["codes"].nbytes, L["norms"].nbytes]
             assert sizes[2:] == [L["q8"].nbytes, L["scale"].nbytes, L["idx"].nbytes]
-    assert bisco.bisco_encoded_sizes_axis(64, 64, 2, 5, 0) == bisco.bisco_encoded_sizes(64, 64, 2, 5)
+    W = synth.layer_weights(48, 256, seed=8)
+    for fmt in (bisco.PROT_INT8, bisco.PROT_E4M3, bisco.PROT_E5M2, bisco.PROT_BF16):
+        sizes = bisco.bisco_layer_sizes(48, 256, 2, 5, axis=0, fmt=fmt)
+        assert sizes[:2] == bisco.bisco_encoded_sizes(48, 256, 2, 5)[:2]
+        idx = oracle.select_protected(W, 5)[0]
+        q, scale = oracle.quantize_protected_fmt(W, idx, fmt)
+        padded = q.itemsize * 48 * oracle.pad16(5)          # the oracle returns q[:, :p_pad]
+        assert sizes[2:] == [padded, scale.nbytes, 4 * 5]
+    assert bisco.bisco_layer_sizes(64, 64, 2, 5) == bisco.bisco_encoded_sizes(64, 64, 2, 5)
+    f = lib.bisco_layer_sizes
     out = (ctypes.c_size_t * 5)()
-    f = lib.bisco_encoded_sizes_axis
-    assert f(64, 64, 8, 2, 65, 1, out) == bisco.ERR_INVALID_ARG        # p > N
-    assert f(64, 128, 8, 2, 65, 1, out) == bisco.ERR_INVALID_ARG       # p > N although <= K
-    assert f(128, 64, 8, 2, 65, 1, out) == bisco.OK                    # rows may exceed K
-    assert f(64, 64, 8, 2, 4, 2, out) == bisco.ERR_INVALID_ARG         # axis
-    assert f(64, 64, 16, 2, 4, 1, out) == bisco.ERR_UNSUPPORTED
-    assert f(64, 64, 8, 2, 4, 1, None) == bisco.ERR_INVALID_ARG
+
+    def c(**kw):
+        base = dict(n_out=64, k_in=64, chunk_dim=8, stages=2, n_protected=4, protect_axis=0,
+                    protect_format=0)
+        base.update(kw)
+        return ctypes.byref(bisco.bisco_layer(**base))
+
+    assert f(c(), out) == bisco.OK
+    assert f(c(protect_axis=1, n_protected=65), out) == bisco.ERR_INVALID_ARG   # p > N
+    assert f(c(protect_axis=1, k_in=128, n_protected=65), out) == bisco.ERR_INVALID_ARG
+    assert f(c(protect_axis=1, n_out=128, n_protected=65), out) == bisco.OK      # rows may exceed K
+    assert f(c(protect_axis=2), out) == bisco.ERR_INVALID_ARG
+    assert f(c(chunk_dim=16), out) == bisco.ERR_UNSUPPORTED
+    assert f(c(protect_format=4), out) == bisco.ERR_INVALID_ARG
+    assert f(c(protect_format=-1), out) == bisco.ERR_INVALID_ARG
+    assert f(c(protect_format=1, protect_axis=1), out) == bisco.ERR_UNSUPPORTED  # FP8 rows
+    assert f(c(), None) == bisco.ERR_INVALID_ARG
+    assert f(None, out) == bisco.ERR_INVALID_ARG
+
+
+def test_protect_format_validation_before_any_device_call(lib):
+    x, y = ctypes.c_void_p(0x60000), ctypes.c_void_p(0x70000)
+    tab = ctypes.c_void_p(0x90000)
+    for fmt, code in ((5, bisco.ERR_INVALID_ARG), (-2, bisco.ERR_INVALID_ARG)):
+        L = _fake_layer(protect_format=fmt)
+        assert lib.bisco_gemv(ctypes.byref(L), x, 1, y, None) == code
+        assert lib.bisco_gemm(ctypes.byref(L), x, 4, y, None, 0, None) == code
+        assert lib.bisco_decode_dense(ctypes.byref(L), y, bisco.DENSE_F32, None) == code
+    L = _fake_layer(protect_format=bisco.PROT_E4M3, protect_axis=1)
+    assert lib.bisco_gemv(ctypes.byref(L), x, 1, y, None) == bisco.ERR_UNSUPPORTED
+    for fmt in (bisco.PROT_E4M3, bisco.PROT_E5M2, bisco.PROT_BF16):       # tables: INT8 only
+        L = _fake_layer(protect_format=fmt)
+        assert lib.bisco_gemv_table(ctypes.byref(L), tab, x, 1, y, None) == bisco.ERR_UNSUPPORTED
+        assert lib.bisco_decode_dense_table(ctypes.byref(L), tab, y, 0, None) == bisco.ERR_UNSUPPORTED
+        assert lib.bisco_encode_noalloc(x, None, ctypes.byref(L), None) == bisco.ERR_UNSUPPORTED
 
 
 def test_encode_workspace_by_axis(lib):
