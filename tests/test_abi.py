@@ -324,3 +324,20 @@ def test_decoder_table_validation(lib):
     assert d(ctypes.byref(L), tab, None, bisco.DENSE_BF16, None) == E
     assert d(ctypes.byref(L), tab, ctypes.c_void_p(0x70004), bisco.DENSE_F16, None) == E
     assert d(ctypes.byref(_fake_layer(stages=4)), tab, y, bisco.DENSE_F32, None) == E
+
+
+def test_struct_layout_matches_the_header(tmp_path):
+    """The ctypes mirror of bisco_layer has the C struct's size and field
+    offsets (an array of them crosses the ABI in bisco_gemv_multi)."""
+    import subprocess
+    fields = [f for f, _ in bisco.bisco_layer._fields_]
+    src = tmp_path / "layout.c"
+    src.write_text('#include <stdio.h>\n#include <stddef.h>\n#include "bisco.h"\nint main(void) {\n'
+                   '  printf("%zu\\n", sizeof(bisco_layer));\n' +
+                   "".join('  printf("%%zu\\n", offsetof(bisco_layer, %s));\n' % f for f in fields) +
+                   "  return 0;\n}\n")
+    exe = tmp_path / "layout"
+    subprocess.check_call(["gcc", "-std=c11", "-I", os.path.join(ROOT, "include"), "-o", str(exe), str(src)])
+    out = [int(v) for v in subprocess.check_output([str(exe)]).split()]
+    assert out[0] == ctypes.sizeof(bisco.bisco_layer)
+    assert out[1:] == [getattr(bisco.bisco_layer, f).offset for f in fields]
