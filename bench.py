@@ -45,11 +45,13 @@ def parse():
     ap.add_argument("--impl", choices=("bisco", "reference"), default="bisco")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
-    ap.add_argument("--mode", choices=("both", "decode", "prefill", "shapes", "dense", "lora"),
+    ap.add_argument("--mode", choices=("both", "decode", "prefill", "shapes", "dense", "lora",
+                                       "stack"),
                     default="both",
                     help="decode: the GEMV step only; prefill: the tcgen05 GEMM only; "
                          "shapes: batch-1 GEMV per Qwen3-8B layer shape; lora: the decode step "
-                         "with a low-rank compensation on every projection")
+                         "with a low-rank compensation on every projection; stack: the full "
+                         "7-projection stack at batch 1/4/16 and the GEMV/GEMM crossover")
     ap.add_argument("--lora-rank", type=int, default=16)
     ap.add_argument("--shape-mb", type=float, default=500.0,
                     help="--mode shapes: MB of distinct coded layers per shape (> L2)")
@@ -697,6 +699,116 @@ def run_shapes(args, local_rank):
     return out
 
 
+# ------------------------------------------------------------------ stack
+
+STACK = ("q_proj", "k_proj", "v_proj", "o_proj", "gate_proj", "up_proj", "down_proj")
+
+
+def run_stack(args, local_rank):
+    """The full linear stack of Qwen3-8B: 7 projections x --layers layers,
+    each a distinct random layer (N(0,0.02) + 8 outlier columns x20), d = 8,
+    S = 2, 1 % protected columns (5.28 GB coded for 36 layers, far more than
+    L2).  Decode sweep at batch 1, 4 and 16 through bisco_gemv_multi (q/k/v;
+    gate/up) and bisco_gemv (o; down), four launches per layer; then the
+    GEMV/GEMM crossover, bisco_gemm on every projection at M = 1, 4, 16, 64
+    (decode kernels) and 128 (tensor cores).  Each is a CUDA graph of the
+    whole stack, CUDA events over `steps` replays."""
+    import torch
+    from paper_2607_08643_gb300 import bisco, synth
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    layers = []
+    ws = None
+    for l in range(args.layers):
+        for j, name in enumerate(STACK):
+            N, K = synth.QWEN3_8B_SHAPES[name]
+            p = synth.protected_count(K, RHO_PCT)
+            W = synth.layer_weights_torch(N, K, seed=1000 * l + j, device=dev)
+            need = bisco.bisco_encode_workspace_bytes(N, K)
+            if ws is None or ws.numel() < need:
+                ws = torch.empty(need, dtype=torch.uint8, device=dev)
+            layers.append(bisco.bisco_encode(W, S_STAGES, p, workspace=ws))
+            del W
+    torch.cuda.synchronize()
+    if bisco.bisco_get_device_error() != bisco.OK:
+        raise RuntimeError("device error while encoding the stack")
+    total = sum(L.compressed_bytes for L in layers)
+    peak, peak_kind = peaks()
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(77)
+    stream = torch.cuda.Stream(device=dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(step):
+        with torch.cuda.stream(stream):
+            step()
+            torch.cuda.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                step()
+        torch.cuda.synchronize()
+        for _ in range(max(args.warmup, 3)):
+            g.replay()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(args.steps):
+                g.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        if bisco.bisco_get_device_error(stream) != bisco.OK:
+            raise RuntimeError("device error in the stack step")
+        return e0.elapsed_time(e1) / args.steps
+
+    def inputs(B):
+        xk = torch.randn((B, 4096), generator=gen, device=dev).to(torch.bfloat16).view(torch.int16)
+        xf = torch.randn((B, 12288), generator=gen, device=dev).to(torch.bfloat16).view(torch.int16)
+        ys = {nm: torch.empty((B, synth.QWEN3_8B_SHAPES[nm][0]), device=dev) for nm in STACK}
+        return xk, xf, ys
+
+    sweep = []
+    for B in (1, 4, 16):
+        xk, xf, ys = inputs(B)
+
+        def step():
+            for l in range(args.layers):
+                Ls = layers[7 * l:7 * l + 7]
+                bisco.bisco_gemv_multi(Ls[0:3], xk, ys=[ys[nm] for nm in STACK[0:3]], stream=stream)
+                bisco.bisco_gemv(Ls[3], xk, y=ys["o_proj"], stream=stream)
+                bisco.bisco_gemv_multi(Ls[4:6], xk, ys=[ys[nm] for nm in STACK[4:6]], stream=stream)
+                bisco.bisco_gemv(Ls[6], xf, y=ys["down_proj"], stream=stream)
+        ms = timed(step)
+        gbs = total / (ms * 1e-3) / 1e9
+        sweep.append({"batch": B, "ms_per_step": ms, "gbs": gbs, "frac_of_hbm": gbs / peak,
+                      "tokens_per_s": B / (ms * 1e-3), "calls_per_step": 4 * args.layers})
+        del xk, xf, ys
+    cross = []
+    for M in (1, 4, 16, 64, 128):
+        xk, xf, ys = inputs(M)
+        need = max(bisco.bisco_gemm_workspace_bytes(L, M) for L in layers)
+        gws = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+
+        def step():
+            for l in range(args.layers):
+                for j, nm in enumerate(STACK):
+                    L = layers[7 * l + j]
+                    bisco.bisco_gemm(L, xf if nm == "down_proj" else xk, Y=ys[nm],
+                                     workspace=gws, stream=stream)
+        ms = timed(step)
+        cross.append({"tokens": M, "ms_per_step": ms, "tokens_per_s": M / (ms * 1e-3),
+                      "gbs": total / (ms * 1e-3) / 1e9,
+                      "path": "tcgen05 GEMM" if M > 64 else "decode kernels"})
+        del xk, xf, ys, gws
+    return {"metric": "Qwen3-8B linear stack decode sweep and GEMV/GEMM crossover",
+            "unit": "GB/s", "layers": args.layers, "projections": list(STACK),
+            "compressed_bytes": total, "hbm_peak_gbs": peak, "peak_source": peak_kind,
+            "decode": sweep, "crossover_gemm": cross,
+            "config": {"workload": "Qwen3-8B linear stack, 7 projections x %d layers" % args.layers,
+                       "chunk_dim": 8, "stages": S_STAGES, "protected_pct": RHO_PCT,
+                       "weights": "N(0,0.02) + 8 outlier cols x20, seeded on device",
+                       "l2": "inputs larger than L2 (distinct coded layers per step, no flush)"}}
+
+
 # ------------------------------------------------------------ CPU oracle
 
 def cpu_oracle_sample(seconds, batch):
@@ -783,6 +895,12 @@ def main():
             print(json.dumps({"metric": "batch-1 GEMV GB/s per Qwen3-8B shape (compressed bytes)",
                               "unit": "GB/s", "hbm_peak_gbs": peaks()[0], "steps": args.steps,
                               "data": "synthetic", "shapes": res}))
+        return
+    if args.mode == "stack":
+        st = run_stack(args, local_rank)
+        if rank == 0:
+            print(json.dumps(dict(st, n_gpus=world, steps=args.steps, warmup=args.warmup,
+                                  data="synthetic")))
         return
     if args.mode == "lora":
         lr = run_lora(args, local_rank)
