@@ -19,20 +19,10 @@
 
 #include "bisco_dev.cuh"
 #include "bisco_host.h"
+#include "fp8.cuh"
 
 namespace bisco {
 namespace {
-
-struct Fp8Format {
-    int mbits, bias;
-    double maxf;
-    uint8_t maxcode;
-};
-
-__device__ __forceinline__ Fp8Format fp8_format(int fmt) {
-    if (fmt == BISCO_PROT_E4M3) return {3, 7, 448.0, 0x7E};
-    return {2, 15, 57344.0, 0x7B};   // BISCO_PROT_E5M2
-}
 
 __device__ __forceinline__ uint16_t f64_to_f16_rn(double x) {
     unsigned short r;
@@ -48,43 +38,11 @@ __device__ __forceinline__ double bf16_to_f64(uint16_t b) {
     return static_cast<double>(__uint_as_float(static_cast<uint32_t>(b) << 16));
 }
 
-// binary64 -> FP8 bits, nearest even: the significand scaled so that the
-// kept bits are its integer part (exact, a power of two), rounded once by
-// rint; subnormals share the least normal exponent; above F saturates.
-__device__ __forceinline__ uint8_t f64_to_fp8(double x, const Fp8Format &f) {
-    const uint8_t sign = signbit(x) ? 0x80 : 0x00;
-    const double a = fabs(x);
-    if (a == 0.0) return sign;
-    int E = ilogb(a);
-    if (E < 1 - f.bias) E = 1 - f.bias;
-    double m = rint(ldexp(a, f.mbits - E));
-    if (m == ldexp(1.0, f.mbits + 1)) {   // rounded up to the next binade
-        m = ldexp(1.0, f.mbits);
-        E += 1;
-    }
-    if (ldexp(m, E - f.mbits) > f.maxf) return sign | f.maxcode;
-    const int mi = static_cast<int>(m);
-    if (mi >= (1 << f.mbits))
-        return sign | static_cast<uint8_t>(((E + f.bias) << f.mbits) | (mi - (1 << f.mbits)));
-    return sign | static_cast<uint8_t>(mi);
-}
-
 // The value of a protected payload element (exact in fp32).
 __device__ __forceinline__ float payload_value(const void *q, int64_t e, int fmt) {
     if (fmt == BISCO_PROT_BF16)
         return __uint_as_float(static_cast<uint32_t>(static_cast<const uint16_t *>(q)[e]) << 16);
-    const uint32_t v = static_cast<const uint8_t *>(q)[e];
-    if (fmt == BISCO_PROT_E5M2)   // E5M2 is the upper byte of a binary16
-        return __half2float(__ushort_as_half(static_cast<uint16_t>(v << 8)));
-    const uint32_t ex = (v >> 3) & 0xFu, mn = v & 7u;   // E4M3
-    float r;
-    if (ex == 15u && mn == 7u)
-        r = __uint_as_float(0x7FC00000u);
-    else if (ex == 0u)
-        r = ldexpf(static_cast<float>(mn), -9);
-    else
-        r = ldexpf(static_cast<float>(8u + mn), static_cast<int>(ex) - 10);
-    return (v & 0x80u) ? -r : r;
+    return fp8_to_f32(static_cast<const uint8_t *>(q)[e], fmt);
 }
 
 // Encoder: one CTA per payload column t < p_pad (t >= p: zero padding).
