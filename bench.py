@@ -46,12 +46,13 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--mode", choices=("both", "decode", "prefill", "shapes", "dense", "lora",
-                                       "stack"),
+                                       "stack", "variants"),
                     default="both",
                     help="decode: the GEMV step only; prefill: the tcgen05 GEMM only; "
                          "shapes: batch-1 GEMV per Qwen3-8B layer shape; lora: the decode step "
                          "with a low-rank compensation on every projection; stack: the full "
-                         "7-projection stack at batch 1/4/16 and the GEMV/GEMM crossover")
+                         "7-projection stack at batch 1/4/16 and the GEMV/GEMM crossover; "
+                         "variants: the decode step per protected-set / decoder variant")
     ap.add_argument("--lora-rank", type=int, default=16)
     ap.add_argument("--shape-mb", type=float, default=500.0,
                     help="--mode shapes: MB of distinct coded layers per shape (> L2)")
@@ -809,6 +810,87 @@ def run_stack(args, local_rank):
                        "l2": "inputs larger than L2 (distinct coded layers per step, no flush)"}}
 
 
+# --------------------------------------------------------------- variants
+
+def run_variants(args, local_rank):
+    """The batch-B decode step of the 36-layer q/k/v/o stack (as in the
+    default line) with each protected-set and decoder variant of the
+    library: INT8 protected columns (the default), FP8 E4M3 and BF16
+    payloads (protected-format ablation), 1 % protected output rows
+    (Eq. 9 / Eq. 10 on rows) and the learned decoder step as per-stage
+    tables (bisco_gemv_table, one call per projection).  One CUDA graph per
+    variant, CUDA events over `steps` replays; GB/s on each variant's own
+    compressed bytes (the decoder tables, 8 KB per layer, are not counted)."""
+    import torch
+    from paper_2607_08643_gb300 import bisco, synth
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    peak, peak_kind = peaks()
+    B = args.batch
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(31)
+    x = torch.randn((B, 4096), generator=gen, device=dev).to(torch.bfloat16).view(torch.int16)
+    stream = torch.cuda.Stream(device=dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    tabs = (torch.randn((S_STAGES, 256, 8), generator=gen, device=dev) * 0.35).to(torch.float16)
+    out = []
+    for name, axis, fmt, table in (("int8 columns", 0, bisco.PROT_INT8, False),
+                                   ("fp8 e4m3 columns", 0, bisco.PROT_E4M3, False),
+                                   ("bf16 columns", 0, bisco.PROT_BF16, False),
+                                   ("int8 rows", 1, bisco.PROT_INT8, False),
+                                   ("decoder tables", 0, bisco.PROT_INT8, True)):
+        layers = []
+        for l in range(args.layers):
+            for j, proj in enumerate(ATTN):
+                N, K = synth.QWEN3_8B_SHAPES[proj]
+                p = synth.protected_count(N if axis else K, RHO_PCT)
+                W = synth.layer_weights_torch(N, K, seed=1000 * l + j, device=dev)
+                layers.append(bisco.bisco_encode(W, S_STAGES, p, axis=axis, fmt=fmt))
+                del W
+        ys = [torch.empty((B, L.N), device=dev) for L in layers]
+        torch.cuda.synchronize()
+
+        def step():
+            for l in range(args.layers):
+                q = list(range(4 * l, 4 * l + 4))
+                if table:
+                    for i in q:
+                        bisco.bisco_gemv_table(layers[i], tabs, x, y=ys[i], stream=stream)
+                else:
+                    bisco.bisco_gemv_multi([layers[i] for i in q[:3]], x,
+                                           ys=[ys[i] for i in q[:3]], stream=stream)
+                    bisco.bisco_gemv(layers[q[3]], x, y=ys[q[3]], stream=stream)
+
+        with torch.cuda.stream(stream):
+            step()
+            torch.cuda.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                step()
+        torch.cuda.synchronize()
+        for _ in range(max(args.warmup, 3)):
+            g.replay()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(args.steps):
+                g.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        if bisco.bisco_get_device_error(stream) != bisco.OK:
+            raise RuntimeError("device error in variant " + name)
+        ms = e0.elapsed_time(e1) / args.steps
+        total = sum(L.compressed_bytes for L in layers)
+        gbs = total / (ms * 1e-3) / 1e9
+        out.append({"variant": name, "bytes_per_step": total, "ms_per_step": ms, "gbs": gbs,
+                    "frac_of_hbm": gbs / peak, "tokens_per_s": B / (ms * 1e-3)})
+        del layers, ys, g
+        torch.cuda.empty_cache()
+    return {"metric": "decode step per protected-set / decoder variant", "unit": "GB/s",
+            "batch": B, "layers": args.layers, "hbm_peak_gbs": peak, "peak_source": peak_kind,
+            "variants": out}
+
+
 # ------------------------------------------------------------ CPU oracle
 
 def cpu_oracle_sample(seconds, batch):
@@ -895,6 +977,12 @@ def main():
             print(json.dumps({"metric": "batch-1 GEMV GB/s per Qwen3-8B shape (compressed bytes)",
                               "unit": "GB/s", "hbm_peak_gbs": peaks()[0], "steps": args.steps,
                               "data": "synthetic", "shapes": res}))
+        return
+    if args.mode == "variants":
+        vr = run_variants(args, local_rank)
+        if rank == 0:
+            print(json.dumps(dict(vr, n_gpus=world, steps=args.steps, warmup=args.warmup,
+                                  data="synthetic", config=workload_config(args))))
         return
     if args.mode == "stack":
         st = run_stack(args, local_rank)
