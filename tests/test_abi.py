@@ -341,3 +341,34 @@ def test_struct_layout_matches_the_header(tmp_path):
     out = [int(v) for v in subprocess.check_output([str(exe)]).split()]
     assert out[0] == ctypes.sizeof(bisco.bisco_layer)
     assert out[1:] == [getattr(bisco.bisco_layer, f).offset for f in fields]
+
+
+@pytest.mark.parametrize("axis,fmt", [(0, bisco.PROT_INT8), (0, bisco.PROT_E4M3), (0, bisco.PROT_E5M2),
+                                      (0, bisco.PROT_BF16), (1, bisco.PROT_INT8)])
+def test_layer_marshalling_round_trip(lib, axis, fmt):
+    """Layer.from_numpy / to_numpy carry the oracle's layer dicts exactly for
+    every protection axis and payload format (host tensors; no device call),
+    and the C struct describes the tensors it points at."""
+    import numpy as np
+    N, K, S, p = 40, 136, 2, 3
+    W = synth.layer_weights(N, K, seed=5)
+    if axis == 1:
+        ref = oracle.encode_rows(W, S, p)
+    else:
+        ref = oracle.encode(W, S=S, p=p)
+        if fmt != bisco.PROT_INT8:
+            q, scale = oracle.quantize_protected_fmt(W, ref["idx"], fmt)
+            ref = dict(ref, q8=q, scale=scale, fmt=fmt)
+    L = bisco.Layer.from_numpy(ref, device="cpu")
+    got = L.to_numpy()
+    for k in ("codes", "norms", "q8", "scale", "idx"):
+        assert got[k].dtype == ref[k].dtype and np.array_equal(got[k], ref[k]), k
+    assert got.get("axis", 0) == axis and got.get("fmt", 0) == ref.get("fmt", 0)
+    c = L.c
+    assert (c.n_out, c.k_in, c.stages, c.n_protected, c.protect_axis, c.protect_format) == \
+        (N, K, S, p, axis, fmt)
+    assert c.codes == L.codes.data_ptr() and c.q8 == L.q8.data_ptr() and c.prot_idx == L.idx.data_ptr()
+    sizes = bisco.bisco_layer_sizes(N, K, S, p, axis, fmt)
+    assert sizes[2] <= L.q8.numel() * L.q8.element_size()
+    extra = 2 if fmt == bisco.PROT_BF16 else 1
+    assert L.compressed_bytes == S * N * (K // 8) * 3 + p * (K if axis else N) * extra + 6 * p
