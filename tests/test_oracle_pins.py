@@ -838,3 +838,28 @@ def test_mlp_decoder_odd_residual_and_limits():
     assert np.allclose(T / eps, lin_r, rtol=0, atol=1e-8 * np.abs(lin_r).max())
     with pytest.raises(oracle.OracleError):
         oracle.decoder_table_mlp(np.zeros((0, 8)), np.zeros((8, 0)))
+
+
+def test_encode_with_given_columns_reduces_to_eq8_encode():
+    """Given the very set Eq. 8 selects, the given-set encoder is the
+    ordinary encoder byte for byte; a different set moves the masking."""
+    W = synth.layer_weights(48, 136, seed=101, dist="t4")
+    for S, p in ((1, 3), (2, 5), (3, 17)):
+        ref = oracle.encode(W, S=S, p=p)
+        got = oracle.encode_given(W, S, ref["idx"])
+        for k in ("codes", "norms", "q8", "scale", "idx"):
+            assert np.array_equal(got[k], ref[k]), (S, p, k)
+    other = np.array([0, 7, 8, 135], np.int32)
+    L = oracle.encode_given(W, 2, other)
+    What = oracle.decode_rows(L)
+    sc = L["scale"].view(np.float16).astype(np.float64)
+    assert np.array_equal(What[:, other], sc[None, :] * L["q8"][:, :4].astype(np.float64))
+    Wm = f64(W)
+    Wm[:, other] = 0.0
+    # the stage-1 norms are those of the chunks with the given columns zeroed
+    n1 = np.sqrt((Wm.reshape(48, 17, 8) ** 2).sum(axis=2)).astype(np.float16)
+    assert np.array_equal(L["norms"][0], n1.view(np.uint16))
+    with pytest.raises(oracle.OracleError):
+        oracle.encode_given(W, 2, np.array([5, 3], np.int32))        # not ascending
+    with pytest.raises(oracle.OracleError):
+        oracle.encode_given(W, 2, np.array([136], np.int32))         # out of range
