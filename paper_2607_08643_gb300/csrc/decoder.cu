@@ -126,6 +126,118 @@ __global__ void __launch_bounds__(256) k_gemv_table(const uint8_t *__restrict__ 
     }
 }
 
+// k_gemv_table for K % 32 == 0: each lane takes groups of 4 consecutive
+// chunks, one 32-bit code word and one 8-byte norm word per stage, and
+// issues the loads of UNROLL groups before decoding any of them; S is a
+// template parameter so that the words stay in registers.
+template <int S, int UNROLL>
+__global__ void __launch_bounds__(256) k_gemv_table_v(const uint8_t *__restrict__ codes,
+                                                      const uint16_t *__restrict__ norms,
+                                                      const uint16_t *__restrict__ tables,
+                                                      const int8_t *__restrict__ q8,
+                                                      const uint16_t *__restrict__ q8_scale,
+                                                      const int32_t *__restrict__ prot_idx, int N,
+                                                      int K, int p,
+                                                      const uint16_t *__restrict__ x, int B,
+                                                      float *__restrict__ y, int *err) {
+    __shared__ uint4 s_tab[3 * kTableEntries / 8];
+    stage_tables(tables, S, s_tab);
+    const int C = K / 8, G = C / 4, p_pad = (p + 15) / 16 * 16;
+    const int lane = threadIdx.x & 31;
+    const int i = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
+    if (i >= N) return;
+    const uint32_t *cw32 = reinterpret_cast<const uint32_t *>(codes);
+    const uint2 *nw64 = reinterpret_cast<const uint2 *>(norms);
+    float acc[16];
+#pragma unroll
+    for (int b = 0; b < 16; ++b) acc[b] = 0.f;
+    for (int g0 = lane; g0 < G; g0 += 32 * UNROLL) {
+        uint32_t cw[UNROLL][S];
+        uint2 nw[UNROLL][S];
+#pragma unroll
+        for (int u = 0; u < UNROLL; ++u) {
+            const int g = min(g0 + 32 * u, G - 1);   // groups past the row reload the last one
+#pragma unroll
+            for (int s = 0; s < S; ++s) {
+                const int64_t e = (static_cast<int64_t>(s) * N + i) * G + g;
+                cw[u][s] = cw32[e];
+                nw[u][s] = nw64[e];
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < UNROLL; ++u) {
+            const int g = g0 + 32 * u;
+            if (g >= G) break;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                float w[8];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) w[k] = 0.f;
+#pragma unroll
+                for (int s = 0; s < S; ++s) {
+                    const uint32_t v = (cw[u][s] >> (8 * q)) & 0xFFu;
+                    const uint32_t nh = q < 2 ? nw[u][s].x : nw[u][s].y;
+                    const float n = __half2float(__ushort_as_half(
+                        static_cast<uint16_t>((q & 1) ? (nh >> 16) : (nh & 0xFFFFu))));
+                    const uint4 row = s_tab[s * 256 + v];
+                    const uint32_t hw[4] = {row.x, row.y, row.z, row.w};
+#pragma unroll
+                    for (int h = 0; h < 4; ++h) {
+                        const float2 t = __half22float2(*reinterpret_cast<const __half2 *>(&hw[h]));
+                        w[2 * h] = fmaf(n, t.x, w[2 * h]);
+                        w[2 * h + 1] = fmaf(n, t.y, w[2 * h + 1]);
+                    }
+                }
+                const int c = 4 * g + q;
+#pragma unroll
+                for (int b = 0; b < 16; ++b) {
+                    if (b >= B) break;
+                    const uint4 xr =
+                        *reinterpret_cast<const uint4 *>(x + static_cast<int64_t>(b) * K + 8 * c);
+                    const uint32_t xw[4] = {xr.x, xr.y, xr.z, xr.w};
+                    float d = 0.f;
+#pragma unroll
+                    for (int h = 0; h < 4; ++h) {
+                        d = fmaf(w[2 * h], __uint_as_float(xw[h] << 16), d);
+                        d = fmaf(w[2 * h + 1], __uint_as_float(xw[h] & 0xFFFF0000u), d);
+                    }
+                    acc[b] += d;
+                }
+            }
+        }
+    }
+    // Eq. 10, as in k_gemv_table
+    const int64_t stride = static_cast<int64_t>(N) * C;
+    for (int t = lane; t < p; t += 32) {
+        const int j = prot_idx[t];
+        if (j < 0 || j >= K) {
+            latch_error(err, BISCO_ERR_INVALID_ARG);
+            continue;
+        }
+        float w[8];
+        decode_chunk(codes, norms, s_tab, S, static_cast<int64_t>(i) * C + j / 8, stride, w);
+        float wb = 0.f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) wb = (k == j % 8) ? w[k] : wb;
+        const float wq = __half2float(__ushort_as_half(q8_scale[t])) *
+                         static_cast<float>(q8[static_cast<int64_t>(i) * p_pad + t]);
+#pragma unroll
+        for (int b = 0; b < 16; ++b) {
+            if (b >= B) break;
+            acc[b] += (wq - wb) * bf16_to_f32(x[static_cast<int64_t>(b) * K + j]);
+        }
+    }
+#pragma unroll
+    for (int b = 0; b < 16; ++b)
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) acc[b] += __shfl_xor_sync(0xffffffffu, acc[b], o);
+    if (lane == 0) {
+#pragma unroll
+        for (int b = 0; b < 16; ++b)
+            if (b < B) y[static_cast<int64_t>(b) * N + i] = acc[b];
+    }
+}
+
 template <typename T>
 __device__ __forceinline__ T from_f32(float v);
 template <>
@@ -196,9 +308,28 @@ bisco_status launch_dense_table_t(const bisco_layer &L, const uint16_t *tables, 
 bisco_status launch_gemv_table(const bisco_layer &L, const uint16_t *tables, const uint16_t *x,
                                int B, float *y, int *err, cudaStream_t stream) {
     const int rows_per_block = 8;
-    k_gemv_table<<<(L.n_out + rows_per_block - 1) / rows_per_block, 32 * rows_per_block, 0,
-                   stream>>>(L.codes, L.norms, tables, L.q8, L.q8_scale, L.prot_idx, L.n_out,
-                             L.k_in, L.stages, L.n_protected, x, B, y, err);
+    const unsigned grid = (L.n_out + rows_per_block - 1) / rows_per_block;
+    const int N = L.n_out, K = L.k_in, p = L.n_protected;
+    if (K % 32 == 0) {   // 4-chunk code and norm words are aligned
+        switch (L.stages) {
+            case 1:
+                k_gemv_table_v<1, 2><<<grid, 32 * rows_per_block, 0, stream>>>(
+                    L.codes, L.norms, tables, L.q8, L.q8_scale, L.prot_idx, N, K, p, x, B, y, err);
+                break;
+            case 2:
+                k_gemv_table_v<2, 2><<<grid, 32 * rows_per_block, 0, stream>>>(
+                    L.codes, L.norms, tables, L.q8, L.q8_scale, L.prot_idx, N, K, p, x, B, y, err);
+                break;
+            default:
+                k_gemv_table_v<3, 2><<<grid, 32 * rows_per_block, 0, stream>>>(
+                    L.codes, L.norms, tables, L.q8, L.q8_scale, L.prot_idx, N, K, p, x, B, y, err);
+                break;
+        }
+    } else {
+        k_gemv_table<<<grid, 32 * rows_per_block, 0, stream>>>(L.codes, L.norms, tables, L.q8,
+                                                              L.q8_scale, L.prot_idx, N, K,
+                                                              L.stages, p, x, B, y, err);
+    }
     return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
 }
 
