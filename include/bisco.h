@@ -10,13 +10,18 @@
  * Eq. 10), and inference decodes the stages independently and sums them
  * (Sec. III-G, Eq. 12) before the linear map y = W x.  This library runs
  * that linear map straight from the coded bytes, without ever writing the
- * dense weight to memory.
+ * dense weight to memory.  Beside that path it takes the method's variants:
+ * output rows as the protected channels, with the coupled gate/up/down set
+ * of a gated MLP (Eq. 9); FP8 and BF16 protected payloads; the learned
+ * decoder of Eq. 1 given as per-stage tables; the materialised weight; and
+ * the optional low-rank compensation.
  *
  * Conventions for every entry point:
  *   - All pointers are caller-owned DEVICE memory unless stated otherwise;
  *     the library allocates nothing and keeps no state between calls other
  *     than a per-device error word.
- *   - Pointers must be 16-byte aligned, else BISCO_ERR_INVALID_ARG.
+ *   - Pointers must be 16-byte aligned, else BISCO_ERR_INVALID_ARG; the
+ *     per-channel float weights g and caller-given index lists need 4.
  *   - Calls are asynchronous on `stream` (NULL = the legacy default stream).
  *     Argument errors are returned synchronously and nothing is launched.
  *     Errors found on the device (fp16 overflow in encode, an expired
