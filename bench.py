@@ -820,7 +820,9 @@ def run_variants(args, local_rank):
     (Eq. 9 / Eq. 10 on rows) and the learned decoder step as per-stage
     tables (bisco_gemv_table, one call per projection).  One CUDA graph per
     variant, CUDA events over `steps` replays; GB/s on each variant's own
-    compressed bytes (the decoder tables, 8 KB per layer, are not counted)."""
+    compressed bytes (the decoder tables, 8 KB per layer, are not counted).
+    Then the gated MLP of the same layers (gate/up grouped, down) with
+    per-layer INT8 columns and with the coupled set of Eq. 9."""
     import torch
     from paper_2607_08643_gb300 import bisco, synth
     dev = torch.device("cuda", local_rank)
@@ -886,9 +888,64 @@ def run_variants(args, local_rank):
                     "frac_of_hbm": gbs / peak, "tokens_per_s": B / (ms * 1e-3)})
         del layers, ys, g
         torch.cuda.empty_cache()
+    # the gated MLP (gate/up 12288x4096, down 4096x12288): 1 % protected input
+    # columns per layer, against the coupled set of Eq. 9 (rows of gate and
+    # up, columns of down, 1 % of the 12288 channels)
+    xf = torch.randn((B, 12288), generator=gen, device=dev).to(torch.bfloat16).view(torch.int16)
+    mlp = []
+    for name in ("int8 columns", "coupled rows + columns"):
+        layers = []
+        for l in range(args.layers):
+            Ws = [synth.layer_weights_torch(*synth.QWEN3_8B_SHAPES[proj], seed=1000 * l + 4 + j,
+                                            device=dev)
+                  for j, proj in enumerate(("gate_proj", "up_proj", "down_proj"))]
+            if name == "int8 columns":
+                layers += [bisco.bisco_encode(W, S_STAGES, synth.protected_count(W.shape[1], RHO_PCT))
+                           for W in Ws]
+            else:
+                idx = bisco.bisco_select_coupled(Ws[0], Ws[1], Ws[2],
+                                                 synth.protected_count(Ws[0].shape[0], RHO_PCT))
+                layers += [bisco.bisco_encode_with_set(Ws[0], S_STAGES, idx, axis=1),
+                           bisco.bisco_encode_with_set(Ws[1], S_STAGES, idx, axis=1),
+                           bisco.bisco_encode_with_set(Ws[2], S_STAGES, idx, axis=0)]
+            del Ws
+        ys = [torch.empty((B, L.N), device=dev) for L in layers]
+        torch.cuda.synchronize()
+
+        def step():
+            for l in range(args.layers):
+                g = 3 * l
+                bisco.bisco_gemv_multi(layers[g:g + 2], x, ys=ys[g:g + 2], stream=stream)
+                bisco.bisco_gemv(layers[g + 2], xf, y=ys[g + 2], stream=stream)
+
+        with torch.cuda.stream(stream):
+            step()
+            torch.cuda.synchronize()
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, stream=stream):
+                step()
+        torch.cuda.synchronize()
+        for _ in range(max(args.warmup, 3)):
+            gr.replay()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(args.steps):
+                gr.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        if bisco.bisco_get_device_error(stream) != bisco.OK:
+            raise RuntimeError("device error in MLP variant " + name)
+        ms = e0.elapsed_time(e1) / args.steps
+        total = sum(L.compressed_bytes for L in layers)
+        gbs = total / (ms * 1e-3) / 1e9
+        mlp.append({"variant": name, "bytes_per_step": total, "ms_per_step": ms, "gbs": gbs,
+                    "frac_of_hbm": gbs / peak, "tokens_per_s": B / (ms * 1e-3)})
+        del layers, ys, gr
+        torch.cuda.empty_cache()
     return {"metric": "decode step per protected-set / decoder variant", "unit": "GB/s",
             "batch": B, "layers": args.layers, "hbm_peak_gbs": peak, "peak_source": peak_kind,
-            "variants": out}
+            "variants": out, "mlp_variants": mlp}
 
 
 # ------------------------------------------------------------ CPU oracle
