@@ -109,59 +109,63 @@ __global__ void __launch_bounds__(256) k_prot_fix(const uint8_t *__restrict__ co
     __shared__ float s_x[kFixTok][kFixT + 1];
     const int tid = threadIdx.x;
     const int r = tid >> 3, c = tid & 7;
-    const int i0 = blockIdx.x * kFixRows, m0 = blockIdx.y * kFixTok;
+    const int i0 = blockIdx.x * kFixRows;
     const int C = K / 8, p_pad = (p + 15) / 16 * 16;
     const float inv_sqrt8 = 0.35355339059327373f;   // the decode kernels' 1/sqrt(8) in fp32
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
-    for (int t0 = 0; t0 < p; t0 += kFixT) {
+    // token tiles stride by the grid (its y extent is capped at 65535)
+    for (int m0 = blockIdx.y * kFixTok; m0 < M; m0 += gridDim.y * kFixTok) {
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int t0 = 0; t0 < p; t0 += kFixT) {
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int tt = 4 * c + u, t = t0 + tt;
-            // d = scale * value(q) - (stage value of that weight), row i0 + r
-            float d = 0.f;
-            const int i = i0 + r;
-            if (t < p && i < N) {
-                const int j = idx[t];
-                if (j >= 0 && j < K) {
-                    float wb = 0.f;
-                    for (int s = 0; s < S; ++s) {
-                        const int64_t e = (static_cast<int64_t>(s) * N + i) * C + j / 8;
-                        const float n = __half2float(__ushort_as_half(norms[e]));
-                        wb += ((codes[e] >> (j % 8)) & 1u) ? -n : n;
+            for (int u = 0; u < 4; ++u) {
+                const int tt = 4 * c + u, t = t0 + tt;
+                // d = scale * value(q) - (stage value of that weight), row i0 + r
+                float d = 0.f;
+                const int i = i0 + r;
+                if (t < p && i < N) {
+                    const int j = idx[t];
+                    if (j >= 0 && j < K) {
+                        float wb = 0.f;
+                        for (int s = 0; s < S; ++s) {
+                            const int64_t e = (static_cast<int64_t>(s) * N + i) * C + j / 8;
+                            const float n = __half2float(__ushort_as_half(norms[e]));
+                            wb += ((codes[e] >> (j % 8)) & 1u) ? -n : n;
+                        }
+                        const float sc = __half2float(__ushort_as_half(scale[t]));
+                        d = sc * payload_value(q, static_cast<int64_t>(i) * p_pad + t, fmt) -
+                            wb * inv_sqrt8;
+                    } else if (r == 0) {
+                        latch_error(err, BISCO_ERR_INVALID_ARG);   // not a column of this layer
                     }
-                    const float sc = __half2float(__ushort_as_half(scale[t]));
-                    d = sc * payload_value(q, static_cast<int64_t>(i) * p_pad + t, fmt) -
-                        wb * inv_sqrt8;
-                } else if (r == 0) {
-                    latch_error(err, BISCO_ERR_INVALID_ARG);   // not a column of this layer
                 }
+                s_d[r][tt] = d;
+                // activation (m0 + r, column j_t)
+                float xv = 0.f;
+                const int m = m0 + r;
+                if (t < p && m < M) {
+                    const int j = idx[t];
+                    if (j >= 0 && j < K)
+                        xv = __uint_as_float(static_cast<uint32_t>(X[static_cast<int64_t>(m) * K + j]) << 16);
+                }
+                s_x[r][tt] = xv;
             }
-            s_d[r][tt] = d;
-            // activation (m0 + r, column j_t)
-            float xv = 0.f;
-            const int m = m0 + r;
-            if (t < p && m < M) {
-                const int j = idx[t];
-                if (j >= 0 && j < K)
-                    xv = __uint_as_float(static_cast<uint32_t>(X[static_cast<int64_t>(m) * K + j]) << 16);
-            }
-            s_x[r][tt] = xv;
-        }
-        __syncthreads();
+            __syncthreads();
 #pragma unroll 8
-        for (int tt = 0; tt < kFixT; ++tt) {
-            const float d = s_d[r][tt];
+            for (int tt = 0; tt < kFixT; ++tt) {
+                const float d = s_d[r][tt];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) acc[u] = fmaf(d, s_x[4 * c + u][tt], acc[u]);
+                for (int u = 0; u < 4; ++u) acc[u] = fmaf(d, s_x[4 * c + u][tt], acc[u]);
+            }
+            __syncthreads();
         }
-        __syncthreads();
-    }
-    const int i = i0 + r;
-    if (i >= N) return;
+        const int i = i0 + r;
+        if (i < N) {
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-        const int m = m0 + 4 * c + u;
-        if (m < M) Y[static_cast<int64_t>(m) * N + i] += acc[u];
+            for (int u = 0; u < 4; ++u) {
+                const int m = m0 + 4 * c + u;
+                if (m < M) Y[static_cast<int64_t>(m) * N + i] += acc[u];
+            }
+        }
     }
 }
 
@@ -215,7 +219,8 @@ bisco_status launch_q_fmt(const uint16_t *W, const bisco_layer &L, int *err, cud
 bisco_status launch_prot_fix(const bisco_layer &L, const uint16_t *X, int M, float *Y, int *err,
                              cudaStream_t stream) {
     if (L.n_protected <= 0 || M <= 0) return BISCO_OK;
-    const dim3 grid((L.n_out + kFixRows - 1) / kFixRows, (M + kFixTok - 1) / kFixTok);
+    const int tiles = (M + kFixTok - 1) / kFixTok;
+    const dim3 grid((L.n_out + kFixRows - 1) / kFixRows, tiles < 65535 ? tiles : 65535);
     k_prot_fix<<<grid, 256, 0, stream>>>(L.codes, L.norms, L.q8, L.q8_scale, L.prot_idx,
                                          L.protect_format, L.n_out, L.k_in, L.stages,
                                          L.n_protected, X, M, Y, err);
