@@ -12,7 +12,9 @@ paper's definitions can be compared bit for bit:
   Eq. 3   each stage's bits are the signs of its target (+0 and -0 code
           positive) and its norm the fp16 of the target chunk's L2 norm;
   Eq. 5-7 the next target is the previous one minus the decoded stage, with
-          the protected positions held at zero.
+          the protected positions held at zero;
+  Eq. 9   the coupled score is the gate row, up row and down column norms
+          added in that order, and protected rows take Eq. 10 per row.
 """
 import math
 
@@ -107,3 +109,54 @@ def test_product_is_linear_and_row_separable(layer, B):
     assert np.allclose(y, xd @ What.T, rtol=1e-12, atol=1e-12)
     for r in range(N):                                        # any row block alone
         assert np.array_equal(oracle.decode_rows(L, row0=r, nrows=1)[0], What[r])
+
+
+@hyp.settings(max_examples=200, deadline=None)
+@hyp.given(layers())
+def test_row_encoder_follows_the_definitions(layer):
+    """Eq. 10 on rows: the top-p rows by norm (ties to the lower index), one
+    scale per row, and the stages of the row-masked weight."""
+    Wd, S, p = layer
+    N, K = Wd.shape
+    p = min(p, N)
+    W = _bf16(Wd)
+    L = oracle.encode_rows(W, S, p)
+    norms = np.sqrt((Wd * Wd).sum(axis=1))
+    idx = np.array(sorted(sorted(range(N), key=lambda i: (-norms[i], i))[:p]), np.int32)
+    assert np.array_equal(L["idx"], idx)
+    for t, i in enumerate(idx):
+        s16 = np.float16(np.abs(Wd[i]).max() / 127.0)
+        assert L["scale"][t] == s16.view(np.uint16)
+        s = float(s16)
+        q = np.clip(np.rint(Wd[i] / s), -127, 127) if s != 0.0 else np.zeros(K)
+        assert np.array_equal(L["q8"][t, :K].astype(np.float64), q)
+    Wm = W.copy()
+    Wm[idx] = 0
+    ref = oracle.encode(Wm, S=S, p=0)
+    assert np.array_equal(L["codes"], ref["codes"]) and np.array_equal(L["norms"], ref["norms"])
+
+
+@st.composite
+def mlps(draw):
+    F = draw(st.integers(1, 12))
+    H = draw(st.integers(1, 6))
+    p = draw(st.integers(0, F))
+
+    def mat(r, c):
+        ks = draw(st.lists(st.integers(-16, 16), min_size=r * c, max_size=r * c))
+        return np.array(ks, np.float64).reshape(r, c) / 4.0
+    return mat(F, H), mat(F, H), mat(H, F), p
+
+
+@hyp.settings(max_examples=200, deadline=None)
+@hyp.given(mlps())
+def test_coupled_selection_follows_eq9(mlp):
+    """Eq. 9: gate row norm + up row norm + down column norm, added in that
+    order; the top p channels, ties to the lower index, ascending."""
+    G, U, D, p = mlp
+    F = G.shape[0]
+    idx, scores = oracle.select_coupled(_bf16(G), _bf16(U), _bf16(D), p)
+    want = (np.sqrt((G * G).sum(axis=1)) + np.sqrt((U * U).sum(axis=1))) + np.sqrt((D * D).sum(axis=0))
+    assert np.array_equal(np.asarray(scores), want)
+    top = sorted(sorted(range(F), key=lambda j: (-want[j], j))[:p])
+    assert list(idx) == top
