@@ -107,11 +107,12 @@ typedef struct {
  * (saturation).  The q8 buffer then holds FP8 bytes in the same [N][p_pad]
  * layout (E4M3: bias 7, no infinities; E5M2: bias 15).  For BF16 the
  * payload is the weight itself, scale 1.0, and the buffer is [N][p_pad]
- * uint16 (twice the bytes).  Formats other than INT8 are supported for
- * protected columns (protect_axis 0) only, else BISCO_ERR_UNSUPPORTED.
- * The decode kernels run the binary spherical stages without the protected
- * set and then replace each protected column's decoded value by
- * scale * value(q) in a second kernel.
+ * uint16 (twice the bytes).  On protected rows (protect_axis 1) the same
+ * per-channel rules apply with the row as the channel: q [p][kp] elements
+ * of the format, one scale per row.  The decode kernels run the binary
+ * spherical stages without the protected set and then, in a second kernel,
+ * replace each protected column's decoded value by scale * value(q) (or
+ * overwrite each protected row).
  */
 #define BISCO_PROT_INT8 0
 #define BISCO_PROT_E4M3 1
@@ -137,8 +138,8 @@ bisco_status bisco_encoded_sizes(int32_t N, int32_t K, int32_t d, int32_t S,
 /*
  * Byte sizes of the five buffers of the layer *L describes (its sizes,
  * protect_axis and protect_format; the pointers are not read): the q8
- * buffer is N * p_pad bytes for columns (twice that for BF16) and
- * p * roundup(K, 16) bytes for rows.  INVALID_ARG or UNSUPPORTED as for the
+ * buffer is N * p_pad elements for columns and p * roundup(K, 16) for
+ * rows, of 1 byte (INT8, FP8) or 2 (BF16).  INVALID_ARG or UNSUPPORTED as for the
  * decode calls.  Host-only.
  */
 bisco_status bisco_layer_sizes(const bisco_layer *L, size_t out_bytes[5]);

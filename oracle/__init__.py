@@ -19,10 +19,10 @@ Functions and the paper passages they follow:
                             channel score (Sec. III-E Eq. 9) with Eq. 10 on
                             rows; the CUDA library does not take this axis yet
 * :func:`double_to_fp8`, :func:`fp8_to_double`, :func:`quantize_protected_fmt`,
-  :func:`protected_values_fmt`
+  :func:`quantize_protected_rows_fmt`, :func:`protected_values_fmt`
                             FP8 E4M3 / E5M2 and BF16 protected payloads (the
                             paper's protected-format ablation) as variants of
-                            Eq. 10; not taken by the CUDA library yet
+                            Eq. 10, on protected columns or rows
 * :func:`decoder_table_linear`, :func:`decoder_table_mlp`, :func:`decode_rows_table`
                             the decoder step of Eq. 1 as a table over the 256
                             code bytes (linear, or odd tanh perceptron with an
@@ -383,6 +383,22 @@ def quantize_protected_fmt(W_bits, idx, fmt):
     if rc:
         raise OracleError(rc)
     return q[:, :pad16(p)].copy(), scale[:p].copy()
+
+
+def quantize_protected_rows_fmt(W_bits, idx, fmt):
+    """Eq. 10 on protected output rows with the payload in format ``fmt``
+    (the row axis of Eq. 9 under the protected-format ablation): row i of W
+    is column i of W^T, so this is :func:`quantize_protected_fmt` on the
+    transpose.  Returns (q [p][pad16(K)], scale uint16[p]); one scale per
+    row, zero padding past K."""
+    W_bits = _c(W_bits, np.uint16)
+    N, K = W_bits.shape
+    idx = _c(idx, np.int32)
+    p = len(idx)
+    qt, scale = quantize_protected_fmt(np.ascontiguousarray(W_bits.T), idx, fmt)
+    q = np.zeros((p, pad16(K)), qt.dtype)
+    q[:, :K] = qt[:, :p].T
+    return q, scale
 
 
 def protected_values_fmt(q, scale, fmt):

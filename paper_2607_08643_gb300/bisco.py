@@ -178,11 +178,11 @@ class Layer:
         dev = torch.device(device)
         self.codes = torch.empty((S, N, K // 8), dtype=torch.uint8, device=dev)
         self.norms = torch.empty((S, N, K // 8), dtype=torch.int16, device=dev)
+        qdt = {PROT_INT8: torch.int8, PROT_E4M3: torch.uint8, PROT_E5M2: torch.uint8,
+               PROT_BF16: torch.int16}[fmt]
         if axis == 1:
-            self.q8 = torch.empty((max(p, 1), self.kp), dtype=torch.int8, device=dev)
+            self.q8 = torch.empty((max(p, 1), self.kp), dtype=qdt, device=dev)
         else:
-            qdt = {PROT_INT8: torch.int8, PROT_E4M3: torch.uint8, PROT_E5M2: torch.uint8,
-                   PROT_BF16: torch.int16}[fmt]
             self.q8 = torch.empty((N, max(self.p_pad, 16)), dtype=qdt, device=dev)
         self.scale = torch.empty((max(p, 8),), dtype=torch.int16, device=dev)
         self.idx = torch.empty((max(p, 4),), dtype=torch.int32, device=dev)
@@ -210,8 +210,8 @@ class Layer:
             L["q8"] = self.q8[:p].cpu().numpy()
         else:
             L["q8"] = self.q8[:, :self.p_pad].cpu().numpy()
-            if self.fmt == PROT_BF16:
-                L["q8"] = L["q8"].view("uint16")
+        if self.fmt == PROT_BF16:
+            L["q8"] = L["q8"].view("uint16")
         if self.fmt != PROT_INT8:
             L["fmt"] = self.fmt
         return L
@@ -264,15 +264,16 @@ def bisco_encode(W_bits, S, p, g=None, workspace=None, stream=None, axis=0,
     return L
 
 
-def bisco_encode_with_set(W_bits, S, idx, axis, workspace=None, stream=None) -> Layer:
+def bisco_encode_with_set(W_bits, S, idx, axis, workspace=None, stream=None,
+                          fmt=PROT_INT8) -> Layer:
     """Encodes with the protected set given (device int32 [p], ascending):
-    columns for axis 0, rows for axis 1."""
+    columns for axis 0, rows for axis 1; fmt is the payload's format."""
     import torch
     W_bits = _bits2d(W_bits)
     N, K = W_bits.shape
     p = int(idx.numel())
     assert idx.dtype == torch.int32 and idx.is_cuda and idx.is_contiguous()
-    L = Layer(N, K, S, p, W_bits.device, axis=axis)
+    L = Layer(N, K, S, p, W_bits.device, axis=axis, fmt=fmt)
     need = bisco_encode_workspace_bytes_axis(N, K, axis)
     if workspace is None:
         workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=W_bits.device)

@@ -42,7 +42,6 @@ bisco_status check_layer(const bisco_layer *L, bool check_buffers) {
     if (L->protect_format < BISCO_PROT_INT8 || L->protect_format > BISCO_PROT_BF16)
         return BISCO_ERR_INVALID_ARG;
     if (L->chunk_dim != 8) return BISCO_ERR_UNSUPPORTED;
-    if (L->protect_format != BISCO_PROT_INT8 && L->protect_axis != 0) return BISCO_ERR_UNSUPPORTED;
     if (static_cast<int64_t>(L->n_out) * L->k_in > (int64_t(1) << 40)) return BISCO_ERR_INVALID_ARG;
     if (!check_buffers) return BISCO_OK;
     if (!L->codes || !L->norms || !aligned16(L->codes) || !aligned16(L->norms))
@@ -193,10 +192,11 @@ bisco_status bisco_layer_sizes(const bisco_layer *L, size_t out_bytes[5]) {
     const size_t C = K / 8;
     out_bytes[0] = S * N * C;
     out_bytes[1] = S * N * C * 2;
+    const size_t elem = L->protect_format == BISCO_PROT_BF16 ? 2 : 1;
     if (L->protect_axis == 1)
-        out_bytes[2] = p * ((K + 15) / 16 * 16);
+        out_bytes[2] = p * ((K + 15) / 16 * 16) * elem;
     else
-        out_bytes[2] = N * ((p + 15) / 16 * 16) * (L->protect_format == BISCO_PROT_BF16 ? 2 : 1);
+        out_bytes[2] = N * ((p + 15) / 16 * 16) * elem;
     out_bytes[3] = p * 2;
     out_bytes[4] = p * 4;
     return BISCO_OK;

@@ -48,6 +48,8 @@ bisco_status launch_rows_dense(const bisco_layer &L, void *out, int dtype, int *
 // quantiser, the correction after the stage-only decode kernels, and the
 // dense overwrite.
 bisco_status launch_q_fmt(const uint16_t *W, const bisco_layer &L, int *err, cudaStream_t stream);
+bisco_status launch_q_fmt_rows(const uint16_t *W, const bisco_layer &L, int *err,
+                               cudaStream_t stream);
 bisco_status launch_prot_fix(const bisco_layer &L, const uint16_t *X, int M, float *Y, int *err,
                              cudaStream_t stream);
 bisco_status launch_dense_fmt(const bisco_layer &L, void *out, int dtype, int *err,

@@ -410,7 +410,11 @@ bisco_status launch_encode_rows(const uint16_t *W, const float *g, const bisco_l
     k_rowscore<<<(N + 127) / 128, 128, 0, stream>>>(W, g, N, K, score, err);
     k_rank<<<(N + kRankThreads - 1) / kRankThreads, kRankThreads, 0, stream>>>(score, N, p, rank);
     k_compact<<<1, kCompactThreads, 0, stream>>>(rank, N, p, prot, L.prot_idx);
-    if (p > 0) k_q8_rows<<<p, 256, 0, stream>>>(W, N, K, kp, L.prot_idx, L.q8, L.q8_scale, err);
+    if (L.protect_format != BISCO_PROT_INT8) {
+        if (launch_q_fmt_rows(W, L, err, stream) != BISCO_OK) return BISCO_ERR_CUDA;
+    } else if (p > 0) {
+        k_q8_rows<<<p, 256, 0, stream>>>(W, N, K, kp, L.prot_idx, L.q8, L.q8_scale, err);
+    }
     const int64_t chunks = static_cast<int64_t>(N) * (K / 8);
     k_stages<true><<<static_cast<unsigned>((chunks + 255) / 256), 256, 0, stream>>>(
         W, N, K, S, prot, L.codes, L.norms, err);
@@ -433,7 +437,11 @@ bisco_status launch_encode_with_set(const uint16_t *W, const int32_t *idx_in,
     const unsigned sgrid = static_cast<unsigned>((chunks + 255) / 256);
     if (rows) {
         const int kp = (K + 15) / 16 * 16;
-        if (p > 0) k_q8_rows<<<p, 256, 0, stream>>>(W, N, K, kp, L.prot_idx, L.q8, L.q8_scale, err);
+        if (L.protect_format != BISCO_PROT_INT8) {
+            if (launch_q_fmt_rows(W, L, err, stream) != BISCO_OK) return BISCO_ERR_CUDA;
+        } else if (p > 0) {
+            k_q8_rows<<<p, 256, 0, stream>>>(W, N, K, kp, L.prot_idx, L.q8, L.q8_scale, err);
+        }
         k_stages<true><<<sgrid, 256, 0, stream>>>(W, N, K, S, prot, L.codes, L.norms, err);
     } else {
         const int p_pad = (p + 15) / 16 * 16;

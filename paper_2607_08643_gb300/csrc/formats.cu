@@ -91,6 +91,50 @@ __global__ void __launch_bounds__(256) k_q_fmt(const uint16_t *__restrict__ W, i
     }
 }
 
+// Encoder on protected output rows: one CTA per protected row t < p, one
+// scale per row (the row is the protected channel), q [p][kp] with
+// kp = roundup(K, 16) and zero padding past K.
+__global__ void __launch_bounds__(256) k_q_fmt_rows(const uint16_t *__restrict__ W, int N, int K,
+                                                    int kp, const int32_t *__restrict__ idx,
+                                                    int fmt, void *__restrict__ q,
+                                                    uint16_t *__restrict__ scale, int *err) {
+    const int t = blockIdx.x;
+    const int i = idx[t];
+    uint8_t *q8 = static_cast<uint8_t *>(q) + static_cast<int64_t>(t) * kp;
+    uint16_t *q16 = static_cast<uint16_t *>(q) + static_cast<int64_t>(t) * kp;
+    if (i < 0 || i >= N) {   // only after a latched k_set_map error
+        for (int k = threadIdx.x; k < kp; k += blockDim.x) {
+            if (fmt == BISCO_PROT_BF16) q16[k] = 0; else q8[k] = 0;
+        }
+        return;
+    }
+    const uint16_t *wrow = W + static_cast<int64_t>(i) * K;
+    if (fmt == BISCO_PROT_BF16) {
+        if (threadIdx.x == 0) scale[t] = 0x3C00u;   // 1.0
+        for (int k = threadIdx.x; k < kp; k += blockDim.x) q16[k] = k < K ? wrow[k] : 0;
+        return;
+    }
+    const Fp8Format f = fp8_format(fmt);
+    double m = 0.0;
+    for (int k = threadIdx.x; k < K; k += blockDim.x) m = fmax(m, fabs(bf16_to_f64(wrow[k])));
+    __shared__ double red[256];
+    red[threadIdx.x] = m;
+    __syncthreads();
+    for (int w = 128; w > 0; w >>= 1) {
+        if (threadIdx.x < w) red[threadIdx.x] = fmax(red[threadIdx.x], red[threadIdx.x + w]);
+        __syncthreads();
+    }
+    const uint16_t s16 = f64_to_f16_rn(__ddiv_rn(red[0], f.maxf));
+    if ((s16 & 0x7C00u) == 0x7C00u) {
+        if (threadIdx.x == 0) latch_error(err, BISCO_ERR_RANGE);
+        return;
+    }
+    if (threadIdx.x == 0) scale[t] = s16;
+    const double s = f16_to_f64(s16);
+    for (int k = threadIdx.x; k < kp; k += blockDim.x)
+        q8[k] = (k < K && s != 0.0) ? f64_to_fp8(__ddiv_rn(bf16_to_f64(wrow[k]), s), f) : 0;
+}
+
 constexpr int kFixRows = 32, kFixTok = 32, kFixT = 32;
 
 // The correction of the decode kernels' output, for a tile of 32 output
@@ -213,6 +257,15 @@ bisco_status launch_q_fmt(const uint16_t *W, const bisco_layer &L, int *err, cud
     if (p_pad == 0) return BISCO_OK;
     k_q_fmt<<<p_pad, 256, 0, stream>>>(W, L.n_out, L.k_in, p, p_pad, L.prot_idx, L.protect_format,
                                        L.q8, L.q8_scale, err);
+    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+}
+
+bisco_status launch_q_fmt_rows(const uint16_t *W, const bisco_layer &L, int *err,
+                               cudaStream_t stream) {
+    if (L.n_protected <= 0) return BISCO_OK;
+    const int kp = (L.k_in + 15) / 16 * 16;
+    k_q_fmt_rows<<<L.n_protected, 256, 0, stream>>>(W, L.n_out, L.k_in, kp, L.prot_idx,
+                                                    L.protect_format, L.q8, L.q8_scale, err);
     return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
 }
 

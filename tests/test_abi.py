@@ -226,7 +226,9 @@ def test_layer_sizes_match_oracle_layouts(lib):
     assert f(c(chunk_dim=16), out) == bisco.ERR_UNSUPPORTED
     assert f(c(protect_format=4), out) == bisco.ERR_INVALID_ARG
     assert f(c(protect_format=-1), out) == bisco.ERR_INVALID_ARG
-    assert f(c(protect_format=1, protect_axis=1), out) == bisco.ERR_UNSUPPORTED  # FP8 rows
+    assert f(c(protect_format=1, protect_axis=1), out) == bisco.OK               # FP8 rows
+    f(c(protect_format=3, protect_axis=1, n_protected=5), out)                   # BF16 rows
+    assert out[2] == 5 * 64 * 2
     assert f(c(), None) == bisco.ERR_INVALID_ARG
     assert f(None, out) == bisco.ERR_INVALID_ARG
 
@@ -239,8 +241,6 @@ def test_protect_format_validation_before_any_device_call(lib):
         assert lib.bisco_gemv(ctypes.byref(L), x, 1, y, None) == code
         assert lib.bisco_gemm(ctypes.byref(L), x, 4, y, None, 0, None) == code
         assert lib.bisco_decode_dense(ctypes.byref(L), y, bisco.DENSE_F32, None) == code
-    L = _fake_layer(protect_format=bisco.PROT_E4M3, protect_axis=1)
-    assert lib.bisco_gemv(ctypes.byref(L), x, 1, y, None) == bisco.ERR_UNSUPPORTED
     for fmt in (bisco.PROT_E4M3, bisco.PROT_E5M2, bisco.PROT_BF16):       # tables: INT8 only
         L = _fake_layer(protect_format=fmt)
         assert lib.bisco_gemv_table(ctypes.byref(L), tab, x, 1, y, None) == bisco.ERR_UNSUPPORTED
@@ -344,7 +344,8 @@ def test_struct_layout_matches_the_header(tmp_path):
 
 
 @pytest.mark.parametrize("axis,fmt", [(0, bisco.PROT_INT8), (0, bisco.PROT_E4M3), (0, bisco.PROT_E5M2),
-                                      (0, bisco.PROT_BF16), (1, bisco.PROT_INT8)])
+                                      (0, bisco.PROT_BF16), (1, bisco.PROT_INT8), (1, bisco.PROT_E4M3),
+                                      (1, bisco.PROT_BF16)])
 def test_layer_marshalling_round_trip(lib, axis, fmt):
     """Layer.from_numpy / to_numpy carry the oracle's layer dicts exactly for
     every protection axis and payload format (host tensors; no device call),
@@ -354,6 +355,9 @@ def test_layer_marshalling_round_trip(lib, axis, fmt):
     W = synth.layer_weights(N, K, seed=5)
     if axis == 1:
         ref = oracle.encode_rows(W, S, p)
+        if fmt != bisco.PROT_INT8:
+            q, scale = oracle.quantize_protected_rows_fmt(W, ref["idx"], fmt)
+            ref = dict(ref, q8=q, scale=scale, fmt=fmt)
     else:
         ref = oracle.encode(W, S=S, p=p)
         if fmt != bisco.PROT_INT8:

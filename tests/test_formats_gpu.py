@@ -1,7 +1,8 @@
 """Protected payloads in FP8 E4M3, FP8 E5M2 and BF16 on the GPU (the
 protected-format ablation, variants of Eq. 10) against the fp64 oracle:
 the encoder's bytes bit for bit, and GEMV / GEMM / dense decode with the
-protected columns replaced by scale * value(q), within the 2e-3 bar."""
+protected columns replaced by scale * value(q) -- or the protected rows
+overwritten (Eq. 9's row axis) -- within the 2e-3 bar."""
 import numpy as np
 import pytest
 
@@ -134,3 +135,60 @@ def test_full_size_q_proj_e4m3_sampled(env):
                                                          q8=ref["q8"][r:r + 1], N=1)), x)[:, 0]
                          for r in rows], axis=1)
         assert max_rel_rows(y.cpu().numpy()[:, rows], want) <= TOL
+
+
+def oracle_rows_layer(W, S, p, fmt, idx=None):
+    L = oracle.encode_rows(W, S, p, idx=idx)
+    q, scale = oracle.quantize_protected_rows_fmt(W, L["idx"], fmt)
+    return dict(L, q8=q, scale=scale, fmt=fmt)
+
+
+def oracle_rows_dense(L):
+    """Stages of the row-masked weight, protected rows = scale * value(q)."""
+    N, K, p = L["N"], L["K"], L["p"]
+    base = dict(L, p=0, axis=0, q8=np.zeros((N, 0), np.int8), scale=np.zeros(0, np.uint16),
+                idx=np.zeros(0, np.int32))
+    What = oracle.decode_rows(base)
+    if p:
+        qc = np.zeros((K, oracle.pad16(p)), L["q8"].dtype)        # rows as protected columns
+        qc[:, :p] = L["q8"][:, :K].T
+        What[L["idx"]] = oracle.protected_values_fmt(qc, L["scale"], L["fmt"]).T
+    return What
+
+
+@pytest.mark.parametrize("fmt", FORMATS)
+def test_encode_rows_formats_bit_exact(env, fmt):
+    import torch
+    bisco, dev = env
+    for (N, K, S, p, seed) in ((300, 1024, 2, 3, 1), (64, 136, 3, 5, 2)):
+        W = synth.layer_weights(N, K, seed=seed)
+        Wd = to_dev(W, dev)
+        L = bisco.bisco_encode(Wd, S, p, axis=1, fmt=fmt)
+        idx = torch.tensor([1, 7, N - 1], dtype=torch.int32, device=dev)
+        Lg = bisco.bisco_encode_with_set(Wd, S, idx, axis=1, fmt=fmt)
+        torch.cuda.synchronize()
+        assert bisco.bisco_get_device_error() == 0
+        for got, ref in ((L.to_numpy(), oracle_rows_layer(W, S, p, fmt)),
+                         (Lg.to_numpy(), oracle_rows_layer(W, S, 3, fmt, idx=[1, 7, N - 1]))):
+            for k in ("codes", "norms", "q8", "scale", "idx"):
+                assert got[k].dtype == ref[k].dtype and np.array_equal(got[k], ref[k]), k
+
+
+@pytest.mark.parametrize("fmt", FORMATS)
+def test_gemv_gemm_rows_formats_match_oracle(env, fmt):
+    import torch
+    bisco, dev = env
+    N, K = 512, 1024
+    ref = oracle_rows_layer(synth.layer_weights(N, K, seed=61), 2, 6, fmt)
+    L = bisco.Layer.from_numpy(ref, dev)
+    What = oracle_rows_dense(ref)
+    for M in (1, 16, 300):
+        X = synth.activations(M, K, seed=62 + M)
+        Y = bisco.bisco_gemv(L, to_dev(X, dev)) if M <= 16 else bisco.bisco_gemm(L, to_dev(X, dev))
+        torch.cuda.synchronize()
+        assert bisco.bisco_get_device_error() == 0
+        assert max_rel_rows(Y.cpu().numpy(), oracle.matmul(What, X)) <= TOL
+    out = bisco.bisco_decode_dense(L, "f32")
+    torch.cuda.synchronize()
+    got = out.cpu().numpy().astype(np.float64)
+    assert np.array_equal(got[ref["idx"]], What[ref["idx"]])     # scale * value(q): exact in fp32

@@ -863,3 +863,36 @@ def test_encode_with_given_columns_reduces_to_eq8_encode():
         oracle.encode_given(W, 2, np.array([5, 3], np.int32))        # not ascending
     with pytest.raises(oracle.OracleError):
         oracle.encode_given(W, 2, np.array([136], np.int32))         # out of range
+
+
+@pytest.mark.parametrize("fmt", [oracle.FMT_INT8, oracle.FMT_E4M3, oracle.FMT_E5M2, oracle.FMT_BF16])
+def test_row_quantiser_in_every_format(fmt):
+    """Eq. 10 on rows in any payload format: INT8 equals the row encoder's
+    own quantiser (or_quantize_protected_rows) byte for byte; every format
+    keeps one scale per row with the format's closed form, and the decoded
+    rows are within half a step of the weights."""
+    N, K = 40, 136
+    W = synth.layer_weights(N, K, seed=111)
+    idx = np.array([3, 17, 39], np.int32)
+    q, scale = oracle.quantize_protected_rows_fmt(W, idx, fmt)
+    assert q.shape == (3, oracle.pad16(K)) and not q[:, K:].any()
+    if fmt == oracle.FMT_INT8:
+        L = oracle.encode_rows(W, 2, 3, idx=idx)
+        assert np.array_equal(q, L["q8"]) and np.array_equal(scale, L["scale"])
+    fw = f64(W)[idx]
+    F = {oracle.FMT_INT8: 127.0, oracle.FMT_E4M3: 448.0, oracle.FMT_E5M2: 57344.0}
+    if fmt == oracle.FMT_BF16:
+        assert np.all(scale == 0x3C00) and np.array_equal(q[:, :K], W[idx])
+    else:
+        s16 = (np.abs(fw).max(axis=1) / F[fmt]).astype(np.float16)
+        assert np.array_equal(scale, s16.view(np.uint16))
+    qc = np.zeros((K, oracle.pad16(3)), q.dtype)                       # as protected columns
+    qc[:, :3] = q[:, :K].T
+    vals = oracle.protected_values_fmt(qc, scale, fmt).T                  # [p][K]
+    sd = scale.view(np.float16).astype(np.float64)[:, None]
+    rel = {oracle.FMT_INT8: None, oracle.FMT_E4M3: 2.0 ** -4, oracle.FMT_E5M2: 2.0 ** -3,
+           oracle.FMT_BF16: 0.0}[fmt]
+    if rel is None:
+        assert np.all(np.abs(vals - fw) <= sd / 2 * (1 + 1e-12))
+    else:
+        assert np.all(np.abs(vals - fw) <= rel * np.abs(fw) + sd * 2.0 ** -9)
