@@ -330,7 +330,8 @@ bisco_status bisco_decode_dense(const bisco_layer *L, void *out, int32_t dtype,
  * bisco_decode_dense_table: What as a dense [N][K] fp32 / bf16 / fp16
  * matrix (BISCO_DENSE_*), rounded once from fp32.
  * Arguments and errors are otherwise those of bisco_gemv and
- * bisco_decode_dense.
+ * bisco_decode_dense; protected columns need the INT8 payload
+ * (BISCO_ERR_UNSUPPORTED otherwise), protected rows take any format.
  */
 bisco_status bisco_gemv_table(const bisco_layer *L, const uint16_t *tables, const uint16_t *x_bf16,
                               int32_t B, float *y, bisco_stream_t stream);

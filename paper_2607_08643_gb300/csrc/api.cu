@@ -365,7 +365,9 @@ bisco_status bisco_gemv_table(const bisco_layer *L, const uint16_t *tables, cons
                               int32_t B, float *y, bisco_stream_t stream) {
     bisco_status st = check_layer(L, true);
     if (st != BISCO_OK) return st;
-    if (L->protect_format != BISCO_PROT_INT8) return BISCO_ERR_UNSUPPORTED;
+    // a column payload other than INT8 is corrected against the identity
+    // decoder's stage value (formats.cu), not a table's: rows only
+    if (L->protect_format != BISCO_PROT_INT8 && L->protect_axis == 0) return BISCO_ERR_UNSUPPORTED;
     if (B < 0 || B > 16) return BISCO_ERR_INVALID_ARG;
     if (!tables || !aligned16(tables)) return BISCO_ERR_INVALID_ARG;
     if (B == 0) return BISCO_OK;
@@ -385,7 +387,7 @@ bisco_status bisco_decode_dense_table(const bisco_layer *L, const uint16_t *tabl
                                       int32_t dtype, bisco_stream_t stream) {
     bisco_status st = check_layer(L, true);
     if (st != BISCO_OK) return st;
-    if (L->protect_format != BISCO_PROT_INT8) return BISCO_ERR_UNSUPPORTED;
+    if (L->protect_format != BISCO_PROT_INT8 && L->protect_axis == 0) return BISCO_ERR_UNSUPPORTED;
     if (dtype != BISCO_DENSE_F32 && dtype != BISCO_DENSE_BF16 && dtype != BISCO_DENSE_F16)
         return BISCO_ERR_INVALID_ARG;
     if (!tables || !aligned16(tables) || !out || !aligned16(out)) return BISCO_ERR_INVALID_ARG;
