@@ -17,15 +17,15 @@
 
 #include "bisco_dev.cuh"
 #include "bisco_host.h"
+#include "convert.cuh"
 
 namespace bisco {
 namespace {
 
 constexpr int kTableEntries = 256 * 8;   // halves per stage
 
-__device__ __forceinline__ float bf16_to_f32(uint16_t b) {
-    return __uint_as_float(static_cast<uint32_t>(b) << 16);
-}
+using cvt::bf16_to_f32;
+using cvt::from_f32;
 
 // Stages S tables into shared memory (S * 4 KB, 16-byte copies).
 __device__ __forceinline__ void stage_tables(const uint16_t *__restrict__ tables, int S,
@@ -237,15 +237,6 @@ __global__ void __launch_bounds__(256) k_gemv_table_v(const uint8_t *__restrict_
             if (b < B) y[static_cast<int64_t>(b) * N + i] = acc[b];
     }
 }
-
-template <typename T>
-__device__ __forceinline__ T from_f32(float v);
-template <>
-__device__ __forceinline__ float from_f32<float>(float v) { return v; }
-template <>
-__device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
-template <>
-__device__ __forceinline__ __half from_f32<__half>(float v) { return __float2half_rn(v); }
 
 // Dense decode with a decoder table: one thread per chunk.
 template <typename T>

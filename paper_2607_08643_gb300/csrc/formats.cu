@@ -19,24 +19,16 @@
 
 #include "bisco_dev.cuh"
 #include "bisco_host.h"
+#include "convert.cuh"
 #include "fp8.cuh"
 
 namespace bisco {
 namespace {
 
-__device__ __forceinline__ uint16_t f64_to_f16_rn(double x) {
-    unsigned short r;
-    asm("cvt.rn.f16.f64 %0, %1;" : "=h"(r) : "d"(x));
-    return r;
-}
-
-__device__ __forceinline__ double f16_to_f64(uint16_t h) {
-    return static_cast<double>(__half2float(__ushort_as_half(h)));
-}
-
-__device__ __forceinline__ double bf16_to_f64(uint16_t b) {
-    return static_cast<double>(__uint_as_float(static_cast<uint32_t>(b) << 16));
-}
+using cvt::bf16_to_f64;
+using cvt::f16_to_f64;
+using cvt::f64_to_f16_rn;
+using cvt::from_f32;
 
 // The value of a protected payload element (exact in fp32).
 __device__ __forceinline__ float payload_value(const void *q, int64_t e, int fmt) {
@@ -212,15 +204,6 @@ __global__ void __launch_bounds__(256) k_prot_fix(const uint8_t *__restrict__ co
         }
     }
 }
-
-template <typename T>
-__device__ __forceinline__ T from_f32(float v);
-template <>
-__device__ __forceinline__ float from_f32<float>(float v) { return v; }
-template <>
-__device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
-template <>
-__device__ __forceinline__ __half from_f32<__half>(float v) { return __float2half_rn(v); }
 
 // Dense decode: out[i][idx[u]] = scale_u * value(q[i][u]), one thread per (i, u).
 template <typename T>

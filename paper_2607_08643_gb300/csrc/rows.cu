@@ -16,6 +16,7 @@
 
 #include "bisco_dev.cuh"
 #include "bisco_host.h"
+#include "convert.cuh"
 #include "fp8.cuh"
 
 namespace bisco {
@@ -23,8 +24,9 @@ namespace {
 
 constexpr int kRowWarps = 8;
 
-__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+using cvt::bf16_hi;
+using cvt::bf16_lo;
+using cvt::from_f32;
 
 // Eight consecutive payload elements of a protected row, from element `off`
 // (a multiple of 8): INT8 and FP8 are one 8-byte load, BF16 one 16-byte
@@ -132,15 +134,6 @@ __global__ void __launch_bounds__(32 * kRowWarps) k_rows_apply(
         }
     }
 }
-
-template <typename T>
-__device__ __forceinline__ T from_f32(float v);
-template <>
-__device__ __forceinline__ float from_f32<float>(float v) { return v; }
-template <>
-__device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
-template <>
-__device__ __forceinline__ __half from_f32<__half>(float v) { return __float2half_rn(v); }
 
 // Dense protected rows, one CTA per row t: out[idx[t]][k] = scale[t] * value(q8[t][k])
 // (exact in fp32, rounded once to the output type).
