@@ -822,7 +822,9 @@ def run_variants(args, local_rank):
     variant, CUDA events over `steps` replays; GB/s on each variant's own
     compressed bytes (the decoder tables, 8 KB per layer, are not counted).
     Then the gated MLP of the same layers (gate/up grouped, down) with
-    per-layer INT8 columns and with the coupled set of Eq. 9."""
+    per-layer INT8 columns and with the coupled set of Eq. 9, and the
+    prefill GEMM of q_proj-shaped layers per variant (its epilogue kernels
+    included)."""
     import torch
     from paper_2607_08643_gb300 import bisco, synth
     dev = torch.device("cuda", local_rank)
@@ -943,9 +945,57 @@ def run_variants(args, local_rank):
                     "frac_of_hbm": gbs / peak, "tokens_per_s": B / (ms * 1e-3)})
         del layers, ys, gr
         torch.cuda.empty_cache()
+    # prefill: bisco_gemm on 8 distinct q_proj-shaped layers per variant at
+    # --prefill-tokens, the variants' epilogue kernels included
+    M = args.prefill_tokens
+    Xp = torch.randn((M, 4096), generator=gen, device=dev).to(torch.bfloat16).view(torch.int16)
+    tf_burst, _, _ = tensor_peaks()
+    pre = []
+    for name, axis, fmt in (("int8 columns", 0, bisco.PROT_INT8),
+                            ("fp8 e4m3 columns", 0, bisco.PROT_E4M3),
+                            ("int8 rows", 1, bisco.PROT_INT8)):
+        layers = []
+        for l in range(8):
+            W = synth.layer_weights_torch(4096, 4096, seed=5000 + l, device=dev)
+            layers.append(bisco.bisco_encode(W, S_STAGES, synth.protected_count(4096, RHO_PCT),
+                                             axis=axis, fmt=fmt))
+            del W
+        need = max(bisco.bisco_gemm_workspace_bytes(L, M) for L in layers)
+        gws = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+        Y = torch.empty((M, 4096), device=dev)
+        torch.cuda.synchronize()
+
+        def step():
+            for L in layers:
+                bisco.bisco_gemm(L, Xp, Y=Y, workspace=gws, stream=stream)
+
+        with torch.cuda.stream(stream):
+            step()
+            torch.cuda.synchronize()
+            gp = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gp, stream=stream):
+                step()
+        torch.cuda.synchronize()
+        for _ in range(max(args.warmup, 3)):
+            gp.replay()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(args.steps):
+                gp.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        if bisco.bisco_get_device_error(stream) != bisco.OK:
+            raise RuntimeError("device error in prefill variant " + name)
+        us = e0.elapsed_time(e1) * 1e3 / (args.steps * len(layers))
+        tflops = 2.0 * M * 4096 * 4096 / (us * 1e-6) / 1e12
+        pre.append({"variant": name, "tokens": M, "us_per_layer": us, "tflops": tflops,
+                    "frac_of_tensor_burst": tflops / tf_burst})
+        del layers, gws, Y, gp
+        torch.cuda.empty_cache()
     return {"metric": "decode step per protected-set / decoder variant", "unit": "GB/s",
             "batch": B, "layers": args.layers, "hbm_peak_gbs": peak, "peak_source": peak_kind,
-            "variants": out, "mlp_variants": mlp}
+            "variants": out, "mlp_variants": mlp, "prefill_q_proj": pre}
 
 
 # ------------------------------------------------------------ CPU oracle
