@@ -47,6 +47,7 @@ def example():
 
 
 if __name__ == "__main__":
-    with open(os.path.join(HERE, "oracle_small_layer.json"), "w") as f:
-        json.dump(example(), f, indent=0)
-        f.write("\n")
+    g = example()
+    with open(os.path.join(HERE, "oracle_small_layer.json"), "w") as f:   # one key per line
+        f.write("{\n" + ",\n".join("%s: %s" % (json.dumps(k), json.dumps(v)) for k, v in g.items())
+                + "\n}\n")
