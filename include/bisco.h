@@ -91,7 +91,7 @@ typedef struct {
     int32_t protect_axis; /* 0 = input columns; 1 = output rows            */
     uint8_t *codes;
     uint16_t *norms;
-    int8_t *q8;
+    int8_t *q8;           /* the protected payload, in protect_format      */
     uint16_t *q8_scale;
     int32_t *prot_idx;
     int32_t protect_format; /* BISCO_PROT_*: the protected payload's type */
@@ -139,8 +139,8 @@ bisco_status bisco_encoded_sizes(int32_t N, int32_t K, int32_t d, int32_t S,
  * Byte sizes of the five buffers of the layer *L describes (its sizes,
  * protect_axis and protect_format; the pointers are not read): the q8
  * buffer is N * p_pad elements for columns and p * roundup(K, 16) for
- * rows, of 1 byte (INT8, FP8) or 2 (BF16).  INVALID_ARG or UNSUPPORTED as for the
- * decode calls.  Host-only.
+ * rows, of 1 byte (INT8, FP8) or 2 (BF16).  INVALID_ARG or UNSUPPORTED
+ * as for the decode calls.  Host-only.
  */
 bisco_status bisco_layer_sizes(const bisco_layer *L, size_t out_bytes[5]);
 
