@@ -230,8 +230,11 @@ bisco_status bisco_select_coupled(const uint16_t *Wg_bf16, const uint16_t *Wu_bf
  * the array's device address (cudaGetSymbolAddress) with that device
  * current; make that first call before any stream capture.  All calls share
  * the one array, so calls that overlap on the GPU race and must be
- * serialised by the caller.  Arguments, outputs and errors are otherwise
- * those of bisco_encode.
+ * serialised by the caller.  It takes input-column protection with INT8
+ * payloads only: protect_axis = 1 or another protect_format returns
+ * BISCO_ERR_UNSUPPORTED.  It validates the layer as bisco_encode does
+ * (the same BISCO_ERR_INVALID_ARG cases), and its outputs and device
+ * errors are those of bisco_encode.
  */
 #define BISCO_ENCODE_NOALLOC_MAX_K 32768
 bisco_status bisco_encode_noalloc(const uint16_t *W_bf16, const float *g, const bisco_layer *L,

@@ -31,28 +31,6 @@ int current_device() {
     return d;
 }
 
-// Validates the sizes of a layer; buffers too when check_buffers.
-bisco_status check_layer(const bisco_layer *L, bool check_buffers) {
-    if (!L) return BISCO_ERR_INVALID_ARG;
-    if (L->n_out < 1 || L->k_in < 8 || L->k_in % 8 != 0) return BISCO_ERR_INVALID_ARG;
-    if (L->stages < 1 || L->stages > 3) return BISCO_ERR_INVALID_ARG;
-    if (L->protect_axis != 0 && L->protect_axis != 1) return BISCO_ERR_INVALID_ARG;
-    const int32_t p_max = L->protect_axis == 1 ? L->n_out : L->k_in;
-    if (L->n_protected < 0 || L->n_protected > p_max) return BISCO_ERR_INVALID_ARG;
-    if (L->protect_format < BISCO_PROT_INT8 || L->protect_format > BISCO_PROT_BF16)
-        return BISCO_ERR_INVALID_ARG;
-    if (L->chunk_dim != 8) return BISCO_ERR_UNSUPPORTED;
-    if (static_cast<int64_t>(L->n_out) * L->k_in > (int64_t(1) << 40)) return BISCO_ERR_INVALID_ARG;
-    if (!check_buffers) return BISCO_OK;
-    if (!L->codes || !L->norms || !aligned16(L->codes) || !aligned16(L->norms))
-        return BISCO_ERR_INVALID_ARG;
-    if (L->n_protected > 0) {
-        if (!L->q8 || !L->q8_scale || !L->prot_idx) return BISCO_ERR_INVALID_ARG;
-        if (!aligned16(L->q8) || !aligned16(L->q8_scale) || !aligned16(L->prot_idx))
-            return BISCO_ERR_INVALID_ARG;
-    }
-    return BISCO_OK;
-}
 
 // Layers whose protected set the decode kernels do not take themselves:
 // output rows (rows.cu) and payloads other than INT8 (formats.cu).
@@ -84,6 +62,29 @@ bisco_status dense_epilogue(const bisco_layer &L, void *out, int dtype, int *err
 }
 
 }  // namespace
+
+// Validates the sizes of a layer; buffers too when check_buffers.
+bisco_status check_layer(const bisco_layer *L, bool check_buffers) {
+    if (!L) return BISCO_ERR_INVALID_ARG;
+    if (L->n_out < 1 || L->k_in < 8 || L->k_in % 8 != 0) return BISCO_ERR_INVALID_ARG;
+    if (L->stages < 1 || L->stages > 3) return BISCO_ERR_INVALID_ARG;
+    if (L->protect_axis != 0 && L->protect_axis != 1) return BISCO_ERR_INVALID_ARG;
+    const int32_t p_max = L->protect_axis == 1 ? L->n_out : L->k_in;
+    if (L->n_protected < 0 || L->n_protected > p_max) return BISCO_ERR_INVALID_ARG;
+    if (L->protect_format < BISCO_PROT_INT8 || L->protect_format > BISCO_PROT_BF16)
+        return BISCO_ERR_INVALID_ARG;
+    if (L->chunk_dim != 8) return BISCO_ERR_UNSUPPORTED;
+    if (static_cast<int64_t>(L->n_out) * L->k_in > (int64_t(1) << 40)) return BISCO_ERR_INVALID_ARG;
+    if (!check_buffers) return BISCO_OK;
+    if (!L->codes || !L->norms || !aligned16(L->codes) || !aligned16(L->norms))
+        return BISCO_ERR_INVALID_ARG;
+    if (L->n_protected > 0) {
+        if (!L->q8 || !L->q8_scale || !L->prot_idx) return BISCO_ERR_INVALID_ARG;
+        if (!aligned16(L->q8) || !aligned16(L->q8_scale) || !aligned16(L->prot_idx))
+            return BISCO_ERR_INVALID_ARG;
+    }
+    return BISCO_OK;
+}
 
 int *device_error_word(bisco_status *st) {
     const int d = current_device();

@@ -11,6 +11,10 @@
 
 namespace bisco {
 
+// Validates the sizes of a layer (api.cu); its buffers too when
+// check_buffers.
+bisco_status check_layer(const bisco_layer *L, bool check_buffers);
+
 // Device error word of the current device (set up on first use).
 int *device_error_word(bisco_status *st);
 

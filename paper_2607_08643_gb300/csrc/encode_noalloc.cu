@@ -58,25 +58,17 @@ bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 extern "C" bisco_status bisco_encode_noalloc(const uint16_t *W_bf16, const float *g,
                                              const bisco_layer *L, bisco_stream_t stream) {
     using namespace bisco;
-    if (!L || !W_bf16 || !aligned16(W_bf16) || (g && (reinterpret_cast<uintptr_t>(g) & 3u)))
+    bisco_status st = check_layer(L, true);   // the same checks as bisco_encode
+    if (st != BISCO_OK) return st;
+    if (!W_bf16 || !aligned16(W_bf16) || (g && (reinterpret_cast<uintptr_t>(g) & 3u)))
         return BISCO_ERR_INVALID_ARG;
-    if (L->n_out < 1 || L->k_in < 8 || L->k_in % 8 != 0 || L->stages < 1 || L->stages > 3 ||
-        L->n_protected < 0 || L->n_protected > L->k_in ||
-        (L->protect_axis != 0 && L->protect_axis != 1))
-        return BISCO_ERR_INVALID_ARG;
-    if (L->chunk_dim != 8 || L->protect_axis != 0 || L->protect_format != BISCO_PROT_INT8)
-        return BISCO_ERR_UNSUPPORTED;
-    if (L->k_in > BISCO_ENCODE_NOALLOC_MAX_K) return BISCO_ERR_UNSUPPORTED;   // beyond the array
-    if (static_cast<int64_t>(L->n_out) * L->k_in > (int64_t(1) << 40)) return BISCO_ERR_INVALID_ARG;
-    if (!L->codes || !L->norms || !aligned16(L->codes) || !aligned16(L->norms))
-        return BISCO_ERR_INVALID_ARG;
-    if (L->n_protected > 0 &&
-        (!L->q8 || !L->q8_scale || !L->prot_idx || !aligned16(L->q8) ||
-         !aligned16(L->q8_scale) || !aligned16(L->prot_idx)))
-        return BISCO_ERR_INVALID_ARG;
+    // What this entry point leaves out: output-row protection, payloads
+    // other than INT8, and K beyond the array.
+    if (L->protect_axis != 0 || L->protect_format != BISCO_PROT_INT8) return BISCO_ERR_UNSUPPORTED;
+    if (L->k_in > BISCO_ENCODE_NOALLOC_MAX_K) return BISCO_ERR_UNSUPPORTED;
     if (encode_workspace_bytes(L->n_out, L->k_in) > kNoallocScratchBytes) return BISCO_ERR_UNSUPPORTED;
     void *scratch = nullptr;
-    bisco_status st = scratch_address(&scratch);
+    st = scratch_address(&scratch);
     if (st != BISCO_OK) return st;
     int *err = device_error_word(&st);
     if (!err) return st;

@@ -248,6 +248,21 @@ def test_protect_format_validation_before_any_device_call(lib):
         assert lib.bisco_encode_noalloc(x, None, ctypes.byref(L), None) == bisco.ERR_UNSUPPORTED
 
 
+def test_noalloc_validates_the_layer_as_bisco_encode_does(lib):
+    """Sizes, axis and format outside the layer's range give the same
+    INVALID_ARG as bisco_encode; the row axis alone is UNSUPPORTED."""
+    w, ws = ctypes.c_void_p(0x30000), ctypes.c_void_p(0x40000)
+    for bad in (dict(protect_format=5), dict(protect_format=-1), dict(protect_axis=2),
+                dict(k_in=12), dict(stages=4), dict(n_protected=-1), dict(n_protected=257)):
+        L = _fake_layer(**bad)
+        assert lib.bisco_encode(w, None, ctypes.byref(L), ws, 1 << 20, None) == bisco.ERR_INVALID_ARG
+        assert lib.bisco_encode_noalloc(w, None, ctypes.byref(L), None) == bisco.ERR_INVALID_ARG, bad
+    L = _fake_layer(protect_axis=1, n_protected=3)
+    assert lib.bisco_encode_noalloc(w, None, ctypes.byref(L), None) == bisco.ERR_UNSUPPORTED
+    assert lib.bisco_encode_noalloc(None, None, ctypes.byref(_fake_layer()), None) \
+        == bisco.ERR_INVALID_ARG
+
+
 def test_encode_workspace_by_axis(lib):
     assert bisco.bisco_encode_workspace_bytes_axis(300, 64, 0) == bisco.bisco_encode_workspace_bytes(300, 64)
     ws = bisco.bisco_encode_workspace_bytes_axis(300, 64, 1)
