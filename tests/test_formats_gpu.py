@@ -11,11 +11,7 @@ from paper_2607_08643_gb300 import synth
 
 from _helpers import TOL, max_rel_rows, sample_rows, to_dev
 
-pytestmark = [
-    pytest.mark.gpu,
-    pytest.mark.skip(reason="protected-format kernels not yet run on a GB300; enable after the "
-                            "first passing GPU run"),
-]
+pytestmark = pytest.mark.gpu
 
 FORMATS = [oracle.FMT_E4M3, oracle.FMT_E5M2, oracle.FMT_BF16]
 

@@ -108,8 +108,6 @@ def test_lora_after_gemv_end_to_end(env, B):
     assert max_rel_rows(y.cpu().numpy(), ref) <= TOL
 
 
-@pytest.mark.skip(reason="K-split down projection not yet run on a GB300; enable after the first "
-                         "passing GPU run")
 @pytest.mark.parametrize("N,K,rank,B,scale", CASES)
 def test_lora_split_down_matches_oracle(env, N, K, rank, B, scale, monkeypatch):
     """BISCO_LORA_SPLIT=1 (each rank row's K over the 8 warps of a CTA, added

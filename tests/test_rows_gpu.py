@@ -10,11 +10,7 @@ from paper_2607_08643_gb300 import synth
 
 from _helpers import TOL, max_rel_rows, to_dev
 
-pytestmark = [
-    pytest.mark.gpu,
-    pytest.mark.skip(reason="row-protection kernels not yet run on a GB300; enable after the "
-                            "first passing GPU run"),
-]
+pytestmark = pytest.mark.gpu
 
 
 @pytest.fixture(scope="module")
