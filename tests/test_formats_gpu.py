@@ -9,7 +9,7 @@ import pytest
 import oracle
 from paper_2607_08643_gb300 import synth
 
-from _helpers import TOL, max_rel_rows, sample_rows, to_dev
+from _helpers import assert_parity, gemm_tight, gemv_tight, sample_rows, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -73,7 +73,7 @@ def test_gemv_formats_match_oracle(env, fmt, N, K, B):
     y = bisco.bisco_gemv(L, to_dev(x, dev))
     torch.cuda.synchronize()
     assert bisco.bisco_get_device_error() == 0
-    assert max_rel_rows(y.cpu().numpy(), oracle.matmul(oracle_dense(ref), x)) <= TOL
+    assert_parity(y.cpu().numpy(), oracle.matmul(oracle_dense(ref), x), gemv_tight(B))
 
 
 @pytest.mark.parametrize("fmt", FORMATS)
@@ -90,9 +90,9 @@ def test_gemm_and_multi_formats_match_oracle(env, fmt):
     ys = bisco.bisco_gemv_multi([L, L8], to_dev(x, dev))
     torch.cuda.synchronize()
     assert bisco.bisco_get_device_error() == 0
-    assert max_rel_rows(Y.cpu().numpy(), oracle.matmul(oracle_dense(ref), X)) <= TOL
-    assert max_rel_rows(ys[0].cpu().numpy(), oracle.matmul(oracle_dense(ref), x)) <= TOL
-    assert max_rel_rows(ys[1].cpu().numpy(), oracle.matmul(oracle.decode_rows(ref8), x)) <= TOL
+    assert_parity(Y.cpu().numpy(), oracle.matmul(oracle_dense(ref), X), gemm_tight(300, K))
+    assert_parity(ys[0].cpu().numpy(), oracle.matmul(oracle_dense(ref), x), gemv_tight(8))
+    assert_parity(ys[1].cpu().numpy(), oracle.matmul(oracle.decode_rows(ref8), x), gemv_tight(8))
 
 
 @pytest.mark.parametrize("fmt", FORMATS)
@@ -118,8 +118,8 @@ def test_full_size_q_proj_e4m3_sampled(env):
     N, K = synth.QWEN3_8B_SHAPES["q_proj"]
     p = synth.protected_count(K, 1)
     W = synth.layer_weights(N, K, seed=41)
-    L = bisco.bisco_encode(to_dev(W, dev), 2, p, fmt=oracle.FMT_E4M3)
-    ref = L.to_numpy()
+    ref = oracle_layer(W, 2, p, oracle.FMT_E4M3)
+    L = bisco.Layer.from_numpy(ref, dev)
     rows = sample_rows(N)
     for B in (1, 16):
         x = synth.activations(B, K, seed=42 + B)
@@ -130,7 +130,7 @@ def test_full_size_q_proj_e4m3_sampled(env):
                                                          norms=ref["norms"][:, r:r + 1],
                                                          q8=ref["q8"][r:r + 1], N=1)), x)[:, 0]
                          for r in rows], axis=1)
-        assert max_rel_rows(y.cpu().numpy()[:, rows], want) <= TOL
+        assert_parity(y.cpu().numpy()[:, rows], want, gemv_tight(B))
 
 
 def oracle_rows_layer(W, S, p, fmt, idx=None):
@@ -183,7 +183,8 @@ def test_gemv_gemm_rows_formats_match_oracle(env, fmt):
         Y = bisco.bisco_gemv(L, to_dev(X, dev)) if M <= 16 else bisco.bisco_gemm(L, to_dev(X, dev))
         torch.cuda.synchronize()
         assert bisco.bisco_get_device_error() == 0
-        assert max_rel_rows(Y.cpu().numpy(), oracle.matmul(What, X)) <= TOL
+        assert_parity(Y.cpu().numpy(), oracle.matmul(What, X),
+                      gemv_tight(M) if M <= 16 else gemm_tight(M, K))
     out = bisco.bisco_decode_dense(L, "f32")
     torch.cuda.synchronize()
     got = out.cpu().numpy().astype(np.float64)

@@ -5,7 +5,7 @@ import pytest
 import oracle
 from paper_2607_08643_gb300 import synth
 
-from _helpers import TOL, max_rel_rows, sample_rows, to_dev
+from _helpers import assert_parity, gemm_tight, max_rel_rows, rows_per_tile, sample_rows, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -47,21 +47,43 @@ def test_gemm_matches_oracle(env, N, K, S, p, M):
     X = synth.activations(M, K, seed=M)
     Lref = oracle.encode(W, S=S, p=p)
     Y, _ = run_gemm(env, Lref, X)
-    assert max_rel_rows(Y, oracle.gemv(Lref, X)) <= TOL
+    assert_parity(Y, oracle.gemv(Lref, X), gemm_tight(M, K))
 
 
-@pytest.mark.parametrize("name", ["q_proj", "k_proj", "down_proj"])
+@pytest.mark.parametrize("name", ["q_proj", "k_proj", "gate_proj", "up_proj", "down_proj"])
 def test_gemm_full_size_sampled(env, name):
+    """Every Qwen3-8B shape at 2048 tokens.  gate/up (12288 x 4096: 768
+    tiles of 128 features x 256 tokens) make each persistent CTA walk five or
+    six tiles; the sample takes two features of every 128-feature tile and
+    five tokens of every 256-token tile, so every tile is checked."""
     N, K = synth.QWEN3_8B_SHAPES[name]
     S, p = 2, synth.protected_count(K, 1)
-    W = synth.layer_weights(N, K, seed=23)
+    W = synth.layer_weights(N, K, seed=23 + N % 7)
     X = synth.activations(2048, K, seed=24)
     Lref = oracle.encode(W, S=S, p=p)
     Y, _ = run_gemm(env, Lref, X)
-    rows = sample_rows(N, n=12)
-    toks = sample_rows(2048, n=40, seed=1)
+    rows = rows_per_tile(N, 128, per=2, seed=N)
+    toks = rows_per_tile(2048, 256, per=5, seed=1)
     ref = oracle.apply_rows(Lref, rows, X[toks])
-    assert max_rel_rows(Y[toks][:, rows], ref) <= TOL
+    assert_parity(Y[toks][:, rows], ref, gemm_tight(2048, K), name)
+
+
+@pytest.mark.parametrize("N,K,S,p,M", [
+    (4096, 256, 2, 3, 4096),        # 512 tiles: every CTA runs three or four
+    (2048, 512, 3, 6, 8192),        # 512 tiles, three stages
+    (1152, 384, 1, 0, 8000),        # ragged last token tile, S = 1, no protection
+])
+def test_gemm_many_tiles_per_cta(env, N, K, S, p, M):
+    """Far more tiles than SMs at small K: accumulator reuse, the TMEM
+    phases and the rings carried from tile to tile, checked on every
+    output feature against 320 tokens spread over all token tiles."""
+    W = synth.layer_weights(N, K, seed=N + K + M)
+    X = synth.activations(M, K, seed=M + 1)
+    Lref = oracle.encode(W, S=S, p=p)
+    Y, _ = run_gemm(env, Lref, X)
+    toks = rows_per_tile(M, 256, per=10, seed=M)
+    ref = oracle.gemv(Lref, X[toks])
+    assert_parity(Y[toks], ref, gemm_tight(M, K), f"{N}x{K} M={M}")
 
 
 def test_gemm_equals_gemv(env):
