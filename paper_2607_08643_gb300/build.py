@@ -13,7 +13,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libbisco.so")
-SOURCES = ["api.cu", "encode.cu", "encode_noalloc.cu", "gemv.cu", "gemm.cu", "dense.cu", "lora.cu",
+SOURCES = ["api.cu", "encode.cu", "encode_noalloc.cu", "gemv.cu", "gemv_b1.cu", "gemm.cu", "dense.cu", "lora.cu",
            "rows.cu", "decoder.cu", "formats.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",

@@ -92,6 +92,29 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
     }
 }
 
+// mbar_wait with a suspend-time hint (ns) on every poll: a waiting warp
+// yields its issue slots to the others instead of spinning.
+__device__ __forceinline__ bool mbar_try_wait_hint(uint32_t bar, uint32_t parity, uint32_t ns) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok) : "r"(bar), "r"(parity), "r"(ns) : "memory");
+    return ok != 0;
+}
+
+__device__ __forceinline__ bool mbar_wait_sleep(uint32_t bar, uint32_t parity, uint32_t ns) {
+    if (mbar_try_wait_hint(bar, parity, ns)) return true;
+    const uint64_t t0 = globaltimer();
+    for (;;) {
+#pragma unroll 1
+        for (int i = 0; i < 8; ++i)
+            if (mbar_try_wait_hint(bar, parity, ns)) return true;
+        if (globaltimer() - t0 > BISCO_WAIT_NS) return false;
+    }
+}
+
 // Whole-warp form: every lane waits (each acquires), and the warp leaves
 // converged with one verdict, so a lane that gave up cannot split the warp
 // before a warp-aligned instruction.
@@ -148,6 +171,15 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_
     asm volatile(
         "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
         ::"r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
+}
+
+// The same with an L2 policy for the source (data read once: evict first).
+__device__ __forceinline__ void bulk_load_hint(uint32_t dst, const void *src, uint32_t bytes,
+                                               uint32_t bar, uint64_t pol) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1], %2, [%3], %4;"
+        ::"r"(dst), "l"(src), "r"(bytes), "r"(bar), "l"(pol) : "memory");
 }
 
 // Warms L2 with [src, src + bytes) (16-byte aligned, bytes % 16 == 0).  A
@@ -358,17 +390,11 @@ __device__ __forceinline__ uint32_t lop3_and_or(uint32_t a, uint32_t mask, uint3
     return r;
 }
 
-__device__ __forceinline__ uint16_t lo_half(uint32_t w) {
-    uint16_t l, h;
-    asm("mov.b32 {%0, %1}, %2;" : "=h"(l), "=h"(h) : "r"(w));
-    return l;
-}
+// Halves of a 32-bit word as plain integer operations, so that the compiler
+// can fold the selection into the instruction that consumes the half.
+__device__ __forceinline__ uint16_t lo_half(uint32_t w) { return static_cast<uint16_t>(w & 0xFFFFu); }
 
-__device__ __forceinline__ uint16_t hi_half(uint32_t w) {
-    uint16_t l, h;
-    asm("mov.b32 {%0, %1}, %2;" : "=h"(l), "=h"(h) : "r"(w));
-    return h;
-}
+__device__ __forceinline__ uint16_t hi_half(uint32_t w) { return static_cast<uint16_t>(w >> 16); }
 
 // c + a * b for fp16 a, b (bit patterns) and fp32 c: the product of two fp16
 // values is exact in fp32, so the result is rounded once, to fp32

@@ -1720,8 +1720,16 @@ bisco_status launch_gemv(const bisco_layer &L, const uint16_t *x, int B, float *
     a.B = B;
     a.p = p;
 
-    // streaming kernel: small batch and at least one 16-row tile per SM
+    // batch 1: the row-split kernel of gemv_b1.cu where it applies (K a
+    // multiple of 4096), unless a kernel of this file is forced
     const char *mode = getenv("BISCO_GEMV_MODE");
+    if (B == 1 && !mode) {
+        bool launched = false;
+        const bisco_status st = launch_gemv_b1(&L, 1, x, &y, err, stream, &launched);
+        if (launched || st != BISCO_OK) return st;
+    }
+
+    // streaming kernel: small batch and at least one 16-row tile per SM
     const int sms = num_sms();
     bool use_stream = B <= 16 && (N + 15) / 16 >= sms;
     if (mode && mode[0] == 's') use_stream = B <= 16;
@@ -1803,6 +1811,11 @@ bisco_status launch_gemv(const bisco_layer &L, const uint16_t *x, int B, float *
 
 bisco_status launch_gemv_multi(const bisco_layer *Ls, int G, const uint16_t *x, int B,
                                float *const *y, int *err, cudaStream_t stream) {
+    if (B == 1 && !getenv("BISCO_GEMV_MODE")) {
+        bool launched = false;
+        const bisco_status st = launch_gemv_b1(Ls, G, x, y, err, stream, &launched);
+        if (launched || st != BISCO_OK) return st;
+    }
     if (B <= 8 && Ls[0].k_in % 128 == 0) {
         bool launched = false;
         const bisco_status st = launch_stream(Ls, G, x, B, y, err, num_sms(), stream, &launched);

@@ -1,0 +1,523 @@
+// gemv_b1.cu -- batch-1 decode-time y = What x straight from the coded
+// layer (Sec. III-G Eq. 12 with Eq. 10's protected columns) for G <= 4
+// layers that share x and have K a multiple of 4096 (every Qwen3-8B
+// projection).
+//
+// Work split.  The CTAs of a one-per-SM grid are shared out among the G
+// layers so that the longest row run per CTA is as short as it can be
+// (q/k/v of Qwen3-8B: 101/25/26 CTAs of 40-41 rows); each CTA takes a
+// contiguous run of one layer's rows.  A row's work is S * K/4096 items, one
+// per (stage, 4096-column span): 512 sign bytes and 512 fp16 norms, 1536
+// bytes.  A CTA orders its items stage by stage, row by row, span by span --
+// the order of the [S][N][K/8] buffers -- and each of its 16 warps takes one
+// contiguous run of that list.
+//
+// Data path.  Every warp owns a ring of `depth` item slots in shared memory.
+// Lane 0 fills a slot with two 1-D bulk copies (cp.async.bulk: 512 B of
+// signs, 1 KB of norms) that complete on the slot's mbarrier, and refills it
+// with the item `depth` further on as soon as the warp has read it.  The
+// first `depth` items of every warp are requested before the wait on the
+// previous kernel, so a CTA has up to 16 * depth * 1.5 KB of its layer in
+// flight while that kernel finishes.  On GB300 this layout streams at the
+// HBM copy rate with 16 decoding warps; 8 warps reach about 80 % of it and a
+// register-staged load pipeline about half.
+//
+// Decode (Eq. 12 per chunk-stage): for a sign byte b of chunk c the signed
+// sum of the chunk's 8 activations is T_lo(c, b & 15) + T_hi(c, b >> 4),
+// where T_lo(c, v) = sum_{e<4} (bit e of v ? -x[8c+e] : x[8c+e]) and T_hi the
+// same over x[8c+4..8c+7].  Each is rounded once to fp16 (2^-11 relative),
+// held as one fp16 pair (T_lo, T_hi) per (c, v), and meets the chunk's fp16
+// norm in an fp16 x fp16 -> fp32 FMA (exact product).  The layer's protected
+// columns are zero in its tables, which is Eq. 10's overwrite of their BSQ
+// value; the 1/sqrt(8) of Eq. 3 is applied once per output.
+//
+// Table placement.  Lane l of an item handles chunks 8l+j (j = 0..7) of each
+// 256-chunk half h of its span; chunk c = 512*span + 256*h + 8l + j sits at
+// position P = 512*span + 256*h + 32*j + l, and entry (P, v) at byte
+//   (P >> 6) * 4096 + v * 256 + (P & 63) * 4,
+// so a lane's lookups always hit bank l.  With the table 4 KB aligned, the
+// lane's base address has bits 8..11 clear and the lookup address is one
+// shift and one LOP3 ((w >> s) & 0xF00 | base) plus a compile-time offset.
+//
+// Outputs.  Each item's lane sums are added across the warp (fixed shuffle
+// order) into one float per item; after a CTA barrier a warp per row adds
+// its items in item order, scales by 1/sqrt(8) and adds the protected term
+// sum_u q8[r][u] * (scale_u * x[idx_u]) (int8 rows staged in shared memory
+// before the wait).  No atomics: the result depends only on the sizes.
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <stdlib.h>
+
+#include "bisco_dev.cuh"
+#include "bisco_host.h"
+
+namespace bisco {
+namespace {
+
+constexpr int kB1Warps = 16;
+constexpr int kB1Span = 512;                  // chunks per item
+constexpr uint32_t kB1Item = 1536;            // bytes per item slot: signs, then norms
+constexpr int kB1MaxG = 4;                    // layers per launch
+constexpr float kB1InvSqrt8 = 0.35355339059327373f;
+// Two CTAs (this layer's and the next one's) share an SM when each takes at
+// most this much dynamic shared memory (228 KB per SM, 1 KB reserved per CTA).
+constexpr size_t kB1Coresident = 112 * 1024;
+constexpr size_t kB1MaxSmem = 227 * 1024;
+
+struct B1Layer {
+    const uint8_t *codes;      // [S][N][K/8]
+    const uint16_t *norms;     // [S][N][K/8] fp16
+    const int8_t *q8;          // [N][p_pad]
+    const uint16_t *q8_scale;  // [p] fp16
+    const int32_t *prot_idx;   // [p]
+    float *y;                  // [N]
+    int N, p, p_pad;
+    int cta0, ctas;            // the CTAs of the grid that take this layer's rows
+};
+
+struct B1Args {
+    B1Layer L[kB1MaxG];
+    const uint16_t *x;
+    int *err;
+    int K, G;
+    int nspan;                 // K / 4096
+    int S;                     // stages
+    int depth;                 // item slots per warp
+    int q8_staged;             // int8 rows in shared memory (else read at the end)
+    uint32_t sleep_ns;         // suspend-time hint of the item waits
+    uint32_t off_ring, off_pm, off_pidx, off_sx, off_part, off_q8, off_bar;   // tables at 0
+};
+
+template <uint32_t A>
+__device__ __forceinline__ unsigned char *align_smem(unsigned char *raw) {
+    return raw + ((A - (smem_u32(raw) & (A - 1u))) & (A - 1u));
+}
+
+__device__ __forceinline__ uint4 lds_u128(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+    return v;
+}
+
+// (w >> sh) for sh >= 0, (w << -sh) otherwise (sh a compile-time constant)
+template <int SH>
+__device__ __forceinline__ uint32_t shift_by(uint32_t w) {
+    if constexpr (SH >= 0) return w >> SH;
+    else return w << (-SH);
+}
+
+// Lane sums of one item: 16 chunks (8 per half) through the tables at base0.
+__device__ __forceinline__ float b1_item(const uint2 (&cw)[2], const uint4 (&nw)[2], uint32_t base0) {
+    float acc4[2][2] = {{0.f, 0.f}, {0.f, 0.f}};   // four short FMA chains, one per word
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+#pragma unroll
+        for (int jw = 0; jw < 2; ++jw) {
+            const uint32_t w = jw ? cw[h].y : cw[h].x;
+            const uint32_t n01 = jw ? nw[h].z : nw[h].x;
+            const uint32_t n23 = jw ? nw[h].w : nw[h].y;
+            uint32_t lo[4], hi[4];
+            // v << 8 for the low and high nibble of byte jj: bits 8jj.. and 8jj+4..
+            lo[0] = lop3_and_or(shift_by<-8>(w), 0xF00u, base0);
+            lo[1] = lop3_and_or(w, 0xF00u, base0);
+            lo[2] = lop3_and_or(shift_by<8>(w), 0xF00u, base0);
+            lo[3] = lop3_and_or(shift_by<16>(w), 0xF00u, base0);
+            hi[0] = lop3_and_or(shift_by<-4>(w), 0xF00u, base0);
+            hi[1] = lop3_and_or(shift_by<4>(w), 0xF00u, base0);
+            hi[2] = lop3_and_or(shift_by<12>(w), 0xF00u, base0);
+            hi[3] = lop3_and_or(shift_by<20>(w), 0xF00u, base0);
+            uint32_t tl[4], th[4];
+#pragma unroll
+            for (int jj = 0; jj < 4; ++jj) {
+                const int j = 4 * jw + jj;
+                const uint32_t off = h * 16384u + (j >> 1) * 4096u + (j & 1) * 128u;
+                tl[jj] = lds_u32(lo[jj] + off);
+                th[jj] = lds_u32(hi[jj] + off);
+            }
+            float &acc = acc4[h][jw];
+#pragma unroll
+            for (int jj = 0; jj < 4; ++jj) {
+                const uint32_t nn = jj < 2 ? n01 : n23;
+                const uint16_t n = (jj & 1) ? hi_half(nn) : lo_half(nn);
+                acc = fma_f16_f32(lo_half(tl[jj]), n, acc);
+                acc = fma_f16_f32(hi_half(th[jj]), n, acc);
+            }
+        }
+    }
+    return (acc4[0][0] + acc4[0][1]) + (acc4[1][0] + acc4[1][1]);
+}
+
+// Lane 0 of the warp arms a slot's mbarrier for 1536 bytes and issues its
+// two bulk copies (signs, norms); the other lanes run the same instruction
+// stream with the predicate off, so the warp never diverges.
+__device__ __forceinline__ void b1_issue(bool leader, uint32_t slot, uint32_t bar, const void *codes,
+                                         const void *norms, uint64_t pol) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.u32 p, %0, 0;\n\t"
+        "@p fence.proxy.async.shared::cta;\n\t"
+        "@p mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%2], 1536;\n\t"
+        "@p cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%1], [%3], 512, [%2], %5;\n\t"
+        "@p cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%6], [%4], 1024, [%2], %5;\n\t}"
+        ::"r"(static_cast<uint32_t>(leader)), "r"(slot), "r"(bar), "l"(codes), "l"(norms), "l"(pol),
+          "r"(slot + 512u)
+        : "memory");
+}
+
+// D item slots per warp; NSPAN 4096-column spans per row (0: a.nspan, at
+// run time).  Both fixed at compile time make every ring address an
+// immediate offset.
+template <int D, int NSPAN>
+__global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_constant__ B1Args a) {
+    constexpr int kB1Threads = kB1Warps * 32;
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *sm = align_smem<4096>(smem_raw);
+    const uint32_t sbase = smem_u32(sm);
+    __shared__ int s_abort;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int K = a.K, C = K / 8, nspan = NSPAN ? NSPAN : a.nspan, S = a.S;
+    // this CTA's layer and rows [ra, ra + nrows)
+    int g = 0;
+#pragma unroll
+    for (int i = 1; i < kB1MaxG; ++i)
+        if (i < a.G && static_cast<int>(blockIdx.x) >= a.L[i].cta0) g = i;
+    const B1Layer &L = a.L[g];
+    const int N = L.N, p = L.p, p_pad = L.p_pad;
+    const int ci = static_cast<int>(blockIdx.x) - L.cta0;
+    const int ra = static_cast<int>(static_cast<int64_t>(N) * ci / L.ctas);
+    const int rb = static_cast<int>(static_cast<int64_t>(N) * (ci + 1) / L.ctas);
+    const int nrows = rb - ra;
+    const int nitems = nrows * S * nspan;
+    const uint8_t *const codes = L.codes;
+    const uint16_t *const norms = L.norms;
+    const int8_t *const q8 = L.q8;
+    float *const y = L.y;
+
+    uint32_t *pm = reinterpret_cast<uint32_t *>(sm + a.off_pm);   // protected bits, 32 columns a word
+    int *spidx = reinterpret_cast<int *>(sm + a.off_pidx);        // [p]
+    float *ssc = reinterpret_cast<float *>(spidx + (p + 3) / 4 * 4);
+    float *sx = reinterpret_cast<float *>(sm + a.off_sx);         // scale * x [p]
+    float *part = reinterpret_cast<float *>(sm + a.off_part);     // [nitems]
+    int8_t *q8s = reinterpret_cast<int8_t *>(sm + a.off_q8);
+    const uint64_t pol = l2_evict_first_policy();
+
+    // this warp's items [kb, kb + cnt), in memory order, through its ring.
+    // Within a stage the items of consecutive rows are consecutive in memory
+    // (512 elements apart); a stage boundary jumps to the next [N][K/8] plane.
+    const int kb = static_cast<int>(static_cast<int64_t>(nitems) * warp / kB1Warps);
+    const int cnt = static_cast<int>(static_cast<int64_t>(nitems) * (warp + 1) / kB1Warps) - kb;
+    const int per_stage = nrows * nspan;
+    const uint32_t wring = sbase + a.off_ring + static_cast<uint32_t>(warp * D) * kB1Item;
+    const uint32_t wbar = sbase + a.off_bar + static_cast<uint32_t>(warp * D) * 8u;
+    // issue cursor: element offset of the next item to request, the items
+    // left in its stage, and that stage
+    int is = per_stage > 0 ? kb / per_stage : 0;
+    int ileft = per_stage - (kb - is * per_stage);
+    int64_t ie = (static_cast<int64_t>(is) * N + ra) * C + static_cast<int64_t>(kb - is * per_stage) * kB1Span;
+    // every lane keeps the cursor (uniform), lane 0 alone issues
+    auto advance = [&]() {
+        ie += kB1Span;
+        if (--ileft == 0) {
+            ++is;
+            ie = (static_cast<int64_t>(is) * N + ra) * C;
+            ileft = per_stage;
+        }
+    };
+
+    // ---- before the wait: barriers, first items, protected metadata, int8 rows
+    int issued = 0;
+    if (lane == 0) {
+        for (int d = 0; d < D; ++d) mbar_init(wbar + 8 * d, 1);
+        fence_mbar_init();
+    }
+    __syncwarp();
+#pragma unroll
+    for (int d = 0; d < D; ++d)
+        if (d < cnt) {
+            b1_issue(lane == 0, wring + d * kB1Item, wbar + d * 8u, codes + ie, norms + ie, pol);
+            advance();
+            ++issued;
+        }
+    if (threadIdx.x == 0) s_abort = 0;
+    for (int i = threadIdx.x; i < C / 4; i += kB1Threads) pm[i] = 0u;
+    __syncthreads();
+    for (int u = threadIdx.x; u < p; u += kB1Threads) {
+        int j = L.prot_idx[u];
+        float sc = __half2float(__ushort_as_half(L.q8_scale[u]));
+        if (j < 0 || j >= K) {   // not a valid layer: reported, and the entry dropped
+            latch_error(a.err, BISCO_ERR_INVALID_ARG);
+            j = -1;
+            sc = 0.f;
+        } else {
+            atomicOr(&pm[j >> 5], 1u << (j & 31));
+        }
+        spidx[u] = j;
+        ssc[u] = sc;
+    }
+    if (p > 0 && nrows > 0) {
+        if (a.q8_staged) {
+            const int n16 = nrows * p_pad / 16;
+            const uint4 *src = reinterpret_cast<const uint4 *>(q8 + static_cast<int64_t>(ra) * p_pad);
+            for (int i = threadIdx.x; i < n16; i += kB1Threads) reinterpret_cast<uint4 *>(q8s)[i] = src[i];
+        } else if (threadIdx.x == 0) {
+            // read at the end from global memory: into L2 now
+            prefetch_l2(q8 + static_cast<int64_t>(ra) * p_pad, static_cast<uint32_t>(nrows * p_pad));
+        }
+    }
+    __syncthreads();
+    pdl_launch_dependents();
+
+    // ---- after the wait: this layer's tables of x, scale * x
+    pdl_wait();
+    // x of this thread's protected column, loaded with its first table job
+    // (one round trip for both)
+    const int uj = threadIdx.x < p ? spidx[threadIdx.x] : -1;
+    const uint16_t xj = uj >= 0 ? a.x[uj] : static_cast<uint16_t>(0);
+    for (int J = warp; J < C / 32; J += kB1Warps) {   // job: one (span, half, j) for 32 lanes
+        const int span = J >> 4, h = (J >> 3) & 1, j = J & 7;
+        const int c = span * kB1Span + h * 256 + 8 * lane + j;
+        const uint4 u = *reinterpret_cast<const uint4 *>(a.x + 8 * c);
+        const uint32_t m = (pm[c >> 2] >> ((c & 3) * 8)) & 0xFFu;
+        float e[8] = {__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xFFFF0000u),
+                      __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xFFFF0000u),
+                      __uint_as_float(u.z << 16), __uint_as_float(u.z & 0xFFFF0000u),
+                      __uint_as_float(u.w << 16), __uint_as_float(u.w & 0xFFFF0000u)};
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            if ((m >> k) & 1u) e[k] = 0.f;
+        // signed sums of element pairs: index bit 0 negates the first, bit 1 the second
+        float p01[2][4], p23[2][4];
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const float x0 = e[4 * hh], x1 = e[4 * hh + 1], x2 = e[4 * hh + 2], x3 = e[4 * hh + 3];
+            p01[hh][0] = x0 + x1; p01[hh][1] = x1 - x0; p01[hh][2] = x0 - x1; p01[hh][3] = -(x0 + x1);
+            p23[hh][0] = x2 + x3; p23[hh][1] = x3 - x2; p23[hh][2] = x2 - x3; p23[hh][3] = -(x2 + x3);
+        }
+        const int P = span * kB1Span + h * 256 + 32 * j + lane;
+        const uint32_t dst = sbase + static_cast<uint32_t>((P >> 6) * 4096 + (P & 63) * 4);
+#pragma unroll
+        for (int v = 0; v < 16; ++v) {
+            const __half2 hv = __floats2half2_rn(p01[0][v & 3] + p23[0][v >> 2],
+                                                 p01[1][v & 3] + p23[1][v >> 2]);
+            asm volatile("st.shared.b32 [%0], %1;" ::"r"(dst + v * 256),
+                         "r"(*reinterpret_cast<const uint32_t *>(&hv)));
+        }
+    }
+    // scale * x of the protected columns (exact in fp32: 11 x 8 significant bits)
+    if (threadIdx.x < p) sx[threadIdx.x] = uj >= 0 ? ssc[threadIdx.x] * bf16_bits_to_f32(xj) : 0.f;
+    for (int u = threadIdx.x + kB1Threads; u < p; u += kB1Threads) {
+        const int j = spidx[u];
+        sx[u] = j >= 0 ? ssc[u] * bf16_bits_to_f32(a.x[j]) : 0.f;
+    }
+    __syncthreads();
+
+    // ---- decode: this warp's items through its ring, D at a time
+    {
+        const uint32_t base0 = sbase + lane * 4u;
+        int i = 0, span = kb - (kb / nspan) * nspan;
+        uint32_t phase = 0;
+        bool ok = true;
+        for (int i0 = 0; i0 < cnt && ok; i0 += D, phase ^= 1u) {
+#pragma unroll
+            for (int d = 0; d < D; ++d) {
+                if (i0 + d >= cnt) break;
+                const uint32_t slot = wring + d * kB1Item;
+                const uint32_t bar = wbar + d * 8u;
+                if (!__all_sync(0xFFFFFFFFu, mbar_try_wait(bar, phase)) &&
+                    !__all_sync(0xFFFFFFFFu, mbar_wait_sleep(bar, phase, a.sleep_ns))) {
+                    if (lane == 0) {
+                        latch_error(a.err, BISCO_ERR_TIMEOUT);
+                        atomicExch(&s_abort, 1);
+                    }
+                    ok = false;
+                    break;
+                }
+                uint2 cw[2];
+                uint4 nw[2];
+                cw[0] = lds_u64(slot + lane * 8u);
+                cw[1] = lds_u64(slot + 256u + lane * 8u);
+                nw[0] = lds_u128(slot + 512u + lane * 16u);
+                nw[1] = lds_u128(slot + 1024u + lane * 16u);
+                float v = b1_item(cw, nw, NSPAN == 1 ? base0 : base0 + static_cast<uint32_t>(span) * 32768u);
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+                if (lane == 0) part[kb + i0 + d] = v;
+                // the slot's reads are done (the values are in registers): refill it
+                __syncwarp();
+                if (issued < cnt) {
+                    b1_issue(lane == 0, slot, bar, codes + ie, norms + ie, pol);
+                    advance();
+                    ++issued;
+                }
+                if (NSPAN != 1) span = span + 1 == nspan ? 0 : span + 1;
+                i = i0 + d + 1;
+            }
+        }
+        // every copy this warp issued has landed before it leaves the ring
+        if (lane == 0)
+            for (int j = i; j < issued; ++j)
+                mbar_wait(wbar + static_cast<uint32_t>(j % D) * 8u, static_cast<uint32_t>(j / D) & 1u);
+    }
+    __syncthreads();
+    if (*reinterpret_cast<volatile int *>(&s_abort)) return;
+
+    // ---- outputs: a warp per row; items in order, then the protected term
+    for (int rr = warp; rr < nrows; rr += kB1Warps) {
+        float pr = 0.f;
+        if (p > 0) {
+            const int8_t *q8r = a.q8_staged ? q8s + rr * p_pad : q8 + static_cast<int64_t>(ra + rr) * p_pad;
+            for (int u = lane; u < p; u += 32) pr = fmaf(static_cast<float>(q8r[u]), sx[u], pr);
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) pr += __shfl_xor_sync(0xFFFFFFFFu, pr, o);
+        }
+        if (lane == 0) {
+            float v = 0.f;
+            for (int s = 0; s < S; ++s)
+                for (int sp = 0; sp < nspan; ++sp) v += part[(s * nrows + rr) * nspan + sp];
+            y[ra + rr] = v * kB1InvSqrt8 + pr;
+        }
+    }
+}
+
+size_t align_up_b1(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+template <int D, int NSPAN>
+bisco_status launch_b1_t(const B1Args &a, int grid, size_t smem, cudaStream_t stream) {
+    auto kern = k_gemv_b1<D, NSPAN>;
+    static size_t configured[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return BISCO_ERR_CUDA;
+    if (smem > configured[dev]) {
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(smem)) != cudaSuccess)
+            return BISCO_ERR_CUDA;
+        configured[dev] = smem;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid, 1, 1);
+    cfg.blockDim = dim3(kB1Warps * 32, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, a) == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+}
+
+// Shared memory of one CTA with `depth` item slots per warp, past the 4 KB
+// aligned base (tables first); fills the offsets of `a`.
+size_t b1_layout(int C, int depth, int p_max, int items_max, size_t q8_bytes, B1Args *a) {
+    size_t off = static_cast<size_t>(C) * 64;   // tables: 64 bytes per chunk
+    a->off_ring = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(kB1Warps) * depth * kB1Item;
+    a->off_pm = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(C);                          // one bit per column
+    a->off_pidx = static_cast<uint32_t>(off);
+    off += static_cast<size_t>((p_max + 3) / 4 * 4) * 8;    // indices, scales
+    a->off_sx = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(p_max) * 4;
+    off = align_up_b1(off, 16);
+    a->off_part = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(items_max) * 4;
+    off = align_up_b1(off, 16);
+    a->off_q8 = static_cast<uint32_t>(off);
+    off += q8_bytes;
+    off = align_up_b1(off, 8);
+    a->off_bar = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(kB1Warps) * depth * 8;
+    return off + 4096;   // slack for the 4 KB aligned base
+}
+
+}  // namespace
+
+bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, float *const *y,
+                            int *err, cudaStream_t stream, bool *launched) {
+    *launched = false;
+    if (const char *e = getenv("BISCO_GEMV_B1"))
+        if (e[0] == '0') return BISCO_OK;
+    if (G < 1 || G > kB1MaxG) return BISCO_OK;
+    const int K = Ls[0].k_in, S = Ls[0].stages;
+    if (K % 4096 != 0 || S < 1 || S > 3) return BISCO_OK;
+    B1Args a = {};
+    a.x = x;
+    a.err = err;
+    a.K = K;
+    a.G = G;
+    a.nspan = K / 4096;
+    int p_max = 0;
+    for (int g = 0; g < G; ++g) {
+        const bisco_layer &L = Ls[g];
+        if (L.k_in != K || L.stages != S || L.protect_axis != 0 || L.protect_format != BISCO_PROT_INT8)
+            return BISCO_OK;
+        B1Layer &b = a.L[g];
+        b.codes = reinterpret_cast<const uint8_t *>(L.codes);
+        b.norms = L.norms;
+        b.q8 = L.q8;
+        b.q8_scale = L.q8_scale;
+        b.prot_idx = L.prot_idx;
+        b.y = y[g];
+        b.N = L.n_out;
+        b.p = L.n_protected;
+        b.p_pad = (L.n_protected + 15) / 16 * 16;
+        p_max = p_max > b.p ? p_max : b.p;
+    }
+    // CTAs per layer: one each, then one at a time to the layer with the
+    // longest row run per CTA, up to one CTA per SM
+    const int sms = num_sms();
+    if (G > sms) return BISCO_OK;
+    int ctas[kB1MaxG] = {}, total = G;
+    for (int g = 0; g < G; ++g) ctas[g] = 1;
+    auto run = [&](int g) { return (a.L[g].N + ctas[g] - 1) / ctas[g]; };
+    while (total < sms) {
+        int best = -1;
+        for (int g = 0; g < G; ++g)
+            if (ctas[g] < a.L[g].N && (best < 0 || run(g) > run(best))) best = g;
+        if (best < 0) break;
+        ++ctas[best];
+        ++total;
+    }
+    int rows_max = 0;
+    size_t q8_max = 0;
+    for (int g = 0, c0 = 0; g < G; ++g) {
+        a.L[g].cta0 = c0;
+        a.L[g].ctas = ctas[g];
+        c0 += ctas[g];
+        rows_max = rows_max > run(g) ? rows_max : run(g);
+        const size_t q8b = static_cast<size_t>(run(g)) * a.L[g].p_pad;
+        q8_max = q8_max > q8b ? q8_max : q8b;
+    }
+    const int C = K / 8;
+    const int items_max = rows_max * S * a.nspan;
+    // the deepest ring (three or two item slots per warp) that leaves room
+    // for the next kernel's CTA on the SM, else one CTA per SM
+    int depth = 0;
+    size_t smem = 0;
+    for (int pass = 0; pass < 2 && depth == 0; ++pass) {
+        const size_t budget = pass == 0 ? kB1Coresident : kB1MaxSmem;
+        for (int d = 3; d >= 2 && depth == 0; --d)
+            for (int staged = 1; staged >= 0 && depth == 0; --staged) {
+                const size_t need = b1_layout(C, d, p_max, items_max, staged ? q8_max : 0, &a);
+                if (need <= budget) {
+                    depth = d;
+                    smem = need;
+                    a.q8_staged = staged;
+                }
+            }
+    }
+    if (depth == 0) return BISCO_OK;
+    a.depth = depth;
+    a.S = S;
+    a.sleep_ns = 200;
+    b1_layout(C, depth, p_max, items_max, a.q8_staged ? q8_max : 0, &a);
+    *launched = true;
+    const bool one = a.nspan == 1;
+    if (depth == 3) return one ? launch_b1_t<3, 1>(a, total, smem, stream) : launch_b1_t<3, 0>(a, total, smem, stream);
+    return one ? launch_b1_t<2, 1>(a, total, smem, stream) : launch_b1_t<2, 0>(a, total, smem, stream);
+}
+}  // namespace bisco

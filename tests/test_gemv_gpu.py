@@ -286,3 +286,60 @@ def test_gemv_batch1_zero_activations(env):
     Lref = oracle.encode(synth.layer_weights(N, K, seed=99), S=S, p=p)
     y = run_gemv(env, Lref, np.zeros((1, K), np.uint16))
     assert np.all(y == 0)
+
+
+# ------------------------------------------------- batch 1, row-split kernel
+# K a multiple of 4096 at batch 1 goes to the row-split kernel: every CTA
+# takes an equal run of the launch's rows (across the layers of a group),
+# codes and norms go straight to registers, and each CTA builds masked
+# tables for the (at most two) layers its rows touch.  The cases cover rows
+# fewer than SMs, ragged row runs, S = 1..3, K = 4096 / 8192 / 12288, layers
+# without protection, int8 rows too large to stage in shared memory, and
+# groups whose layer boundaries fall inside CTAs.
+
+@pytest.mark.parametrize("N,K,S,p", [
+    (16, 4096, 1, 0),          # 16 rows: 16 one-row CTAs
+    (150, 4096, 2, 41),        # one row per CTA, two left idle
+    (153, 4096, 3, 41),        # 152 CTAs, one with two rows
+    (1000, 4096, 2, 0),        # no protection
+    (2500, 4096, 3, 82),       # ragged row runs, S = 3
+    (500, 8192, 2, 82),        # two 4096-column spans per stage
+    (300, 12288, 2, 123),      # three spans (down_proj width)
+    (4000, 4096, 2, 2000),     # int8 rows read from global memory at the end
+])
+def test_gemv_b1_matches_oracle(env, N, K, S, p):
+    W = synth.layer_weights(N, K, seed=N + K + S + p, dist="t4" if S == 3 else "normal")
+    X = synth.activations(1, K, seed=N + 5)
+    Lref = oracle.encode(W, S=S, p=p)
+    y = run_gemv(env, Lref, X)
+    assert_parity(y, oracle.gemv(Lref, X), gemv_tight(1))
+    # the same bits on a second call (no atomics, a fixed summation order)
+    assert np.array_equal(y, run_gemv(env, Lref, X))
+
+
+@pytest.mark.parametrize("shapes", [
+    [(300, 21), (64, 0), (1000, 33)],                 # layer boundaries inside CTAs
+    [(4096, 41), (1024, 41), (1024, 41)],             # q/k/v of one attention layer
+    [(3000, 41), (2000, 0), (1500, 41), (4000, 10)],  # four layers
+    [(200, 5), (7, 3), (150, 0)],                     # a CTA over three layers: other kernel
+])
+def test_gemv_b1_groups_match_oracle(env, shapes):
+    K, S = 4096, 2
+    Lrefs = [oracle.encode(synth.layer_weights(N, K, seed=200 + i), S=S, p=p)
+             for i, (N, p) in enumerate(shapes)]
+    X = synth.activations(1, K, seed=201)
+    ys = _multi(env, Lrefs, X)
+    for y, L in zip(ys, Lrefs):
+        rows = sample_rows(L["N"], n=64) if L["N"] > 2000 else np.arange(L["N"], dtype=np.int32)
+        assert_parity(y[:, rows], oracle.apply_rows(L, rows, X), gemv_tight(1))
+
+
+def test_gemv_b1_equals_streaming_kernel(env):
+    """The row-split kernel and the streaming kernel's table decode (same
+    tables, other summation order) agree far inside the table bound."""
+    N, K, S, p = 2500, 4096, 2, 41
+    Lref = oracle.encode(synth.layer_weights(N, K, seed=211), S=S, p=p)
+    X = synth.activations(1, K, seed=212)
+    y1 = run_gemv(env, Lref, X)
+    y0 = run_gemv(env, Lref, X, extra_env={"BISCO_GEMV_B1": "0"})
+    assert max_rel_rows(y1, y0) <= 2e-5
