@@ -1,13 +1,16 @@
-"""Decode benchmark: BiSCo-coded Qwen3-8B attention projections on GB300.
+"""Decode benchmark: BiSCo-coded Qwen3-8B linear stack on GB300.
 
-Workload (one "step" = one decode token through every projection):
-  q_proj/o_proj 4096x4096 and k_proj/v_proj 1024x4096 (N x K) for each of
-  the 36 layers of Qwen3-8B, each a distinct random layer (N(0, 0.02)
-  weights with 8 outlier input columns x20, drawn on the device from a
-  seeded generator), coded with d = 8, base + 1 residual stage (S = 2) and
-  1 % int8 protected columns (p = 41); batch 1 bf16 N(0,1) activations.
-  The 144 coded layers hold 1.15 GB, far more than the 129 MB L2, so every
-  step streams its weights from HBM (no L2 flush needed).
+Workload (one "step" = one decode token through every linear layer):
+  the 36 layers x 7 projections of Qwen3-8B -- q_proj/o_proj 4096x4096,
+  k_proj/v_proj 1024x4096, gate_proj/up_proj 12288x4096, down_proj
+  4096x12288 (N x K) -- each a distinct random layer (N(0, 0.02) weights
+  with 8 outlier input columns x20, drawn on the device from a seeded
+  generator), coded with d = 8, base + 1 residual stage (S = 2) and 1 %
+  int8 protected columns; batch 1 bf16 N(0,1) activations.  Four library
+  calls per layer: bisco_gemv_multi(q, k, v), bisco_gemv(o),
+  bisco_gemv_multi(gate, up), bisco_gemv(down).  The 252 coded layers hold
+  5.28 GB, far more than the 129 MB L2, so every step streams its weights
+  from HBM (no L2 flush needed).
 
 Metric: decode GEMV GB/s on compressed bytes (signs + norms + int8 payload +
 scales + indices) and tokens/s; value = whole-job GB/s over all ranks.
@@ -30,6 +33,11 @@ sys.path.insert(0, ROOT)
 
 METRIC = "decode GEMV GB/s (compressed bytes) & tokens/s, % of HBM/tensor roofline"
 ATTN = ("q_proj", "k_proj", "v_proj", "o_proj")
+STACK = ("q_proj", "k_proj", "v_proj", "o_proj", "gate_proj", "up_proj", "down_proj")
+# the four library calls of one layer: name, projections (indices into
+# STACK) that read the same activation, and that activation's width
+CALLS = (("qkv", (0, 1, 2), 4096), ("o", (3,), 4096), ("gate_up", (4, 5), 4096),
+         ("down", (6,), 12288))
 N_LAYERS = 36
 S_STAGES = 2
 RHO_PCT = 1
@@ -46,7 +54,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--mode", choices=("both", "decode", "prefill", "shapes", "dense", "lora",
-                                       "stack", "variants"),
+                                       "stack", "variants", "dominant"),
                     default="both",
                     help="decode: the GEMV step only; prefill: the tcgen05 GEMM only; "
                          "shapes: batch-1 GEMV per Qwen3-8B layer shape; lora: the decode step "
@@ -57,8 +65,6 @@ def parse():
     ap.add_argument("--shape-mb", type=float, default=500.0,
                     help="--mode shapes: MB of distinct coded layers per shape (> L2)")
     ap.add_argument("--prefill-tokens", type=int, default=2048)
-    ap.add_argument("--ungrouped", action="store_true",
-                    help="one bisco_gemv per projection instead of bisco_gemv_multi for q/k/v")
     return ap.parse_args()
 
 
@@ -82,61 +88,50 @@ def tensor_peaks():
         return 1900.0, 1700.0, "fallback"
 
 
-# DRAM bytes (read + write) of one grouped q/k/v launch of the dominant
-# kernel (batch 1, table-lookup decode), from the ncu capture summarised in
-# profiles/ (the file gives the command), valid while the kernel source
-# hashes to the recorded digest.
-DOMINANT_TRAFFIC = {"bytes": 19244800, "gemv_cu_sha256": "2867c80526b9b883c986b2fad2201d855ab36872765081c3540cfba08217d946",
-                    "profile": "profiles/k_gemv_stream_qkv_group_b1.md"}
+# DRAM bytes (read + write) of one launch of the dominant call (bisco_gemv_multi
+# over gate_proj + up_proj of one layer, batch 1), from the ncu capture
+# summarised in profiles/ (the file gives the command), valid while the
+# kernel source hashes to the recorded digest.
+DOMINANT_TRAFFIC = {"bytes": 77178624, "gemv_b1_cu_sha256": "5707433fc765bf66a7ce3b86c617e3882094bc5b2d4ce28663d271626e009908",
+                    "profile": "profiles/k_gemv_b1_gate_up_b1.md"}
 
 
-def decode_kind(B):
-    """Template flag and name of the streaming kernel's decode for batch B."""
-    table = B == 1 and os.environ.get("BISCO_GEMV_LUT", "1")[:1] != "0"
-    return ("1", "table-lookup decode") if table else ("0", "mma decode")
-
-
-def dominant_label(B, ungrouped):
-    """What one timed dominant call launches.  A grouped q/k/v call is one
-    streaming launch while the three layers' staged activations fit shared
-    memory (always at batch 1, where x is staged as lookup tables); past that
-    the library launches each layer on its own, so the label names the call."""
-    flag, kind = decode_kind(B)
-    if ungrouped:
-        return ("k_gemv_stream<4,2,2,1,%s> (bisco_gemv, q_proj/o_proj 4096x4096, batch %d, %s)"
-                % (flag, B, kind))
-    if B == 1:
-        return ("k_gemv_stream<4,2,2,4,%s> (bisco_gemv_multi, q+k+v 6144x4096, batch 1, %s)"
-                % (flag, kind))
-    return ("bisco_gemv_multi call (q+k+v 6144x4096, batch %d, %s): one grouped k_gemv_stream "
-            "launch when the three layers' staged activations fit shared memory, else one launch "
-            "per layer" % (B, kind))
-
-
-def dominant_traffic(B, grouped):
-    """DRAM bytes of one dominant launch from the committed ncu capture, or None
-    when the capture does not describe the kernel being timed (another
-    gemv.cu, batch, decode or launch grouping)."""
+def dominant_traffic(B, call):
+    """DRAM bytes of one dominant launch from the committed ncu capture, or
+    None when the capture does not describe the kernel being timed."""
     import hashlib
-    if DOMINANT_TRAFFIC["bytes"] is None or B != 1 or not grouped or decode_kind(B)[0] != "1":
+    if DOMINANT_TRAFFIC["bytes"] is None or B != 1 or call != "gate_up":
         return None
-    with open(os.path.join(ROOT, "paper_2607_08643_gb300", "csrc", "gemv.cu"), "rb") as f:
+    with open(os.path.join(ROOT, "paper_2607_08643_gb300", "csrc", "gemv_b1.cu"), "rb") as f:
         digest = hashlib.sha256(f.read()).hexdigest()
-    return DOMINANT_TRAFFIC["bytes"] if digest == DOMINANT_TRAFFIC["gemv_cu_sha256"] else None
+    return DOMINANT_TRAFFIC["bytes"] if digest == DOMINANT_TRAFFIC["gemv_b1_cu_sha256"] else None
+
+
+def call_label(call, B):
+    """The kernel one call of the step launches."""
+    names = {"qkv": "bisco_gemv_multi q+k+v 6144x4096", "o": "bisco_gemv o_proj 4096x4096",
+             "gate_up": "bisco_gemv_multi gate+up 24576x4096", "down": "bisco_gemv down_proj 4096x12288"}
+    if B == 1:
+        return "k_gemv_b1 (%s, batch 1, row-split table decode)" % names[call]
+    return "%s, batch %d (k_gemv_stream / k_gemv MMA decode)" % (names[call], B)
 
 
 def workload_config(args):
     return {
-        "workload": "Qwen3-8B attention projections q/k/v/o x %d layers, decode batch %d"
-                    % (args.layers, args.batch),
-        "shapes_NxK": {"q_proj": [4096, 4096], "k_proj": [1024, 4096],
-                       "v_proj": [1024, 4096], "o_proj": [4096, 4096]},
+        "workload": "Qwen3-8B linear stack: %d layers x 7 projections (q/k/v/o/gate/up/down), "
+                    "decode batch %d" % (args.layers, args.batch),
+        "shapes_NxK": {n: list(SHAPES[n]) for n in STACK},
+        "calls_per_layer": "bisco_gemv_multi(q,k,v), bisco_gemv(o), bisco_gemv_multi(gate,up), "
+                           "bisco_gemv(down)",
         "chunk_dim": 8, "stages": S_STAGES, "protected_pct": RHO_PCT, "batch": args.batch,
         "weights": "N(0,0.02) + 8 outlier cols x20, seeded on device",
         "l2": "inputs larger than L2 (distinct coded layers per step, no flush)",
-        "launches": ("one bisco_gemv per projection" if args.ungrouped else
-                     "q/k/v in one bisco_gemv_multi launch per layer, o_proj in its own"),
     }
+
+
+SHAPES = {"q_proj": (4096, 4096), "k_proj": (1024, 4096), "v_proj": (1024, 4096),
+          "o_proj": (4096, 4096), "gate_proj": (12288, 4096), "up_proj": (12288, 4096),
+          "down_proj": (4096, 12288)}
 
 
 # ---------------------------------------------------------------- clocks
@@ -242,55 +237,114 @@ def replica_rates(world, bytes_per_step, batch, steps, ms_total, ms_e2e):
             "e2e_gbs": world * bytes_per_step / (ms_e2e / steps * 1e-3) / 1e9}
 
 
+def build_stack(nl, dev):
+    """nl layers x the 7 projections, coded with S_STAGES and RHO_PCT; list
+    of per-layer lists in STACK order."""
+    import torch
+    from paper_2607_08643_gb300 import bisco, synth
+    out, ws = [], None
+    for l in range(nl):
+        row = []
+        for j, name in enumerate(STACK):
+            N, K = SHAPES[name]
+            W = synth.layer_weights_torch(N, K, seed=1000 * l + j, device=dev)
+            need = bisco.bisco_encode_workspace_bytes(N, K)
+            if ws is None or ws.numel() < need:
+                ws = torch.empty(need, dtype=torch.uint8, device=dev)
+            row.append(bisco.bisco_encode(W, S_STAGES, synth.protected_count(K, RHO_PCT), workspace=ws))
+            del W
+        out.append(row)
+    torch.cuda.synchronize()
+    if bisco.bisco_get_device_error() != bisco.OK:
+        raise RuntimeError("device error while encoding the stack")
+    return out
+
+
+class StackIO:
+    """One flat bf16 input buffer and one flat fp32 output buffer for a batch-B
+    step: per layer the activations of its four calls and the outputs of its
+    seven projections, with views for the calls."""
+
+    def __init__(self, stack, B, dev, seed):
+        import torch
+        nl = len(stack)
+        per_x = sum(k for _, _, k in CALLS) * B
+        per_y = sum(SHAPES[n][0] for n in STACK) * B
+        self.x = torch.empty(nl * per_x, dtype=torch.int16, device=dev)
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(seed)
+        self.x.copy_(torch.randn(self.x.numel(), generator=gen, device=dev).to(torch.bfloat16).view(torch.int16))
+        self.y = torch.empty(nl * per_y, dtype=torch.float32, device=dev)
+        self.xv, self.yv = [], []
+        for l in range(nl):
+            xo, yo, xs, ys = l * per_x, l * per_y, {}, []
+            for name, _, k in CALLS:
+                xs[name] = self.x[xo:xo + k * B].view(B, k)
+                xo += k * B
+            for n in STACK:
+                N = SHAPES[n][0]
+                ys.append(self.y[yo:yo + N * B].view(B, N))
+                yo += N * B
+            self.xv.append(xs)
+            self.yv.append(ys)
+
+
+def stack_step(bisco, stack, io, stream, only=None):
+    """The library calls of one step (or only those of one call type)."""
+    for l, row in enumerate(stack):
+        for name, idx, _ in CALLS:
+            if only is not None and name != only:
+                continue
+            x, ys = io.xv[l][name], [io.yv[l][i] for i in idx]
+            if len(idx) == 1:
+                bisco.bisco_gemv(row[idx[0]], x, y=ys[0], stream=stream)
+            else:
+                bisco.bisco_gemv_multi([row[i] for i in idx], x, ys=ys, stream=stream)
+
+
+def graph_of(torch, stream, fn):
+    with torch.cuda.stream(stream):
+        fn()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            fn()
+    torch.cuda.synchronize()
+    return g
+
+
+def time_graph(torch, stream, g, steps, warmup):
+    """ms per replay: CUDA events on the launching stream over `steps`
+    back-to-back replays, after `warmup` untimed ones."""
+    for _ in range(max(warmup, 3)):
+        g.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(steps):
+            g.replay()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / steps
+
+
 def run_bisco(args, rank, world, local_rank):
+    """The full-stack decode step (see the module docstring): timed line,
+    end-to-end line, per-call rates and the dominant call's roofline."""
     import torch
     import torch.distributed as dist
-    from paper_2607_08643_gb300 import bisco, synth
+    from paper_2607_08643_gb300 import bisco
 
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
     bisco.load()
-    layers = build_layers(args, dev)
+    stack = build_stack(args.layers, dev)
     B = args.batch
-    K = 4096
-    # per step: one activation shared by q/k/v and one for o_proj, per layer
-    n_in = 2 * args.layers
-    x_dev = torch.empty((n_in, B, K), dtype=torch.int16, device=dev)
-    gen = torch.Generator(device=dev)
-    gen.manual_seed(7 + rank)
-    x_dev.copy_(torch.randn((n_in, B, K), generator=gen, device=dev).to(torch.bfloat16).view(torch.int16))
-    outs = [torch.empty((B, L.N), dtype=torch.float32, device=dev) for _, L in layers]
-    y_total = sum(o.numel() for o in outs)
-    y_flat = torch.empty(y_total, dtype=torch.float32, device=dev)
-    views, off = [], 0
-    for o in outs:
-        views.append(y_flat[off:off + o.numel()].view(o.shape))
-        off += o.numel()
-    bytes_step = sum(L.compressed_bytes for _, L in layers)
+    io = StackIO(stack, B, dev, seed=7 + rank)
+    bytes_step = sum(L.compressed_bytes for row in stack for L in row)
     stream = torch.cuda.Stream(device=dev)
-
-    def step():
-        if args.ungrouped:
-            for i, (name, L) in enumerate(layers):
-                li = i // 4
-                xi = 2 * li + (1 if name == "o_proj" else 0)
-                bisco.bisco_gemv(L, x_dev[xi], y=views[i], stream=stream)
-            return
-        for li in range(args.layers):
-            # q/k/v read the same activation: one grouped launch; o_proj its own
-            qkv = [layers[4 * li + j][1] for j in range(3)]
-            bisco.bisco_gemv_multi(qkv, x_dev[2 * li], ys=views[4 * li:4 * li + 3], stream=stream)
-            bisco.bisco_gemv(layers[4 * li + 3][1], x_dev[2 * li + 1], y=views[4 * li + 3],
-                             stream=stream)
-
-    # capture one step (144 launches through the public API) in a CUDA graph
-    with torch.cuda.stream(stream):
-        step()
-        torch.cuda.synchronize()
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=stream):
-            step()
-    torch.cuda.synchronize()
+    g = graph_of(torch, stream, lambda: stack_step(bisco, stack, io, stream))
     if bisco.bisco_get_device_error(stream) != bisco.OK:
         raise RuntimeError("device error in warm-up")
 
@@ -319,14 +373,14 @@ def run_bisco(args, rank, world, local_rank):
         raise RuntimeError("device error in timed region")
 
     # end to end: pinned host inputs in, graph of public-API calls, outputs out
-    x_host = torch.empty(x_dev.shape, dtype=torch.int16, pin_memory=True)
-    x_host.copy_(x_dev.cpu())
-    y_host = torch.empty(y_total, dtype=torch.float32, pin_memory=True)
+    x_host = torch.empty(io.x.shape, dtype=torch.int16, pin_memory=True)
+    x_host.copy_(io.x.cpu())
+    y_host = torch.empty(io.y.shape, dtype=torch.float32, pin_memory=True)
     for _ in range(2):
         with torch.cuda.stream(stream):
-            x_dev.copy_(x_host, non_blocking=True)
+            io.x.copy_(x_host, non_blocking=True)
             g.replay()
-            y_host.copy_(y_flat, non_blocking=True)
+            y_host.copy_(io.y, non_blocking=True)
     barrier()
     t0 = time.perf_counter()
     f0 = torch.cuda.Event(enable_timing=True)
@@ -334,65 +388,187 @@ def run_bisco(args, rank, world, local_rank):
     with torch.cuda.stream(stream):
         f0.record(stream)
         for _ in range(args.steps):
-            x_dev.copy_(x_host, non_blocking=True)
+            io.x.copy_(x_host, non_blocking=True)
             g.replay()
-            y_host.copy_(y_flat, non_blocking=True)
+            y_host.copy_(io.y, non_blocking=True)
         f1.record(stream)
     stream.synchronize()
     wall_e2e = time.perf_counter() - t0
     barrier()
     ms_e2e = max(f0.elapsed_time(f1), wall_e2e * 1e3)
-
     ms_total, ms_e2e = max_over_ranks([ms_total, ms_e2e], world, device=dev)
 
-    # dominant kernel: the grouped q/k/v launch (60 % of the step's bytes;
-    # the q/o projections when ungrouped), timed alone on the same stream
-    if args.ungrouped:
-        dom_calls = [[i] for i, (name, _) in enumerate(layers) if name in ("q_proj", "o_proj")]
-    else:
-        dom_calls = [[4 * li, 4 * li + 1, 4 * li + 2] for li in range(args.layers)]
-    with torch.cuda.stream(stream):
-        g_dom = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g_dom, stream=stream):
-            for idx in dom_calls:
-                li = idx[0] // 4
-                xi = 2 * li + (1 if layers[idx[0]][0] == "o_proj" else 0)
-                if len(idx) == 1:
-                    bisco.bisco_gemv(layers[idx[0]][1], x_dev[xi], y=views[idx[0]], stream=stream)
-                else:
-                    bisco.bisco_gemv_multi([layers[i][1] for i in idx], x_dev[xi],
-                                           ys=[views[i] for i in idx], stream=stream)
-    for _ in range(3):
-        g_dom.replay()
-    barrier()
-    d0 = torch.cuda.Event(enable_timing=True)
-    d1 = torch.cuda.Event(enable_timing=True)
-    with torch.cuda.stream(stream):
-        d0.record(stream)
-        for _ in range(args.steps):
-            g_dom.replay()
-        d1.record(stream)
-    barrier()
-    us_dom = d0.elapsed_time(d1) * 1e3 / (args.steps * len(dom_calls))
-    bytes_dom = sum(layers[i][1].compressed_bytes for i in dom_calls[0])
-
-    rates = replica_rates(world, bytes_step, B, args.steps, ms_total, ms_e2e)
-    ms_step, gbs, tok_s, e2e_gbs = (rates["ms_per_step"], rates["gbs"], rates["tokens_per_s"],
-                                    rates["e2e_gbs"])
-    launches = len(layers) if args.ungrouped else 2 * args.layers
+    # each call type alone (a graph of its launches over all layers): the
+    # dominant one is the roofline line
+    per_call = {}
+    for name, idx, _ in CALLS:
+        gc = graph_of(torch, stream, lambda n=name: stack_step(bisco, stack, io, stream, only=n))
+        ms = time_graph(torch, stream, gc, args.steps, args.warmup)
+        nbytes = sum(stack[0][i].compressed_bytes for i in idx)
+        us = ms * 1e3 / len(stack)
+        per_call[name] = {"kernel": call_label(name, B), "bytes_per_launch": nbytes,
+                          "us_per_launch": us, "gbs": nbytes / (us * 1e-6) / 1e9,
+                          "launches_timed": args.steps * len(stack)}
+        del gc
+    if bisco.bisco_get_device_error(stream) != bisco.OK:
+        raise RuntimeError("device error in the per-call timing")
+    dom = max(per_call, key=lambda n: per_call[n]["us_per_launch"])
     peak, peak_kind = peaks()
-    achieved = bytes_dom / (us_dom * 1e-6) / 1e9
+    for v in per_call.values():
+        v["frac_of_hbm"] = v["gbs"] / peak
+    d = per_call[dom]
+    rates = replica_rates(world, bytes_step, B, args.steps, ms_total, ms_e2e)
     return dict(
-        value=gbs, ms_per_step=ms_step, tokens_per_s=tok_s, bytes_per_step=bytes_step,
-        launches=launches, e2e_gbs=e2e_gbs, h2d=x_dev.numel() * 2, d2h=y_total * 4,
-        roofline={"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                  "frac": achieved / peak, "traffic": dominant_traffic(B, not args.ungrouped),
+        value=rates["gbs"], ms_per_step=rates["ms_per_step"], tokens_per_s=rates["tokens_per_s"],
+        bytes_per_step=bytes_step, launches=len(CALLS) * len(stack), e2e_gbs=rates["e2e_gbs"],
+        h2d=io.x.numel() * 2, d2h=io.y.numel() * 4,
+        roofline={"bound": "hbm", "achieved": d["gbs"], "peak": peak, "unit": "GB/s",
+                  "frac": d["gbs"] / peak, "traffic": dominant_traffic(B, dom),
                   "peak_source": "%s hbm_gbs (MEASURED_PEAKS.json, copy burst)" % peak_kind
                   if peak_kind == "measured" else "fallback 6.8 TB/s",
-                  "kernel": dominant_label(B, args.ungrouped),
-                  "bytes_per_launch": bytes_dom, "us_per_launch": us_dom,
-                  "launches_timed": args.steps * len(dom_calls)},
-        clocks=clk, ms_e2e=ms_e2e / args.steps)
+                  "kernel": d["kernel"], "bytes_per_launch": d["bytes_per_launch"],
+                  "us_per_launch": d["us_per_launch"], "launches_timed": d["launches_timed"],
+                  "step_frac_of_hbm": rates["gbs"] / world / peak},
+        per_call=per_call, clocks=clk, ms_e2e=ms_e2e / args.steps, stack=stack, io=io,
+        stream=stream)
+
+
+def run_sweeps(args, stack, stream, dev):
+    """Sub-records on the same coded stack: the decode step at batch 4 and 16
+    (GEMV), and the GEMV/GEMM crossover (bisco_gemm on every projection at
+    M = 1, 4, 16, 64 through the decode kernels and 128 on the tensor
+    cores)."""
+    import torch
+    from paper_2607_08643_gb300 import bisco
+    peak, _ = peaks()
+    total = sum(L.compressed_bytes for row in stack for L in row)
+    steps, warm = max(3, min(args.steps, 10)), 3
+    sweep = []
+    for B in (4, 16):
+        io = StackIO(stack, B, dev, seed=100 + B)
+        g = graph_of(torch, stream, lambda: stack_step(bisco, stack, io, stream))
+        ms = time_graph(torch, stream, g, steps, warm)
+        gbs = total / (ms * 1e-3) / 1e9
+        sweep.append({"batch": B, "ms_per_step": ms, "gbs": gbs, "frac_of_hbm": gbs / peak,
+                      "tokens_per_s": B / (ms * 1e-3)})
+        del g, io
+    cross = []
+    for M in (1, 4, 16, 64, 128):
+        io = StackIO(stack, M, dev, seed=200 + M)
+        need = max(bisco.bisco_gemm_workspace_bytes(L, M) for row in stack for L in row)
+        ws = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+
+        def step():
+            for l, row in enumerate(stack):
+                for name, idx, _ in CALLS:
+                    for i in idx:
+                        bisco.bisco_gemm(row[i], io.xv[l][name], Y=io.yv[l][i], workspace=ws,
+                                         stream=stream)
+        g = graph_of(torch, stream, step)
+        ms = time_graph(torch, stream, g, steps, warm)
+        cross.append({"tokens": M, "ms_per_step": ms, "tokens_per_s": M / (ms * 1e-3),
+                      "gbs": total / (ms * 1e-3) / 1e9,
+                      "path": "tcgen05 GEMM" if M > 64 else "decode kernels"})
+        del g, io, ws
+    if bisco.bisco_get_device_error(stream) != bisco.OK:
+        raise RuntimeError("device error in the sweeps")
+    torch.cuda.empty_cache()
+    return {"decode_batch_sweep": sweep, "gemv_gemm_crossover": cross}
+
+
+def run_dense_stack(args, stack, stream, dev):
+    """The paper's own inference path on the same stack: every coded layer
+    decoded once to dense bf16 (bisco_decode_dense), then the step as one
+    cuBLAS product (torch.matmul) per call of the fused step (q/k/v and
+    gate/up concatenated), at batch 1 and 16."""
+    import torch
+    from paper_2607_08643_gb300 import bisco
+    dense = []
+    for row in stack:
+        mats = []
+        for _, idx, k in CALLS:
+            W = torch.empty((sum(row[i].N for i in idx), k), dtype=torch.bfloat16, device=dev)
+            mats.append((idx, W))
+        dense.append(mats)
+
+    def materialise():
+        for row, mats in zip(stack, dense):
+            for idx, W in mats:
+                r0 = 0
+                for i in idx:
+                    bisco.bisco_decode_dense(row[i], "bf16", out=W[r0:r0 + row[i].N], stream=stream)
+                    r0 += row[i].N
+
+    with torch.cuda.stream(stream):
+        materialise()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        materialise()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    if bisco.bisco_get_device_error(stream) != bisco.OK:
+        raise RuntimeError("device error in bisco_decode_dense")
+    ms_mat = e0.elapsed_time(e1)
+    dense_bytes = sum(W.numel() * 2 for mats in dense for _, W in mats)
+    out = {"how": "bisco_decode_dense to bf16 once, then torch.matmul (cuBLAS) per call: q/k/v and "
+                  "gate/up concatenated, o and down alone, CUDA graph of the step",
+           "materialise_ms": ms_mat, "dense_bytes_per_step": dense_bytes}
+    steps = max(3, min(args.steps, 10))
+    for B in (1, 16):
+        xs = [[torch.randn((k, B), device=dev).to(torch.bfloat16) for _, _, k in CALLS] for _ in stack]
+        ys = [[torch.empty((W.shape[0], B), dtype=torch.bfloat16, device=dev) for _, W in mats] for mats in dense]
+
+        def step():
+            for l, mats in enumerate(dense):
+                for c, (_, W) in enumerate(mats):
+                    torch.matmul(W, xs[l][c], out=ys[l][c])
+        g = graph_of(torch, stream, step)
+        ms = time_graph(torch, stream, g, steps, 3)
+        out["batch_%d" % B] = {"ms_per_step": ms, "tokens_per_s": B / (ms * 1e-3),
+                               "dense_gbs": dense_bytes / (ms * 1e-3) / 1e9}
+        del g, xs, ys
+    del dense
+    torch.cuda.empty_cache()
+    return out
+
+
+def run_prefill_stack(args, stack, stream, dev):
+    """Prefill on the tensor cores: bisco_gemm on the 7 projections of the
+    first 4 layers of the stack at --prefill-tokens tokens, a CUDA graph of
+    the 28 calls; TFLOP/s on the algorithmic 2*M*N*K."""
+    import torch
+    from paper_2607_08643_gb300 import bisco
+    M = args.prefill_tokens
+    rows = stack[:4]
+    X = {k: torch.randn((M, k), device=dev).to(torch.bfloat16).view(torch.int16) for k in (4096, 12288)}
+    Ys = [[torch.empty((M, L.N), device=dev) for L in row] for row in rows]
+    ws = torch.empty(max(bisco.bisco_gemm_workspace_bytes(L, M) for row in rows for L in row),
+                     dtype=torch.uint8, device=dev)
+
+    def step():
+        for row, ys in zip(rows, Ys):
+            for L, Y in zip(row, ys):
+                bisco.bisco_gemm(L, X[L.K], Y=Y, workspace=ws, stream=stream)
+    g = graph_of(torch, stream, step)
+    ms = time_graph(torch, stream, g, max(3, min(args.steps, 10)), 3)
+    if bisco.bisco_get_device_error(stream) != bisco.OK:
+        raise RuntimeError("device error in prefill")
+    flops = sum(2.0 * M * L.N * L.K for row in rows for L in row)
+    tf = flops / (ms * 1e-3) / 1e12
+    burst, sustained, kind = tensor_peaks()
+    del g, X, Ys, ws
+    torch.cuda.empty_cache()
+    return {"metric": "prefill GEMM TFLOP/s (2*M*N*K, decoded weight never written)",
+            "workload": "Qwen3-8B 7 projections x 4 layers, %d tokens, S=%d, %d%% protected"
+                        % (M, S_STAGES, RHO_PCT),
+            "value": tf, "unit": "TFLOP/s", "ms_per_step": ms,
+            "roofline": {"bound": "tensor", "achieved": tf, "peak": burst, "unit": "TFLOP/s",
+                         "frac": tf / burst, "frac_of_sustained": tf / sustained,
+                         "peak_source": "%s bf16_tflops (MEASURED_PEAKS.json; fp16 rate = bf16)" % kind,
+                         "kernels": "k_gemm_prep + k_gemm per projection"},
+            "dtype": "f16 x f16 -> f32"}
 
 
 # ---------------------------------------------------------------- prefill
@@ -700,116 +876,6 @@ def run_shapes(args, local_rank):
     return out
 
 
-# ------------------------------------------------------------------ stack
-
-STACK = ("q_proj", "k_proj", "v_proj", "o_proj", "gate_proj", "up_proj", "down_proj")
-
-
-def run_stack(args, local_rank):
-    """The full linear stack of Qwen3-8B: 7 projections x --layers layers,
-    each a distinct random layer (N(0,0.02) + 8 outlier columns x20), d = 8,
-    S = 2, 1 % protected columns (5.28 GB coded for 36 layers, far more than
-    L2).  Decode sweep at batch 1, 4 and 16 through bisco_gemv_multi (q/k/v;
-    gate/up) and bisco_gemv (o; down), four launches per layer; then the
-    GEMV/GEMM crossover, bisco_gemm on every projection at M = 1, 4, 16, 64
-    (decode kernels) and 128 (tensor cores).  Each is a CUDA graph of the
-    whole stack, CUDA events over `steps` replays."""
-    import torch
-    from paper_2607_08643_gb300 import bisco, synth
-    dev = torch.device("cuda", local_rank)
-    torch.cuda.set_device(dev)
-    layers = []
-    ws = None
-    for l in range(args.layers):
-        for j, name in enumerate(STACK):
-            N, K = synth.QWEN3_8B_SHAPES[name]
-            p = synth.protected_count(K, RHO_PCT)
-            W = synth.layer_weights_torch(N, K, seed=1000 * l + j, device=dev)
-            need = bisco.bisco_encode_workspace_bytes(N, K)
-            if ws is None or ws.numel() < need:
-                ws = torch.empty(need, dtype=torch.uint8, device=dev)
-            layers.append(bisco.bisco_encode(W, S_STAGES, p, workspace=ws))
-            del W
-    torch.cuda.synchronize()
-    if bisco.bisco_get_device_error() != bisco.OK:
-        raise RuntimeError("device error while encoding the stack")
-    total = sum(L.compressed_bytes for L in layers)
-    peak, peak_kind = peaks()
-    gen = torch.Generator(device=dev)
-    gen.manual_seed(77)
-    stream = torch.cuda.Stream(device=dev)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-
-    def timed(step):
-        with torch.cuda.stream(stream):
-            step()
-            torch.cuda.synchronize()
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g, stream=stream):
-                step()
-        torch.cuda.synchronize()
-        for _ in range(max(args.warmup, 3)):
-            g.replay()
-        torch.cuda.synchronize()
-        with torch.cuda.stream(stream):
-            e0.record(stream)
-            for _ in range(args.steps):
-                g.replay()
-            e1.record(stream)
-        torch.cuda.synchronize()
-        if bisco.bisco_get_device_error(stream) != bisco.OK:
-            raise RuntimeError("device error in the stack step")
-        return e0.elapsed_time(e1) / args.steps
-
-    def inputs(B):
-        xk = torch.randn((B, 4096), generator=gen, device=dev).to(torch.bfloat16).view(torch.int16)
-        xf = torch.randn((B, 12288), generator=gen, device=dev).to(torch.bfloat16).view(torch.int16)
-        ys = {nm: torch.empty((B, synth.QWEN3_8B_SHAPES[nm][0]), device=dev) for nm in STACK}
-        return xk, xf, ys
-
-    sweep = []
-    for B in (1, 4, 16):
-        xk, xf, ys = inputs(B)
-
-        def step():
-            for l in range(args.layers):
-                Ls = layers[7 * l:7 * l + 7]
-                bisco.bisco_gemv_multi(Ls[0:3], xk, ys=[ys[nm] for nm in STACK[0:3]], stream=stream)
-                bisco.bisco_gemv(Ls[3], xk, y=ys["o_proj"], stream=stream)
-                bisco.bisco_gemv_multi(Ls[4:6], xk, ys=[ys[nm] for nm in STACK[4:6]], stream=stream)
-                bisco.bisco_gemv(Ls[6], xf, y=ys["down_proj"], stream=stream)
-        ms = timed(step)
-        gbs = total / (ms * 1e-3) / 1e9
-        sweep.append({"batch": B, "ms_per_step": ms, "gbs": gbs, "frac_of_hbm": gbs / peak,
-                      "tokens_per_s": B / (ms * 1e-3), "calls_per_step": 4 * args.layers})
-        del xk, xf, ys
-    cross = []
-    for M in (1, 4, 16, 64, 128):
-        xk, xf, ys = inputs(M)
-        need = max(bisco.bisco_gemm_workspace_bytes(L, M) for L in layers)
-        gws = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
-
-        def step():
-            for l in range(args.layers):
-                for j, nm in enumerate(STACK):
-                    L = layers[7 * l + j]
-                    bisco.bisco_gemm(L, xf if nm == "down_proj" else xk, Y=ys[nm],
-                                     workspace=gws, stream=stream)
-        ms = timed(step)
-        cross.append({"tokens": M, "ms_per_step": ms, "tokens_per_s": M / (ms * 1e-3),
-                      "gbs": total / (ms * 1e-3) / 1e9,
-                      "path": "tcgen05 GEMM" if M > 64 else "decode kernels"})
-        del xk, xf, ys, gws
-    return {"metric": "Qwen3-8B linear stack decode sweep and GEMV/GEMM crossover",
-            "unit": "GB/s", "layers": args.layers, "projections": list(STACK),
-            "compressed_bytes": total, "hbm_peak_gbs": peak, "peak_source": peak_kind,
-            "decode": sweep, "crossover_gemm": cross,
-            "config": {"workload": "Qwen3-8B linear stack, 7 projections x %d layers" % args.layers,
-                       "chunk_dim": 8, "stages": S_STAGES, "protected_pct": RHO_PCT,
-                       "weights": "N(0,0.02) + 8 outlier cols x20, seeded on device",
-                       "l2": "inputs larger than L2 (distinct coded layers per step, no flush)"}}
-
-
 # --------------------------------------------------------------- variants
 
 def run_variants(args, local_rank):
@@ -1000,64 +1066,124 @@ def run_variants(args, local_rank):
 
 # ------------------------------------------------------------ CPU oracle
 
-def cpu_oracle_sample(seconds, batch):
-    """The fp64 oracle (decode to dense + naive matmul, single thread) on a
-    bounded sample of the same workload: whole projections of layer 0, in
-    q/k/v/o order, repeated until `seconds` of CPU time have passed."""
-    import numpy as np
+# Rows of each projection shape a CPU worker codes and applies repeatedly: a
+# bounded sample of the same workload (every byte of a coded layer costs the
+# oracle the same work, so a slab of rows stands for the layer).
+ORACLE_ROWS = {4096: 256, 12288: 128}
+_WORKER_LAYER = {}
+
+
+def _oracle_worker(task):
+    """One CPU process of the oracle baseline: codes a slab of rows of one
+    projection shape with the fp64 oracle (once per process), then applies it
+    to a batch of activations (decode to dense + naive matmul) until
+    `seconds` have passed.  Returns (compressed bytes processed, seconds,
+    calls)."""
+    name, seconds, batch = task
     import oracle
     from paper_2607_08643_gb300 import synth
-    layers = []
-    for j, name in enumerate(ATTN):
-        N, K = synth.QWEN3_8B_SHAPES[name]
-        p = synth.protected_count(K, RHO_PCT)
-        W = synth.layer_weights(N, K, seed=j)
-        layers.append(oracle.encode(W, S=S_STAGES, p=p))
-    X = synth.activations(batch, 4096, seed=99)
-    done_bytes, n_calls, t0 = 0, 0, time.perf_counter()
+    N, K = SHAPES[name]
+    key = (name, batch)
+    if key not in _WORKER_LAYER:
+        rows = ORACLE_ROWS[K]
+        L = oracle.encode(synth.layer_weights(rows, K, seed=STACK.index(name)), S=S_STAGES,
+                          p=synth.protected_count(K, RHO_PCT))
+        _WORKER_LAYER[key] = (L, synth.activations(batch, K, seed=99))
+    L, X = _WORKER_LAYER[key]
+    per_call = S_STAGES * L["N"] * (K // 8) * 3 + L["N"] * L["p"] + 6 * L["p"]
+    n, t0 = 0, time.perf_counter()
     while True:
-        L = layers[n_calls % 4]
         oracle.gemv(L, X)
-        done_bytes += S_STAGES * L["N"] * (L["K"] // 8) * 3 + L["N"] * L["p"] + 6 * L["p"]
-        n_calls += 1
+        n += 1
         el = time.perf_counter() - t0
-        if el >= seconds and n_calls >= 1:
-            break
-    return {"value": done_bytes / el / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
-            "sample": "%d whole-projection calls of layer 0 (q/k/v/o cycle), %.1f s, "
-                      "fp64 decode-to-dense + naive matmul, batch %d" % (n_calls, el, batch)}
+        if el >= seconds:
+            return n * per_call, el, n
+
+
+class OraclePool:
+    """The oracle on `workers` host processes (spawned, so that no process
+    forks after CUDA work), each on one projection shape of the stack in
+    turn; rate = all bytes / the slowest worker's time."""
+
+    def __init__(self, workers):
+        import multiprocessing as mp
+        self.workers = workers
+        self.pool = mp.get_context("spawn").Pool(workers) if workers > 1 else None
+
+    def sample(self, seconds, batch):
+        tasks = [(STACK[w % len(STACK)], seconds, batch) for w in range(self.workers)]
+        res = self.pool.map(_oracle_worker, tasks) if self.pool else [_oracle_worker(tasks[0])]
+        nbytes = sum(r[0] for r in res)
+        el = max(r[1] for r in res)
+        return nbytes / el / 1e9, el, sum(r[2] for r in res)
+
+    def close(self):
+        if self.pool:
+            self.pool.close()
+            self.pool.join()
+
+
+def host_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(seconds, batch):
+    """The fp64 oracle as it stands on the host cores, single-process and on
+    every core, on a bounded sample of the stack's workload."""
+    cores = host_cores()
+    one = OraclePool(1)
+    gbs1, el1, n1 = one.sample(seconds / 2, batch)
+    allp = OraclePool(cores)
+    allp.sample(0.5, batch)   # every worker codes its slab once
+    gbs, el, n = allp.sample(seconds / 2, batch)
+    allp.close()
+    slab = ", ".join("%d rows of %s" % (ORACLE_ROWS[SHAPES[nm][1]], nm) for nm in STACK)
+    return {"value": gbs, "unit": "GB/s", "cores": cores, "kind": "oracle",
+            "sample": "fp64 decode-to-dense + naive matmul of coded row slabs (%s), one shape "
+                      "per process, %d processes for %.1f s (%d calls), batch %d" % (slab, cores, el, n, batch),
+            "single_core": {"value": gbs1, "unit": "GB/s", "cores": 1,
+                            "sample": "q_proj slab, %.1f s (%d calls)" % (el1, n1)},
+            "host_cores_available": cores}
 
 
 def run_reference(args, rank, world):
-    """Reference arm: the CPU oracle as it stands, on the same metric."""
+    """Reference arm: the CPU oracle as it stands, on every host core, on the
+    same metric; each step is a bounded sample of the workload (all workers
+    for a fixed time), timed as a step."""
     if rank != 0:
         return None
-    per_step = max(2.0, min(20.0, 120.0 / max(1, args.steps + args.warmup)))
+    cores = host_cores()
+    pool = OraclePool(cores)
+    per_step = max(0.5, min(10.0, 120.0 / max(1, args.steps + args.warmup)))
     for _ in range(args.warmup):
-        cpu_oracle_sample(min(per_step, 2.0), args.batch)
-    vals, t0 = [], time.perf_counter()
+        pool.sample(per_step, args.batch)
+    vals, secs, t0 = [], [], time.perf_counter()
     for _ in range(args.steps):
-        vals.append(cpu_oracle_sample(per_step, args.batch))
-    el = time.perf_counter() - t0
-    gbs = statistics.median(v["value"] for v in vals)
-    bytes_step_full = 0
-    for name in ATTN:
-        N, K = (4096, 4096) if name in ("q_proj", "o_proj") else (1024, 4096)
-        bytes_step_full += S_STAGES * N * (K // 8) * 3 + N * 41 + 6 * 41
-    bytes_step_full *= args.layers
-    ms_step = bytes_step_full / (gbs * 1e9) * 1e3
-    line = {
+        gbs, el, _ = pool.sample(per_step, args.batch)
+        vals.append(gbs)
+        secs.append(el)
+    wall = time.perf_counter() - t0
+    pool.close()
+    gbs = statistics.median(vals)
+    slab = ", ".join("%d rows of %s" % (ORACLE_ROWS[SHAPES[nm][1]], nm) for nm in STACK)
+    return {
         "impl": "reference", "metric": METRIC, "value": gbs, "unit": "GB/s", "n_gpus": 1,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": statistics.median(secs) * 1e3,
+        "step": "a bounded sample of the workload: every host core runs the oracle on coded row "
+                "slabs of one projection shape for %.1f s; value = the sample's compressed bytes "
+                "/ its time" % per_step,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": workload_config(args),
-        "tokens_per_s": args.batch / (ms_step * 1e-3),
-        "cpu_baseline": {"kind": "oracle", "cores": 1, "value": gbs, "unit": "GB/s",
-                         "sample": vals[0]["sample"] + "; each step a bounded sample"},
+        "cpu_baseline": {"kind": "oracle", "cores": cores, "value": gbs, "unit": "GB/s",
+                         "sample": "fp64 decode-to-dense + naive matmul on %s; %d processes"
+                                   % (slab, cores)},
         "e2e": {"value": gbs, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
-        "wall_s": el,
+        "wall_s": wall,
     }
-    return line
 
 
 def main():
@@ -1091,11 +1217,26 @@ def main():
             print(json.dumps(dict(vr, n_gpus=world, steps=args.steps, warmup=args.warmup,
                                   data="synthetic", config=workload_config(args))))
         return
-    if args.mode == "stack":
-        st = run_stack(args, local_rank)
-        if rank == 0:
-            print(json.dumps(dict(st, n_gpus=world, steps=args.steps, warmup=args.warmup,
-                                  data="synthetic")))
+    if args.mode == "dominant":
+        # the dominant call alone, launched directly (no graph), for an ncu
+        # capture of one launch on a small stack: python bench.py --mode
+        # dominant --layers 2 --steps 2 --warmup 1
+        import torch
+        from paper_2607_08643_gb300 import bisco
+        dev = torch.device("cuda", local_rank)
+        torch.cuda.set_device(dev)
+        stack = build_stack(args.layers, dev)
+        io = StackIO(stack, args.batch, dev, seed=7)
+        stream = torch.cuda.Stream(device=dev)
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup + args.steps):
+                stack_step(bisco, stack, io, stream, only="gate_up")
+        torch.cuda.synchronize()
+        if bisco.bisco_get_device_error(stream) != bisco.OK:
+            raise RuntimeError("device error")
+        print(json.dumps({"mode": "dominant", "kernel": call_label("gate_up", args.batch),
+                          "launches": len(stack) * (args.warmup + args.steps),
+                          "bytes_per_launch": sum(stack[0][i].compressed_bytes for i in (4, 5))}))
         return
     if args.mode == "lora":
         lr = run_lora(args, local_rank)
@@ -1122,14 +1263,17 @@ def main():
     # CPU baseline first (before any CUDA work), rank 0 at N = 1 only
     cpu = None
     if world == 1 and rank == 0 and not args.no_cpu_baseline:
-        cpu = cpu_oracle_sample(args.cpu_seconds, args.batch)
+        cpu = cpu_baseline(args.cpu_seconds, args.batch)
     r = run_bisco(args, rank, world, local_rank)
-    prefill = run_prefill(args, local_rank) if args.mode == "both" else None
-    dense_cmp = None
-    if args.mode == "both" and world == 1:
-        dn = run_dense(args, local_rank)
-        dense_cmp = dict(dn, fused_tokens_per_s=r["tokens_per_s"],
-                         fused_over_dense=r["tokens_per_s"] / dn["tokens_per_s"])
+    subs, dense_cmp, prefill = {}, None, None
+    if args.mode in ("both", "stack") and world == 1:
+        import torch
+        dev = torch.device("cuda", local_rank)
+        subs = run_sweeps(args, r["stack"], r["stream"], dev)
+        prefill = run_prefill_stack(args, r["stack"], r["stream"], dev)
+        dense_cmp = run_dense_stack(args, r["stack"], r["stream"], dev)
+        dense_cmp["fused_over_dense_batch1"] = (r["tokens_per_s"] / (args.batch / (dense_cmp["batch_1"]["ms_per_step"] * 1e-3))
+                                                if args.batch == 1 else None)
     if rank == 0:
         line = {
             "metric": METRIC, "value": r["value"], "unit": "GB/s", "n_gpus": world,
@@ -1140,17 +1284,20 @@ def main():
             "e2e": {"value": r["e2e_gbs"], "unit": "GB/s",
                     "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"],
                     "how": "pinned H2D of the step's activations + CUDA graph of the step's "
-                           "bisco_gemv_multi (q/k/v) and bisco_gemv (o) calls + D2H of all "
-                           "outputs, per step",
+                           "4 calls per layer (bisco_gemv_multi q/k/v, bisco_gemv o, "
+                           "bisco_gemv_multi gate/up, bisco_gemv down) + D2H of all outputs, "
+                           "per step",
                     "ms_per_step": r["ms_e2e"]},
             "gpu_launches": r["launches"] * args.steps,
             "roofline": r["roofline"],
+            "per_call": r["per_call"],
             "clocks": r["clocks"],
             "cpu_baseline": cpu,
             "parallelism": "replicas" if world > 1 else "single GPU",
             "prefill": prefill,
             "dense_comparison": dense_cmp,
         }
+        line.update(subs)
         print(json.dumps(line))
     if world > 1:
         import torch.distributed as dist
