@@ -167,11 +167,53 @@ __device__ __forceinline__ void b1_issue(bool leader, uint32_t slot, uint32_t ba
         : "memory");
 }
 
-// D item slots per warp; NSPAN 4096-column spans per row (0: a.nspan, at
-// run time).  Both fixed at compile time make every ring address an
-// immediate offset.
+// The table of one 4096-column span (32 KB): job J of warp J (16 jobs for
+// 16 warps), lane l: chunk 256*h + 8l + j of the span, h = J >> 3 & 1,
+// j = J & 7, from its 8 activations xv (bf16, the span's column base c0)
+// with the layer's protected columns (bits of pm) zeroed.
+__device__ __forceinline__ void b1_table_job(uint32_t tab, const uint32_t *pm, int c0, int J, int lane,
+                                             uint4 xv) {
+    const int h = (J >> 3) & 1, j = J & 7;
+    const int c = c0 + h * 256 + 8 * lane + j;   // chunk of the layer
+    const uint32_t m = (pm[c >> 2] >> ((c & 3) * 8)) & 0xFFu;
+    float e[8] = {__uint_as_float(xv.x << 16), __uint_as_float(xv.x & 0xFFFF0000u),
+                  __uint_as_float(xv.y << 16), __uint_as_float(xv.y & 0xFFFF0000u),
+                  __uint_as_float(xv.z << 16), __uint_as_float(xv.z & 0xFFFF0000u),
+                  __uint_as_float(xv.w << 16), __uint_as_float(xv.w & 0xFFFF0000u)};
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+        if ((m >> k) & 1u) e[k] = 0.f;
+    // signed sums of element pairs: index bit 0 negates the first, bit 1 the second
+    float p01[2][4], p23[2][4];
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+        const float x0 = e[4 * hh], x1 = e[4 * hh + 1], x2 = e[4 * hh + 2], x3 = e[4 * hh + 3];
+        p01[hh][0] = x0 + x1; p01[hh][1] = x1 - x0; p01[hh][2] = x0 - x1; p01[hh][3] = -(x0 + x1);
+        p23[hh][0] = x2 + x3; p23[hh][1] = x3 - x2; p23[hh][2] = x2 - x3; p23[hh][3] = -(x2 + x3);
+    }
+    const int P = h * 256 + 32 * j + lane;
+    const uint32_t dst = tab + static_cast<uint32_t>((P >> 6) * 4096 + (P & 63) * 4);
+#pragma unroll
+    for (int v = 0; v < 16; ++v) {
+        const __half2 hv = __floats2half2_rn(p01[0][v & 3] + p23[0][v >> 2], p01[1][v & 3] + p23[1][v >> 2]);
+        asm volatile("st.shared.b32 [%0], %1;" ::"r"(dst + v * 256), "r"(*reinterpret_cast<const uint32_t *>(&hv)));
+    }
+}
+
+// x of job J's chunk in span sp (see b1_table_job).
+__device__ __forceinline__ uint4 b1_table_x(const uint16_t *x, int sp, int J, int lane) {
+    const int c = sp * kB1Span + ((J >> 3) & 1) * 256 + 8 * lane + (J & 7);
+    return *reinterpret_cast<const uint4 *>(x + 8 * c);
+}
+
+// D item slots per warp; NSPAN 4096-column spans per row (0: a.nspan > 1,
+// at run time).  With one span, every ring address is an immediate offset;
+// with several, a CTA holds the table of one span at a time and walks its
+// items span by span, rebuilding the table between spans (x of the next
+// span is loaded while the current one is decoded).
 template <int D, int NSPAN>
 __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_constant__ B1Args a) {
+    static_assert(kB1Warps == 16, "one table job per warp per span");
     constexpr int kB1Threads = kB1Warps * 32;
     extern __shared__ unsigned char smem_raw[];
     unsigned char *sm = align_smem<4096>(smem_raw);
@@ -191,7 +233,6 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
     const int ra = static_cast<int>(static_cast<int64_t>(N) * ci / L.ctas);
     const int rb = static_cast<int>(static_cast<int64_t>(N) * (ci + 1) / L.ctas);
     const int nrows = rb - ra;
-    const int nitems = nrows * S * nspan;
     const uint8_t *const codes = L.codes;
     const uint16_t *const norms = L.norms;
     const int8_t *const q8 = L.q8;
@@ -201,30 +242,38 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
     int *spidx = reinterpret_cast<int *>(sm + a.off_pidx);        // [p]
     float *ssc = reinterpret_cast<float *>(spidx + (p + 3) / 4 * 4);
     float *sx = reinterpret_cast<float *>(sm + a.off_sx);         // scale * x [p]
-    float *part = reinterpret_cast<float *>(sm + a.off_part);     // [nitems]
+    float *part = reinterpret_cast<float *>(sm + a.off_part);     // [S * nrows * nspan]
     int8_t *q8s = reinterpret_cast<int8_t *>(sm + a.off_q8);
     const uint64_t pol = l2_evict_first_policy();
 
-    // this warp's items [kb, kb + cnt), in memory order, through its ring.
-    // Within a stage the items of consecutive rows are consecutive in memory
-    // (512 elements apart); a stage boundary jumps to the next [N][K/8] plane.
-    const int kb = static_cast<int>(static_cast<int64_t>(nitems) * warp / kB1Warps);
-    const int cnt = static_cast<int>(static_cast<int64_t>(nitems) * (warp + 1) / kB1Warps) - kb;
-    const int per_stage = nrows * nspan;
+    // Items, span by span; within a span stage by stage, row by row (the
+    // order of the [S][N][K/8] buffers for one span).  Every warp takes the
+    // same contiguous run [kb0, kb0 + cnt0) of each span's S * nrows items.
+    const int per_span = S * nrows;
+    const int kb0 = per_span * warp / kB1Warps;
+    const int cnt0 = per_span * (warp + 1) / kB1Warps - kb0;
+    const int total = cnt0 * nspan;   // this warp's items
     const uint32_t wring = sbase + a.off_ring + static_cast<uint32_t>(warp * D) * kB1Item;
     const uint32_t wbar = sbase + a.off_bar + static_cast<uint32_t>(warp * D) * 8u;
-    // issue cursor: element offset of the next item to request, the items
-    // left in its stage, and that stage
-    int is = per_stage > 0 ? kb / per_stage : 0;
-    int ileft = per_stage - (kb - is * per_stage);
-    int64_t ie = (static_cast<int64_t>(is) * N + ra) * C + static_cast<int64_t>(kb - is * per_stage) * kB1Span;
-    // every lane keeps the cursor (uniform), lane 0 alone issues
+    // issue cursor (uniform over the warp): span, stage, row and items left in
+    // this span's run of the next item to request, and its element offset
+    const int s0 = nrows > 0 ? kb0 / nrows : 0, rr0 = kb0 - s0 * nrows;
+    int csp = 0, cs = s0, crr = rr0, cleft = cnt0;
+    int64_t ie = (static_cast<int64_t>(cs) * N + ra + crr) * C;
     auto advance = [&]() {
-        ie += kB1Span;
-        if (--ileft == 0) {
-            ++is;
-            ie = (static_cast<int64_t>(is) * N + ra) * C;
-            ileft = per_stage;
+        ++crr;
+        ie += C;
+        if (crr == nrows) {
+            crr = 0;
+            ++cs;
+            ie = (static_cast<int64_t>(cs) * N + ra) * C + csp * kB1Span;
+        }
+        if (--cleft == 0) {
+            ++csp;
+            cs = s0;
+            crr = rr0;
+            cleft = cnt0;
+            ie = (static_cast<int64_t>(cs) * N + ra + crr) * C + csp * kB1Span;
         }
     };
 
@@ -237,7 +286,7 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
     __syncwarp();
 #pragma unroll
     for (int d = 0; d < D; ++d)
-        if (d < cnt) {
+        if (d < total) {
             b1_issue(lane == 0, wring + d * kB1Item, wbar + d * 8u, codes + ie, norms + ie, pol);
             advance();
             ++issued;
@@ -271,43 +320,12 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
     __syncthreads();
     pdl_launch_dependents();
 
-    // ---- after the wait: this layer's tables of x, scale * x
+    // ---- after the wait: the first span's table, scale * x.  The x of this
+    // thread's protected column and of its table job share one round trip.
     pdl_wait();
-    // x of this thread's protected column, loaded with its first table job
-    // (one round trip for both)
     const int uj = threadIdx.x < p ? spidx[threadIdx.x] : -1;
     const uint16_t xj = uj >= 0 ? a.x[uj] : static_cast<uint16_t>(0);
-    for (int J = warp; J < C / 32; J += kB1Warps) {   // job: one (span, half, j) for 32 lanes
-        const int span = J >> 4, h = (J >> 3) & 1, j = J & 7;
-        const int c = span * kB1Span + h * 256 + 8 * lane + j;
-        const uint4 u = *reinterpret_cast<const uint4 *>(a.x + 8 * c);
-        const uint32_t m = (pm[c >> 2] >> ((c & 3) * 8)) & 0xFFu;
-        float e[8] = {__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xFFFF0000u),
-                      __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xFFFF0000u),
-                      __uint_as_float(u.z << 16), __uint_as_float(u.z & 0xFFFF0000u),
-                      __uint_as_float(u.w << 16), __uint_as_float(u.w & 0xFFFF0000u)};
-#pragma unroll
-        for (int k = 0; k < 8; ++k)
-            if ((m >> k) & 1u) e[k] = 0.f;
-        // signed sums of element pairs: index bit 0 negates the first, bit 1 the second
-        float p01[2][4], p23[2][4];
-#pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-            const float x0 = e[4 * hh], x1 = e[4 * hh + 1], x2 = e[4 * hh + 2], x3 = e[4 * hh + 3];
-            p01[hh][0] = x0 + x1; p01[hh][1] = x1 - x0; p01[hh][2] = x0 - x1; p01[hh][3] = -(x0 + x1);
-            p23[hh][0] = x2 + x3; p23[hh][1] = x3 - x2; p23[hh][2] = x2 - x3; p23[hh][3] = -(x2 + x3);
-        }
-        const int P = span * kB1Span + h * 256 + 32 * j + lane;
-        const uint32_t dst = sbase + static_cast<uint32_t>((P >> 6) * 4096 + (P & 63) * 4);
-#pragma unroll
-        for (int v = 0; v < 16; ++v) {
-            const __half2 hv = __floats2half2_rn(p01[0][v & 3] + p23[0][v >> 2],
-                                                 p01[1][v & 3] + p23[1][v >> 2]);
-            asm volatile("st.shared.b32 [%0], %1;" ::"r"(dst + v * 256),
-                         "r"(*reinterpret_cast<const uint32_t *>(&hv)));
-        }
-    }
-    // scale * x of the protected columns (exact in fp32: 11 x 8 significant bits)
+    b1_table_job(sbase, pm, 0, warp, lane, b1_table_x(a.x, 0, warp, lane));
     if (threadIdx.x < p) sx[threadIdx.x] = uj >= 0 ? ssc[threadIdx.x] * bf16_bits_to_f32(xj) : 0.f;
     for (int u = threadIdx.x + kB1Threads; u < p; u += kB1Threads) {
         const int j = spidx[u];
@@ -315,53 +333,77 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
     }
     __syncthreads();
 
-    // ---- decode: this warp's items through its ring, D at a time
-    {
-        const uint32_t base0 = sbase + lane * 4u;
-        int i = 0, span = kb - (kb / nspan) * nspan;
+    const uint32_t base0 = sbase + lane * 4u;
+    int i = 0;   // items consumed
+    auto item = [&](uint32_t slot, uint32_t bar, uint32_t phase, int pidx) -> bool {
+        if (!__all_sync(0xFFFFFFFFu, mbar_try_wait(bar, phase)) &&
+            !__all_sync(0xFFFFFFFFu, mbar_wait_sleep(bar, phase, a.sleep_ns))) {
+            if (lane == 0) {
+                latch_error(a.err, BISCO_ERR_TIMEOUT);
+                atomicExch(&s_abort, 1);
+            }
+            return false;
+        }
+        uint2 cw[2];
+        uint4 nw[2];
+        cw[0] = lds_u64(slot + lane * 8u);
+        cw[1] = lds_u64(slot + 256u + lane * 8u);
+        nw[0] = lds_u128(slot + 512u + lane * 16u);
+        nw[1] = lds_u128(slot + 1024u + lane * 16u);
+        float v = b1_item(cw, nw, base0);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+        if (lane == 0) part[pidx] = v;
+        // the slot's reads are done (the values are in registers): refill it
+        __syncwarp();
+        if (issued < total) {
+            b1_issue(lane == 0, slot, bar, codes + ie, norms + ie, pol);
+            advance();
+            ++issued;
+        }
+        return true;
+    };
+    if constexpr (NSPAN == 1) {
+        // ---- decode: this warp's items through its ring, D at a time
         uint32_t phase = 0;
         bool ok = true;
-        for (int i0 = 0; i0 < cnt && ok; i0 += D, phase ^= 1u) {
+        for (int i0 = 0; i0 < total && ok; i0 += D, phase ^= 1u) {
 #pragma unroll
             for (int d = 0; d < D; ++d) {
-                if (i0 + d >= cnt) break;
-                const uint32_t slot = wring + d * kB1Item;
-                const uint32_t bar = wbar + d * 8u;
-                if (!__all_sync(0xFFFFFFFFu, mbar_try_wait(bar, phase)) &&
-                    !__all_sync(0xFFFFFFFFu, mbar_wait_sleep(bar, phase, a.sleep_ns))) {
-                    if (lane == 0) {
-                        latch_error(a.err, BISCO_ERR_TIMEOUT);
-                        atomicExch(&s_abort, 1);
-                    }
+                if (i0 + d >= total) break;
+                if (!item(wring + d * kB1Item, wbar + d * 8u, phase, kb0 + i0 + d)) {
                     ok = false;
                     break;
                 }
-                uint2 cw[2];
-                uint4 nw[2];
-                cw[0] = lds_u64(slot + lane * 8u);
-                cw[1] = lds_u64(slot + 256u + lane * 8u);
-                nw[0] = lds_u128(slot + 512u + lane * 16u);
-                nw[1] = lds_u128(slot + 1024u + lane * 16u);
-                float v = b1_item(cw, nw, NSPAN == 1 ? base0 : base0 + static_cast<uint32_t>(span) * 32768u);
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
-                if (lane == 0) part[kb + i0 + d] = v;
-                // the slot's reads are done (the values are in registers): refill it
-                __syncwarp();
-                if (issued < cnt) {
-                    b1_issue(lane == 0, slot, bar, codes + ie, norms + ie, pol);
-                    advance();
-                    ++issued;
-                }
-                if (NSPAN != 1) span = span + 1 == nspan ? 0 : span + 1;
                 i = i0 + d + 1;
             }
         }
-        // every copy this warp issued has landed before it leaves the ring
-        if (lane == 0)
-            for (int j = i; j < issued; ++j)
-                mbar_wait(wbar + static_cast<uint32_t>(j % D) * 8u, static_cast<uint32_t>(j / D) & 1u);
+    } else {
+        // ---- decode span by span; the table of span sp replaces that of sp - 1
+        bool ok = true;
+        uint4 xn = nspan > 1 ? b1_table_x(a.x, 1, warp, lane) : make_uint4(0, 0, 0, 0);
+        for (int sp = 0; sp < nspan; ++sp) {
+            if (sp > 0) {
+                __syncthreads();   // every warp is done with the table of span sp - 1
+                b1_table_job(sbase, pm, sp * kB1Span, warp, lane, xn);
+                __syncthreads();
+                if (sp + 1 < nspan) xn = b1_table_x(a.x, sp + 1, warp, lane);
+            }
+            for (int j = 0; j < cnt0 && ok; ++j) {
+                const int d = i % D;
+                if (!item(wring + d * kB1Item, wbar + d * 8u, static_cast<uint32_t>(i / D) & 1u,
+                          sp * per_span + kb0 + j)) {
+                    ok = false;
+                    break;
+                }
+                ++i;
+            }
+        }
     }
+    // every copy this warp issued has landed before it leaves the ring
+    if (lane == 0)
+        for (int j = i; j < issued; ++j)
+            mbar_wait(wbar + static_cast<uint32_t>(j % D) * 8u, static_cast<uint32_t>(j / D) & 1u);
     __syncthreads();
     if (*reinterpret_cast<volatile int *>(&s_abort)) return;
 
@@ -376,8 +418,8 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
         }
         if (lane == 0) {
             float v = 0.f;
-            for (int s = 0; s < S; ++s)
-                for (int sp = 0; sp < nspan; ++sp) v += part[(s * nrows + rr) * nspan + sp];
+            for (int sp = 0; sp < nspan; ++sp)
+                for (int s = 0; s < S; ++s) v += part[sp * per_span + s * nrows + rr];
             y[ra + rr] = v * kB1InvSqrt8 + pr;
         }
     }
@@ -413,7 +455,7 @@ bisco_status launch_b1_t(const B1Args &a, int grid, size_t smem, cudaStream_t st
 // Shared memory of one CTA with `depth` item slots per warp, past the 4 KB
 // aligned base (tables first); fills the offsets of `a`.
 size_t b1_layout(int C, int depth, int p_max, int items_max, size_t q8_bytes, B1Args *a) {
-    size_t off = static_cast<size_t>(C) * 64;   // tables: 64 bytes per chunk
+    size_t off = static_cast<size_t>(kB1Span) * 64;   // the table of one span: 64 bytes per chunk
     a->off_ring = static_cast<uint32_t>(off);
     off += static_cast<size_t>(kB1Warps) * depth * kB1Item;
     a->off_pm = static_cast<uint32_t>(off);
