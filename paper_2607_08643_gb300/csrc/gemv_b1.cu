@@ -200,6 +200,23 @@ __device__ __forceinline__ void b1_table_job(uint32_t tab, const uint32_t *pm, i
     }
 }
 
+// Sums of four values over the warp with six shuffles: the values are folded
+// in halves (lanes with bit 4 set keep c, d; with bit 3 set, the second of
+// their pair), then added over the remaining eight lanes.  Every lane returns
+// the total of value lane >> 3 (a, b, c, d); the order of the additions is
+// fixed.
+__device__ __forceinline__ float warp_sum4(float a, float b, float c, float d, int lane) {
+    const bool h4 = (lane & 16) != 0, h3 = (lane & 8) != 0;
+    const float r0 = __shfl_xor_sync(0xFFFFFFFFu, h4 ? a : c, 16);
+    const float r1 = __shfl_xor_sync(0xFFFFFFFFu, h4 ? b : d, 16);
+    const float k0 = (h4 ? c : a) + r0, k1 = (h4 ? d : b) + r1;
+    float k = (h3 ? k1 : k0) + __shfl_xor_sync(0xFFFFFFFFu, h3 ? k0 : k1, 8);
+    k += __shfl_xor_sync(0xFFFFFFFFu, k, 4);
+    k += __shfl_xor_sync(0xFFFFFFFFu, k, 2);
+    k += __shfl_xor_sync(0xFFFFFFFFu, k, 1);
+    return k;
+}
+
 // x of job J's chunk in span sp (see b1_table_job).
 __device__ __forceinline__ uint4 b1_table_x(const uint16_t *x, int sp, int J, int lane) {
     const int c = sp * kB1Span + ((J >> 3) & 1) * 256 + 8 * lane + (J & 7);
@@ -335,7 +352,9 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
 
     const uint32_t base0 = sbase + lane * 4u;
     int i = 0;   // items consumed
-    auto item = [&](uint32_t slot, uint32_t bar, uint32_t phase, int pidx) -> bool {
+    // item in `slot`: wait for it, decode it into this lane's partial sum,
+    // hand the slot back for the item D further on; false on a timeout
+    auto item = [&](uint32_t slot, uint32_t bar, uint32_t phase, float &v) -> bool {
         if (!__all_sync(0xFFFFFFFFu, mbar_try_wait(bar, phase)) &&
             !__all_sync(0xFFFFFFFFu, mbar_wait_sleep(bar, phase, a.sleep_ns))) {
             if (lane == 0) {
@@ -350,10 +369,7 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
         cw[1] = lds_u64(slot + 256u + lane * 8u);
         nw[0] = lds_u128(slot + 512u + lane * 16u);
         nw[1] = lds_u128(slot + 1024u + lane * 16u);
-        float v = b1_item(cw, nw, base0);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
-        if (lane == 0) part[pidx] = v;
+        v = b1_item(cw, nw, base0);
         // the slot's reads are done (the values are in registers): refill it
         __syncwarp();
         if (issued < total) {
@@ -364,19 +380,26 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
         return true;
     };
     if constexpr (NSPAN == 1) {
-        // ---- decode: this warp's items through its ring, D at a time
+        // ---- decode: this warp's items through its ring, D at a time; the D
+        // partial sums of a pass are added over the warp together
+        static_assert(D <= 4, "one folded reduction covers four items");
         uint32_t phase = 0;
         bool ok = true;
         for (int i0 = 0; i0 < total && ok; i0 += D, phase ^= 1u) {
+            float v[4] = {0.f, 0.f, 0.f, 0.f};
+            int n = 0;
 #pragma unroll
             for (int d = 0; d < D; ++d) {
                 if (i0 + d >= total) break;
-                if (!item(wring + d * kB1Item, wbar + d * 8u, phase, kb0 + i0 + d)) {
+                if (!item(wring + d * kB1Item, wbar + d * 8u, phase, v[d])) {
                     ok = false;
                     break;
                 }
-                i = i0 + d + 1;
+                n = d + 1;
             }
+            const float r = warp_sum4(v[0], v[1], v[2], v[3], lane);   // value lane >> 3, every lane
+            if ((lane & 7) == 0 && (lane >> 3) < n) part[kb0 + i0 + (lane >> 3)] = r;
+            i = i0 + n;
         }
     } else {
         // ---- decode span by span; the table of span sp replaces that of sp - 1
@@ -389,14 +412,23 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
                 __syncthreads();
                 if (sp + 1 < nspan) xn = b1_table_x(a.x, sp + 1, warp, lane);
             }
-            for (int j = 0; j < cnt0 && ok; ++j) {
-                const int d = i % D;
-                if (!item(wring + d * kB1Item, wbar + d * 8u, static_cast<uint32_t>(i / D) & 1u,
-                          sp * per_span + kb0 + j)) {
-                    ok = false;
-                    break;
+            // four items at a time, their partial sums added over the warp together
+            for (int j0 = 0; j0 < cnt0 && ok; j0 += 4) {
+                float v[4] = {0.f, 0.f, 0.f, 0.f};
+                int n = 0;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    if (j0 + q >= cnt0) break;
+                    const int d = i % D;
+                    if (!item(wring + d * kB1Item, wbar + d * 8u, static_cast<uint32_t>(i / D) & 1u, v[q])) {
+                        ok = false;
+                        break;
+                    }
+                    ++i;
+                    n = q + 1;
                 }
-                ++i;
+                const float r = warp_sum4(v[0], v[1], v[2], v[3], lane);
+                if ((lane & 7) == 0 && (lane >> 3) < n) part[sp * per_span + kb0 + j0 + (lane >> 3)] = r;
             }
         }
     }
