@@ -17,7 +17,8 @@ Functions and the paper passages they follow:
   :func:`encode_given`, :func:`encode_coupled`
                             output-row protection and the coupled MLP
                             channel score (Sec. III-E Eq. 9) with Eq. 10 on
-                            rows; the CUDA library does not take this axis yet
+                            rows (the CUDA library's protect_axis = 1 and
+                            bisco_select_coupled are checked against these)
 * :func:`double_to_fp8`, :func:`fp8_to_double`, :func:`quantize_protected_fmt`,
   :func:`quantize_protected_rows_fmt`, :func:`protected_values_fmt`
                             FP8 E4M3 / E5M2 and BF16 protected payloads (the
@@ -26,8 +27,9 @@ Functions and the paper passages they follow:
 * :func:`decoder_table_linear`, :func:`decoder_table_mlp`, :func:`decode_rows_table`
                             the decoder step of Eq. 1 as a table over the 256
                             code bytes (linear, or odd tanh perceptron with an
-                            optional residual block), decoded per Eq. 12; not
-                            taken by the CUDA library yet
+                            optional residual block), decoded per Eq. 12 (the
+                            CUDA library's bisco_gemv_table and
+                            bisco_decode_dense_table are checked against these)
 * :func:`lora_apply`        y0 + scale * Bm (A x), the optional low-rank
                             compensation of Sec. III-F (plain definition)
 * :func:`apply_rows`        decode + matmul on a list of rows
