@@ -534,6 +534,45 @@ def run_dense_stack(args, stack, stream, dev):
     return out
 
 
+def run_residual_decode(args, stack, stream, dev):
+    """Load-time decode of the whole stack to fp32 (Sec. III-G): packed (all
+    stages in one pass, bisco_decode_dense) against sequential (one pass per
+    stage, bisco_decode_dense_stage accumulating into the output).  Every
+    layer is decoded into one reused fp32 buffer of its shape."""
+    import torch
+    from paper_2607_08643_gb300 import bisco
+    bufs = {SHAPES[n]: torch.empty(SHAPES[n], dtype=torch.float32, device=dev) for n in STACK}
+
+    def packed():
+        for row in stack:
+            for L in row:
+                bisco.bisco_decode_dense(L, "f32", out=bufs[(L.N, L.K)], stream=stream)
+
+    def sequential():
+        for row in stack:
+            for L in row:
+                bisco.bisco_decode_dense_sequential(L, out=bufs[(L.N, L.K)], stream=stream)
+
+    out = {}
+    for name, fn in (("packed", packed), ("sequential", sequential)):
+        g = graph_of(torch, stream, fn)
+        out[name + "_ms"] = time_graph(torch, stream, g, 3, 2)
+        del g
+    if bisco.bisco_get_device_error(stream) != bisco.OK:
+        raise RuntimeError("device error in the residual decode")
+    elems = sum(L.N * L.K for row in stack for L in row)
+    coded = sum(L.compressed_bytes for row in stack for L in row)
+    out.update({"layers": len(stack) * len(STACK), "stages": S_STAGES, "dense_fp32_bytes": 4 * elems,
+                "compressed_bytes": coded,
+                "packed_gbs": (coded + 4 * elems) / (out["packed_ms"] * 1e-3) / 1e9,
+                "sequential_over_packed": out["sequential_ms"] / out["packed_ms"],
+                "how": "CUDA graph of one decode of every layer of the stack into a reused fp32 "
+                       "buffer per shape; sequential = S passes (write, then read-add-write)"})
+    del bufs
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_prefill_stack(args, stack, stream, dev):
     """Prefill on the tensor cores: bisco_gemm on the 7 projections of the
     first 4 layers of the stack at --prefill-tokens tokens, a CUDA graph of
@@ -1272,6 +1311,7 @@ def main():
         subs = run_sweeps(args, r["stack"], r["stream"], dev)
         prefill = run_prefill_stack(args, r["stack"], r["stream"], dev)
         dense_cmp = run_dense_stack(args, r["stack"], r["stream"], dev)
+        subs["residual_decode"] = run_residual_decode(args, r["stack"], r["stream"], dev)
         dense_cmp["fused_over_dense_batch1"] = (r["tokens_per_s"] / (args.batch / (dense_cmp["batch_1"]["ms_per_step"] * 1e-3))
                                                 if args.batch == 1 else None)
     if rank == 0:

@@ -316,6 +316,22 @@ bisco_status bisco_decode_dense(const bisco_layer *L, void *out, int32_t dtype,
                                 bisco_stream_t stream);
 
 /*
+ * One stage of the dense decode (Sec. III-G Eq. 12 term by term), for the
+ * sequential residual decode that the packed decode of bisco_decode_dense
+ * replaces (Sec. III-G, batched parallel residual decoding):
+ *     out[i][j]  = (bit_{stage,i,j} ? -1 : +1) * n16_{stage,i,j/8} / sqrt(8)   accumulate == 0
+ *     out[i][j] += the same                                                    accumulate != 0
+ * for every column, each term rounded once to fp32.  When stage is the last
+ * one (S - 1) the protected columns (rows, protect_axis = 1) are then
+ * overwritten as in bisco_decode_dense, so calling stages 0 .. S-1 in order
+ * with accumulate = (stage > 0) yields What, the stage terms added in stage
+ * order.  out: [N][K] fp32 device, 16-byte aligned.  stage outside
+ * [0, S) returns BISCO_ERR_INVALID_ARG.  Asynchronous on `stream`.
+ */
+bisco_status bisco_decode_dense_stage(const bisco_layer *L, int32_t stage, float *out,
+                                      int32_t accumulate, bisco_stream_t stream);
+
+/*
  * The learned decoder step (Sec. III-A Eq. 1; the decoder ablation compares
  * a symmetric, sign-symmetric decoder with a linear one).  A stage's chunk
  * decodes to n16 * D_s(q); with b = 8 the code q takes 256 values, so D_s is

@@ -21,7 +21,8 @@ EXPORTS = (
     "bisco_encode_workspace_bytes_axis", "bisco_encode", "bisco_encode_with_set",
     "bisco_select_coupled_workspace_bytes", "bisco_select_coupled",
     "bisco_encode_noalloc", "bisco_gemv", "bisco_gemv_multi",
-    "bisco_gemm_workspace_bytes", "bisco_gemm", "bisco_decode_dense", "bisco_gemv_table",
+    "bisco_gemm_workspace_bytes", "bisco_gemm", "bisco_decode_dense", "bisco_decode_dense_stage",
+    "bisco_gemv_table",
     "bisco_decode_dense_table", "bisco_lora_apply",
     "bisco_get_device_error",
 )
@@ -93,6 +94,8 @@ def load(path: str = LIB_PATH):
     lib.bisco_gemm.argtypes = [Lp, P, i32, P, P, sz, P]
     lib.bisco_decode_dense.restype = st
     lib.bisco_decode_dense.argtypes = [Lp, P, i32, P]
+    lib.bisco_decode_dense_stage.restype = st
+    lib.bisco_decode_dense_stage.argtypes = [Lp, i32, P, i32, P]
     lib.bisco_gemv_table.restype = st
     lib.bisco_gemv_table.argtypes = [Lp, P, P, i32, P, P]
     lib.bisco_decode_dense_table.restype = st
@@ -386,6 +389,26 @@ def bisco_decode_dense(L: Layer, dtype: str = "f32", out=None, stream=None):
     assert out.is_contiguous() and out.dtype == tdt and tuple(out.shape) == (L.N, L.K)
     _check(load().bisco_decode_dense(ctypes.byref(L.c), _ptr(out), code, _stream(stream)),
            "bisco_decode_dense")
+    return out
+
+
+def bisco_decode_dense_stage(L: Layer, stage: int, out, accumulate: bool, stream=None):
+    """Adds (or writes) one stage's term of What into the fp32 [N][K] tensor
+    `out`; the last stage also writes the protected set."""
+    import torch
+    assert out.is_contiguous() and out.dtype == torch.float32 and tuple(out.shape) == (L.N, L.K)
+    _check(load().bisco_decode_dense_stage(ctypes.byref(L.c), int(stage), _ptr(out), int(bool(accumulate)),
+                                           _stream(stream)), "bisco_decode_dense_stage")
+    return out
+
+
+def bisco_decode_dense_sequential(L: Layer, out=None, stream=None):
+    """What [N][K] fp32 decoded stage by stage (one pass per stage)."""
+    import torch
+    if out is None:
+        out = torch.empty((L.N, L.K), dtype=torch.float32, device=L.codes.device)
+    for s in range(L.c.stages):
+        bisco_decode_dense_stage(L, s, out, s > 0, stream)
     return out
 
 

@@ -362,6 +362,22 @@ bisco_status bisco_decode_dense(const bisco_layer *L, void *out, int32_t dtype,
     return launch_decode_dense(*L, out, dtype, err, s);
 }
 
+bisco_status bisco_decode_dense_stage(const bisco_layer *L, int32_t stage, float *out,
+                                      int32_t accumulate, bisco_stream_t stream) {
+    bisco_status st = check_layer(L, true);
+    if (st != BISCO_OK) return st;
+    if (stage < 0 || stage >= L->stages) return BISCO_ERR_INVALID_ARG;
+    if (!out || !aligned16(out)) return BISCO_ERR_INVALID_ARG;
+    int *err = device_error_word(&st);
+    if (!err) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    st = launch_decode_stage(*L, stage, out, accumulate != 0, s);
+    if (st != BISCO_OK || stage != L->stages - 1 || L->n_protected == 0) return st;
+    // after the last stage the protected set overwrites its columns (or rows)
+    if (needs_epilogue(*L)) return dense_epilogue(*L, out, BISCO_DENSE_F32, err, s);
+    return launch_dense_protected_f32(*L, out, err, s);
+}
+
 bisco_status bisco_gemv_table(const bisco_layer *L, const uint16_t *tables, const uint16_t *x_bf16,
                               int32_t B, float *y, bisco_stream_t stream) {
     bisco_status st = check_layer(L, true);

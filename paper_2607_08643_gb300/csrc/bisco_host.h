@@ -72,6 +72,11 @@ bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *
                          void *workspace, size_t ws_bytes, int *err, cudaStream_t stream);
 bisco_status launch_decode_dense(const bisco_layer &L, void *out, int dtype, int *err,
                                  cudaStream_t stream);
+// One stage into a dense fp32 matrix, and the INT8 protected-column
+// overwrite of that matrix (dense.cu).
+bisco_status launch_decode_stage(const bisco_layer &L, int stage, float *out, bool accumulate,
+                                 cudaStream_t stream);
+bisco_status launch_dense_protected_f32(const bisco_layer &L, float *out, int *err, cudaStream_t stream);
 
 // bisco_lora_apply's two kernels (arguments already validated).
 bisco_status launch_lora_apply(const uint16_t *A, const uint16_t *Bm, int rank, int N, int K,

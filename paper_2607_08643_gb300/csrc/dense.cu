@@ -100,6 +100,30 @@ __global__ void __launch_bounds__(kDenseThreads) k_dense_protected(const int8_t 
         from_f32<T>(sc * static_cast<float>(q8[static_cast<int64_t>(i) * p_pad + u]));
 }
 
+// One stage of Eq. 12 into a dense fp32 matrix: out (=, or += when ACC)
+// (bit ? -1 : +1) * n16 / sqrt(8), one thread per 8-column chunk.  Calling it
+// stage after stage is the sequential residual decode that Sec. III-G's
+// packed decode (k_decode_dense: every stage in one pass) replaces.
+template <bool ACC>
+__global__ void __launch_bounds__(kDenseThreads) k_decode_stage(const uint8_t *__restrict__ codes,
+                                                                const uint16_t *__restrict__ norms,
+                                                                int64_t chunks, float *__restrict__ out) {
+    const int64_t e = static_cast<int64_t>(blockIdx.x) * kDenseThreads + threadIdx.x;
+    if (e >= chunks) return;
+    const uint32_t b = codes[e];
+    const float t = __half2float(__ushort_as_half(norms[e])) * kInvSqrt8;
+    float v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = ((b >> k) & 1u) ? -t : t;
+    if constexpr (ACC) {
+        const float4 a = reinterpret_cast<const float4 *>(out + e * 8)[0];
+        const float4 c = reinterpret_cast<const float4 *>(out + e * 8)[1];
+        v[0] += a.x; v[1] += a.y; v[2] += a.z; v[3] += a.w;
+        v[4] += c.x; v[5] += c.y; v[6] += c.z; v[7] += c.w;
+    }
+    store8(out + e * 8, v);
+}
+
 template <typename T>
 bisco_status launch_dense_t(const bisco_layer &L, T *out, int *err, cudaStream_t stream) {
     const int N = L.n_out, K = L.k_in, S = L.stages, p = L.n_protected;
@@ -118,6 +142,28 @@ bisco_status launch_dense_t(const bisco_layer &L, T *out, int *err, cudaStream_t
 }
 
 }  // namespace
+
+bisco_status launch_decode_stage(const bisco_layer &L, int stage, float *out, bool accumulate,
+                                 cudaStream_t stream) {
+    const int64_t chunks = static_cast<int64_t>(L.n_out) * (L.k_in / 8);
+    const uint8_t *codes = reinterpret_cast<const uint8_t *>(L.codes) + stage * chunks;
+    const uint16_t *norms = L.norms + stage * chunks;
+    const unsigned grid = static_cast<unsigned>((chunks + kDenseThreads - 1) / kDenseThreads);
+    if (accumulate)
+        k_decode_stage<true><<<grid, kDenseThreads, 0, stream>>>(codes, norms, chunks, out);
+    else
+        k_decode_stage<false><<<grid, kDenseThreads, 0, stream>>>(codes, norms, chunks, out);
+    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+}
+
+bisco_status launch_dense_protected_f32(const bisco_layer &L, float *out, int *err, cudaStream_t stream) {
+    const int N = L.n_out, K = L.k_in, p = L.n_protected;
+    if (p == 0) return BISCO_OK;
+    const int64_t n = static_cast<int64_t>(N) * p;
+    k_dense_protected<float><<<static_cast<unsigned>((n + kDenseThreads - 1) / kDenseThreads), kDenseThreads,
+                               0, stream>>>(L.q8, L.q8_scale, L.prot_idx, N, K, p, (p + 15) / 16 * 16, out, err);
+    return cudaGetLastError() == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
+}
 
 bisco_status launch_decode_dense(const bisco_layer &L, void *out, int dtype, int *err,
                                  cudaStream_t stream) {

@@ -85,6 +85,7 @@ struct B1Args {
     int depth;                 // item slots per warp
     int q8_staged;             // int8 rows in shared memory (else read at the end)
     uint32_t sleep_ns;         // suspend-time hint of the item waits
+    int withhold;              // test of the bounded waits: request no copies
     uint32_t off_ring, off_pm, off_pidx, off_sx, off_part, off_q8, off_bar;   // tables at 0
 };
 
@@ -301,9 +302,10 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
         fence_mbar_init();
     }
     __syncwarp();
+    const int to_issue = a.withhold ? 0 : total;   // withheld: every wait runs out, nothing in flight
 #pragma unroll
     for (int d = 0; d < D; ++d)
-        if (d < total) {
+        if (d < to_issue) {
             b1_issue(lane == 0, wring + d * kB1Item, wbar + d * 8u, codes + ie, norms + ie, pol);
             advance();
             ++issued;
@@ -372,7 +374,7 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
         v = b1_item(cw, nw, base0);
         // the slot's reads are done (the values are in registers): refill it
         __syncwarp();
-        if (issued < total) {
+        if (issued < to_issue) {
             b1_issue(lane == 0, slot, bar, codes + ie, norms + ie, pol);
             advance();
             ++issued;
@@ -588,6 +590,10 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
     a.depth = depth;
     a.S = S;
     a.sleep_ns = 200;
+    // test hook for the bounded waits: with BISCO_TEST_WITHHOLD_COPIES set the
+    // kernel requests no data, so its waits expire, it latches
+    // BISCO_ERR_TIMEOUT and returns with no copy in flight
+    a.withhold = getenv("BISCO_TEST_WITHHOLD_COPIES") != nullptr;
     b1_layout(C, depth, p_max, items_max, a.q8_staged ? q8_max : 0, &a);
     *launched = true;
     const bool one = a.nspan == 1;

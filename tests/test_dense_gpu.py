@@ -93,3 +93,56 @@ def test_dense_then_matmul_meets_the_bar(env):
     x = to_dev(X, dev).view(torch.bfloat16).float()
     y = (x @ W.t()).cpu().numpy()
     assert max_rel_rows(y, oracle.gemv(Lref, X)) <= TOL
+
+
+@pytest.mark.parametrize("N,K,S,p,dist", CASES)
+def test_sequential_stage_decode_matches_oracle(env, N, K, S, p, dist):
+    """bisco_decode_dense_stage stage after stage (the sequential residual
+    decode): each stage term is rounded once to fp32 and added in stage
+    order, S - 1 more fp32 roundings than the packed decode -- within
+    S * 2^-23 relative of the oracle, protected columns exact."""
+    import torch
+    bisco, dev = env
+    Lref = oracle.encode(synth.layer_weights(N, K, seed=N + K + S, dist=dist), S=S, p=p)
+    ref = oracle.decode_rows(Lref)
+    L = bisco.Layer.from_numpy(Lref, dev)
+    got = bisco.bisco_decode_dense_sequential(L)
+    torch.cuda.synchronize()
+    assert bisco.bisco_get_device_error() == 0
+    got = got.cpu().numpy().astype(np.float64)
+    floor = 2.0 ** -40 * np.abs(ref).max()
+    # each term |n16/sqrt(8)| is at most the chunk's largest |What| bound: use
+    # the sum of term magnitudes, S * max term, as the scale of the rounding
+    terms = np.zeros_like(ref)
+    for s in range(S):
+        n = Lref["norms"][s].view(np.float16).astype(np.float64)       # [N][K/8]
+        terms += np.repeat(n, 8, axis=1) / np.sqrt(8.0)
+    bad = np.abs(got - ref) > S * 2.0 ** -23 * terms + floor
+    assert not bad.any(), (bad.sum(), got[bad][:4], ref[bad][:4])
+    if p > 0:
+        assert np.array_equal(got[:, Lref["idx"]], ref[:, Lref["idx"]])
+
+
+def test_sequential_and_packed_decode_agree(env):
+    import torch
+    bisco, dev = env
+    Lref = oracle.encode(synth.layer_weights(300, 1024, seed=77, dist="t4"), S=3, p=11)
+    L = bisco.Layer.from_numpy(Lref, dev)
+    seq = bisco.bisco_decode_dense_sequential(L)
+    packed = bisco.bisco_decode_dense(L, "f32")
+    torch.cuda.synchronize()
+    d = (seq - packed).abs().max().item()
+    assert d <= 4 * 2.0 ** -23 * packed.abs().max().item()
+
+
+def test_stage_decode_rejects_a_stage_out_of_range(env):
+    import torch
+    bisco, dev = env
+    Lref = oracle.encode(synth.layer_weights(16, 64, seed=5), S=2, p=1)
+    L = bisco.Layer.from_numpy(Lref, dev)
+    out = torch.empty((16, 64), dtype=torch.float32, device=dev)
+    lib = bisco.load()
+    import ctypes
+    for st in (-1, 2):
+        assert lib.bisco_decode_dense_stage(ctypes.byref(L.c), st, ctypes.c_void_p(out.data_ptr()), 0,
+                                            None) == bisco.ERR_INVALID_ARG
