@@ -149,27 +149,36 @@ __device__ __forceinline__ float b1_item(const uint2 (&cw)[2], const uint4 (&nw)
     return (acc4[0][0] + acc4[0][1]) + (acc4[1][0] + acc4[1][1]);
 }
 
-// Lane 0 of the warp arms a slot's mbarrier for 1536 bytes and issues its
-// two bulk copies (signs, norms); the other lanes run the same instruction
-// stream with the predicate off, so the warp never diverges.
-__device__ __forceinline__ void b1_issue(bool leader, uint32_t slot, uint32_t bar, const void *codes,
-                                         const void *norms, uint64_t pol) {
+// Lane 0 of the warp arms a slot's mbarrier for `bytes` (after a proxy fence:
+// the warp's reads of the slot are done) and, in b1_copy, issues one item's
+// two bulk copies (signs to cdst, norms to ndst); the other lanes run the
+// same instruction stream with the predicate off, so the warp never
+// diverges.
+__device__ __forceinline__ void b1_arm(bool leader, uint32_t bar, uint32_t bytes) {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "setp.ne.u32 p, %0, 0;\n\t"
         "@p fence.proxy.async.shared::cta;\n\t"
-        "@p mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%2], 1536;\n\t"
+        "@p mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%1], %2;\n\t}"
+        ::"r"(static_cast<uint32_t>(leader)), "r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void b1_copy(bool leader, uint32_t cdst, uint32_t ndst, uint32_t bar,
+                                        const void *codes, const void *norms, uint64_t pol) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.u32 p, %0, 0;\n\t"
         "@p cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-        " [%1], [%3], 512, [%2], %5;\n\t"
+        " [%1], [%4], 512, [%3], %6;\n\t"
         "@p cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-        " [%6], [%4], 1024, [%2], %5;\n\t}"
-        ::"r"(static_cast<uint32_t>(leader)), "r"(slot), "r"(bar), "l"(codes), "l"(norms), "l"(pol),
-          "r"(slot + 512u)
+        " [%2], [%5], 1024, [%3], %6;\n\t}"
+        ::"r"(static_cast<uint32_t>(leader)), "r"(cdst), "r"(ndst), "r"(bar), "l"(codes), "l"(norms),
+          "l"(pol)
         : "memory");
 }
 
-// The table of one 4096-column span (32 KB): job J of warp J (16 jobs for
-// 16 warps), lane l: chunk 256*h + 8l + j of the span, h = J >> 3 & 1,
+// The table of one 4096-column span (32 KB): job J (of 16) of a warp,
+// lane l: chunk 256*h + 8l + j of the span, h = J >> 3 & 1,
 // j = J & 7, from its 8 activations xv (bf16, the span's column base c0)
 // with the layer's protected columns (bits of pm) zeroed.
 __device__ __forceinline__ void b1_table_job(uint32_t tab, const uint32_t *pm, int c0, int J, int lane,
@@ -224,15 +233,18 @@ __device__ __forceinline__ uint4 b1_table_x(const uint16_t *x, int sp, int J, in
     return *reinterpret_cast<const uint4 *>(x + 8 * c);
 }
 
-// D item slots per warp; NSPAN 4096-column spans per row (0: a.nspan > 1,
-// at run time).  With one span, every ring address is an immediate offset;
-// with several, a CTA holds the table of one span at a time and walks its
-// items span by span, rebuilding the table between spans (x of the next
-// span is loaded while the current one is decoded).
-template <int D, int NSPAN>
-__global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_constant__ B1Args a) {
-    static_assert(kB1Warps == 16, "one table job per warp per span");
-    constexpr int kB1Threads = kB1Warps * 32;
+// NW warps; D ring slots per warp of IPS items each; NSPAN 4096-column spans
+// per row (0: a.nspan > 1, at run time).  With one span, every ring address
+// is an immediate offset; with several, a CTA holds the table of one span at
+// a time and walks its items span by span, rebuilding the table between
+// spans (x of the next span is loaded while the current one is decoded).
+template <int NW, int D, int IPS, int NSPAN>
+__global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ B1Args a) {
+    static_assert(D * IPS <= 4, "one folded reduction covers a ring pass");
+    static_assert(NSPAN == 1 || IPS == 1, "several spans: one item per slot");
+    constexpr int kThreads = NW * 32;
+    constexpr uint32_t kSlot = IPS * kB1Item;          // [signs of IPS items][norms of IPS items]
+    constexpr uint32_t kNormOff = IPS * 512u;
     extern __shared__ unsigned char smem_raw[];
     unsigned char *sm = align_smem<4096>(smem_raw);
     const uint32_t sbase = smem_u32(sm);
@@ -268,10 +280,10 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
     // order of the [S][N][K/8] buffers for one span).  Every warp takes the
     // same contiguous run [kb0, kb0 + cnt0) of each span's S * nrows items.
     const int per_span = S * nrows;
-    const int kb0 = per_span * warp / kB1Warps;
-    const int cnt0 = per_span * (warp + 1) / kB1Warps - kb0;
+    const int kb0 = per_span * warp / NW;
+    const int cnt0 = per_span * (warp + 1) / NW - kb0;
     const int total = cnt0 * nspan;   // this warp's items
-    const uint32_t wring = sbase + a.off_ring + static_cast<uint32_t>(warp * D) * kB1Item;
+    const uint32_t wring = sbase + a.off_ring + static_cast<uint32_t>(warp * D) * kSlot;
     const uint32_t wbar = sbase + a.off_bar + static_cast<uint32_t>(warp * D) * 8u;
     // issue cursor (uniform over the warp): span, stage, row and items left in
     // this span's run of the next item to request, and its element offset
@@ -294,26 +306,37 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
             ie = (static_cast<int64_t>(cs) * N + ra + crr) * C + csp * kB1Span;
         }
     };
+    // slot d: the next up to IPS items (withheld: none, every wait runs out
+    // with nothing in flight)
+    const int to_issue = a.withhold ? 0 : total;
+    int issued = 0;
+    auto fill = [&](int d) {
+        const int n = min(IPS, to_issue - issued);
+        if (n <= 0) return;
+        const uint32_t slot = wring + d * kSlot, bar = wbar + d * 8u;
+        b1_arm(lane == 0, bar, n * kB1Item);
+#pragma unroll
+        for (int it = 0; it < IPS; ++it)
+            if (it < n) {
+                b1_copy(lane == 0, slot + it * 512u, slot + kNormOff + it * 1024u, bar, codes + ie,
+                        norms + ie, pol);
+                advance();
+            }
+        issued += n;
+    };
 
     // ---- before the wait: barriers, first items, protected metadata, int8 rows
-    int issued = 0;
     if (lane == 0) {
         for (int d = 0; d < D; ++d) mbar_init(wbar + 8 * d, 1);
         fence_mbar_init();
     }
     __syncwarp();
-    const int to_issue = a.withhold ? 0 : total;   // withheld: every wait runs out, nothing in flight
 #pragma unroll
-    for (int d = 0; d < D; ++d)
-        if (d < to_issue) {
-            b1_issue(lane == 0, wring + d * kB1Item, wbar + d * 8u, codes + ie, norms + ie, pol);
-            advance();
-            ++issued;
-        }
+    for (int d = 0; d < D; ++d) fill(d);
     if (threadIdx.x == 0) s_abort = 0;
-    for (int i = threadIdx.x; i < C / 4; i += kB1Threads) pm[i] = 0u;
+    for (int i = threadIdx.x; i < C / 4; i += kThreads) pm[i] = 0u;
     __syncthreads();
-    for (int u = threadIdx.x; u < p; u += kB1Threads) {
+    for (int u = threadIdx.x; u < p; u += kThreads) {
         int j = L.prot_idx[u];
         float sc = __half2float(__ushort_as_half(L.q8_scale[u]));
         if (j < 0 || j >= K) {   // not a valid layer: reported, and the entry dropped
@@ -330,7 +353,7 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
         if (a.q8_staged) {
             const int n16 = nrows * p_pad / 16;
             const uint4 *src = reinterpret_cast<const uint4 *>(q8 + static_cast<int64_t>(ra) * p_pad);
-            for (int i = threadIdx.x; i < n16; i += kB1Threads) reinterpret_cast<uint4 *>(q8s)[i] = src[i];
+            for (int i = threadIdx.x; i < n16; i += kThreads) reinterpret_cast<uint4 *>(q8s)[i] = src[i];
         } else if (threadIdx.x == 0) {
             // read at the end from global memory: into L2 now
             prefetch_l2(q8 + static_cast<int64_t>(ra) * p_pad, static_cast<uint32_t>(nrows * p_pad));
@@ -340,13 +363,21 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
     pdl_launch_dependents();
 
     // ---- after the wait: the first span's table, scale * x.  The x of this
-    // thread's protected column and of its table job share one round trip.
+    // thread's protected column and of its table jobs share one round trip.
     pdl_wait();
     const int uj = threadIdx.x < p ? spidx[threadIdx.x] : -1;
     const uint16_t xj = uj >= 0 ? a.x[uj] : static_cast<uint16_t>(0);
-    b1_table_job(sbase, pm, 0, warp, lane, b1_table_x(a.x, 0, warp, lane));
+    {
+        uint4 xv[(16 + NW - 1) / NW];
+#pragma unroll
+        for (int q = 0; q < (16 + NW - 1) / NW; ++q)
+            if (warp + q * NW < 16) xv[q] = b1_table_x(a.x, 0, warp + q * NW, lane);
+#pragma unroll
+        for (int q = 0; q < (16 + NW - 1) / NW; ++q)
+            if (warp + q * NW < 16) b1_table_job(sbase, pm, 0, warp + q * NW, lane, xv[q]);
+    }
     if (threadIdx.x < p) sx[threadIdx.x] = uj >= 0 ? ssc[threadIdx.x] * bf16_bits_to_f32(xj) : 0.f;
-    for (int u = threadIdx.x + kB1Threads; u < p; u += kB1Threads) {
+    for (int u = threadIdx.x + kThreads; u < p; u += kThreads) {
         const int j = spidx[u];
         sx[u] = j >= 0 ? ssc[u] * bf16_bits_to_f32(a.x[j]) : 0.f;
     }
@@ -354,9 +385,10 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
 
     const uint32_t base0 = sbase + lane * 4u;
     int i = 0;   // items consumed
-    // item in `slot`: wait for it, decode it into this lane's partial sum,
-    // hand the slot back for the item D further on; false on a timeout
-    auto item = [&](uint32_t slot, uint32_t bar, uint32_t phase, float &v) -> bool {
+    // slot d: wait for it, decode its n items into this lane's partial sums
+    // v[0..n), refill it; false on a timeout
+    auto slot_items = [&](int d, uint32_t phase, int n, float *v) -> bool {
+        const uint32_t slot = wring + d * kSlot, bar = wbar + d * 8u;
         if (!__all_sync(0xFFFFFFFFu, mbar_try_wait(bar, phase)) &&
             !__all_sync(0xFFFFFFFFu, mbar_wait_sleep(bar, phase, a.sleep_ns))) {
             if (lane == 0) {
@@ -365,39 +397,39 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
             }
             return false;
         }
-        uint2 cw[2];
-        uint4 nw[2];
-        cw[0] = lds_u64(slot + lane * 8u);
-        cw[1] = lds_u64(slot + 256u + lane * 8u);
-        nw[0] = lds_u128(slot + 512u + lane * 16u);
-        nw[1] = lds_u128(slot + 1024u + lane * 16u);
-        v = b1_item(cw, nw, base0);
+#pragma unroll
+        for (int it = 0; it < IPS; ++it)
+            if (it < n) {
+                uint2 cw[2];
+                uint4 nw[2];
+                cw[0] = lds_u64(slot + it * 512u + lane * 8u);
+                cw[1] = lds_u64(slot + it * 512u + 256u + lane * 8u);
+                nw[0] = lds_u128(slot + kNormOff + it * 1024u + lane * 16u);
+                nw[1] = lds_u128(slot + kNormOff + it * 1024u + 512u + lane * 16u);
+                v[it] = b1_item(cw, nw, base0);
+            }
         // the slot's reads are done (the values are in registers): refill it
         __syncwarp();
-        if (issued < to_issue) {
-            b1_issue(lane == 0, slot, bar, codes + ie, norms + ie, pol);
-            advance();
-            ++issued;
-        }
+        fill(d);
         return true;
     };
     if constexpr (NSPAN == 1) {
-        // ---- decode: this warp's items through its ring, D at a time; the D
-        // partial sums of a pass are added over the warp together
-        static_assert(D <= 4, "one folded reduction covers four items");
+        // ---- decode: D slots (D * IPS items) a pass; the partial sums of a
+        // pass are added over the warp together
         uint32_t phase = 0;
         bool ok = true;
-        for (int i0 = 0; i0 < total && ok; i0 += D, phase ^= 1u) {
+        for (int i0 = 0; i0 < total && ok; i0 += D * IPS, phase ^= 1u) {
             float v[4] = {0.f, 0.f, 0.f, 0.f};
             int n = 0;
 #pragma unroll
             for (int d = 0; d < D; ++d) {
-                if (i0 + d >= total) break;
-                if (!item(wring + d * kB1Item, wbar + d * 8u, phase, v[d])) {
+                const int m = min(IPS, total - (i0 + d * IPS));
+                if (m <= 0) break;
+                if (!slot_items(d, phase, m, v + d * IPS)) {
                     ok = false;
                     break;
                 }
-                n = d + 1;
+                n = d * IPS + m;
             }
             const float r = warp_sum4(v[0], v[1], v[2], v[3], lane);   // value lane >> 3, every lane
             if ((lane & 7) == 0 && (lane >> 3) < n) part[kb0 + i0 + (lane >> 3)] = r;
@@ -406,13 +438,20 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
     } else {
         // ---- decode span by span; the table of span sp replaces that of sp - 1
         bool ok = true;
-        uint4 xn = nspan > 1 ? b1_table_x(a.x, 1, warp, lane) : make_uint4(0, 0, 0, 0);
+        uint4 xn[(16 + NW - 1) / NW];
+#pragma unroll
+        for (int q = 0; q < (16 + NW - 1) / NW; ++q)
+            if (warp + q * NW < 16 && nspan > 1) xn[q] = b1_table_x(a.x, 1, warp + q * NW, lane);
         for (int sp = 0; sp < nspan; ++sp) {
             if (sp > 0) {
                 __syncthreads();   // every warp is done with the table of span sp - 1
-                b1_table_job(sbase, pm, sp * kB1Span, warp, lane, xn);
+#pragma unroll
+                for (int q = 0; q < (16 + NW - 1) / NW; ++q)
+                    if (warp + q * NW < 16) b1_table_job(sbase, pm, sp * kB1Span, warp + q * NW, lane, xn[q]);
                 __syncthreads();
-                if (sp + 1 < nspan) xn = b1_table_x(a.x, sp + 1, warp, lane);
+#pragma unroll
+                for (int q = 0; q < (16 + NW - 1) / NW; ++q)
+                    if (warp + q * NW < 16 && sp + 1 < nspan) xn[q] = b1_table_x(a.x, sp + 1, warp + q * NW, lane);
             }
             // four items at a time, their partial sums added over the warp together
             for (int j0 = 0; j0 < cnt0 && ok; j0 += 4) {
@@ -421,8 +460,7 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
                     if (j0 + q >= cnt0) break;
-                    const int d = i % D;
-                    if (!item(wring + d * kB1Item, wbar + d * 8u, static_cast<uint32_t>(i / D) & 1u, v[q])) {
+                    if (!slot_items(i % D, static_cast<uint32_t>(i / D) & 1u, 1, v + q)) {
                         ok = false;
                         break;
                     }
@@ -434,15 +472,16 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
             }
         }
     }
-    // every copy this warp issued has landed before it leaves the ring
+    // every copy this warp issued has landed before it leaves the ring: the
+    // slots of the items requested and not consumed
     if (lane == 0)
-        for (int j = i; j < issued; ++j)
+        for (int j = (i + IPS - 1) / IPS; j < (issued + IPS - 1) / IPS; ++j)
             mbar_wait(wbar + static_cast<uint32_t>(j % D) * 8u, static_cast<uint32_t>(j / D) & 1u);
     __syncthreads();
     if (*reinterpret_cast<volatile int *>(&s_abort)) return;
 
     // ---- outputs: a warp per row; items in order, then the protected term
-    for (int rr = warp; rr < nrows; rr += kB1Warps) {
+    for (int rr = warp; rr < nrows; rr += NW) {
         float pr = 0.f;
         if (p > 0) {
             const int8_t *q8r = a.q8_staged ? q8s + rr * p_pad : q8 + static_cast<int64_t>(ra + rr) * p_pad;
@@ -461,9 +500,9 @@ __global__ void __launch_bounds__(kB1Warps * 32, 2) k_gemv_b1(const __grid_const
 
 size_t align_up_b1(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
-template <int D, int NSPAN>
+template <int NW, int D, int IPS, int NSPAN>
 bisco_status launch_b1_t(const B1Args &a, int grid, size_t smem, cudaStream_t stream) {
-    auto kern = k_gemv_b1<D, NSPAN>;
+    auto kern = k_gemv_b1<NW, D, IPS, NSPAN>;
     static size_t configured[64] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return BISCO_ERR_CUDA;
@@ -475,7 +514,7 @@ bisco_status launch_b1_t(const B1Args &a, int grid, size_t smem, cudaStream_t st
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid, 1, 1);
-    cfg.blockDim = dim3(kB1Warps * 32, 1, 1);
+    cfg.blockDim = dim3(NW * 32, 1, 1);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
@@ -486,12 +525,14 @@ bisco_status launch_b1_t(const B1Args &a, int grid, size_t smem, cudaStream_t st
     return cudaLaunchKernelEx(&cfg, kern, a) == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
 }
 
-// Shared memory of one CTA with `depth` item slots per warp, past the 4 KB
-// aligned base (tables first); fills the offsets of `a`.
-size_t b1_layout(int C, int depth, int p_max, int items_max, size_t q8_bytes, B1Args *a) {
+// Shared memory of one CTA of nw warps with `depth` slots of ips items per
+// warp, past the 4 KB aligned base (the span table first); fills the offsets
+// of `a`.
+size_t b1_layout(int C, int nw, int depth, int ips, int p_max, int items_max, size_t q8_bytes,
+                 B1Args *a) {
     size_t off = static_cast<size_t>(kB1Span) * 64;   // the table of one span: 64 bytes per chunk
     a->off_ring = static_cast<uint32_t>(off);
-    off += static_cast<size_t>(kB1Warps) * depth * kB1Item;
+    off += static_cast<size_t>(nw) * depth * ips * kB1Item;
     a->off_pm = static_cast<uint32_t>(off);
     off += static_cast<size_t>(C);                          // one bit per column
     a->off_pidx = static_cast<uint32_t>(off);
@@ -506,9 +547,20 @@ size_t b1_layout(int C, int depth, int p_max, int items_max, size_t q8_bytes, B1
     off += q8_bytes;
     off = align_up_b1(off, 8);
     a->off_bar = static_cast<uint32_t>(off);
-    off += static_cast<size_t>(kB1Warps) * depth * 8;
+    off += static_cast<size_t>(nw) * depth * 8;
     return off + 4096;   // slack for the 4 KB aligned base
 }
+
+// The instantiated (warps, slots per warp, items per slot) shapes, in order
+// of preference: one span per row, then several.  Measured on GB300: 12
+// warps with two-item slots (the per-slot work paid once per two items, 80
+// registers) run the 36x7 step 8 % slower than 16 warps with one item per
+// slot -- latency is hidden by warps more than by the slot work saved.
+struct B1Shape {
+    int nw, depth, ips;
+};
+constexpr B1Shape kB1One[] = {{16, 3, 1}, {16, 2, 1}};
+constexpr B1Shape kB1Many[] = {{16, 3, 1}, {16, 2, 1}};
 
 }  // namespace
 
@@ -570,34 +622,42 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
     }
     const int C = K / 8;
     const int items_max = rows_max * S * a.nspan;
-    // the deepest ring (three or two item slots per warp) that leaves room
-    // for the next kernel's CTA on the SM, else one CTA per SM
-    int depth = 0;
+    // the first shape that leaves room for the next kernel's CTA on the SM
+    // (int8 rows staged if they fit), else the first that fits one CTA per SM
+    const bool one = a.nspan == 1;
+    const B1Shape *shapes = one ? kB1One : kB1Many;
+    const int nshapes = 2;
+    B1Shape pick = {0, 0, 0};
     size_t smem = 0;
-    for (int pass = 0; pass < 2 && depth == 0; ++pass) {
+    for (int pass = 0; pass < 2 && pick.nw == 0; ++pass) {
         const size_t budget = pass == 0 ? kB1Coresident : kB1MaxSmem;
-        for (int d = 3; d >= 2 && depth == 0; --d)
-            for (int staged = 1; staged >= 0 && depth == 0; --staged) {
-                const size_t need = b1_layout(C, d, p_max, items_max, staged ? q8_max : 0, &a);
+        for (int k = 0; k < nshapes && pick.nw == 0; ++k)
+            for (int staged = 1; staged >= 0 && pick.nw == 0; --staged) {
+                const B1Shape &sh = shapes[k];
+                const size_t need = b1_layout(C, sh.nw, sh.depth, sh.ips, p_max, items_max,
+                                              staged ? q8_max : 0, &a);
                 if (need <= budget) {
-                    depth = d;
+                    pick = sh;
                     smem = need;
                     a.q8_staged = staged;
                 }
             }
     }
-    if (depth == 0) return BISCO_OK;
-    a.depth = depth;
+    if (pick.nw == 0) return BISCO_OK;
+    a.depth = pick.depth;
     a.S = S;
     a.sleep_ns = 200;
     // test hook for the bounded waits: with BISCO_TEST_WITHHOLD_COPIES set the
     // kernel requests no data, so its waits expire, it latches
     // BISCO_ERR_TIMEOUT and returns with no copy in flight
     a.withhold = getenv("BISCO_TEST_WITHHOLD_COPIES") != nullptr;
-    b1_layout(C, depth, p_max, items_max, a.q8_staged ? q8_max : 0, &a);
+    b1_layout(C, pick.nw, pick.depth, pick.ips, p_max, items_max, a.q8_staged ? q8_max : 0, &a);
     *launched = true;
-    const bool one = a.nspan == 1;
-    if (depth == 3) return one ? launch_b1_t<3, 1>(a, total, smem, stream) : launch_b1_t<3, 0>(a, total, smem, stream);
-    return one ? launch_b1_t<2, 1>(a, total, smem, stream) : launch_b1_t<2, 0>(a, total, smem, stream);
+    if (one) {
+        if (pick.depth == 3) return launch_b1_t<16, 3, 1, 1>(a, total, smem, stream);
+        return launch_b1_t<16, 2, 1, 1>(a, total, smem, stream);
+    }
+    if (pick.depth == 3) return launch_b1_t<16, 3, 1, 0>(a, total, smem, stream);
+    return launch_b1_t<16, 2, 1, 0>(a, total, smem, stream);
 }
 }  // namespace bisco
