@@ -349,6 +349,9 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
         spidx[u] = j;
         ssc[u] = sc;
     }
+    // x into L2 now (a prefetch moves no data into the CTA, so it is safe
+    // ahead of the wait on a kernel that may still be writing x); read after
+    if (threadIdx.x == 32) prefetch_l2(a.x, static_cast<uint32_t>(K) * 2u);
     if (p > 0 && nrows > 0) {
         if (a.q8_staged) {
             const int n16 = nrows * p_pad / 16;
