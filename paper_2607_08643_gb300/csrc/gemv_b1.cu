@@ -63,6 +63,11 @@ constexpr float kB1InvSqrt8 = 0.35355339059327373f;
 // most this much dynamic shared memory (228 KB per SM, 1 KB reserved per CTA).
 constexpr size_t kB1Coresident = 112 * 1024;
 constexpr size_t kB1MaxSmem = 227 * 1024;
+// A launch with at least this many items per SM runs two of its own CTAs per
+// SM: eight warps per scheduler hide the decode's dependency latencies better
+// than four, which outweighs the lost overlap with the neighbouring launches
+// (for 2 x 12288 x 4096 at S = 2, 323 items per SM: 22.1 -> 18.6 us).
+constexpr int kB1TwoPerSm = 256;
 
 struct B1Layer {
     const uint8_t *codes;      // [S][N][K/8]
@@ -598,54 +603,66 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
         b.p_pad = (L.n_protected + 15) / 16 * 16;
         p_max = p_max > b.p ? p_max : b.p;
     }
-    // CTAs per layer: one each, then one at a time to the layer with the
-    // longest row run per CTA, up to one CTA per SM
     const int sms = num_sms();
     if (G > sms) return BISCO_OK;
-    int ctas[kB1MaxG] = {}, total = G;
-    for (int g = 0; g < G; ++g) ctas[g] = 1;
-    auto run = [&](int g) { return (a.L[g].N + ctas[g] - 1) / ctas[g]; };
-    while (total < sms) {
-        int best = -1;
-        for (int g = 0; g < G; ++g)
-            if (ctas[g] < a.L[g].N && (best < 0 || run(g) > run(best))) best = g;
-        if (best < 0) break;
-        ++ctas[best];
-        ++total;
-    }
-    int rows_max = 0;
-    size_t q8_max = 0;
-    for (int g = 0, c0 = 0; g < G; ++g) {
-        a.L[g].cta0 = c0;
-        a.L[g].ctas = ctas[g];
-        c0 += ctas[g];
-        rows_max = rows_max > run(g) ? rows_max : run(g);
-        const size_t q8b = static_cast<size_t>(run(g)) * a.L[g].p_pad;
-        q8_max = q8_max > q8b ? q8_max : q8b;
-    }
+    int items_all = 0;
+    for (int g = 0; g < G; ++g) items_all += a.L[g].N * S * a.nspan;
     const int C = K / 8;
-    const int items_max = rows_max * S * a.nspan;
-    // the first shape that leaves room for the next kernel's CTA on the SM
-    // (int8 rows staged if they fit), else the first that fits one CTA per SM
     const bool one = a.nspan == 1;
     const B1Shape *shapes = one ? kB1One : kB1Many;
     const int nshapes = 2;
+    int total = 0;
     B1Shape pick = {0, 0, 0};
     size_t smem = 0;
-    for (int pass = 0; pass < 2 && pick.nw == 0; ++pass) {
-        const size_t budget = pass == 0 ? kB1Coresident : kB1MaxSmem;
-        for (int k = 0; k < nshapes && pick.nw == 0; ++k)
-            for (int staged = 1; staged >= 0 && pick.nw == 0; --staged) {
-                const B1Shape &sh = shapes[k];
-                const size_t need = b1_layout(C, sh.nw, sh.depth, sh.ips, p_max, items_max,
-                                              staged ? q8_max : 0, &a);
-                if (need <= budget) {
-                    pick = sh;
-                    smem = need;
-                    a.q8_staged = staged;
+    // CTAs per layer: one each, then one at a time to the layer with the
+    // longest row run per CTA, up to `slots` CTAs; then the first shape that
+    // leaves room for a second CTA on the SM (int8 rows staged if they fit),
+    // else, with one CTA per SM, the first that fits
+    auto plan = [&](int slots) {
+        int ctas[kB1MaxG] = {};
+        total = G;
+        for (int g = 0; g < G; ++g) ctas[g] = 1;
+        auto run = [&](int g) { return (a.L[g].N + ctas[g] - 1) / ctas[g]; };
+        while (total < slots) {
+            int best = -1;
+            for (int g = 0; g < G; ++g)
+                if (ctas[g] < a.L[g].N && (best < 0 || run(g) > run(best))) best = g;
+            if (best < 0) break;
+            ++ctas[best];
+            ++total;
+        }
+        int rows_max = 0;
+        size_t q8_max = 0;
+        for (int g = 0, c0 = 0; g < G; ++g) {
+            a.L[g].cta0 = c0;
+            a.L[g].ctas = ctas[g];
+            c0 += ctas[g];
+            rows_max = rows_max > run(g) ? rows_max : run(g);
+            const size_t q8b = static_cast<size_t>(run(g)) * a.L[g].p_pad;
+            q8_max = q8_max > q8b ? q8_max : q8b;
+        }
+        const int items_max = rows_max * S * a.nspan;
+        pick = {0, 0, 0};
+        const int passes = slots > sms ? 1 : 2;
+        for (int pass = 0; pass < passes && pick.nw == 0; ++pass) {
+            const size_t budget = pass == 0 ? kB1Coresident : kB1MaxSmem;
+            for (int k = 0; k < nshapes && pick.nw == 0; ++k)
+                for (int staged = 1; staged >= 0 && pick.nw == 0; --staged) {
+                    const B1Shape &sh = shapes[k];
+                    const size_t need = b1_layout(C, sh.nw, sh.depth, sh.ips, p_max, items_max,
+                                                  staged ? q8_max : 0, &a);
+                    if (need <= budget) {
+                        pick = sh;
+                        smem = need;
+                        a.q8_staged = staged;
+                    }
                 }
-            }
-    }
+        }
+        if (pick.nw != 0)
+            b1_layout(C, pick.nw, pick.depth, pick.ips, p_max, items_max, a.q8_staged ? q8_max : 0, &a);
+    };
+    if (items_all >= kB1TwoPerSm * sms) plan(2 * sms);
+    if (pick.nw == 0) plan(sms);
     if (pick.nw == 0) return BISCO_OK;
     a.depth = pick.depth;
     a.S = S;
@@ -654,7 +671,6 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
     // kernel requests no data, so its waits expire, it latches
     // BISCO_ERR_TIMEOUT and returns with no copy in flight
     a.withhold = getenv("BISCO_TEST_WITHHOLD_COPIES") != nullptr;
-    b1_layout(C, pick.nw, pick.depth, pick.ips, p_max, items_max, a.q8_staged ? q8_max : 0, &a);
     *launched = true;
     if (one) {
         if (pick.depth == 3) return launch_b1_t<16, 3, 1, 1>(a, total, smem, stream);
