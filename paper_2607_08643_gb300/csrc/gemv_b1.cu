@@ -54,7 +54,6 @@
 namespace bisco {
 namespace {
 
-constexpr int kB1Warps = 16;
 constexpr int kB1Span = 512;                  // chunks per item
 constexpr uint32_t kB1Item = 1536;            // bytes per item slot: signs, then norms
 constexpr int kB1MaxG = 4;                    // layers per launch
@@ -91,7 +90,7 @@ struct B1Args {
     int q8_staged;             // int8 rows in shared memory (else read at the end)
     uint32_t sleep_ns;         // suspend-time hint of the item waits
     int withhold;              // test of the bounded waits: request no copies
-    uint32_t off_ring, off_pm, off_pidx, off_sx, off_part, off_q8, off_bar;   // tables at 0
+    uint32_t off_ring, off_pm, off_pidx, off_sx, off_part, off_prot, off_q8, off_bar;   // tables at 0
 };
 
 template <uint32_t A>
@@ -154,31 +153,23 @@ __device__ __forceinline__ float b1_item(const uint2 (&cw)[2], const uint4 (&nw)
     return (acc4[0][0] + acc4[0][1]) + (acc4[1][0] + acc4[1][1]);
 }
 
-// Lane 0 of the warp arms a slot's mbarrier for `bytes` (after a proxy fence:
-// the warp's reads of the slot are done) and, in b1_copy, issues one item's
-// two bulk copies (signs to cdst, norms to ndst); the other lanes run the
-// same instruction stream with the predicate off, so the warp never
-// diverges.
-__device__ __forceinline__ void b1_arm(bool leader, uint32_t bar, uint32_t bytes) {
+// Lane 0 of the warp requests one item into a ring slot: after a proxy fence
+// (the warp's reads of the slot are done) it arms the slot's mbarrier for
+// 1536 bytes and issues the two bulk copies (signs to the slot, norms 512
+// bytes on); the other lanes run the same instructions with the predicate
+// off, so the warp never diverges.
+__device__ __forceinline__ void b1_request(uint32_t lead, uint32_t slot, uint32_t bar, const void *csrc,
+                                           const void *nsrc, uint64_t pol) {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "setp.ne.u32 p, %0, 0;\n\t"
         "@p fence.proxy.async.shared::cta;\n\t"
-        "@p mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%1], %2;\n\t}"
-        ::"r"(static_cast<uint32_t>(leader)), "r"(bar), "r"(bytes) : "memory");
-}
-
-__device__ __forceinline__ void b1_copy(bool leader, uint32_t cdst, uint32_t ndst, uint32_t bar,
-                                        const void *codes, const void *norms, uint64_t pol) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.u32 p, %0, 0;\n\t"
+        "@p mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%2], 1536;\n\t"
         "@p cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-        " [%1], [%4], 512, [%3], %6;\n\t"
+        " [%1], [%3], 512, [%2], %5;\n\t"
         "@p cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-        " [%2], [%5], 1024, [%3], %6;\n\t}"
-        ::"r"(static_cast<uint32_t>(leader)), "r"(cdst), "r"(ndst), "r"(bar), "l"(codes), "l"(norms),
-          "l"(pol)
+        " [%6], [%4], 1024, [%2], %5;\n\t}"
+        ::"r"(lead), "r"(slot), "r"(bar), "l"(csrc), "l"(nsrc), "l"(pol), "r"(slot + 512u)
         : "memory");
 }
 
@@ -238,18 +229,15 @@ __device__ __forceinline__ uint4 b1_table_x(const uint16_t *x, int sp, int J, in
     return *reinterpret_cast<const uint4 *>(x + 8 * c);
 }
 
-// NW warps; D ring slots per warp of IPS items each; NSPAN 4096-column spans
+// NW warps; D ring slots (one item each) per warp; NSPAN 4096-column spans
 // per row (0: a.nspan > 1, at run time).  With one span, every ring address
 // is an immediate offset; with several, a CTA holds the table of one span at
 // a time and walks its items span by span, rebuilding the table between
 // spans (x of the next span is loaded while the current one is decoded).
-template <int NW, int D, int IPS, int NSPAN>
+template <int NW, int D, int NSPAN>
 __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ B1Args a) {
-    static_assert(D * IPS <= 4, "one folded reduction covers a ring pass");
-    static_assert(NSPAN == 1 || IPS == 1, "several spans: one item per slot");
+    static_assert(D <= 4, "one folded reduction covers a ring pass");
     constexpr int kThreads = NW * 32;
-    constexpr uint32_t kSlot = IPS * kB1Item;          // [signs of IPS items][norms of IPS items]
-    constexpr uint32_t kNormOff = IPS * 512u;
     extern __shared__ unsigned char smem_raw[];
     unsigned char *sm = align_smem<4096>(smem_raw);
     const uint32_t sbase = smem_u32(sm);
@@ -278,6 +266,7 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     float *ssc = reinterpret_cast<float *>(spidx + (p + 3) / 4 * 4);
     float *sx = reinterpret_cast<float *>(sm + a.off_sx);         // scale * x [p]
     float *part = reinterpret_cast<float *>(sm + a.off_part);     // [S * nrows * nspan]
+    float *prot = reinterpret_cast<float *>(sm + a.off_prot);     // protected term [nrows]
     int8_t *q8s = reinterpret_cast<int8_t *>(sm + a.off_q8);
     const uint64_t pol = l2_evict_first_policy();
 
@@ -288,46 +277,39 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     const int kb0 = per_span * warp / NW;
     const int cnt0 = per_span * (warp + 1) / NW - kb0;
     const int total = cnt0 * nspan;   // this warp's items
-    const uint32_t wring = sbase + a.off_ring + static_cast<uint32_t>(warp * D) * kSlot;
+    const uint32_t wring = sbase + a.off_ring + static_cast<uint32_t>(warp * D) * kB1Item;
     const uint32_t wbar = sbase + a.off_bar + static_cast<uint32_t>(warp * D) * 8u;
-    // issue cursor (uniform over the warp): span, stage, row and items left in
-    // this span's run of the next item to request, and its element offset
-    const int s0 = nrows > 0 ? kb0 / nrows : 0, rr0 = kb0 - s0 * nrows;
-    int csp = 0, cs = s0, crr = rr0, cleft = cnt0;
-    int64_t ie = (static_cast<int64_t>(cs) * N + ra + crr) * C;
-    auto advance = [&]() {
-        ++crr;
-        ie += C;
-        if (crr == nrows) {
-            crr = 0;
-            ++cs;
-            ie = (static_cast<int64_t>(cs) * N + ra) * C + csp * kB1Span;
-        }
-        if (--cleft == 0) {
-            ++csp;
-            cs = s0;
-            crr = rr0;
-            cleft = cnt0;
-            ie = (static_cast<int64_t>(cs) * N + ra + crr) * C + csp * kB1Span;
-        }
-    };
-    // slot d: the next up to IPS items (withheld: none, every wait runs out
-    // with nothing in flight)
-    const int to_issue = a.withhold ? 0 : total;
-    int issued = 0;
+    // request cursor (uniform over the warp): byte offset of the next item's
+    // signs in codes (its norms at twice that in norms; below 2^32, checked
+    // on the host), items left in its row run (at the end of a run the next
+    // stage's rows follow, N - nrows rows on) and in its span's run
+    const int s0 = nrows > 0 ? kb0 / nrows : 0, r0 = kb0 - s0 * nrows;
+    const uint32_t off0 = (static_cast<uint32_t>(s0) * N + ra + r0) * static_cast<uint32_t>(C);
+    const uint32_t gap = static_cast<uint32_t>(N - nrows) * C;
+    uint32_t off = off0;
+    int rleft = nrows - r0, cleft = cnt0, csp = 0;
+    const uint32_t lead = lane == 0;
+    const unsigned char *const nbytes = reinterpret_cast<const unsigned char *>(norms);
+    // items still to request (withheld: none, every wait runs out with
+    // nothing in flight)
+    const int to_request = a.withhold ? 0 : total;
+    int left = to_request;
     auto fill = [&](int d) {
-        const int n = min(IPS, to_issue - issued);
-        if (n <= 0) return;
-        const uint32_t slot = wring + d * kSlot, bar = wbar + d * 8u;
-        b1_arm(lane == 0, bar, n * kB1Item);
-#pragma unroll
-        for (int it = 0; it < IPS; ++it)
-            if (it < n) {
-                b1_copy(lane == 0, slot + it * 512u, slot + kNormOff + it * 1024u, bar, codes + ie,
-                        norms + ie, pol);
-                advance();
+        b1_request(lead, wring + d * kB1Item, wbar + d * 8u, codes + off, nbytes + 2ull * off, pol);
+        --left;
+        off += C;
+        if (--rleft == 0) {
+            off += gap;
+            rleft = nrows;
+        }
+        if constexpr (NSPAN != 1) {
+            if (--cleft == 0) {
+                ++csp;
+                off = off0 + static_cast<uint32_t>(csp) * kB1Span;
+                rleft = nrows - r0;
+                cleft = cnt0;
             }
-        issued += n;
+        }
     };
 
     // ---- before the wait: barriers, first items, protected metadata, int8 rows
@@ -337,7 +319,8 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     }
     __syncwarp();
 #pragma unroll
-    for (int d = 0; d < D; ++d) fill(d);
+    for (int d = 0; d < D; ++d)
+        if (left > 0) fill(d);
     if (threadIdx.x == 0) s_abort = 0;
     for (int i = threadIdx.x; i < C / 4; i += kThreads) pm[i] = 0u;
     __syncthreads();
@@ -393,10 +376,10 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
 
     const uint32_t base0 = sbase + lane * 4u;
     int i = 0;   // items consumed
-    // slot d: wait for it, decode its n items into this lane's partial sums
-    // v[0..n), refill it; false on a timeout
-    auto slot_items = [&](int d, uint32_t phase, int n, float *v) -> bool {
-        const uint32_t slot = wring + d * kSlot, bar = wbar + d * 8u;
+    // slot d: wait for it, decode its item into this lane's partial sum,
+    // request the next item into it; false on a timeout
+    auto slot_item = [&](int d, uint32_t phase, float &v) -> bool {
+        const uint32_t slot = wring + d * kB1Item, bar = wbar + d * 8u;
         if (!__all_sync(0xFFFFFFFFu, mbar_try_wait(bar, phase)) &&
             !__all_sync(0xFFFFFFFFu, mbar_wait_sleep(bar, phase, a.sleep_ns))) {
             if (lane == 0) {
@@ -405,40 +388,32 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
             }
             return false;
         }
-#pragma unroll
-        for (int it = 0; it < IPS; ++it)
-            if (it < n) {
-                uint2 cw[2];
-                uint4 nw[2];
-                cw[0] = lds_u64(slot + it * 512u + lane * 8u);
-                cw[1] = lds_u64(slot + it * 512u + 256u + lane * 8u);
-                nw[0] = lds_u128(slot + kNormOff + it * 1024u + lane * 16u);
-                nw[1] = lds_u128(slot + kNormOff + it * 1024u + 512u + lane * 16u);
-                v[it] = b1_item(cw, nw, base0);
-            }
-        // the slot's reads are done (the values are in registers): refill it
+        uint2 cw[2];
+        uint4 nw[2];
+        cw[0] = lds_u64(slot + lane * 8u);
+        cw[1] = lds_u64(slot + 256u + lane * 8u);
+        nw[0] = lds_u128(slot + 512u + lane * 16u);
+        nw[1] = lds_u128(slot + 1024u + lane * 16u);
+        // the slot's reads are done (the values are in registers, ordered
+        // before the refill by the warp barrier and the proxy fence): refill
+        // it before the decode, so the copy's latency overlaps the decode
         __syncwarp();
-        fill(d);
+        if (left > 0) fill(d);
+        v = b1_item(cw, nw, base0);
         return true;
     };
     if constexpr (NSPAN == 1) {
-        // ---- decode: D slots (D * IPS items) a pass; the partial sums of a
-        // pass are added over the warp together
+        // ---- decode: D items a pass; their partial sums are added over the
+        // warp together
         uint32_t phase = 0;
-        bool ok = true;
-        for (int i0 = 0; i0 < total && ok; i0 += D * IPS, phase ^= 1u) {
+        for (int i0 = 0; i0 < total; i0 += D, phase ^= 1u) {
             float v[4] = {0.f, 0.f, 0.f, 0.f};
-            int n = 0;
+            const int n = min(D, total - i0);
+            bool ok = true;
 #pragma unroll
-            for (int d = 0; d < D; ++d) {
-                const int m = min(IPS, total - (i0 + d * IPS));
-                if (m <= 0) break;
-                if (!slot_items(d, phase, m, v + d * IPS)) {
-                    ok = false;
-                    break;
-                }
-                n = d * IPS + m;
-            }
+            for (int d = 0; d < D; ++d)
+                if (ok && d < n) ok = slot_item(d, phase, v[d]);
+            if (!ok) break;
             const float r = warp_sum4(v[0], v[1], v[2], v[3], lane);   // value lane >> 3, every lane
             if ((lane & 7) == 0 && (lane >> 3) < n) part[kb0 + i0 + (lane >> 3)] = r;
             i = i0 + n;
@@ -446,10 +421,13 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     } else {
         // ---- decode span by span; the table of span sp replaces that of sp - 1
         bool ok = true;
+        int d = 0;
+        uint32_t phase = 0;
         uint4 xn[(16 + NW - 1) / NW];
 #pragma unroll
         for (int q = 0; q < (16 + NW - 1) / NW; ++q)
             if (warp + q * NW < 16 && nspan > 1) xn[q] = b1_table_x(a.x, 1, warp + q * NW, lane);
+        // (after a timeout the warp still passes every span's barriers)
         for (int sp = 0; sp < nspan; ++sp) {
             if (sp > 0) {
                 __syncthreads();   // every warp is done with the table of span sp - 1
@@ -464,53 +442,81 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
             // four items at a time, their partial sums added over the warp together
             for (int j0 = 0; j0 < cnt0 && ok; j0 += 4) {
                 float v[4] = {0.f, 0.f, 0.f, 0.f};
-                int n = 0;
+                const int n = min(4, cnt0 - j0);
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    if (j0 + q >= cnt0) break;
-                    if (!slot_items(i % D, static_cast<uint32_t>(i / D) & 1u, 1, v + q)) {
-                        ok = false;
-                        break;
+                for (int q = 0; q < 4; ++q)
+                    if (ok && q < n) {
+                        ok = slot_item(d, phase, v[q]);
+                        if (++d == D) {
+                            d = 0;
+                            phase ^= 1u;
+                        }
                     }
-                    ++i;
-                    n = q + 1;
-                }
+                if (!ok) break;
                 const float r = warp_sum4(v[0], v[1], v[2], v[3], lane);
                 if ((lane & 7) == 0 && (lane >> 3) < n) part[sp * per_span + kb0 + j0 + (lane >> 3)] = r;
+                i += n;
             }
         }
     }
-    // every copy this warp issued has landed before it leaves the ring: the
-    // slots of the items requested and not consumed
+    // every copy this warp requested has landed before it leaves the ring:
+    // the slots of the items requested and not consumed (only after a
+    // timeout; their slot for item j is j % D, its phase (j / D) & 1)
+    const int requested = to_request - left;
     if (lane == 0)
-        for (int j = (i + IPS - 1) / IPS; j < (issued + IPS - 1) / IPS; ++j)
+        for (int j = i; j < requested; ++j)
             mbar_wait(wbar + static_cast<uint32_t>(j % D) * 8u, static_cast<uint32_t>(j / D) & 1u);
+
+    // ---- the protected term of rows warp, warp + NW, ... (Eq. 10), while
+    // other warps may still decode: four rows at a time, all their int8
+    // loads issued before the first product, then added over the warp
+    // together
+    if (p > 0) {
+        for (int rr0 = warp; rr0 < nrows; rr0 += 4 * NW) {
+            float pr[4] = {0.f, 0.f, 0.f, 0.f};
+            for (int u0 = 0; u0 < p; u0 += 64) {
+                int qv[4][2];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const int rr = rr0 + k * NW;
+                    const int8_t *q8r = a.q8_staged ? q8s + rr * p_pad : q8 + static_cast<int64_t>(ra + rr) * p_pad;
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const int u = u0 + 32 * h + lane;
+                        qv[k][h] = rr < nrows && u < p ? q8r[u] : 0;
+                    }
+                }
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const int u = u0 + 32 * h + lane;
+                        if (u < p) pr[k] = fmaf(static_cast<float>(qv[k][h]), sx[u], pr[k]);
+                    }
+            }
+            const float r = warp_sum4(pr[0], pr[1], pr[2], pr[3], lane);   // row rr0 + (lane >> 3) * NW
+            const int rr = rr0 + (lane >> 3) * NW;
+            if ((lane & 7) == 0 && rr < nrows) prot[rr] = r;
+        }
+    }
     __syncthreads();
     if (*reinterpret_cast<volatile int *>(&s_abort)) return;
 
-    // ---- outputs: a warp per row; items in order, then the protected term
-    for (int rr = warp; rr < nrows; rr += NW) {
-        float pr = 0.f;
-        if (p > 0) {
-            const int8_t *q8r = a.q8_staged ? q8s + rr * p_pad : q8 + static_cast<int64_t>(ra + rr) * p_pad;
-            for (int u = lane; u < p; u += 32) pr = fmaf(static_cast<float>(q8r[u]), sx[u], pr);
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) pr += __shfl_xor_sync(0xFFFFFFFFu, pr, o);
-        }
-        if (lane == 0) {
-            float v = 0.f;
-            for (int sp = 0; sp < nspan; ++sp)
-                for (int s = 0; s < S; ++s) v += part[sp * per_span + s * nrows + rr];
-            y[ra + rr] = v * kB1InvSqrt8 + pr;
-        }
+    // ---- outputs: a thread per row; the row's item sums in order, then the
+    // protected term
+    for (int rr = threadIdx.x; rr < nrows; rr += kThreads) {
+        float v = 0.f;
+        for (int sp = 0; sp < nspan; ++sp)
+            for (int s = 0; s < S; ++s) v += part[sp * per_span + s * nrows + rr];
+        y[ra + rr] = v * kB1InvSqrt8 + (p > 0 ? prot[rr] : 0.f);
     }
 }
 
 size_t align_up_b1(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
-template <int NW, int D, int IPS, int NSPAN>
+template <int NW, int D, int NSPAN>
 bisco_status launch_b1_t(const B1Args &a, int grid, size_t smem, cudaStream_t stream) {
-    auto kern = k_gemv_b1<NW, D, IPS, NSPAN>;
+    auto kern = k_gemv_b1<NW, D, NSPAN>;
     static size_t configured[64] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return BISCO_ERR_CUDA;
@@ -533,14 +539,14 @@ bisco_status launch_b1_t(const B1Args &a, int grid, size_t smem, cudaStream_t st
     return cudaLaunchKernelEx(&cfg, kern, a) == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
 }
 
-// Shared memory of one CTA of nw warps with `depth` slots of ips items per
+// Shared memory of one CTA of nw warps with `depth` one-item slots per
 // warp, past the 4 KB aligned base (the span table first); fills the offsets
 // of `a`.
-size_t b1_layout(int C, int nw, int depth, int ips, int p_max, int items_max, size_t q8_bytes,
+size_t b1_layout(int C, int nw, int depth, int p_max, int rows_max, int items_max, size_t q8_bytes,
                  B1Args *a) {
     size_t off = static_cast<size_t>(kB1Span) * 64;   // the table of one span: 64 bytes per chunk
     a->off_ring = static_cast<uint32_t>(off);
-    off += static_cast<size_t>(nw) * depth * ips * kB1Item;
+    off += static_cast<size_t>(nw) * depth * kB1Item;
     a->off_pm = static_cast<uint32_t>(off);
     off += static_cast<size_t>(C);                          // one bit per column
     a->off_pidx = static_cast<uint32_t>(off);
@@ -550,6 +556,8 @@ size_t b1_layout(int C, int nw, int depth, int ips, int p_max, int items_max, si
     off = align_up_b1(off, 16);
     a->off_part = static_cast<uint32_t>(off);
     off += static_cast<size_t>(items_max) * 4;
+    a->off_prot = static_cast<uint32_t>(off);
+    off += static_cast<size_t>(rows_max) * 4;
     off = align_up_b1(off, 16);
     a->off_q8 = static_cast<uint32_t>(off);
     off += q8_bytes;
@@ -565,10 +573,9 @@ size_t b1_layout(int C, int nw, int depth, int ips, int p_max, int items_max, si
 // registers) run the 36x7 step 8 % slower than 16 warps with one item per
 // slot -- latency is hidden by warps more than by the slot work saved.
 struct B1Shape {
-    int nw, depth, ips;
+    int nw, depth;
 };
-constexpr B1Shape kB1One[] = {{16, 3, 1}, {16, 2, 1}};
-constexpr B1Shape kB1Many[] = {{16, 3, 1}, {16, 2, 1}};
+constexpr B1Shape kB1Shapes[] = {{16, 3}, {16, 2}};
 
 }  // namespace
 
@@ -591,6 +598,8 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
         const bisco_layer &L = Ls[g];
         if (L.k_in != K || L.stages != S || L.protect_axis != 0 || L.protect_format != BISCO_PROT_INT8)
             return BISCO_OK;
+        // the kernel's byte offsets into the sign planes are 32-bit
+        if (static_cast<uint64_t>(S) * L.n_out * (K / 8) >= (1ull << 32)) return BISCO_OK;
         B1Layer &b = a.L[g];
         b.codes = reinterpret_cast<const uint8_t *>(L.codes);
         b.norms = L.norms;
@@ -609,10 +618,10 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
     for (int g = 0; g < G; ++g) items_all += a.L[g].N * S * a.nspan;
     const int C = K / 8;
     const bool one = a.nspan == 1;
-    const B1Shape *shapes = one ? kB1One : kB1Many;
+    const B1Shape *shapes = kB1Shapes;
     const int nshapes = 2;
     int total = 0;
-    B1Shape pick = {0, 0, 0};
+    B1Shape pick = {0, 0};
     size_t smem = 0;
     // CTAs per layer: one each, then one at a time to the layer with the
     // longest row run per CTA, up to `slots` CTAs; then the first shape that
@@ -642,14 +651,14 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
             q8_max = q8_max > q8b ? q8_max : q8b;
         }
         const int items_max = rows_max * S * a.nspan;
-        pick = {0, 0, 0};
+        pick = {0, 0};
         const int passes = slots > sms ? 1 : 2;
         for (int pass = 0; pass < passes && pick.nw == 0; ++pass) {
             const size_t budget = pass == 0 ? kB1Coresident : kB1MaxSmem;
             for (int k = 0; k < nshapes && pick.nw == 0; ++k)
                 for (int staged = 1; staged >= 0 && pick.nw == 0; --staged) {
                     const B1Shape &sh = shapes[k];
-                    const size_t need = b1_layout(C, sh.nw, sh.depth, sh.ips, p_max, items_max,
+                    const size_t need = b1_layout(C, sh.nw, sh.depth, p_max, rows_max, items_max,
                                                   staged ? q8_max : 0, &a);
                     if (need <= budget) {
                         pick = sh;
@@ -659,7 +668,7 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
                 }
         }
         if (pick.nw != 0)
-            b1_layout(C, pick.nw, pick.depth, pick.ips, p_max, items_max, a.q8_staged ? q8_max : 0, &a);
+            b1_layout(C, pick.nw, pick.depth, p_max, rows_max, items_max, a.q8_staged ? q8_max : 0, &a);
     };
     if (items_all >= kB1TwoPerSm * sms) plan(2 * sms);
     if (pick.nw == 0) plan(sms);
@@ -673,10 +682,10 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
     a.withhold = getenv("BISCO_TEST_WITHHOLD_COPIES") != nullptr;
     *launched = true;
     if (one) {
-        if (pick.depth == 3) return launch_b1_t<16, 3, 1, 1>(a, total, smem, stream);
-        return launch_b1_t<16, 2, 1, 1>(a, total, smem, stream);
+        if (pick.depth == 3) return launch_b1_t<16, 3, 1>(a, total, smem, stream);
+        return launch_b1_t<16, 2, 1>(a, total, smem, stream);
     }
-    if (pick.depth == 3) return launch_b1_t<16, 3, 1, 0>(a, total, smem, stream);
-    return launch_b1_t<16, 2, 1, 0>(a, total, smem, stream);
+    if (pick.depth == 3) return launch_b1_t<16, 3, 0>(a, total, smem, stream);
+    return launch_b1_t<16, 2, 0>(a, total, smem, stream);
 }
 }  // namespace bisco
