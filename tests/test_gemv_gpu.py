@@ -289,13 +289,13 @@ def test_gemv_batch1_zero_activations(env):
 
 
 # ------------------------------------------------- batch 1, row-split kernel
-# K a multiple of 4096 at batch 1 goes to the row-split kernel: every CTA
-# takes an equal run of the launch's rows (across the layers of a group),
-# codes and norms go straight to registers, and each CTA builds masked
-# tables for the (at most two) layers its rows touch.  The cases cover rows
-# fewer than SMs, ragged row runs, S = 1..3, K = 4096 / 8192 / 12288, layers
+# K a multiple of 4096 at batch 1 goes to the row-split kernel: each layer
+# of a launch gets whole CTAs, each CTA a run of rows that it walks span by
+# span (4096 columns, one table at a time), each warp a run of the CTA's
+# items through its own ring of bulk copies.  The cases cover rows fewer
+# than SMs, ragged row runs, S = 1..3, K = 4096 / 8192 / 12288, layers
 # without protection, int8 rows too large to stage in shared memory, and
-# groups whose layer boundaries fall inside CTAs.
+# groups of several layers.
 
 @pytest.mark.parametrize("N,K,S,p", [
     (16, 4096, 1, 0),          # 16 rows: 16 one-row CTAs
@@ -317,14 +317,15 @@ def test_gemv_b1_matches_oracle(env, N, K, S, p):
     assert np.array_equal(y, run_gemv(env, Lref, X))
 
 
-@pytest.mark.parametrize("shapes", [
-    [(300, 21), (64, 0), (1000, 33)],                 # layer boundaries inside CTAs
-    [(4096, 41), (1024, 41), (1024, 41)],             # q/k/v of one attention layer
-    [(3000, 41), (2000, 0), (1500, 41), (4000, 10)],  # four layers
-    [(200, 5), (7, 3), (150, 0)],                     # a CTA over three layers: other kernel
+@pytest.mark.parametrize("K,shapes", [
+    (4096, [(300, 21), (64, 0), (1000, 33)]),                 # layers of unequal row counts
+    (4096, [(4096, 41), (1024, 41), (1024, 41)]),             # q/k/v of one attention layer
+    (4096, [(3000, 41), (2000, 0), (1500, 41), (4000, 10)]),  # four layers
+    (4096, [(200, 5), (7, 3), (150, 0)]),                     # a 7-row layer between larger ones
+    (12288, [(700, 123), (90, 0), (333, 60)]),                # three spans, three layers
 ])
-def test_gemv_b1_groups_match_oracle(env, shapes):
-    K, S = 4096, 2
+def test_gemv_b1_groups_match_oracle(env, K, shapes):
+    S = 2
     Lrefs = [oracle.encode(synth.layer_weights(N, K, seed=200 + i), S=S, p=p)
              for i, (N, p) in enumerate(shapes)]
     X = synth.activations(1, K, seed=201)

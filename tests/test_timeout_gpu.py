@@ -25,10 +25,13 @@ def env():
     return bisco, dev
 
 
-def test_expired_wait_reports_timeout_and_the_next_call_is_correct(env, monkeypatch):
+@pytest.mark.parametrize("N,K,S,p", [
+    (600, 4096, 2, 41),       # one span
+    (400, 12288, 2, 123),     # three spans: the barriers between spans are still passed
+])
+def test_expired_wait_reports_timeout_and_the_next_call_is_correct(env, monkeypatch, N, K, S, p):
     import torch
     bisco, dev = env
-    N, K, S, p = 600, 4096, 2, 41          # the batch-1 row-split kernel
     Lref = oracle.encode(synth.layer_weights(N, K, seed=301), S=S, p=p)
     L = bisco.Layer.from_numpy(Lref, dev)
     X = synth.activations(1, K, seed=302)
