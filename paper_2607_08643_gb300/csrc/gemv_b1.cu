@@ -58,14 +58,13 @@ constexpr int kB1Span = 512;                  // chunks per item
 constexpr uint32_t kB1Item = 1536;            // bytes per item slot: signs, then norms
 constexpr int kB1MaxG = 4;                    // layers per launch
 constexpr float kB1InvSqrt8 = 0.35355339059327373f;
-// Two CTAs (this layer's and the next one's) share an SM when each takes at
-// most this much dynamic shared memory (228 KB per SM, 1 KB reserved per CTA).
-constexpr size_t kB1Coresident = 112 * 1024;
-constexpr size_t kB1MaxSmem = 227 * 1024;
+// dynamic shared memory of one CTA at most (227 KB per block less the
+// kernel's static shared memory, rounded down)
+constexpr size_t kB1MaxSmem = 226 * 1024;
 // A launch with at least this many items per SM runs two of its own CTAs per
-// SM: eight warps per scheduler hide the decode's dependency latencies better
-// than four, which outweighs the lost overlap with the neighbouring launches
-// (for 2 x 12288 x 4096 at S = 2, 323 items per SM: 22.1 -> 18.6 us).
+// SM: twice the copies in flight and twice the decoding warps outweigh the
+// lost overlap with the neighbouring launches (for 2 x 12288 x 4096 at S = 2,
+// 323 items per SM: 22.1 -> 18.6 us).
 constexpr int kB1TwoPerSm = 256;
 
 struct B1Layer {
@@ -539,6 +538,38 @@ bisco_status launch_b1_t(const B1Args &a, int grid, size_t smem, cudaStream_t st
     return cudaLaunchKernelEx(&cfg, kern, a) == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
 }
 
+// The most dynamic shared memory at which two CTAs of the kernel (this
+// layer's and the next one's) share an SM, from the runtime's occupancy
+// calculator (every instantiation has the same block size and static
+// shared memory); found once per device.
+size_t b1_coresident_budget() {
+    static size_t budget[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    if (budget[dev] != 0) return budget[dev];
+    auto kern = k_gemv_b1<16, 3, 1>;
+    constexpr size_t kHi = 160 * 1024;   // more than two CTAs of an SM can hold
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kHi)) !=
+        cudaSuccess) {
+        (void)cudaGetLastError();
+        return 0;
+    }
+    auto two = [&](size_t smem) {
+        int n = 0;
+        const bool ok = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, 16 * 32, smem) == cudaSuccess;
+        if (!ok) (void)cudaGetLastError();
+        return ok && n >= 2;
+    };
+    size_t lo = 0, hi = kHi;   // two(lo) or lo = 0; not two(hi)
+    while (hi - lo > 16) {
+        const size_t mid = (lo + hi) / 2 / 16 * 16;
+        if (two(mid)) lo = mid;
+        else hi = mid;
+    }
+    budget[dev] = lo > 0 ? lo : 1;
+    return budget[dev];
+}
+
 // Shared memory of one CTA of nw warps with `depth` one-item slots per
 // warp, past the 4 KB aligned base (the span table first); fills the offsets
 // of `a`.
@@ -614,6 +645,7 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
     }
     const int sms = num_sms();
     if (G > sms) return BISCO_OK;
+    const size_t coresident = b1_coresident_budget();
     int items_all = 0;
     for (int g = 0; g < G; ++g) items_all += a.L[g].N * S * a.nspan;
     const int C = K / 8;
@@ -654,7 +686,7 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
         pick = {0, 0};
         const int passes = slots > sms ? 1 : 2;
         for (int pass = 0; pass < passes && pick.nw == 0; ++pass) {
-            const size_t budget = pass == 0 ? kB1Coresident : kB1MaxSmem;
+            const size_t budget = pass == 0 ? coresident : kB1MaxSmem;
             for (int k = 0; k < nshapes && pick.nw == 0; ++k)
                 for (int staged = 1; staged >= 0 && pick.nw == 0; --staged) {
                     const B1Shape &sh = shapes[k];
