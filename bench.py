@@ -756,14 +756,17 @@ def run_dense(args, local_rank):
 # ------------------------------------------------------------------- lora
 
 def run_lora(args, local_rank):
-    """Low-rank compensation (bisco_lora_apply, rank --lora-rank) on every
-    projection of the 36-layer q/k/v/o decode step.  Times the step with and
-    without it (CUDA graphs of the same calls, CUDA events over `steps`
-    replays) and the compensation alone: a graph of its calls for every
-    projection, timed replay by replay with L2 flushed in between (the
-    adapters of the stack are smaller than L2).  Adapter bytes are
-    rank * (K + N) bf16 per projection; the roofline counts those plus x, t
-    and the read-modify-write of y."""
+    """Low-rank compensation (rank --lora-rank) on every projection of the
+    36-layer q/k/v/o decode step.  Times the step without it, with it fused
+    into the GEMV at batch 1 (bisco_gemv_multi_lora for q/k/v,
+    bisco_gemv_lora for o: one launch each, as without it), and with the
+    two-kernel bisco_lora_apply after each GEMV (CUDA graphs of the same
+    calls, CUDA events over `steps` replays); and that two-kernel
+    compensation alone: a graph of its calls for every projection, timed
+    replay by replay with L2 flushed in between (the adapters of the stack
+    are smaller than L2).  Adapter bytes are rank * (K + N) bf16 per
+    projection; the roofline counts those plus x, t and the read-modify-
+    write of y."""
     import torch
     from paper_2607_08643_gb300 import bisco
     dev = torch.device("cuda", local_rank)
@@ -783,7 +786,19 @@ def run_lora(args, local_rank):
     t = torch.empty((B, R), dtype=torch.float32, device=dev)
     stream = torch.cuda.Stream(device=dev)
 
-    def step(with_lora, with_gemv=True):
+    fused_ok = B == 1
+
+    def step(with_lora, with_gemv=True, fused=False):
+        if fused:
+            for li in range(args.layers):
+                q = [4 * li + j for j in range(3)]
+                bisco.bisco_gemv_multi_lora([layers[i][1] for i in q],
+                                            [adapters[i] + (1.0,) for i in q], x[2 * li],
+                                            ys=[ys[i] for i in q], stream=stream)
+                o = 4 * li + 3
+                bisco.bisco_gemv_lora(layers[o][1], adapters[o] + (1.0,), x[2 * li + 1], y=ys[o],
+                                      stream=stream)
+            return
         for li in range(args.layers):
             q = [4 * li + j for j in range(3)]
             if with_gemv:
@@ -799,20 +814,23 @@ def run_lora(args, local_rank):
                 bisco.bisco_lora_apply(*adapters[o], x[2 * li + 1], ys[o], 1.0, t=t, stream=stream)
 
     graphs = {}
-    for key, (wl, wg) in {"plain": (False, True), "lora": (True, True), "only": (True, False)}.items():
+    variants = {"plain": (False, True, False), "lora": (True, True, False), "only": (True, False, False)}
+    if fused_ok:
+        variants["fused"] = (True, True, True)
+    for key, (wl, wg, fu) in variants.items():
         with torch.cuda.stream(stream):
-            step(wl, wg)
+            step(wl, wg, fu)
             torch.cuda.synchronize()
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g, stream=stream):
-                step(wl, wg)
+                step(wl, wg, fu)
         graphs[key] = g
     torch.cuda.synchronize()
     if bisco.bisco_get_device_error(stream) != bisco.OK:
         raise RuntimeError("device error in the lora step")
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ms = {}
-    for key in ("plain", "lora"):
+    for key in [k for k in ("plain", "lora", "fused") if k in graphs]:
         for _ in range(max(args.warmup, 3)):
             graphs[key].replay()
         torch.cuda.synchronize()
@@ -842,7 +860,12 @@ def run_lora(args, local_rank):
     gbs = (adapter_bytes + io_bytes) / (ms_only * 1e-3) / 1e9
     return {"metric": "decode step with low-rank compensation on every projection",
             "rank": R, "batch": B, "layers": args.layers,
-            "step_ms_without": ms["plain"], "step_ms_with": ms["lora"],
+            "step_ms_without": ms["plain"],
+            "fused": ({"step_ms": ms["fused"], "overhead_pct": 100.0 * (ms["fused"] / ms["plain"] - 1.0),
+                       "tokens_per_s": B / (ms["fused"] * 1e-3),
+                       "kernels": "k_gemv_b1 with t = A x and Bm t in the same launch"}
+                      if "fused" in ms else None),
+            "step_ms_with": ms["lora"],
             "overhead_pct": 100.0 * (ms["lora"] / ms["plain"] - 1.0),
             "tokens_per_s_with": B / (ms["lora"] * 1e-3),
             "compensation_alone": {"ms_per_step": ms_only, "calls": calls,
@@ -851,7 +874,7 @@ def run_lora(args, local_rank):
                                    "gbs": gbs, "frac_of_hbm": gbs / peak,
                                    "peak_source": peak_kind,
                                    "l2": "flushed (256 MB write) before every replay"},
-            "kernels": "k_lora_down + k_lora_up per projection"}
+            "kernels": "step_ms_with: the GEMV, then k_lora_down + k_lora_up per projection"}
 
 
 # ----------------------------------------------------------------- shapes

@@ -278,6 +278,40 @@ bisco_status bisco_gemv_multi(const bisco_layer *layers, int32_t G, const uint16
                               int32_t B, float *const *y, bisco_stream_t stream);
 
 /*
+ * A layer's low-rank compensation (Sec. II-D, Sec. III-F), for the fused
+ * entry points below: A [rank][K] and Bm [N][rank] bf16 device arrays (the
+ * layouts of bisco_lora_apply), 16-byte aligned, and a finite scale.
+ * rank 0 means no compensation for that layer (A and Bm are then ignored).
+ */
+typedef struct bisco_lora {
+    const uint16_t *A;
+    const uint16_t *Bm;
+    int32_t rank;
+    float scale;
+} bisco_lora;
+
+/*
+ * bisco_gemv_multi with each layer's compensation in the same launch:
+ *     y[g][i] = sum_j What_g[i][j] * x[j]
+ *               + scale_g * sum_r Bm_g[i][r] * sum_k A_g[r][k] * x[k]
+ * the quantity bisco_gemv_multi followed by bisco_lora_apply on every
+ * layer computes, at batch 1 in one kernel: every CTA forms t = A x for its
+ * layer (fp32, summed in a fixed order, so the result does not depend on
+ * the launch) and adds Bm t to its rows when it writes them.  loras: host
+ * array of G structs.  Taken by the batch-1 row-split kernel only: batch 1,
+ * k_in == 4096, stages 1..3, int8 column protection, every rank a multiple
+ * of 8 in [0, BISCO_GEMV_LORA_MAX_RANK]; other combinations return
+ * BISCO_ERR_UNSUPPORTED (run bisco_gemv_multi and bisco_lora_apply then).
+ * Malformed arguments: BISCO_ERR_INVALID_ARG.  Layers, x and y as for
+ * bisco_gemv_multi.  bisco_gemv_lora is the G = 1 case.
+ */
+#define BISCO_GEMV_LORA_MAX_RANK 64
+bisco_status bisco_gemv_multi_lora(const bisco_layer *layers, const bisco_lora *loras, int32_t G,
+                                   const uint16_t *x_bf16, float *const *y, bisco_stream_t stream);
+bisco_status bisco_gemv_lora(const bisco_layer *L, const bisco_lora *lora, const uint16_t *x_bf16,
+                             float *y, bisco_stream_t stream);
+
+/*
  * Prefill matrix product Y[m][i] = sum_j What[i][j] * X[m][j] for any M >= 0
  * (Sec. III-G Eq. 12 with Eq. 10), the same quantity as bisco_gemv.  For
  * M > 64 and K % 128 == 0 it runs on the tcgen05 tensor cores: the decoded

@@ -20,7 +20,8 @@ EXPORTS = (
     "bisco_layer_sizes", "bisco_encode_workspace_bytes",
     "bisco_encode_workspace_bytes_axis", "bisco_encode", "bisco_encode_with_set",
     "bisco_select_coupled_workspace_bytes", "bisco_select_coupled",
-    "bisco_encode_noalloc", "bisco_gemv", "bisco_gemv_multi",
+    "bisco_encode_noalloc", "bisco_gemv", "bisco_gemv_multi", "bisco_gemv_multi_lora",
+    "bisco_gemv_lora",
     "bisco_gemm_workspace_bytes", "bisco_gemm", "bisco_decode_dense", "bisco_decode_dense_stage",
     "bisco_gemv_table",
     "bisco_decode_dense_table", "bisco_lora_apply",
@@ -35,6 +36,12 @@ class BiscoError(RuntimeError):
     def __init__(self, code: int, where: str = ""):
         self.code = code
         super().__init__("%s: bisco status %d (%s)" % (where, code, status_string(code)))
+
+
+class bisco_lora(ctypes.Structure):
+    """struct bisco_lora of include/bisco.h."""
+    _fields_ = [("A", ctypes.c_void_p), ("Bm", ctypes.c_void_p), ("rank", ctypes.c_int32),
+                ("scale", ctypes.c_float)]
 
 
 class bisco_layer(ctypes.Structure):
@@ -88,6 +95,10 @@ def load(path: str = LIB_PATH):
     lib.bisco_gemv.argtypes = [Lp, P, i32, P, P]
     lib.bisco_gemv_multi.restype = st
     lib.bisco_gemv_multi.argtypes = [Lp, i32, P, i32, ctypes.POINTER(P), P]
+    lib.bisco_gemv_multi_lora.restype = st
+    lib.bisco_gemv_multi_lora.argtypes = [Lp, ctypes.POINTER(bisco_lora), i32, P, ctypes.POINTER(P), P]
+    lib.bisco_gemv_lora.restype = st
+    lib.bisco_gemv_lora.argtypes = [Lp, ctypes.POINTER(bisco_lora), P, P, P]
     lib.bisco_gemm_workspace_bytes.restype = sz
     lib.bisco_gemm_workspace_bytes.argtypes = [Lp, i32]
     lib.bisco_gemm.restype = st
@@ -358,6 +369,53 @@ def bisco_gemv_multi(layers, x_bits, ys=None, stream=None):
     _check(load().bisco_gemv_multi(structs, G, _ptr(x_bits), B, yp, _stream(stream)),
            "bisco_gemv_multi")
     return ys
+
+
+def _lora_struct(lora):
+    """(A, Bm, scale) of bf16 device tensors, or None for no compensation."""
+    if lora is None:
+        return bisco_lora(None, None, 0, 0.0)
+    A, Bm, scale = lora
+    return bisco_lora(A.data_ptr(), Bm.data_ptr(), int(A.shape[0]), float(scale))
+
+
+def bisco_gemv_multi_lora(layers, loras, x_bits, ys=None, stream=None):
+    """[y_g] = x What_g^T + scale_g (x A_g^T) Bm_g^T at batch 1 in one launch;
+    loras[g] = (A [rank][K] bf16, Bm [N][rank] bf16, scale) or None."""
+    import torch
+    if x_bits.dtype == torch.bfloat16:
+        x_bits = x_bits.view(torch.int16)
+    if x_bits.dim() == 1:
+        x_bits = x_bits.unsqueeze(0)
+    G = len(layers)
+    assert x_bits.shape[0] == 1 and x_bits.is_contiguous() and len(loras) == G
+    for r in loras:
+        if r is not None:
+            assert r[0].is_contiguous() and r[1].is_contiguous()
+    if ys is None:
+        ys = [torch.empty((1, L.N), dtype=torch.float32, device=x_bits.device) for L in layers]
+    structs = (bisco_layer * G)(*[L.c for L in layers])
+    lstructs = (bisco_lora * G)(*[_lora_struct(r) for r in loras])
+    yp = (ctypes.c_void_p * G)(*[y.data_ptr() for y in ys])
+    _check(load().bisco_gemv_multi_lora(structs, lstructs, G, _ptr(x_bits), yp, _stream(stream)),
+           "bisco_gemv_multi_lora")
+    return ys
+
+
+def bisco_gemv_lora(L: Layer, lora, x_bits, y=None, stream=None):
+    """y = x What^T + scale (x A^T) Bm^T at batch 1 (lora = (A, Bm, scale))."""
+    import torch
+    if x_bits.dtype == torch.bfloat16:
+        x_bits = x_bits.view(torch.int16)
+    if x_bits.dim() == 1:
+        x_bits = x_bits.unsqueeze(0)
+    assert x_bits.shape[0] == 1 and x_bits.is_contiguous()
+    if y is None:
+        y = torch.empty((1, L.N), dtype=torch.float32, device=x_bits.device)
+    ls = _lora_struct(lora)
+    _check(load().bisco_gemv_lora(ctypes.byref(L.c), ctypes.byref(ls), _ptr(x_bits), y.data_ptr(),
+                                  _stream(stream)), "bisco_gemv_lora")
+    return y
 
 
 def bisco_gemm(L: Layer, X_bits, Y=None, workspace=None, stream=None):

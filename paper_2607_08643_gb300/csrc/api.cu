@@ -320,6 +320,38 @@ bisco_status bisco_gemv_multi(const bisco_layer *layers, int32_t G, const uint16
     return st;
 }
 
+bisco_status bisco_gemv_multi_lora(const bisco_layer *layers, const bisco_lora *loras, int32_t G,
+                                   const uint16_t *x_bf16, float *const *y, bisco_stream_t stream) {
+    if (!layers || !loras || !y || G < 1 || G > BISCO_GEMV_MULTI_MAX) return BISCO_ERR_INVALID_ARG;
+    if (!x_bf16 || !aligned16(x_bf16)) return BISCO_ERR_INVALID_ARG;
+    for (int g = 0; g < G; ++g) {
+        const bisco_status st = check_layer(&layers[g], true);
+        if (st != BISCO_OK) return st;
+        if (layers[g].k_in != layers[0].k_in || layers[g].stages != layers[0].stages)
+            return BISCO_ERR_INVALID_ARG;
+        if (!y[g] || !aligned16(y[g])) return BISCO_ERR_INVALID_ARG;
+        const bisco_lora &r = loras[g];
+        if (r.rank < 0 || r.rank > BISCO_GEMV_LORA_MAX_RANK || r.rank % 8 != 0) return BISCO_ERR_INVALID_ARG;
+        if (r.rank > 0 && (!r.A || !r.Bm || !aligned16(r.A) || !aligned16(r.Bm) || !std::isfinite(r.scale)))
+            return BISCO_ERR_INVALID_ARG;
+        if (needs_epilogue(layers[g])) return BISCO_ERR_UNSUPPORTED;
+    }
+    if (layers[0].k_in != 4096) return BISCO_ERR_UNSUPPORTED;
+    bisco_status st;
+    int *err = device_error_word(&st);
+    if (!err) return st;
+    bool launched = false;
+    st = launch_gemv_b1(layers, G, x_bf16, y, err, reinterpret_cast<cudaStream_t>(stream), &launched, loras);
+    if (st != BISCO_OK) return st;
+    return launched ? BISCO_OK : BISCO_ERR_UNSUPPORTED;
+}
+
+bisco_status bisco_gemv_lora(const bisco_layer *L, const bisco_lora *lora, const uint16_t *x_bf16,
+                             float *y, bisco_stream_t stream) {
+    if (!L || !lora || !y) return BISCO_ERR_INVALID_ARG;
+    return bisco_gemv_multi_lora(L, lora, 1, x_bf16, &y, stream);
+}
+
 size_t bisco_gemm_workspace_bytes(const bisco_layer *L, int32_t M) {
     if (M < 0 || check_layer(L, false) != BISCO_OK) return 0;
     return gemm_workspace_bytes(needs_epilogue(*L) ? bsq_only(*L) : *L, M);

@@ -74,6 +74,10 @@ struct B1Layer {
     const uint16_t *q8_scale;  // [p] fp16
     const int32_t *prot_idx;   // [p]
     float *y;                  // [N]
+    const uint16_t *la;        // low-rank compensation: A [rank][K] bf16
+    const uint16_t *lb;        //                        Bm [N][rank] bf16
+    int rank;                  // 0: none
+    float lscale;
     int N, p, p_pad;
     int cta0, ctas;            // the CTAs of the grid that take this layer's rows
 };
@@ -89,7 +93,8 @@ struct B1Args {
     int q8_staged;             // int8 rows in shared memory (else read at the end)
     uint32_t sleep_ns;         // suspend-time hint of the item waits
     int withhold;              // test of the bounded waits: request no copies
-    uint32_t off_ring, off_pm, off_pidx, off_sx, off_part, off_prot, off_q8, off_bar;   // tables at 0
+    int lrank;                 // the largest compensation rank of the launch (0: none)
+    uint32_t off_ring, off_pm, off_pidx, off_sx, off_part, off_prot, off_lt, off_q8, off_bar;   // table at 0
 };
 
 template <uint32_t A>
@@ -240,7 +245,7 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     extern __shared__ unsigned char smem_raw[];
     unsigned char *sm = align_smem<4096>(smem_raw);
     const uint32_t sbase = smem_u32(sm);
-    __shared__ int s_abort;
+    __shared__ int s_abort, s_lnext;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int K = a.K, C = K / 8, nspan = NSPAN ? NSPAN : a.nspan, S = a.S;
@@ -320,7 +325,10 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
 #pragma unroll
     for (int d = 0; d < D; ++d)
         if (left > 0) fill(d);
-    if (threadIdx.x == 0) s_abort = 0;
+    if (threadIdx.x == 0) {
+        s_abort = 0;
+        s_lnext = 0;
+    }
     for (int i = threadIdx.x; i < C / 4; i += kThreads) pm[i] = 0u;
     __syncthreads();
     for (int u = threadIdx.x; u < p; u += kThreads) {
@@ -339,6 +347,17 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     // x into L2 now (a prefetch moves no data into the CTA, so it is safe
     // ahead of the wait on a kernel that may still be writing x); read after
     if (threadIdx.x == 32) prefetch_l2(a.x, static_cast<uint32_t>(K) * 2u);
+    // the compensation's weights into L2 as well: this CTA's share of A
+    // (every CTA of the layer reads all of it) and Bm's rows of its rows
+    if (L.rank > 0 && threadIdx.x == 64) {
+        const uint32_t abytes = static_cast<uint32_t>(L.rank) * K * 2u;
+        const uint32_t share = (abytes / L.ctas + 15u) / 16u * 16u;
+        const uint32_t b0 = share * static_cast<uint32_t>(ci);
+        if (b0 < abytes)
+            prefetch_l2(reinterpret_cast<const unsigned char *>(L.la) + b0, min(share, abytes - b0));
+        if (nrows > 0)
+            prefetch_l2(L.lb + static_cast<size_t>(ra) * L.rank, static_cast<uint32_t>(nrows * L.rank) * 2u);
+    }
     if (p > 0 && nrows > 0) {
         if (a.q8_staged) {
             const int n16 = nrows * p_pad / 16;
@@ -498,16 +517,86 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
             if ((lane & 7) == 0 && rr < nrows) prot[rr] = r;
         }
     }
+
+    // ---- the layer's low-rank compensation (Sec. III-F), first t = A x:
+    // units of eight ranks x 256 columns, each taken by whichever warp is
+    // free first (a unit's result does not depend on the warp), its sums
+    // into lt[column slice][rank]
+    float *lt = reinterpret_cast<float *>(sm + a.off_lt);   // [K / 256][rank], then t [rank]
+    const int nsl = K / 256;
+    if (L.rank > 0) {
+        const int nunit = (L.rank / 8) * nsl;
+        for (;;) {
+            int u = 0;
+            if (lane == 0) u = atomicAdd(&s_lnext, 1);
+            u = __shfl_sync(0xFFFFFFFFu, u, 0);
+            if (u >= nunit) break;
+            const int sl = u % nsl, r0 = (u / nsl) * 8;
+            const int col = sl * 256 + lane * 8;
+            const uint4 xv = *reinterpret_cast<const uint4 *>(a.x + col);
+            uint4 av[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                av[q] = *reinterpret_cast<const uint4 *>(L.la + static_cast<size_t>(r0 + q) * K + col);
+            const float xf[8] = {bf16_bits_to_f32(static_cast<uint16_t>(xv.x)), bf16_bits_to_f32(static_cast<uint16_t>(xv.x >> 16)),
+                                 bf16_bits_to_f32(static_cast<uint16_t>(xv.y)), bf16_bits_to_f32(static_cast<uint16_t>(xv.y >> 16)),
+                                 bf16_bits_to_f32(static_cast<uint16_t>(xv.z)), bf16_bits_to_f32(static_cast<uint16_t>(xv.z >> 16)),
+                                 bf16_bits_to_f32(static_cast<uint16_t>(xv.w)), bf16_bits_to_f32(static_cast<uint16_t>(xv.w >> 16))};
+            float d[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const uint32_t w[4] = {av[q].x, av[q].y, av[q].z, av[q].w};
+                float acc = 0.f;
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    acc = fmaf(bf16_bits_to_f32(static_cast<uint16_t>(w[e])), xf[2 * e], acc);
+                    acc = fmaf(bf16_bits_to_f32(static_cast<uint16_t>(w[e] >> 16)), xf[2 * e + 1], acc);
+                }
+                d[q] = acc;
+            }
+            const float s0 = warp_sum4(d[0], d[1], d[2], d[3], lane);   // rank r0 + (lane >> 3)
+            const float s1 = warp_sum4(d[4], d[5], d[6], d[7], lane);   // rank r0 + 4 + (lane >> 3)
+            if ((lane & 7) == 0) {
+                lt[sl * L.rank + r0 + (lane >> 3)] = s0;
+                lt[sl * L.rank + r0 + 4 + (lane >> 3)] = s1;
+            }
+        }
+    }
     __syncthreads();
     if (*reinterpret_cast<volatile int *>(&s_abort)) return;
+    // t[r]: the slices' sums in slice order
+    float *lt_t = lt + nsl * a.lrank;
+    if (L.rank > 0) {
+        if (static_cast<int>(threadIdx.x) < L.rank) {
+            float t = 0.f;
+            for (int sl = 0; sl < nsl; ++sl) t += lt[sl * L.rank + threadIdx.x];
+            lt_t[threadIdx.x] = t;
+        }
+        __syncthreads();
+    }
 
     // ---- outputs: a thread per row; the row's item sums in order, then the
-    // protected term
+    // protected term, then scale * (Bm t) of the compensation
     for (int rr = threadIdx.x; rr < nrows; rr += kThreads) {
         float v = 0.f;
         for (int sp = 0; sp < nspan; ++sp)
             for (int s = 0; s < S; ++s) v += part[sp * per_span + s * nrows + rr];
-        y[ra + rr] = v * kB1InvSqrt8 + (p > 0 ? prot[rr] : 0.f);
+        v = v * kB1InvSqrt8 + (p > 0 ? prot[rr] : 0.f);
+        if (L.rank > 0) {
+            const uint16_t *bm = L.lb + static_cast<size_t>(ra + rr) * L.rank;
+            float bt = 0.f;
+            for (int r0 = 0; r0 < L.rank; r0 += 8) {
+                const uint4 bv = *reinterpret_cast<const uint4 *>(bm + r0);
+                const uint32_t w[4] = {bv.x, bv.y, bv.z, bv.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    bt = fmaf(bf16_bits_to_f32(static_cast<uint16_t>(w[e])), lt_t[r0 + 2 * e], bt);
+                    bt = fmaf(bf16_bits_to_f32(static_cast<uint16_t>(w[e] >> 16)), lt_t[r0 + 2 * e + 1], bt);
+                }
+            }
+            v = fmaf(L.lscale, bt, v);
+        }
+        y[ra + rr] = v;
     }
 }
 
@@ -589,6 +678,8 @@ size_t b1_layout(int C, int nw, int depth, int p_max, int rows_max, int items_ma
     off += static_cast<size_t>(items_max) * 4;
     a->off_prot = static_cast<uint32_t>(off);
     off += static_cast<size_t>(rows_max) * 4;
+    a->off_lt = static_cast<uint32_t>(off);                 // compensation: slice sums, t
+    off += a->lrank > 0 ? static_cast<size_t>(C / 32 + 1) * a->lrank * 4 : 0;
     off = align_up_b1(off, 16);
     a->off_q8 = static_cast<uint32_t>(off);
     off += q8_bytes;
@@ -611,7 +702,7 @@ constexpr B1Shape kB1Shapes[] = {{16, 3}, {16, 2}};
 }  // namespace
 
 bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, float *const *y,
-                            int *err, cudaStream_t stream, bool *launched) {
+                            int *err, cudaStream_t stream, bool *launched, const bisco_lora *loras) {
     *launched = false;
     if (const char *e = getenv("BISCO_GEMV_B1"))
         if (e[0] == '0') return BISCO_OK;
@@ -642,6 +733,15 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
         b.p = L.n_protected;
         b.p_pad = (L.n_protected + 15) / 16 * 16;
         p_max = p_max > b.p ? p_max : b.p;
+        if (loras != nullptr && loras[g].rank > 0) {
+            // the compensation's slices are 256 columns of one span
+            if (a.nspan != 1) return BISCO_OK;
+            b.la = loras[g].A;
+            b.lb = loras[g].Bm;
+            b.rank = loras[g].rank;
+            b.lscale = loras[g].scale;
+            a.lrank = a.lrank > b.rank ? a.lrank : b.rank;
+        }
     }
     const int sms = num_sms();
     if (G > sms) return BISCO_OK;

@@ -174,6 +174,39 @@ def test_lora_validation(lib):
             assert f(p[0], p[1], 16, 64, 64, 1.0, p[2], 1, p[3], p[4], None) == E
 
 
+def test_gemv_lora_validation(lib):
+    """The fused compensation entry points check every argument before any
+    device call; shapes the batch-1 kernel does not take are UNSUPPORTED."""
+    L = _fake_layer()                                                   # k_in 256
+    L4 = _fake_layer(k_in=4096)
+    x = ctypes.c_void_p(0x60000)
+    ys = (ctypes.c_void_p * 2)(0x70000, 0x80000)
+    ok = bisco.bisco_lora(0x90000, 0xA0000, 16, 1.0)
+    E = bisco.ERR_INVALID_ARG
+    f = lib.bisco_gemv_multi_lora
+    arr = (bisco.bisco_layer * 2)(L, L)
+    lor = (bisco.bisco_lora * 2)(ok, ok)
+    assert f(arr, lor, 2, x, ys, None) == bisco.ERR_UNSUPPORTED       # K != 4096
+    for bad in (bisco.bisco_lora(0x90000, 0xA0000, r, 1.0) for r in (4, 12, 72, -8)):
+        assert f(arr, (bisco.bisco_lora * 2)(ok, bad), 2, x, ys, None) == E
+    for bad in (bisco.bisco_lora(0x90008, 0xA0000, 16, 1.0), bisco.bisco_lora(0x90000, None, 16, 1.0),
+                bisco.bisco_lora(0x90000, 0xA0000, 16, float("nan"))):
+        assert f(arr, (bisco.bisco_lora * 2)(bad, ok), 2, x, ys, None) == E
+    # rank 0: no compensation, A and Bm not looked at
+    none = bisco.bisco_lora(None, None, 0, float("nan"))
+    assert f(arr, (bisco.bisco_lora * 2)(none, none), 2, x, ys, None) == bisco.ERR_UNSUPPORTED
+    assert f(arr, None, 2, x, ys, None) == E
+    assert f(arr, lor, 0, x, ys, None) == E
+    assert f(arr, lor, 5, x, ys, None) == E
+    assert f(arr, lor, 2, ctypes.c_void_p(0x60002), ys, None) == E      # x misaligned
+    mixed = (bisco.bisco_layer * 2)(L4, L)                              # K differs
+    assert f(mixed, lor, 2, x, ys, None) == E
+    g = lib.bisco_gemv_lora
+    assert g(ctypes.byref(L), ctypes.byref(ok), x, ctypes.c_void_p(0x70000), None) == bisco.ERR_UNSUPPORTED
+    assert g(ctypes.byref(L), None, x, ctypes.c_void_p(0x70000), None) == E
+    assert g(ctypes.byref(L), ctypes.byref(ok), x, ctypes.c_void_p(0x70004), None) == E
+
+
 def test_binding_argument_counts_match_header(lib):
     """Every prototype in bisco.h has as many parameters as the ctypes
     binding declares for it (a drifted binding would pass garbage)."""
@@ -341,21 +374,24 @@ def test_decoder_table_validation(lib):
     assert d(ctypes.byref(_fake_layer(stages=4)), tab, y, bisco.DENSE_F32, None) == E
 
 
-def test_struct_layout_matches_the_header(tmp_path):
-    """The ctypes mirror of bisco_layer has the C struct's size and field
-    offsets (an array of them crosses the ABI in bisco_gemv_multi)."""
+@pytest.mark.parametrize("name", ["bisco_layer", "bisco_lora"])
+def test_struct_layout_matches_the_header(tmp_path, name):
+    """The ctypes mirrors of bisco_layer and bisco_lora have the C structs'
+    sizes and field offsets (arrays of them cross the ABI in
+    bisco_gemv_multi and bisco_gemv_multi_lora)."""
     import subprocess
-    fields = [f for f, _ in bisco.bisco_layer._fields_]
+    cls = getattr(bisco, name)
+    fields = [f for f, _ in cls._fields_]
     src = tmp_path / "layout.c"
     src.write_text('#include <stdio.h>\n#include <stddef.h>\n#include "bisco.h"\nint main(void) {\n'
-                   '  printf("%zu\\n", sizeof(bisco_layer));\n' +
-                   "".join('  printf("%%zu\\n", offsetof(bisco_layer, %s));\n' % f for f in fields) +
+                   '  printf("%%zu\\n", sizeof(%s));\n' % name +
+                   "".join('  printf("%%zu\\n", offsetof(%s, %s));\n' % (name, f) for f in fields) +
                    "  return 0;\n}\n")
     exe = tmp_path / "layout"
     subprocess.check_call(["gcc", "-std=c11", "-I", os.path.join(ROOT, "include"), "-o", str(exe), str(src)])
     out = [int(v) for v in subprocess.check_output([str(exe)]).split()]
-    assert out[0] == ctypes.sizeof(bisco.bisco_layer)
-    assert out[1:] == [getattr(bisco.bisco_layer, f).offset for f in fields]
+    assert out[0] == ctypes.sizeof(cls)
+    assert out[1:] == [getattr(cls, f).offset for f in fields]
 
 
 @pytest.mark.parametrize("axis,fmt", [(0, bisco.PROT_INT8), (0, bisco.PROT_E4M3), (0, bisco.PROT_E5M2),

@@ -1,5 +1,6 @@
 """bisco_lora_apply (the low-rank compensation of Sec. III-F) against the
-fp64 oracle's lora_apply.
+fp64 oracle's lora_apply, and the compensation fused into the batch-1 GEMV
+(bisco_gemv_lora, bisco_gemv_multi_lora) at the end of the file.
 
 The kernels sum in fp32, and every product they form (bf16 x bf16 in the
 down projection, bf16 x fp32 inside an fma in the up projection) is exact.
@@ -15,7 +16,7 @@ import pytest
 import oracle
 from paper_2607_08643_gb300 import synth
 
-from _helpers import TOL, max_rel_rows, to_dev
+from _helpers import TOL, assert_parity, gemv_tight, max_rel_rows, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -120,3 +121,72 @@ def test_lora_split_down_matches_oracle(env, N, K, rank, B, scale, monkeypatch):
     got = _run(env, A, Bm, X, Y0, scale)
     assert np.all(np.abs(got - ref) <= _bound(A, Bm, X, Y0, scale))
     assert np.array_equal(got, _run(env, A, Bm, X, Y0, scale))
+
+
+# ------------------------------------------ compensation fused into the GEMV
+# bisco_gemv_lora / bisco_gemv_multi_lora: the batch-1 row-split kernel adds
+# scale * Bm (A x) to each row it writes (t = A x formed in every CTA, in
+# units of 8 ranks x 256 columns summed in a fixed order).  Against the
+# oracle's layer output plus the oracle's compensation at the table decode's
+# bound; against bisco_gemv + bisco_lora_apply (the same decode, the
+# compensation's sums in another order) far inside it; the same bits on a
+# second call.
+
+def _fused(env, Lrefs, loras, X):
+    import torch
+    bisco, dev = env
+    Ls = [bisco.Layer.from_numpy(L, dev) for L in Lrefs]
+    dl = [None if r is None else (to_dev(r[0], dev), to_dev(r[1], dev), r[2]) for r in loras]
+    xd = to_dev(X, dev)
+    if len(Ls) == 1:
+        ys = [bisco.bisco_gemv_lora(Ls[0], dl[0], xd)]
+    else:
+        ys = bisco.bisco_gemv_multi_lora(Ls, dl, xd)
+    torch.cuda.synchronize()
+    assert bisco.bisco_get_device_error() == 0
+    return [y.cpu().numpy() for y in ys], Ls, dl, xd
+
+
+@pytest.mark.parametrize("shapes", [
+    [(4096, 41, 16, 0.5)],                                   # o_proj
+    [(4096, 41, 16, 1.0), (1024, 41, 8, -2.0), (1024, 41, 0, 0.0)],   # q/k/v, v without one
+    [(150, 5, 64, 0.25)],                                    # one row per CTA, largest rank
+    [(12288, 41, 16, 1.0), (12288, 41, 32, 0.5)],            # gate/up: two CTAs per SM
+])
+def test_gemv_lora_fused_matches_oracle(env, shapes):
+    import torch
+    bisco, dev = env
+    K, S = 4096, 2
+    Lrefs, loras = [], []
+    for i, (N, p, rank, scale) in enumerate(shapes):
+        Lrefs.append(oracle.encode(synth.layer_weights(N, K, seed=600 + i), S=S, p=p))
+        loras.append(None if rank == 0 else synth.lora_adapter(N, K, rank, seed=610 + i) + (scale,))
+    X = synth.activations(1, K, seed=620)
+    ys, Ls, dl, xd = _fused(env, Lrefs, loras, X)
+    for y, L, r, Ld, rd in zip(ys, Lrefs, loras, Ls, dl):
+        y0 = oracle.gemv(L, X)
+        ref = y0 if r is None else oracle.lora_apply(r[0], r[1], X, y0, r[2])
+        assert_parity(y, ref, gemv_tight(1))
+        # the unfused chain: the same decode, then the two-kernel compensation
+        yc = bisco.bisco_gemv(Ld, xd)
+        if rd is not None:
+            bisco.bisco_lora_apply(rd[0], rd[1], xd, yc, rd[2])
+        torch.cuda.synchronize()
+        assert max_rel_rows(y, yc.cpu().numpy()) <= 2e-6
+    again, _, _, _ = _fused(env, Lrefs, loras, X)
+    for y, y2 in zip(ys, again):
+        assert np.array_equal(y, y2)
+
+
+def test_gemv_lora_unsupported_shapes(env):
+    """K other than 4096 is not taken by the fused kernel: UNSUPPORTED, and
+    the two-kernel chain is the way to run it."""
+    import torch
+    bisco, dev = env
+    Lref = oracle.encode(synth.layer_weights(256, 8192, seed=630), S=2, p=11)
+    A, Bm = synth.lora_adapter(256, 8192, 16, seed=631)
+    L = bisco.Layer.from_numpy(Lref, dev)
+    x = to_dev(synth.activations(1, 8192, seed=632), dev)
+    with pytest.raises(bisco.BiscoError) as e:
+        bisco.bisco_gemv_lora(L, (to_dev(A, dev), to_dev(Bm, dev), 1.0), x)
+    assert e.value.code == bisco.ERR_UNSUPPORTED
