@@ -120,7 +120,7 @@ typedef struct {
 #define BISCO_PROT_BF16 3
 
 /* ABI version of this header (major * 100 + minor). */
-#define BISCO_ABI_VERSION 105
+#define BISCO_ABI_VERSION 106
 int32_t bisco_abi_version(void);
 
 /* Static string for a status code (never NULL). */
