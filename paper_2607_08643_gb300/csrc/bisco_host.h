@@ -32,9 +32,10 @@ bisco_status launch_gemv(const bisco_layer &L, const uint16_t *x, int B, float *
                          cudaStream_t stream);
 bisco_status launch_gemv_multi(const bisco_layer *Ls, int G, const uint16_t *x, int B,
                                float *const *y, int *err, cudaStream_t stream);
-// Batch-1 decode for G <= 4 layers sharing x with K % 4096 == 0 (gemv_b1.cu),
-// with each layer's low-rank compensation when loras is not null (K == 4096
-// only); *launched stays false when the layers do not fit its plan.
+// Batch-1 decode for G <= 4 layers sharing x with K % 4096 == 0 and column
+// protection in any payload format (gemv_b1.cu), with each layer's low-rank
+// compensation when loras is not null (K == 4096 only); *launched stays
+// false when the layers do not fit its plan.
 bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, float *const *y,
                             int *err, cudaStream_t stream, bool *launched,
                             const bisco_lora *loras = nullptr);

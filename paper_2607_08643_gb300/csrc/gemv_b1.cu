@@ -1,26 +1,28 @@
 // gemv_b1.cu -- batch-1 decode-time y = What x straight from the coded
 // layer (Sec. III-G Eq. 12 with Eq. 10's protected columns) for G <= 4
 // layers that share x and have K a multiple of 4096 (every Qwen3-8B
-// projection).
+// projection); optionally with each layer's low-rank compensation
+// (Sec. III-F) in the same launch.
 //
-// Work split.  The CTAs of a one-per-SM grid are shared out among the G
-// layers so that the longest row run per CTA is as short as it can be
-// (q/k/v of Qwen3-8B: 101/25/26 CTAs of 40-41 rows); each CTA takes a
-// contiguous run of one layer's rows.  A row's work is S * K/4096 items, one
-// per (stage, 4096-column span): 512 sign bytes and 512 fp16 norms, 1536
-// bytes.  A CTA orders its items stage by stage, row by row, span by span --
-// the order of the [S][N][K/8] buffers -- and each of its 16 warps takes one
-// contiguous run of that list.
+// Work split.  The CTAs of the grid are shared out among the G layers so
+// that the longest row run per CTA is as short as it can be (q/k/v of
+// Qwen3-8B: 102/25/25 CTAs of 40-41 rows); each CTA takes a contiguous run
+// of one layer's rows.  A launch with at least kB1TwoPerSm items per SM runs
+// two of its own CTAs per SM, others one.  A row's work is S * K/4096 items,
+// one per (stage, 4096-column span): 512 sign bytes and 512 fp16 norms,
+// 1536 bytes.  A CTA orders its items span by span, then stage by stage and
+// row by row (within a span and stage, consecutive rows are consecutive in
+// memory), and each of its 16 warps takes the same contiguous run of every
+// span.
 //
-// Data path.  Every warp owns a ring of `depth` item slots in shared memory.
-// Lane 0 fills a slot with two 1-D bulk copies (cp.async.bulk: 512 B of
-// signs, 1 KB of norms) that complete on the slot's mbarrier, and refills it
-// with the item `depth` further on as soon as the warp has read it.  The
-// first `depth` items of every warp are requested before the wait on the
-// previous kernel, so a CTA has up to 16 * depth * 1.5 KB of its layer in
-// flight while that kernel finishes.  On GB300 this layout streams at the
-// HBM copy rate with 16 decoding warps; 8 warps reach about 80 % of it and a
-// register-staged load pipeline about half.
+// Data path.  Every warp owns a ring of `depth` one-item slots in shared
+// memory.  Lane 0 fills a slot with two 1-D bulk copies (cp.async.bulk:
+// 512 B of signs, 1 KB of norms) that complete on the slot's mbarrier, and
+// refills it with the item `depth` further on as soon as the warp has read
+// it into registers, before decoding it.  The first `depth` items of every
+// warp are requested before the wait on the previous kernel, and a CTA
+// takes at most the shared memory at which two CTAs share an SM, so the
+// next call's CTAs request theirs while this one finishes.
 //
 // Decode (Eq. 12 per chunk-stage): for a sign byte b of chunk c the signed
 // sum of the chunk's 8 activations is T_lo(c, b & 15) + T_hi(c, b >> 4),
@@ -29,27 +31,34 @@
 // held as one fp16 pair (T_lo, T_hi) per (c, v), and meets the chunk's fp16
 // norm in an fp16 x fp16 -> fp32 FMA (exact product).  The layer's protected
 // columns are zero in its tables, which is Eq. 10's overwrite of their BSQ
-// value; the 1/sqrt(8) of Eq. 3 is applied once per output.
+// value; the 1/sqrt(8) of Eq. 3 is applied once per output.  A CTA holds
+// the table of one span at a time (32 KB) and rebuilds it between spans.
 //
 // Table placement.  Lane l of an item handles chunks 8l+j (j = 0..7) of each
 // 256-chunk half h of its span; chunk c = 512*span + 256*h + 8l + j sits at
-// position P = 512*span + 256*h + 32*j + l, and entry (P, v) at byte
+// position P = 256*h + 32*j + l of the span's table, and entry (P, v) at
+// byte
 //   (P >> 6) * 4096 + v * 256 + (P & 63) * 4,
 // so a lane's lookups always hit bank l.  With the table 4 KB aligned, the
 // lane's base address has bits 8..11 clear and the lookup address is one
 // shift and one LOP3 ((w >> s) & 0xF00 | base) plus a compile-time offset.
 //
-// Outputs.  Each item's lane sums are added across the warp (fixed shuffle
-// order) into one float per item; after a CTA barrier a warp per row adds
-// its items in item order, scales by 1/sqrt(8) and adds the protected term
-// sum_u q8[r][u] * (scale_u * x[idx_u]) (int8 rows staged in shared memory
-// before the wait).  No atomics: the result depends only on the sizes.
+// Outputs.  The lane sums of a ring pass's items are added across the warp
+// (fixed shuffle order) into one float per item.  A warp that has decoded
+// its items computes the protected term sum_u value(q[r][u]) * (scale_u *
+// x[idx_u]) of its share of the rows (int8, FP8 E4M3 / E5M2 or bf16
+// payloads; staged in shared memory before the wait where they fit) while
+// the others may still decode; after one CTA barrier a thread per row adds
+// the row's items in item order, scales by 1/sqrt(8) and adds the protected
+// term (and the compensation).  No atomics: the result depends only on the
+// sizes.
 #include <cuda_runtime.h>
 #include <stdint.h>
 #include <stdlib.h>
 
 #include "bisco_dev.cuh"
 #include "bisco_host.h"
+#include "fp8.cuh"
 
 namespace bisco {
 namespace {
@@ -70,7 +79,7 @@ constexpr int kB1TwoPerSm = 256;
 struct B1Layer {
     const uint8_t *codes;      // [S][N][K/8]
     const uint16_t *norms;     // [S][N][K/8] fp16
-    const int8_t *q8;          // [N][p_pad]
+    const int8_t *q8;          // [N][p_pad] elements of the protected format
     const uint16_t *q8_scale;  // [p] fp16
     const int32_t *prot_idx;   // [p]
     float *y;                  // [N]
@@ -79,6 +88,8 @@ struct B1Layer {
     int rank;                  // 0: none
     float lscale;
     int N, p, p_pad;
+    int fmt;                   // BISCO_PROT_*: int8, FP8 E4M3 / E5M2 or bf16 payload
+    int prow;                  // payload bytes per row: p_pad elements of 1 or 2 bytes
     int cta0, ctas;            // the CTAs of the grid that take this layer's rows
 };
 
@@ -238,7 +249,9 @@ __device__ __forceinline__ uint4 b1_table_x(const uint16_t *x, int sp, int J, in
 // is an immediate offset; with several, a CTA holds the table of one span at
 // a time and walks its items span by span, rebuilding the table between
 // spans (x of the next span is loaded while the current one is decoded).
-template <int NW, int D, int NSPAN>
+// FMT: the protected payloads may be FP8 or bf16 (their conversions compiled
+// in); without it every payload is int8.
+template <int NW, int D, int NSPAN, bool FMT>
 __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ B1Args a) {
     static_assert(D <= 4, "one folded reduction covers a ring pass");
     constexpr int kThreads = NW * 32;
@@ -255,7 +268,7 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     for (int i = 1; i < kB1MaxG; ++i)
         if (i < a.G && static_cast<int>(blockIdx.x) >= a.L[i].cta0) g = i;
     const B1Layer &L = a.L[g];
-    const int N = L.N, p = L.p, p_pad = L.p_pad;
+    const int N = L.N, p = L.p, prow = L.prow, fmt = L.fmt;
     const int ci = static_cast<int>(blockIdx.x) - L.cta0;
     const int ra = static_cast<int>(static_cast<int64_t>(N) * ci / L.ctas);
     const int rb = static_cast<int>(static_cast<int64_t>(N) * (ci + 1) / L.ctas);
@@ -360,12 +373,12 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     }
     if (p > 0 && nrows > 0) {
         if (a.q8_staged) {
-            const int n16 = nrows * p_pad / 16;
-            const uint4 *src = reinterpret_cast<const uint4 *>(q8 + static_cast<int64_t>(ra) * p_pad);
+            const int n16 = nrows * prow / 16;
+            const uint4 *src = reinterpret_cast<const uint4 *>(q8 + static_cast<int64_t>(ra) * prow);
             for (int i = threadIdx.x; i < n16; i += kThreads) reinterpret_cast<uint4 *>(q8s)[i] = src[i];
         } else if (threadIdx.x == 0) {
             // read at the end from global memory: into L2 now
-            prefetch_l2(q8 + static_cast<int64_t>(ra) * p_pad, static_cast<uint32_t>(nrows * p_pad));
+            prefetch_l2(q8 + static_cast<int64_t>(ra) * prow, static_cast<uint32_t>(nrows * prow));
         }
     }
     __syncthreads();
@@ -486,22 +499,24 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
             mbar_wait(wbar + static_cast<uint32_t>(j % D) * 8u, static_cast<uint32_t>(j / D) & 1u);
 
     // ---- the protected term of rows warp, warp + NW, ... (Eq. 10), while
-    // other warps may still decode: four rows at a time, all their int8
+    // other warps may still decode: four rows at a time, all their payload
     // loads issued before the first product, then added over the warp
-    // together
-    if (p > 0) {
+    // together (load: a payload element's bits; value: its value, exact in
+    // fp32 -- Eq. 10's int8, or the FP8 / bf16 payload of the protected-
+    // format variants; one instance per format)
+    auto prot_term = [&](auto load, auto value) {
         for (int rr0 = warp; rr0 < nrows; rr0 += 4 * NW) {
             float pr[4] = {0.f, 0.f, 0.f, 0.f};
             for (int u0 = 0; u0 < p; u0 += 64) {
-                int qv[4][2];
+                uint32_t qv[4][2];
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
                     const int rr = rr0 + k * NW;
-                    const int8_t *q8r = a.q8_staged ? q8s + rr * p_pad : q8 + static_cast<int64_t>(ra + rr) * p_pad;
+                    const int8_t *q8r = a.q8_staged ? q8s + rr * prow : q8 + static_cast<int64_t>(ra + rr) * prow;
 #pragma unroll
                     for (int h = 0; h < 2; ++h) {
                         const int u = u0 + 32 * h + lane;
-                        qv[k][h] = rr < nrows && u < p ? q8r[u] : 0;
+                        qv[k][h] = rr < nrows && u < p ? load(q8r, u) : 0u;
                     }
                 }
 #pragma unroll
@@ -509,13 +524,23 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
 #pragma unroll
                     for (int h = 0; h < 2; ++h) {
                         const int u = u0 + 32 * h + lane;
-                        if (u < p) pr[k] = fmaf(static_cast<float>(qv[k][h]), sx[u], pr[k]);
+                        if (u < p) pr[k] = fmaf(value(qv[k][h]), sx[u], pr[k]);
                     }
             }
             const float r = warp_sum4(pr[0], pr[1], pr[2], pr[3], lane);   // row rr0 + (lane >> 3) * NW
             const int rr = rr0 + (lane >> 3) * NW;
             if ((lane & 7) == 0 && rr < nrows) prot[rr] = r;
         }
+    };
+    auto load_byte = [](const int8_t *r, int u) { return static_cast<uint32_t>(static_cast<uint8_t>(r[u])); };
+    if (p > 0) {
+        if (!FMT || fmt == BISCO_PROT_INT8)
+            prot_term(load_byte, [](uint32_t b) { return static_cast<float>(static_cast<int8_t>(b)); });
+        else if (fmt == BISCO_PROT_BF16)
+            prot_term([](const int8_t *r, int u) { return static_cast<uint32_t>(reinterpret_cast<const uint16_t *>(r)[u]); },
+                      [](uint32_t b) { return __uint_as_float(b << 16); });
+        else
+            prot_term(load_byte, [fmt](uint32_t b) { return fp8_to_f32(b, fmt); });
     }
 
     // ---- the layer's low-rank compensation (Sec. III-F), first t = A x:
@@ -602,9 +627,9 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
 
 size_t align_up_b1(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
-template <int NW, int D, int NSPAN>
+template <int NW, int D, int NSPAN, bool FMT>
 bisco_status launch_b1_t(const B1Args &a, int grid, size_t smem, cudaStream_t stream) {
-    auto kern = k_gemv_b1<NW, D, NSPAN>;
+    auto kern = k_gemv_b1<NW, D, NSPAN, FMT>;
     static size_t configured[64] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return BISCO_ERR_CUDA;
@@ -636,7 +661,7 @@ size_t b1_coresident_budget() {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
     if (budget[dev] != 0) return budget[dev];
-    auto kern = k_gemv_b1<16, 3, 1>;
+    auto kern = k_gemv_b1<16, 3, 1, false>;
     constexpr size_t kHi = 160 * 1024;   // more than two CTAs of an SM can hold
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kHi)) !=
         cudaSuccess) {
@@ -718,8 +743,7 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
     int p_max = 0;
     for (int g = 0; g < G; ++g) {
         const bisco_layer &L = Ls[g];
-        if (L.k_in != K || L.stages != S || L.protect_axis != 0 || L.protect_format != BISCO_PROT_INT8)
-            return BISCO_OK;
+        if (L.k_in != K || L.stages != S || L.protect_axis != 0) return BISCO_OK;
         // the kernel's byte offsets into the sign planes are 32-bit
         if (static_cast<uint64_t>(S) * L.n_out * (K / 8) >= (1ull << 32)) return BISCO_OK;
         B1Layer &b = a.L[g];
@@ -732,6 +756,8 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
         b.N = L.n_out;
         b.p = L.n_protected;
         b.p_pad = (L.n_protected + 15) / 16 * 16;
+        b.fmt = L.protect_format;
+        b.prow = b.p_pad * (L.protect_format == BISCO_PROT_BF16 ? 2 : 1);
         p_max = p_max > b.p ? p_max : b.p;
         if (loras != nullptr && loras[g].rank > 0) {
             // the compensation's slices are 256 columns of one span
@@ -779,7 +805,7 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
             a.L[g].ctas = ctas[g];
             c0 += ctas[g];
             rows_max = rows_max > run(g) ? rows_max : run(g);
-            const size_t q8b = static_cast<size_t>(run(g)) * a.L[g].p_pad;
+            const size_t q8b = static_cast<size_t>(run(g)) * a.L[g].prow;
             q8_max = q8_max > q8b ? q8_max : q8b;
         }
         const int items_max = rows_max * S * a.nspan;
@@ -813,11 +839,23 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
     // BISCO_ERR_TIMEOUT and returns with no copy in flight
     a.withhold = getenv("BISCO_TEST_WITHHOLD_COPIES") != nullptr;
     *launched = true;
-    if (one) {
-        if (pick.depth == 3) return launch_b1_t<16, 3, 1>(a, total, smem, stream);
-        return launch_b1_t<16, 2, 1>(a, total, smem, stream);
+    // int8 payloads only (the common case) or any format (FMT: the other
+    // formats' conversions compiled in)
+    bool fmt = false;
+    for (int g = 0; g < G; ++g) fmt |= a.L[g].p > 0 && a.L[g].fmt != BISCO_PROT_INT8;
+    if (fmt) {
+        if (one) {
+            if (pick.depth == 3) return launch_b1_t<16, 3, 1, true>(a, total, smem, stream);
+            return launch_b1_t<16, 2, 1, true>(a, total, smem, stream);
+        }
+        if (pick.depth == 3) return launch_b1_t<16, 3, 0, true>(a, total, smem, stream);
+        return launch_b1_t<16, 2, 0, true>(a, total, smem, stream);
     }
-    if (pick.depth == 3) return launch_b1_t<16, 3, 0>(a, total, smem, stream);
-    return launch_b1_t<16, 2, 0>(a, total, smem, stream);
+    if (one) {
+        if (pick.depth == 3) return launch_b1_t<16, 3, 1, false>(a, total, smem, stream);
+        return launch_b1_t<16, 2, 1, false>(a, total, smem, stream);
+    }
+    if (pick.depth == 3) return launch_b1_t<16, 3, 0, false>(a, total, smem, stream);
+    return launch_b1_t<16, 2, 0, false>(a, total, smem, stream);
 }
 }  // namespace bisco

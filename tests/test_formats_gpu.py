@@ -77,6 +77,45 @@ def test_gemv_formats_match_oracle(env, fmt, N, K, B):
 
 
 @pytest.mark.parametrize("fmt", FORMATS)
+@pytest.mark.parametrize("N,K", [(1000, 4096), (300, 8192)])
+def test_gemv_batch1_kernel_formats_match_oracle(env, fmt, N, K):
+    """Batch 1 with K a multiple of 4096: the row-split kernel takes the
+    payload format itself (value(q) * scale * x in its protected term, one
+    launch), against the oracle at the table decode's bound; the same bits
+    on a second call."""
+    import torch
+    bisco, dev = env
+    p = synth.protected_count(K, 2)
+    ref = oracle_layer(synth.layer_weights(N, K, seed=N + 3), 2, p, fmt)
+    L = bisco.Layer.from_numpy(ref, dev)
+    x = synth.activations(1, K, seed=7)
+    y = bisco.bisco_gemv(L, to_dev(x, dev))
+    y2 = bisco.bisco_gemv(L, to_dev(x, dev))
+    torch.cuda.synchronize()
+    assert bisco.bisco_get_device_error() == 0
+    assert_parity(y.cpu().numpy(), oracle.matmul(oracle_dense(ref), x), gemv_tight(1))
+    assert torch.equal(y, y2)
+
+
+def test_gemv_multi_batch1_mixed_formats(env):
+    """q/k/v-like group at batch 1 with INT8, E4M3 and bf16 payloads in one
+    launch of the row-split kernel."""
+    import torch
+    bisco, dev = env
+    K = 4096
+    refs = [oracle_layer(synth.layer_weights(N, K, seed=70 + i), 2, 41, fmt)
+            for i, (N, fmt) in enumerate([(1500, oracle.FMT_INT8), (512, oracle.FMT_E4M3),
+                                           (700, oracle.FMT_BF16)])]
+    Ls = [bisco.Layer.from_numpy(r, dev) for r in refs]
+    x = synth.activations(1, K, seed=71)
+    ys = bisco.bisco_gemv_multi(Ls, to_dev(x, dev))
+    torch.cuda.synchronize()
+    assert bisco.bisco_get_device_error() == 0
+    for y, r in zip(ys, refs):
+        assert_parity(y.cpu().numpy(), oracle.matmul(oracle_dense(r), x), gemv_tight(1))
+
+
+@pytest.mark.parametrize("fmt", FORMATS)
 def test_gemm_and_multi_formats_match_oracle(env, fmt):
     import torch
     bisco, dev = env
