@@ -441,6 +441,12 @@ bisco_status bisco_gemv_table(const bisco_layer *L, const uint16_t *tables, cons
     int *err = device_error_word(&st);
     if (!err) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    // batch 1, K a multiple of 4096: the row-split kernel in table mode
+    if (B == 1 && L->protect_axis == 0 && !getenv("BISCO_GEMV_MODE")) {
+        bool launched = false;
+        st = launch_gemv_b1(L, 1, x_bf16, &y, err, s, &launched, nullptr, tables);
+        if (launched || st != BISCO_OK) return st;
+    }
     if (L->protect_axis == 1) {
         st = launch_gemv_table(bsq_only(*L), tables, x_bf16, B, y, err, s);
         if (st != BISCO_OK) return st;

@@ -36,9 +36,12 @@ bisco_status launch_gemv_multi(const bisco_layer *Ls, int G, const uint16_t *x, 
 // protection in any payload format (gemv_b1.cu), with each layer's low-rank
 // compensation when loras is not null (K == 4096 only); *launched stays
 // false when the layers do not fit its plan.
+// With tables (the decoder tables of bisco_gemv_table, [S][256][8] fp16) it
+// runs the learned decoder step instead of the sign decode (one layer, int8
+// payloads).
 bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, float *const *y,
                             int *err, cudaStream_t stream, bool *launched,
-                            const bisco_lora *loras = nullptr);
+                            const bisco_lora *loras = nullptr, const uint16_t *tables = nullptr);
 // Output-row protection and the coupled MLP set (encode.cu, rows.cu).
 size_t encode_workspace_bytes_axis(int N, int K, int axis);
 size_t select_coupled_workspace_bytes(int F);

@@ -96,6 +96,7 @@ struct B1Layer {
 struct B1Args {
     B1Layer L[kB1MaxG];
     const uint16_t *x;
+    const uint16_t *tab;       // decoder tables [S][256][8] fp16 (table mode), else null
     int *err;
     int K, G;
     int nspan;                 // K / 4096
@@ -244,14 +245,80 @@ __device__ __forceinline__ uint4 b1_table_x(const uint16_t *x, int sp, int J, in
     return *reinterpret_cast<const uint4 *>(x + 8 * c);
 }
 
+// Table mode (the learned decoder step, Eq. 1 with Eq. 12): a chunk of
+// stage s with code byte v decodes to n * T_s[v][0..7], so its term is
+// n * sum_k T_s[v][k] x[8c+k].  The span's activations (protected columns
+// zeroed, fp16) sit at position P = 256h + 32j + l of a 16-byte-per-chunk
+// buffer, so lane l's loads hit consecutive words; the S decoder tables
+// (4 KB each) follow it.
+constexpr uint32_t kB1TabOff = 8192;   // the tables' offset in the table region
+
+// Job J of the span's activation buffer (see b1_table_job for J and lane):
+// chunk c = c0 + 256h + 8l + j, its 8 activations with the layer's
+// protected columns zeroed, as fp16, at position 256h + 32j + l.
+__device__ __forceinline__ void b1_xspan_job(uint32_t xs, const uint32_t *pm, int c0, int J, int lane,
+                                             uint4 xv) {
+    const int h = (J >> 3) & 1, j = J & 7;
+    const int c = c0 + h * 256 + 8 * lane + j;
+    const uint32_t m = (pm[c >> 2] >> ((c & 3) * 8)) & 0xFFu;
+    const uint32_t w[4] = {xv.x, xv.y, xv.z, xv.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const float lo = (m >> (2 * q)) & 1u ? 0.f : __uint_as_float(w[q] << 16);
+        const float hi = (m >> (2 * q + 1)) & 1u ? 0.f : __uint_as_float(w[q] & 0xFFFF0000u);
+        const __half2 hv = __floats2half2_rn(lo, hi);
+        o[q] = *reinterpret_cast<const uint32_t *>(&hv);
+    }
+    const uint32_t dst = xs + static_cast<uint32_t>((h * 256 + 32 * j + lane) * 16);
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(o[0]), "r"(o[1]), "r"(o[2]), "r"(o[3]));
+}
+
+// Lane sums of one item in table mode: chunks 8l + j of each half through
+// the stage's table at tb and the activations at xs_lane (the buffer plus
+// 16 * lane).  fp16 x fp16 products are exact in fp32.
+__device__ __forceinline__ float b1_item_tab(const uint2 (&cw)[2], const uint4 (&nw)[2], uint32_t xs_lane,
+                                             uint32_t tb) {
+    float acc4[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+#pragma unroll
+        for (int jw = 0; jw < 2; ++jw) {
+            const uint32_t w = jw ? cw[h].y : cw[h].x;
+            const uint32_t n01 = jw ? nw[h].z : nw[h].x;
+            const uint32_t n23 = jw ? nw[h].w : nw[h].y;
+            float &acc = acc4[h][jw];
+#pragma unroll
+            for (int jj = 0; jj < 4; ++jj) {
+                const int j = 4 * jw + jj;
+                const uint32_t v = (w >> (8 * jj)) & 0xFFu;
+                const uint4 t = lds_u128(tb + v * 16u);
+                const uint4 xx = lds_u128(xs_lane + static_cast<uint32_t>((h * 256 + 32 * j) * 16));
+                const uint32_t tw[4] = {t.x, t.y, t.z, t.w}, xw[4] = {xx.x, xx.y, xx.z, xx.w};
+                float d = 0.f;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    d = fma_f16_f32(lo_half(tw[q]), lo_half(xw[q]), d);
+                    d = fma_f16_f32(hi_half(tw[q]), hi_half(xw[q]), d);
+                }
+                const uint32_t nn = jj < 2 ? n01 : n23;
+                const uint16_t n = (jj & 1) ? hi_half(nn) : lo_half(nn);
+                acc = fmaf(__half2float(__ushort_as_half(n)), d, acc);
+            }
+        }
+    }
+    return (acc4[0][0] + acc4[0][1]) + (acc4[1][0] + acc4[1][1]);
+}
+
 // NW warps; D ring slots (one item each) per warp; NSPAN 4096-column spans
 // per row (0: a.nspan > 1, at run time).  With one span, every ring address
 // is an immediate offset; with several, a CTA holds the table of one span at
 // a time and walks its items span by span, rebuilding the table between
 // spans (x of the next span is loaded while the current one is decoded).
 // FMT: the protected payloads may be FP8 or bf16 (their conversions compiled
-// in); without it every payload is int8.
-template <int NW, int D, int NSPAN, bool FMT>
+// in); without it every payload is int8.  TAB: table mode (the decoder
+// tables of a.tab instead of the sign decode; one layer, int8 payloads).
+template <int NW, int D, int NSPAN, bool FMT, bool TAB>
 __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ B1Args a) {
     static_assert(D <= 4, "one folded reduction covers a ring pass");
     constexpr int kThreads = NW * 32;
@@ -394,9 +461,22 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
 #pragma unroll
         for (int q = 0; q < (16 + NW - 1) / NW; ++q)
             if (warp + q * NW < 16) xv[q] = b1_table_x(a.x, 0, warp + q * NW, lane);
+        if constexpr (TAB) {
+            // the decoder tables, S x 4 KB, beside the activation buffer
+            for (int q = threadIdx.x; q < S * 256; q += kThreads) {
+                const uint4 t = reinterpret_cast<const uint4 *>(a.tab)[q];
+                asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(sbase + kB1TabOff + q * 16u),
+                             "r"(t.x), "r"(t.y), "r"(t.z), "r"(t.w));
+            }
+        }
 #pragma unroll
         for (int q = 0; q < (16 + NW - 1) / NW; ++q)
-            if (warp + q * NW < 16) b1_table_job(sbase, pm, 0, warp + q * NW, lane, xv[q]);
+            if (warp + q * NW < 16) {
+                if constexpr (TAB)
+                    b1_xspan_job(sbase, pm, 0, warp + q * NW, lane, xv[q]);
+                else
+                    b1_table_job(sbase, pm, 0, warp + q * NW, lane, xv[q]);
+            }
     }
     if (threadIdx.x < p) sx[threadIdx.x] = uj >= 0 ? ssc[threadIdx.x] * bf16_bits_to_f32(xj) : 0.f;
     for (int u = threadIdx.x + kThreads; u < p; u += kThreads) {
@@ -406,6 +486,11 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     __syncthreads();
 
     const uint32_t base0 = sbase + lane * 4u;
+    // table mode: this lane's activation words, and the stage and the items
+    // left in the row run of the next item to decode (the consumer's walk of
+    // the same run the requests take)
+    const uint32_t xs_lane = sbase + lane * 16u;
+    int tst = s0, trl = nrows - r0;
     int i = 0;   // items consumed
     // slot d: wait for it, decode its item into this lane's partial sum,
     // request the next item into it; false on a timeout
@@ -430,7 +515,16 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
         // it before the decode, so the copy's latency overlaps the decode
         __syncwarp();
         if (left > 0) fill(d);
-        v = b1_item(cw, nw, base0);
+        if constexpr (TAB) {
+            // this item's stage: the consumer's own walk of the run
+            v = b1_item_tab(cw, nw, xs_lane, sbase + kB1TabOff + static_cast<uint32_t>(tst) * 4096u);
+            if (--trl == 0) {
+                ++tst;
+                trl = nrows;
+            }
+        } else {
+            v = b1_item(cw, nw, base0);
+        }
         return true;
     };
     if constexpr (NSPAN == 1) {
@@ -460,11 +554,18 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
             if (warp + q * NW < 16 && nspan > 1) xn[q] = b1_table_x(a.x, 1, warp + q * NW, lane);
         // (after a timeout the warp still passes every span's barriers)
         for (int sp = 0; sp < nspan; ++sp) {
+            tst = s0;   // every span walks the same run of stages and rows
+            trl = nrows - r0;
             if (sp > 0) {
                 __syncthreads();   // every warp is done with the table of span sp - 1
 #pragma unroll
                 for (int q = 0; q < (16 + NW - 1) / NW; ++q)
-                    if (warp + q * NW < 16) b1_table_job(sbase, pm, sp * kB1Span, warp + q * NW, lane, xn[q]);
+                    if (warp + q * NW < 16) {
+                        if constexpr (TAB)
+                            b1_xspan_job(sbase, pm, sp * kB1Span, warp + q * NW, lane, xn[q]);
+                        else
+                            b1_table_job(sbase, pm, sp * kB1Span, warp + q * NW, lane, xn[q]);
+                    }
                 __syncthreads();
 #pragma unroll
                 for (int q = 0; q < (16 + NW - 1) / NW; ++q)
@@ -606,7 +707,9 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
         float v = 0.f;
         for (int sp = 0; sp < nspan; ++sp)
             for (int s = 0; s < S; ++s) v += part[sp * per_span + s * nrows + rr];
-        v = v * kB1InvSqrt8 + (p > 0 ? prot[rr] : 0.f);
+        // (the sign decode's 1/sqrt(8) of Eq. 3; a decoder table holds its
+        // outputs as they are)
+        v = v * (TAB ? 1.f : kB1InvSqrt8) + (p > 0 ? prot[rr] : 0.f);
         if (L.rank > 0) {
             const uint16_t *bm = L.lb + static_cast<size_t>(ra + rr) * L.rank;
             float bt = 0.f;
@@ -627,9 +730,9 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
 
 size_t align_up_b1(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
-template <int NW, int D, int NSPAN, bool FMT>
+template <int NW, int D, int NSPAN, bool FMT, bool TAB = false>
 bisco_status launch_b1_t(const B1Args &a, int grid, size_t smem, cudaStream_t stream) {
-    auto kern = k_gemv_b1<NW, D, NSPAN, FMT>;
+    auto kern = k_gemv_b1<NW, D, NSPAN, FMT, TAB>;
     static size_t configured[64] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return BISCO_ERR_CUDA;
@@ -661,7 +764,7 @@ size_t b1_coresident_budget() {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
     if (budget[dev] != 0) return budget[dev];
-    auto kern = k_gemv_b1<16, 3, 1, false>;
+    auto kern = k_gemv_b1<16, 3, 1, false, false>;
     constexpr size_t kHi = 160 * 1024;   // more than two CTAs of an SM can hold
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kHi)) !=
         cudaSuccess) {
@@ -727,7 +830,8 @@ constexpr B1Shape kB1Shapes[] = {{16, 3}, {16, 2}};
 }  // namespace
 
 bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, float *const *y,
-                            int *err, cudaStream_t stream, bool *launched, const bisco_lora *loras) {
+                            int *err, cudaStream_t stream, bool *launched, const bisco_lora *loras,
+                            const uint16_t *tables) {
     *launched = false;
     if (const char *e = getenv("BISCO_GEMV_B1"))
         if (e[0] == '0') return BISCO_OK;
@@ -839,6 +943,20 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
     // BISCO_ERR_TIMEOUT and returns with no copy in flight
     a.withhold = getenv("BISCO_TEST_WITHHOLD_COPIES") != nullptr;
     *launched = true;
+    if (tables != nullptr) {
+        // table mode: one layer, int8 payloads
+        if (G != 1 || (a.L[0].p > 0 && a.L[0].fmt != BISCO_PROT_INT8) || a.lrank > 0) {
+            *launched = false;
+            return BISCO_OK;
+        }
+        a.tab = tables;
+        if (one) {
+            if (pick.depth == 3) return launch_b1_t<16, 3, 1, false, true>(a, total, smem, stream);
+            return launch_b1_t<16, 2, 1, false, true>(a, total, smem, stream);
+        }
+        if (pick.depth == 3) return launch_b1_t<16, 3, 0, false, true>(a, total, smem, stream);
+        return launch_b1_t<16, 2, 0, false, true>(a, total, smem, stream);
+    }
     // int8 payloads only (the common case) or any format (FMT: the other
     // formats' conversions compiled in)
     bool fmt = false;

@@ -62,6 +62,35 @@ def test_gemv_table_matches_oracle(env, N, K, S, p, B, kind):
     assert max_rel_rows(y.cpu().numpy(), want) <= TOL
 
 
+@pytest.mark.parametrize("N,K,S,p,kind", [
+    (1000, 4096, 2, 41, "mlp"), (4096, 4096, 2, 41, "linear"), (300, 8192, 3, 82, "linear"),
+    (150, 4096, 1, 0, "mlp"),
+])
+def test_gemv_table_batch1_kernel(env, N, K, S, p, kind, monkeypatch):
+    """Batch 1 with K a multiple of 4096: the row-split kernel in table mode
+    (the span's activations and the S tables in shared memory; fp16 x fp16
+    products, exact, summed in fp32).  Against the oracle far inside the
+    bar (fp32 sums over K terms), against the one-warp-per-row kernel
+    (BISCO_GEMV_MODE forces it), and the same bits on a second call."""
+    import torch
+    bisco, dev = env
+    ref = oracle.encode(synth.layer_weights(N, K, seed=N + 17), S=S, p=p)
+    L = bisco.Layer.from_numpy(ref, dev)
+    tabs = mlp_tables(S, seed=K + 1) if kind == "mlp" else linear_tables(S, seed=K + 1)
+    x = synth.activations(1, K, seed=6)
+    td, xd = to_dev(tabs, dev), to_dev(x, dev)
+    y = bisco.bisco_gemv_table(L, td, xd)
+    y2 = bisco.bisco_gemv_table(L, td, xd)
+    monkeypatch.setenv("BISCO_GEMV_MODE", "stream")
+    y_rows = bisco.bisco_gemv_table(L, td, xd)
+    torch.cuda.synchronize()
+    assert bisco.bisco_get_device_error() == 0
+    want = oracle.matmul(oracle.decode_rows_table(ref, tabs), x)
+    assert max_rel_rows(y.cpu().numpy(), want) <= 2e-5
+    assert max_rel_rows(y.cpu().numpy(), y_rows.cpu().numpy()) <= 2e-5
+    assert torch.equal(y, y2)
+
+
 def test_identity_table_is_the_norm_rescale_decoder(env):
     """The binary16 table of +-1/sqrt(8) gives bisco_gemv's result up to the
     table's rounding (|fp16(1/sqrt 8) - 1/sqrt 8| relative, about 1.6e-4)."""
