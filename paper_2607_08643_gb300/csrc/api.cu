@@ -34,8 +34,8 @@ int current_device() {
 
 // Layers whose protected set the decode kernels do not take themselves:
 // output rows (rows.cu) and payloads other than INT8 (formats.cu) -- except
-// at batch 1, where the row-split kernel takes protected columns in every
-// payload format.
+// at batch 1, where the row-split kernel takes protected columns and rows in
+// every payload format.
 bool needs_epilogue(const bisco_layer &L) {
     return L.n_protected > 0 &&
            (L.protect_axis == 1 || L.protect_format != BISCO_PROT_INT8);
@@ -283,9 +283,9 @@ bisco_status bisco_gemv(const bisco_layer *L, const uint16_t *x_bf16, int32_t B,
     if (!err) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     if (needs_epilogue(*L)) {
-        // batch 1, protected columns in an FP8 / bf16 payload: the batch-1
-        // kernel takes those formats itself, in one launch
-        if (B == 1 && L->protect_axis == 0 && !getenv("BISCO_GEMV_MODE")) {
+        // batch 1, protected columns in an FP8 / bf16 payload or protected
+        // rows: the batch-1 kernel takes those itself, in one launch
+        if (B == 1 && !getenv("BISCO_GEMV_MODE")) {
             bool launched = false;
             st = launch_gemv_b1(L, 1, x_bf16, &y, err, s, &launched);
             if (launched || st != BISCO_OK) return st;
@@ -316,17 +316,16 @@ bisco_status bisco_gemv_multi(const bisco_layer *layers, int32_t G, const uint16
     if (!err) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     bisco_layer stages[BISCO_GEMV_MULTI_MAX];
-    bool any = false, rows = false;
+    bool any = false;
     for (int g = 0; g < G; ++g) {
         const bool e = needs_epilogue(layers[g]);
         any |= e;
-        rows |= layers[g].protect_axis == 1 && layers[g].n_protected > 0;
         stages[g] = e ? bsq_only(layers[g]) : layers[g];
     }
     if (!any) return launch_gemv_multi(layers, G, x_bf16, B, y, err, s);
-    // batch 1, protected columns in any payload format: one launch of the
-    // batch-1 kernel
-    if (B == 1 && !rows && !getenv("BISCO_GEMV_MODE")) {
+    // batch 1, protected columns or rows in any payload format: one launch
+    // of the batch-1 kernel
+    if (B == 1 && !getenv("BISCO_GEMV_MODE")) {
         bool launched = false;
         st = launch_gemv_b1(layers, G, x_bf16, y, err, s, &launched);
         if (launched || st != BISCO_OK) return st;

@@ -56,6 +56,8 @@
 #include <stdint.h>
 #include <stdlib.h>
 
+#include <type_traits>
+
 #include "bisco_dev.cuh"
 #include "bisco_host.h"
 #include "fp8.cuh"
@@ -67,6 +69,8 @@ constexpr int kB1Span = 512;                  // chunks per item
 constexpr uint32_t kB1Item = 1536;            // bytes per item slot: signs, then norms
 constexpr int kB1MaxG = 4;                    // layers per launch
 constexpr float kB1InvSqrt8 = 0.35355339059327373f;
+// kernel instances by the protected set's kind (see k_gemv_b1)
+constexpr int kB1Int8 = 0, kB1Fmt = 1, kB1Rows = 2, kB1Tab = 3;
 // dynamic shared memory of one CTA at most (227 KB per block less the
 // kernel's static shared memory, rounded down)
 constexpr size_t kB1MaxSmem = 226 * 1024;
@@ -90,6 +94,8 @@ struct B1Layer {
     int N, p, p_pad;
     int fmt;                   // BISCO_PROT_*: int8, FP8 E4M3 / E5M2 or bf16 payload
     int prow;                  // payload bytes per row: p_pad elements of 1 or 2 bytes
+    int axis;                  // 1: the protected channels are output rows (payload
+                               // [p][kp], kp = roundup(K, 16) elements a row)
     int cta0, ctas;            // the CTAs of the grid that take this layer's rows
 };
 
@@ -315,17 +321,19 @@ __device__ __forceinline__ float b1_item_tab(const uint2 (&cw)[2], const uint4 (
 // is an immediate offset; with several, a CTA holds the table of one span at
 // a time and walks its items span by span, rebuilding the table between
 // spans (x of the next span is loaded while the current one is decoded).
-// FMT: the protected payloads may be FP8 or bf16 (their conversions compiled
-// in); without it every payload is int8.  TAB: table mode (the decoder
-// tables of a.tab instead of the sign decode; one layer, int8 payloads).
-template <int NW, int D, int NSPAN, bool FMT, bool TAB>
+// MODE: the protected set's kind, one instance each -- kB1Int8 (int8
+// columns, the common case), kB1Fmt (columns in any payload format: the
+// FP8 / bf16 conversions compiled in), kB1Rows (output rows in any format)
+// or kB1Tab (table mode: the decoder tables of a.tab instead of the sign
+// decode; one layer, int8 columns).
+template <int NW, int D, int NSPAN, int MODE>
 __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ B1Args a) {
     static_assert(D <= 4, "one folded reduction covers a ring pass");
     constexpr int kThreads = NW * 32;
     extern __shared__ unsigned char smem_raw[];
     unsigned char *sm = align_smem<4096>(smem_raw);
     const uint32_t sbase = smem_u32(sm);
-    __shared__ int s_abort, s_lnext;
+    __shared__ int s_abort, s_lnext, s_r0, s_r1;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int K = a.K, C = K / 8, nspan = NSPAN ? NSPAN : a.nspan, S = a.S;
@@ -335,7 +343,11 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     for (int i = 1; i < kB1MaxG; ++i)
         if (i < a.G && static_cast<int>(blockIdx.x) >= a.L[i].cta0) g = i;
     const B1Layer &L = a.L[g];
-    const int N = L.N, p = L.p, prow = L.prow, fmt = L.fmt;
+    const int N = L.N, prow = L.prow, fmt = L.fmt;
+    // protected input columns (Eq. 10) or, with axis 1, output rows (Eq. 9;
+    // taken by the FMT instances only)
+    constexpr bool FMT = MODE == kB1Fmt || MODE == kB1Rows, ROWS = MODE == kB1Rows, TAB = MODE == kB1Tab;
+    const int p = ROWS ? 0 : L.p, prows = ROWS ? L.p : 0;
     const int ci = static_cast<int>(blockIdx.x) - L.cta0;
     const int ra = static_cast<int>(static_cast<int64_t>(N) * ci / L.ctas);
     const int rb = static_cast<int>(static_cast<int64_t>(N) * (ci + 1) / L.ctas);
@@ -408,7 +420,29 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     if (threadIdx.x == 0) {
         s_abort = 0;
         s_lnext = 0;
+        // protected output rows of this CTA: [s_r0, s_r1) of the ascending list
+        int t0 = 0, t1 = 0;
+        if (ROWS && prows > 0) {
+            int lo = 0, hi = prows;
+            while (lo < hi) {
+                const int mid = (lo + hi) >> 1;
+                if (L.prot_idx[mid] < ra) lo = mid + 1;
+                else hi = mid;
+            }
+            t0 = lo;
+            hi = prows;
+            while (lo < hi) {
+                const int mid = (lo + hi) >> 1;
+                if (L.prot_idx[mid] < rb) lo = mid + 1;
+                else hi = mid;
+            }
+            t1 = lo;
+        }
+        s_r0 = t0;
+        s_r1 = t1;
     }
+    if (ROWS && prows > 0)
+        for (int rr = threadIdx.x; rr < nrows; rr += kThreads) prot[rr] = 0.f;
     for (int i = threadIdx.x; i < C / 4; i += kThreads) pm[i] = 0u;
     __syncthreads();
     for (int u = threadIdx.x; u < p; u += kThreads) {
@@ -690,6 +724,69 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     }
     __syncthreads();
     if (*reinterpret_cast<volatile int *>(&s_abort)) return;
+    // ---- protected output rows (Eq. 9 with Eq. 10 on rows): their chunks
+    // store norm 0, so the decode gave them 0; each is the dot product of
+    // its payload row with x, times the row's scale.  Every warp takes K/16
+    // columns of each of the CTA's protected rows (lane l eight of them per
+    // 256), its sums go to the now idle ring, and a thread per row adds the
+    // 16 in warp order.
+    if constexpr (ROWS) {
+        // rows in batches the ring holds (depth * 1536 bytes a warp)
+        const int cap = a.depth * static_cast<int>(kB1Item) / 4;
+        for (int b0 = s_r0; b0 < s_r1; b0 += cap) {
+            const int b1 = min(s_r1, b0 + cap), nr = b1 - b0;
+            float *rp = reinterpret_cast<float *>(sm + a.off_ring);   // [row][warp]
+            const int kp = (K + 15) / 16 * 16, kw = K / NW;
+            const bool bf = fmt == BISCO_PROT_BF16;
+            for (int t = b0; t < b1; ++t) {
+                const unsigned char *qr =
+                    reinterpret_cast<const unsigned char *>(q8) + static_cast<int64_t>(t) * kp * (bf ? 2 : 1);
+                float d = 0.f;
+                for (int k0 = warp * kw + lane * 8; k0 < (warp + 1) * kw; k0 += 256) {
+                    const uint4 xv = *reinterpret_cast<const uint4 *>(a.x + k0);
+                    const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
+                    float qf[8];
+                    if (bf) {
+                        const uint4 q = *reinterpret_cast<const uint4 *>(qr + 2 * k0);
+                        const uint32_t qw[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            qf[2 * e] = __uint_as_float(qw[e] << 16);
+                            qf[2 * e + 1] = __uint_as_float(qw[e] & 0xFFFF0000u);
+                        }
+                    } else {
+                        const uint2 q = *reinterpret_cast<const uint2 *>(qr + k0);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            const uint32_t b8 = ((e < 4 ? q.x : q.y) >> (8 * (e & 3))) & 0xFFu;
+                            qf[e] = fmt == BISCO_PROT_INT8 ? static_cast<float>(static_cast<int8_t>(b8))
+                                                           : fp8_to_f32(b8, fmt);
+                        }
+                    }
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        d = fmaf(qf[2 * e], __uint_as_float(xw[e] << 16), d);
+                        d = fmaf(qf[2 * e + 1], __uint_as_float(xw[e] & 0xFFFF0000u), d);
+                    }
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) d += __shfl_xor_sync(0xFFFFFFFFu, d, o);
+                if (lane == 0) rp[(t - b0) * NW + warp] = d;
+            }
+            __syncthreads();
+            for (int i = threadIdx.x; i < nr; i += kThreads) {
+                const int rr = L.prot_idx[b0 + i] - ra;
+                if (rr < 0 || rr >= nrows) {   // not an ascending list
+                    latch_error(a.err, BISCO_ERR_INVALID_ARG);
+                    continue;
+                }
+                float d = 0.f;
+                for (int w = 0; w < NW; ++w) d += rp[i * NW + w];
+                prot[rr] = __half2float(__ushort_as_half(L.q8_scale[b0 + i])) * d;
+            }
+            __syncthreads();
+        }
+    }
     // t[r]: the slices' sums in slice order
     float *lt_t = lt + nsl * a.lrank;
     if (L.rank > 0) {
@@ -709,7 +806,7 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
             for (int s = 0; s < S; ++s) v += part[sp * per_span + s * nrows + rr];
         // (the sign decode's 1/sqrt(8) of Eq. 3; a decoder table holds its
         // outputs as they are)
-        v = v * (TAB ? 1.f : kB1InvSqrt8) + (p > 0 ? prot[rr] : 0.f);
+        v = v * (TAB ? 1.f : kB1InvSqrt8) + (L.p > 0 ? prot[rr] : 0.f);
         if (L.rank > 0) {
             const uint16_t *bm = L.lb + static_cast<size_t>(ra + rr) * L.rank;
             float bt = 0.f;
@@ -730,9 +827,9 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
 
 size_t align_up_b1(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
-template <int NW, int D, int NSPAN, bool FMT, bool TAB = false>
+template <int NW, int D, int NSPAN, int MODE>
 bisco_status launch_b1_t(const B1Args &a, int grid, size_t smem, cudaStream_t stream) {
-    auto kern = k_gemv_b1<NW, D, NSPAN, FMT, TAB>;
+    auto kern = k_gemv_b1<NW, D, NSPAN, MODE>;
     static size_t configured[64] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return BISCO_ERR_CUDA;
@@ -764,7 +861,7 @@ size_t b1_coresident_budget() {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
     if (budget[dev] != 0) return budget[dev];
-    auto kern = k_gemv_b1<16, 3, 1, false, false>;
+    auto kern = k_gemv_b1<16, 3, 1, kB1Int8>;
     constexpr size_t kHi = 160 * 1024;   // more than two CTAs of an SM can hold
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kHi)) !=
         cudaSuccess) {
@@ -847,7 +944,7 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
     int p_max = 0;
     for (int g = 0; g < G; ++g) {
         const bisco_layer &L = Ls[g];
-        if (L.k_in != K || L.stages != S || L.protect_axis != 0) return BISCO_OK;
+        if (L.k_in != K || L.stages != S) return BISCO_OK;
         // the kernel's byte offsets into the sign planes are 32-bit
         if (static_cast<uint64_t>(S) * L.n_out * (K / 8) >= (1ull << 32)) return BISCO_OK;
         B1Layer &b = a.L[g];
@@ -861,8 +958,10 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
         b.p = L.n_protected;
         b.p_pad = (L.n_protected + 15) / 16 * 16;
         b.fmt = L.protect_format;
-        b.prow = b.p_pad * (L.protect_format == BISCO_PROT_BF16 ? 2 : 1);
-        p_max = p_max > b.p ? p_max : b.p;
+        b.axis = L.protect_axis;
+        // int8 rows staged per CTA: the column payload only
+        b.prow = L.protect_axis ? 0 : b.p_pad * (L.protect_format == BISCO_PROT_BF16 ? 2 : 1);
+        if (!b.axis) p_max = p_max > b.p ? p_max : b.p;   // the column sets' metadata
         if (loras != nullptr && loras[g].rank > 0) {
             // the compensation's slices are 256 columns of one span
             if (a.nspan != 1) return BISCO_OK;
@@ -943,37 +1042,47 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
     // BISCO_ERR_TIMEOUT and returns with no copy in flight
     a.withhold = getenv("BISCO_TEST_WITHHOLD_COPIES") != nullptr;
     *launched = true;
+    int mode = kB1Int8;
     if (tables != nullptr) {
-        // table mode: one layer, int8 payloads
-        if (G != 1 || (a.L[0].p > 0 && a.L[0].fmt != BISCO_PROT_INT8) || a.lrank > 0) {
+        // table mode: one layer, int8 columns
+        if (G != 1 || (a.L[0].p > 0 && (a.L[0].fmt != BISCO_PROT_INT8 || a.L[0].axis != 0)) || a.lrank > 0) {
             *launched = false;
             return BISCO_OK;
         }
         a.tab = tables;
-        if (one) {
-            if (pick.depth == 3) return launch_b1_t<16, 3, 1, false, true>(a, total, smem, stream);
-            return launch_b1_t<16, 2, 1, false, true>(a, total, smem, stream);
+        mode = kB1Tab;
+    } else {
+        // the kind of every protected set of the launch: one instance takes
+        // int8 columns, one any column format, one rows (not mixed)
+        bool cols_fmt = false, rows = false, cols = false;
+        for (int g = 0; g < G; ++g) {
+            if (a.L[g].p == 0) continue;
+            if (a.L[g].axis) rows = true;
+            else {
+                cols = true;
+                cols_fmt |= a.L[g].fmt != BISCO_PROT_INT8;
+            }
         }
-        if (pick.depth == 3) return launch_b1_t<16, 3, 0, false, true>(a, total, smem, stream);
-        return launch_b1_t<16, 2, 0, false, true>(a, total, smem, stream);
-    }
-    // int8 payloads only (the common case) or any format (FMT: the other
-    // formats' conversions compiled in)
-    bool fmt = false;
-    for (int g = 0; g < G; ++g) fmt |= a.L[g].p > 0 && a.L[g].fmt != BISCO_PROT_INT8;
-    if (fmt) {
-        if (one) {
-            if (pick.depth == 3) return launch_b1_t<16, 3, 1, true>(a, total, smem, stream);
-            return launch_b1_t<16, 2, 1, true>(a, total, smem, stream);
+        if (rows && cols) {
+            *launched = false;
+            return BISCO_OK;
         }
-        if (pick.depth == 3) return launch_b1_t<16, 3, 0, true>(a, total, smem, stream);
-        return launch_b1_t<16, 2, 0, true>(a, total, smem, stream);
+        mode = rows ? kB1Rows : cols_fmt ? kB1Fmt : kB1Int8;
     }
-    if (one) {
-        if (pick.depth == 3) return launch_b1_t<16, 3, 1, false>(a, total, smem, stream);
-        return launch_b1_t<16, 2, 1, false>(a, total, smem, stream);
+    auto go = [&](auto mode_c) {
+        constexpr int M = decltype(mode_c)::value;
+        if (one) {
+            if (pick.depth == 3) return launch_b1_t<16, 3, 1, M>(a, total, smem, stream);
+            return launch_b1_t<16, 2, 1, M>(a, total, smem, stream);
+        }
+        if (pick.depth == 3) return launch_b1_t<16, 3, 0, M>(a, total, smem, stream);
+        return launch_b1_t<16, 2, 0, M>(a, total, smem, stream);
+    };
+    switch (mode) {
+        case kB1Fmt: return go(std::integral_constant<int, kB1Fmt>());
+        case kB1Rows: return go(std::integral_constant<int, kB1Rows>());
+        case kB1Tab: return go(std::integral_constant<int, kB1Tab>());
+        default: return go(std::integral_constant<int, kB1Int8>());
     }
-    if (pick.depth == 3) return launch_b1_t<16, 3, 0, false>(a, total, smem, stream);
-    return launch_b1_t<16, 2, 0, false>(a, total, smem, stream);
 }
 }  // namespace bisco

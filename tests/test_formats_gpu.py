@@ -210,10 +210,13 @@ def test_encode_rows_formats_bit_exact(env, fmt):
 
 
 @pytest.mark.parametrize("fmt", FORMATS)
-def test_gemv_gemm_rows_formats_match_oracle(env, fmt):
+@pytest.mark.parametrize("K", [1024, 4096])
+def test_gemv_gemm_rows_formats_match_oracle(env, fmt, K):
+    """Protected rows in each payload format; at K = 4096 batch 1 goes to the
+    row-split kernel (the rows' payload dot products after its decode)."""
     import torch
     bisco, dev = env
-    N, K = 512, 1024
+    N = 512
     ref = oracle_rows_layer(synth.layer_weights(N, K, seed=61), 2, 6, fmt)
     L = bisco.Layer.from_numpy(ref, dev)
     What = oracle_rows_dense(ref)

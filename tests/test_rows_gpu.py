@@ -152,6 +152,8 @@ def _row_layer(env, N, K, S, p, seed):
 @pytest.mark.parametrize("N,K,S,p,B", [
     (1024, 1024, 2, 11, 1), (1024, 1024, 2, 11, 16), (300, 4096, 2, 3, 4),
     (64, 136, 2, 3, 2), (48, 256, 3, 48, 1), (4096, 512, 2, 0, 8),
+    # batch 1, K a multiple of 4096: the row-split kernel takes the rows
+    (1000, 4096, 2, 10, 1), (300, 8192, 3, 30, 1), (48, 4096, 2, 48, 1),
 ])
 def test_gemv_rows_matches_oracle(env, N, K, S, p, B):
     import torch
@@ -172,10 +174,11 @@ def test_gemv_rows_matches_oracle(env, N, K, S, p, B):
         assert np.all(np.abs(got - want) <= bound + 1e-30)
 
 
-def test_gemv_multi_mixes_row_and_column_layers(env):
+@pytest.mark.parametrize("K", [1024, 4096])
+def test_gemv_multi_mixes_row_and_column_layers(env, K):
     import torch
     bisco, dev = env
-    K, S = 1024, 2
+    S = 2
     Lr, rr = _row_layer(env, 512, K, S, 6, seed=71)
     Wc = synth.layer_weights(256, K, seed=72)
     rc = oracle.encode(Wc, S=S, p=11)
