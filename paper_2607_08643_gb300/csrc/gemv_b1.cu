@@ -294,7 +294,8 @@ __device__ __forceinline__ float b1_item_tab(const uint2 (&cw)[2], const uint4 (
             const uint32_t n01 = jw ? nw[h].z : nw[h].x;
             const uint32_t n23 = jw ? nw[h].w : nw[h].y;
             float &acc = acc4[h][jw];
-#pragma unroll
+            // (unrolled by two: fully unrolled, the kernel spills)
+#pragma unroll 2
             for (int jj = 0; jj < 4; ++jj) {
                 const int j = 4 * jw + jj;
                 const uint32_t v = (w >> (8 * jj)) & 0xFFu;
