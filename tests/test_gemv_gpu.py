@@ -323,6 +323,7 @@ def test_gemv_b1_matches_oracle(env, N, K, S, p):
     (4096, [(3000, 41), (2000, 0), (1500, 41), (4000, 10)]),  # four layers
     (4096, [(200, 5), (7, 3), (150, 0)]),                     # a 7-row layer between larger ones
     (12288, [(700, 123), (90, 0), (333, 60)]),                # three spans, three layers
+    (4096, [(12288, 41), (12288, 41)]),                       # gate/up: two CTAs per SM (the step's dominant call)
 ])
 def test_gemv_b1_groups_match_oracle(env, K, shapes):
     S = 2
