@@ -299,9 +299,8 @@ typedef struct bisco_lora {
  * layer (fp32, summed in a fixed order, so the result does not depend on
  * the launch) and adds Bm t to its rows when it writes them.  loras: host
  * array of G structs.  Taken by the batch-1 row-split kernel only: batch 1,
- * k_in == 4096, stages 1..3, protected columns (any payload format), every
- * rank a multiple of 8 in [0, BISCO_GEMV_LORA_MAX_RANK]; other combinations
- * return
+ * k_in == 4096, stages 1..3, int8 protected columns, every rank a multiple
+ * of 8 in [0, BISCO_GEMV_LORA_MAX_RANK]; other combinations return
  * BISCO_ERR_UNSUPPORTED (run bisco_gemv_multi and bisco_lora_apply then).
  * Malformed arguments: BISCO_ERR_INVALID_ARG.  Layers, x and y as for
  * bisco_gemv_multi.  bisco_gemv_lora is the G = 1 case.

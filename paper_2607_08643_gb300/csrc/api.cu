@@ -350,7 +350,7 @@ bisco_status bisco_gemv_multi_lora(const bisco_layer *layers, const bisco_lora *
         if (r.rank < 0 || r.rank > BISCO_GEMV_LORA_MAX_RANK || r.rank % 8 != 0) return BISCO_ERR_INVALID_ARG;
         if (r.rank > 0 && (!r.A || !r.Bm || !aligned16(r.A) || !aligned16(r.Bm) || !std::isfinite(r.scale)))
             return BISCO_ERR_INVALID_ARG;
-        if (layers[g].protect_axis == 1 && layers[g].n_protected > 0) return BISCO_ERR_UNSUPPORTED;
+        if (needs_epilogue(layers[g])) return BISCO_ERR_UNSUPPORTED;   // int8 columns only
     }
     if (layers[0].k_in != 4096) return BISCO_ERR_UNSUPPORTED;
     bisco_status st;

@@ -70,7 +70,7 @@ constexpr uint32_t kB1Item = 1536;            // bytes per item slot: signs, the
 constexpr int kB1MaxG = 4;                    // layers per launch
 constexpr float kB1InvSqrt8 = 0.35355339059327373f;
 // kernel instances by the protected set's kind (see k_gemv_b1)
-constexpr int kB1Int8 = 0, kB1Fmt = 1, kB1Rows = 2, kB1Tab = 3;
+constexpr int kB1Int8 = 0, kB1Fmt = 1, kB1Rows = 2, kB1Tab = 3, kB1Lora = 4;
 // dynamic shared memory of one CTA at most (227 KB per block less the
 // kernel's static shared memory, rounded down)
 constexpr size_t kB1MaxSmem = 226 * 1024;
@@ -326,7 +326,8 @@ __device__ __forceinline__ float b1_item_tab(const uint2 (&cw)[2], const uint4 (
 // columns, the common case), kB1Fmt (columns in any payload format: the
 // FP8 / bf16 conversions compiled in), kB1Rows (output rows in any format)
 // or kB1Tab (table mode: the decoder tables of a.tab instead of the sign
-// decode; one layer, int8 columns).
+// decode; one layer, int8 columns), or kB1Lora (int8 columns with each
+// layer's low-rank compensation).
 template <int NW, int D, int NSPAN, int MODE>
 __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ B1Args a) {
     static_assert(D <= 4, "one folded reduction covers a ring pass");
@@ -347,7 +348,9 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     const int N = L.N, prow = L.prow, fmt = L.fmt;
     // protected input columns (Eq. 10) or, with axis 1, output rows (Eq. 9;
     // taken by the FMT instances only)
-    constexpr bool FMT = MODE == kB1Fmt || MODE == kB1Rows, ROWS = MODE == kB1Rows, TAB = MODE == kB1Tab;
+    constexpr bool FMT = MODE == kB1Fmt || MODE == kB1Rows, ROWS = MODE == kB1Rows,
+                   TAB = MODE == kB1Tab, LORA = MODE == kB1Lora;
+    const int lrank = LORA ? L.rank : 0;   // the compensation's rank (0: none)
     const int p = ROWS ? 0 : L.p, prows = ROWS ? L.p : 0;
     const int ci = static_cast<int>(blockIdx.x) - L.cta0;
     const int ra = static_cast<int>(static_cast<int64_t>(N) * ci / L.ctas);
@@ -464,14 +467,14 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     if (threadIdx.x == 32) prefetch_l2(a.x, static_cast<uint32_t>(K) * 2u);
     // the compensation's weights into L2 as well: this CTA's share of A
     // (every CTA of the layer reads all of it) and Bm's rows of its rows
-    if (L.rank > 0 && threadIdx.x == 64) {
-        const uint32_t abytes = static_cast<uint32_t>(L.rank) * K * 2u;
+    if (lrank > 0 && threadIdx.x == 64) {
+        const uint32_t abytes = static_cast<uint32_t>(lrank) * K * 2u;
         const uint32_t share = (abytes / L.ctas + 15u) / 16u * 16u;
         const uint32_t b0 = share * static_cast<uint32_t>(ci);
         if (b0 < abytes)
             prefetch_l2(reinterpret_cast<const unsigned char *>(L.la) + b0, min(share, abytes - b0));
         if (nrows > 0)
-            prefetch_l2(L.lb + static_cast<size_t>(ra) * L.rank, static_cast<uint32_t>(nrows * L.rank) * 2u);
+            prefetch_l2(L.lb + static_cast<size_t>(ra) * lrank, static_cast<uint32_t>(nrows * lrank) * 2u);
     }
     if (p > 0 && nrows > 0) {
         if (a.q8_staged) {
@@ -685,8 +688,8 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
     // into lt[column slice][rank]
     float *lt = reinterpret_cast<float *>(sm + a.off_lt);   // [K / 256][rank], then t [rank]
     const int nsl = K / 256;
-    if (L.rank > 0) {
-        const int nunit = (L.rank / 8) * nsl;
+    if (lrank > 0) {
+        const int nunit = (lrank / 8) * nsl;
         for (;;) {
             int u = 0;
             if (lane == 0) u = atomicAdd(&s_lnext, 1);
@@ -718,13 +721,23 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
             const float s0 = warp_sum4(d[0], d[1], d[2], d[3], lane);   // rank r0 + (lane >> 3)
             const float s1 = warp_sum4(d[4], d[5], d[6], d[7], lane);   // rank r0 + 4 + (lane >> 3)
             if ((lane & 7) == 0) {
-                lt[sl * L.rank + r0 + (lane >> 3)] = s0;
-                lt[sl * L.rank + r0 + 4 + (lane >> 3)] = s1;
+                lt[sl * lrank + r0 + (lane >> 3)] = s0;
+                lt[sl * lrank + r0 + 4 + (lane >> 3)] = s1;
             }
         }
     }
     __syncthreads();
     if (*reinterpret_cast<volatile int *>(&s_abort)) return;
+    // t[r]: the slices' sums in slice order
+    float *lt_t = lt + nsl * a.lrank;
+    if (lrank > 0) {
+        if (static_cast<int>(threadIdx.x) < lrank) {
+            float t = 0.f;
+            for (int sl = 0; sl < nsl; ++sl) t += lt[sl * lrank + threadIdx.x];
+            lt_t[threadIdx.x] = t;
+        }
+        __syncthreads();
+    }
     // ---- protected output rows (Eq. 9 with Eq. 10 on rows): their chunks
     // store norm 0, so the decode gave them 0; each is the dot product of
     // its payload row with x, times the row's scale.  Every warp takes K/16
@@ -788,16 +801,6 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
             __syncthreads();
         }
     }
-    // t[r]: the slices' sums in slice order
-    float *lt_t = lt + nsl * a.lrank;
-    if (L.rank > 0) {
-        if (static_cast<int>(threadIdx.x) < L.rank) {
-            float t = 0.f;
-            for (int sl = 0; sl < nsl; ++sl) t += lt[sl * L.rank + threadIdx.x];
-            lt_t[threadIdx.x] = t;
-        }
-        __syncthreads();
-    }
 
     // ---- outputs: a thread per row; the row's item sums in order, then the
     // protected term, then scale * (Bm t) of the compensation
@@ -808,10 +811,10 @@ __global__ void __launch_bounds__(NW * 32, 2) k_gemv_b1(const __grid_constant__ 
         // (the sign decode's 1/sqrt(8) of Eq. 3; a decoder table holds its
         // outputs as they are)
         v = v * (TAB ? 1.f : kB1InvSqrt8) + (L.p > 0 ? prot[rr] : 0.f);
-        if (L.rank > 0) {
-            const uint16_t *bm = L.lb + static_cast<size_t>(ra + rr) * L.rank;
+        if (lrank > 0) {
+            const uint16_t *bm = L.lb + static_cast<size_t>(ra + rr) * lrank;
             float bt = 0.f;
-            for (int r0 = 0; r0 < L.rank; r0 += 8) {
+            for (int r0 = 0; r0 < lrank; r0 += 8) {
                 const uint4 bv = *reinterpret_cast<const uint4 *>(bm + r0);
                 const uint32_t w[4] = {bv.x, bv.y, bv.z, bv.w};
 #pragma unroll
@@ -1064,11 +1067,11 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
                 cols_fmt |= a.L[g].fmt != BISCO_PROT_INT8;
             }
         }
-        if (rows && cols) {
+        if ((rows && cols) || (a.lrank > 0 && (rows || cols_fmt))) {
             *launched = false;
             return BISCO_OK;
         }
-        mode = rows ? kB1Rows : cols_fmt ? kB1Fmt : kB1Int8;
+        mode = a.lrank > 0 ? kB1Lora : rows ? kB1Rows : cols_fmt ? kB1Fmt : kB1Int8;
     }
     auto go = [&](auto mode_c) {
         constexpr int M = decltype(mode_c)::value;
@@ -1083,6 +1086,7 @@ bisco_status launch_gemv_b1(const bisco_layer *Ls, int G, const uint16_t *x, flo
         case kB1Fmt: return go(std::integral_constant<int, kB1Fmt>());
         case kB1Rows: return go(std::integral_constant<int, kB1Rows>());
         case kB1Tab: return go(std::integral_constant<int, kB1Tab>());
+        case kB1Lora: return go(std::integral_constant<int, kB1Lora>());
         default: return go(std::integral_constant<int, kB1Int8>());
     }
 }
