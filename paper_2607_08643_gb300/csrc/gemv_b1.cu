@@ -108,7 +108,7 @@ struct B1Args {
     int nspan;                 // K / 4096
     int S;                     // stages
     int depth;                 // item slots per warp
-    int q8_staged;             // int8 rows in shared memory (else read at the end)
+    int q8_staged;             // payload rows in shared memory (else read at the end)
     uint32_t sleep_ns;         // suspend-time hint of the item waits
     int withhold;              // test of the bounded waits: request no copies
     int lrank;                 // the largest compensation rank of the launch (0: none)
