@@ -120,7 +120,7 @@ typedef struct {
 #define BISCO_PROT_BF16 3
 
 /* ABI version of this header (major * 100 + minor). */
-#define BISCO_ABI_VERSION 106
+#define BISCO_ABI_VERSION 107
 int32_t bisco_abi_version(void);
 
 /* Static string for a status code (never NULL). */
@@ -321,10 +321,13 @@ bisco_status bisco_gemv_lora(const bisco_layer *L, const bisco_lora *lora, const
  * M, or other K, run the decode kernels of bisco_gemv.
  * X_bf16: [M][K] device; Y: [M][N] float32 device, fully overwritten.
  * workspace: device, 16-byte aligned, at least
- * bisco_gemm_workspace_bytes(L, M) bytes (M * (roundup(K,128) +
- * 2 * roundup(p,64)) * 2 on the tensor-core path, with p = 0 for a
- * row-protected layer; NULL when that is 0).  It holds the fp16 copy of X
- * and is overwritten.
+ * bisco_gemm_workspace_bytes(L, M) bytes (NULL when that is 0).  On the
+ * tensor-core path that is the fp16 copy of X, M * (roundup(K,128) +
+ * 2 * roundup(p,64)) * 2 bytes (p = 0 for a row-protected layer) rounded up
+ * to 256, followed by the partial tiles of the split of the work over the
+ * SMs, 160 * 2 * TN * 128 * 4 bytes with TN = 128 for M <= 128 and 256
+ * otherwise.  It is overwritten.  Tiles split between SMs are summed by a
+ * second kernel in a fixed order, so the result does not depend on timing.
  */
 size_t bisco_gemm_workspace_bytes(const bisco_layer *L, int32_t M);
 bisco_status bisco_gemm(const bisco_layer *L, const uint16_t *X_bf16, int32_t M, float *Y,

@@ -18,8 +18,10 @@
 // int8 q8 values (exact in fp16), so the protected term is a few more k
 // steps of the same MMA, and the epilogue is Y = D / sqrt(8).
 //
-// CTA roles (512 threads, one CTA per SM, persistent over output tiles):
-//   warps 0-3  epilogue: TMEM -> registers -> Y (fp32), lane quarter w
+// CTA roles (512 threads, one CTA per SM, persistent over a contiguous
+// range of whole tiles, or of the tiles' k-steps in a stream-K split):
+//   warps 0-3  epilogue: TMEM -> registers -> Y (fp32), or to a partial
+//              tile in the workspace; lane quarter w
 //   warp 4     TMA producer of the compressed-weight ring
 //   warp 5     TMEM allocator and MMA issuer (one thread)
 //   warp 6     TMA producer of the activation ring
@@ -34,7 +36,7 @@ namespace bisco {
 namespace {
 
 constexpr int GM = 128;     // output features per tile (MMA M, TMEM lanes)
-constexpr int GN = 256;     // tokens per tile (MMA N); 128 when 256 leaves SMs idle
+constexpr int GN = 256;     // tokens per tile (MMA N); 128 when M <= 128
 constexpr int GK = 128;     // K columns per weight step (one TMEM A stage)
 // Ring depths are template parameters (NX activation stages of 64 columns
 // = 32 KB, NW compressed-weight stages of 128 columns): the activation ring
@@ -50,15 +52,79 @@ constexpr uint32_t x_stage_bytes(int tn) { return static_cast<uint32_t>(tn) * 12
 constexpr float kInvSqrt8 = 0.35355339059327373f;
 constexpr float kSqrt8 = 2.8284271247461903f;
 
+// Work split over the persistent CTAs.  Whole tiles: CTA c takes tiles c,
+// c + G, c + 2G, ...  Stream-K: the tiles' k-steps are laid end to end
+// (tile t holds steps [t*KS, (t+1)*KS)) and CTA c takes the steps
+// [c*W/G, (c+1)*W/G), so every CTA has the same work.  A tile covered by
+// one CTA is written to Y directly; a tile
+// split between CTAs has each piece's fp32 sum written to the workspace (the
+// first piece of a CTA's range in its slot 0, the last in slot 1), and
+// k_gemm_fixup, launched after the GEMM, adds the pieces in CTA order and
+// writes Y.  No CTA waits for another, and the order of the sum depends only
+// on the sizes and the grid.
+constexpr int kSkMaxCtas = 160;   // partial-tile slots in the workspace: 2 per CTA
+constexpr int kSkMinSteps = 8;    // fewer CTAs when the pieces would be shorter
+// Stream-K is taken when its range plus this many k-steps is shorter than
+// the whole-tile schedule's longest range: the cost of the extra pieces (the
+// partial tiles' stores, the pipeline drains at the piece boundaries, the
+// fixup kernel), measured on Qwen3-8B shapes at 2048 tokens as 16-27 k-steps.
+constexpr int kSkOverheadSteps = 16;
+
 struct GemmArgs {
     float *Y;
     int *err;
+    float *part;    // partial tiles: [G][2][TN tokens][GM features] fp32
     int M, N, S;
     int ks_main;    // 128-column weight steps over K (K_pad / 128)
     int ks_ext;     // extension steps (one per 64 protected columns)
+    int KS;         // ks_main + ks_ext
     int tiles_t;    // token tiles
     int ntiles;
+    int G;          // CTAs
+    int whole;      // 1: whole tiles per CTA; 0: stream-K
+    int64_t W;      // ntiles * KS
     uint32_t w_stage;   // bytes of one compressed-weight stage
+};
+
+// stream-K: the first step of CTA c's range
+__device__ __forceinline__ int64_t sk_begin(int c, const GemmArgs &a) {
+    return static_cast<int64_t>(c) * a.W / a.G;
+}
+// stream-K: the CTA whose range holds step w (the largest c with sk_begin(c) <= w)
+__device__ __forceinline__ int sk_owner(int64_t w, const GemmArgs &a) {
+    return static_cast<int>(((w + 1) * a.G - 1) / a.W);
+}
+struct Piece {
+    int t, k0, k1;   // tile, k-steps [k0, k1)
+};
+// The pieces of CTA c, in the order it runs them.
+struct Sched {
+    int n;              // pieces
+    int64_t w0, w1;     // stream-K range
+    __device__ __forceinline__ Sched(int c, const GemmArgs &a) {
+        if (a.whole) {
+            n = c < a.ntiles ? (a.ntiles - c + a.G - 1) / a.G : 0;
+            w0 = w1 = 0;
+        } else {
+            w0 = sk_begin(c, a);
+            w1 = sk_begin(c + 1, a);
+            n = static_cast<int>((w1 - 1) / a.KS - w0 / a.KS) + 1;
+        }
+    }
+    __device__ __forceinline__ Piece at(int j, int c, const GemmArgs &a) const {
+        Piece pc;
+        if (a.whole) {
+            pc.t = c + j * a.G;
+            pc.k0 = 0;
+            pc.k1 = a.KS;
+        } else {
+            const int ta = static_cast<int>(w0 / a.KS), tb = static_cast<int>((w1 - 1) / a.KS);
+            pc.t = ta + j;
+            pc.k0 = pc.t == ta ? static_cast<int>(w0 - static_cast<int64_t>(ta) * a.KS) : 0;
+            pc.k1 = pc.t == tb ? static_cast<int>(w1 - static_cast<int64_t>(tb) * a.KS) : a.KS;
+        }
+        return pc;
+    }
 };
 
 // idesc of kind::f16: D f32, A = B = f16, both K-major, N = tn, M = GM.
@@ -140,8 +206,8 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
     const uint32_t wfull = xempty + 8 * NX, wempty = wfull + 8 * NW;
     const uint32_t afull = wempty + 8 * NW, aempty = afull + 8 * NA;
     const uint32_t dfull = aempty + 8 * NA, dempty = dfull + 8, drain = dempty + 8;
-    const int ksteps = a.ks_main + a.ks_ext;
     const int S = a.S;
+    const Sched sch(blockIdx.x, a);
     const uint32_t wbytes_main = static_cast<uint32_t>(S) * GM * 48;
 
     if (threadIdx.x == 0) {
@@ -183,9 +249,10 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
             prefetch_tmap(&tm_norms);
             int wi = 0;
             bool ok = true;
-            for (int t = blockIdx.x; ok && t < a.ntiles; t += gridDim.x) {
-                const int f0 = (t / a.tiles_t) * GM;
-                for (int ks = 0; ks < ksteps; ++ks) {
+            for (int j = 0; ok && j < sch.n; ++j) {
+                const Piece pc = sch.at(j, blockIdx.x, a);
+                const int f0 = (pc.t / a.tiles_t) * GM;
+                for (int ks = pc.k0; ks < pc.k1; ++ks) {
                     const int ws = wi % NW;
                     if (wi >= NW && !mbar_wait(wempty + 8 * ws, ((wi / NW) - 1) & 1)) { ok = false; break; }
                     if (aborted()) { ok = false; break; }
@@ -217,9 +284,10 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
             pdl_wait();
             int xi = 0;
             bool ok = true;
-            for (int t = blockIdx.x; ok && t < a.ntiles; t += gridDim.x) {
-                const int t0 = (t % a.tiles_t) * TN;
-                for (int ks = 0; ok && ks < ksteps; ++ks) {
+            for (int j = 0; ok && j < sch.n; ++j) {
+                const Piece pc = sch.at(j, blockIdx.x, a);
+                const int t0 = (pc.t % a.tiles_t) * TN;
+                for (int ks = pc.k0; ok && ks < pc.k1; ++ks) {
                     for (int hh = 0; hh < 2; ++hh) {
                         const int xs = xi % NX;
                         if (xi >= NX && !mbar_wait(xempty + 8 * xs, ((xi / NX) - 1) & 1)) { ok = false; break; }
@@ -236,12 +304,13 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
     } else if (warp == 5) {
         // --------------------------------------------------- MMA issuer
         if (lane == 0) {
-            int xi = 0, ai = 0, ti = 0;
+            int xi = 0, ai = 0;
             bool ok = true;
-            for (int t = blockIdx.x; ok && t < a.ntiles; t += gridDim.x, ++ti) {
+            for (int ti = 0; ok && ti < sch.n; ++ti) {
+                const Piece pc = sch.at(ti, blockIdx.x, a);
                 if (ti > 0 && !mbar_wait(dempty, (ti - 1) & 1)) { ok = false; break; }
                 tc_fence_after();
-                for (int ks = 0; ks < ksteps && ok; ++ks) {
+                for (int ks = pc.k0; ks < pc.k1 && ok; ++ks) {
                     const int as = ai % NA;
                     if (!mbar_wait(afull + 8 * as, (ai / NA) & 1) || aborted()) { ok = false; break; }
                     tc_fence_after();
@@ -253,7 +322,7 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
                         for (int kk = 0; kk < 4; ++kk) {
                             const uint32_t a_tmem = tmem + kColA + as * 64 + hh * 32 + kk * 8;
                             const uint64_t bdesc = smem_desc_sw128(x_ring + xs * kXStage + kk * 32);
-                            tc_mma_f16_ta(tmem + kColD, a_tmem, bdesc, kIdesc, (ks | hh | kk) != 0);
+                            tc_mma_f16_ta(tmem + kColD, a_tmem, bdesc, kIdesc, (ks != pc.k0) | hh | kk);
                         }
                         tc_commit(xempty + 8 * xs);
                         ++xi;
@@ -273,9 +342,10 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
         const int q = warp & 3, h = (warp - 8) >> 2;
         const int r = 32 * q + lane;
         int wi = 0, ai = 0;
-        for (int t = blockIdx.x; t < a.ntiles; t += gridDim.x) {
+        for (int j = 0; j < sch.n; ++j) {
+            const Piece pc = sch.at(j, blockIdx.x, a);
             bool ok = true;
-            for (int ks = 0; ks < ksteps; ++ks) {
+            for (int ks = pc.k0; ks < pc.k1; ++ks) {
                 const int ws = wi % NW, as = ai % NA;
                 if (!mbar_wait_all(wfull + 8 * ws, (wi / NW) & 1)) { ok = false; break; }
                 if (__any_sync(0xFFFFFFFFu, aborted())) { ok = false; break; }
@@ -307,28 +377,47 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
     } else if (warp < 4) {
         // ------------------------------------------------------ epilogue
         const int q = warp;
-        int ti = 0;
-        for (int t = blockIdx.x; t < a.ntiles; t += gridDim.x, ++ti) {
+        for (int ti = 0; ti < sch.n; ++ti) {
+            const Piece pc = sch.at(ti, blockIdx.x, a);
             if (!mbar_wait_all(dfull, ti & 1) || __any_sync(0xFFFFFFFFu, aborted())) {
                 if (lane == 0) fail();
                 break;
             }
             tc_fence_after();
-            const int f0 = (t / a.tiles_t) * GM, t0 = (t % a.tiles_t) * TN;
+            const int f0 = (pc.t / a.tiles_t) * GM, t0 = (pc.t % a.tiles_t) * TN;
             const int feat = f0 + 32 * q + lane;
+            const uint32_t dcol = tmem + (static_cast<uint32_t>(32 * q) << 16) + kColD;
+            if (pc.k0 == 0 && pc.k1 == a.KS) {
+                // the whole tile: Y directly
+#pragma unroll 1
+                for (int c = 0; c < TN / 32; ++c) {
+                    uint32_t v[32];
+                    tmem_ld32(dcol + c * 32, v);
+                    tmem_wait_ld();
+                    if (feat < a.N) {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) {
+                            const int tok = t0 + c * 32 + i;
+                            if (tok < a.M)
+                                a.Y[static_cast<int64_t>(tok) * a.N + feat] = __uint_as_float(v[i]) * kInvSqrt8;
+                        }
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(dempty);
+                continue;
+            }
+            // a piece of a split tile: its sum to this CTA's slot (the first
+            // piece of the range in slot 0, the last in slot 1)
+            float *mine = a.part + (static_cast<int64_t>(blockIdx.x) * 2 + (ti == 0 ? 0 : 1)) * (GM * TN);
 #pragma unroll 1
             for (int c = 0; c < TN / 32; ++c) {
                 uint32_t v[32];
-                tmem_ld32(tmem + (static_cast<uint32_t>(32 * q) << 16) + kColD + c * 32, v);
+                tmem_ld32(dcol + c * 32, v);
                 tmem_wait_ld();
-                if (feat < a.N) {
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        const int tok = t0 + c * 32 + i;
-                        if (tok < a.M)
-                            a.Y[static_cast<int64_t>(tok) * a.N + feat] = __uint_as_float(v[i]) * kInvSqrt8;
-                    }
-                }
+                for (int i = 0; i < 32; ++i) __stcg(mine + (c * 32 + i) * GM + 32 * q + lane, __uint_as_float(v[i]));
             }
             tc_fence_before();
             __syncwarp();
@@ -340,6 +429,56 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
     __syncthreads();
     tc_fence_after();
     if (warp == 5) tmem_dealloc(tmem, kTmemCols);
+}
+
+// Sum of the pieces of the tiles split by the stream-K schedule, in CTA
+// order, into Y.  Block (c - 1, j) takes the tile that holds the boundary
+// between CTAs c - 1 and c, if that boundary is the first inside it, and its
+// 32-token chunk j: 256 threads, 4 features x 4 tokens each.
+constexpr int kFixThreads = 256;
+
+__global__ void __launch_bounds__(kFixThreads) k_gemm_fixup(const GemmArgs a, int TN) {
+    // the partial tiles are written by the GEMM launched just before
+    pdl_wait();
+    const int c = blockIdx.x + 1;
+    const int64_t b = sk_begin(c, a);
+    const int t = static_cast<int>(b / a.KS);
+    const int64_t ts = static_cast<int64_t>(t) * a.KS;
+    if (b == ts || sk_begin(c - 1, a) > ts) return;   // no split here, or not the first boundary
+    const int c_lo = sk_owner(ts, a), c_hi = sk_owner(ts + a.KS - 1, a);
+    const int f0 = (t / a.tiles_t) * GM, t0 = (t % a.tiles_t) * TN;
+    const int fl = (threadIdx.x & 31) * 4, tl0 = blockIdx.y * 32 + (threadIdx.x >> 5) * 4;
+    float4 acc[4];
+#pragma unroll 1
+    for (int cc = c_lo; cc <= c_hi; ++cc) {
+        // the tile is the first of CTA cc's range (slot 0), or its last
+        const int slot = sk_begin(cc, a) / a.KS == t ? 0 : 1;
+        const float *src = a.part + (static_cast<int64_t>(cc) * 2 + slot) * (GM * TN);
+        float4 v[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) v[i] = __ldcg(reinterpret_cast<const float4 *>(src + (tl0 + i) * GM + fl));
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            if (cc == c_lo) {
+                acc[i] = v[i];
+            } else {
+                acc[i].x += v[i].x;
+                acc[i].y += v[i].y;
+                acc[i].z += v[i].z;
+                acc[i].w += v[i].w;
+            }
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int tok = t0 + tl0 + i;
+        if (tok >= a.M) break;
+        float *yr = a.Y + static_cast<int64_t>(tok) * a.N + f0 + fl;
+        const float o[4] = {acc[i].x, acc[i].y, acc[i].z, acc[i].w};
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+            if (f0 + fl + u < a.N) yr[u] = o[u] * kInvSqrt8;
+    }
 }
 
 // Activation pre-pass: X16[m][k] = fp16(x[m][k]) for k < K (0 for
@@ -436,6 +575,28 @@ int k_ext_of(int K, int p) { return k_pad_of(K) + 2 * p_ext_of(p); }
 // small prefills go through the decode kernels instead.
 bool tensor_path(const bisco_layer &L, int M) { return M > 64 && L.k_in % 128 == 0; }
 
+// Token tile: 256 (the decode of a weight step feeds the most MMA work);
+// 128 when M fits in it.  The stream-K split keeps every SM busy either way.
+int tile_tokens(int M) { return M <= 128 ? 128 : GN; }
+
+size_t round256(size_t b) { return (b + 255) / 256 * 256; }
+
+// Workspace: [X16: M x K_ext fp16][partial tiles: kSkMaxCtas x 2 x TN x GM
+// fp32], each part rounded up to 256 bytes.
+struct GemmWs {
+    size_t x16, part, total;
+    int ntiles;
+};
+GemmWs gemm_ws(const bisco_layer &L, int M) {
+    GemmWs w;
+    const int TN = tile_tokens(M);
+    w.ntiles = ((M + TN - 1) / TN) * ((L.n_out + GM - 1) / GM);
+    w.x16 = 0;
+    w.part = round256(static_cast<size_t>(M) * k_ext_of(L.k_in, L.n_protected) * 2);
+    w.total = w.part + static_cast<size_t>(kSkMaxCtas) * 2 * GM * TN * 4;
+    return w;
+}
+
 bisco_status gemm_via_gemv(const bisco_layer &L, const uint16_t *X, int M, float *Y, int *err,
                            cudaStream_t stream) {
     for (int m0 = 0; m0 < M; m0 += 16) {
@@ -483,7 +644,7 @@ bisco_status launch_gemm_t(const CUtensorMap &mx, const CUtensorMap &mc, const C
 
 size_t gemm_workspace_bytes(const bisco_layer &L, int M) {
     if (!tensor_path(L, M)) return 0;
-    return static_cast<size_t>(M) * k_ext_of(L.k_in, L.n_protected) * 2;
+    return gemm_ws(L, M).total;
 }
 
 bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *Y,
@@ -491,8 +652,10 @@ bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *
     if (!tensor_path(L, M)) return gemm_via_gemv(L, X, M, Y, err, stream);
     const int N = L.n_out, K = L.k_in, S = L.stages, p = L.n_protected;
     const int K_pad = k_pad_of(K), K_ext = k_ext_of(K, p);
-    if (ws_bytes < gemm_workspace_bytes(L, M)) return BISCO_ERR_INVALID_ARG;
-    uint16_t *X16 = static_cast<uint16_t *>(workspace);
+    const GemmWs wl = gemm_ws(L, M);
+    if (ws_bytes < wl.total) return BISCO_ERR_INVALID_ARG;
+    unsigned char *wsb = static_cast<unsigned char *>(workspace);
+    uint16_t *X16 = reinterpret_cast<uint16_t *>(wsb + wl.x16);
 
     const size_t prep_smem = static_cast<size_t>(K_pad / 32) * 4;
     if (prep_smem > 48 * 1024) {
@@ -512,12 +675,7 @@ bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *
         X, M, K, K_pad, K_ext, p, L.prot_idx, L.q8_scale, X16, err);
     if (cudaGetLastError() != cudaSuccess) return BISCO_ERR_CUDA;
 
-    // token tile: 256, or 128 when 256-token tiles would leave SMs idle
-    // (e.g. k_proj / v_proj: 8 feature tiles); the decode per k-step is the
-    // same, the MMA work halves
-    const int sms = num_sms();
-    const int feat_tiles = (N + GM - 1) / GM;
-    const int TN = (static_cast<long>((M + GN - 1) / GN) * feat_tiles < sms && M > 128) ? 128 : GN;
+    const int TN = tile_tokens(M);
     CUtensorMap mx, mc, mn, mq;
     {
         const uint64_t dims[2] = {static_cast<uint64_t>(K_ext), static_cast<uint64_t>(M)};
@@ -554,20 +712,45 @@ bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *
     GemmArgs a = {};
     a.Y = Y;
     a.err = err;
+    a.part = reinterpret_cast<float *>(wsb + wl.part);
     a.M = M;
     a.N = N;
     a.S = S;
     a.ks_main = K_pad / GK;
     a.ks_ext = p_ext_of(p) / 64;
+    a.KS = a.ks_main + a.ks_ext;
     a.tiles_t = (M + TN - 1) / TN;
-    a.ntiles = a.tiles_t * feat_tiles;
+    a.ntiles = wl.ntiles;
+    a.W = static_cast<int64_t>(a.ntiles) * a.KS;
+    const int sms = num_sms() < kSkMaxCtas ? num_sms() : kSkMaxCtas;
+    int64_t g = a.W / kSkMinSteps;
+    if (g > sms) g = sms;
+    if (g < 1) g = 1;
+    const int g_whole = a.ntiles < sms ? a.ntiles : sms;
+    const int64_t whole_steps = static_cast<int64_t>((a.ntiles + g_whole - 1) / g_whole) * a.KS;
+    a.whole = whole_steps <= a.W / g + kSkOverheadSteps ? 1 : 0;
+    a.G = a.whole ? g_whole : static_cast<int>(g);
     a.w_stage = static_cast<uint32_t>(S * GM * 48 > GM * 64 ? S * GM * 48 : GM * 64);
-    const int grid = a.ntiles < sms ? a.ntiles : sms;
+    const int grid = a.G;
     // 256 tokens: S = 1: 6 x 32 KB + 3 x 8 KB; S = 2, 3: 5 x 32 KB + 3 x 12/18 KB;
     // 128 tokens: 8 x 16 KB + 3 x 8/12/18 KB (all <= 227 KB)
-    if (TN == 128) return launch_gemm_t<8, 3, 128>(mx, mc, mn, mq, a, grid, stream);
-    if (S == 1) return launch_gemm_t<6, 3, GN>(mx, mc, mn, mq, a, grid, stream);
-    return launch_gemm_t<5, 3, GN>(mx, mc, mn, mq, a, grid, stream);
+    bisco_status st;
+    if (TN == 128) st = launch_gemm_t<8, 3, 128>(mx, mc, mn, mq, a, grid, stream);
+    else if (S == 1) st = launch_gemm_t<6, 3, GN>(mx, mc, mn, mq, a, grid, stream);
+    else st = launch_gemm_t<5, 3, GN>(mx, mc, mn, mq, a, grid, stream);
+    if (st != BISCO_OK || a.whole || a.G < 2) return st;
+    // the split tiles, summed once the GEMM is done (programmatic dependent
+    // launch: its set-up overlaps the GEMM's last CTAs)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(a.G - 1, TN / 32, 1);
+    cfg.blockDim = dim3(kFixThreads, 1, 1);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_gemm_fixup, a, TN) == cudaSuccess ? BISCO_OK : BISCO_ERR_CUDA;
 }
 
 }  // namespace bisco

@@ -35,7 +35,7 @@ def test_header_declarations_are_exported(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert bisco.bisco_abi_version() == 106
+    assert bisco.bisco_abi_version() == 107
     for code in range(6):
         assert bisco.status_string(code)
     assert bisco.status_string(99) == "unknown status"
@@ -112,9 +112,16 @@ def test_call_argument_validation(lib):
     assert lib.bisco_gemm_workspace_bytes(ctypes.byref(_fake_layer(k_in=12)), 128) == 0
     assert lib.bisco_gemm_workspace_bytes(ctypes.byref(L), -1) == 0
     assert lib.bisco_gemm_workspace_bytes(ctypes.byref(L), 64) == 0        # decode-kernel path
-    # tensor-core path: fp16 activations plus hi/lo protected columns
+    # tensor-core path: fp16 activations plus hi/lo protected columns (rounded
+    # up to 256 bytes), then the partial tiles of the stream-K split (160 CTAs
+    # x 2 slots x TN tokens x 128 features, fp32)
     L2 = _fake_layer(k_in=4096, n_protected=41)
-    assert lib.bisco_gemm_workspace_bytes(ctypes.byref(L2), 2048) == 2048 * (4096 + 128) * 2
+    assert lib.bisco_gemm_workspace_bytes(ctypes.byref(L2), 2048) == \
+        2048 * (4096 + 128) * 2 + 160 * 2 * 256 * 128 * 4
+    assert lib.bisco_gemm_workspace_bytes(ctypes.byref(L2), 100) == \
+        100 * (4096 + 128) * 2 + 160 * 2 * 128 * 128 * 4
+    assert lib.bisco_gemm_workspace_bytes(ctypes.byref(_fake_layer(k_in=128, n_protected=1)), 65) == \
+        (65 * 256 * 2 + 255) // 256 * 256 + 160 * 2 * 128 * 128 * 4
     assert lib.bisco_gemm(ctypes.byref(L2), x, 2048, y, None, 0, None) == bisco.ERR_INVALID_ARG
 
 

@@ -96,3 +96,24 @@ def test_gemm_equals_gemv(env):
     Y, L = run_gemm(env, Lref, X)
     y = bisco.bisco_gemv(L, to_dev(X, dev)).cpu().numpy()
     assert max_rel_rows(Y, y) <= 1e-4
+
+
+@pytest.mark.parametrize("N,K,S,p,M", [
+    (128, 4096, 2, 41, 200),        # one tile of 33 k-steps, split over 4 CTAs
+    (256, 4096, 3, 41, 100),        # M <= 128: 128-token tiles, 2 tiles over 8 CTAs
+    (1024, 4096, 2, 41, 2048),      # k_proj: 64 tiles over every SM, 2-3 pieces a tile
+])
+def test_gemm_split_tiles(env, N, K, S, p, M):
+    """Tiles split between CTAs by the stream-K schedule, the partial sums
+    added by the warp that brings a tile's last piece: the outputs against
+    the oracle (every token up to 200, 5 tokens of every 256 beyond), and a
+    second call equal bit for bit (the pieces are summed in CTA order)."""
+    W = synth.layer_weights(N, K, seed=N + 7 * K)
+    X = synth.activations(M, K, seed=M + 3)
+    Lref = oracle.encode(W, S=S, p=p)
+    Y, _ = run_gemm(env, Lref, X)
+    Y2, _ = run_gemm(env, Lref, X)
+    assert np.array_equal(Y, Y2)
+    toks = np.arange(M) if M <= 200 else rows_per_tile(M, 256, per=5, seed=M)
+    ref = oracle.gemv(Lref, X[toks])
+    assert_parity(Y[toks], ref, gemm_tight(M, K), f"{N}x{K} M={M}")
