@@ -65,6 +65,8 @@ def parse():
     ap.add_argument("--shape-mb", type=float, default=500.0,
                     help="--mode shapes: MB of distinct coded layers per shape (> L2)")
     ap.add_argument("--prefill-tokens", type=int, default=2048)
+    ap.add_argument("--prefill-proj", default=",".join(ATTN),
+                    help="--mode prefill: comma-separated Qwen3-8B projections, one layer of each")
     return ap.parse_args()
 
 
@@ -606,29 +608,35 @@ def run_prefill_stack(args, stack, stream, dev):
             "roofline": {"bound": "tensor", "achieved": tf, "peak": burst, "unit": "TFLOP/s",
                          "frac": tf / burst, "frac_of_sustained": tf / sustained,
                          "peak_source": "%s bf16_tflops (MEASURED_PEAKS.json; fp16 rate = bf16)" % kind,
-                         "kernels": "k_gemm_prep + k_gemm per projection"},
+                         "kernels": "k_gemm_prep + k_gemm per projection, + k_gemm_fixup where "
+                                    "the call splits tiles (stream-K)"},
             "dtype": "f16 x f16 -> f32"}
 
 
 # ---------------------------------------------------------------- prefill
 
 def run_prefill(args, local_rank):
-    """Prefill (bisco_gemm on the tensor cores): the four attention
-    projections of one layer at M tokens, a CUDA graph of the four calls
-    (fp16 pre-pass + tcgen05 kernel each), CUDA events over `steps` replays.
-    TFLOP/s on the algorithmic 2*M*N*K."""
+    """Prefill (bisco_gemm on the tensor cores): one layer of each projection
+    in --prefill-proj (default the four attention projections) at M tokens, a
+    CUDA graph of the calls (fp16 pre-pass + tcgen05 kernel each, plus the
+    fixup kernel where a call splits tiles), CUDA events over `steps`
+    replays.  TFLOP/s on the algorithmic 2*M*N*K."""
     import torch
     from paper_2607_08643_gb300 import bisco, synth
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
     M = args.prefill_tokens
+    names = [n for n in args.prefill_proj.split(",") if n]
+    if not names or any(n not in synth.QWEN3_8B_SHAPES for n in names):
+        raise SystemExit("--prefill-proj: names from %s" % ",".join(synth.QWEN3_8B_SHAPES))
     layers = []
-    for j, name in enumerate(ATTN):
+    for j, name in enumerate(names):
         N, K = synth.QWEN3_8B_SHAPES[name]
         W = synth.layer_weights_torch(N, K, seed=500 + j, device=dev)
         layers.append((name, bisco.bisco_encode(W, S_STAGES, synth.protected_count(K, RHO_PCT))))
         del W
-    X = torch.randn((M, 4096), device=dev).to(torch.bfloat16).view(torch.int16)
+    Xk = {K: torch.randn((M, K), device=dev).to(torch.bfloat16).view(torch.int16)
+          for K in sorted({L.K for _, L in layers})}
     Ys = [torch.empty((M, L.N), device=dev) for _, L in layers]
     ws = torch.empty(max(bisco.bisco_gemm_workspace_bytes(L, M) for _, L in layers),
                      dtype=torch.uint8, device=dev)
@@ -636,12 +644,12 @@ def run_prefill(args, local_rank):
     stream = torch.cuda.Stream(device=dev)
     with torch.cuda.stream(stream):
         for (_, L), Y in zip(layers, Ys):
-            bisco.bisco_gemm(L, X, Y=Y, workspace=ws, stream=stream)
+            bisco.bisco_gemm(L, Xk[L.K], Y=Y, workspace=ws, stream=stream)
         torch.cuda.synchronize()
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
             for (_, L), Y in zip(layers, Ys):
-                bisco.bisco_gemm(L, X, Y=Y, workspace=ws, stream=stream)
+                bisco.bisco_gemm(L, Xk[L.K], Y=Y, workspace=ws, stream=stream)
     torch.cuda.synchronize()
     for _ in range(max(args.warmup, 3)):
         g.replay()
@@ -661,14 +669,15 @@ def run_prefill(args, local_rank):
     tf = flops / (ms * 1e-3) / 1e12
     burst, sustained, kind = tensor_peaks()
     return {"metric": "prefill GEMM TFLOP/s (2*M*N*K, decoded weight never written)",
-            "workload": "Qwen3-8B q/k/v/o projections, %d tokens, S=%d, %d%% protected"
-                        % (M, S_STAGES, RHO_PCT),
+            "workload": "Qwen3-8B %s, one layer each, %d tokens, S=%d, %d%% protected"
+                        % ("/".join(names), M, S_STAGES, RHO_PCT),
             "value": tf, "unit": "TFLOP/s", "ms_per_step": ms, "tokens_per_s": M / (ms * 1e-3),
             "roofline": {"bound": "tensor", "achieved": tf, "peak": burst, "unit": "TFLOP/s",
                          "frac": tf / burst, "frac_of_sustained": tf / sustained,
                          "peak_source": "%s bf16_tflops (MEASURED_PEAKS.json; fp16 rate = bf16)" % kind,
-                         "kernels": "k_gemm_prep + k_gemm per projection"},
-            "dtype": "f16 x f16 -> f32", "launches_per_step": 2 * len(layers)}
+                         "kernels": "k_gemm_prep + k_gemm per projection, + k_gemm_fixup where "
+                                    "the call splits tiles (stream-K)"},
+            "dtype": "f16 x f16 -> f32"}
 
 
 # ------------------------------------------------------------------ dense
