@@ -598,6 +598,20 @@ def run_prefill_stack(args, stack, stream, dev):
         raise RuntimeError("device error in prefill")
     flops = sum(2.0 * M * L.N * L.K for row in rows for L in row)
     tf = flops / (ms * 1e-3) / 1e12
+    # each projection alone: a graph of its 4 calls
+    per_proj = {}
+    for j, name in enumerate(STACK):
+        def one(j=j):
+            for row, ys in zip(rows, Ys):
+                bisco.bisco_gemm(row[j], X[row[j].K], Y=ys[j], workspace=ws, stream=stream)
+        gj = graph_of(torch, stream, one)
+        msj = time_graph(torch, stream, gj, max(3, min(args.steps, 10)), 3)
+        fj = sum(2.0 * M * row[j].N * row[j].K for row in rows)
+        per_proj[name] = {"us_per_call": round(msj * 1e3 / len(rows), 2),
+                          "tflops": round(fj / (msj * 1e-3) / 1e12, 1)}
+        del gj
+    if bisco.bisco_get_device_error(stream) != bisco.OK:
+        raise RuntimeError("device error in prefill")
     burst, sustained, kind = tensor_peaks()
     del g, X, Ys, ws
     torch.cuda.empty_cache()
@@ -610,6 +624,7 @@ def run_prefill_stack(args, stack, stream, dev):
                          "peak_source": "%s bf16_tflops (MEASURED_PEAKS.json; fp16 rate = bf16)" % kind,
                          "kernels": "k_gemm_prep + k_gemm per projection, + k_gemm_fixup where "
                                     "the call splits tiles (stream-K)"},
+            "per_projection": per_proj,
             "dtype": "f16 x f16 -> f32"}
 
 

@@ -31,6 +31,7 @@
 
 #include "bisco_dev.cuh"
 #include "bisco_host.h"
+#include "gemm_sched.cuh"
 
 namespace bisco {
 namespace {
@@ -52,79 +53,16 @@ constexpr uint32_t x_stage_bytes(int tn) { return static_cast<uint32_t>(tn) * 12
 constexpr float kInvSqrt8 = 0.35355339059327373f;
 constexpr float kSqrt8 = 2.8284271247461903f;
 
-// Work split over the persistent CTAs.  Whole tiles: CTA c takes tiles c,
-// c + G, c + 2G, ...  Stream-K: the tiles' k-steps are laid end to end
-// (tile t holds steps [t*KS, (t+1)*KS)) and CTA c takes the steps
-// [c*W/G, (c+1)*W/G), so every CTA has the same work.  A tile covered by
-// one CTA is written to Y directly; a tile
-// split between CTAs has each piece's fp32 sum written to the workspace (the
-// first piece of a CTA's range in its slot 0, the last in slot 1), and
-// k_gemm_fixup, launched after the GEMM, adds the pieces in CTA order and
-// writes Y.  No CTA waits for another, and the order of the sum depends only
-// on the sizes and the grid.
-constexpr int kSkMaxCtas = 160;   // partial-tile slots in the workspace: 2 per CTA
-constexpr int kSkMinSteps = 8;    // fewer CTAs when the pieces would be shorter
-// Stream-K is taken when its range plus this many k-steps is shorter than
-// the whole-tile schedule's longest range: the cost of the extra pieces (the
-// partial tiles' stores, the pipeline drains at the piece boundaries, the
-// fixup kernel), measured on Qwen3-8B shapes at 2048 tokens as 16-27 k-steps.
-constexpr int kSkOverheadSteps = 16;
-
 struct GemmArgs {
     float *Y;
     int *err;
-    float *part;    // partial tiles: [G][2][TN tokens][GM features] fp32
+    float *part;    // partial tiles of the stream-K split: [G][2][TN tokens][GM features] fp32
     int M, N, S;
     int ks_main;    // 128-column weight steps over K (K_pad / 128)
     int ks_ext;     // extension steps (one per 64 protected columns)
-    int KS;         // ks_main + ks_ext
     int tiles_t;    // token tiles
-    int ntiles;
-    int G;          // CTAs
-    int whole;      // 1: whole tiles per CTA; 0: stream-K
-    int64_t W;      // ntiles * KS
+    SkPlan sk;      // the split of the tiles' k-steps over the CTAs (gemm_sched.cuh)
     uint32_t w_stage;   // bytes of one compressed-weight stage
-};
-
-// stream-K: the first step of CTA c's range
-__device__ __forceinline__ int64_t sk_begin(int c, const GemmArgs &a) {
-    return static_cast<int64_t>(c) * a.W / a.G;
-}
-// stream-K: the CTA whose range holds step w (the largest c with sk_begin(c) <= w)
-__device__ __forceinline__ int sk_owner(int64_t w, const GemmArgs &a) {
-    return static_cast<int>(((w + 1) * a.G - 1) / a.W);
-}
-struct Piece {
-    int t, k0, k1;   // tile, k-steps [k0, k1)
-};
-// The pieces of CTA c, in the order it runs them.
-struct Sched {
-    int n;              // pieces
-    int64_t w0, w1;     // stream-K range
-    __device__ __forceinline__ Sched(int c, const GemmArgs &a) {
-        if (a.whole) {
-            n = c < a.ntiles ? (a.ntiles - c + a.G - 1) / a.G : 0;
-            w0 = w1 = 0;
-        } else {
-            w0 = sk_begin(c, a);
-            w1 = sk_begin(c + 1, a);
-            n = static_cast<int>((w1 - 1) / a.KS - w0 / a.KS) + 1;
-        }
-    }
-    __device__ __forceinline__ Piece at(int j, int c, const GemmArgs &a) const {
-        Piece pc;
-        if (a.whole) {
-            pc.t = c + j * a.G;
-            pc.k0 = 0;
-            pc.k1 = a.KS;
-        } else {
-            const int ta = static_cast<int>(w0 / a.KS), tb = static_cast<int>((w1 - 1) / a.KS);
-            pc.t = ta + j;
-            pc.k0 = pc.t == ta ? static_cast<int>(w0 - static_cast<int64_t>(ta) * a.KS) : 0;
-            pc.k1 = pc.t == tb ? static_cast<int>(w1 - static_cast<int64_t>(tb) * a.KS) : a.KS;
-        }
-        return pc;
-    }
 };
 
 // idesc of kind::f16: D f32, A = B = f16, both K-major, N = tn, M = GM.
@@ -207,7 +145,7 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
     const uint32_t afull = wempty + 8 * NW, aempty = afull + 8 * NA;
     const uint32_t dfull = aempty + 8 * NA, dempty = dfull + 8, drain = dempty + 8;
     const int S = a.S;
-    const Sched sch(blockIdx.x, a);
+    const SkSched sch(blockIdx.x, a.sk);
     const uint32_t wbytes_main = static_cast<uint32_t>(S) * GM * 48;
 
     if (threadIdx.x == 0) {
@@ -250,7 +188,7 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
             int wi = 0;
             bool ok = true;
             for (int j = 0; ok && j < sch.n; ++j) {
-                const Piece pc = sch.at(j, blockIdx.x, a);
+                const SkPiece pc = sch.at(j, blockIdx.x, a.sk);
                 const int f0 = (pc.t / a.tiles_t) * GM;
                 for (int ks = pc.k0; ks < pc.k1; ++ks) {
                     const int ws = wi % NW;
@@ -285,7 +223,7 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
             int xi = 0;
             bool ok = true;
             for (int j = 0; ok && j < sch.n; ++j) {
-                const Piece pc = sch.at(j, blockIdx.x, a);
+                const SkPiece pc = sch.at(j, blockIdx.x, a.sk);
                 const int t0 = (pc.t % a.tiles_t) * TN;
                 for (int ks = pc.k0; ok && ks < pc.k1; ++ks) {
                     for (int hh = 0; hh < 2; ++hh) {
@@ -307,7 +245,7 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
             int xi = 0, ai = 0;
             bool ok = true;
             for (int ti = 0; ok && ti < sch.n; ++ti) {
-                const Piece pc = sch.at(ti, blockIdx.x, a);
+                const SkPiece pc = sch.at(ti, blockIdx.x, a.sk);
                 if (ti > 0 && !mbar_wait(dempty, (ti - 1) & 1)) { ok = false; break; }
                 tc_fence_after();
                 for (int ks = pc.k0; ks < pc.k1 && ok; ++ks) {
@@ -343,7 +281,7 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
         const int r = 32 * q + lane;
         int wi = 0, ai = 0;
         for (int j = 0; j < sch.n; ++j) {
-            const Piece pc = sch.at(j, blockIdx.x, a);
+            const SkPiece pc = sch.at(j, blockIdx.x, a.sk);
             bool ok = true;
             for (int ks = pc.k0; ks < pc.k1; ++ks) {
                 const int ws = wi % NW, as = ai % NA;
@@ -378,7 +316,7 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
         // ------------------------------------------------------ epilogue
         const int q = warp;
         for (int ti = 0; ti < sch.n; ++ti) {
-            const Piece pc = sch.at(ti, blockIdx.x, a);
+            const SkPiece pc = sch.at(ti, blockIdx.x, a.sk);
             if (!mbar_wait_all(dfull, ti & 1) || __any_sync(0xFFFFFFFFu, aborted())) {
                 if (lane == 0) fail();
                 break;
@@ -387,7 +325,7 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
             const int f0 = (pc.t / a.tiles_t) * GM, t0 = (pc.t % a.tiles_t) * TN;
             const int feat = f0 + 32 * q + lane;
             const uint32_t dcol = tmem + (static_cast<uint32_t>(32 * q) << 16) + kColD;
-            if (pc.k0 == 0 && pc.k1 == a.KS) {
+            if (pc.k0 == 0 && pc.k1 == a.sk.KS) {
                 // the whole tile: Y directly
 #pragma unroll 1
                 for (int c = 0; c < TN / 32; ++c) {
@@ -408,8 +346,8 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
                 if (lane == 0) mbar_arrive(dempty);
                 continue;
             }
-            // a piece of a split tile: its sum to this CTA's slot (the first
-            // piece of the range in slot 0, the last in slot 1)
+            // a piece of a split tile: its sum to this CTA's slot (sk_slot: the
+            // first piece of the range in slot 0, a later one in slot 1)
             float *mine = a.part + (static_cast<int64_t>(blockIdx.x) * 2 + (ti == 0 ? 0 : 1)) * (GM * TN);
 #pragma unroll 1
             for (int c = 0; c < TN / 32; ++c) {
@@ -441,19 +379,16 @@ __global__ void __launch_bounds__(kFixThreads) k_gemm_fixup(const GemmArgs a, in
     // the partial tiles are written by the GEMM launched just before
     pdl_wait();
     const int c = blockIdx.x + 1;
-    const int64_t b = sk_begin(c, a);
-    const int t = static_cast<int>(b / a.KS);
-    const int64_t ts = static_cast<int64_t>(t) * a.KS;
-    if (b == ts || sk_begin(c - 1, a) > ts) return;   // no split here, or not the first boundary
-    const int c_lo = sk_owner(ts, a), c_hi = sk_owner(ts + a.KS - 1, a);
+    const int t = sk_fixup_tile(c, a.sk);
+    if (t < 0) return;   // no split here, or not the first boundary inside the tile
+    const int64_t ts = static_cast<int64_t>(t) * a.sk.KS;
+    const int c_lo = sk_owner(ts, a.sk), c_hi = sk_owner(ts + a.sk.KS - 1, a.sk);
     const int f0 = (t / a.tiles_t) * GM, t0 = (t % a.tiles_t) * TN;
     const int fl = (threadIdx.x & 31) * 4, tl0 = blockIdx.y * 32 + (threadIdx.x >> 5) * 4;
     float4 acc[4];
 #pragma unroll 1
     for (int cc = c_lo; cc <= c_hi; ++cc) {
-        // the tile is the first of CTA cc's range (slot 0), or its last
-        const int slot = sk_begin(cc, a) / a.KS == t ? 0 : 1;
-        const float *src = a.part + (static_cast<int64_t>(cc) * 2 + slot) * (GM * TN);
+        const float *src = a.part + (static_cast<int64_t>(cc) * 2 + sk_slot(cc, t, a.sk)) * (GM * TN);
         float4 v[4];
 #pragma unroll
         for (int i = 0; i < 4; ++i) v[i] = __ldcg(reinterpret_cast<const float4 *>(src + (tl0 + i) * GM + fl));
@@ -718,31 +653,21 @@ bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *
     a.S = S;
     a.ks_main = K_pad / GK;
     a.ks_ext = p_ext_of(p) / 64;
-    a.KS = a.ks_main + a.ks_ext;
     a.tiles_t = (M + TN - 1) / TN;
-    a.ntiles = wl.ntiles;
-    a.W = static_cast<int64_t>(a.ntiles) * a.KS;
-    const int sms = num_sms() < kSkMaxCtas ? num_sms() : kSkMaxCtas;
-    int64_t g = a.W / kSkMinSteps;
-    if (g > sms) g = sms;
-    if (g < 1) g = 1;
-    const int g_whole = a.ntiles < sms ? a.ntiles : sms;
-    const int64_t whole_steps = static_cast<int64_t>((a.ntiles + g_whole - 1) / g_whole) * a.KS;
-    a.whole = whole_steps <= a.W / g + kSkOverheadSteps ? 1 : 0;
-    a.G = a.whole ? g_whole : static_cast<int>(g);
+    a.sk = sk_plan(wl.ntiles, a.ks_main + a.ks_ext, num_sms());
     a.w_stage = static_cast<uint32_t>(S * GM * 48 > GM * 64 ? S * GM * 48 : GM * 64);
-    const int grid = a.G;
+    const int grid = a.sk.G;
     // 256 tokens: S = 1: 6 x 32 KB + 3 x 8 KB; S = 2, 3: 5 x 32 KB + 3 x 12/18 KB;
     // 128 tokens: 8 x 16 KB + 3 x 8/12/18 KB (all <= 227 KB)
     bisco_status st;
     if (TN == 128) st = launch_gemm_t<8, 3, 128>(mx, mc, mn, mq, a, grid, stream);
     else if (S == 1) st = launch_gemm_t<6, 3, GN>(mx, mc, mn, mq, a, grid, stream);
     else st = launch_gemm_t<5, 3, GN>(mx, mc, mn, mq, a, grid, stream);
-    if (st != BISCO_OK || a.whole || a.G < 2) return st;
+    if (st != BISCO_OK || a.sk.whole || a.sk.G < 2) return st;
     // the split tiles, summed once the GEMM is done (programmatic dependent
     // launch: its set-up overlaps the GEMM's last CTAs)
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(a.G - 1, TN / 32, 1);
+    cfg.gridDim = dim3(a.sk.G - 1, TN / 32, 1);
     cfg.blockDim = dim3(kFixThreads, 1, 1);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
