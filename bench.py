@@ -470,7 +470,7 @@ def run_sweeps(args, stack, stream, dev):
         ms = time_graph(torch, stream, g, steps, warm)
         cross.append({"tokens": M, "ms_per_step": ms, "tokens_per_s": M / (ms * 1e-3),
                       "gbs": total / (ms * 1e-3) / 1e9,
-                      "path": "tcgen05 GEMM" if M > 64 else "decode kernels"})
+                      "path": "tcgen05 GEMM" if M > 16 else "decode kernels"})
         del g, io, ws
     if bisco.bisco_get_device_error(stream) != bisco.OK:
         raise RuntimeError("device error in the sweeps")

@@ -314,7 +314,7 @@ bisco_status bisco_gemv_lora(const bisco_layer *L, const bisco_lora *lora, const
 /*
  * Prefill matrix product Y[m][i] = sum_j What[i][j] * X[m][j] for any M >= 0
  * (Sec. III-G Eq. 12 with Eq. 10), the same quantity as bisco_gemv.  For
- * M > 64 and K % 128 == 0 it runs on the tcgen05 tensor cores: the decoded
+ * M > 16 and K % 128 == 0 it runs on the tcgen05 tensor cores: the decoded
  * weight (fp16, the S stages summed in fp16 -- one rounding of relative
  * size <= 2^-11 per weight for S >= 2) against fp16 activations, fp32
  * accumulation; the protected columns use the int8 values exactly.  Smaller

@@ -506,9 +506,11 @@ int k_pad_of(int K) { return (K + GK - 1) / GK * GK; }
 int p_ext_of(int p) { return (p + 63) / 64 * 64; }
 int k_ext_of(int K, int p) { return k_pad_of(K) + 2 * p_ext_of(p); }
 
-// The tcgen05 path needs TMA-legal strides and enough tokens to fill tiles;
-// small prefills go through the decode kernels instead.
-bool tensor_path(const bisco_layer &L, int M) { return M > 64 && L.k_in % 128 == 0; }
+// The tcgen05 path needs TMA-legal strides.  Up to 16 tokens the batch-16
+// decode kernels are faster (one pass over the weights that feeds every
+// token); from 17 on they need a second pass, while the stream-K split keeps
+// every SM busy on the tensor cores even with one token tile.
+bool tensor_path(const bisco_layer &L, int M) { return M > 16 && L.k_in % 128 == 0; }
 
 // Token tile: 256 (the decode of a weight step feeds the most MMA work);
 // 128 when M fits in it.  The stream-K split keeps every SM busy either way.

@@ -40,9 +40,9 @@ def gemv_tight(B, tables=True):
 
 
 def gemm_tight(M, K):
-    """The bound of bisco_gemm: the tensor-core path for M > 64 and
+    """The bound of bisco_gemm: the tensor-core path for M > 16 and
     K % 128 == 0, otherwise the decode kernels of bisco_gemv."""
-    return TIGHT_GEMM if (M > 64 and K % 128 == 0) else gemv_tight(M)
+    return TIGHT_GEMM if (M > 16 and K % 128 == 0) else gemv_tight(M)
 
 
 def max_rel_rows(y, ref):

@@ -111,7 +111,9 @@ def test_call_argument_validation(lib):
     assert lib.bisco_encode_workspace_bytes(0, 64) == 0
     assert lib.bisco_gemm_workspace_bytes(ctypes.byref(_fake_layer(k_in=12)), 128) == 0
     assert lib.bisco_gemm_workspace_bytes(ctypes.byref(L), -1) == 0
-    assert lib.bisco_gemm_workspace_bytes(ctypes.byref(L), 64) == 0        # decode-kernel path
+    assert lib.bisco_gemm_workspace_bytes(ctypes.byref(L), 16) == 0        # decode-kernel path
+    assert lib.bisco_gemm_workspace_bytes(ctypes.byref(L), 17) == \
+        17 * (256 + 128) * 2 + 160 * 2 * 128 * 128 * 4                    # tensor cores from 17
     # tensor-core path: fp16 activations plus hi/lo protected columns (rounded
     # up to 256 bytes), then the partial tiles of the stream-K split (160 CTAs
     # x 2 slots x TN tokens x 128 features, fp32)

@@ -33,7 +33,10 @@ def run_gemm(env, Lref, X):
 
 @pytest.mark.parametrize("N,K,S,p,M", [
     (1024, 1024, 2, 11, 2048),      # single layer 1024 x 1024, 2048 tokens (tensor cores)
-    (1024, 1024, 2, 11, 37),        # small prefill: decode kernels
+    (1024, 1024, 2, 11, 37),        # 37 tokens: tensor cores, one 128-token tile
+    (512, 1024, 2, 11, 16),         # 16 tokens: decode kernels
+    (384, 2048, 3, 41, 17),         # 17 tokens: tensor cores
+    (1024, 4096, 2, 41, 64),        # 64 tokens: tensor cores, stream-K
     (200, 1536, 3, 20, 130),        # ragged N and M, three stages
     (128, 512, 1, 0, 100),          # S = 1, no protected columns
     (384, 2048, 2, 130, 300),       # three 64-column protected blocks, two token tiles
