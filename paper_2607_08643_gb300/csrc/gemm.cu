@@ -171,6 +171,10 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    // the kernel launched after this one (the fixup, or the next call's
+    // pre-pass) may take its place on the SMs now and wait there for this
+    // grid's completion
+    pdl_launch_dependents();
     const uint32_t tmem = s_tmem;
     auto aborted = [&]() { return *reinterpret_cast<volatile int *>(&s_abort) != 0; };
     auto fail = [&]() {
@@ -376,7 +380,9 @@ k_gemm(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtenso
 constexpr int kFixThreads = 256;
 
 __global__ void __launch_bounds__(kFixThreads) k_gemm_fixup(const GemmArgs a, int TN) {
-    // the partial tiles are written by the GEMM launched just before
+    // the partial tiles are written by the GEMM launched just before; the
+    // next kernel may launch meanwhile
+    pdl_launch_dependents();
     pdl_wait();
     const int c = blockIdx.x + 1;
     const int t = sk_fixup_tile(c, a.sk);
@@ -432,6 +438,10 @@ __global__ void __launch_bounds__(kPrepThreads) k_gemm_prep(const uint16_t *__re
     // the GEMM launched after this kernel may set itself up meanwhile; it
     // waits for this grid's completion before it reads X16
     pdl_launch_dependents();
+    // launched as a programmatic dependent of the kernel before it (which
+    // may write X, or still read the X16 of an earlier call): nothing is
+    // read or written before that kernel has completed
+    pdl_wait();
     const int groups = K_ext / 8;
     const int64_t njobs = static_cast<int64_t>(M) * groups;
     const int64_t base = static_cast<int64_t>(blockIdx.x) * kPrepThreads * kPrepJobs + threadIdx.x;
@@ -608,9 +618,21 @@ bisco_status launch_gemm(const bisco_layer &L, const uint16_t *X, int M, float *
     }
     const int64_t prep_jobs = static_cast<int64_t>(M) * (K_ext / 8);
     const int prep_grid = static_cast<int>((prep_jobs + kPrepThreads * kPrepJobs - 1) / (kPrepThreads * kPrepJobs));
-    k_gemm_prep<<<prep_grid, kPrepThreads, prep_smem, stream>>>(
-        X, M, K, K_pad, K_ext, p, L.prot_idx, L.q8_scale, X16, err);
-    if (cudaGetLastError() != cudaSuccess) return BISCO_ERR_CUDA;
+    {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(prep_grid, 1, 1);
+        cfg.blockDim = dim3(kPrepThreads, 1, 1);
+        cfg.dynamicSmemBytes = prep_smem;
+        cfg.stream = stream;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        if (cudaLaunchKernelEx(&cfg, k_gemm_prep, X, M, K, K_pad, K_ext, p, L.prot_idx, L.q8_scale, X16,
+                               err) != cudaSuccess)
+            return BISCO_ERR_CUDA;
+    }
 
     const int TN = tile_tokens(M);
     CUtensorMap mx, mc, mn, mq;
