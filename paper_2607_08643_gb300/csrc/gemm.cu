@@ -18,8 +18,9 @@
 // int8 q8 values (exact in fp16), so the protected term is a few more k
 // steps of the same MMA, and the epilogue is Y = D / sqrt(8).
 //
-// CTA roles (512 threads, one CTA per SM, persistent over a contiguous
-// range of whole tiles, or of the tiles' k-steps in a stream-K split):
+// CTA roles (512 threads, one CTA per SM, persistent over whole tiles
+// taken round robin, or over a range of the tiles' k-steps in a stream-K
+// split; gemm_sched.cuh):
 //   warps 0-3  epilogue: TMEM -> registers -> Y (fp32), or to a partial
 //              tile in the workspace; lane quarter w
 //   warp 4     TMA producer of the compressed-weight ring
